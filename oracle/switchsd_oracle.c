@@ -1,0 +1,195 @@
+/*
+ * switchsd_oracle.c -- plain, slow CPU oracle of the SwitchSD per-step controller.
+ *
+ * TEST INFRASTRUCTURE ONLY.  This file is the reference the CUDA path is checked against.  Only the
+ * test suite, __graft_entry__.smoke() and bench.py's CPU-baseline leg may load it.  It shares no code,
+ * header, table or constant with the CUDA library (paper_2609_20186_gb300/csrc), and it includes
+ * nothing from there.  Every function follows one passage of the paper ("To Copy or Not to Copy:
+ * Controlling Speculative Decoding via Intrinsic Model Signals"), cited beside it, and is written as the
+ * plain definition: no blocking, no early reordering, floating point in double.
+ *
+ * Conventions (shared with the CUDA path only through the documented C ABI, not through code):
+ *   - a context row is int32 tokens x[0..L-1]; the current token is x[L-1];
+ *   - bf16 values arrive as their 16-bit patterns (uint16_t);
+ *   - modes: 0 = no repetition, 1 = copy draft, 2 = repetition without copy intent (Fig. 1 cases i-iii).
+ *
+ * Parity status: every function below is pinned by tests that do not re-run its own formula
+ * (brute-force enumeration, hand-built cases, library routines, closed forms); see tests/test_oracle_*.py.
+ */
+#include <stdint.h>
+#include <string.h>
+
+#define ORACLE_MODE_NO_REP 0
+#define ORACLE_MODE_COPY 1
+#define ORACLE_MODE_REP_NO_COPY 2
+
+#define ORACLE_ROW_OK 0
+#define ORACLE_ROW_CAPACITY 1
+
+/*
+ * Longest-suffix n-gram search.  §3.3 "Copy-Intent Decision Rule": the n-gram ending at the current
+ * token x_i must match a prior occurrence in the context; §3.3 "Copy-Based Speculative Generation":
+ * candidates are ranked by recency.  Reading of the open points: n is tried from n_max down to n_min
+ * and the first n with an occurrence wins; for that n the most recent occurrence (largest end e) wins;
+ * a prior occurrence ends at e <= L-2 so that at least one continuation token exists; occurrences may
+ * overlap the suffix itself.
+ * Returns 1 with (*n_out, *e_out) on a hit, else 0 with (0, -1).
+ */
+int oracle_longest_suffix_match(const int32_t *x, int32_t L, int32_t n_min, int32_t n_max,
+                                int32_t *n_out, int32_t *e_out)
+{
+    for (int32_t n = n_max; n >= n_min; --n) {
+        if (L < n + 1) continue;               /* the suffix and one earlier end must both fit */
+        for (int32_t e = L - 2; e >= n - 1; --e) {
+            int32_t i = 0;
+            while (i < n && x[e - i] == x[L - 1 - i]) ++i;
+            if (i == n) {
+                *n_out = n;
+                *e_out = e;
+                return 1;
+            }
+        }
+    }
+    *n_out = 0;
+    *e_out = -1;
+    return 0;
+}
+
+/* bf16 bit pattern -> double: a bf16 is the upper half of an IEEE binary32. */
+double oracle_bf16_to_double(uint16_t v)
+{
+    uint32_t bits = ((uint32_t)v) << 16;
+    float f;
+    memcpy(&f, &bits, sizeof f);
+    return (double)f;
+}
+
+/*
+ * Linear copy-intent probe, Eq. 3: p = sigma(w^T H), no bias.  The oracle returns the logit
+ * z = w^T H, summed in double in index order.
+ */
+double oracle_probe_linear(const uint16_t *h, const uint16_t *w, int32_t d)
+{
+    double z = 0.0;
+    for (int32_t j = 0; j < d; ++j)
+        z += oracle_bf16_to_double(w[j]) * oracle_bf16_to_double(h[j]);
+    return z;
+}
+
+/*
+ * Two-layer probe z = w2 . ReLU(W1 h + b1) + b2 (an extension beyond Eq. 3's linear probe, used by
+ * the 256-row / 5120-wide workload).  W1 is [H1, d] row-major bf16, w2 is [H1] bf16, b1 is [H1] float
+ * or NULL, b2 a float.  All arithmetic in double; the hidden layer is never rounded.
+ */
+double oracle_probe_mlp(const uint16_t *h, const uint16_t *W1, const float *b1, const uint16_t *w2,
+                        float b2, int32_t d, int32_t H1)
+{
+    double z = (double)b2;
+    for (int32_t u = 0; u < H1; ++u) {
+        double a = (b1 != NULL) ? (double)b1[u] : 0.0;
+        for (int32_t j = 0; j < d; ++j)
+            a += oracle_bf16_to_double(W1[(int64_t)u * d + j]) * oracle_bf16_to_double(h[j]);
+        if (a < 0.0) a = 0.0;
+        z += oracle_bf16_to_double(w2[u]) * a;
+    }
+    return z;
+}
+
+/*
+ * Three-way switch and copy draft.  Fig. 1: (i) no repetition -> neural draft; (ii) repetition with
+ * copy intent -> copy draft; (iii) repetition without copy intent -> neural draft.  Eq. 4 and the
+ * kappa-gram condition of §3.3: copy iff sigma(z) >= tau and the kappa-gram ending at x_{L-1} occurs
+ * earlier.  Since sigma is monotone, sigma(z) >= tau is decided as z >= logit(tau); the comparison is
+ * taken in binary32, the precision the device path decides in.  A match shorter than kappa counts as
+ * a repetition without copy intent.  The copy draft is the continuation after the matched occurrence,
+ * x[e*+1 ...], clipped at k and at the end of the context (§3.3 "Copy-Based Speculative Generation").
+ * Returns the mode; writes draft[0..len) and *len (0 unless copy).
+ */
+int32_t oracle_switch(int32_t has_match, int32_t n_star, int32_t e_star, double z, float logit_tau,
+                      int32_t kappa, int32_t k, const int32_t *x, int32_t L, int32_t *draft,
+                      int32_t *len)
+{
+    int32_t mode;
+    if (!has_match)
+        mode = ORACLE_MODE_NO_REP;
+    else if (n_star >= kappa && (float)z >= logit_tau)
+        mode = ORACLE_MODE_COPY;
+    else
+        mode = ORACLE_MODE_REP_NO_COPY;
+
+    *len = 0;
+    if (mode == ORACLE_MODE_COPY) {
+        int32_t avail = L - 1 - e_star;
+        int32_t n = avail < k ? avail : k;
+        for (int32_t i = 0; i < n; ++i) draft[i] = x[e_star + 1 + i];
+        *len = n;
+    }
+    return mode;
+}
+
+/*
+ * Greedy verification and append (§3.3 "Parallel Verification", "Overall Framework"; temperature 0 as
+ * in the main experiments, App. A).  target has len+1 meaningful entries: the target model's argmax
+ * after each draft prefix.  a = number of leading draft tokens equal to the target's argmax; the
+ * context receives draft[0..a) and then target[a], the target's own next token.  If that does not fit
+ * in cap the row is left untouched, *accept = -1 and the row status is ORACLE_ROW_CAPACITY.
+ */
+int32_t oracle_verify_row(int32_t *row, int32_t *L, int32_t cap, const int32_t *draft, int32_t len,
+                          const int32_t *target, int32_t *accept)
+{
+    int32_t a = 0;
+    while (a < len && draft[a] == target[a]) ++a;
+    if (*L + a + 1 > cap) {
+        *accept = -1;
+        return ORACLE_ROW_CAPACITY;
+    }
+    for (int32_t i = 0; i < a; ++i) row[*L + i] = draft[i];
+    row[*L + a] = target[a];
+    *L += a + 1;
+    *accept = a;
+    return ORACLE_ROW_OK;
+}
+
+/*
+ * One controller step over rows [b0, b1) of a batch: search, probe, switch, draft.  Layouts are the
+ * documented ABI layouts: ctx [B, cap] int32, hidden [B, d] bf16, out_draft [B, k].  probe_kind 0 uses
+ * probe_w = w[d]; probe_kind 1 uses probe_w = W1[H1, d] followed by w2[H1].  kappa <= 0 means
+ * kappa = n_min.  out_score receives the double logit; out_n / out_e the match (0 / -1 if none).
+ */
+void oracle_step_rows(const int32_t *ctx, const int32_t *lens, int32_t b0, int32_t b1, int32_t cap,
+                      const uint16_t *hidden, int32_t d, const uint16_t *probe_w, int32_t probe_kind,
+                      int32_t H1, const float *b1v, float b2, int32_t k, int32_t n_min, int32_t n_max,
+                      int32_t kappa, float logit_tau, int32_t *out_draft, int32_t *out_len,
+                      int32_t *out_mode, double *out_score, int32_t *out_n, int32_t *out_e)
+{
+    if (kappa <= 0) kappa = n_min;
+    for (int32_t b = b0; b < b1; ++b) {
+        const int32_t *x = ctx + (int64_t)b * cap;
+        int32_t L = lens[b];
+        int32_t n_star, e_star;
+        int32_t hit = oracle_longest_suffix_match(x, L, n_min, n_max, &n_star, &e_star);
+        const uint16_t *h = hidden + (int64_t)b * d;
+        double z;
+        if (probe_kind == 0)
+            z = oracle_probe_linear(h, probe_w, d);
+        else
+            z = oracle_probe_mlp(h, probe_w, b1v, probe_w + (int64_t)H1 * d, b2, d, H1);
+        out_mode[b] = oracle_switch(hit, n_star, e_star, z, logit_tau, kappa, k, x, L,
+                                    out_draft + (int64_t)b * k, &out_len[b]);
+        out_score[b] = z;
+        out_n[b] = n_star;
+        out_e[b] = e_star;
+    }
+}
+
+/* Verification over rows [b0, b1): draft [B, k], draft_len [B], target [B, k+1]. */
+void oracle_verify_rows(int32_t *ctx, int32_t *lens, int32_t b0, int32_t b1, int32_t cap, int32_t k,
+                        const int32_t *draft, const int32_t *draft_len, const int32_t *target,
+                        int32_t *out_accept, int32_t *status)
+{
+    for (int32_t b = b0; b < b1; ++b) {
+        int32_t st = oracle_verify_row(ctx + (int64_t)b * cap, &lens[b], cap, draft + (int64_t)b * k,
+                                       draft_len[b], target + (int64_t)b * (k + 1), &out_accept[b]);
+        if (status != NULL) status[b] = st;
+    }
+}

@@ -1,0 +1,96 @@
+"""Checks of the seeded input generators and the host harness (no controller arithmetic here)."""
+import numpy as np
+
+import synth
+from synth.rng import splitmix64, splitmix64_int, harness_key
+
+
+def test_splitmix64_published_sequence():
+    # SplitMix64 seeded with 0 (Vigna's reference generator): the state advances by the golden gamma
+    # and each output is the finaliser of the state; the first three outputs are:
+    g = 0x9E3779B97F4A7C15
+    expect = [0xE220A8397B1DCDAF, 0x6E789E6AA1B965F4, 0x06C45D188009454F]
+    assert [splitmix64_int((i * g) % (1 << 64)) for i in range(3)] == expect
+    got = splitmix64(np.array([(i * g) % (1 << 64) for i in range(3)], np.uint64))
+    assert [int(v) for v in got] == expect
+
+
+def test_harness_key_is_a_chain():
+    a = harness_key(7, 3, 11, np.arange(5, dtype=np.uint64))
+    k = splitmix64_int(7)
+    k = splitmix64_int(k ^ 3)
+    k = splitmix64_int(k ^ 11)
+    assert [int(v) for v in a] == [splitmix64_int(k ^ s) for s in range(5)]
+
+
+def test_bf16_rounding():
+    f = np.array([1.0, -2.0, 1.00390625, 1.005859375, 3.0e38, 0.0], np.float32)
+    bits = synth.bf16_bits_from_f32(f)
+    # 1 + 2^-8 is a tie between 1 and 1 + 2^-7: round to even (1.0); 1 + 3*2^-9 rounds up
+    assert bits.tolist() == [0x3F80, 0xC000, 0x3F80, 0x3F81, 0x7F62, 0x0000]
+    assert np.array_equal(synth.f32_from_bf16_bits(bits[:2]), np.array([1.0, -2.0], np.float32))
+
+
+def test_workload_shapes_and_determinism():
+    for name, wl in synth.WORKLOADS.items():
+        assert wl.cap % 4 == 0 and wl.cap >= wl.L0 + wl.steps * (wl.k + 1)
+        small = wl.scaled(B=min(wl.B, 2), L0=min(wl.L0, 4096), steps=2)
+        a = small.context_row(1 if small.B > 1 else 0)
+        b = small.context_row(1 if small.B > 1 else 0)
+        assert np.array_equal(a, b) and a.min() >= 0 and a.max() < wl.V
+    wl = synth.get_workload("uniform_8k")
+    assert wl.probe_weights().shape == (wl.d,)
+    assert wl.hidden(3).shape == (wl.B, wl.d)
+    mlp = synth.get_workload("code_16k")
+    assert mlp.probe_weights().shape == (mlp.probe_hidden * mlp.d + mlp.probe_hidden,)
+
+
+def test_planted_spans_are_verbatim_earlier_copies():
+    wl = synth.get_workload("uniform_8k").scaled(B=1)
+    x = wl.context_row(0)
+    # with uniform ids over 128K, an 8-gram repeat only arises from a planted copy; about 10 % of
+    # positions end such a repeat
+    seen = {}
+    ends = 0
+    for e in range(7, x.shape[0]):
+        g = tuple(x[e - 7: e + 1].tolist())
+        if g in seen:
+            ends += 1
+        seen.setdefault(g, e)
+    assert 0.05 * x.shape[0] < ends < 0.12 * x.shape[0]
+
+
+def test_labels_coverage():
+    wl = synth.get_workload("mixed_128k").scaled(B=2)
+    lab = wl.labels()
+    assert lab.shape == (2, wl.cap - wl.L0)
+    assert 0.1 < lab.mean() < 0.5
+
+
+def test_harness_law():
+    wl = synth.get_workload("uniform_8k").scaled(B=64, steps=4)
+    params = wl.harness_params()
+    B, k = wl.B, wl.k
+    rng = np.random.default_rng(0)
+    draft = rng.integers(0, wl.V, (B, k)).astype(np.int32)
+    mode = np.array([1, 0, 2] * 21 + [1], np.int32)
+    dlen = np.where(mode == 1, k, 0).astype(np.int32)
+    lens = np.full(B, wl.L0, np.int32)
+    labels = np.ones((B, wl.cap - wl.L0), np.uint8)
+    vd, vl, t = synth.harness_targets(params, 0, lens, mode, draft, dlen, labels)
+    assert np.all(vl == k)
+    assert np.array_equal(vd[mode == 1], draft[mode == 1])
+    agree = (vd == t[:, :k])
+    assert 0.8 < agree.mean() < 0.97           # p_in = 0.9 everywhere here
+    # a disagreeing target never equals the draft token
+    assert np.all((t[:, :k] != vd) | agree)
+    # outside spans the agreement law is p_out = 0.05
+    vd, vl, t = synth.harness_targets(params, 1, lens, mode, draft, dlen, labels * 0)
+    assert (vd == t[:, :k]).mean() < 0.12
+    # agree_cap forces a disagreement at index 5 (the planted workload)
+    pw = synth.get_workload("planted_copy")
+    p = pw.harness_params()
+    d1 = rng.integers(0, pw.V, (1, pw.k)).astype(np.int32)
+    vd, vl, t = synth.harness_targets(p, 0, np.array([pw.L0], np.int32), np.array([1], np.int32),
+                                      d1, np.array([pw.k], np.int32), pw.labels())
+    assert t[0, :5].tolist() == d1[0, :5].tolist() and t[0, 5] != d1[0, 5]
