@@ -1,0 +1,173 @@
+/*
+ * switchsd.h -- C ABI of the SwitchSD per-step controller on one GB300 (sm_103a).
+ *
+ * SwitchSD ("To Copy or Not to Copy: Controlling Speculative Decoding via Intrinsic Model Signals")
+ * decides after every verification step whether the next draft is copied from the context or left to
+ * a neural drafter (Fig. 1).  This library runs that controller for B independent sequences:
+ *
+ *   switchsd_step    longest-suffix n-gram search (§3.3 kappa-gram gate, recency ranking), the
+ *                    copy-intent probe logit (Eq. 3, or a two-layer extension), the three-way switch
+ *                    (Fig. 1, Eq. 4) and the copy draft gather (§3.3 "Copy-Based Speculative
+ *                    Generation");
+ *   switchsd_verify  greedy verification and append (§3.3 "Parallel Verification", temperature 0 as
+ *                    in App. A): accepted prefix length, then the accepted tokens and the target's own
+ *                    next token are appended to the context.
+ *
+ * The target model and the neural drafter are outside the library; their outputs (hidden state at the
+ * probed layer, the target's greedy tokens, the neural draft) arrive as arguments.
+ *
+ * General conventions
+ *   - Every array pointer is a caller-owned DEVICE pointer (cudaMalloc / torch CUDA tensor memory) on
+ *     the current CUDA device.  The library never frees or retains them.
+ *   - Calls are asynchronous on `stream` (a cudaStream_t passed as void*; NULL = legacy default
+ *     stream).  They return SWITCHSD_OK once the work is enqueued, or a negative host error code
+ *     before anything is enqueued (bad argument, unsupported shape) or SWITCHSD_ERR_CUDA if a launch
+ *     failed.  Outputs are valid once the stream reaches the call.
+ *   - Per-row problems found on the device (bad length, capacity overflow) are reported in the
+ *     optional per-row `status` array (SWITCHSD_ROW_*); the kernels never trap.
+ *   - Token ids are opaque int32 values: only equality is used.
+ *   - bf16 values are passed as their 16-bit patterns (uint16_t), the upper half of an IEEE binary32.
+ *   - All calls may be captured into a CUDA graph: they allocate nothing and synchronise nothing.
+ */
+#ifndef SWITCHSD_H_
+#define SWITCHSD_H_
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#define SWITCHSD_ABI_VERSION 1
+
+#define SWITCHSD_NMAX 32 /* largest supported n_max */
+#define SWITCHSD_KMAX 64 /* largest supported draft length k */
+
+/* Modes: the three cases of Fig. 1. */
+#define SWITCHSD_MODE_NO_REP 0      /* (i) no repetition: neural draft */
+#define SWITCHSD_MODE_COPY 1        /* (ii) repetition with copy intent: copy draft */
+#define SWITCHSD_MODE_REP_NO_COPY 2 /* (iii) repetition without copy intent: neural draft */
+
+/* Probe kinds. */
+#define SWITCHSD_PROBE_LINEAR 0 /* Eq. 3: z = w^T h, probe_w = w[d] */
+#define SWITCHSD_PROBE_MLP 1    /* z = w2 . ReLU(W1 h + b1) + b2, probe_w = W1[H1, d] then w2[H1] */
+
+/* Host return codes. */
+#define SWITCHSD_OK 0
+#define SWITCHSD_ERR_ARG (-1)   /* NULL or misaligned pointer, bad enum */
+#define SWITCHSD_ERR_SHAPE (-2) /* unsupported size */
+#define SWITCHSD_ERR_CUDA (-3)  /* a CUDA call failed; cudaGetLastError() has the cause */
+
+/* Per-row device status. */
+#define SWITCHSD_ROW_OK 0
+#define SWITCHSD_ROW_CAPACITY 1 /* verify: the append does not fit in cap; row left untouched */
+#define SWITCHSD_ROW_BAD_LEN 2  /* ctx_lens[b] outside [1, cap] or draft_len[b] outside [0, k] */
+#define SWITCHSD_ROW_TIMEOUT 3  /* an on-chip copy did not complete within its wait limit */
+
+/*
+ * Parameters of switchsd_step.
+ *
+ *   B            number of rows (sequences), >= 1
+ *   cap          row capacity in tokens (row stride of ctx_tokens), a multiple of 4, >= 4
+ *   d            hidden size, a multiple of 8
+ *   k            largest copy draft, 1..SWITCHSD_KMAX (the paper's D, App. D)
+ *   n_min,n_max  n-gram lengths searched, 1 <= n_min <= n_max <= SWITCHSD_NMAX
+ *   kappa        shortest match that may copy (§3.3, the paper sets 5); <= 0 means n_min
+ *   logit_tau    decision threshold in logit space: copy iff z >= logit_tau (Eq. 4 with tau;
+ *                tau = 0.5 gives 0.0; -INFINITY copies on every match, +INFINITY never copies)
+ *   probe_kind   SWITCHSD_PROBE_LINEAR or SWITCHSD_PROBE_MLP
+ *   probe_hidden H1 of the two-layer probe (1..1024); ignored for the linear probe
+ *   b1, b2       two-layer probe biases: b1 device float[H1] or NULL (zero), b2 a float
+ *   split        CTAs per row (1, 2, 4, 8 or 16); 0 lets the library choose
+ *   out_match_n, out_match_end   optional device int32[B]: the winning match length n* and the end
+ *                position e* of its most recent earlier occurrence (0 / -1 when none); may be NULL
+ *   status       optional device int32[B] per-row status (SWITCHSD_ROW_*); may be NULL
+ *   stream       cudaStream_t as void*
+ */
+typedef struct {
+    int32_t B, cap, d, k, n_min, n_max, kappa;
+    float logit_tau;
+    int32_t probe_kind;
+    int32_t probe_hidden;
+    const float *b1;
+    float b2;
+    int32_t split;
+    int32_t *out_match_n;
+    int32_t *out_match_end;
+    int32_t *status;
+    void *stream;
+} switchsd_params;
+
+/*
+ * One controller step for B rows (§3.3, Fig. 1).
+ *
+ *   ctx_tokens  int32 [B, cap] row-major, 16-byte aligned; row b holds its context x[0..L_b-1]
+ *   ctx_lens    int32 [B]; L_b = ctx_lens[b], 1 <= L_b <= cap
+ *   hidden      bf16 [B, d] row-major, 16-byte aligned: the target model's hidden state at the probed
+ *               layer for the row's current (last) token
+ *   probe_w     bf16, 16-byte aligned: w[d] (linear) or W1[H1, d] row-major followed by w2[H1]
+ *
+ * For each row: (n*, e*) = the longest n in [n_min, n_max] whose suffix x[L-n..L-1] also ends at an
+ * earlier position e <= L-2, and for that n the most recent such e.  z = the probe logit (fp32
+ * accumulation of bf16 products).  mode = NO_REP if no match, COPY if n* >= kappa and
+ * z >= logit_tau, else REP_NO_COPY.  For COPY rows the draft is x[e*+1 .. e*+len] with
+ * len = min(k, L-1-e*); other rows get len 0 (the caller's neural drafter takes over).
+ *
+ *   out_draft   int32 [B, k]: entries at and beyond out_len[b] are unspecified
+ *   out_len     int32 [B]
+ *   out_mode    int32 [B]   (SWITCHSD_MODE_*)
+ *   out_score   float [B]   the probe logit z (written for every row)
+ *
+ * Rows with a bad length get mode NO_REP, len 0 and status SWITCHSD_ROW_BAD_LEN.
+ */
+int switchsd_step(const int32_t *ctx_tokens, const int32_t *ctx_lens, const uint16_t *hidden,
+                  const uint16_t *probe_w, const switchsd_params *params, int32_t *out_draft,
+                  int32_t *out_len, int32_t *out_mode, float *out_score);
+
+/*
+ * Parameters of switchsd_verify.
+ *
+ *   B, cap, k    as for switchsd_step
+ *   draft_len    device int32 [B]: tokens of the draft to verify per row, 0..k (a copy row passes
+ *                switchsd_step's out_len, a neural row its own draft length)
+ *   ctx_tokens   device int32 [B, cap] (modified: accepted tokens are appended)
+ *   ctx_lens     device int32 [B]      (modified: grows by accepted + 1)
+ *   status       optional device int32 [B]; may be NULL
+ *   stream       cudaStream_t as void*
+ */
+typedef struct {
+    int32_t B, cap, k;
+    const int32_t *draft_len;
+    int32_t *ctx_tokens;
+    int32_t *ctx_lens;
+    int32_t *status;
+    void *stream;
+} switchsd_verify_params;
+
+/*
+ * Greedy verification and append (§3.3 "Parallel Verification", temperature 0, App. A).
+ *
+ *   draft          int32 [B, k]: the draft that was verified (copy or neural)
+ *   target_argmax  int32 [B, k+1]: the target model's greedy token after each draft prefix; entry i
+ *                  is its prediction for the position of draft[i], entry len its next token after a
+ *                  fully accepted draft
+ *   out_accept     int32 [B]: a = number of leading draft tokens equal to target_argmax
+ *
+ * The row's context receives draft[0..a) then target_argmax[a]; ctx_lens grows by a+1.  If that does
+ * not fit in cap, the row is untouched, out_accept = -1 and status = SWITCHSD_ROW_CAPACITY.
+ */
+int switchsd_verify(const int32_t *draft, const int32_t *target_argmax, int32_t *out_accept,
+                    const switchsd_verify_params *vp);
+
+/* Human-readable text of a host return code or a row status (static storage, never NULL). */
+const char *switchsd_strerror(int code);
+
+/* SWITCHSD_ABI_VERSION of the loaded library. */
+int switchsd_abi_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* SWITCHSD_H_ */

@@ -1,0 +1,200 @@
+"""ctypes binding of libswitchsd.so: the C ABI of include/switchsd.h and include/switchsd_harness.h.
+
+Argument marshalling only: every function takes torch CUDA tensors, checks dtype / device / layout,
+and passes raw device pointers and the current CUDA stream to the library.  All computation runs in
+the library's kernels.  If the library is missing the first call raises; there is no fallback.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import threading
+
+import torch
+
+from . import build as _build
+
+MODE_NO_REP, MODE_COPY, MODE_REP_NO_COPY = 0, 1, 2
+PROBE_LINEAR, PROBE_MLP = 0, 1
+OK, ERR_ARG, ERR_SHAPE, ERR_CUDA = 0, -1, -2, -3
+ROW_OK, ROW_CAPACITY, ROW_BAD_LEN, ROW_TIMEOUT = 0, 1, 2, 3
+NMAX, KMAX = 32, 64
+
+_c_i32p = ctypes.c_void_p
+
+
+class switchsd_params(ctypes.Structure):
+    _fields_ = [
+        ("B", ctypes.c_int32), ("cap", ctypes.c_int32), ("d", ctypes.c_int32), ("k", ctypes.c_int32),
+        ("n_min", ctypes.c_int32), ("n_max", ctypes.c_int32), ("kappa", ctypes.c_int32),
+        ("logit_tau", ctypes.c_float),
+        ("probe_kind", ctypes.c_int32), ("probe_hidden", ctypes.c_int32),
+        ("b1", ctypes.c_void_p), ("b2", ctypes.c_float),
+        ("split", ctypes.c_int32),
+        ("out_match_n", ctypes.c_void_p), ("out_match_end", ctypes.c_void_p),
+        ("status", ctypes.c_void_p),
+        ("stream", ctypes.c_void_p),
+    ]
+
+
+class switchsd_verify_params(ctypes.Structure):
+    _fields_ = [
+        ("B", ctypes.c_int32), ("cap", ctypes.c_int32), ("k", ctypes.c_int32),
+        ("draft_len", ctypes.c_void_p), ("ctx_tokens", ctypes.c_void_p),
+        ("ctx_lens", ctypes.c_void_p), ("status", ctypes.c_void_p), ("stream", ctypes.c_void_p),
+    ]
+
+
+class switchsd_harness_params(ctypes.Structure):
+    _fields_ = [
+        ("B", ctypes.c_int32), ("k", ctypes.c_int32), ("V", ctypes.c_int32), ("L0", ctypes.c_int32),
+        ("n_labels", ctypes.c_int32), ("agree_cap", ctypes.c_int32), ("step", ctypes.c_int32),
+        ("seed", ctypes.c_uint64), ("thr_in", ctypes.c_uint64), ("thr_out", ctypes.c_uint64),
+        ("stream", ctypes.c_void_p),
+    ]
+
+
+_lock = threading.Lock()
+_lib = None
+
+# Every symbol the headers declare, with its ctypes signature.
+_SIGNATURES = {
+    "switchsd_step": (ctypes.c_int, [ctypes.c_void_p] * 4 + [ctypes.POINTER(switchsd_params)]
+                      + [ctypes.c_void_p] * 4),
+    "switchsd_verify": (ctypes.c_int, [ctypes.c_void_p] * 3
+                        + [ctypes.POINTER(switchsd_verify_params)]),
+    "switchsd_strerror": (ctypes.c_char_p, [ctypes.c_int]),
+    "switchsd_abi_version": (ctypes.c_int, []),
+    "switchsd_harness_target": (ctypes.c_int, [ctypes.c_void_p] * 8
+                                + [ctypes.POINTER(switchsd_harness_params)]),
+}
+
+
+def library_path() -> str:
+    return _build.LIB
+
+
+def load(path: str | None = None):
+    """Loads (once) and returns the ctypes handle.  Raises if the library was not built."""
+    global _lib
+    with _lock:
+        if _lib is not None:
+            return _lib
+        p = path or _build.LIB
+        if not os.path.exists(p):
+            raise RuntimeError(f"{p} is missing: build it with __graft_entry__.build() "
+                               "(python -m paper_2609_20186_gb300.build); there is no fallback")
+        lib = ctypes.CDLL(p)
+        for name, (res, args) in _SIGNATURES.items():
+            fn = getattr(lib, name)
+            fn.restype = res
+            fn.argtypes = args
+        _lib = lib
+        return lib
+
+
+def strerror(code: int) -> str:
+    return load().switchsd_strerror(code).decode()
+
+
+def abi_version() -> int:
+    return load().switchsd_abi_version()
+
+
+def _check(code: int, what: str):
+    if code != OK:
+        raise RuntimeError(f"{what} failed: {code} ({strerror(code)})")
+
+
+def _dev(t: torch.Tensor | None, dtype, name: str, shape=None):
+    if t is None:
+        return None
+    if not isinstance(t, torch.Tensor) or not t.is_cuda:
+        raise TypeError(f"{name} must be a CUDA tensor")
+    if t.dtype != dtype:
+        raise TypeError(f"{name} must be {dtype}, got {t.dtype}")
+    if not t.is_contiguous():
+        raise ValueError(f"{name} must be contiguous")
+    if shape is not None and tuple(t.shape) != tuple(shape):
+        raise ValueError(f"{name} has shape {tuple(t.shape)}, expected {tuple(shape)}")
+    return t.data_ptr()
+
+
+def _stream_ptr(stream) -> int:
+    s = stream if stream is not None else torch.cuda.current_stream()
+    return s.cuda_stream
+
+
+def _bf16(t: torch.Tensor, name: str, shape=None):
+    return _dev(t, torch.bfloat16, name, shape)
+
+
+def switchsd_step(ctx_tokens, ctx_lens, hidden, probe_w, out_draft, out_len, out_mode, out_score, *,
+                  k: int, n_min: int, n_max: int, kappa: int = 0, logit_tau: float = 0.0,
+                  probe_kind: int = PROBE_LINEAR, probe_hidden: int = 0, b1=None, b2: float = 0.0,
+                  split: int = 0, out_match_n=None, out_match_end=None, status=None,
+                  stream=None) -> None:
+    """switchsd_step of include/switchsd.h on torch tensors (see the header for semantics).
+
+    ctx_tokens int32 [B, cap]; ctx_lens int32 [B]; hidden bf16 [B, d]; probe_w bf16 (w[d] or
+    W1[H1, d] + w2[H1] flattened); outputs int32 [B, k], int32 [B], int32 [B], float32 [B].
+    """
+    B, cap = ctx_tokens.shape
+    d = hidden.shape[1]
+    p = switchsd_params()
+    p.B, p.cap, p.d, p.k = B, cap, d, k
+    p.n_min, p.n_max, p.kappa = n_min, n_max, kappa
+    p.logit_tau = logit_tau
+    p.probe_kind, p.probe_hidden = probe_kind, probe_hidden
+    p.b1 = _dev(b1, torch.float32, "b1", (probe_hidden,)) if b1 is not None else None
+    p.b2 = b2
+    p.split = split
+    p.out_match_n = _dev(out_match_n, torch.int32, "out_match_n", (B,))
+    p.out_match_end = _dev(out_match_end, torch.int32, "out_match_end", (B,))
+    p.status = _dev(status, torch.int32, "status", (B,))
+    p.stream = _stream_ptr(stream)
+    nw = d if probe_kind == PROBE_LINEAR else probe_hidden * d + probe_hidden
+    code = load().switchsd_step(
+        _dev(ctx_tokens, torch.int32, "ctx_tokens"), _dev(ctx_lens, torch.int32, "ctx_lens", (B,)),
+        _bf16(hidden, "hidden", (B, d)), _bf16(probe_w, "probe_w", (nw,)), ctypes.byref(p),
+        _dev(out_draft, torch.int32, "out_draft", (B, k)), _dev(out_len, torch.int32, "out_len", (B,)),
+        _dev(out_mode, torch.int32, "out_mode", (B,)), _dev(out_score, torch.float32, "out_score", (B,)))
+    _check(code, "switchsd_step")
+
+
+def switchsd_verify(draft, target_argmax, out_accept, *, draft_len, ctx_tokens, ctx_lens,
+                    status=None, stream=None) -> None:
+    """switchsd_verify of include/switchsd.h on torch tensors."""
+    B, cap = ctx_tokens.shape
+    k = draft.shape[1]
+    vp = switchsd_verify_params()
+    vp.B, vp.cap, vp.k = B, cap, k
+    vp.draft_len = _dev(draft_len, torch.int32, "draft_len", (B,))
+    vp.ctx_tokens = _dev(ctx_tokens, torch.int32, "ctx_tokens")
+    vp.ctx_lens = _dev(ctx_lens, torch.int32, "ctx_lens", (B,))
+    vp.status = _dev(status, torch.int32, "status", (B,))
+    vp.stream = _stream_ptr(stream)
+    code = load().switchsd_verify(_dev(draft, torch.int32, "draft", (B, k)),
+                                  _dev(target_argmax, torch.int32, "target_argmax", (B, k + 1)),
+                                  _dev(out_accept, torch.int32, "out_accept", (B,)), ctypes.byref(vp))
+    _check(code, "switchsd_verify")
+
+
+def switchsd_harness_target(ctx_lens, mode, draft, draft_len, labels, vdraft, vlen, target, *,
+                            seed: int, V: int, L0: int, agree_cap: int, thr_in: int, thr_out: int,
+                            step: int, stream=None) -> None:
+    """switchsd_harness_target of include/switchsd_harness.h (the target-model stand-in)."""
+    B, k = draft.shape
+    hp = switchsd_harness_params()
+    hp.B, hp.k, hp.V, hp.L0 = B, k, V, L0
+    hp.n_labels = labels.shape[1]
+    hp.agree_cap, hp.step = agree_cap, step
+    hp.seed, hp.thr_in, hp.thr_out = seed, thr_in, thr_out
+    hp.stream = _stream_ptr(stream)
+    code = load().switchsd_harness_target(
+        _dev(ctx_lens, torch.int32, "ctx_lens", (B,)), _dev(mode, torch.int32, "mode", (B,)),
+        _dev(draft, torch.int32, "draft", (B, k)), _dev(draft_len, torch.int32, "draft_len", (B,)),
+        _dev(labels, torch.uint8, "labels"), _dev(vdraft, torch.int32, "vdraft", (B, k)),
+        _dev(vlen, torch.int32, "vlen", (B,)), _dev(target, torch.int32, "target", (B, k + 1)),
+        ctypes.byref(hp))
+    _check(code, "switchsd_harness_target")

@@ -1,0 +1,91 @@
+// harness.cu -- device stand-in for the neural drafter and the target model (not the controller).
+//
+// Synthesises the target's greedy tokens for each row's draft with the seeded agreement law stated
+// in switchsd_harness.h.  One warp per row; lane i handles draft indices i, i + 32, ...
+#include "common.cuh"
+#include "switchsd_harness.h"
+
+namespace switchsd {
+
+constexpr int kHarnessThreads = 256;
+
+struct HarnessArgs {
+    const int32_t *lens, *mode, *draft, *draft_len;
+    const uint8_t *labels;
+    int32_t *vdraft, *vlen, *target;
+    switchsd_harness_params p;
+};
+
+// splitmix64 finaliser (Steele, Lea and Flood; Vigna's published constants).
+__device__ __forceinline__ uint64_t splitmix64(uint64_t z) {
+    z += 0x9E3779B97F4A7C15ull;
+    z = (z ^ (z >> 30)) * 0xBF58476D1CE4E5B9ull;
+    z = (z ^ (z >> 27)) * 0x94D049BB133111EBull;
+    return z ^ (z >> 31);
+}
+
+__device__ __forceinline__ int32_t token_of(uint64_t r, int32_t V) {
+    return int32_t((r >> 32) % uint64_t(V));
+}
+
+__global__ void __launch_bounds__(kHarnessThreads) harness_kernel(const HarnessArgs a) {
+    const int lane = threadIdx.x & 31;
+    const int b = (blockIdx.x * kHarnessThreads + threadIdx.x) >> 5;
+    const switchsd_harness_params &p = a.p;
+    if (b >= p.B) return;
+    const int k = p.k;
+    const bool copy = a.mode[b] == SWITCHSD_MODE_COPY;
+    int len = copy ? a.draft_len[b] : k;
+    len = len < 0 ? 0 : (len > k ? k : len);
+    const int32_t L = a.lens[b];
+    const uint64_t row_key = splitmix64(splitmix64(splitmix64(p.seed) ^ uint64_t(b)) ^ uint64_t(p.step));
+    for (int i = lane; i <= k; i += kWarp) {
+        const uint64_t slot = 4ull * uint64_t(i);
+        int32_t d = 0;
+        if (i < len) d = copy ? a.draft[size_t(b) * k + i] : token_of(splitmix64(row_key ^ (slot + 2)), p.V);
+        if (i < k) a.vdraft[size_t(b) * k + i] = i < len ? d : 0;
+        int32_t t;
+        if (i < len) {
+            const int64_t pos = int64_t(L) + i - p.L0;
+            const bool lab = pos >= 0 && pos < p.n_labels && a.labels[size_t(b) * p.n_labels + pos] != 0;
+            const uint64_t thr = lab ? p.thr_in : p.thr_out;
+            const uint64_t coin = splitmix64(row_key ^ (slot + 0)) & 0xffffffffull;
+            const bool agree = i < p.agree_cap && coin < thr;
+            if (agree) {
+                t = d;
+            } else {
+                t = token_of(splitmix64(row_key ^ (slot + 1)), p.V);
+                if (t == d) t = (t + 1) % p.V;
+            }
+        } else {
+            t = token_of(splitmix64(row_key ^ (slot + 3)), p.V);
+        }
+        a.target[size_t(b) * (k + 1) + i] = t;
+    }
+    if (lane == 0) a.vlen[b] = len;
+}
+
+}  // namespace switchsd
+
+using namespace switchsd;
+
+extern "C" int switchsd_harness_target(const int32_t *ctx_lens, const int32_t *mode, const int32_t *draft,
+                                       const int32_t *draft_len, const uint8_t *labels, int32_t *vdraft,
+                                       int32_t *vlen, int32_t *target, const switchsd_harness_params *hp) {
+    if (!hp || !ctx_lens || !mode || !draft || !draft_len || !vdraft || !vlen || !target) return SWITCHSD_ERR_ARG;
+    if (hp->n_labels > 0 && !labels) return SWITCHSD_ERR_ARG;
+    if (hp->B < 1 || hp->k < 1 || hp->k > SWITCHSD_KMAX || hp->V < 2 || hp->n_labels < 0) return SWITCHSD_ERR_SHAPE;
+    HarnessArgs a;
+    a.lens = ctx_lens;
+    a.mode = mode;
+    a.draft = draft;
+    a.draft_len = draft_len;
+    a.labels = labels;
+    a.vdraft = vdraft;
+    a.vlen = vlen;
+    a.target = target;
+    a.p = *hp;
+    const int wpb = kHarnessThreads / kWarp;
+    harness_kernel<<<(hp->B + wpb - 1) / wpb, kHarnessThreads, 0, static_cast<cudaStream_t>(hp->stream)>>>(a);
+    return cudaGetLastError() == cudaSuccess ? SWITCHSD_OK : SWITCHSD_ERR_CUDA;
+}

@@ -1,0 +1,419 @@
+// step.cu -- switchsd_step: n-gram search, probe, switch and copy-draft gather for B rows.
+//
+// Paper: §3.3 (kappa-gram gate, recency-ranked copy candidates, Eq. 4 decision rule), Eq. 3 (linear
+// probe), Fig. 1 (three cases).
+//
+// Layout of the work.  Row b is handled by one thread-block cluster of C CTAs (grid = C x B).  The
+// candidate end positions e in [0, L-1) are split into C contiguous 16-byte-aligned ranges.  Each CTA
+// streams its range through shared memory in tiles of kTile tokens with bulk TMA copies (one copy per
+// tile, kHalo tokens of look-back included), so the whole range is in flight at once.  A position e
+// is a candidate when x[e] equals the current token; the thread then compares backwards against the
+// suffix (held in shared memory) to get m(e) = the common suffix length, capped at n_max.  The row's
+// answer is the maximum of the packed key (m << 32 | e) over candidates with m >= n_min: the largest
+// m first, then the most recent e -- exactly the longest-then-most-recent rule.
+//
+// The same CTAs also compute the linear probe: CTA r dots its 1/C slice of the hidden state with the
+// probe weights in fp32.  Each CTA writes its key and its probe partial into the leader CTA's shared
+// memory over DSMEM; after one cluster barrier the leader reduces them (fixed order), applies the
+// switch and gathers the draft.  No global scratch, no atomics, no inter-CTA spin-waits.
+#include "common.cuh"
+
+namespace switchsd {
+
+constexpr int kStepThreads = 256;
+constexpr int kStepWarps = kStepThreads / kWarp;
+constexpr int kTile = 4096;  // tokens per staged tile
+constexpr int kHalo = 32;    // look-back staged before each tile: >= SWITCHSD_NMAX - 1, multiple of 4
+constexpr int kStages = 2;
+constexpr int kStageInts = kHalo + kTile;
+constexpr int kMaxSplit = 16;
+constexpr size_t kStepSmemBytes = size_t(kStages) * kStageInts * sizeof(int32_t);
+constexpr unsigned long long kTimeoutBit = 1ull << 62;
+
+static_assert(kHalo >= SWITCHSD_NMAX - 1 && kHalo % 4 == 0, "halo must cover the longest n-gram");
+
+struct StepArgs {
+    const int32_t *ctx;
+    const int32_t *lens;
+    const uint16_t *hidden;
+    const uint16_t *probe_w;
+    const float *z_pre;  // logits from the two-layer probe kernel, or null for the linear probe
+    int32_t B, cap, d, k, n_min, n_max, kappa;
+    float logit_tau;
+    int32_t *out_draft, *out_len, *out_mode;
+    float *out_score;
+    int32_t *out_match_n, *out_match_end, *status;
+};
+
+__device__ __forceinline__ float dot8_bf16(uint4 w, uint4 h, float acc) {
+    acc = fmaf(bf16_lo(w.x), bf16_lo(h.x), acc);
+    acc = fmaf(bf16_hi(w.x), bf16_hi(h.x), acc);
+    acc = fmaf(bf16_lo(w.y), bf16_lo(h.y), acc);
+    acc = fmaf(bf16_hi(w.y), bf16_hi(h.y), acc);
+    acc = fmaf(bf16_lo(w.z), bf16_lo(h.z), acc);
+    acc = fmaf(bf16_hi(w.z), bf16_hi(h.z), acc);
+    acc = fmaf(bf16_lo(w.w), bf16_lo(h.w), acc);
+    acc = fmaf(bf16_hi(w.w), bf16_hi(h.w), acc);
+    return acc;
+}
+
+__global__ void __launch_bounds__(kStepThreads) step_kernel(const StepArgs a) {
+    extern __shared__ __align__(128) int32_t tiles[];  // kStages x kStageInts
+    __shared__ __align__(8) uint64_t bars[kStages];
+    __shared__ int32_t s_suf[SWITCHSD_NMAX];
+    __shared__ unsigned long long s_wkey[kStepWarps];
+    __shared__ float s_wz[kStepWarps];
+    __shared__ unsigned long long s_key[kMaxSplit];  // leader: one slot per CTA of the cluster
+    __shared__ float s_zp[kMaxSplit];
+    __shared__ int32_t s_out[3];                     // leader: mode, len, e*
+
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    const uint32_t rank = cluster_ctarank();
+    const uint32_t C = cluster_nctarank();
+    const int b = blockIdx.y;
+
+    // Phase 1 of the cluster barrier: waited on right before the first DSMEM store, by which time
+    // every CTA of the cluster is guaranteed to be running.
+    cluster_arrive_relaxed();
+
+    const int32_t *row = a.ctx + size_t(b) * size_t(a.cap);
+    const int32_t L = a.lens[b];
+    const bool len_ok = (L >= 1 && L <= a.cap);
+    const int32_t E = len_ok ? L - 1 : 0;  // candidate ends e in [0, E)
+
+    int32_t chunk = (E + int32_t(C) - 1) / int32_t(C);
+    chunk = (chunk + 3) & ~3;
+    const int32_t e_lo = min(E, int32_t(rank) * chunk);
+    const int32_t e_hi = min(E, e_lo + chunk);
+    const int32_t ntiles = (e_hi - e_lo + kTile - 1) / kTile;
+
+    if (tid == 0) {
+        for (int s = 0; s < kStages; ++s) mbar_init(&bars[s], 1);
+        fence_mbar_init();
+    }
+    if (tid < SWITCHSD_NMAX) s_suf[tid] = (len_ok && tid < L) ? row[L - 1 - tid] : 0;
+    __syncthreads();
+
+    // Stage tile t: tokens [max(0, t0 - kHalo), roundup4(t1)) land so that tokens[p] sits at
+    // stage[kHalo + p - t0].  roundup4(t1) <= cap because t1 <= L-1 < cap and cap % 4 == 0.
+    auto issue = [&](int t) {
+        const int s = t % kStages;
+        const int32_t t0 = e_lo + t * kTile;
+        const int32_t t1 = min(e_hi, t0 + kTile);
+        const int32_t lo = max(0, t0 - kHalo);
+        const int32_t hi = (t1 + 3) & ~3;
+        const uint32_t bytes = uint32_t(hi - lo) * 4u;
+        mbar_arrive_expect_tx(&bars[s], bytes);
+        bulk_g2s(tiles + s * kStageInts + (kHalo + lo - t0), row + lo, bytes, &bars[s]);
+    };
+    if (tid == 0)
+        for (int t = 0; t < min(ntiles, kStages); ++t) issue(t);
+
+    // Linear probe partial over this CTA's slice of the hidden vector (overlaps the copies).
+    float zp = 0.f;
+    if (a.z_pre == nullptr) {
+        const int nv = a.d >> 3;
+        const int per = (nv + int(C) - 1) / int(C);
+        const int v0 = int(rank) * per, v1 = min(nv, v0 + per);
+        const uint4 *h4 = reinterpret_cast<const uint4 *>(a.hidden + size_t(b) * size_t(a.d));
+        const uint4 *w4 = reinterpret_cast<const uint4 *>(a.probe_w);
+        for (int v = v0 + tid; v < v1; v += kStepThreads) zp = dot8_bf16(__ldg(w4 + v), __ldg(h4 + v), zp);
+    }
+
+    // Scan.
+    const int32_t s0 = s_suf[0];
+    const int32_t n_max = a.n_max, n_min = a.n_min;
+    unsigned long long best = 0;  // real keys have m >= n_min >= 1, so 0 means "no match"
+    bool ok = true;
+    int t = 0;
+    for (; t < ntiles; ++t) {
+        const int s = t % kStages;
+        ok = __syncthreads_and(mbar_wait(&bars[s], uint32_t(t / kStages) & 1u));
+        if (!ok) break;
+        const int32_t t0 = e_lo + t * kTile;
+        const int32_t t1 = min(e_hi, t0 + kTile);
+        const int32_t *stage = tiles + s * kStageInts;
+        const int32_t off = kHalo - t0;  // stage[off + p] = x[p] over the staged range
+        for (int32_t e4 = t0 + 4 * tid; e4 < t1; e4 += 4 * kStepThreads) {
+            const int4 v = *reinterpret_cast<const int4 *>(stage + (off + e4));
+            const int32_t vals[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+            for (int q = 0; q < 4; ++q) {
+                const int32_t e = e4 + q;
+                if (vals[q] == s0 && e < t1) {
+                    const int32_t lim = min(n_max, e + 1);
+                    int32_t m = 1;
+                    while (m < lim && stage[off + e - m] == s_suf[m]) ++m;
+                    if (m >= n_min) {
+                        const unsigned long long key = (static_cast<unsigned long long>(m) << 32) | uint32_t(e);
+                        best = key > best ? key : best;
+                    }
+                }
+            }
+        }
+        if (t + kStages < ntiles) {
+            __syncthreads();  // every thread is done with stage s
+            if (tid == 0) {
+                asm volatile("fence.proxy.async.shared::cta;\n" ::: "memory");
+                issue(t + kStages);
+            }
+        }
+    }
+    if (!ok) {
+        best = kTimeoutBit;
+        // Give the copies still in flight a second bounded wait before the CTA's memory goes away.
+        if (tid == 0)
+            for (int u = t; u < min(ntiles, t + kStages); ++u)
+                (void)mbar_wait(&bars[u % kStages], uint32_t(u / kStages) & 1u);
+    }
+
+    // CTA reduction (fixed order).
+    best = warp_max_u64(best);
+    zp = warp_sum_f32(zp);
+    if (lane == 0) {
+        s_wkey[warp] = best;
+        s_wz[warp] = zp;
+    }
+    __syncthreads();
+    unsigned long long cta_key = 0;
+    float cta_z = 0.f;
+    if (warp == 0) {
+        cta_key = lane < kStepWarps ? s_wkey[lane] : 0ull;
+        cta_z = lane < kStepWarps ? s_wz[lane] : 0.f;
+        cta_key = warp_max_u64(cta_key);
+        cta_z = warp_sum_f32(cta_z);
+    }
+
+    cluster_wait_acquire();  // phase 1: all CTAs of the cluster are running
+    if (tid == 0) {
+        st_cluster_u64(map_to_rank(&s_key[rank], 0), cta_key);
+        st_cluster_f32(map_to_rank(&s_zp[rank], 0), cta_z);
+    }
+    cluster_arrive_release();
+    cluster_wait_acquire();  // phase 2: every CTA's key and partial are in the leader
+    if (rank != 0) return;
+
+    if (tid == 0) {
+        unsigned long long key = 0;
+        float z = 0.f;
+        for (uint32_t r = 0; r < C; ++r) {
+            key = s_key[r] > key ? s_key[r] : key;
+            z += s_zp[r];
+        }
+        if (a.z_pre != nullptr) z = a.z_pre[b];
+        const bool timeout = (key & kTimeoutBit) != 0;
+        const bool hit = len_ok && !timeout && key != 0;
+        const int32_t n = hit ? int32_t(key >> 32) : 0;
+        const int32_t e = hit ? int32_t(key & 0xffffffffu) : -1;
+        const int32_t kappa = a.kappa > 0 ? a.kappa : a.n_min;
+        int32_t mode = SWITCHSD_MODE_NO_REP;
+        if (hit) mode = (n >= kappa && z >= a.logit_tau) ? SWITCHSD_MODE_COPY : SWITCHSD_MODE_REP_NO_COPY;
+        const int32_t len = mode == SWITCHSD_MODE_COPY ? min(a.k, L - 1 - e) : 0;
+        s_out[0] = mode;
+        s_out[1] = len;
+        s_out[2] = e;
+        a.out_mode[b] = mode;
+        a.out_len[b] = len;
+        a.out_score[b] = z;
+        if (a.out_match_n) a.out_match_n[b] = n;
+        if (a.out_match_end) a.out_match_end[b] = e;
+        if (a.status)
+            a.status[b] = !len_ok ? SWITCHSD_ROW_BAD_LEN : (timeout ? SWITCHSD_ROW_TIMEOUT : SWITCHSD_ROW_OK);
+    }
+    __syncthreads();
+    const int32_t len = s_out[1], e = s_out[2];
+    for (int i = tid; i < len; i += kStepThreads) a.out_draft[size_t(b) * a.k + i] = row[e + 1 + i];
+}
+
+// ------------------------------------------------------------------------------------------------
+// Two-layer probe z = w2 . ReLU(W1 h + b1) + b2 on CUDA cores (fp32 accumulation, fp32 hidden
+// layer).  Block = kMlpRows rows; warp w handles hidden units u = w, w + 8, ...; each lane streams
+// 16-byte slices of the W1 row and dots them with the rows' hidden vectors staged in shared memory.
+// ------------------------------------------------------------------------------------------------
+constexpr int kMlpRows = 4;
+constexpr int kMlpThreads = 256;
+
+struct MlpArgs {
+    const uint16_t *hidden;
+    const uint16_t *W1;
+    const uint16_t *w2;
+    const float *b1;
+    float b2;
+    int32_t B, d, H1;
+    float *z_out;
+};
+
+__global__ void __launch_bounds__(kMlpThreads) mlp_probe_kernel(const MlpArgs a) {
+    extern __shared__ __align__(16) uint4 hs[];  // kMlpRows x d/8
+    __shared__ float s_part[kMlpThreads / kWarp][kMlpRows];
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    const int row0 = blockIdx.x * kMlpRows;
+    const int nv = a.d >> 3;
+    for (int i = tid; i < kMlpRows * nv; i += kMlpThreads) {
+        const int r = i / nv, v = i % nv;
+        const int bb = row0 + r;
+        hs[i] = bb < a.B ? __ldg(reinterpret_cast<const uint4 *>(a.hidden + size_t(bb) * a.d) + v)
+                         : make_uint4(0, 0, 0, 0);
+    }
+    __syncthreads();
+    float zpart[kMlpRows];
+#pragma unroll
+    for (int r = 0; r < kMlpRows; ++r) zpart[r] = 0.f;
+    for (int u = warp; u < a.H1; u += kMlpThreads / kWarp) {
+        const uint4 *wrow = reinterpret_cast<const uint4 *>(a.W1 + size_t(u) * a.d);
+        float acc[kMlpRows];
+#pragma unroll
+        for (int r = 0; r < kMlpRows; ++r) acc[r] = 0.f;
+        for (int v = lane; v < nv; v += kWarp) {
+            const uint4 w = __ldg(wrow + v);
+#pragma unroll
+            for (int r = 0; r < kMlpRows; ++r) acc[r] = dot8_bf16(w, hs[r * nv + v], acc[r]);
+        }
+        const float bias = a.b1 ? a.b1[u] : 0.f;
+        const float w2u = bf16_lo(uint32_t(a.w2[u]));
+#pragma unroll
+        for (int r = 0; r < kMlpRows; ++r) {
+            const float pre = warp_sum_f32(acc[r]) + bias;
+            zpart[r] = fmaf(w2u, fmaxf(pre, 0.f), zpart[r]);
+        }
+    }
+    if (lane == 0)
+#pragma unroll
+        for (int r = 0; r < kMlpRows; ++r) s_part[warp][r] = zpart[r];
+    __syncthreads();
+    if (tid < kMlpRows && row0 + tid < a.B) {
+        float z = a.b2;
+        for (int w = 0; w < kMlpThreads / kWarp; ++w) z += s_part[w][tid];
+        a.z_out[row0 + tid] = z;
+    }
+}
+
+// ------------------------------------------------------------------------------------------------
+// Host side.
+// ------------------------------------------------------------------------------------------------
+static int sm_count_cached() {
+    static int counts[64] = {0};
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return 0;
+    if (counts[dev] == 0) {
+        int n = 0;
+        if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) return 0;
+        counts[dev] = n;
+    }
+    return counts[dev];
+}
+
+static bool aligned16(const void *p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+// CTAs per row: the smallest power of two giving at least two CTAs per SM over the batch, with at
+// least 1024 tokens of capacity per CTA, at most kMaxSplit.
+static int choose_split(int B, int cap) {
+    const int sms = sm_count_cached() > 0 ? sm_count_cached() : 148;
+    int c = 1;
+    while (c < kMaxSplit && int64_t(B) * c < 2ll * sms && cap / (2 * c) >= 1024) c *= 2;
+    return c;
+}
+
+static cudaError_t launch_step(const StepArgs &args, int split, cudaStream_t stream) {
+    static bool attr_done[64] = {false};
+    int dev = 0;
+    cudaGetDevice(&dev);
+    if (dev >= 0 && dev < 64 && !attr_done[dev]) {
+        cudaError_t e = cudaFuncSetAttribute(step_kernel, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
+        if (e != cudaSuccess) return e;
+        attr_done[dev] = true;
+    }
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(unsigned(split), unsigned(args.B), 1);
+    cfg.blockDim = dim3(kStepThreads, 1, 1);
+    cfg.dynamicSmemBytes = kStepSmemBytes;
+    cfg.stream = stream;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = unsigned(split);
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, step_kernel, args);
+}
+
+static cudaError_t launch_mlp(const MlpArgs &m, cudaStream_t stream) {
+    const size_t smem = size_t(kMlpRows) * size_t(m.d) * 2;
+    static bool attr_done[64] = {false};
+    int dev = 0;
+    cudaGetDevice(&dev);
+    if (smem > 48 * 1024 && dev >= 0 && dev < 64 && !attr_done[dev]) {
+        cudaError_t e = cudaFuncSetAttribute(mlp_probe_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                             200 * 1024);
+        if (e != cudaSuccess) return e;
+        attr_done[dev] = true;
+    }
+    mlp_probe_kernel<<<(m.B + kMlpRows - 1) / kMlpRows, kMlpThreads, smem, stream>>>(m);
+    return cudaGetLastError();
+}
+
+}  // namespace switchsd
+
+using namespace switchsd;
+
+extern "C" int switchsd_step(const int32_t *ctx_tokens, const int32_t *ctx_lens, const uint16_t *hidden,
+                             const uint16_t *probe_w, const switchsd_params *p, int32_t *out_draft,
+                             int32_t *out_len, int32_t *out_mode, float *out_score) {
+    if (!p || !ctx_tokens || !ctx_lens || !hidden || !probe_w || !out_draft || !out_len || !out_mode ||
+        !out_score)
+        return SWITCHSD_ERR_ARG;
+    if (!aligned16(ctx_tokens) || !aligned16(hidden) || !aligned16(probe_w)) return SWITCHSD_ERR_ARG;
+    if (p->probe_kind != SWITCHSD_PROBE_LINEAR && p->probe_kind != SWITCHSD_PROBE_MLP) return SWITCHSD_ERR_ARG;
+    if (p->B < 1 || p->B > 65535 || p->cap < 4 || (p->cap & 3) != 0) return SWITCHSD_ERR_SHAPE;
+    if (p->d < 8 || (p->d & 7) != 0) return SWITCHSD_ERR_SHAPE;
+    if (p->k < 1 || p->k > SWITCHSD_KMAX) return SWITCHSD_ERR_SHAPE;
+    if (p->n_min < 1 || p->n_max > SWITCHSD_NMAX || p->n_min > p->n_max) return SWITCHSD_ERR_SHAPE;
+    if (p->split != 0 && p->split != 1 && p->split != 2 && p->split != 4 && p->split != 8 && p->split != 16)
+        return SWITCHSD_ERR_SHAPE;
+    if (p->probe_kind == SWITCHSD_PROBE_MLP && (p->probe_hidden < 1 || p->probe_hidden > 1024))
+        return SWITCHSD_ERR_SHAPE;
+    if (p->probe_kind == SWITCHSD_PROBE_MLP && size_t(kMlpRows) * size_t(p->d) * 2 > 200 * 1024)
+        return SWITCHSD_ERR_SHAPE;
+
+    cudaStream_t stream = static_cast<cudaStream_t>(p->stream);
+    StepArgs args;
+    args.ctx = ctx_tokens;
+    args.lens = ctx_lens;
+    args.hidden = hidden;
+    args.probe_w = probe_w;
+    args.z_pre = nullptr;
+    args.B = p->B;
+    args.cap = p->cap;
+    args.d = p->d;
+    args.k = p->k;
+    args.n_min = p->n_min;
+    args.n_max = p->n_max;
+    args.kappa = p->kappa;
+    args.logit_tau = p->logit_tau;
+    args.out_draft = out_draft;
+    args.out_len = out_len;
+    args.out_mode = out_mode;
+    args.out_score = out_score;
+    args.out_match_n = p->out_match_n;
+    args.out_match_end = p->out_match_end;
+    args.status = p->status;
+
+    if (p->probe_kind == SWITCHSD_PROBE_MLP) {
+        MlpArgs m;
+        m.hidden = hidden;
+        m.W1 = probe_w;
+        m.w2 = probe_w + size_t(p->probe_hidden) * size_t(p->d);
+        m.b1 = p->b1;
+        m.b2 = p->b2;
+        m.B = p->B;
+        m.d = p->d;
+        m.H1 = p->probe_hidden;
+        m.z_out = out_score;
+        if (launch_mlp(m, stream) != cudaSuccess) return SWITCHSD_ERR_CUDA;
+        args.z_pre = out_score;
+    }
+    const int split = p->split > 0 ? p->split : choose_split(p->B, p->cap);
+    if (launch_step(args, split, stream) != cudaSuccess) return SWITCHSD_ERR_CUDA;
+    return SWITCHSD_OK;
+}

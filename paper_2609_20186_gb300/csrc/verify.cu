@@ -1,0 +1,91 @@
+// verify.cu -- switchsd_verify: greedy verification and append (§3.3 "Parallel Verification",
+// temperature 0 as in App. A).
+//
+// One warp per row.  Lanes compare draft[i] with the target's greedy token 32 indices at a time; the
+// first set bit of the ballot of mismatches is the accepted length a.  Lanes then append
+// draft[0..a) and target[a] at ctx[L..L+a] and lane 0 publishes L + a + 1.  The work is O(B k)
+// bytes: latency-bound by design.
+#include "common.cuh"
+
+namespace switchsd {
+
+constexpr int kVerifyThreads = 256;
+
+struct VerifyArgs {
+    const int32_t *draft;
+    const int32_t *target;
+    const int32_t *draft_len;
+    int32_t *ctx;
+    int32_t *lens;
+    int32_t *out_accept;
+    int32_t *status;
+    int32_t B, cap, k;
+};
+
+__global__ void __launch_bounds__(kVerifyThreads) verify_kernel(const VerifyArgs a) {
+    const int lane = threadIdx.x & 31;
+    const int b = (blockIdx.x * kVerifyThreads + threadIdx.x) >> 5;
+    if (b >= a.B) return;
+    const int32_t len = a.draft_len[b];
+    const int32_t L = a.lens[b];
+    if (len < 0 || len > a.k || L < 1 || L > a.cap) {
+        if (lane == 0) {
+            a.out_accept[b] = -1;
+            if (a.status) a.status[b] = SWITCHSD_ROW_BAD_LEN;
+        }
+        return;
+    }
+    const int32_t *dr = a.draft + size_t(b) * a.k;
+    const int32_t *tg = a.target + size_t(b) * (a.k + 1);
+    int32_t acc = len;
+    for (int base = 0; base < len; base += kWarp) {
+        const int i = base + lane;
+        const bool mismatch = i < len && dr[i] != tg[i];
+        const unsigned m = __ballot_sync(kFull, mismatch);
+        if (m) {
+            acc = base + __ffs(m) - 1;
+            break;
+        }
+    }
+    if (L + acc + 1 > a.cap) {
+        if (lane == 0) {
+            a.out_accept[b] = -1;
+            if (a.status) a.status[b] = SWITCHSD_ROW_CAPACITY;
+        }
+        return;
+    }
+    int32_t *row = a.ctx + size_t(b) * size_t(a.cap) + L;
+    for (int i = lane; i <= acc; i += kWarp) row[i] = i < acc ? dr[i] : tg[acc];
+    if (lane == 0) {
+        a.lens[b] = L + acc + 1;
+        a.out_accept[b] = acc;
+        if (a.status) a.status[b] = SWITCHSD_ROW_OK;
+    }
+}
+
+}  // namespace switchsd
+
+using namespace switchsd;
+
+extern "C" int switchsd_verify(const int32_t *draft, const int32_t *target_argmax, int32_t *out_accept,
+                               const switchsd_verify_params *vp) {
+    if (!vp || !draft || !target_argmax || !out_accept || !vp->draft_len || !vp->ctx_tokens || !vp->ctx_lens)
+        return SWITCHSD_ERR_ARG;
+    if (vp->B < 1 || vp->cap < 4 || (vp->cap & 3) != 0 || vp->k < 1 || vp->k > SWITCHSD_KMAX)
+        return SWITCHSD_ERR_SHAPE;
+    VerifyArgs a;
+    a.draft = draft;
+    a.target = target_argmax;
+    a.draft_len = vp->draft_len;
+    a.ctx = vp->ctx_tokens;
+    a.lens = vp->ctx_lens;
+    a.out_accept = out_accept;
+    a.status = vp->status;
+    a.B = vp->B;
+    a.cap = vp->cap;
+    a.k = vp->k;
+    const int warps_per_block = kVerifyThreads / kWarp;
+    const int blocks = (vp->B + warps_per_block - 1) / warps_per_block;
+    verify_kernel<<<blocks, kVerifyThreads, 0, static_cast<cudaStream_t>(vp->stream)>>>(a);
+    return cudaGetLastError() == cudaSuccess ? SWITCHSD_OK : SWITCHSD_ERR_CUDA;
+}

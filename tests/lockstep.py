@@ -1,0 +1,123 @@
+"""Lockstep drivers used by the parity tests.
+
+The oracle side and the GPU side each run the full decoding loop on their own state, from the same
+seeded inputs (synth): step -> harness (target stand-in) -> verify.  Nothing computed by one side is
+fed to the other; the tests compare the two traces step by step.
+
+Near-threshold rule (the reading stated in the design doc): if the modes differ and the oracle's logit is
+within 1e-3 of logit(tau), the row is a permitted flip; both sides have taken a valid decision, their
+contexts diverge from then on, and the row is compared no further.  Any other difference fails.
+"""
+from __future__ import annotations
+
+import numpy as np
+
+import oracle
+import synth
+
+SCORE_TOL = 1e-3
+
+
+def oracle_trace(wl: synth.Workload, rows, steps: int, ctx=None, lens=None):
+    """Runs the oracle loop on the given rows; returns a list (per step) of dicts of per-row arrays
+    plus the final ctx / lens."""
+    if ctx is None:
+        ctx, lens = wl.contexts()
+    ctx = ctx.copy()
+    lens = lens.copy()
+    labels = wl.labels()
+    pw = wl.probe_weights()
+    hp = wl.harness_params()
+    rows = list(rows)
+    trace = []
+    for t in range(steps):
+        h = wl.hidden(t)
+        out = None
+        for b in rows:
+            o = oracle.step(ctx, lens, h, pw, k=wl.k, n_min=wl.n_min, n_max=wl.n_max,
+                            kappa=wl.kappa, logit_tau=wl.logit_tau, probe_kind=wl.probe_kind,
+                            probe_hidden=wl.probe_hidden, rows=(b, b + 1))
+            if out is None:
+                out = o
+            else:
+                for key in out:
+                    out[key][b] = o[key][b]
+        vd, vl, tg = synth.harness_targets(hp, t, lens, out["mode"], out["draft"], out["len"],
+                                           labels, rows=rows)
+        acc = np.zeros(wl.B, np.int32)
+        st = np.zeros(wl.B, np.int32)
+        for b in rows:
+            a, s = oracle.verify(ctx, lens, vd, vl, tg, rows=(b, b + 1))
+            acc[b], st[b] = a[b], s[b]
+        out["accept"] = acc
+        out["vstatus"] = st
+        out["lens_after"] = lens.copy()
+        trace.append(out)
+    return trace, ctx, lens
+
+
+def gpu_trace(wl: synth.Workload, steps: int, split: int = 0, ctx=None, lens=None, device="cuda"):
+    """Runs the GPU loop on all rows; returns the per-step host copies of every output."""
+    import torch
+    from paper_2609_20186_gb300 import Session, bf16_tensor
+
+    if ctx is None:
+        ctx, lens = wl.contexts()
+    sess = Session(ctx, lens, wl.probe_weights(), k=wl.k, n_min=wl.n_min, n_max=wl.n_max,
+                   kappa=wl.kappa, logit_tau=wl.logit_tau, probe_kind=wl.probe_kind,
+                   probe_hidden=wl.probe_hidden, labels=wl.labels(), harness=wl.harness_params(),
+                   split=split, device=device)
+    trace = []
+    for t in range(steps):
+        hidden = bf16_tensor(wl.hidden(t), sess.device)
+        sess.step(hidden)
+        out = sess.step_outputs()
+        sess.harness(t)
+        sess.verify()
+        out["accept"] = sess.accept.cpu().numpy()
+        out["vstatus"] = sess.vstatus.cpu().numpy()
+        out["lens_after"] = sess.lens.cpu().numpy()
+        trace.append(out)
+    torch.cuda.synchronize()
+    return trace, sess.ctx.cpu().numpy(), sess.lens.cpu().numpy()
+
+
+def compare(wl: synth.Workload, o_trace, g_trace, rows, o_ctx=None, g_ctx=None):
+    """Asserts parity on the given rows; returns (flips, stats)."""
+    kappa = wl.kappa_eff
+    active = set(rows)
+    flips = []
+    stats = {"copy": 0, "rep_no_copy": 0, "no_rep": 0, "checked": 0}
+    for t, (o, g) in enumerate(zip(o_trace, g_trace)):
+        for b in sorted(active):
+            where = f"{wl.name} step {t} row {b}"
+            assert g["status"][b] == 0, where
+            # integer outputs of the search: bit-exact
+            assert g["match_n"][b] == o["match_n"][b], (where, g["match_n"][b], o["match_n"][b])
+            assert g["match_end"][b] == o["match_end"][b], (where, g["match_end"][b],
+                                                            o["match_end"][b])
+            # probe logit within tolerance
+            assert abs(float(g["score"][b]) - float(o["score"][b])) <= SCORE_TOL, \
+                (where, g["score"][b], o["score"][b])
+            if g["mode"][b] != o["mode"][b]:
+                near = abs(float(o["score"][b]) - wl.logit_tau) <= SCORE_TOL
+                both_match = o["match_n"][b] >= kappa
+                assert near and both_match, (where, "switch flip outside the threshold band",
+                                             g["mode"][b], o["mode"][b], o["score"][b])
+                flips.append((t, b))
+                active.discard(b)
+                continue
+            m = int(o["mode"][b])
+            stats[("no_rep", "copy", "rep_no_copy")[m]] += 1
+            assert g["len"][b] == o["len"][b], where
+            ln = int(o["len"][b])
+            assert np.array_equal(g["draft"][b, :ln], o["draft"][b, :ln]), where
+            assert g["accept"][b] == o["accept"][b], (where, g["accept"][b], o["accept"][b])
+            assert g["vstatus"][b] == o["vstatus"][b], where
+            assert g["lens_after"][b] == o["lens_after"][b], where
+            stats["checked"] += 1
+    if o_ctx is not None and g_ctx is not None:
+        for b in active:
+            L = int(o_trace[-1]["lens_after"][b])
+            assert np.array_equal(o_ctx[b, :L], g_ctx[b, :L]), f"{wl.name} final context row {b}"
+    return flips, stats

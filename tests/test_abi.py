@@ -1,0 +1,118 @@
+"""The C ABI library without a GPU: it loads, exports every function include/*.h declares, and its
+host-side validation returns the documented codes before any CUDA call is made."""
+import ctypes
+import math
+import os
+import re
+import subprocess
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+INCLUDE = os.path.join(ROOT, "include")
+
+
+@pytest.fixture(scope="module")
+def lib():
+    from paper_2609_20186_gb300 import build, binding
+    build.build()
+    return binding.load()
+
+
+def declared_functions():
+    names = set()
+    for f in os.listdir(INCLUDE):
+        if not f.endswith(".h"):
+            continue
+        text = open(os.path.join(INCLUDE, f)).read()
+        text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+        for m in re.finditer(r"\b(switchsd_\w+)\s*\(", text):
+            names.add(m.group(1))
+    return sorted(names)
+
+
+def test_headers_declare_the_boundary():
+    names = declared_functions()
+    for must in ("switchsd_step", "switchsd_verify", "switchsd_strerror", "switchsd_abi_version",
+                 "switchsd_harness_target"):
+        assert must in names
+
+
+def test_every_declared_symbol_is_exported(lib):
+    from paper_2609_20186_gb300 import build
+    out = subprocess.run(["nm", "-D", "--defined-only", build.LIB], capture_output=True, text=True,
+                         check=True).stdout
+    exported = {line.split()[-1] for line in out.splitlines() if line.strip()}
+    for name in declared_functions():
+        assert name in exported, name
+        assert hasattr(lib, name)
+
+
+def test_abi_version_and_strerror(lib):
+    from paper_2609_20186_gb300 import binding as bd
+    assert bd.abi_version() == 1
+    for code in (0, -1, -2, -3, 1, 2, 3):
+        assert bd.strerror(code) != "unknown code"
+    assert bd.strerror(12345) == "unknown code"
+
+
+def _params(**kw):
+    from paper_2609_20186_gb300 import binding as bd
+    p = bd.switchsd_params()
+    p.B, p.cap, p.d, p.k, p.n_min, p.n_max = 4, 64, 16, 8, 3, 8
+    p.logit_tau = 0.0
+    for key, v in kw.items():
+        setattr(p, key, v)
+    return p
+
+
+FAKE = 0x10000  # a 16-byte-aligned non-NULL address; never dereferenced by host validation
+
+
+def _step(lib, p, ctx=FAKE, hidden=FAKE, probe=FAKE, lens=FAKE):
+    return lib.switchsd_step(ctx, lens, hidden, probe, ctypes.byref(p) if p is not None else None,
+                             FAKE, FAKE, FAKE, FAKE)
+
+
+def test_step_validation(lib):
+    from paper_2609_20186_gb300 import binding as bd
+    assert _step(lib, None) == bd.ERR_ARG
+    assert _step(lib, _params(), ctx=0) == bd.ERR_ARG
+    assert _step(lib, _params(), ctx=FAKE + 4) == bd.ERR_ARG          # misaligned rows
+    assert _step(lib, _params(), hidden=FAKE + 2) == bd.ERR_ARG
+    assert _step(lib, _params(probe_kind=7)) == bd.ERR_ARG
+    assert _step(lib, _params(B=0)) == bd.ERR_SHAPE
+    assert _step(lib, _params(cap=66)) == bd.ERR_SHAPE                 # cap % 4 != 0
+    assert _step(lib, _params(d=12)) == bd.ERR_SHAPE                   # d % 8 != 0
+    assert _step(lib, _params(k=0)) == bd.ERR_SHAPE
+    assert _step(lib, _params(k=65)) == bd.ERR_SHAPE
+    assert _step(lib, _params(n_min=0)) == bd.ERR_SHAPE
+    assert _step(lib, _params(n_min=5, n_max=4)) == bd.ERR_SHAPE
+    assert _step(lib, _params(n_max=33)) == bd.ERR_SHAPE
+    assert _step(lib, _params(split=3)) == bd.ERR_SHAPE
+    assert _step(lib, _params(probe_kind=1, probe_hidden=0)) == bd.ERR_SHAPE
+
+
+def test_verify_validation(lib):
+    from paper_2609_20186_gb300 import binding as bd
+    vp = bd.switchsd_verify_params()
+    vp.B, vp.cap, vp.k = 4, 64, 8
+    vp.draft_len = vp.ctx_tokens = vp.ctx_lens = FAKE
+    assert lib.switchsd_verify(FAKE, FAKE, FAKE, None) == bd.ERR_ARG
+    assert lib.switchsd_verify(0, FAKE, FAKE, ctypes.byref(vp)) == bd.ERR_ARG
+    vp.k = 0
+    assert lib.switchsd_verify(FAKE, FAKE, FAKE, ctypes.byref(vp)) == bd.ERR_SHAPE
+    vp.k, vp.cap = 8, 63
+    assert lib.switchsd_verify(FAKE, FAKE, FAKE, ctypes.byref(vp)) == bd.ERR_SHAPE
+    vp.cap, vp.ctx_lens = 64, None
+    assert lib.switchsd_verify(FAKE, FAKE, FAKE, ctypes.byref(vp)) == bd.ERR_ARG
+
+
+def test_binding_rejects_cpu_tensors(lib):
+    import torch
+    from paper_2609_20186_gb300 import binding as bd
+    t = torch.zeros(2, 8, dtype=torch.int32)
+    with pytest.raises(TypeError):
+        bd.switchsd_verify(t, torch.zeros(2, 9, dtype=torch.int32), torch.zeros(2, dtype=torch.int32),
+                           draft_len=torch.zeros(2, dtype=torch.int32), ctx_tokens=t,
+                           ctx_lens=torch.zeros(2, dtype=torch.int32))

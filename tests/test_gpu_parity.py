@@ -1,0 +1,170 @@
+"""GPU path vs the CPU oracle, through the C ABI (libswitchsd.so via the ctypes binding).
+
+Bar: bit-exact on match length / end position, modes, draft tokens, accepted lengths and contexts;
+probe logits within 1e-3 absolute; no switch flip outside 1e-3 of the threshold (lockstep.compare).
+
+Small cases compare every row at every step and span several staged tiles with ragged tails; the
+full-size workloads run every row on the GPU in the launch configuration the benchmark uses, and the
+oracle replays a sample of rows (rows are independent, so a replayed row is exact).
+"""
+import numpy as np
+import pytest
+
+import synth
+from tests import lockstep
+
+pytestmark = pytest.mark.gpu
+
+W = synth.WORKLOADS
+
+SMALL = {
+    "uniform_small": W["uniform_8k"].scaled(name="uniform_small", B=8, L0=3000, steps=20),
+    "zipf_small": W["zipf_32k"].scaled(name="zipf_small", B=8, L0=9001, steps=24),
+    "code_small": W["code_16k"].scaled(name="code_small", B=12, L0=5000, steps=16),
+    "mixed_small": W["mixed_128k"].scaled(name="mixed_small", B=4, L0=20003, steps=12),
+    "zipf_kappa5": W["zipf_32k"].scaled(name="zipf_kappa5", B=8, L0=6000, steps=16, kappa=5),
+}
+
+
+def _run_small(wl, split=0):
+    rows = range(wl.B)
+    o_trace, o_ctx, _ = lockstep.oracle_trace(wl, rows, wl.steps)
+    g_trace, g_ctx, _ = lockstep.gpu_trace(wl, wl.steps, split=split)
+    return lockstep.compare(wl, o_trace, g_trace, rows, o_ctx, g_ctx)
+
+
+@pytest.mark.parametrize("name", list(SMALL))
+def test_small_lockstep(name):
+    flips, stats = _run_small(SMALL[name])
+    assert stats["checked"] > 0
+    assert len(flips) <= 1
+
+
+@pytest.mark.parametrize("split", [1, 2, 4, 8, 16])
+def test_split_invariance(split):
+    wl = SMALL["zipf_small"].scaled(steps=8)
+    _run_small(wl, split=split)
+
+
+@pytest.mark.parametrize("variant", ["copy", "nocopy", "norep"])
+def test_planted(variant):
+    wl = W[f"planted_{variant}"]
+    exp = wl.expected_planted()
+    o_trace, o_ctx, _ = lockstep.oracle_trace(wl, [0], 1)
+    g_trace, g_ctx, g_lens = lockstep.gpu_trace(wl, 1)
+    lockstep.compare(wl, o_trace, g_trace, [0], o_ctx, g_ctx)
+    g = g_trace[0]
+    assert g["mode"][0] == exp["mode"]
+    assert g["match_n"][0] == exp["match_n"] and g["match_end"][0] == exp["match_end"]
+    assert g["draft"][0, : g["len"][0]].tolist() == exp["draft"]
+    assert g["accept"][0] == exp["accept"] and g_lens[0] == wl.L0 + exp["accept"] + 1
+
+
+FULL_ROWS = {"uniform_8k": [0, 31, 63], "zipf_32k": [0, 29, 63], "code_16k": [0, 101, 255],
+             "mixed_128k": [0, 7, 15]}
+
+
+@pytest.mark.parametrize("name", list(FULL_ROWS))
+def test_full_size_sampled_rows(name):
+    wl = W[name]
+    rows = FULL_ROWS[name]
+    g_trace, g_ctx, _ = lockstep.gpu_trace(wl, wl.steps)
+    o_trace, o_ctx, _ = lockstep.oracle_trace(wl, rows, wl.steps)
+    flips, stats = lockstep.compare(wl, o_trace, g_trace, rows, o_ctx, g_ctx)
+    assert stats["checked"] >= (len(rows) - len(flips)) * 1
+    # every row of the batch stayed healthy on the GPU
+    for t in g_trace:
+        assert np.all(t["status"] == 0) and np.all(t["vstatus"] == 0)
+        assert np.all(t["len"] <= wl.k)
+
+
+def test_threshold_extremes():
+    """tau -> 0 (logit -inf) copies on every kappa-match (prompt-lookup decoding); tau -> 1 never
+    copies."""
+    base = SMALL["zipf_small"].scaled(steps=6)
+    for tau, expect_copy in ((0.0, True), (1.0, False)):
+        wl = base.scaled(tau=tau)
+        _, _ = _run_small(wl)
+        g_trace, _, _ = lockstep.gpu_trace(wl, wl.steps)
+        for t in g_trace:
+            hit = t["match_n"] >= wl.kappa_eff
+            if expect_copy:
+                assert np.array_equal(t["mode"] == 1, hit)
+            else:
+                assert not np.any(t["mode"] == 1)
+
+
+def test_edge_lengths_and_status():
+    """Rows of length 1, 2, n_min, n_min + 1, a full row and out-of-range lengths in one batch."""
+    import torch
+    from paper_2609_20186_gb300 import Session, bf16_tensor
+    import oracle
+
+    wl = W["uniform_8k"].scaled(B=10, L0=256, steps=1)
+    ctx, _ = wl.contexts()
+    ctx[:, :] = np.random.default_rng(0).integers(0, 3, ctx.shape)   # dense small-alphabet repeats
+    cap = wl.cap
+    lens = np.array([1, 2, 3, 4, 9, cap - 4, cap, 0, cap + 1, -7], np.int32)
+    sess = Session(ctx, lens, wl.probe_weights(), k=wl.k, n_min=wl.n_min, n_max=wl.n_max,
+                   logit_tau=wl.logit_tau, labels=wl.labels(), harness=wl.harness_params())
+    h = wl.hidden(0)
+    sess.step(bf16_tensor(h, sess.device))
+    g = sess.step_outputs()
+    for b in range(7):
+        o = oracle.step(ctx, lens, h, wl.probe_weights(), k=wl.k, n_min=wl.n_min, n_max=wl.n_max,
+                        logit_tau=wl.logit_tau, rows=(b, b + 1))
+        assert g["status"][b] == 0
+        assert (g["match_n"][b], g["match_end"][b]) == (o["match_n"][b], o["match_end"][b]), b
+        assert g["mode"][b] == o["mode"][b] and g["len"][b] == o["len"][b]
+        assert np.array_equal(g["draft"][b, : g["len"][b]], o["draft"][b, : o["len"][b]])
+    for b in range(7, 10):
+        assert g["status"][b] == 2 and g["mode"][b] == 0 and g["len"][b] == 0
+    # verification: the full row (L = cap) cannot take even the bonus token
+    sess.vdraft.zero_()
+    sess.target.zero_()
+    sess.vlen.zero_()
+    sess.vlen[5] = 3
+    sess.target[5, :4] = torch.tensor([0, 0, 0, 9], dtype=torch.int32, device=sess.device)
+    before = sess.ctx.clone()
+    sess.verify()
+    acc = sess.accept.cpu().numpy()
+    st = sess.vstatus.cpu().numpy()
+    ln = sess.lens.cpu().numpy()
+    assert st[6] == 1 and acc[6] == -1 and ln[6] == cap
+    assert torch.equal(sess.ctx[6], before[6])
+    # row 5: L = cap - 4, accepts 3 zeros, appends 9 -> exactly full
+    assert st[5] == 0 and acc[5] == 3 and ln[5] == cap
+    assert sess.ctx[5, cap - 4:].tolist() == [0, 0, 0, 9]
+    # rows 0..4: empty drafts append target[0] = 0
+    assert np.all(acc[:5] == 0) and np.all(ln[:5] == lens[:5] + 1)
+    for b in range(7, 10):
+        assert st[b] == 2 and acc[b] == -1
+
+
+def test_device_harness_matches_host():
+    import torch
+    from paper_2609_20186_gb300 import binding as bd
+
+    wl = W["zipf_32k"].scaled(B=64, steps=8)
+    rng = np.random.default_rng(1)
+    B, k = wl.B, wl.k
+    lens = (wl.L0 + rng.integers(0, 50, B)).astype(np.int32)
+    mode = rng.integers(0, 3, B).astype(np.int32)
+    draft = rng.integers(0, wl.V, (B, k)).astype(np.int32)
+    dlen = np.where(mode == 1, rng.integers(1, k + 1, B), 0).astype(np.int32)
+    labels = (rng.random((B, wl.cap - wl.L0)) < 0.5).astype(np.uint8)
+    hp = wl.harness_params()
+    for step in (0, 5):
+        vd, vl, tg = synth.harness_targets(hp, step, lens, mode, draft, dlen, labels)
+        dev = {n: torch.from_numpy(a).cuda() for n, a in
+               (("lens", lens), ("mode", mode), ("draft", draft), ("dlen", dlen), ("labels", labels))}
+        gvd = torch.zeros(B, k, dtype=torch.int32, device="cuda")
+        gvl = torch.zeros(B, dtype=torch.int32, device="cuda")
+        gtg = torch.zeros(B, k + 1, dtype=torch.int32, device="cuda")
+        bd.switchsd_harness_target(dev["lens"], dev["mode"], dev["draft"], dev["dlen"], dev["labels"],
+                                   gvd, gvl, gtg, step=step, **{x: hp[x] for x in
+                                                                ("seed", "V", "L0", "agree_cap",
+                                                                 "thr_in", "thr_out")})
+        assert np.array_equal(gvd.cpu().numpy(), vd)
+        assert np.array_equal(gvl.cpu().numpy(), vl)
+        assert np.array_equal(gtg.cpu().numpy(), tg)
