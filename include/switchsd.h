@@ -11,7 +11,9 @@
  *                    Generation");
  *   switchsd_verify  greedy verification and append (§3.3 "Parallel Verification", temperature 0 as
  *                    in App. A): accepted prefix length, then the accepted tokens and the target's own
- *                    next token are appended to the context.
+ *                    next token are appended to the context;
+ *   switchsd_verify_step  both, fused into one launch (verification of the previous draft, then the
+ *                    next step).
  *
  * The target model and the neural drafter are outside the library; their outputs (hidden state at the
  * probed layer, the target's greedy tokens, the neural draft) arrive as arguments.
@@ -159,6 +161,28 @@ typedef struct {
  */
 int switchsd_verify(const int32_t *draft, const int32_t *target_argmax, int32_t *out_accept,
                     const switchsd_verify_params *vp);
+
+/*
+ * One controller iteration in one launch (§3.3 "Overall Framework": after every verification step the
+ * controller decides the next draft, Fig. 1): greedy verification and append of the previous draft,
+ * exactly as switchsd_verify, then switchsd_step on the extended context.  The result equals
+ * switchsd_verify followed by switchsd_step with the same arguments, at the cost of one launch.
+ *
+ *   draft, target_argmax, draft_len  the previous iteration's verified draft, as for switchsd_verify
+ *                 (device int32 [B, k], [B, k+1], [B])
+ *   out_accept    device int32 [B]: accepted length a, or -1 if the append did not fit / bad lengths
+ *   ctx_tokens, ctx_lens   device, modified in place by the append, then searched by the step
+ *   hidden, probe_w, params, out_draft, out_len, out_mode, out_score   as for switchsd_step
+ *
+ * params->status receives SWITCHSD_ROW_CAPACITY when the append did not fit (the step then runs on
+ * the unchanged context), SWITCHSD_ROW_BAD_LEN for a bad ctx_lens[b] or draft_len[b], else the step's
+ * status.  The draft buffers must not alias out_draft.
+ */
+int switchsd_verify_step(const int32_t *draft, const int32_t *target_argmax, const int32_t *draft_len,
+                         int32_t *out_accept, int32_t *ctx_tokens, int32_t *ctx_lens,
+                         const uint16_t *hidden, const uint16_t *probe_w,
+                         const switchsd_params *params, int32_t *out_draft, int32_t *out_len,
+                         int32_t *out_mode, float *out_score);
 
 /* Human-readable text of a host return code or a row status (static storage, never NULL). */
 const char *switchsd_strerror(int code);

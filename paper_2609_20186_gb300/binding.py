@@ -48,8 +48,8 @@ class switchsd_verify_params(ctypes.Structure):
 class switchsd_harness_params(ctypes.Structure):
     _fields_ = [
         ("B", ctypes.c_int32), ("k", ctypes.c_int32), ("V", ctypes.c_int32), ("L0", ctypes.c_int32),
-        ("n_labels", ctypes.c_int32), ("agree_cap", ctypes.c_int32), ("step", ctypes.c_int32),
-        ("seed", ctypes.c_uint64), ("thr_in", ctypes.c_uint64), ("thr_out", ctypes.c_uint64),
+        ("n_future", ctypes.c_int32), ("gamma", ctypes.c_int32), ("step", ctypes.c_int32),
+        ("seed", ctypes.c_uint64), ("thr_neural", ctypes.c_uint64),
         ("stream", ctypes.c_void_p),
     ]
 
@@ -63,6 +63,8 @@ _SIGNATURES = {
                       + [ctypes.c_void_p] * 4),
     "switchsd_verify": (ctypes.c_int, [ctypes.c_void_p] * 3
                         + [ctypes.POINTER(switchsd_verify_params)]),
+    "switchsd_verify_step": (ctypes.c_int, [ctypes.c_void_p] * 8 + [ctypes.POINTER(switchsd_params)]
+                             + [ctypes.c_void_p] * 4),
     "switchsd_strerror": (ctypes.c_char_p, [ctypes.c_int]),
     "switchsd_abi_version": (ctypes.c_int, []),
     "switchsd_harness_target": (ctypes.c_int, [ctypes.c_void_p] * 8
@@ -162,6 +164,40 @@ def switchsd_step(ctx_tokens, ctx_lens, hidden, probe_w, out_draft, out_len, out
     _check(code, "switchsd_step")
 
 
+def switchsd_verify_step(draft, target_argmax, draft_len, out_accept, ctx_tokens, ctx_lens, hidden,
+                         probe_w, out_draft, out_len, out_mode, out_score, *, k: int, n_min: int,
+                         n_max: int, kappa: int = 0, logit_tau: float = 0.0,
+                         probe_kind: int = PROBE_LINEAR, probe_hidden: int = 0, b1=None,
+                         b2: float = 0.0, split: int = 0, out_match_n=None, out_match_end=None,
+                         status=None, stream=None) -> None:
+    """switchsd_verify_step of include/switchsd.h: verification of the previous draft, then the next
+    step, in one launch."""
+    B, cap = ctx_tokens.shape
+    d = hidden.shape[1]
+    p = switchsd_params()
+    p.B, p.cap, p.d, p.k = B, cap, d, k
+    p.n_min, p.n_max, p.kappa = n_min, n_max, kappa
+    p.logit_tau = logit_tau
+    p.probe_kind, p.probe_hidden = probe_kind, probe_hidden
+    p.b1 = _dev(b1, torch.float32, "b1", (probe_hidden,)) if b1 is not None else None
+    p.b2 = b2
+    p.split = split
+    p.out_match_n = _dev(out_match_n, torch.int32, "out_match_n", (B,))
+    p.out_match_end = _dev(out_match_end, torch.int32, "out_match_end", (B,))
+    p.status = _dev(status, torch.int32, "status", (B,))
+    p.stream = _stream_ptr(stream)
+    nw = d if probe_kind == PROBE_LINEAR else probe_hidden * d + probe_hidden
+    code = load().switchsd_verify_step(
+        _dev(draft, torch.int32, "draft", (B, k)),
+        _dev(target_argmax, torch.int32, "target_argmax", (B, k + 1)),
+        _dev(draft_len, torch.int32, "draft_len", (B,)), _dev(out_accept, torch.int32, "out_accept", (B,)),
+        _dev(ctx_tokens, torch.int32, "ctx_tokens"), _dev(ctx_lens, torch.int32, "ctx_lens", (B,)),
+        _bf16(hidden, "hidden", (B, d)), _bf16(probe_w, "probe_w", (nw,)), ctypes.byref(p),
+        _dev(out_draft, torch.int32, "out_draft", (B, k)), _dev(out_len, torch.int32, "out_len", (B,)),
+        _dev(out_mode, torch.int32, "out_mode", (B,)), _dev(out_score, torch.float32, "out_score", (B,)))
+    _check(code, "switchsd_verify_step")
+
+
 def switchsd_verify(draft, target_argmax, out_accept, *, draft_len, ctx_tokens, ctx_lens,
                     status=None, stream=None) -> None:
     """switchsd_verify of include/switchsd.h on torch tensors."""
@@ -180,21 +216,21 @@ def switchsd_verify(draft, target_argmax, out_accept, *, draft_len, ctx_tokens, 
     _check(code, "switchsd_verify")
 
 
-def switchsd_harness_target(ctx_lens, mode, draft, draft_len, labels, vdraft, vlen, target, *,
-                            seed: int, V: int, L0: int, agree_cap: int, thr_in: int, thr_out: int,
-                            step: int, stream=None) -> None:
+def switchsd_harness_target(ctx_lens, mode, draft, draft_len, future, vdraft, vlen, target, *,
+                            seed: int, V: int, L0: int, gamma: int, thr_neural: int, step: int,
+                            stream=None) -> None:
     """switchsd_harness_target of include/switchsd_harness.h (the target-model stand-in)."""
     B, k = draft.shape
     hp = switchsd_harness_params()
     hp.B, hp.k, hp.V, hp.L0 = B, k, V, L0
-    hp.n_labels = labels.shape[1]
-    hp.agree_cap, hp.step = agree_cap, step
-    hp.seed, hp.thr_in, hp.thr_out = seed, thr_in, thr_out
+    hp.n_future = future.shape[1]
+    hp.gamma, hp.step = gamma, step
+    hp.seed, hp.thr_neural = seed, thr_neural
     hp.stream = _stream_ptr(stream)
     code = load().switchsd_harness_target(
         _dev(ctx_lens, torch.int32, "ctx_lens", (B,)), _dev(mode, torch.int32, "mode", (B,)),
         _dev(draft, torch.int32, "draft", (B, k)), _dev(draft_len, torch.int32, "draft_len", (B,)),
-        _dev(labels, torch.uint8, "labels"), _dev(vdraft, torch.int32, "vdraft", (B, k)),
+        _dev(future, torch.int32, "future"), _dev(vdraft, torch.int32, "vdraft", (B, k)),
         _dev(vlen, torch.int32, "vlen", (B,)), _dev(target, torch.int32, "target", (B, k + 1)),
         ctypes.byref(hp))
     _check(code, "switchsd_harness_target")

@@ -1,7 +1,8 @@
 // harness.cu -- device stand-in for the neural drafter and the target model (not the controller).
 //
-// Synthesises the target's greedy tokens for each row's draft with the seeded agreement law stated
-// in switchsd_harness.h.  One warp per row; lane i handles draft indices i, i + 32, ...
+// Reads the target's greedy tokens for each row from the caller's future stream and draws the neural
+// draft for non-copy rows, with the seeded law stated in switchsd_harness.h.  One warp per row; lane
+// i handles draft indices i, i + 32, ...
 #include "common.cuh"
 #include "switchsd_harness.h"
 
@@ -10,8 +11,7 @@ namespace switchsd {
 constexpr int kHarnessThreads = 256;
 
 struct HarnessArgs {
-    const int32_t *lens, *mode, *draft, *draft_len;
-    const uint8_t *labels;
+    const int32_t *lens, *mode, *draft, *draft_len, *future;
     int32_t *vdraft, *vlen, *target;
     switchsd_harness_params p;
 };
@@ -35,32 +35,32 @@ __global__ void __launch_bounds__(kHarnessThreads) harness_kernel(const HarnessA
     if (b >= p.B) return;
     const int k = p.k;
     const bool copy = a.mode[b] == SWITCHSD_MODE_COPY;
-    int len = copy ? a.draft_len[b] : k;
+    int len = copy ? a.draft_len[b] : p.gamma;
     len = len < 0 ? 0 : (len > k ? k : len);
     const int32_t L = a.lens[b];
     const uint64_t row_key = splitmix64(splitmix64(splitmix64(p.seed) ^ uint64_t(b)) ^ uint64_t(p.step));
     for (int i = lane; i <= k; i += kWarp) {
-        const uint64_t slot = 4ull * uint64_t(i);
-        int32_t d = 0;
-        if (i < len) d = copy ? a.draft[size_t(b) * k + i] : token_of(splitmix64(row_key ^ (slot + 2)), p.V);
-        if (i < k) a.vdraft[size_t(b) * k + i] = i < len ? d : 0;
-        int32_t t;
-        if (i < len) {
-            const int64_t pos = int64_t(L) + i - p.L0;
-            const bool lab = pos >= 0 && pos < p.n_labels && a.labels[size_t(b) * p.n_labels + pos] != 0;
-            const uint64_t thr = lab ? p.thr_in : p.thr_out;
-            const uint64_t coin = splitmix64(row_key ^ (slot + 0)) & 0xffffffffull;
-            const bool agree = i < p.agree_cap && coin < thr;
-            if (agree) {
-                t = d;
-            } else {
-                t = token_of(splitmix64(row_key ^ (slot + 1)), p.V);
-                if (t == d) t = (t + 1) % p.V;
+        const int64_t pos = int64_t(L) - p.L0 + i;
+        const int32_t g = (pos >= 0 && pos < p.n_future) ? a.future[size_t(b) * p.n_future + pos] : 0;
+        a.target[size_t(b) * (k + 1) + i] = g;
+        if (i < k) {
+            int32_t d = 0;
+            if (i < len) {
+                if (copy) {
+                    d = a.draft[size_t(b) * k + i];
+                } else {
+                    const uint64_t slot = 4ull * uint64_t(i);
+                    const uint64_t coin = splitmix64(row_key ^ slot) & 0xffffffffull;
+                    if (coin < p.thr_neural) {
+                        d = g;
+                    } else {
+                        d = token_of(splitmix64(row_key ^ (slot + 1)), p.V);
+                        if (d == g) d = (d + 1) % p.V;
+                    }
+                }
             }
-        } else {
-            t = token_of(splitmix64(row_key ^ (slot + 3)), p.V);
+            a.vdraft[size_t(b) * k + i] = d;
         }
-        a.target[size_t(b) * (k + 1) + i] = t;
     }
     if (lane == 0) a.vlen[b] = len;
 }
@@ -70,17 +70,19 @@ __global__ void __launch_bounds__(kHarnessThreads) harness_kernel(const HarnessA
 using namespace switchsd;
 
 extern "C" int switchsd_harness_target(const int32_t *ctx_lens, const int32_t *mode, const int32_t *draft,
-                                       const int32_t *draft_len, const uint8_t *labels, int32_t *vdraft,
+                                       const int32_t *draft_len, const int32_t *future, int32_t *vdraft,
                                        int32_t *vlen, int32_t *target, const switchsd_harness_params *hp) {
     if (!hp || !ctx_lens || !mode || !draft || !draft_len || !vdraft || !vlen || !target) return SWITCHSD_ERR_ARG;
-    if (hp->n_labels > 0 && !labels) return SWITCHSD_ERR_ARG;
-    if (hp->B < 1 || hp->k < 1 || hp->k > SWITCHSD_KMAX || hp->V < 2 || hp->n_labels < 0) return SWITCHSD_ERR_SHAPE;
+    if (hp->n_future > 0 && !future) return SWITCHSD_ERR_ARG;
+    if (hp->B < 1 || hp->k < 1 || hp->k > SWITCHSD_KMAX || hp->V < 2 || hp->n_future < 0 || hp->gamma < 0 ||
+        hp->gamma > hp->k)
+        return SWITCHSD_ERR_SHAPE;
     HarnessArgs a;
     a.lens = ctx_lens;
     a.mode = mode;
     a.draft = draft;
     a.draft_len = draft_len;
-    a.labels = labels;
+    a.future = future;
     a.vdraft = vdraft;
     a.vlen = vlen;
     a.target = target;

@@ -1,44 +1,61 @@
-// step.cu -- switchsd_step: n-gram search, probe, switch and copy-draft gather for B rows.
+// step.cu -- switchsd_step and switchsd_verify_step: n-gram search, probe, switch and copy-draft gather
+// for B rows, optionally preceded by the greedy verification and append of the previous draft.
 //
-// Paper: §3.3 (kappa-gram gate, recency-ranked copy candidates, Eq. 4 decision rule), Eq. 3 (linear
-// probe), Fig. 1 (three cases).
+// Paper: §3.3 (kappa-gram gate, recency-ranked copy candidates, Eq. 4 decision rule, parallel
+// verification, overall framework), Eq. 3 (linear probe), Fig. 1 (three cases).
 //
 // Layout of the work.  Row b is handled by one thread-block cluster of C CTAs (grid = C x B).  The
 // candidate end positions e in [0, L-1) are split into C contiguous 16-byte-aligned ranges.  Each CTA
-// streams its range through shared memory in tiles of kTile tokens with bulk TMA copies (one copy per
-// tile, kHalo tokens of look-back included), so the whole range is in flight at once.  A position e
-// is a candidate when x[e] equals the current token; the thread then compares backwards against the
-// suffix (held in shared memory) to get m(e) = the common suffix length, capped at n_max.  The row's
-// answer is the maximum of the packed key (m << 32 | e) over candidates with m >= n_min: the largest
-// m first, then the most recent e -- exactly the longest-then-most-recent rule.
+// stages its range in shared memory with bulk TMA copies (normally one copy: the host sizes the tile to
+// the range); a copy also brings kHalo tokens of look-back (for the backward compare) and kFwd tokens
+// of look-ahead (for the copy draft).  The copies are issued as soon as the row length is known,
+// before any other dependent load, so the whole context is in flight at once.  A position e is a
+// candidate when x[e] equals the current token; the thread then compares backwards against the suffix
+// (held in shared memory) to get m(e) = the common suffix length, capped at n_max.  The row's answer is
+// the maximum of the packed key (m << 32 | e) over candidates with m >= n_min: the largest m first,
+// then the most recent e -- exactly the longest-then-most-recent rule.
 //
-// The same CTAs also compute the linear probe: CTA r dots its 1/C slice of the hidden state with the
-// probe weights in fp32.  Each CTA writes its key and its probe partial into the leader CTA's shared
-// memory over DSMEM; after one cluster barrier the leader reduces them (fixed order), applies the
-// switch and gathers the draft.  No global scratch, no atomics, no inter-CTA spin-waits.
+// Fused verification (switchsd_verify_step).  While the copies fly, every CTA of the row recomputes the
+// accepted length a of the previous draft (a warp ballot over draft vs target) and the tokens it
+// appends, draft[0..a) then target[a].  The split is taken on the length before the append and the
+// last CTA's range stretches to the longest possible append, so the copies never wait for the verify.
+// Staged positions at or past the old length are patched with the appended tokens (the leader writes
+// them to global memory in the same launch, so a copy may see either version).  The leader publishes
+// the new length only after every CTA of the cluster has read the old one (cluster barrier phase 1).
+//
+// After each tile the CTA reduces its best key and, when it improves, keeps that match's continuation
+// (the candidate draft) from the staged tile.  The same CTAs compute the linear probe: CTA r dots its
+// 1/C slice of the hidden state with the probe weights in fp32.  Each CTA then writes its key, probe
+// partial and candidate draft into the leader CTA's shared memory over DSMEM; after one cluster
+// barrier the leader reduces them in a fixed order, applies the switch and writes the winner's draft.
+// No global scratch, no atomics, no inter-CTA spin-waits, no global re-read of the context.
 #include "common.cuh"
 
 namespace switchsd {
 
 constexpr int kStepThreads = 256;
 constexpr int kStepWarps = kStepThreads / kWarp;
-constexpr int kTile = 4096;  // tokens per staged tile
-constexpr int kHalo = 32;    // look-back staged before each tile: >= SWITCHSD_NMAX - 1, multiple of 4
-constexpr int kStages = 2;
-constexpr int kStageInts = kHalo + kTile;
+constexpr int kTileMax = 8192;        // largest staged tile (candidate ends)
+constexpr int kHalo = 32;             // look-back staged before a tile: >= SWITCHSD_NMAX, multiple of 4
+constexpr int kFwd = SWITCHSD_KMAX;   // look-ahead staged after a tile: the longest copy draft
+constexpr int kMaxStages = 2;
 constexpr int kMaxSplit = 16;
-constexpr size_t kStepSmemBytes = size_t(kStages) * kStageInts * sizeof(int32_t);
 constexpr unsigned long long kTimeoutBit = 1ull << 62;
 
-static_assert(kHalo >= SWITCHSD_NMAX - 1 && kHalo % 4 == 0, "halo must cover the longest n-gram");
+static_assert(kHalo >= SWITCHSD_NMAX && kHalo % 4 == 0, "halo must cover the longest n-gram");
+static_assert(kFwd % 4 == 0 && kTileMax % 4 == 0, "stages must stay 16-byte aligned");
 
 struct StepArgs {
-    const int32_t *ctx;
-    const int32_t *lens;
+    int32_t *ctx;            // read through TMA; written (append) by the leader when verifying
+    int32_t *lens;           // read; written when verifying
     const uint16_t *hidden;
     const uint16_t *probe_w;
-    const float *z_pre;  // logits from the two-layer probe kernel, or null for the linear probe
-    int32_t B, cap, d, k, n_min, n_max, kappa;
+    const float *z_pre;      // logits from the two-layer probe kernel, or null for the linear probe
+    const int32_t *pv_draft; // previous draft [B, k] / target [B, k+1] / draft length [B]; null = no verify
+    const int32_t *pv_target;
+    const int32_t *pv_len;
+    int32_t *out_accept;
+    int32_t B, cap, d, k, n_min, n_max, kappa, tile, stages;
     float logit_tau;
     int32_t *out_draft, *out_len, *out_mode;
     float *out_score;
@@ -57,59 +74,102 @@ __device__ __forceinline__ float dot8_bf16(uint4 w, uint4 h, float acc) {
     return acc;
 }
 
+__device__ __forceinline__ void st_cluster_i32(uint32_t addr, int32_t v) {
+    asm volatile("st.shared::cluster.s32 [%0], %1;\n" ::"r"(addr), "r"(v) : "memory");
+}
+
 __global__ void __launch_bounds__(kStepThreads) step_kernel(const StepArgs a) {
-    extern __shared__ __align__(128) int32_t tiles[];  // kStages x kStageInts
-    __shared__ __align__(8) uint64_t bars[kStages];
+    extern __shared__ __align__(128) int32_t tiles[];  // stages x (kHalo + tile + kFwd)
+    __shared__ __align__(8) uint64_t bars[kMaxStages];
     __shared__ int32_t s_suf[SWITCHSD_NMAX];
+    __shared__ int32_t s_old[kHalo];                           // the kHalo tokens before the old end
+    __shared__ int32_t s_app[SWITCHSD_KMAX + 1];               // tokens appended by the verification
+    __shared__ int32_t s_ver[3];                               // accepted, new length, verify status
     __shared__ unsigned long long s_wkey[kStepWarps];
     __shared__ float s_wz[kStepWarps];
-    __shared__ unsigned long long s_key[kMaxSplit];  // leader: one slot per CTA of the cluster
+    __shared__ int32_t s_mine[SWITCHSD_KMAX];                  // continuation of this CTA's best match
+    __shared__ unsigned long long s_key[kMaxSplit];            // leader: one slot per CTA of the cluster
     __shared__ float s_zp[kMaxSplit];
-    __shared__ int32_t s_out[3];                     // leader: mode, len, e*
+    __shared__ int32_t s_cand[kMaxSplit][SWITCHSD_KMAX];
+    __shared__ int32_t s_out[2];                               // leader: winner rank, draft length
 
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     const uint32_t rank = cluster_ctarank();
     const uint32_t C = cluster_nctarank();
     const int b = blockIdx.y;
+    const int stage_ints = kHalo + a.tile + kFwd;
+    const bool verifying = a.pv_len != nullptr;
 
-    // Phase 1 of the cluster barrier: waited on right before the first DSMEM store, by which time
-    // every CTA of the cluster is guaranteed to be running.
-    cluster_arrive_relaxed();
-
-    const int32_t *row = a.ctx + size_t(b) * size_t(a.cap);
-    const int32_t L = a.lens[b];
-    const bool len_ok = (L >= 1 && L <= a.cap);
-    const int32_t E = len_ok ? L - 1 : 0;  // candidate ends e in [0, E)
-
-    int32_t chunk = (E + int32_t(C) - 1) / int32_t(C);
+    int32_t *row = a.ctx + size_t(b) * size_t(a.cap);
+    const int32_t L_old = a.lens[b];
+    // Phase 1 of the cluster barrier, released after the row length is read: once the leader has
+    // waited on it, every CTA of the cluster is running and has read ctx_lens[b], so the leader may
+    // publish the new length; it is also waited on before the first DSMEM store.
+    cluster_arrive_release();
+    const bool len_ok = (L_old >= 1 && L_old <= a.cap);
+    // Split on the old length; the last CTA also covers every end the append can add.
+    const int32_t E_split = len_ok ? L_old - 1 : 0;
+    const int32_t E_max = len_ok ? (verifying ? min(L_old + a.k + 1, a.cap) : L_old) - 1 : 0;
+    int32_t chunk = (E_split + int32_t(C) - 1) / int32_t(C);
     chunk = (chunk + 3) & ~3;
-    const int32_t e_lo = min(E, int32_t(rank) * chunk);
-    const int32_t e_hi = min(E, e_lo + chunk);
-    const int32_t ntiles = (e_hi - e_lo + kTile - 1) / kTile;
+    const int32_t e_lo = min(E_split, int32_t(rank) * chunk);
+    const int32_t e_hi = rank + 1 == C ? E_max : min(E_split, e_lo + chunk);
+    const int32_t ntiles = (e_hi - e_lo + a.tile - 1) / a.tile;
 
-    if (tid == 0) {
-        for (int s = 0; s < kStages; ++s) mbar_init(&bars[s], 1);
-        fence_mbar_init();
-    }
-    if (tid < SWITCHSD_NMAX) s_suf[tid] = (len_ok && tid < L) ? row[L - 1 - tid] : 0;
-    __syncthreads();
-
-    // Stage tile t: tokens [max(0, t0 - kHalo), roundup4(t1)) land so that tokens[p] sits at
-    // stage[kHalo + p - t0].  roundup4(t1) <= cap because t1 <= L-1 < cap and cap % 4 == 0.
+    // Stage tile t: tokens [max(0, t0 - kHalo), min(roundup4(t1 + kFwd), cap)) land so that token p
+    // sits at stage[kHalo + p - t0].  cap % 4 == 0 keeps every bound 16-byte aligned.
     auto issue = [&](int t) {
-        const int s = t % kStages;
-        const int32_t t0 = e_lo + t * kTile;
-        const int32_t t1 = min(e_hi, t0 + kTile);
+        const int s = t % a.stages;
+        const int32_t t0 = e_lo + t * a.tile;
+        const int32_t t1 = min(e_hi, t0 + a.tile);
         const int32_t lo = max(0, t0 - kHalo);
-        const int32_t hi = (t1 + 3) & ~3;
+        const int32_t hi = min((t1 + kFwd + 3) & ~3, a.cap);
         const uint32_t bytes = uint32_t(hi - lo) * 4u;
         mbar_arrive_expect_tx(&bars[s], bytes);
-        bulk_g2s(tiles + s * kStageInts + (kHalo + lo - t0), row + lo, bytes, &bars[s]);
+        bulk_g2s(tiles + s * stage_ints + (kHalo + lo - t0), row + lo, bytes, &bars[s]);
     };
-    if (tid == 0)
-        for (int t = 0; t < min(ntiles, kStages); ++t) issue(t);
-
-    // Linear probe partial over this CTA's slice of the hidden vector (overlaps the copies).
+    if (tid == 0) {
+        for (int s = 0; s < a.stages; ++s) mbar_init(&bars[s], 1);
+        fence_mbar_init();
+        for (int t = 0; t < min(ntiles, a.stages); ++t) issue(t);
+    } else if (warp == 1) {
+        // Verification of the previous draft (every CTA of the row computes the same result).
+        int32_t acc = -1, L = L_old, vst = len_ok ? SWITCHSD_ROW_OK : SWITCHSD_ROW_BAD_LEN;
+        if (verifying && len_ok) {
+            const int32_t n = a.pv_len[b];
+            if (n < 0 || n > a.k) {
+                vst = SWITCHSD_ROW_BAD_LEN;
+            } else {
+                const int32_t *dr = a.pv_draft + size_t(b) * a.k;
+                const int32_t *tg = a.pv_target + size_t(b) * (a.k + 1);
+                acc = n;
+                for (int base = 0; base < n; base += kWarp) {
+                    const int i = base + lane;
+                    const unsigned m = __ballot_sync(kFull, i < n && dr[i] != tg[i]);
+                    if (m) {
+                        acc = base + __ffs(m) - 1;
+                        break;
+                    }
+                }
+                if (L_old + acc + 1 > a.cap) {
+                    vst = SWITCHSD_ROW_CAPACITY;
+                    acc = -1;
+                } else {
+                    for (int i = lane; i <= acc; i += kWarp) s_app[i] = i < acc ? dr[i] : tg[acc];
+                    L = L_old + acc + 1;
+                }
+            }
+        }
+        if (lane == 0) {
+            s_ver[0] = acc;
+            s_ver[1] = L;
+            s_ver[2] = vst;
+        }
+    } else if (warp == 2) {
+        const int32_t p = L_old - kHalo + lane;
+        if (lane < kHalo) s_old[lane] = (len_ok && p >= 0) ? row[p] : 0;
+    }
+    // The linear probe partial over this CTA's 1/C slice, while the copies fly.
     float zp = 0.f;
     if (a.z_pre == nullptr) {
         const int nv = a.d >> 3;
@@ -119,85 +179,116 @@ __global__ void __launch_bounds__(kStepThreads) step_kernel(const StepArgs a) {
         const uint4 *w4 = reinterpret_cast<const uint4 *>(a.probe_w);
         for (int v = v0 + tid; v < v1; v += kStepThreads) zp = dot8_bf16(__ldg(w4 + v), __ldg(h4 + v), zp);
     }
+    zp = warp_sum_f32(zp);
+    if (lane == 0) s_wz[warp] = zp;
+    __syncthreads();  // verification, old tail, probe partials and barrier initialisation are visible
 
-    // Scan.
+    const int32_t acc = s_ver[0], L = s_ver[1];
+    const int32_t E = len_ok ? L - 1 : 0;  // candidate ends after the append: [0, E)
+    if (tid < SWITCHSD_NMAX) {
+        const int32_t p = L - 1 - tid;  // suffix position; p >= L_old - kHalo since L >= L_old
+        s_suf[tid] = p < 0 ? 0 : (p >= L_old ? s_app[p - L_old] : s_old[p - (L_old - kHalo)]);
+    }
+    float cta_z = 0.f;
+    if (warp == 0) cta_z = warp_sum_f32(lane < kStepWarps ? s_wz[lane] : 0.f);
+    __syncthreads();
+
     const int32_t s0 = s_suf[0];
     const int32_t n_max = a.n_max, n_min = a.n_min;
-    unsigned long long best = 0;  // real keys have m >= n_min >= 1, so 0 means "no match"
+    unsigned long long best = 0;  // CTA-uniform; real keys have m >= n_min >= 1, so 0 = no match
     bool ok = true;
     int t = 0;
     for (; t < ntiles; ++t) {
-        const int s = t % kStages;
-        ok = __syncthreads_and(mbar_wait(&bars[s], uint32_t(t / kStages) & 1u));
+        const int s = t % a.stages;
+        ok = __syncthreads_and(mbar_wait(&bars[s], uint32_t(t / a.stages) & 1u));
         if (!ok) break;
-        const int32_t t0 = e_lo + t * kTile;
-        const int32_t t1 = min(e_hi, t0 + kTile);
-        const int32_t *stage = tiles + s * kStageInts;
+        const int32_t t0 = e_lo + t * a.tile;
+        const int32_t t1 = min(min(e_hi, t0 + a.tile), E);  // ends scanned in this tile
+        int32_t *stage = tiles + s * stage_ints;
         const int32_t off = kHalo - t0;  // stage[off + p] = x[p] over the staged range
+        if (verifying) {
+            const int32_t lo = max(0, t0 - kHalo), hi = min((min(e_hi, t0 + a.tile) + kFwd + 3) & ~3, a.cap);
+            const int32_t p0 = max(lo, L_old), p1 = min(hi, L);
+            if (p0 < p1) {  // CTA-uniform
+                for (int32_t p = p0 + tid; p < p1; p += kStepThreads) stage[off + p] = s_app[p - L_old];
+                __syncthreads();
+            }
+        }
+        unsigned long long mine = 0;
         for (int32_t e4 = t0 + 4 * tid; e4 < t1; e4 += 4 * kStepThreads) {
             const int4 v = *reinterpret_cast<const int4 *>(stage + (off + e4));
-            const int32_t vals[4] = {v.x, v.y, v.z, v.w};
-#pragma unroll
-            for (int q = 0; q < 4; ++q) {
-                const int32_t e = e4 + q;
-                if (vals[q] == s0 && e < t1) {
-                    const int32_t lim = min(n_max, e + 1);
-                    int32_t m = 1;
-                    while (m < lim && stage[off + e - m] == s_suf[m]) ++m;
-                    if (m >= n_min) {
-                        const unsigned long long key = (static_cast<unsigned long long>(m) << 32) | uint32_t(e);
-                        best = key > best ? key : best;
-                    }
+            unsigned hits = unsigned(v.x == s0) | (unsigned(v.y == s0) << 1) | (unsigned(v.z == s0) << 2) |
+                            (unsigned(v.w == s0) << 3);
+            while (hits) {
+                const int32_t e = e4 + __ffs(hits) - 1;
+                hits &= hits - 1;
+                if (e >= t1) break;
+                const int32_t lim = min(n_max, e + 1);
+                int32_t m = 1;
+                while (m < lim && stage[off + e - m] == s_suf[m]) ++m;
+                if (m >= n_min) {
+                    const unsigned long long key = (static_cast<unsigned long long>(m) << 32) | uint32_t(e);
+                    mine = key > mine ? key : mine;
                 }
             }
         }
-        if (t + kStages < ntiles) {
-            __syncthreads();  // every thread is done with stage s
-            if (tid == 0) {
-                asm volatile("fence.proxy.async.shared::cta;\n" ::: "memory");
-                issue(t + kStages);
-            }
+        // Tile reduction; on improvement keep the match's continuation while the tile is staged.
+        mine = warp_max_u64(mine);
+        if (lane == 0) s_wkey[warp] = mine;
+        __syncthreads();
+        unsigned long long tile_best = 0;
+#pragma unroll
+        for (int w = 0; w < kStepWarps; ++w) tile_best = s_wkey[w] > tile_best ? s_wkey[w] : tile_best;
+        if (tile_best > best) {
+            best = tile_best;
+            const int32_t e = int32_t(best & 0xffffffffu);
+            const int32_t len = min(a.k, L - 1 - e);
+            for (int i = tid; i < len; i += kStepThreads) s_mine[i] = stage[off + e + 1 + i];
+        }
+        __syncthreads();  // stage s and s_wkey are free again
+        if (t + a.stages < ntiles && tid == 0) {
+            asm volatile("fence.proxy.async.shared::cta;\n" ::: "memory");
+            issue(t + a.stages);
         }
     }
     if (!ok) {
         best = kTimeoutBit;
         // Give the copies still in flight a second bounded wait before the CTA's memory goes away.
         if (tid == 0)
-            for (int u = t; u < min(ntiles, t + kStages); ++u)
-                (void)mbar_wait(&bars[u % kStages], uint32_t(u / kStages) & 1u);
+            for (int u = t; u < min(ntiles, t + a.stages); ++u)
+                (void)mbar_wait(&bars[u % a.stages], uint32_t(u / a.stages) & 1u);
     }
 
-    // CTA reduction (fixed order).
-    best = warp_max_u64(best);
-    zp = warp_sum_f32(zp);
-    if (lane == 0) {
-        s_wkey[warp] = best;
-        s_wz[warp] = zp;
+    cluster_wait_acquire();  // phase 1: all CTAs of the cluster are running and have read ctx_lens[b]
+    if (rank == 0 && verifying) {
+        // The leader publishes the append; the other CTAs only patched their staged copies.
+        for (int i = tid; i <= acc; i += kStepThreads) row[L_old + i] = s_app[i];
+        if (tid == 0 && len_ok) {
+            a.lens[b] = L;
+            a.out_accept[b] = acc;
+        }
     }
-    __syncthreads();
-    unsigned long long cta_key = 0;
-    float cta_z = 0.f;
-    if (warp == 0) {
-        cta_key = lane < kStepWarps ? s_wkey[lane] : 0ull;
-        cta_z = lane < kStepWarps ? s_wz[lane] : 0.f;
-        cta_key = warp_max_u64(cta_key);
-        cta_z = warp_sum_f32(cta_z);
-    }
-
-    cluster_wait_acquire();  // phase 1: all CTAs of the cluster are running
     if (tid == 0) {
-        st_cluster_u64(map_to_rank(&s_key[rank], 0), cta_key);
+        st_cluster_u64(map_to_rank(&s_key[rank], 0), best);
         st_cluster_f32(map_to_rank(&s_zp[rank], 0), cta_z);
     }
+    if (best != 0 && !(best & kTimeoutBit)) {
+        const int32_t len = min(a.k, L - 1 - int32_t(best & 0xffffffffu));
+        for (int i = tid; i < len; i += kStepThreads) st_cluster_i32(map_to_rank(&s_cand[rank][i], 0), s_mine[i]);
+    }
     cluster_arrive_release();
-    cluster_wait_acquire();  // phase 2: every CTA's key and partial are in the leader
+    cluster_wait_acquire();  // phase 2: every CTA's key, partial and candidate are in the leader
     if (rank != 0) return;
 
     if (tid == 0) {
         unsigned long long key = 0;
+        uint32_t win = 0;
         float z = 0.f;
         for (uint32_t r = 0; r < C; ++r) {
-            key = s_key[r] > key ? s_key[r] : key;
+            if (s_key[r] > key) {
+                key = s_key[r];
+                win = r;
+            }
             z += s_zp[r];
         }
         if (a.z_pre != nullptr) z = a.z_pre[b];
@@ -209,20 +300,23 @@ __global__ void __launch_bounds__(kStepThreads) step_kernel(const StepArgs a) {
         int32_t mode = SWITCHSD_MODE_NO_REP;
         if (hit) mode = (n >= kappa && z >= a.logit_tau) ? SWITCHSD_MODE_COPY : SWITCHSD_MODE_REP_NO_COPY;
         const int32_t len = mode == SWITCHSD_MODE_COPY ? min(a.k, L - 1 - e) : 0;
-        s_out[0] = mode;
+        s_out[0] = int32_t(win);
         s_out[1] = len;
-        s_out[2] = e;
         a.out_mode[b] = mode;
         a.out_len[b] = len;
         a.out_score[b] = z;
         if (a.out_match_n) a.out_match_n[b] = n;
         if (a.out_match_end) a.out_match_end[b] = e;
-        if (a.status)
-            a.status[b] = !len_ok ? SWITCHSD_ROW_BAD_LEN : (timeout ? SWITCHSD_ROW_TIMEOUT : SWITCHSD_ROW_OK);
+        if (verifying && !len_ok) a.out_accept[b] = -1;
+        if (a.status) {
+            int32_t st = s_ver[2];
+            if (st == SWITCHSD_ROW_OK && timeout) st = SWITCHSD_ROW_TIMEOUT;
+            a.status[b] = st;
+        }
     }
     __syncthreads();
-    const int32_t len = s_out[1], e = s_out[2];
-    for (int i = tid; i < len; i += kStepThreads) a.out_draft[size_t(b) * a.k + i] = row[e + 1 + i];
+    const int32_t win = s_out[0], len = s_out[1];
+    for (int i = tid; i < len; i += kStepThreads) a.out_draft[size_t(b) * a.k + i] = s_cand[win][i];
 }
 
 // ------------------------------------------------------------------------------------------------
@@ -321,12 +415,15 @@ static cudaError_t launch_step(const StepArgs &args, int split, cudaStream_t str
     if (dev >= 0 && dev < 64 && !attr_done[dev]) {
         cudaError_t e = cudaFuncSetAttribute(step_kernel, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
         if (e != cudaSuccess) return e;
+        e = cudaFuncSetAttribute(step_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 int(kMaxStages * (kHalo + kTileMax + kFwd) * sizeof(int32_t)));
+        if (e != cudaSuccess) return e;
         attr_done[dev] = true;
     }
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(unsigned(split), unsigned(args.B), 1);
     cfg.blockDim = dim3(kStepThreads, 1, 1);
-    cfg.dynamicSmemBytes = kStepSmemBytes;
+    cfg.dynamicSmemBytes = size_t(args.stages) * (kHalo + args.tile + kFwd) * sizeof(int32_t);
     cfg.stream = stream;
     cudaLaunchAttribute attr[1];
     attr[0].id = cudaLaunchAttributeClusterDimension;
@@ -353,13 +450,11 @@ static cudaError_t launch_mlp(const MlpArgs &m, cudaStream_t stream) {
     return cudaGetLastError();
 }
 
-}  // namespace switchsd
-
-using namespace switchsd;
-
-extern "C" int switchsd_step(const int32_t *ctx_tokens, const int32_t *ctx_lens, const uint16_t *hidden,
-                             const uint16_t *probe_w, const switchsd_params *p, int32_t *out_draft,
-                             int32_t *out_len, int32_t *out_mode, float *out_score) {
+// Shared validation and launch of switchsd_step / switchsd_verify_step.
+static int step_entry(int32_t *ctx_tokens, int32_t *ctx_lens, const uint16_t *hidden, const uint16_t *probe_w,
+                      const switchsd_params *p, const int32_t *pv_draft, const int32_t *pv_target,
+                      const int32_t *pv_len, int32_t *out_accept, int32_t *out_draft, int32_t *out_len,
+                      int32_t *out_mode, float *out_score) {
     if (!p || !ctx_tokens || !ctx_lens || !hidden || !probe_w || !out_draft || !out_len || !out_mode ||
         !out_score)
         return SWITCHSD_ERR_ARG;
@@ -383,6 +478,10 @@ extern "C" int switchsd_step(const int32_t *ctx_tokens, const int32_t *ctx_lens,
     args.hidden = hidden;
     args.probe_w = probe_w;
     args.z_pre = nullptr;
+    args.pv_draft = pv_draft;
+    args.pv_target = pv_target;
+    args.pv_len = pv_len;
+    args.out_accept = out_accept;
     args.B = p->B;
     args.cap = p->cap;
     args.d = p->d;
@@ -399,6 +498,18 @@ extern "C" int switchsd_step(const int32_t *ctx_tokens, const int32_t *ctx_lens,
     args.out_match_end = p->out_match_end;
     args.status = p->status;
 
+    const int split = p->split > 0 ? p->split : choose_split(p->B, p->cap);
+    // Tile: the largest CTA range (the last CTA may also cover a k + 1 token append), in one stage
+    // when it fits, else a ring of two kTileMax stages.
+    const int64_t range = ((int64_t(p->cap) - 1 + split - 1) / split + 3) / 4 * 4 + p->k + 1;
+    if (range <= kTileMax) {
+        args.tile = int32_t((range + 3) / 4 * 4);
+        args.stages = 1;
+    } else {
+        args.tile = kTileMax;
+        args.stages = 2;
+    }
+
     if (p->probe_kind == SWITCHSD_PROBE_MLP) {
         MlpArgs m;
         m.hidden = hidden;
@@ -413,7 +524,26 @@ extern "C" int switchsd_step(const int32_t *ctx_tokens, const int32_t *ctx_lens,
         if (launch_mlp(m, stream) != cudaSuccess) return SWITCHSD_ERR_CUDA;
         args.z_pre = out_score;
     }
-    const int split = p->split > 0 ? p->split : choose_split(p->B, p->cap);
     if (launch_step(args, split, stream) != cudaSuccess) return SWITCHSD_ERR_CUDA;
     return SWITCHSD_OK;
+}
+
+}  // namespace switchsd
+
+using namespace switchsd;
+
+extern "C" int switchsd_step(const int32_t *ctx_tokens, const int32_t *ctx_lens, const uint16_t *hidden,
+                             const uint16_t *probe_w, const switchsd_params *p, int32_t *out_draft,
+                             int32_t *out_len, int32_t *out_mode, float *out_score) {
+    return step_entry(const_cast<int32_t *>(ctx_tokens), const_cast<int32_t *>(ctx_lens), hidden, probe_w, p,
+                      nullptr, nullptr, nullptr, nullptr, out_draft, out_len, out_mode, out_score);
+}
+
+extern "C" int switchsd_verify_step(const int32_t *draft, const int32_t *target_argmax, const int32_t *draft_len,
+                                    int32_t *out_accept, int32_t *ctx_tokens, int32_t *ctx_lens,
+                                    const uint16_t *hidden, const uint16_t *probe_w, const switchsd_params *p,
+                                    int32_t *out_draft, int32_t *out_len, int32_t *out_mode, float *out_score) {
+    if (!draft || !target_argmax || !draft_len || !out_accept) return SWITCHSD_ERR_ARG;
+    return step_entry(ctx_tokens, ctx_lens, hidden, probe_w, p, draft, target_argmax, draft_len, out_accept,
+                      out_draft, out_len, out_mode, out_score);
 }

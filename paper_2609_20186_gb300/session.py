@@ -8,9 +8,13 @@ one decoding iteration as three library calls on one stream:
     switchsd_verify          (controller: greedy verification and append)
 
 Inputs arrive as numpy arrays (token ids int32, bf16 values as uint16 bit patterns) and are copied to
-the device once; nothing here computes any part of the controller.
+the device once.  The buffers are checked once at construction; each call then passes the cached
+argument list straight to the C function, so the per-call host cost is one foreign call.  Nothing
+here computes any part of the controller.
 """
 from __future__ import annotations
+
+import ctypes
 
 import numpy as np
 import torch
@@ -27,13 +31,14 @@ def bf16_tensor(bits: np.ndarray, device) -> torch.Tensor:
 class Session:
     def __init__(self, ctx: np.ndarray, lens: np.ndarray, probe_w_bits: np.ndarray, *, k: int,
                  n_min: int, n_max: int, kappa: int = 0, logit_tau: float = 0.0,
-                 probe_kind: int = bd.PROBE_LINEAR, probe_hidden: int = 0, labels=None,
-                 harness: dict | None = None, split: int = 0, device="cuda", stream=None):
+                 probe_kind: int = bd.PROBE_LINEAR, probe_hidden: int = 0, future=None,
+                 harness: dict | None = None, split: int = 0, d: int | None = None,
+                 device="cuda", stream: torch.cuda.Stream | None = None):
         self.device = torch.device(device)
+        if self.device.type == "cuda" and self.device.index is None:
+            self.device = torch.device("cuda", torch.cuda.current_device())
         self.B, self.cap = ctx.shape
         self.k = k
-        self.cfg = dict(k=k, n_min=n_min, n_max=n_max, kappa=kappa, logit_tau=logit_tau,
-                        probe_kind=probe_kind, probe_hidden=probe_hidden, split=split)
         dev = self.device
         self.ctx = torch.from_numpy(np.ascontiguousarray(ctx, np.int32)).to(dev)
         self.lens = torch.from_numpy(np.ascontiguousarray(lens, np.int32)).to(dev)
@@ -52,29 +57,100 @@ class Session:
         self.target = torch.zeros(B, k + 1, **i32)
         self.accept = torch.zeros(B, **i32)
         self.vstatus = torch.zeros(B, **i32)
-        lab = labels if labels is not None else np.zeros((B, 0), np.uint8)
-        self.labels = torch.from_numpy(np.ascontiguousarray(lab, np.uint8)).to(dev)
-        self.harness_cfg = harness
+        fut = future if future is not None else np.zeros((B, 0), np.int32)
+        self.future = torch.from_numpy(np.ascontiguousarray(fut, np.int32)).to(dev)
         self.stream = stream
+        sp = (stream or torch.cuda.current_stream(dev)).cuda_stream
+        if d is None:
+            d = probe_w_bits.size if probe_kind == bd.PROBE_LINEAR else None
+        self.d = d
+        self.lib = bd.load()
+
+        # switchsd_step: two cached parameter blocks (with and without the debug outputs)
+        def params(debug: bool):
+            p = bd.switchsd_params()
+            p.B, p.cap, p.d, p.k = B, self.cap, d or 0, k
+            p.n_min, p.n_max, p.kappa, p.logit_tau = n_min, n_max, kappa, logit_tau
+            p.probe_kind, p.probe_hidden, p.b1, p.b2, p.split = probe_kind, probe_hidden, None, 0.0, split
+            p.out_match_n = self.match_n.data_ptr() if debug else None
+            p.out_match_end = self.match_end.data_ptr() if debug else None
+            p.status = self.status.data_ptr() if debug else None
+            p.stream = sp
+            return p
+        self._p_dbg, self._p_fast = params(True), params(False)
+        self._step_head = (self.ctx.data_ptr(), self.lens.data_ptr())
+        self._step_tail = (self.probe_w.data_ptr(),)
+        self._step_outs = (self.draft.data_ptr(), self.len.data_ptr(), self.mode.data_ptr(),
+                           self.score.data_ptr())
+
+        def vparams(debug: bool):
+            vp = bd.switchsd_verify_params()
+            vp.B, vp.cap, vp.k = B, self.cap, k
+            vp.draft_len = self.vlen.data_ptr()
+            vp.ctx_tokens = self.ctx.data_ptr()
+            vp.ctx_lens = self.lens.data_ptr()
+            vp.status = self.vstatus.data_ptr() if debug else None
+            vp.stream = sp
+            return vp
+        self._vp_dbg, self._vp_fast = vparams(True), vparams(False)
+        self._verify_args = (self.vdraft.data_ptr(), self.target.data_ptr(), self.accept.data_ptr())
+        self._vs_head = (self.vdraft.data_ptr(), self.target.data_ptr(), self.vlen.data_ptr(),
+                         self.accept.data_ptr())
+
+        self._hp = None
+        if harness is not None:
+            hp = bd.switchsd_harness_params()
+            hp.B, hp.k, hp.V, hp.L0 = B, k, harness["V"], harness["L0"]
+            hp.n_future = self.future.shape[1]
+            hp.gamma, hp.step = harness["gamma"], 0
+            hp.seed, hp.thr_neural = harness["seed"], harness["thr_neural"]
+            hp.stream = sp
+            self._hp = hp
+            self._harness_args = (self.lens.data_ptr(), self.mode.data_ptr(), self.draft.data_ptr(),
+                                  self.len.data_ptr(),
+                                  self.future.data_ptr() if self.future.numel() else None,
+                                  self.vdraft.data_ptr(), self.vlen.data_ptr(),
+                                  self.target.data_ptr())
 
     # --- the three calls ---------------------------------------------------------------------
+    def _check_hidden(self, hidden: torch.Tensor) -> None:
+        if (hidden.dtype != torch.bfloat16 or hidden.device != self.device
+                or not hidden.is_contiguous() or hidden.shape[0] != self.B
+                or (self.d is not None and hidden.shape[1] != self.d)):
+            raise ValueError("hidden must be a contiguous bf16 [B, d] tensor on the session device")
+        if self.d is None:
+            self._p_dbg.d = self._p_fast.d = hidden.shape[1]
+            self.d = hidden.shape[1]
+
     def step(self, hidden: torch.Tensor, debug: bool = True) -> None:
-        bd.switchsd_step(self.ctx, self.lens, hidden, self.probe_w, self.draft, self.len, self.mode,
-                         self.score, out_match_n=self.match_n if debug else None,
-                         out_match_end=self.match_end if debug else None,
-                         status=self.status if debug else None, stream=self.stream, **self.cfg)
+        self._check_hidden(hidden)
+        p = self._p_dbg if debug else self._p_fast
+        code = self.lib.switchsd_step(*self._step_head, hidden.data_ptr(), *self._step_tail,
+                                      ctypes.byref(p), *self._step_outs)
+        if code != bd.OK:
+            raise RuntimeError(f"switchsd_step failed: {code} ({bd.strerror(code)})")
+
+    def verify_step(self, hidden: torch.Tensor, debug: bool = True) -> None:
+        """Verification of the last harness draft (vdraft / target / vlen) and the next step, fused."""
+        self._check_hidden(hidden)
+        p = self._p_dbg if debug else self._p_fast
+        code = self.lib.switchsd_verify_step(*self._vs_head, self.ctx.data_ptr(), self.lens.data_ptr(),
+                                             hidden.data_ptr(), *self._step_tail, ctypes.byref(p),
+                                             *self._step_outs)
+        if code != bd.OK:
+            raise RuntimeError(f"switchsd_verify_step failed: {code} ({bd.strerror(code)})")
 
     def harness(self, t: int) -> None:
-        h = self.harness_cfg
-        bd.switchsd_harness_target(self.lens, self.mode, self.draft, self.len, self.labels,
-                                   self.vdraft, self.vlen, self.target, seed=h["seed"], V=h["V"],
-                                   L0=h["L0"], agree_cap=h["agree_cap"], thr_in=h["thr_in"],
-                                   thr_out=h["thr_out"], step=t, stream=self.stream)
+        self._hp.step = t
+        code = self.lib.switchsd_harness_target(*self._harness_args, ctypes.byref(self._hp))
+        if code != bd.OK:
+            raise RuntimeError(f"switchsd_harness_target failed: {code} ({bd.strerror(code)})")
 
     def verify(self, debug: bool = True) -> None:
-        bd.switchsd_verify(self.vdraft, self.target, self.accept, draft_len=self.vlen,
-                           ctx_tokens=self.ctx, ctx_lens=self.lens,
-                           status=self.vstatus if debug else None, stream=self.stream)
+        code = self.lib.switchsd_verify(*self._verify_args,
+                                        ctypes.byref(self._vp_dbg if debug else self._vp_fast))
+        if code != bd.OK:
+            raise RuntimeError(f"switchsd_verify failed: {code} ({bd.strerror(code)})")
 
     def iterate(self, hidden: torch.Tensor, t: int, debug: bool = True) -> None:
         self.step(hidden, debug)

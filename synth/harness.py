@@ -1,18 +1,20 @@
 """Stand-in for the neural drafter and the target model's verification forward (host side).
 
-The controller's verification input is the target model's greedy token after each draft prefix
-(``target_argmax``, k+1 entries per row).  The target model is out of scope, so this harness
-synthesises it from the draft with a seeded per-token agreement law:
+Greedy verification (temperature 0) keeps the context equal to the target model's own greedy
+sequence.  The target model is out of scope, so each row's greedy continuation is a seeded token
+stream ``future`` (Workload.future: the row's token law plus planted copies of earlier spans with
+occasional edits).  Then, for a row of current length L:
 
-- rows whose mode is not COPY get a neural draft of k seeded tokens (the drafter is out of scope);
-- for each draft index i < len: the target agrees with draft[i] with probability ``p_in`` if the
-  absolute position L + i lies inside a future span (``labels``), else ``p_out``, and never at
-  i >= ``agree_cap``; a disagreeing target token is a seeded id different from draft[i];
-- target[i] for i >= len (the bonus token and unused slots) is a seeded id.
+- the target's greedy token after draft prefix i is future[L + i] whenever that prefix is the
+  target's own (the only prefixes verification can accept), so target[i] = future[L + i - L0] for
+  i = 0..k;
+- rows whose mode is not COPY get a neural draft of ``gamma`` tokens: draft[i] = future[L + i - L0]
+  with probability ``p_neural`` (a seeded coin), else a seeded token different from it.
 
-All randomness comes from ``harness_key(seed, row, step, 4 * i + slot)`` with slots
-``TOKEN_STREAMS``; the CUDA harness kernel implements the same chain, so both sides see identical
-targets for identical drafts.  No controller arithmetic happens here.
+Randomness comes from ``harness_key(seed, row, step, 4 * i + slot)`` (slot 0: the neural coin, low
+32 bits; slot 1: the replacement token, a token being (word >> 32) mod V).  The CUDA harness kernel
+implements the same chain, so both sides produce identical drafts and targets for identical inputs.
+No controller arithmetic happens here.
 """
 from __future__ import annotations
 
@@ -20,7 +22,6 @@ import numpy as np
 
 from .rng import harness_key
 
-TOKEN_STREAMS = {"agree": 0, "alt": 1, "neural": 2, "bonus": 3}
 MODE_COPY = 1  # the documented ABI value of the copy mode
 
 
@@ -29,54 +30,39 @@ def _token(r: np.ndarray, V: int) -> np.ndarray:
 
 
 def harness_targets(params: dict, step: int, ctx_lens: np.ndarray, mode: np.ndarray,
-                    draft: np.ndarray, draft_len: np.ndarray, labels: np.ndarray,
-                    rows: np.ndarray | None = None):
-    """Returns (vdraft [B, k], vlen [B], target [B, k+1]) as int32 arrays.
-
-    ``rows`` (optional) restricts the work to those row indices (others are left zero); each row's
-    result depends only on its own inputs.
-    """
+                    draft: np.ndarray, draft_len: np.ndarray, future: np.ndarray,
+                    rows=None):
+    """Returns (vdraft [B, k], vlen [B], target [B, k+1]) as int32 arrays; rows outside ``rows``
+    (default: all) are left zero.  Each row's result depends only on its own inputs."""
     B, k = draft.shape
     V = params["V"]
     L0 = params["L0"]
-    thr_in = np.uint64(params["thr_in"])
-    thr_out = np.uint64(params["thr_out"])
-    agree_cap = params["agree_cap"]
+    gamma = params["gamma"]
+    thr = np.uint64(params["thr_neural"])
     seed = params["seed"]
+    nfut = future.shape[1]
     vdraft = np.zeros((B, k), np.int32)
     vlen = np.zeros(B, np.int32)
     target = np.zeros((B, k + 1), np.int32)
-    idx = np.arange(B) if rows is None else np.asarray(rows)
-    i = np.arange(k + 1, dtype=np.uint64)
-    nlab = labels.shape[1]
+    idx = range(B) if rows is None else rows
+    i = np.arange(k + 1, dtype=np.int64)
     for b in idx:
         b = int(b)
         L = int(ctx_lens[b])
-        r_agree = harness_key(seed, b, step, 4 * i + 0)
-        r_alt = harness_key(seed, b, step, 4 * i + 1)
-        r_neural = harness_key(seed, b, step, 4 * i + 2)
-        r_bonus = harness_key(seed, b, step, 4 * i + 3)
+        pos = L - L0 + i
+        ok = (pos >= 0) & (pos < nfut)
+        g = np.where(ok, future[b, np.clip(pos, 0, max(nfut - 1, 0))] if nfut else 0, 0)
+        target[b] = g.astype(np.int32)
         if int(mode[b]) == MODE_COPY:
             ln = int(draft_len[b])
-            d = np.zeros(k, np.int64)
-            d[:ln] = draft[b, :ln]
+            vdraft[b, :ln] = draft[b, :ln]
         else:
-            ln = k
-            d = _token(r_neural[:k], V)
-        vdraft[b, :ln] = d[:ln]
+            ln = gamma
+            slots = 4 * np.arange(ln, dtype=np.uint64)
+            coin = harness_key(seed, b, step, slots) & np.uint64(0xFFFFFFFF)
+            alt = _token(harness_key(seed, b, step, slots + np.uint64(1)), V)
+            gg = g[:ln].astype(np.int64)
+            alt = np.where(alt == gg, (alt + 1) % V, alt)
+            vdraft[b, :ln] = np.where(coin < thr, gg, alt).astype(np.int32)
         vlen[b] = ln
-        t = _token(r_bonus, V)
-        for j in range(ln):
-            p = L + j - L0
-            lab = labels[b, p] if 0 <= p < nlab else 0
-            thr = thr_in if lab else thr_out
-            agree = (j < agree_cap) and ((r_agree[j] & np.uint64(0xFFFFFFFF)) < thr)
-            if agree:
-                t[j] = d[j]
-            else:
-                alt = int(_token(r_alt[j: j + 1], V)[0])
-                if alt == int(d[j]):
-                    alt = (alt + 1) % V
-                t[j] = alt
-        target[b] = t.astype(np.int32)
     return vdraft, vlen, target

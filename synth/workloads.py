@@ -20,7 +20,9 @@ Recipes (one seed per workload):
 - ``mixed`` (B=16, 131,072): first half Zipf(1.1) prose; second half Zipf filler with 30 % planted
   copies of length 16 + Geom(1/256) - 1, at most 4,096, sourced anywhere earlier.
 
-Hidden states are bf16 N(0, 1) per (step, row); the linear probe is w ~ N(0, 1/d) in bf16 so that the
+The target model's greedy continuation of each row (``future``) follows the row's token law with
+``future_coverage`` of planted copies of earlier spans, 10 % of whose tokens are edited; the target
+stand-in (synth.harness) reads it.  Hidden states are bf16 N(0, 1) per (step, row); the linear probe is w ~ N(0, 1/d) in bf16 so that the
 logit is O(1); the two-layer probe is W1 ~ N(0, 1/d) [256, d], w2 ~ N(0, 1/256), no biases.
 """
 from __future__ import annotations
@@ -34,7 +36,7 @@ import numpy as np
 from .rng import bf16_bits_from_f32
 
 # Stream ids mixed into numpy SeedSequences so that each kind of input has its own stream.
-_S_CTX, _S_HIDDEN, _S_PROBE, _S_LABEL, _S_PERM = 1, 2, 3, 4, 9
+_S_CTX, _S_HIDDEN, _S_PROBE, _S_FUTURE, _S_BLOCKS, _S_PERM = 1, 2, 3, 4, 5, 9
 
 
 @dataclass(frozen=True)
@@ -59,10 +61,10 @@ class Workload:
     span_p: float = 1.0 / 64.0
     span_max: int = 512
     accidental_rate: float = 0.0   # explicit accidental short repeats per position
-    future_coverage: float = 0.0   # in-span share of future positions (harness acceptance law)
-    p_in: float = 0.9              # per-token agreement probability inside a span
-    p_out: float = 0.05            # ... outside
-    agree_cap: int = -1            # if >= 0, the target disagrees at this draft index and beyond
+    future_coverage: float = 0.0   # planted-copy share of the target's future tokens
+    p_in: float = 0.9              # per-token survival of a planted future copy (else an edit)
+    p_neural: float = 0.75         # per-token agreement of the neural draft with the target
+    gamma: int = 6                 # neural draft length (the drafter's lookahead, Table 3)
     variant: str = ""              # planted workload: copy | nocopy | norep
 
     @property
@@ -131,36 +133,37 @@ class Workload:
             out[t] = self.hidden(t)
         return out
 
-    def labels(self) -> np.ndarray:
-        """uint8 [B, cap - L0]: 1 where a future absolute position L0 + j lies inside a span."""
+    def future_row(self, b: int) -> np.ndarray:
+        """The target model's greedy continuation of row b: int32 tokens for absolute positions
+        [L0, cap).  Drawn with the row's own token law, then ``future_coverage`` of it is
+        overwritten with planted copies of earlier spans (context or earlier future), each copied
+        token kept with probability ``p_in`` (else replaced: an edit)."""
         n = self.cap - self.L0
-        out = np.zeros((self.B, n), np.uint8)
-        c = self.future_coverage
-        if c <= 0.0:
-            return out
-        if c >= 1.0:
-            out[:] = 1
-            return out
-        mean_span = self.span_min + (1.0 / self.span_p - 1.0)
-        mean_gap = mean_span * (1.0 - c) / c
+        rng = np.random.default_rng([self.seed, _S_FUTURE, b])
+        if self.structure == "planted":
+            return _planted_future(self, rng)
+        x = self.context_row(b)
+        full = np.concatenate([x, _FUTURE_BASE[self.structure](self, rng, b, n)]).astype(np.int32)
+        if self.future_coverage > 0.0:
+            _plant_spans(full, rng, self.future_coverage, self.span_min, self.span_p,
+                         self.span_max, (self.L0, self.cap), keep=self.p_in, V=self.V)
+        return full[self.L0:].copy()
+
+    def future(self) -> np.ndarray:
+        """int32 [B, cap - L0]: every row's future_row."""
+        out = np.zeros((self.B, self.cap - self.L0), np.int32)
         for b in range(self.B):
-            rng = np.random.default_rng([self.seed, _S_LABEL, b])
-            pos = int(rng.geometric(1.0 / (mean_gap + 1.0))) - 1
-            while pos < n:
-                ln = _span_len(rng, self.span_min, self.span_p, self.span_max)
-                out[b, pos: pos + ln] = 1
-                pos += ln + int(rng.geometric(1.0 / (mean_gap + 1.0))) - 1
+            out[b] = self.future_row(b)
         return out
 
     def harness_params(self) -> dict:
-        """Integer parameters of the target-synthesis harness (see synth.harness)."""
+        """Integer parameters of the target stand-in (see synth.harness)."""
         return {
             "seed": self.seed,
             "V": self.V,
             "L0": self.L0,
-            "thr_in": _prob_to_thr(self.p_in),
-            "thr_out": _prob_to_thr(self.p_out),
-            "agree_cap": self.agree_cap if self.agree_cap >= 0 else self.k + 1,
+            "gamma": min(self.gamma, self.k),
+            "thr_neural": _prob_to_thr(self.p_neural),
         }
 
     def expected_planted(self) -> dict:
@@ -176,8 +179,7 @@ class Workload:
         elif self.variant == "nocopy":
             out.update(draft=[], mode=2)
         else:
-            out.update(mode=1)
-        out["accept"] = self.agree_cap
+            out.update(mode=1, accept=_PLANTED_AGREE)
         return out
 
 
@@ -221,8 +223,9 @@ def _zipf(wl: Workload):
 
 
 def _plant_spans(x: np.ndarray, rng, coverage: float, lo: int, p: float, hi: int,
-                 region: tuple[int, int]) -> None:
-    """Overwrite ``coverage`` of positions in ``region`` with verbatim copies of earlier spans."""
+                 region: tuple[int, int], keep: float = 1.0, V: int = 0) -> None:
+    """Overwrite ``coverage`` of positions in ``region`` with copies of earlier spans; with
+    keep < 1 each copied token is replaced by a random id with probability 1 - keep."""
     r0, r1 = region
     target = int(coverage * (r1 - r0))
     used = np.zeros(x.shape[0], bool)
@@ -244,6 +247,9 @@ def _plant_spans(x: np.ndarray, rng, coverage: float, lo: int, p: float, hi: int
         covered += ln
     for dst, src, ln in sorted(spans):
         x[dst: dst + ln] = x[src: src + ln]
+        if keep < 1.0:
+            edit = rng.random(ln) >= keep
+            x[dst: dst + ln][edit] = rng.integers(0, V, int(edit.sum()), dtype=np.int64)
 
 
 def _accidental_repeats(x: np.ndarray, rng, count: int, nlo: int, nhi: int) -> None:
@@ -280,6 +286,21 @@ def _gen_planted(wl: Workload, rng, b: int) -> np.ndarray:
     return x
 
 
+_PLANTED_AGREE = 5      # the target follows the planted continuation for 5 tokens
+
+
+def _planted_future(wl: Workload, rng) -> np.ndarray:
+    """The target continues the planted copy for _PLANTED_AGREE tokens, then departs from it."""
+    n = wl.cap - wl.L0
+    x = wl.context_row(0)
+    cont = x[_PLANTED_SRC2 + 64: _PLANTED_SRC2 + 64 + wl.k]
+    g = rng.integers(0, wl.V, n, dtype=np.int64).astype(np.int32)
+    g[:_PLANTED_AGREE] = cont[:_PLANTED_AGREE]
+    if g[_PLANTED_AGREE] == cont[_PLANTED_AGREE]:
+        g[_PLANTED_AGREE] = (g[_PLANTED_AGREE] + 1) % wl.V
+    return g
+
+
 def _planted_hidden(wl: Workload) -> np.ndarray:
     rng = np.random.default_rng([wl.seed, _S_HIDDEN, 0])
     h = rng.standard_normal((wl.B, wl.d), dtype=np.float32)
@@ -312,19 +333,30 @@ def _gen_zipf_spans(wl: Workload, rng, b: int) -> np.ndarray:
     return x
 
 
-def _gen_code(wl: Workload, rng, b: int) -> np.ndarray:
-    L = wl.L0
-    blocks = rng.integers(0, wl.V, (8, 200), dtype=np.int64).astype(np.int32)
-    n_inst = L // 200
-    filler = L - n_inst * 200
-    x = np.empty(L, np.int32)
-    x[:filler] = rng.integers(0, wl.V, filler, dtype=np.int64)
+def _code_blocks(wl: Workload, b: int) -> np.ndarray:
+    rng = np.random.default_rng([wl.seed, _S_BLOCKS, b])
+    return rng.integers(0, wl.V, (8, 200), dtype=np.int64).astype(np.int32)
+
+
+def _code_instances(wl: Workload, rng, blocks: np.ndarray, n_inst: int) -> np.ndarray:
+    out = np.empty(n_inst * 200, np.int32)
     for i in range(n_inst):
         inst = blocks[int(rng.integers(0, 8))].copy()
         n_edit = int(rng.integers(1, 4))
         pos = rng.integers(0, 200, n_edit)
         inst[pos] = rng.integers(0, wl.V, n_edit, dtype=np.int64)
-        x[filler + 200 * i: filler + 200 * (i + 1)] = inst
+        out[200 * i: 200 * (i + 1)] = inst
+    return out
+
+
+def _gen_code(wl: Workload, rng, b: int) -> np.ndarray:
+    L = wl.L0
+    blocks = _code_blocks(wl, b)
+    n_inst = L // 200
+    filler = L - n_inst * 200
+    x = np.empty(L, np.int32)
+    x[:filler] = rng.integers(0, wl.V, filler, dtype=np.int64)
+    x[filler:] = _code_instances(wl, rng, blocks, n_inst)
     return x
 
 
@@ -333,6 +365,24 @@ def _gen_mixed(wl: Workload, rng, b: int) -> np.ndarray:
     x = _zipf(wl)(rng, L).astype(np.int32)
     _plant_spans(x, rng, wl.coverage, wl.span_min, wl.span_p, wl.span_max, (L // 2, L))
     return x
+
+
+def _fut_uniform(wl, rng, b, n):
+    return rng.integers(0, wl.V, n, dtype=np.int64).astype(np.int32)
+
+
+def _fut_zipf(wl, rng, b, n):
+    return _zipf(wl)(rng, n).astype(np.int32)
+
+
+def _fut_code(wl, rng, b, n):
+    """The code rows keep tiling their eight blocks (with 1-3 edits per instance)."""
+    inst = _code_instances(wl, rng, _code_blocks(wl, b), (n + 199) // 200)
+    return inst[:n]
+
+
+_FUTURE_BASE = {"uniform_spans": _fut_uniform, "zipf_spans": _fut_zipf, "code": _fut_code,
+                "mixed": _fut_zipf}
 
 
 _GENERATORS = {
@@ -346,8 +396,7 @@ _GENERATORS = {
 
 def _planted(variant: str) -> Workload:
     return Workload(name=f"planted_{variant}", B=1, L0=2048, V=128256, d=4096, k=8, n_min=3,
-                    n_max=8, steps=1, seed=1001, structure="planted", p_in=1.0, p_out=1.0,
-                    agree_cap=5, variant=variant)
+                    n_max=8, steps=1, seed=1001, structure="planted", variant=variant)
 
 
 WORKLOADS: dict[str, Workload] = {

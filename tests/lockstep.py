@@ -25,7 +25,7 @@ def oracle_trace(wl: synth.Workload, rows, steps: int, ctx=None, lens=None):
         ctx, lens = wl.contexts()
     ctx = ctx.copy()
     lens = lens.copy()
-    labels = wl.labels()
+    future = wl.future()
     pw = wl.probe_weights()
     hp = wl.harness_params()
     rows = list(rows)
@@ -43,7 +43,7 @@ def oracle_trace(wl: synth.Workload, rows, steps: int, ctx=None, lens=None):
                 for key in out:
                     out[key][b] = o[key][b]
         vd, vl, tg = synth.harness_targets(hp, t, lens, out["mode"], out["draft"], out["len"],
-                                           labels, rows=rows)
+                                           future, rows=rows)
         acc = np.zeros(wl.B, np.int32)
         st = np.zeros(wl.B, np.int32)
         for b in rows:
@@ -56,8 +56,13 @@ def oracle_trace(wl: synth.Workload, rows, steps: int, ctx=None, lens=None):
     return trace, ctx, lens
 
 
-def gpu_trace(wl: synth.Workload, steps: int, split: int = 0, ctx=None, lens=None, device="cuda"):
-    """Runs the GPU loop on all rows; returns the per-step host copies of every output."""
+def gpu_trace(wl: synth.Workload, steps: int, split: int = 0, ctx=None, lens=None, device="cuda",
+              fused: bool = False):
+    """Runs the GPU loop on all rows; returns the per-step host copies of every output.
+
+    fused=False: switchsd_step, target stand-in, switchsd_verify per iteration.
+    fused=True:  switchsd_verify_step (verification of iteration t-1, then step t) and the target
+                 stand-in per iteration; the last draft is verified by switchsd_verify."""
     import torch
     from paper_2609_20186_gb300 import Session, bf16_tensor
 
@@ -65,18 +70,27 @@ def gpu_trace(wl: synth.Workload, steps: int, split: int = 0, ctx=None, lens=Non
         ctx, lens = wl.contexts()
     sess = Session(ctx, lens, wl.probe_weights(), k=wl.k, n_min=wl.n_min, n_max=wl.n_max,
                    kappa=wl.kappa, logit_tau=wl.logit_tau, probe_kind=wl.probe_kind,
-                   probe_hidden=wl.probe_hidden, labels=wl.labels(), harness=wl.harness_params(),
-                   split=split, device=device)
+                   probe_hidden=wl.probe_hidden, future=wl.future(), harness=wl.harness_params(),
+                   split=split, d=wl.d, device=device)
     trace = []
     for t in range(steps):
         hidden = bf16_tensor(wl.hidden(t), sess.device)
-        sess.step(hidden)
+        if fused and t > 0:
+            sess.verify_step(hidden)
+            prev = trace[-1]
+            st = sess.status.cpu().numpy()
+            prev["accept"] = sess.accept.cpu().numpy()
+            prev["vstatus"] = np.where((st == 1) | (st == 2), st, 0)
+            prev["lens_after"] = sess.lens.cpu().numpy()
+        else:
+            sess.step(hidden)
         out = sess.step_outputs()
         sess.harness(t)
-        sess.verify()
-        out["accept"] = sess.accept.cpu().numpy()
-        out["vstatus"] = sess.vstatus.cpu().numpy()
-        out["lens_after"] = sess.lens.cpu().numpy()
+        if not fused or t == steps - 1:
+            sess.verify()
+            out["accept"] = sess.accept.cpu().numpy()
+            out["vstatus"] = sess.vstatus.cpu().numpy()
+            out["lens_after"] = sess.lens.cpu().numpy()
         trace.append(out)
     torch.cuda.synchronize()
     return trace, sess.ctx.cpu().numpy(), sess.lens.cpu().numpy()

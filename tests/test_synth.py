@@ -60,37 +60,51 @@ def test_planted_spans_are_verbatim_earlier_copies():
     assert 0.05 * x.shape[0] < ends < 0.12 * x.shape[0]
 
 
-def test_labels_coverage():
-    wl = synth.get_workload("mixed_128k").scaled(B=2)
-    lab = wl.labels()
-    assert lab.shape == (2, wl.cap - wl.L0)
-    assert 0.1 < lab.mean() < 0.5
+def test_future_stream():
+    """The target's continuation keeps the row's token law and plants copies of earlier spans with
+    about 10 % edits."""
+    wl = synth.get_workload("uniform_8k").scaled(B=1, steps=600, future_coverage=0.5)
+    g = wl.future_row(0)
+    assert g.shape == (wl.cap - wl.L0,) and g.min() >= 0 and g.max() < wl.V
+    assert np.array_equal(g, wl.future_row(0))
+    x = np.concatenate([wl.context_row(0), g])
+    # fraction of future positions that end an 8-gram seen earlier (uniform ids: only copies do)
+    seen = set()
+    ends = 0
+    for e in range(7, x.shape[0]):
+        gram = tuple(x[e - 7: e + 1].tolist())
+        if e >= wl.L0 and gram in seen:
+            ends += 1
+        seen.add(gram)
+    frac = ends / g.shape[0]
+    assert 0.15 < frac < 0.5          # 50 % coverage, 8-grams broken by 10 % edits: ~0.5 * 0.9^8
 
 
 def test_harness_law():
-    wl = synth.get_workload("uniform_8k").scaled(B=64, steps=4)
+    wl = synth.get_workload("uniform_8k").scaled(B=64, steps=16)
     params = wl.harness_params()
     B, k = wl.B, wl.k
     rng = np.random.default_rng(0)
     draft = rng.integers(0, wl.V, (B, k)).astype(np.int32)
     mode = np.array([1, 0, 2] * 21 + [1], np.int32)
-    dlen = np.where(mode == 1, k, 0).astype(np.int32)
-    lens = np.full(B, wl.L0, np.int32)
-    labels = np.ones((B, wl.cap - wl.L0), np.uint8)
-    vd, vl, t = synth.harness_targets(params, 0, lens, mode, draft, dlen, labels)
-    assert np.all(vl == k)
-    assert np.array_equal(vd[mode == 1], draft[mode == 1])
-    agree = (vd == t[:, :k])
-    assert 0.8 < agree.mean() < 0.97           # p_in = 0.9 everywhere here
-    # a disagreeing target never equals the draft token
-    assert np.all((t[:, :k] != vd) | agree)
-    # outside spans the agreement law is p_out = 0.05
-    vd, vl, t = synth.harness_targets(params, 1, lens, mode, draft, dlen, labels * 0)
-    assert (vd == t[:, :k]).mean() < 0.12
-    # agree_cap forces a disagreement at index 5 (the planted workload)
-    pw = synth.get_workload("planted_copy")
-    p = pw.harness_params()
-    d1 = rng.integers(0, pw.V, (1, pw.k)).astype(np.int32)
-    vd, vl, t = synth.harness_targets(p, 0, np.array([pw.L0], np.int32), np.array([1], np.int32),
-                                      d1, np.array([pw.k], np.int32), pw.labels())
-    assert t[0, :5].tolist() == d1[0, :5].tolist() and t[0, 5] != d1[0, 5]
+    dlen = np.where(mode == 1, rng.integers(0, k + 1, B), 0).astype(np.int32)
+    lens = (wl.L0 + rng.integers(0, 100, B)).astype(np.int32)
+    assert wl.cap - wl.L0 >= 100 + k + 1
+    future = rng.integers(0, wl.V, (B, wl.cap - wl.L0)).astype(np.int32)
+    vd, vl, t = synth.harness_targets(params, 0, lens, mode, draft, dlen, future)
+    # the target reads the future stream at the row's current length
+    for b in range(B):
+        assert t[b].tolist() == future[b, lens[b] - wl.L0: lens[b] - wl.L0 + k + 1].tolist()
+    copy = mode == 1
+    assert np.array_equal(vl[copy], dlen[copy]) and np.all(vl[~copy] == params["gamma"])
+    for b in np.nonzero(copy)[0]:
+        assert vd[b, : vl[b]].tolist() == draft[b, : vl[b]].tolist()
+        assert np.all(vd[b, vl[b]:] == 0)
+    g = params["gamma"]
+    agree = (vd[~copy, :g] == t[~copy, :g])
+    assert 0.65 < agree.mean() < 0.85          # p_neural = 0.75
+    assert np.all(vd[~copy, g:] == 0)
+    # positions past the stream read as 0
+    lens2 = np.full(B, wl.cap - 3, np.int32)
+    _, _, t2 = synth.harness_targets(params, 1, lens2, mode, draft, dlen, future)
+    assert np.all(t2[:, 3:] == 0) and np.array_equal(t2[:, :3], future[:, -3:])
