@@ -32,6 +32,8 @@ __global__ void __launch_bounds__(kHarnessThreads) harness_kernel(const HarnessA
     const int lane = threadIdx.x & 31;
     const int b = (blockIdx.x * kHarnessThreads + threadIdx.x) >> 5;
     const switchsd_harness_params &p = a.p;
+    pdl_wait();
+    pdl_trigger();
     if (b >= p.B) return;
     const int k = p.k;
     const bool copy = a.mode[b] == SWITCHSD_MODE_COPY;
@@ -88,6 +90,7 @@ extern "C" int switchsd_harness_target(const int32_t *ctx_lens, const int32_t *m
     a.target = target;
     a.p = *hp;
     const int wpb = kHarnessThreads / kWarp;
-    harness_kernel<<<(hp->B + wpb - 1) / wpb, kHarnessThreads, 0, static_cast<cudaStream_t>(hp->stream)>>>(a);
-    return cudaGetLastError() == cudaSuccess ? SWITCHSD_OK : SWITCHSD_ERR_CUDA;
+    const cudaError_t e = launch_pdl(harness_kernel, dim3((hp->B + wpb - 1) / wpb), dim3(kHarnessThreads), 0,
+                                     static_cast<cudaStream_t>(hp->stream), 0u, a);
+    return e == cudaSuccess ? SWITCHSD_OK : SWITCHSD_ERR_CUDA;
 }

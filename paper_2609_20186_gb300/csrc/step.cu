@@ -25,10 +25,11 @@
 //
 // After each tile the CTA reduces its best key and, when it improves, keeps that match's continuation
 // (the candidate draft) from the staged tile.  The same CTAs compute the linear probe: CTA r dots its
-// 1/C slice of the hidden state with the probe weights in fp32.  Each CTA then writes its key, probe
-// partial and candidate draft into the leader CTA's shared memory over DSMEM; after one cluster
-// barrier the leader reduces them in a fixed order, applies the switch and writes the winner's draft.
-// No global scratch, no atomics, no inter-CTA spin-waits, no global re-read of the context.
+// 1/C slice of the hidden state with the probe weights in fp32.  Each CTA then ships its key, probe
+// partial and candidate draft into the leader CTA's shared memory with asynchronous DSMEM stores that
+// complete on the leader's mbarrier, and exits; the leader waits (bounded) for all C messages, reduces
+// them in a fixed order, applies the switch and writes the winner's draft.  No global scratch, no
+// atomics, no global re-read of the context.
 #include "common.cuh"
 
 namespace switchsd {
@@ -38,7 +39,8 @@ constexpr int kStepWarps = kStepThreads / kWarp;
 constexpr int kTileMax = 8192;        // largest staged tile (candidate ends)
 constexpr int kHalo = 32;             // look-back staged before a tile: >= SWITCHSD_NMAX, multiple of 4
 constexpr int kFwd = SWITCHSD_KMAX;   // look-ahead staged after a tile: the longest copy draft
-constexpr int kMaxStages = 2;
+constexpr int kMaxStages = 6;          // staged tiles in flight per CTA (bounded by shared memory)
+constexpr size_t kStageSmemBudget = 200 * 1024;
 constexpr int kMaxSplit = 16;
 constexpr unsigned long long kTimeoutBit = 1ull << 62;
 
@@ -78,19 +80,27 @@ __device__ __forceinline__ void st_cluster_i32(uint32_t addr, int32_t v) {
     asm volatile("st.shared::cluster.s32 [%0], %1;\n" ::"r"(addr), "r"(v) : "memory");
 }
 
+// Per-CTA message to the leader: a 16-byte header (key, probe partial) and the candidate draft padded
+// to whole 16-byte words.
+struct alignas(16) Slot {
+    unsigned long long key;
+    float z;
+    int32_t pad;
+    int32_t cand[SWITCHSD_KMAX];
+};
+
 __global__ void __launch_bounds__(kStepThreads) step_kernel(const StepArgs a) {
     extern __shared__ __align__(128) int32_t tiles[];  // stages x (kHalo + tile + kFwd)
     __shared__ __align__(8) uint64_t bars[kMaxStages];
+    __shared__ __align__(8) uint64_t s_done;                   // leader: completes when every slot landed
     __shared__ int32_t s_suf[SWITCHSD_NMAX];
     __shared__ int32_t s_old[kHalo];                           // the kHalo tokens before the old end
     __shared__ int32_t s_app[SWITCHSD_KMAX + 1];               // tokens appended by the verification
     __shared__ int32_t s_ver[3];                               // accepted, new length, verify status
     __shared__ unsigned long long s_wkey[kStepWarps];
     __shared__ float s_wz[kStepWarps];
-    __shared__ int32_t s_mine[SWITCHSD_KMAX];                  // continuation of this CTA's best match
-    __shared__ unsigned long long s_key[kMaxSplit];            // leader: one slot per CTA of the cluster
-    __shared__ float s_zp[kMaxSplit];
-    __shared__ int32_t s_cand[kMaxSplit][SWITCHSD_KMAX];
+    __shared__ __align__(16) int32_t s_mine[SWITCHSD_KMAX];    // continuation of this CTA's best match
+    __shared__ Slot s_slot[kMaxSplit];                         // leader: one message per CTA
     __shared__ int32_t s_out[2];                               // leader: winner rank, draft length
 
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
@@ -99,12 +109,48 @@ __global__ void __launch_bounds__(kStepThreads) step_kernel(const StepArgs a) {
     const int b = blockIdx.y;
     const int stage_ints = kHalo + a.tile + kFwd;
     const bool verifying = a.pv_len != nullptr;
+    const int kwords = (a.k + 3) >> 2;                          // 16-byte words of a candidate
+    const uint32_t slot_bytes = 16u * uint32_t(1 + kwords);
+
+    if (tid == 0) {
+        for (int s = 0; s < a.stages; ++s) mbar_init(&bars[s], 1);
+        if (rank == 0) {
+            mbar_init(&s_done, 1);
+            mbar_arrive_expect_tx(&s_done, slot_bytes * C);
+        }
+        fence_mbar_init();
+    }
+    pdl_wait();     // everything below may read what the preceding kernel wrote
+    pdl_trigger();  // the next kernel may start launching
+
+    // Loads whose addresses do not depend on the row length go out first, in one round trip.
+    // Lane i of warp 1 holds draft[i], draft[i+32], target[i], target[i+32] and (lane 0) target[64].
+    int32_t pv_n = 0, d_lo = 0, d_hi = 0, t_lo = 0, t_hi = 0, t_top = 0;
+    if (verifying && warp == 1) {
+        const int32_t *dr = a.pv_draft + size_t(b) * a.k;
+        const int32_t *tg = a.pv_target + size_t(b) * (a.k + 1);
+        pv_n = a.pv_len[b];
+        if (lane < a.k) d_lo = dr[lane];
+        if (lane + 32 < a.k) d_hi = dr[lane + 32];
+        if (lane <= a.k) t_lo = tg[lane];
+        if (lane + 32 <= a.k) t_hi = tg[lane + 32];
+        if (lane == 0 && a.k >= 64) t_top = tg[64];
+    }
+    float zp = 0.f;
+    if (a.z_pre == nullptr) {
+        // the linear probe partial over this CTA's 1/C slice
+        const int nv = a.d >> 3;
+        const int per = (nv + int(C) - 1) / int(C);
+        const int v0 = int(rank) * per, v1 = min(nv, v0 + per);
+        const uint4 *h4 = reinterpret_cast<const uint4 *>(a.hidden + size_t(b) * size_t(a.d));
+        const uint4 *w4 = reinterpret_cast<const uint4 *>(a.probe_w);
+        for (int v = v0 + tid; v < v1; v += kStepThreads) zp = dot8_bf16(__ldg(w4 + v), __ldg(h4 + v), zp);
+    }
 
     int32_t *row = a.ctx + size_t(b) * size_t(a.cap);
     const int32_t L_old = a.lens[b];
-    // Phase 1 of the cluster barrier, released after the row length is read: once the leader has
-    // waited on it, every CTA of the cluster is running and has read ctx_lens[b], so the leader may
-    // publish the new length; it is also waited on before the first DSMEM store.
+    // Cluster barrier arrival, released after the row length is read: once a CTA has waited on it,
+    // every CTA of the cluster is running, has initialised its barriers and has read ctx_lens[b].
     cluster_arrive_release();
     const bool len_ok = (L_old >= 1 && L_old <= a.cap);
     // Split on the old length; the last CTA also covers every end the append can add.
@@ -129,33 +175,27 @@ __global__ void __launch_bounds__(kStepThreads) step_kernel(const StepArgs a) {
         bulk_g2s(tiles + s * stage_ints + (kHalo + lo - t0), row + lo, bytes, &bars[s]);
     };
     if (tid == 0) {
-        for (int s = 0; s < a.stages; ++s) mbar_init(&bars[s], 1);
-        fence_mbar_init();
         for (int t = 0; t < min(ntiles, a.stages); ++t) issue(t);
     } else if (warp == 1) {
         // Verification of the previous draft (every CTA of the row computes the same result).
         int32_t acc = -1, L = L_old, vst = len_ok ? SWITCHSD_ROW_OK : SWITCHSD_ROW_BAD_LEN;
         if (verifying && len_ok) {
-            const int32_t n = a.pv_len[b];
-            if (n < 0 || n > a.k) {
+            if (pv_n < 0 || pv_n > a.k) {
                 vst = SWITCHSD_ROW_BAD_LEN;
             } else {
-                const int32_t *dr = a.pv_draft + size_t(b) * a.k;
-                const int32_t *tg = a.pv_target + size_t(b) * (a.k + 1);
-                acc = n;
-                for (int base = 0; base < n; base += kWarp) {
-                    const int i = base + lane;
-                    const unsigned m = __ballot_sync(kFull, i < n && dr[i] != tg[i]);
-                    if (m) {
-                        acc = base + __ffs(m) - 1;
-                        break;
-                    }
-                }
+                const unsigned m_lo = __ballot_sync(kFull, lane < pv_n && d_lo != t_lo);
+                const unsigned m_hi = __ballot_sync(kFull, lane + 32 < pv_n && d_hi != t_hi);
+                acc = m_lo ? __ffs(m_lo) - 1 : (m_hi ? 32 + __ffs(m_hi) - 1 : pv_n);
                 if (L_old + acc + 1 > a.cap) {
                     vst = SWITCHSD_ROW_CAPACITY;
                     acc = -1;
                 } else {
-                    for (int i = lane; i <= acc; i += kWarp) s_app[i] = i < acc ? dr[i] : tg[acc];
+                    // s_app[i] = draft[i] for i < acc, target[acc] at i = acc
+                    const int32_t t_acc =
+                        __shfl_sync(kFull, acc < 32 ? t_lo : (acc < 64 ? t_hi : t_top), acc & 31);
+                    if (lane < acc) s_app[lane] = d_lo;
+                    if (lane + 32 < acc) s_app[lane + 32] = d_hi;
+                    if (lane == 0) s_app[acc] = t_acc;
                     L = L_old + acc + 1;
                 }
             }
@@ -169,22 +209,22 @@ __global__ void __launch_bounds__(kStepThreads) step_kernel(const StepArgs a) {
         const int32_t p = L_old - kHalo + lane;
         if (lane < kHalo) s_old[lane] = (len_ok && p >= 0) ? row[p] : 0;
     }
-    // The linear probe partial over this CTA's 1/C slice, while the copies fly.
-    float zp = 0.f;
-    if (a.z_pre == nullptr) {
-        const int nv = a.d >> 3;
-        const int per = (nv + int(C) - 1) / int(C);
-        const int v0 = int(rank) * per, v1 = min(nv, v0 + per);
-        const uint4 *h4 = reinterpret_cast<const uint4 *>(a.hidden + size_t(b) * size_t(a.d));
-        const uint4 *w4 = reinterpret_cast<const uint4 *>(a.probe_w);
-        for (int v = v0 + tid; v < v1; v += kStepThreads) zp = dot8_bf16(__ldg(w4 + v), __ldg(h4 + v), zp);
-    }
     zp = warp_sum_f32(zp);
     if (lane == 0) s_wz[warp] = zp;
-    __syncthreads();  // verification, old tail, probe partials and barrier initialisation are visible
+    __syncthreads();  // verification, old tail and probe partials are visible
 
+    // Every CTA has started and read ctx_lens[b] once this returns; it waits while the copies fly.
+    cluster_wait_acquire();
     const int32_t acc = s_ver[0], L = s_ver[1];
     const int32_t E = len_ok ? L - 1 : 0;  // candidate ends after the append: [0, E)
+    if (rank == 0 && verifying) {
+        // The leader publishes the append; the other CTAs only patch their staged copies.
+        for (int i = tid; i <= acc; i += kStepThreads) row[L_old + i] = s_app[i];
+        if (tid == 0 && len_ok) {
+            a.lens[b] = L;
+            a.out_accept[b] = acc;
+        }
+    }
     if (tid < SWITCHSD_NMAX) {
         const int32_t p = L - 1 - tid;  // suffix position; p >= L_old - kHalo since L >= L_old
         s_suf[tid] = p < 0 ? 0 : (p >= L_old ? s_app[p - L_old] : s_old[p - (L_old - kHalo)]);
@@ -196,100 +236,118 @@ __global__ void __launch_bounds__(kStepThreads) step_kernel(const StepArgs a) {
     const int32_t s0 = s_suf[0];
     const int32_t n_max = a.n_max, n_min = a.n_min;
     unsigned long long best = 0;  // CTA-uniform; real keys have m >= n_min >= 1, so 0 = no match
-    bool ok = true;
-    int t = 0;
-    for (; t < ntiles; ++t) {
+    bool bad = false;             // CTA-uniform: a copy did not land in time
+    for (int t = 0; t < ntiles && !bad; ++t) {
         const int s = t % a.stages;
-        ok = __syncthreads_and(mbar_wait(&bars[s], uint32_t(t / a.stages) & 1u));
-        if (!ok) break;
+        const bool landed = mbar_wait(&bars[s], uint32_t(t / a.stages) & 1u);
         const int32_t t0 = e_lo + t * a.tile;
-        const int32_t t1 = min(min(e_hi, t0 + a.tile), E);  // ends scanned in this tile
+        const int32_t tile_end = min(e_hi, t0 + a.tile);
+        const int32_t t1 = min(tile_end, E);  // ends scanned in this tile
         int32_t *stage = tiles + s * stage_ints;
         const int32_t off = kHalo - t0;  // stage[off + p] = x[p] over the staged range
         if (verifying) {
-            const int32_t lo = max(0, t0 - kHalo), hi = min((min(e_hi, t0 + a.tile) + kFwd + 3) & ~3, a.cap);
+            const int32_t lo = max(0, t0 - kHalo), hi = min((tile_end + kFwd + 3) & ~3, a.cap);
             const int32_t p0 = max(lo, L_old), p1 = min(hi, L);
             if (p0 < p1) {  // CTA-uniform
-                for (int32_t p = p0 + tid; p < p1; p += kStepThreads) stage[off + p] = s_app[p - L_old];
+                if (landed)
+                    for (int32_t p = p0 + tid; p < p1; p += kStepThreads) stage[off + p] = s_app[p - L_old];
                 __syncthreads();
             }
         }
         unsigned long long mine = 0;
-        for (int32_t e4 = t0 + 4 * tid; e4 < t1; e4 += 4 * kStepThreads) {
-            const int4 v = *reinterpret_cast<const int4 *>(stage + (off + e4));
-            unsigned hits = unsigned(v.x == s0) | (unsigned(v.y == s0) << 1) | (unsigned(v.z == s0) << 2) |
-                            (unsigned(v.w == s0) << 3);
-            while (hits) {
-                const int32_t e = e4 + __ffs(hits) - 1;
-                hits &= hits - 1;
-                if (e >= t1) break;
-                const int32_t lim = min(n_max, e + 1);
-                int32_t m = 1;
-                while (m < lim && stage[off + e - m] == s_suf[m]) ++m;
-                if (m >= n_min) {
-                    const unsigned long long key = (static_cast<unsigned long long>(m) << 32) | uint32_t(e);
-                    mine = key > mine ? key : mine;
+        if (landed) {
+            const int32_t n4 = (t1 - t0 + 3) >> 2;
+            const int4 *g4 = reinterpret_cast<const int4 *>(stage + kHalo);
+            for (int32_t g0 = tid; g0 < n4; g0 += 4 * kStepThreads) {
+                int4 v[4];
+#pragma unroll
+                for (int u = 0; u < 4; ++u) {
+                    const int32_t g = g0 + u * kStepThreads;
+                    v[u] = g < n4 ? g4[g] : make_int4(0, 0, 0, 0);
+                }
+#pragma unroll
+                for (int u = 0; u < 4; ++u) {
+                    const int32_t e4 = t0 + 4 * (g0 + u * kStepThreads);
+                    unsigned hits = unsigned(v[u].x == s0) | (unsigned(v[u].y == s0) << 1) |
+                                    (unsigned(v[u].z == s0) << 2) | (unsigned(v[u].w == s0) << 3);
+                    while (hits) {
+                        const int32_t e = e4 + __ffs(hits) - 1;
+                        hits &= hits - 1;
+                        if (e >= t1) break;
+                        const int32_t lim = min(n_max, e + 1);
+                        int32_t m = 1;
+                        while (m < lim && stage[off + e - m] == s_suf[m]) ++m;
+                        if (m >= n_min) {
+                            const unsigned long long key =
+                                (static_cast<unsigned long long>(m) << 32) | uint32_t(e);
+                            mine = key > mine ? key : mine;
+                        }
+                    }
                 }
             }
         }
-        // Tile reduction; on improvement keep the match's continuation while the tile is staged.
+        // Tile reduction; on improvement the threads that will ship the candidate copy it while the
+        // tile is still staged (thread j owns candidate words j-1).
         mine = warp_max_u64(mine);
         if (lane == 0) s_wkey[warp] = mine;
-        __syncthreads();
+        bad = __syncthreads_or(!landed);
         unsigned long long tile_best = 0;
 #pragma unroll
         for (int w = 0; w < kStepWarps; ++w) tile_best = s_wkey[w] > tile_best ? s_wkey[w] : tile_best;
-        if (tile_best > best) {
+        if (!bad && tile_best > best) {
             best = tile_best;
-            const int32_t e = int32_t(best & 0xffffffffu);
-            const int32_t len = min(a.k, L - 1 - e);
-            for (int i = tid; i < len; i += kStepThreads) s_mine[i] = stage[off + e + 1 + i];
+            if (tid >= 1 && tid <= kwords) {
+                const int32_t e = int32_t(best & 0xffffffffu);
+                const int32_t len = min(a.k, L - 1 - e);
+#pragma unroll
+                for (int q = 0; q < 4; ++q) {
+                    const int i = 4 * (tid - 1) + q;
+                    s_mine[i] = i < len ? stage[off + e + 1 + i] : 0;
+                }
+            }
         }
-        __syncthreads();  // stage s and s_wkey are free again
-        if (t + a.stages < ntiles && tid == 0) {
-            asm volatile("fence.proxy.async.shared::cta;\n" ::: "memory");
-            issue(t + a.stages);
+        if (!bad && t + a.stages < ntiles) {
+            __syncthreads();  // stage s and s_wkey are free again
+            if (tid == 0) {
+                asm volatile("fence.proxy.async.shared::cta;\n" ::: "memory");
+                issue(t + a.stages);
+            }
         }
     }
-    if (!ok) {
+    if (bad) {
         best = kTimeoutBit;
         // Give the copies still in flight a second bounded wait before the CTA's memory goes away.
         if (tid == 0)
-            for (int u = t; u < min(ntiles, t + a.stages); ++u)
-                (void)mbar_wait(&bars[u % a.stages], uint32_t(u / a.stages) & 1u);
+            for (int u = 0; u < min(ntiles, a.stages); ++u) (void)mbar_wait(&bars[u], 0u);
     }
 
-    cluster_wait_acquire();  // phase 1: all CTAs of the cluster are running and have read ctx_lens[b]
-    if (rank == 0 && verifying) {
-        // The leader publishes the append; the other CTAs only patched their staged copies.
-        for (int i = tid; i <= acc; i += kStepThreads) row[L_old + i] = s_app[i];
-        if (tid == 0 && len_ok) {
-            a.lens[b] = L;
-            a.out_accept[b] = acc;
-        }
-    }
+    // Ship this CTA's message to the leader: asynchronous DSMEM stores that complete on its barrier.
+    const uint32_t done_addr = map_to_rank(&s_done, 0);
     if (tid == 0) {
-        st_cluster_u64(map_to_rank(&s_key[rank], 0), best);
-        st_cluster_f32(map_to_rank(&s_zp[rank], 0), cta_z);
+        uint4 h;
+        h.x = uint32_t(best & 0xffffffffu);
+        h.y = uint32_t(best >> 32);
+        h.z = __float_as_uint(cta_z);
+        h.w = 0u;
+        st_async_v4(map_to_rank(&s_slot[rank], 0), h, done_addr);
+    } else if (tid <= kwords) {
+        const uint4 v = *reinterpret_cast<const uint4 *>(&s_mine[4 * (tid - 1)]);
+        st_async_v4(map_to_rank(&s_slot[rank].cand[4 * (tid - 1)], 0), v, done_addr);
     }
-    if (best != 0 && !(best & kTimeoutBit)) {
-        const int32_t len = min(a.k, L - 1 - int32_t(best & 0xffffffffu));
-        for (int i = tid; i < len; i += kStepThreads) st_cluster_i32(map_to_rank(&s_cand[rank][i], 0), s_mine[i]);
-    }
-    cluster_arrive_release();
-    cluster_wait_acquire();  // phase 2: every CTA's key, partial and candidate are in the leader
     if (rank != 0) return;
 
     if (tid == 0) {
-        unsigned long long key = 0;
+        // Bounded wait for every CTA's message (C x slot_bytes of transaction).
+        const bool all_in = mbar_wait(&s_done, 0);
+        unsigned long long key = all_in ? 0ull : kTimeoutBit;
         uint32_t win = 0;
         float z = 0.f;
-        for (uint32_t r = 0; r < C; ++r) {
-            if (s_key[r] > key) {
-                key = s_key[r];
+        for (uint32_t r = 0; r < C && all_in; ++r) {
+            if (s_slot[r].key > key) {
+                key = s_slot[r].key;
                 win = r;
             }
-            z += s_zp[r];
+            z += s_slot[r].z;
         }
         if (a.z_pre != nullptr) z = a.z_pre[b];
         const bool timeout = (key & kTimeoutBit) != 0;
@@ -316,7 +374,7 @@ __global__ void __launch_bounds__(kStepThreads) step_kernel(const StepArgs a) {
     }
     __syncthreads();
     const int32_t win = s_out[0], len = s_out[1];
-    for (int i = tid; i < len; i += kStepThreads) a.out_draft[size_t(b) * a.k + i] = s_cand[win][i];
+    for (int i = tid; i < len; i += kStepThreads) a.out_draft[size_t(b) * a.k + i] = s_slot[win].cand[i];
 }
 
 // ------------------------------------------------------------------------------------------------
@@ -342,6 +400,8 @@ __global__ void __launch_bounds__(kMlpThreads) mlp_probe_kernel(const MlpArgs a)
     __shared__ float s_part[kMlpThreads / kWarp][kMlpRows];
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     const int row0 = blockIdx.x * kMlpRows;
+    pdl_wait();
+    pdl_trigger();
     const int nv = a.d >> 3;
     for (int i = tid; i < kMlpRows * nv; i += kMlpThreads) {
         const int r = i / nv, v = i % nv;
@@ -415,24 +475,13 @@ static cudaError_t launch_step(const StepArgs &args, int split, cudaStream_t str
     if (dev >= 0 && dev < 64 && !attr_done[dev]) {
         cudaError_t e = cudaFuncSetAttribute(step_kernel, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
         if (e != cudaSuccess) return e;
-        e = cudaFuncSetAttribute(step_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                 int(kMaxStages * (kHalo + kTileMax + kFwd) * sizeof(int32_t)));
+        e = cudaFuncSetAttribute(step_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, int(kStageSmemBudget));
         if (e != cudaSuccess) return e;
         attr_done[dev] = true;
     }
-    cudaLaunchConfig_t cfg = {};
-    cfg.gridDim = dim3(unsigned(split), unsigned(args.B), 1);
-    cfg.blockDim = dim3(kStepThreads, 1, 1);
-    cfg.dynamicSmemBytes = size_t(args.stages) * (kHalo + args.tile + kFwd) * sizeof(int32_t);
-    cfg.stream = stream;
-    cudaLaunchAttribute attr[1];
-    attr[0].id = cudaLaunchAttributeClusterDimension;
-    attr[0].val.clusterDim.x = unsigned(split);
-    attr[0].val.clusterDim.y = 1;
-    attr[0].val.clusterDim.z = 1;
-    cfg.attrs = attr;
-    cfg.numAttrs = 1;
-    return cudaLaunchKernelEx(&cfg, step_kernel, args);
+    const size_t smem = size_t(args.stages) * (kHalo + args.tile + kFwd) * sizeof(int32_t);
+    return launch_pdl(step_kernel, dim3(unsigned(split), unsigned(args.B), 1), dim3(kStepThreads, 1, 1), smem,
+                      stream, unsigned(split), args);
 }
 
 static cudaError_t launch_mlp(const MlpArgs &m, cudaStream_t stream) {
@@ -446,8 +495,8 @@ static cudaError_t launch_mlp(const MlpArgs &m, cudaStream_t stream) {
         if (e != cudaSuccess) return e;
         attr_done[dev] = true;
     }
-    mlp_probe_kernel<<<(m.B + kMlpRows - 1) / kMlpRows, kMlpThreads, smem, stream>>>(m);
-    return cudaGetLastError();
+    return launch_pdl(mlp_probe_kernel, dim3((m.B + kMlpRows - 1) / kMlpRows), dim3(kMlpThreads), smem, stream, 0u,
+                      m);
 }
 
 // Shared validation and launch of switchsd_step / switchsd_verify_step.
@@ -500,14 +549,19 @@ static int step_entry(int32_t *ctx_tokens, int32_t *ctx_lens, const uint16_t *hi
 
     const int split = p->split > 0 ? p->split : choose_split(p->B, p->cap);
     // Tile: the largest CTA range (the last CTA may also cover a k + 1 token append), in one stage
-    // when it fits, else a ring of two kTileMax stages.
+    // when it fits, else a ring of kTileMax stages, as many as the range needs up to kMaxStages and
+    // the shared-memory budget.
     const int64_t range = ((int64_t(p->cap) - 1 + split - 1) / split + 3) / 4 * 4 + p->k + 1;
     if (range <= kTileMax) {
         args.tile = int32_t((range + 3) / 4 * 4);
         args.stages = 1;
     } else {
         args.tile = kTileMax;
-        args.stages = 2;
+        const int64_t need = (range + kTileMax - 1) / kTileMax;
+        const int64_t fit = int64_t(kStageSmemBudget / ((kHalo + kTileMax + kFwd) * sizeof(int32_t)));
+        args.stages = int32_t(need < fit ? need : fit);
+        if (args.stages > kMaxStages) args.stages = kMaxStages;
+        if (args.stages < 2) args.stages = 2;
     }
 
     if (p->probe_kind == SWITCHSD_PROBE_MLP) {

@@ -25,6 +25,8 @@ struct VerifyArgs {
 __global__ void __launch_bounds__(kVerifyThreads) verify_kernel(const VerifyArgs a) {
     const int lane = threadIdx.x & 31;
     const int b = (blockIdx.x * kVerifyThreads + threadIdx.x) >> 5;
+    pdl_wait();
+    pdl_trigger();
     if (b >= a.B) return;
     const int32_t len = a.draft_len[b];
     const int32_t L = a.lens[b];
@@ -86,6 +88,7 @@ extern "C" int switchsd_verify(const int32_t *draft, const int32_t *target_argma
     a.k = vp->k;
     const int warps_per_block = kVerifyThreads / kWarp;
     const int blocks = (vp->B + warps_per_block - 1) / warps_per_block;
-    verify_kernel<<<blocks, kVerifyThreads, 0, static_cast<cudaStream_t>(vp->stream)>>>(a);
-    return cudaGetLastError() == cudaSuccess ? SWITCHSD_OK : SWITCHSD_ERR_CUDA;
+    const cudaError_t e = launch_pdl(verify_kernel, dim3(blocks), dim3(kVerifyThreads), 0,
+                                     static_cast<cudaStream_t>(vp->stream), 0u, a);
+    return e == cudaSuccess ? SWITCHSD_OK : SWITCHSD_ERR_CUDA;
 }
