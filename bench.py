@@ -329,6 +329,16 @@ class ReplicaLoop:
         p.probe_kind, p.probe_hidden, p.b1, p.b2, p.split = wl.probe_kind, wl.probe_hidden, None, 0.0, split
         p.out_match_n = p.out_match_end = p.status = None
         p.stream = sp
+        # one workspace per batch, so consecutive launches never share one
+        probe = bd.switchsd_params()
+        probe.B, probe.probe_kind, probe.probe_hidden = B, wl.probe_kind, wl.probe_hidden
+        ws = max(256, int(self.lib.switchsd_workspace_bytes(ctypes.byref(probe))))
+        self.workspace = torch.empty(R, ws, dtype=torch.uint8, device=dev)
+        self.params = []
+        for r in range(R):
+            q = bd.switchsd_params.from_buffer_copy(p)
+            q.workspace, q.workspace_bytes = self.workspace[r].data_ptr(), ws
+            self.params.append(q)
         self.p = p
         hp = bd.switchsd_harness_params()
         h = wl.harness_params()
@@ -354,11 +364,13 @@ class ReplicaLoop:
         hid = self.hidden.data_ptr() + step_index * self.hstride
         if first:
             code = self.lib.switchsd_step(c["ctx"], c["lens"], hid, self.probe_w.data_ptr(),
-                                          self.ct.byref(self.p), c["draft"], c["len"], c["mode"], c["score"])
+                                          self.ct.byref(self.params[r]), c["draft"], c["len"], c["mode"],
+                                          c["score"])
         else:
             code = self.lib.switchsd_verify_step(c["vdraft"], c["target"], c["vlen"], c["accept"], c["ctx"],
-                                                 c["lens"], hid, self.probe_w.data_ptr(), self.ct.byref(self.p),
-                                                 c["draft"], c["len"], c["mode"], c["score"])
+                                                 c["lens"], hid, self.probe_w.data_ptr(),
+                                                 self.ct.byref(self.params[r]), c["draft"], c["len"],
+                                                 c["mode"], c["score"])
         if code != 0:
             raise RuntimeError(f"launch failed: {code} ({self.bd.strerror(code)})")
 
@@ -482,6 +494,12 @@ def run_ours(args, world, rank, local):
         outputs = 12 * B + 4 * B * k                       # mode, len, score, draft (bound)
         launch_bytes.extend((ctx_read + probe_bytes + verify_rw + outputs).tolist())
     launch_bytes = np.array(launch_bytes, dtype=np.float64)
+    # Every fused launch appends at least one token per row: a timed region in which some row did not
+    # grow did not run its launches.
+    for j in range(rounds):
+        n_this = min(R, K - j * R)
+        if np.any(Lh[j + 1][:n_this] <= Lh[j][:n_this]):
+            raise SystemExit(f"timed graph round {j}: rows did not grow; the launches did not run")
     peaks = measured_peaks()
     per_launch_s = region_s / K
     achieved = float(launch_bytes.mean() / per_launch_s / 1e9)

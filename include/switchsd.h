@@ -79,9 +79,14 @@ extern "C" {
  *   logit_tau    decision threshold in logit space: copy iff z >= logit_tau (Eq. 4 with tau;
  *                tau = 0.5 gives 0.0; -INFINITY copies on every match, +INFINITY never copies)
  *   probe_kind   SWITCHSD_PROBE_LINEAR or SWITCHSD_PROBE_MLP
- *   probe_hidden H1 of the two-layer probe (1..1024); ignored for the linear probe
+ *   probe_hidden H1 of the two-layer probe (1..1024); ignored for the linear probe.  The two-layer
+ *                probe also needs d <= 8192 (its first layer runs on the tensor cores).
  *   b1, b2       two-layer probe biases: b1 device float[H1] or NULL (zero), b2 a float
  *   split        CTAs per row (1, 2, 4, 8 or 16); 0 lets the library choose
+ *   workspace, workspace_bytes   device scratch for the two-layer probe: at least
+ *                switchsd_workspace_bytes(params) bytes, 16-byte aligned, caller-owned; may be NULL for
+ *                the linear probe.  It holds the probe's per-tile partial logits between its two kernels,
+ *                so calls sharing one workspace must not overlap on the GPU
  *   out_match_n, out_match_end   optional device int32[B]: the winning match length n* and the end
  *                position e* of its most recent earlier occurrence (0 / -1 when none); may be NULL
  *   status       optional device int32[B] per-row status (SWITCHSD_ROW_*); may be NULL
@@ -95,6 +100,8 @@ typedef struct {
     const float *b1;
     float b2;
     int32_t split;
+    void *workspace;
+    size_t workspace_bytes;
     int32_t *out_match_n;
     int32_t *out_match_end;
     int32_t *status;
@@ -183,6 +190,13 @@ int switchsd_verify_step(const int32_t *draft, const int32_t *target_argmax, con
                          const uint16_t *hidden, const uint16_t *probe_w,
                          const switchsd_params *params, int32_t *out_draft, int32_t *out_len,
                          int32_t *out_mode, float *out_score);
+
+/*
+ * Bytes of device workspace switchsd_step / switchsd_verify_step need for `params` (0 for the linear
+ * probe; for the two-layer probe, one float per row and 64-unit tile of the hidden layer, rounded up to
+ * 256 bytes).  Reads B, probe_kind and probe_hidden only.
+ */
+size_t switchsd_workspace_bytes(const switchsd_params *params);
 
 /* Human-readable text of a host return code or a row status (static storage, never NULL). */
 const char *switchsd_strerror(int code);

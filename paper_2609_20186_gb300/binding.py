@@ -31,6 +31,7 @@ class switchsd_params(ctypes.Structure):
         ("probe_kind", ctypes.c_int32), ("probe_hidden", ctypes.c_int32),
         ("b1", ctypes.c_void_p), ("b2", ctypes.c_float),
         ("split", ctypes.c_int32),
+        ("workspace", ctypes.c_void_p), ("workspace_bytes", ctypes.c_size_t),
         ("out_match_n", ctypes.c_void_p), ("out_match_end", ctypes.c_void_p),
         ("status", ctypes.c_void_p),
         ("stream", ctypes.c_void_p),
@@ -66,6 +67,7 @@ _SIGNATURES = {
     "switchsd_verify_step": (ctypes.c_int, [ctypes.c_void_p] * 8 + [ctypes.POINTER(switchsd_params)]
                              + [ctypes.c_void_p] * 4),
     "switchsd_strerror": (ctypes.c_char_p, [ctypes.c_int]),
+    "switchsd_workspace_bytes": (ctypes.c_size_t, [ctypes.POINTER(switchsd_params)]),
     "switchsd_abi_version": (ctypes.c_int, []),
     "switchsd_harness_target": (ctypes.c_int, [ctypes.c_void_p] * 8
                                 + [ctypes.POINTER(switchsd_harness_params)]),
@@ -135,7 +137,7 @@ def switchsd_step(ctx_tokens, ctx_lens, hidden, probe_w, out_draft, out_len, out
                   k: int, n_min: int, n_max: int, kappa: int = 0, logit_tau: float = 0.0,
                   probe_kind: int = PROBE_LINEAR, probe_hidden: int = 0, b1=None, b2: float = 0.0,
                   split: int = 0, out_match_n=None, out_match_end=None, status=None,
-                  stream=None) -> None:
+                  workspace=None, stream=None) -> None:
     """switchsd_step of include/switchsd.h on torch tensors (see the header for semantics).
 
     ctx_tokens int32 [B, cap]; ctx_lens int32 [B]; hidden bf16 [B, d]; probe_w bf16 (w[d] or
@@ -156,6 +158,7 @@ def switchsd_step(ctx_tokens, ctx_lens, hidden, probe_w, out_draft, out_len, out
     p.status = _dev(status, torch.int32, "status", (B,))
     p.stream = _stream_ptr(stream)
     nw = d if probe_kind == PROBE_LINEAR else probe_hidden * d + probe_hidden
+    ws = _attach_workspace(p, workspace, ctx_tokens.device)  # noqa: F841 (kept alive for the call)
     code = load().switchsd_step(
         _dev(ctx_tokens, torch.int32, "ctx_tokens"), _dev(ctx_lens, torch.int32, "ctx_lens", (B,)),
         _bf16(hidden, "hidden", (B, d)), _bf16(probe_w, "probe_w", (nw,)), ctypes.byref(p),
@@ -164,12 +167,34 @@ def switchsd_step(ctx_tokens, ctx_lens, hidden, probe_w, out_draft, out_len, out
     _check(code, "switchsd_step")
 
 
+def switchsd_workspace_bytes(B: int, probe_kind: int = PROBE_LINEAR, probe_hidden: int = 0) -> int:
+    """switchsd_workspace_bytes of include/switchsd.h for a batch of B rows."""
+    p = switchsd_params()
+    p.B, p.probe_kind, p.probe_hidden = B, probe_kind, probe_hidden
+    return int(load().switchsd_workspace_bytes(ctypes.byref(p)))
+
+
+def _attach_workspace(p: switchsd_params, workspace, device) -> torch.Tensor | None:
+    """Points p at `workspace` (a CUDA uint8 tensor), allocating one from torch when the probe needs it
+    and none was given.  Returns the tensor so the caller keeps it alive for the call."""
+    need = int(load().switchsd_workspace_bytes(ctypes.byref(p)))
+    if need == 0 and workspace is None:
+        return None
+    if workspace is None:
+        workspace = torch.empty(need, dtype=torch.uint8, device=device)
+    if not workspace.is_cuda or workspace.numel() * workspace.element_size() < need:
+        raise ValueError(f"workspace must be a CUDA tensor of at least {need} bytes")
+    p.workspace = workspace.data_ptr()
+    p.workspace_bytes = workspace.numel() * workspace.element_size()
+    return workspace
+
+
 def switchsd_verify_step(draft, target_argmax, draft_len, out_accept, ctx_tokens, ctx_lens, hidden,
                          probe_w, out_draft, out_len, out_mode, out_score, *, k: int, n_min: int,
                          n_max: int, kappa: int = 0, logit_tau: float = 0.0,
                          probe_kind: int = PROBE_LINEAR, probe_hidden: int = 0, b1=None,
                          b2: float = 0.0, split: int = 0, out_match_n=None, out_match_end=None,
-                         status=None, stream=None) -> None:
+                         status=None, workspace=None, stream=None) -> None:
     """switchsd_verify_step of include/switchsd.h: verification of the previous draft, then the next
     step, in one launch."""
     B, cap = ctx_tokens.shape
@@ -187,6 +212,7 @@ def switchsd_verify_step(draft, target_argmax, draft_len, out_accept, ctx_tokens
     p.status = _dev(status, torch.int32, "status", (B,))
     p.stream = _stream_ptr(stream)
     nw = d if probe_kind == PROBE_LINEAR else probe_hidden * d + probe_hidden
+    ws = _attach_workspace(p, workspace, ctx_tokens.device)  # noqa: F841 (kept alive for the call)
     code = load().switchsd_verify_step(
         _dev(draft, torch.int32, "draft", (B, k)),
         _dev(target_argmax, torch.int32, "target_argmax", (B, k + 1)),

@@ -31,6 +31,7 @@
 // them in a fixed order, applies the switch and writes the winner's draft.  No global scratch, no
 // atomics, no global re-read of the context.
 #include "common.cuh"
+#include "mlp.cuh"
 
 namespace switchsd {
 
@@ -52,7 +53,9 @@ struct StepArgs {
     int32_t *lens;           // read; written when verifying
     const uint16_t *hidden;
     const uint16_t *probe_w;
-    const float *z_pre;      // logits from the two-layer probe kernel, or null for the linear probe
+    const float *z_pre;      // two-layer probe: per-tile partial logits [z_tiles][B] (workspace), else null
+    int32_t z_tiles;
+    float b2;
     const int32_t *pv_draft; // previous draft [B, k] / target [B, k+1] / draft length [B]; null = no verify
     const int32_t *pv_target;
     const int32_t *pv_len;
@@ -349,7 +352,10 @@ __global__ void __launch_bounds__(kStepThreads) step_kernel(const StepArgs a) {
             }
             z += s_slot[r].z;
         }
-        if (a.z_pre != nullptr) z = a.z_pre[b];
+        if (a.z_pre != nullptr) {
+            z = a.b2;
+            for (int n = 0; n < a.z_tiles; ++n) z += a.z_pre[size_t(n) * a.B + b];
+        }
         const bool timeout = (key & kTimeoutBit) != 0;
         const bool hit = len_ok && !timeout && key != 0;
         const int32_t n = hit ? int32_t(key >> 32) : 0;
@@ -375,71 +381,6 @@ __global__ void __launch_bounds__(kStepThreads) step_kernel(const StepArgs a) {
     __syncthreads();
     const int32_t win = s_out[0], len = s_out[1];
     for (int i = tid; i < len; i += kStepThreads) a.out_draft[size_t(b) * a.k + i] = s_slot[win].cand[i];
-}
-
-// ------------------------------------------------------------------------------------------------
-// Two-layer probe z = w2 . ReLU(W1 h + b1) + b2 on CUDA cores (fp32 accumulation, fp32 hidden
-// layer).  Block = kMlpRows rows; warp w handles hidden units u = w, w + 8, ...; each lane streams
-// 16-byte slices of the W1 row and dots them with the rows' hidden vectors staged in shared memory.
-// ------------------------------------------------------------------------------------------------
-constexpr int kMlpRows = 4;
-constexpr int kMlpThreads = 256;
-
-struct MlpArgs {
-    const uint16_t *hidden;
-    const uint16_t *W1;
-    const uint16_t *w2;
-    const float *b1;
-    float b2;
-    int32_t B, d, H1;
-    float *z_out;
-};
-
-__global__ void __launch_bounds__(kMlpThreads) mlp_probe_kernel(const MlpArgs a) {
-    extern __shared__ __align__(16) uint4 hs[];  // kMlpRows x d/8
-    __shared__ float s_part[kMlpThreads / kWarp][kMlpRows];
-    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-    const int row0 = blockIdx.x * kMlpRows;
-    pdl_wait();
-    pdl_trigger();
-    const int nv = a.d >> 3;
-    for (int i = tid; i < kMlpRows * nv; i += kMlpThreads) {
-        const int r = i / nv, v = i % nv;
-        const int bb = row0 + r;
-        hs[i] = bb < a.B ? __ldg(reinterpret_cast<const uint4 *>(a.hidden + size_t(bb) * a.d) + v)
-                         : make_uint4(0, 0, 0, 0);
-    }
-    __syncthreads();
-    float zpart[kMlpRows];
-#pragma unroll
-    for (int r = 0; r < kMlpRows; ++r) zpart[r] = 0.f;
-    for (int u = warp; u < a.H1; u += kMlpThreads / kWarp) {
-        const uint4 *wrow = reinterpret_cast<const uint4 *>(a.W1 + size_t(u) * a.d);
-        float acc[kMlpRows];
-#pragma unroll
-        for (int r = 0; r < kMlpRows; ++r) acc[r] = 0.f;
-        for (int v = lane; v < nv; v += kWarp) {
-            const uint4 w = __ldg(wrow + v);
-#pragma unroll
-            for (int r = 0; r < kMlpRows; ++r) acc[r] = dot8_bf16(w, hs[r * nv + v], acc[r]);
-        }
-        const float bias = a.b1 ? a.b1[u] : 0.f;
-        const float w2u = bf16_lo(uint32_t(a.w2[u]));
-#pragma unroll
-        for (int r = 0; r < kMlpRows; ++r) {
-            const float pre = warp_sum_f32(acc[r]) + bias;
-            zpart[r] = fmaf(w2u, fmaxf(pre, 0.f), zpart[r]);
-        }
-    }
-    if (lane == 0)
-#pragma unroll
-        for (int r = 0; r < kMlpRows; ++r) s_part[warp][r] = zpart[r];
-    __syncthreads();
-    if (tid < kMlpRows && row0 + tid < a.B) {
-        float z = a.b2;
-        for (int w = 0; w < kMlpThreads / kWarp; ++w) z += s_part[w][tid];
-        a.z_out[row0 + tid] = z;
-    }
 }
 
 // ------------------------------------------------------------------------------------------------
@@ -484,21 +425,6 @@ static cudaError_t launch_step(const StepArgs &args, int split, cudaStream_t str
                       stream, unsigned(split), args);
 }
 
-static cudaError_t launch_mlp(const MlpArgs &m, cudaStream_t stream) {
-    const size_t smem = size_t(kMlpRows) * size_t(m.d) * 2;
-    static bool attr_done[64] = {false};
-    int dev = 0;
-    cudaGetDevice(&dev);
-    if (smem > 48 * 1024 && dev >= 0 && dev < 64 && !attr_done[dev]) {
-        cudaError_t e = cudaFuncSetAttribute(mlp_probe_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                             200 * 1024);
-        if (e != cudaSuccess) return e;
-        attr_done[dev] = true;
-    }
-    return launch_pdl(mlp_probe_kernel, dim3((m.B + kMlpRows - 1) / kMlpRows), dim3(kMlpThreads), smem, stream, 0u,
-                      m);
-}
-
 // Shared validation and launch of switchsd_step / switchsd_verify_step.
 static int step_entry(int32_t *ctx_tokens, int32_t *ctx_lens, const uint16_t *hidden, const uint16_t *probe_w,
                       const switchsd_params *p, const int32_t *pv_draft, const int32_t *pv_target,
@@ -515,10 +441,12 @@ static int step_entry(int32_t *ctx_tokens, int32_t *ctx_lens, const uint16_t *hi
     if (p->n_min < 1 || p->n_max > SWITCHSD_NMAX || p->n_min > p->n_max) return SWITCHSD_ERR_SHAPE;
     if (p->split != 0 && p->split != 1 && p->split != 2 && p->split != 4 && p->split != 8 && p->split != 16)
         return SWITCHSD_ERR_SHAPE;
-    if (p->probe_kind == SWITCHSD_PROBE_MLP && (p->probe_hidden < 1 || p->probe_hidden > 1024))
-        return SWITCHSD_ERR_SHAPE;
-    if (p->probe_kind == SWITCHSD_PROBE_MLP && size_t(kMlpRows) * size_t(p->d) * 2 > 200 * 1024)
-        return SWITCHSD_ERR_SHAPE;
+    if (p->probe_kind == SWITCHSD_PROBE_MLP) {
+        if (!mlp_shape_ok(p->d, p->probe_hidden)) return SWITCHSD_ERR_SHAPE;
+        if (!p->workspace || !aligned16(p->workspace) ||
+            p->workspace_bytes < switchsd_workspace_bytes(p))
+            return SWITCHSD_ERR_ARG;
+    }
 
     cudaStream_t stream = static_cast<cudaStream_t>(p->stream);
     StepArgs args;
@@ -564,19 +492,15 @@ static int step_entry(int32_t *ctx_tokens, int32_t *ctx_lens, const uint16_t *hi
         if (args.stages < 2) args.stages = 2;
     }
 
+    args.z_tiles = 0;
+    args.b2 = p->b2;
     if (p->probe_kind == SWITCHSD_PROBE_MLP) {
-        MlpArgs m;
-        m.hidden = hidden;
-        m.W1 = probe_w;
-        m.w2 = probe_w + size_t(p->probe_hidden) * size_t(p->d);
-        m.b1 = p->b1;
-        m.b2 = p->b2;
-        m.B = p->B;
-        m.d = p->d;
-        m.H1 = p->probe_hidden;
-        m.z_out = out_score;
-        if (launch_mlp(m, stream) != cudaSuccess) return SWITCHSD_ERR_CUDA;
-        args.z_pre = out_score;
+        float *zpart = static_cast<float *>(p->workspace);
+        if (launch_mlp_tc(hidden, probe_w, probe_w + size_t(p->probe_hidden) * size_t(p->d), p->b1, zpart, p->B, p->d,
+                          p->probe_hidden, stream) != cudaSuccess)
+            return SWITCHSD_ERR_CUDA;
+        args.z_pre = zpart;
+        args.z_tiles = mlp_tiles_n(p->probe_hidden);
     }
     if (launch_step(args, split, stream) != cudaSuccess) return SWITCHSD_ERR_CUDA;
     return SWITCHSD_OK;
@@ -585,6 +509,12 @@ static int step_entry(int32_t *ctx_tokens, int32_t *ctx_lens, const uint16_t *hi
 }  // namespace switchsd
 
 using namespace switchsd;
+
+extern "C" size_t switchsd_workspace_bytes(const switchsd_params *p) {
+    if (!p || p->probe_kind != SWITCHSD_PROBE_MLP || p->B < 1) return 0;
+    const int tiles = mlp_tiles_n(p->probe_hidden < 1 ? 1 : p->probe_hidden);
+    return (size_t(tiles) * size_t(p->B) * sizeof(float) + 255) / 256 * 256;
+}
 
 extern "C" int switchsd_step(const int32_t *ctx_tokens, const int32_t *ctx_lens, const uint16_t *hidden,
                              const uint16_t *probe_w, const switchsd_params *p, int32_t *out_draft,

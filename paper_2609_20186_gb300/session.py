@@ -34,6 +34,7 @@ class Session:
                  probe_kind: int = bd.PROBE_LINEAR, probe_hidden: int = 0, future=None,
                  harness: dict | None = None, split: int = 0, d: int | None = None,
                  device="cuda", stream: torch.cuda.Stream | None = None):
+        self.lib = bd.load()
         self.device = torch.device(device)
         if self.device.type == "cuda" and self.device.index is None:
             self.device = torch.device("cuda", torch.cuda.current_device())
@@ -64,7 +65,12 @@ class Session:
         if d is None:
             d = probe_w_bits.size if probe_kind == bd.PROBE_LINEAR else None
         self.d = d
-        self.lib = bd.load()
+
+        # workspace of the two-layer probe (none for the linear probe)
+        probe = bd.switchsd_params()
+        probe.B, probe.probe_kind, probe.probe_hidden = B, probe_kind, probe_hidden
+        ws_bytes = int(self.lib.switchsd_workspace_bytes(ctypes.byref(probe)))
+        self.workspace = torch.empty(max(ws_bytes, 256), dtype=torch.uint8, device=dev)
 
         # switchsd_step: two cached parameter blocks (with and without the debug outputs)
         def params(debug: bool):
@@ -72,6 +78,7 @@ class Session:
             p.B, p.cap, p.d, p.k = B, self.cap, d or 0, k
             p.n_min, p.n_max, p.kappa, p.logit_tau = n_min, n_max, kappa, logit_tau
             p.probe_kind, p.probe_hidden, p.b1, p.b2, p.split = probe_kind, probe_hidden, None, 0.0, split
+            p.workspace, p.workspace_bytes = self.workspace.data_ptr(), self.workspace.numel()
             p.out_match_n = self.match_n.data_ptr() if debug else None
             p.out_match_end = self.match_end.data_ptr() if debug else None
             p.status = self.status.data_ptr() if debug else None

@@ -91,6 +91,14 @@ def test_step_validation(lib):
     assert _step(lib, _params(n_max=33)) == bd.ERR_SHAPE
     assert _step(lib, _params(split=3)) == bd.ERR_SHAPE
     assert _step(lib, _params(probe_kind=1, probe_hidden=0)) == bd.ERR_SHAPE
+    # the two-layer probe needs its workspace
+    assert _step(lib, _params(probe_kind=1, probe_hidden=256)) == bd.ERR_ARG
+    need = bd.switchsd_workspace_bytes(4, 1, 256)
+    assert need >= 4 * 4 * 4 and need % 256 == 0
+    assert bd.switchsd_workspace_bytes(4, 0, 0) == 0
+    assert _step(lib, _params(probe_kind=1, probe_hidden=256, workspace=FAKE,
+                              workspace_bytes=need - 1)) == bd.ERR_ARG
+    assert _step(lib, _params(probe_kind=1, probe_hidden=256, d=8200)) == bd.ERR_SHAPE
 
 
 def test_verify_validation(lib):

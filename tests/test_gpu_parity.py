@@ -187,3 +187,38 @@ def test_device_harness_matches_host():
         assert np.array_equal(gvd.cpu().numpy(), vd)
         assert np.array_equal(gvl.cpu().numpy(), vl)
         assert np.array_equal(gtg.cpu().numpy(), tg)
+
+
+@pytest.mark.parametrize("B,d,H1,bias", [(256, 5120, 256, False), (130, 4096, 100, True),
+                                         (7, 1000, 64, True), (1, 64, 1, False),
+                                         (300, 8192, 1024, True), (129, 5120, 200, True)])
+def test_two_layer_probe_tensor_cores(B, d, H1, bias):
+    """The tcgen05 two-layer probe vs the oracle (double), through switchsd_step: ragged B (M tiles),
+    H1 (N tiles) and d (K chunks), with and without biases."""
+    import math
+    import torch
+    import oracle
+    from paper_2609_20186_gb300 import binding as bd, bf16_tensor
+
+    rng = np.random.default_rng(B * 7 + d + H1)
+    h = synth.bf16_bits_from_f32(rng.standard_normal((B, d)).astype(np.float32))
+    W1 = synth.bf16_bits_from_f32((rng.standard_normal((H1, d)) / math.sqrt(d)).astype(np.float32))
+    w2 = synth.bf16_bits_from_f32((rng.standard_normal(H1) / math.sqrt(H1)).astype(np.float32))
+    b1 = (rng.standard_normal(H1) * 0.2).astype(np.float32) if bias else None
+    b2 = 0.125 if bias else 0.0
+    cap = 64
+    ctx = torch.zeros(B, cap, dtype=torch.int32, device="cuda")
+    lens = torch.full((B,), 10, dtype=torch.int32, device="cuda")
+    out = dict(draft=torch.zeros(B, 8, dtype=torch.int32, device="cuda"),
+               len=torch.zeros(B, dtype=torch.int32, device="cuda"),
+               mode=torch.zeros(B, dtype=torch.int32, device="cuda"),
+               score=torch.zeros(B, dtype=torch.float32, device="cuda"))
+    pw = np.concatenate([W1.reshape(-1), w2])
+    bd.switchsd_step(ctx, lens, bf16_tensor(h, "cuda"), bf16_tensor(pw, "cuda"), out["draft"],
+                     out["len"], out["mode"], out["score"], k=8, n_min=2, n_max=4,
+                     probe_kind=bd.PROBE_MLP, probe_hidden=H1,
+                     b1=torch.from_numpy(b1).cuda() if bias else None, b2=b2)
+    got = out["score"].cpu().numpy()
+    for b in range(B):
+        ref = oracle.probe_mlp(h[b], W1, w2, b1=b1, b2=b2)
+        assert abs(got[b] - ref) <= 1e-3 * max(1.0, abs(ref)), (b, got[b], ref)
