@@ -1,0 +1,72 @@
+"""Host-side logic of bench.py: replica throughput over ranks (gloo, world size 2, CPU), replica
+count for the inputs-larger-than-L2 protocol, and the reference arm's JSON line."""
+import json
+import os
+import socket
+import subprocess
+import sys
+
+import pytest
+import torch.multiprocessing as mp
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+def _free_port():
+    with socket.socket() as s:
+        s.bind(("127.0.0.1", 0))
+        return s.getsockname()[1]
+
+
+def _worker(rank, world, port, out):
+    import torch.distributed as dist
+    sys.path.insert(0, ROOT)
+    import bench
+    os.environ.update(MASTER_ADDR="127.0.0.1", MASTER_PORT=str(port), RANK=str(rank),
+                      WORLD_SIZE=str(world), LOCAL_RANK=str(rank))
+    dist.init_process_group("gloo", rank=rank, world_size=world)
+    secs = [0.5, 2.0][rank]                     # rank 1 is the slow one
+    out[rank] = (bench.replica_throughput(100.0, secs, world), bench.reduce_max(secs, world))
+    dist.barrier()
+    dist.destroy_process_group()
+
+
+def test_replica_throughput_gloo_world2():
+    ctx = mp.get_context("spawn")
+    manager = ctx.Manager()
+    out = manager.dict()
+    port = _free_port()
+    procs = [ctx.Process(target=_worker, args=(r, 2, port, out)) for r in range(2)]
+    for p in procs:
+        p.start()
+    for p in procs:
+        p.join(120)
+        assert p.exitcode == 0
+    # whole-job throughput: all units of both replicas over the slowest rank's time
+    for r in range(2):
+        value, tmax = out[r]
+        assert tmax == 2.0
+        assert value == pytest.approx(200.0 / 2.0)
+
+
+def test_choose_replicas():
+    sys.path.insert(0, ROOT)
+    import bench
+    l2 = 126 << 20
+    r = bench.choose_replicas(10 << 20, l2, 512)
+    assert r & (r - 1) == 0 and r * (10 << 20) >= 2.2 * l2 and (r // 2) * (10 << 20) < 2.2 * l2
+    assert bench.choose_replicas(10 << 20, l2, 8) == 8        # never more batches than launches
+    assert bench.choose_replicas(1 << 30, l2, 512) == 1
+
+
+def test_reference_arm_line():
+    """--impl reference times the CPU oracle and prints one JSON line with the contract's keys."""
+    r = subprocess.run([sys.executable, os.path.join(ROOT, "bench.py"), "--impl", "reference",
+                        "--steps", "3", "--warmup", "1", "--workload", "uniform_8k"],
+                       capture_output=True, text=True, timeout=600, cwd=ROOT)
+    assert r.returncode == 0, r.stderr
+    line = json.loads(r.stdout.strip().splitlines()[-1])
+    assert line["impl"] == "reference" and line["steps"] == 3 and line["warmup"] == 1
+    assert line["value"] > 0 and line["cpu_baseline"]["kind"] == "oracle"
+    assert line["e2e"]["h2d_bytes_per_step"] == 0 and line["e2e"]["value"] == line["value"]
+    assert line["config"]["workload"] == "uniform_8k"
