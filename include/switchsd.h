@@ -198,6 +198,29 @@ int switchsd_verify_step(const int32_t *draft, const int32_t *target_argmax, con
  */
 size_t switchsd_workspace_bytes(const switchsd_params *params);
 
+/*
+ * switchsd_step for callers that cannot allocate device memory.  The paper has no counterpart: this is
+ * a convenience of the library.  Some callers cannot hand the library a workspace at call time (an
+ * inference server that gives all of the GPU's memory to its own pool when it starts, or a host program
+ * with no CUDA allocator of its own); this entry point takes the same arguments as switchsd_step, ignores
+ * params->workspace and uses a fixed 256 KiB array compiled into the library instead.  It allocates
+ * nothing (no cudaMalloc, no cudaFree).
+ *
+ *   Limit: the two-layer probe needs B * ceil(probe_hidden / 64) <= 65,536 (for example B <= 16,384
+ *   with 256 hidden units); larger requests return SWITCHSD_ERR_SHAPE.  The linear probe has no limit
+ *   beyond switchsd_step's.
+ *   Set-up: the first call on each device looks up the array's device address (cudaGetSymbolAddress,
+ *   with that device current); make that first call before any stream capture.
+ *   Sharing: every call on a device uses the same array, and the array keeps whatever the last call
+ *   left there.  Nothing in it needs to start at zero (each call writes every entry it reads), but calls
+ *   that overlap on the GPU race on it: issue them on one stream, or order them.
+ *   Every GPU that loads the library holds the array until the process exits.
+ */
+int switchsd_step_static_workspace(const int32_t *ctx_tokens, const int32_t *ctx_lens,
+                                   const uint16_t *hidden, const uint16_t *probe_w,
+                                   const switchsd_params *params, int32_t *out_draft,
+                                   int32_t *out_len, int32_t *out_mode, float *out_score);
+
 /* Human-readable text of a host return code or a row status (static storage, never NULL). */
 const char *switchsd_strerror(int code);
 

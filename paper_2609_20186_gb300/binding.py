@@ -66,6 +66,8 @@ _SIGNATURES = {
                         + [ctypes.POINTER(switchsd_verify_params)]),
     "switchsd_verify_step": (ctypes.c_int, [ctypes.c_void_p] * 8 + [ctypes.POINTER(switchsd_params)]
                              + [ctypes.c_void_p] * 4),
+    "switchsd_step_static_workspace": (ctypes.c_int, [ctypes.c_void_p] * 4
+                                       + [ctypes.POINTER(switchsd_params)] + [ctypes.c_void_p] * 4),
     "switchsd_strerror": (ctypes.c_char_p, [ctypes.c_int]),
     "switchsd_workspace_bytes": (ctypes.c_size_t, [ctypes.POINTER(switchsd_params)]),
     "switchsd_abi_version": (ctypes.c_int, []),
