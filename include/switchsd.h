@@ -67,6 +67,9 @@ extern "C" {
 #define SWITCHSD_ROW_BAD_LEN 2  /* ctx_lens[b] outside [1, cap] or draft_len[b] outside [0, k] */
 #define SWITCHSD_ROW_TIMEOUT 3  /* an on-chip copy did not complete within its wait limit */
 
+/* Incremental n-gram index (switchsd_index_create); opaque. */
+typedef struct switchsd_index switchsd_index;
+
 /*
  * Parameters of switchsd_step.
  *
@@ -87,6 +90,10 @@ extern "C" {
  *                switchsd_workspace_bytes(params) bytes, 16-byte aligned, caller-owned; may be NULL for
  *                the linear probe.  It holds the probe's per-tile partial logits between its two kernels,
  *                so calls sharing one workspace must not overlap on the GPU
+ *   index        NULL: search by rescanning the context.  Else an index from switchsd_index_create for
+ *                the same B, cap, n_min and n_max, kept current by switchsd_index_build and by the
+ *                verification entry points given the same index; the search then walks its chains
+ *                (same results as the rescan).  Ignores split.
  *   out_match_n, out_match_end   optional device int32[B]: the winning match length n* and the end
  *                position e* of its most recent earlier occurrence (0 / -1 when none); may be NULL
  *   status       optional device int32[B] per-row status (SWITCHSD_ROW_*); may be NULL
@@ -102,6 +109,7 @@ typedef struct {
     int32_t split;
     void *workspace;
     size_t workspace_bytes;
+    switchsd_index *index;
     int32_t *out_match_n;
     int32_t *out_match_end;
     int32_t *status;
@@ -143,6 +151,7 @@ int switchsd_step(const int32_t *ctx_tokens, const int32_t *ctx_lens, const uint
  *   ctx_tokens   device int32 [B, cap] (modified: accepted tokens are appended)
  *   ctx_lens     device int32 [B]      (modified: grows by accepted + 1)
  *   status       optional device int32 [B]; may be NULL
+ *   index        NULL, or the row index (see switchsd_params): the appended positions are inserted
  *   stream       cudaStream_t as void*
  */
 typedef struct {
@@ -151,6 +160,7 @@ typedef struct {
     int32_t *ctx_tokens;
     int32_t *ctx_lens;
     int32_t *status;
+    switchsd_index *index;
     void *stream;
 } switchsd_verify_params;
 
@@ -220,6 +230,31 @@ int switchsd_step_static_workspace(const int32_t *ctx_tokens, const int32_t *ctx
                                    const uint16_t *hidden, const uint16_t *probe_w,
                                    const switchsd_params *params, int32_t *out_draft,
                                    int32_t *out_len, int32_t *out_mode, float *out_score);
+
+/*
+ * Incremental n-gram index: the search of §3.3 without rescanning the context.  Not in the paper (it
+ * states only the search's result); the index returns exactly the rescan's (n*, e*).
+ *
+ * For every row and every n in [n_min, n_max] it keeps hash heads (the most recent end position of
+ * each bucket of n-grams, at least 2 cap buckets) and a chain of previous end positions per bucket.
+ * A lookup walks the suffix's chain from the most recent entry and verifies candidates token by token,
+ * so collisions cost time, never correctness.  Appended tokens are inserted by switchsd_verify and
+ * switchsd_verify_step when their params carry the index.
+ *
+ *   switchsd_index_create   allocates the index for params' B, cap, n_min, n_max (device memory, the
+ *                           library's only allocation: see switchsd_index_bytes); SWITCHSD_ERR_CUDA if
+ *                           the allocation fails.  The index belongs to the current device.
+ *   switchsd_index_build    (re)builds it from ctx_tokens / ctx_lens on `stream` (asynchronous); call
+ *                           it once for the initial contexts and after any change made outside the
+ *                           library's verification entry points.
+ *   switchsd_index_bytes    device bytes the index holds.
+ *   switchsd_index_destroy  frees it (NULL is a no-op); no call using it may still be in flight.
+ */
+int switchsd_index_create(const switchsd_params *params, switchsd_index **out);
+int switchsd_index_build(switchsd_index *index, const int32_t *ctx_tokens, const int32_t *ctx_lens,
+                         void *stream);
+size_t switchsd_index_bytes(const switchsd_index *index);
+void switchsd_index_destroy(switchsd_index *index);
 
 /* Human-readable text of a host return code or a row status (static storage, never NULL). */
 const char *switchsd_strerror(int code);

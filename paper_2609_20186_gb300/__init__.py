@@ -9,7 +9,7 @@ loudly if it was not built.
 """
 from .binding import (  # noqa: F401
     switchsd_step, switchsd_verify, switchsd_verify_step, switchsd_harness_target, switchsd_params,
-    switchsd_verify_params, switchsd_harness_params, load, strerror, abi_version,
+    switchsd_verify_params, switchsd_harness_params, NgramIndex, load, strerror, abi_version,
     MODE_NO_REP, MODE_COPY, MODE_REP_NO_COPY, PROBE_LINEAR, PROBE_MLP,
 )
 from .session import Session, bf16_tensor  # noqa: F401

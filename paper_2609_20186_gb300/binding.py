@@ -32,6 +32,7 @@ class switchsd_params(ctypes.Structure):
         ("b1", ctypes.c_void_p), ("b2", ctypes.c_float),
         ("split", ctypes.c_int32),
         ("workspace", ctypes.c_void_p), ("workspace_bytes", ctypes.c_size_t),
+        ("index", ctypes.c_void_p),
         ("out_match_n", ctypes.c_void_p), ("out_match_end", ctypes.c_void_p),
         ("status", ctypes.c_void_p),
         ("stream", ctypes.c_void_p),
@@ -42,7 +43,8 @@ class switchsd_verify_params(ctypes.Structure):
     _fields_ = [
         ("B", ctypes.c_int32), ("cap", ctypes.c_int32), ("k", ctypes.c_int32),
         ("draft_len", ctypes.c_void_p), ("ctx_tokens", ctypes.c_void_p),
-        ("ctx_lens", ctypes.c_void_p), ("status", ctypes.c_void_p), ("stream", ctypes.c_void_p),
+        ("ctx_lens", ctypes.c_void_p), ("status", ctypes.c_void_p), ("index", ctypes.c_void_p),
+        ("stream", ctypes.c_void_p),
     ]
 
 
@@ -68,6 +70,11 @@ _SIGNATURES = {
                              + [ctypes.c_void_p] * 4),
     "switchsd_step_static_workspace": (ctypes.c_int, [ctypes.c_void_p] * 4
                                        + [ctypes.POINTER(switchsd_params)] + [ctypes.c_void_p] * 4),
+    "switchsd_index_create": (ctypes.c_int, [ctypes.POINTER(switchsd_params),
+                                             ctypes.POINTER(ctypes.c_void_p)]),
+    "switchsd_index_build": (ctypes.c_int, [ctypes.c_void_p] * 4),
+    "switchsd_index_bytes": (ctypes.c_size_t, [ctypes.c_void_p]),
+    "switchsd_index_destroy": (None, [ctypes.c_void_p]),
     "switchsd_strerror": (ctypes.c_char_p, [ctypes.c_int]),
     "switchsd_workspace_bytes": (ctypes.c_size_t, [ctypes.POINTER(switchsd_params)]),
     "switchsd_abi_version": (ctypes.c_int, []),
@@ -174,6 +181,40 @@ def switchsd_workspace_bytes(B: int, probe_kind: int = PROBE_LINEAR, probe_hidde
     p = switchsd_params()
     p.B, p.probe_kind, p.probe_hidden = B, probe_kind, probe_hidden
     return int(load().switchsd_workspace_bytes(ctypes.byref(p)))
+
+
+class NgramIndex:
+    """switchsd_index_* of include/switchsd.h: the incremental n-gram index of B rows (device memory
+    owned by the library, freed by close() or when the object is collected)."""
+
+    def __init__(self, B: int, cap: int, n_min: int, n_max: int):
+        p = switchsd_params()
+        p.B, p.cap, p.n_min, p.n_max = B, cap, n_min, n_max
+        h = ctypes.c_void_p()
+        _check(load().switchsd_index_create(ctypes.byref(p), ctypes.byref(h)), "switchsd_index_create")
+        self.handle = h.value
+        self.B, self.cap, self.n_min, self.n_max = B, cap, n_min, n_max
+
+    def build(self, ctx_tokens: torch.Tensor, ctx_lens: torch.Tensor, stream=None) -> None:
+        _check(load().switchsd_index_build(self.handle, _dev(ctx_tokens, torch.int32, "ctx_tokens",
+                                                             (self.B, self.cap)),
+                                           _dev(ctx_lens, torch.int32, "ctx_lens", (self.B,)),
+                                           _stream_ptr(stream)), "switchsd_index_build")
+
+    @property
+    def nbytes(self) -> int:
+        return int(load().switchsd_index_bytes(self.handle))
+
+    def close(self) -> None:
+        if self.handle:
+            load().switchsd_index_destroy(self.handle)
+            self.handle = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
 
 
 def _attach_workspace(p: switchsd_params, workspace, device) -> torch.Tensor | None:

@@ -1,0 +1,379 @@
+// index.cu -- incremental n-gram index: the same (n*, e*) as the rescan, from hash chains.
+//
+// For every row b and every n in [n_min, n_max] the index keeps
+//   heads[n][b][bucket]  the most recent end position e whose n-gram x[e-n+1..e] hashes to bucket,
+//   prev[n][b][e]        the previous end position with the same bucket (-1 at the end of a chain).
+// Contexts only grow and positions are inserted in increasing order, so every chain lists end
+// positions in decreasing order.  Looking up the suffix n-gram walks its bucket's chain from the head,
+// skips the suffix's own end (L-1) and compares candidates token by token; the first exact match is
+// the most recent earlier occurrence (§3.3's recency ranking).  n* is the largest n with a match and
+// e* its end: exactly the rescan's answer, hash collisions included (they only lengthen the walk).
+//
+// index_kernel runs one CTA per row with one warp per n and does, in order:
+//   verification of the previous draft (as switchsd_verify) and its append, when verifying;
+//   insertion of the appended end positions (all lanes at once; positions of one run that fall into
+//   the same bucket are linked through __match_any_sync, so one read of the old heads suffices);
+//   the lookup, the probe and the switch / copy draft (as switchsd_step), when stepping.
+#include <new>
+
+#include "common.cuh"
+#include "mlp.cuh"
+
+struct switchsd_index {
+    int32_t B, cap, n_min, n_max, nn, log2_buckets;
+    int32_t *heads;  // [nn][B][1 << log2_buckets]
+    int32_t *prev;   // [nn][B][cap]
+    int device;
+};
+
+namespace switchsd {
+
+constexpr int kIdxMaxWarps = SWITCHSD_NMAX;
+constexpr int kIdxTail = SWITCHSD_NMAX + SWITCHSD_KMAX + 1;  // staged context tail: old end +- the append
+
+// Multiply-xorshift hash of the n tokens ending at the last one (`tok(i)` = token i steps back).
+template <typename Tok>
+__device__ __forceinline__ uint32_t gram_hash(int n, Tok tok, int log2_buckets) {
+    uint64_t h = 0x243F6A8885A308D3ull ^ uint64_t(n);
+    for (int i = 0; i < n; ++i) {
+        h = (h ^ uint64_t(uint32_t(tok(i)))) * 0x9E3779B97F4A7C15ull;
+        h ^= h >> 29;
+    }
+    return uint32_t(h >> (64 - log2_buckets));
+}
+
+struct IndexArgs {
+    int32_t *ctx, *lens;
+    const uint16_t *hidden, *probe_w;
+    const float *z_pre;  // two-layer probe partial logits, else null
+    int32_t z_tiles;
+    float b2;
+    const int32_t *pv_draft, *pv_target, *pv_len;  // verification inputs (null: no verification)
+    int32_t *out_accept;
+    int32_t *out_draft, *out_len, *out_mode;
+    float *out_score;
+    int32_t *out_match_n, *out_match_end, *status;
+    int32_t *heads, *prev;
+    int32_t B, cap, d, k, n_min, n_max, kappa, log2_buckets, stepping;
+    float logit_tau;
+};
+
+__global__ void __launch_bounds__(kIdxMaxWarps * kWarp) index_kernel(const IndexArgs a) {
+    __shared__ int32_t s_tail[kIdxTail];     // x[L_old - NMAX .. L_old + KMAX]
+    __shared__ int32_t s_ver[3];             // accepted, new length, status
+    __shared__ int32_t s_found[kIdxMaxWarps];
+    __shared__ float s_wz[kIdxMaxWarps];
+    __shared__ int32_t s_out[3];
+
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    const int nwarps = blockDim.x >> 5;
+    const int b = blockIdx.x;
+    const bool verifying = a.pv_len != nullptr;
+    pdl_wait();
+    pdl_trigger();
+
+    int32_t *row = a.ctx + size_t(b) * a.cap;
+    const int32_t L_old = a.lens[b];
+    const bool len_ok = L_old >= 1 && L_old <= a.cap;
+    const int32_t tail0 = L_old - SWITCHSD_NMAX;  // s_tail[i] = x[tail0 + i]
+    for (int i = tid; i < SWITCHSD_NMAX; i += blockDim.x) {
+        const int32_t p = tail0 + i;
+        s_tail[i] = (len_ok && p >= 0) ? row[p] : 0;
+    }
+    if (warp == 0) {
+        int32_t acc = -1, L = L_old, vst = len_ok ? SWITCHSD_ROW_OK : SWITCHSD_ROW_BAD_LEN;
+        if (verifying && len_ok) {
+            const int32_t n = a.pv_len[b];
+            if (n < 0 || n > a.k) {
+                vst = SWITCHSD_ROW_BAD_LEN;
+            } else {
+                const int32_t *dr = a.pv_draft + size_t(b) * a.k;
+                const int32_t *tg = a.pv_target + size_t(b) * (a.k + 1);
+                acc = n;
+                for (int base = 0; base < n; base += kWarp) {
+                    const int i = base + lane;
+                    const unsigned m = __ballot_sync(kFull, i < n && dr[i] != tg[i]);
+                    if (m) {
+                        acc = base + __ffs(m) - 1;
+                        break;
+                    }
+                }
+                if (L_old + acc + 1 > a.cap) {
+                    vst = SWITCHSD_ROW_CAPACITY;
+                    acc = -1;
+                } else {
+                    for (int i = lane; i <= acc; i += kWarp) {
+                        const int32_t t = i < acc ? dr[i] : tg[acc];
+                        s_tail[SWITCHSD_NMAX + i] = t;
+                        row[L_old + i] = t;
+                    }
+                    L = L_old + acc + 1;
+                }
+            }
+        }
+        if (lane == 0) {
+            s_ver[0] = acc;
+            s_ver[1] = L;
+            s_ver[2] = vst;
+            if (verifying && len_ok) {
+                a.lens[b] = L;
+                a.out_accept[b] = acc;
+            } else if (verifying) {
+                a.out_accept[b] = -1;
+            }
+            if (!a.stepping && a.status) a.status[b] = vst;
+        }
+    }
+    __syncthreads();
+    const int32_t L = s_ver[1];
+    const int n = a.n_min + warp;  // this warp's gram length
+    const bool has_n = warp < a.n_max - a.n_min + 1;
+    const size_t nb = size_t(1) << a.log2_buckets;
+    int32_t *heads = a.heads + (size_t(warp) * a.B + b) * nb;
+    int32_t *prev = a.prev + (size_t(warp) * a.B + b) * a.cap;
+    auto tail_tok = [&](int32_t p) { return s_tail[p - tail0]; };  // valid for p in [tail0, L)
+
+    // Insert the appended end positions p in [L_old, L) (lanes over p, chained through match_any).
+    if (has_n && L > L_old) {
+        for (int32_t base = L_old; base < L; base += kWarp) {
+            const int32_t p = base + lane;
+            const bool valid = p < L && p >= n - 1;
+            uint32_t bucket = 0xffffffffu;
+            if (valid) bucket = gram_hash(n, [&](int i) { return tail_tok(p - i); }, a.log2_buckets);
+            const unsigned peers = __match_any_sync(kFull, bucket) & __ballot_sync(kFull, valid);
+            const int32_t old_head = valid ? heads[bucket] : -1;
+            __syncwarp();  // every lane has read its head before any lane replaces one
+            if (valid) {
+                const unsigned earlier = peers & ((1u << lane) - 1u);
+                prev[p] = earlier ? base + (31 - __clz(earlier)) : old_head;
+                if ((peers >> lane) == 1u) heads[bucket] = p;  // the latest position of the run
+            }
+            __syncwarp();
+        }
+    }
+    if (!a.stepping) return;
+
+    // Lookup: the most recent earlier occurrence of the suffix n-gram, if any.
+    int32_t found = -1;
+    if (has_n && len_ok && L >= n + 1) {
+        const uint32_t bucket = gram_hash(n, [&](int i) { return tail_tok(L - 1 - i); }, a.log2_buckets);
+        const int32_t mine = lane < n ? tail_tok(L - 1 - lane) : 0;
+        int32_t e = heads[bucket];
+        // A valid chain strictly decreases and ends at -1 within L hops; the bounds keep a stale or
+        // unbuilt index from reading outside its tables.
+        for (int32_t hops = 0; e >= 0 && e < a.cap && hops < a.cap; ++hops) {
+            if (e <= L - 2 && e >= n - 1) {
+                const bool eq = lane >= n || row[e - lane] == mine;
+                if (__all_sync(kFull, eq)) {
+                    found = e;
+                    break;
+                }
+            }
+            e = prev[e];
+        }
+    }
+    if (lane == 0 && warp < kIdxMaxWarps) s_found[warp] = found;
+
+    // Probe partial over the whole hidden vector (linear probe).
+    float zp = 0.f;
+    if (a.z_pre == nullptr) {
+        const uint4 *h4 = reinterpret_cast<const uint4 *>(a.hidden + size_t(b) * a.d);
+        const uint4 *w4 = reinterpret_cast<const uint4 *>(a.probe_w);
+        for (int v = tid; v < (a.d >> 3); v += blockDim.x) {
+            const uint4 w = __ldg(w4 + v), h = __ldg(h4 + v);
+            zp = fmaf(bf16_lo(w.x), bf16_lo(h.x), zp);
+            zp = fmaf(bf16_hi(w.x), bf16_hi(h.x), zp);
+            zp = fmaf(bf16_lo(w.y), bf16_lo(h.y), zp);
+            zp = fmaf(bf16_hi(w.y), bf16_hi(h.y), zp);
+            zp = fmaf(bf16_lo(w.z), bf16_lo(h.z), zp);
+            zp = fmaf(bf16_hi(w.z), bf16_hi(h.z), zp);
+            zp = fmaf(bf16_lo(w.w), bf16_lo(h.w), zp);
+            zp = fmaf(bf16_hi(w.w), bf16_hi(h.w), zp);
+        }
+    }
+    zp = warp_sum_f32(zp);
+    if (lane == 0) s_wz[warp] = zp;
+    __syncthreads();
+
+    if (tid == 0) {
+        float z = 0.f;
+        if (a.z_pre != nullptr) {
+            z = a.b2;
+            for (int t = 0; t < a.z_tiles; ++t) z += a.z_pre[size_t(t) * a.B + b];
+        } else {
+            for (int w = 0; w < nwarps; ++w) z += s_wz[w];
+        }
+        int32_t nstar = 0, estar = -1;
+        for (int w = a.n_max - a.n_min; w >= 0; --w)
+            if (s_found[w] >= 0) {
+                nstar = a.n_min + w;
+                estar = s_found[w];
+                break;
+            }
+        const bool hit = len_ok && nstar > 0;
+        const int32_t kappa = a.kappa > 0 ? a.kappa : a.n_min;
+        int32_t mode = SWITCHSD_MODE_NO_REP;
+        if (hit) mode = (nstar >= kappa && z >= a.logit_tau) ? SWITCHSD_MODE_COPY : SWITCHSD_MODE_REP_NO_COPY;
+        const int32_t len = mode == SWITCHSD_MODE_COPY ? min(a.k, L - 1 - estar) : 0;
+        s_out[0] = estar;
+        s_out[1] = len;
+        a.out_mode[b] = mode;
+        a.out_len[b] = len;
+        a.out_score[b] = z;
+        if (a.out_match_n) a.out_match_n[b] = nstar;
+        if (a.out_match_end) a.out_match_end[b] = estar;
+        if (a.status) a.status[b] = s_ver[2];
+    }
+    __syncthreads();
+    const int32_t e = s_out[0], len = s_out[1];
+    // The copy draft x[e+1 .. e+len]: positions below L_old are in global memory, the rest in s_tail.
+    for (int i = tid; i < len; i += blockDim.x) {
+        const int32_t p = e + 1 + i;
+        a.out_draft[size_t(b) * a.k + i] = p >= L_old ? tail_tok(p) : row[p];
+    }
+}
+
+// Build: positions n-1 .. L-1 of every (row, n) inserted in increasing order, 32 per warp iteration.
+__global__ void __launch_bounds__(256) index_build_kernel(const int32_t *ctx, const int32_t *lens, int32_t *heads_all,
+                                                          int32_t *prev_all, int32_t B, int32_t cap, int32_t n_min,
+                                                          int32_t nn, int32_t log2_buckets) {
+    const int lane = threadIdx.x & 31;
+    const int gw = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;  // one warp per (n, row)
+    pdl_wait();
+    pdl_trigger();
+    if (gw >= nn * B) return;
+    const int w = gw / B, b = gw % B;
+    const int n = n_min + w;
+    const size_t nb = size_t(1) << log2_buckets;
+    int32_t *heads = heads_all + (size_t(w) * B + b) * nb;
+    int32_t *prev = prev_all + (size_t(w) * B + b) * cap;
+    const int32_t *row = ctx + size_t(b) * cap;
+    int32_t L = lens[b];
+    if (L < 0 || L > cap) L = 0;
+    for (int32_t base = 0; base < L; base += kWarp) {
+        const int32_t p = base + lane;
+        const bool valid = p < L && p >= n - 1;
+        uint32_t bucket = 0xffffffffu;
+        if (valid) bucket = gram_hash(n, [&](int i) { return row[p - i]; }, log2_buckets);
+        const unsigned peers = __match_any_sync(kFull, bucket) & __ballot_sync(kFull, valid);
+        const int32_t old_head = valid ? heads[bucket] : -1;
+        __syncwarp();  // every lane has read its head before any lane replaces one
+        if (valid) {
+            const unsigned earlier = peers & ((1u << lane) - 1u);
+            prev[p] = earlier ? base + (31 - __clz(earlier)) : old_head;
+            if ((peers >> lane) == 1u) heads[bucket] = p;
+        }
+        __syncwarp();
+    }
+}
+
+// ------------------------------------------------------------------------------------------------
+// Host side.
+// ------------------------------------------------------------------------------------------------
+int index_n_min(const switchsd_index *idx) { return idx->n_min; }
+int index_n_max(const switchsd_index *idx) { return idx->n_max; }
+
+int index_launch(switchsd_index *idx, int32_t *ctx, int32_t *lens, const uint16_t *hidden, const uint16_t *probe_w,
+                 const float *z_pre, int z_tiles, float b2, const int32_t *pv_draft, const int32_t *pv_target,
+                 const int32_t *pv_len, int32_t *out_accept, int32_t *out_draft, int32_t *out_len, int32_t *out_mode,
+                 float *out_score, int32_t *out_match_n, int32_t *out_match_end, int32_t *status, int B, int cap,
+                 int d, int k, int n_min, int n_max, int kappa, float logit_tau, bool stepping, cudaStream_t stream) {
+    if (idx->B != B || idx->cap != cap || idx->n_min != n_min || idx->n_max != n_max) return SWITCHSD_ERR_SHAPE;
+    IndexArgs a;
+    a.ctx = ctx;
+    a.lens = lens;
+    a.hidden = hidden;
+    a.probe_w = probe_w;
+    a.z_pre = z_pre;
+    a.z_tiles = z_tiles;
+    a.b2 = b2;
+    a.pv_draft = pv_draft;
+    a.pv_target = pv_target;
+    a.pv_len = pv_len;
+    a.out_accept = out_accept;
+    a.out_draft = out_draft;
+    a.out_len = out_len;
+    a.out_mode = out_mode;
+    a.out_score = out_score;
+    a.out_match_n = out_match_n;
+    a.out_match_end = out_match_end;
+    a.status = status;
+    a.heads = idx->heads;
+    a.prev = idx->prev;
+    a.B = B;
+    a.cap = cap;
+    a.d = d;
+    a.k = k;
+    a.n_min = n_min;
+    a.n_max = n_max;
+    a.kappa = kappa;
+    a.log2_buckets = idx->log2_buckets;
+    a.stepping = stepping ? 1 : 0;
+    a.logit_tau = logit_tau;
+    const cudaError_t e = launch_pdl(index_kernel, dim3(unsigned(B)), dim3(unsigned(idx->nn * kWarp)), 0, stream, 0u, a);
+    return e == cudaSuccess ? SWITCHSD_OK : SWITCHSD_ERR_CUDA;
+}
+
+}  // namespace switchsd
+
+using namespace switchsd;
+
+extern "C" int switchsd_index_create(const switchsd_params *p, switchsd_index **out) {
+    if (!p || !out) return SWITCHSD_ERR_ARG;
+    *out = nullptr;
+    if (p->B < 1 || p->B > 65535 || p->cap < 4 || (p->cap & 3) != 0) return SWITCHSD_ERR_SHAPE;
+    if (p->n_min < 1 || p->n_max > SWITCHSD_NMAX || p->n_min > p->n_max) return SWITCHSD_ERR_SHAPE;
+    switchsd_index *idx = new (std::nothrow) switchsd_index();
+    if (!idx) return SWITCHSD_ERR_CUDA;
+    idx->B = p->B;
+    idx->cap = p->cap;
+    idx->n_min = p->n_min;
+    idx->n_max = p->n_max;
+    idx->nn = p->n_max - p->n_min + 1;
+    int lg = 4;
+    while ((int64_t(1) << lg) < 2 * int64_t(p->cap) && lg < 30) ++lg;  // load factor <= 1/2
+    idx->log2_buckets = lg;
+    cudaGetDevice(&idx->device);
+    const size_t heads = size_t(idx->nn) * size_t(p->B) * (size_t(1) << lg) * sizeof(int32_t);
+    const size_t prev = size_t(idx->nn) * size_t(p->B) * size_t(p->cap) * sizeof(int32_t);
+    if (cudaMalloc(&idx->heads, heads) != cudaSuccess) {
+        delete idx;
+        return SWITCHSD_ERR_CUDA;
+    }
+    if (cudaMalloc(&idx->prev, prev) != cudaSuccess) {
+        cudaFree(idx->heads);
+        delete idx;
+        return SWITCHSD_ERR_CUDA;
+    }
+    *out = idx;
+    return SWITCHSD_OK;
+}
+
+extern "C" int switchsd_index_build(switchsd_index *idx, const int32_t *ctx_tokens, const int32_t *ctx_lens,
+                                    void *stream) {
+    if (!idx || !ctx_tokens || !ctx_lens) return SWITCHSD_ERR_ARG;
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    const size_t heads = size_t(idx->nn) * size_t(idx->B) * (size_t(1) << idx->log2_buckets) * sizeof(int32_t);
+    if (cudaMemsetAsync(idx->heads, 0xff, heads, s) != cudaSuccess) return SWITCHSD_ERR_CUDA;  // every head = -1
+    const int warps = idx->nn * idx->B;
+    const cudaError_t e = launch_pdl(index_build_kernel, dim3(unsigned((warps + 7) / 8)), dim3(256), 0, s, 0u,
+                                     ctx_tokens, ctx_lens, idx->heads, idx->prev, idx->B, idx->cap, idx->n_min,
+                                     idx->nn, idx->log2_buckets);
+    return e == cudaSuccess ? SWITCHSD_OK : SWITCHSD_ERR_CUDA;
+}
+
+extern "C" size_t switchsd_index_bytes(const switchsd_index *idx) {
+    if (!idx) return 0;
+    return size_t(idx->nn) * size_t(idx->B) * ((size_t(1) << idx->log2_buckets) + size_t(idx->cap)) * sizeof(int32_t);
+}
+
+extern "C" void switchsd_index_destroy(switchsd_index *idx) {
+    if (!idx) return;
+    int cur = 0;
+    cudaGetDevice(&cur);
+    if (cur != idx->device) cudaSetDevice(idx->device);
+    cudaFree(idx->heads);
+    cudaFree(idx->prev);
+    if (cur != idx->device) cudaSetDevice(cur);
+    delete idx;
+}

@@ -35,6 +35,12 @@
 
 namespace switchsd {
 
+int index_launch(switchsd_index *idx, int32_t *ctx, int32_t *lens, const uint16_t *hidden, const uint16_t *probe_w,
+                 const float *z_pre, int z_tiles, float b2, const int32_t *pv_draft, const int32_t *pv_target,
+                 const int32_t *pv_len, int32_t *out_accept, int32_t *out_draft, int32_t *out_len, int32_t *out_mode,
+                 float *out_score, int32_t *out_match_n, int32_t *out_match_end, int32_t *status, int B, int cap,
+                 int d, int k, int n_min, int n_max, int kappa, float logit_tau, bool stepping, cudaStream_t stream);
+
 constexpr int kStepThreads = 256;
 constexpr int kStepWarps = kStepThreads / kWarp;
 constexpr int kTileMax = 8192;        // largest staged tile (candidate ends)
@@ -502,6 +508,11 @@ static int step_entry(int32_t *ctx_tokens, int32_t *ctx_lens, const uint16_t *hi
         args.z_pre = zpart;
         args.z_tiles = mlp_tiles_n(p->probe_hidden);
     }
+    if (p->index != nullptr)
+        return index_launch(p->index, ctx_tokens, ctx_lens, hidden, probe_w, args.z_pre, args.z_tiles, args.b2, pv_draft,
+                            pv_target, pv_len, out_accept, out_draft, out_len, out_mode, out_score, p->out_match_n,
+                            p->out_match_end, p->status, p->B, p->cap, p->d, p->k, p->n_min, p->n_max, p->kappa,
+                            p->logit_tau, true, stream);
     if (launch_step(args, split, stream) != cudaSuccess) return SWITCHSD_ERR_CUDA;
     return SWITCHSD_OK;
 }

@@ -33,7 +33,7 @@ class Session:
                  n_min: int, n_max: int, kappa: int = 0, logit_tau: float = 0.0,
                  probe_kind: int = bd.PROBE_LINEAR, probe_hidden: int = 0, future=None,
                  harness: dict | None = None, split: int = 0, d: int | None = None,
-                 device="cuda", stream: torch.cuda.Stream | None = None):
+                 use_index: bool = False, device="cuda", stream: torch.cuda.Stream | None = None):
         self.lib = bd.load()
         self.device = torch.device(device)
         if self.device.type == "cuda" and self.device.index is None:
@@ -72,6 +72,13 @@ class Session:
         ws_bytes = int(self.lib.switchsd_workspace_bytes(ctypes.byref(probe)))
         self.workspace = torch.empty(max(ws_bytes, 256), dtype=torch.uint8, device=dev)
 
+        # incremental n-gram index (optional): built once from the initial contexts, then kept current
+        # by the verification calls
+        self.index = None
+        if use_index:
+            self.index = bd.NgramIndex(B, self.cap, n_min, n_max)
+            self.index.build(self.ctx, self.lens, stream=stream)
+
         # switchsd_step: two cached parameter blocks (with and without the debug outputs)
         def params(debug: bool):
             p = bd.switchsd_params()
@@ -79,6 +86,7 @@ class Session:
             p.n_min, p.n_max, p.kappa, p.logit_tau = n_min, n_max, kappa, logit_tau
             p.probe_kind, p.probe_hidden, p.b1, p.b2, p.split = probe_kind, probe_hidden, None, 0.0, split
             p.workspace, p.workspace_bytes = self.workspace.data_ptr(), self.workspace.numel()
+            p.index = self.index.handle if self.index is not None else None
             p.out_match_n = self.match_n.data_ptr() if debug else None
             p.out_match_end = self.match_end.data_ptr() if debug else None
             p.status = self.status.data_ptr() if debug else None
@@ -97,6 +105,7 @@ class Session:
             vp.ctx_tokens = self.ctx.data_ptr()
             vp.ctx_lens = self.lens.data_ptr()
             vp.status = self.vstatus.data_ptr() if debug else None
+            vp.index = self.index.handle if self.index is not None else None
             vp.stream = sp
             return vp
         self._vp_dbg, self._vp_fast = vparams(True), vparams(False)

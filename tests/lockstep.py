@@ -57,7 +57,7 @@ def oracle_trace(wl: synth.Workload, rows, steps: int, ctx=None, lens=None):
 
 
 def gpu_trace(wl: synth.Workload, steps: int, split: int = 0, ctx=None, lens=None, device="cuda",
-              fused: bool = False):
+              fused: bool = False, use_index: bool = False):
     """Runs the GPU loop on all rows; returns the per-step host copies of every output.
 
     fused=False: switchsd_step, target stand-in, switchsd_verify per iteration.
@@ -71,7 +71,7 @@ def gpu_trace(wl: synth.Workload, steps: int, split: int = 0, ctx=None, lens=Non
     sess = Session(ctx, lens, wl.probe_weights(), k=wl.k, n_min=wl.n_min, n_max=wl.n_max,
                    kappa=wl.kappa, logit_tau=wl.logit_tau, probe_kind=wl.probe_kind,
                    probe_hidden=wl.probe_hidden, future=wl.future(), harness=wl.harness_params(),
-                   split=split, d=wl.d, device=device)
+                   split=split, d=wl.d, use_index=use_index, device=device)
     trace = []
     for t in range(steps):
         hidden = bf16_tensor(wl.hidden(t), sess.device)

@@ -96,6 +96,36 @@ def test_full_size_sampled_rows(name):
         assert np.all(t["len"] <= wl.k)
 
 
+@pytest.mark.parametrize("fused", [False, True], ids=["separate", "fused"])
+@pytest.mark.parametrize("name", ["mixed_small", "zipf_small", "code_small", "zipf_kappa5"])
+def test_index_lockstep(name, fused):
+    """The incremental n-gram index against the oracle's rescan, in lockstep (build, inserts on every
+    verification, lookups), with the two-layer probe for the code workload."""
+    wl = SMALL[name]
+    rows = range(wl.B)
+    o_trace, o_ctx, _ = lockstep.oracle_trace(wl, rows, wl.steps)
+    g_trace, g_ctx, _ = lockstep.gpu_trace(wl, wl.steps, fused=fused, use_index=True)
+    flips, stats = lockstep.compare(wl, o_trace, g_trace, rows, o_ctx, g_ctx)
+    assert stats["checked"] > 0 and len(flips) <= 1
+
+
+@pytest.mark.parametrize("name", ["mixed_128k", "zipf_32k"])
+def test_index_equals_rescan_full_size(name):
+    """Every row at every step of the full workload: the index path and the rescan path (both on the
+    GPU, fused launches) produce identical matches, modes, drafts and contexts."""
+    wl = W[name]
+    a, a_ctx, _ = lockstep.gpu_trace(wl, wl.steps, fused=True)
+    b, b_ctx, _ = lockstep.gpu_trace(wl, wl.steps, fused=True, use_index=True)
+    for t, (x, y) in enumerate(zip(a, b)):
+        for key in ("match_n", "match_end", "mode", "len", "accept", "lens_after", "status"):
+            assert np.array_equal(x[key], y[key]), (name, t, key)
+        for r in range(wl.B):
+            n = int(x["len"][r])
+            assert np.array_equal(x["draft"][r, :n], y["draft"][r, :n]), (name, t, r)
+        assert np.allclose(x["score"], y["score"], atol=1e-3)
+    assert np.array_equal(a_ctx, b_ctx)
+
+
 def test_threshold_extremes():
     """tau -> 0 (logit -inf) copies on every kappa-match (prompt-lookup decoding); tau -> 1 never
     copies."""
