@@ -59,6 +59,8 @@ def parse_args(argv=None):
     ap.add_argument("--workload", default="zipf_32k", choices=sorted(synth.WORKLOADS))
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--split", type=int, default=0, help="CTAs per row (0 = library choice)")
+    ap.add_argument("--search", default="scan", choices=["scan", "index"],
+                    help="rescan the contexts every step, or keep the incremental n-gram index")
     ap.add_argument("--cpu-seconds", type=float, default=15.0,
                     help="budget of the CPU-baseline sample")
     ap.add_argument("--no-cpu-baseline", action="store_true")
@@ -244,8 +246,8 @@ def cpu_baseline(wl: synth.Workload, budget_s: float) -> dict:
                       f"verify timed, single thread; the host target stand-in is not timed)"}
 
 
-def config_of(wl: synth.Workload, world: int, split: int) -> dict:
-    return {"workload": wl.name, "B": wl.B, "L0": wl.L0, "V": wl.V, "d": wl.d, "k": wl.k,
+def config_of(wl: synth.Workload, world: int, split: int, search: str = "scan") -> dict:
+    return {"workload": wl.name, "search": search, "B": wl.B, "L0": wl.L0, "V": wl.V, "d": wl.d, "k": wl.k,
             "n_min": wl.n_min, "n_max": wl.n_max, "kappa": wl.kappa_eff, "tau": wl.tau,
             "probe": "linear" if wl.probe_kind == 0 else f"mlp{wl.d}x{wl.probe_hidden}",
             "global_batch": wl.B * world, "seq_len": wl.L0, "parallelism": f"replicas{world}",
@@ -270,7 +272,7 @@ def run_reference(args, world, rank):
             "ms_per_step": secs / steps * 1e3, "higher_is_better": True, "scaling": "weak",
             "vs_baseline": None, "dtype": "int32 (search/verify), f64 (probe)", "data": "synthetic",
             "impl": "reference",
-            "config": config_of(base, world, args.split),
+            "config": config_of(base, world, args.split, args.search),
             "cpu_baseline": {"value": value, "unit": UNIT, "cores": 1, "kind": "oracle",
                              "sample": f"{wl.name}: rows 0..{R - 1}, {args.warmup} untimed + "
                                        f"{steps} timed steps, single thread"},
@@ -295,7 +297,8 @@ class ReplicaLoop:
     """R independent batches of B rows stored as one [R*B, cap] state.  Launch i of a round runs
     switchsd_verify_step on batch i (its rows only); then one target stand-in covers all R*B rows."""
 
-    def __init__(self, wl, R, cap, ctx1, lens1, pw, future1, hidden, split, dev, stream):
+    def __init__(self, wl, R, cap, ctx1, lens1, pw, future1, hidden, split, dev, stream,
+                 search="scan"):
         import ctypes
         import torch
         from paper_2609_20186_gb300 import binding as bd, bf16_tensor
@@ -335,9 +338,19 @@ class ReplicaLoop:
         ws = max(256, int(self.lib.switchsd_workspace_bytes(ctypes.byref(probe))))
         self.workspace = torch.empty(R, ws, dtype=torch.uint8, device=dev)
         self.params = []
+        # one incremental n-gram index per batch (search = index), built from its initial contexts
+        self.indexes = []
         for r in range(R):
             q = bd.switchsd_params.from_buffer_copy(p)
             q.workspace, q.workspace_bytes = self.workspace[r].data_ptr(), ws
+            if search == "index":
+                idx = bd.NgramIndex(B, cap, wl.n_min, wl.n_max)
+                code = self.lib.switchsd_index_build(idx.handle, self.ctx.data_ptr() + r * B * cap * 4,
+                                                     self.lens.data_ptr() + r * B * 4, sp)
+                if code != 0:
+                    raise RuntimeError(f"index build failed: {code}")
+                self.indexes.append(idx)
+                q.index = idx.handle
             self.params.append(q)
         self.p = p
         hp = bd.switchsd_harness_params()
@@ -427,7 +440,8 @@ def run_ours(args, world, rank, local):
         hidden_host[i] = wl.hidden(i)
     hidden = bf16_tensor(hidden_host, dev)
     cs = torch.cuda.Stream(dev)
-    loop = ReplicaLoop(wl, R, cap, ctx1, lens1, pw, future1, hidden, args.split, dev, cs)
+    loop = ReplicaLoop(wl, R, cap, ctx1, lens1, pw, future1, hidden, args.split, dev, cs,
+                       search=args.search)
     ctx_bytes_all = R * B * cap * 4
 
     with torch.cuda.stream(cs):
@@ -492,6 +506,12 @@ def run_ours(args, world, rank, local):
         ctx_read = 4 * Lh[j + 1][:n_this].sum(axis=1)
         verify_rw = 8 * B + 16 * grow.sum(axis=1)          # lens r/w, draft + target read, append
         outputs = 12 * B + 4 * B * k                       # mode, len, score, draft (bound)
+        if args.search == "index":
+            # index path: per row the context tail, and per n one head read and one candidate
+            # compare (at least), plus one head and chain write per appended position
+            nn = wl.n_max - wl.n_min + 1
+            ctx_read = np.full(n_this, 4 * B * (32 + nn * (4 + 4 * wl.n_max)), np.int64) + \
+                12 * nn * grow.sum(axis=1)
         launch_bytes.extend((ctx_read + probe_bytes + verify_rw + outputs).tolist())
     launch_bytes = np.array(launch_bytes, dtype=np.float64)
     # Every fused launch appends at least one token per row: a timed region in which some row did not
@@ -519,11 +539,12 @@ def run_ours(args, world, rank, local):
         "ms_per_step": ms_per_step, "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "dtype": "int32 (search/verify), bf16 in / fp32 accumulate (probe)",
         "data": "synthetic",
-        "config": dict(config_of(base, world, args.split), replicas=R,
+        "config": dict(config_of(base, world, args.split, args.search), replicas=R,
                        l2=f"inputs larger than L2: {R} independent batches of B={B} "
                           f"({ctx_bytes_all / 2**20:.0f} MiB of contexts vs {l2 / 2**20:.0f} MiB L2), "
                           f"launch i reads batch i mod {R}"),
-        "roofline": {"kernel": "switchsd_verify_step", "bound": "hbm", "achieved": achieved,
+        "roofline": {"kernel": "switchsd_verify_step" + (" (index)" if args.search == "index" else ""),
+                     "bound": "hbm", "achieved": achieved,
                      "peak": peaks["hbm_gbs"], "unit": "GB/s", "frac": achieved / peaks["hbm_gbs"],
                      "traffic": traffic,
                      "algorithmic_bytes_per_launch": float(launch_bytes.mean()),
@@ -531,7 +552,8 @@ def run_ours(args, world, rank, local):
                      "duration": "timed region / K launches (the region also holds one target "
                                  "stand-in launch and one 4 KB length snapshot per round)",
                      "peak_source": peaks["source"] + " hbm_gbs (copy)"},
-        "controller": {"cold_single_launch_us": cold,
+        "controller": {"cold_single_launch_us": cold, "search": args.search,
+                       "scan_equivalent_gbs": float(4 * Lh[1:].sum(axis=2).mean() / per_launch_s / 1e9),
                        "mean_context_tokens": float(Lh[1:].mean()),
                        "launches_per_step": 1 if wl.probe_kind == 0 else 2},
         "gpu_launches": K * (1 if wl.probe_kind == 0 else 2) + rounds,

@@ -246,7 +246,9 @@ int switchsd_step_static_workspace(const int32_t *ctx_tokens, const int32_t *ctx
  *                           the allocation fails.  The index belongs to the current device.
  *   switchsd_index_build    (re)builds it from ctx_tokens / ctx_lens on `stream` (asynchronous); call
  *                           it once for the initial contexts and after any change made outside the
- *                           library's verification entry points.
+ *                           library's verification entry points.  Lowering ctx_lens and appending the
+ *                           same tokens again needs no rebuild (those insertions are no-ops); appending
+ *                           different tokens after lowering ctx_lens does.
  *   switchsd_index_bytes    device bytes the index holds.
  *   switchsd_index_destroy  frees it (NULL is a no-op); no call using it may still be in flight.
  */

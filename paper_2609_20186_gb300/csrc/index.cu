@@ -143,7 +143,10 @@ __global__ void __launch_bounds__(kIdxMaxWarps * kWarp) index_kernel(const Index
             const unsigned peers = __match_any_sync(kFull, bucket) & __ballot_sync(kFull, valid);
             const int32_t old_head = valid ? heads[bucket] : -1;
             __syncwarp();  // every lane has read its head before any lane replaces one
-            if (valid) {
+            // A head at or past p means these positions were inserted before (the same tokens appended
+            // again after the lengths were rewound): the chains already hold them, so leave them be.
+            // This keeps prev[p] < p, so every chain stays acyclic.
+            if (valid && old_head < p) {
                 const unsigned earlier = peers & ((1u << lane) - 1u);
                 prev[p] = earlier ? base + (31 - __clz(earlier)) : old_head;
                 if ((peers >> lane) == 1u) heads[bucket] = p;  // the latest position of the run

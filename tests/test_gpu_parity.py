@@ -109,6 +109,44 @@ def test_index_lockstep(name, fused):
     assert stats["checked"] > 0 and len(flips) <= 1
 
 
+def test_index_rewind_and_replay():
+    """Lowering ctx_lens and appending the same tokens again leaves the index consistent: the replayed
+    steps reproduce the first pass exactly (the insertions of known positions are no-ops)."""
+    import torch
+    from paper_2609_20186_gb300 import Session, bf16_tensor
+
+    wl = SMALL["mixed_small"].scaled(steps=10)
+    ctx, lens = wl.contexts()
+    sess = Session(ctx, lens, wl.probe_weights(), k=wl.k, n_min=wl.n_min, n_max=wl.n_max,
+                   logit_tau=wl.logit_tau, future=wl.future(), harness=wl.harness_params(), d=wl.d,
+                   use_index=True)
+    hid = [bf16_tensor(wl.hidden(t), sess.device) for t in range(wl.steps)]
+    sess.step(hid[0])
+    sess.harness(0)
+    for t in range(1, 4):
+        sess.verify_step(hid[t])
+        sess.harness(t)
+    state = [(x, x.clone()) for x in (sess.lens, sess.vdraft, sess.vlen, sess.target, sess.mode,
+                                      sess.draft, sess.len)]
+
+    def run():
+        outs = []
+        for t in range(4, wl.steps):
+            sess.verify_step(hid[t])
+            outs.append({n: getattr(sess, n).clone() for n in ("mode", "len", "draft", "match_n",
+                                                               "match_end", "accept", "lens")})
+            sess.harness(t)
+        return outs
+
+    first = run()
+    for dst, src in state:
+        dst.copy_(src)
+    second = run()
+    for a, b in zip(first, second):
+        for n in a:
+            assert torch.equal(a[n], b[n]), n
+
+
 @pytest.mark.parametrize("name", ["mixed_128k", "zipf_32k"])
 def test_index_equals_rescan_full_size(name):
     """Every row at every step of the full workload: the index path and the rescan path (both on the
