@@ -54,43 +54,61 @@ def build(force: bool = False) -> str:
     return _LIB_PATH
 
 
+def compile_library(src: str, out: str) -> str:
+    """Compiles an oracle source file (this one, or a copy under test) into a shared library."""
+    subprocess.run(["gcc", "-O2", "-std=c11", "-fPIC", "-shared", "-o", out, src], check=True)
+    return out
+
+
+def configure(lib):
+    """Declares the C signatures on a loaded oracle library; returns it."""
+    lib.oracle_longest_suffix_match.argtypes = [_i32p, ctypes.c_int32, ctypes.c_int32,
+                                                ctypes.c_int32, _i32p, _i32p]
+    lib.oracle_longest_suffix_match.restype = ctypes.c_int
+    lib.oracle_bf16_to_double.argtypes = [ctypes.c_uint16]
+    lib.oracle_bf16_to_double.restype = ctypes.c_double
+    lib.oracle_probe_linear.argtypes = [_u16p, _u16p, ctypes.c_int32]
+    lib.oracle_probe_linear.restype = ctypes.c_double
+    lib.oracle_probe_mlp.argtypes = [_u16p, _u16p, _f32p, _u16p, ctypes.c_float,
+                                     ctypes.c_int32, ctypes.c_int32]
+    lib.oracle_probe_mlp.restype = ctypes.c_double
+    lib.oracle_switch.argtypes = [ctypes.c_int32, ctypes.c_int32, ctypes.c_int32,
+                                  ctypes.c_double, ctypes.c_float, ctypes.c_int32,
+                                  ctypes.c_int32, _i32p, ctypes.c_int32, _i32p, _i32p]
+    lib.oracle_switch.restype = ctypes.c_int32
+    lib.oracle_verify_row.argtypes = [_i32p, _i32p, ctypes.c_int32, _i32p, ctypes.c_int32,
+                                      _i32p, _i32p]
+    lib.oracle_verify_row.restype = ctypes.c_int32
+    lib.oracle_step_rows.argtypes = [
+        _i32p, _i32p, ctypes.c_int32, ctypes.c_int32, ctypes.c_int32,  # ctx lens b0 b1 cap
+        _u16p, ctypes.c_int32, _u16p, ctypes.c_int32,                   # hidden d probe_w kind
+        ctypes.c_int32, _f32p, ctypes.c_float,                          # H1 b1 b2
+        ctypes.c_int32, ctypes.c_int32, ctypes.c_int32, ctypes.c_int32,  # k n_min n_max kappa
+        ctypes.c_float,                                                 # logit_tau
+        _i32p, _i32p, _i32p, _f64p, _i32p, _i32p]
+    lib.oracle_step_rows.restype = None
+    lib.oracle_verify_rows.argtypes = [_i32p, _i32p, ctypes.c_int32, ctypes.c_int32,
+                                       ctypes.c_int32, ctypes.c_int32, _i32p, _i32p, _i32p,
+                                       _i32p, _i32p]
+    lib.oracle_verify_rows.restype = None
+    return lib
+
+
 def _load():
     global _lib
     with _lock:
-        if _lib is not None:
-            return _lib
-        lib = ctypes.CDLL(build())
-        lib.oracle_longest_suffix_match.argtypes = [_i32p, ctypes.c_int32, ctypes.c_int32,
-                                                    ctypes.c_int32, _i32p, _i32p]
-        lib.oracle_longest_suffix_match.restype = ctypes.c_int
-        lib.oracle_bf16_to_double.argtypes = [ctypes.c_uint16]
-        lib.oracle_bf16_to_double.restype = ctypes.c_double
-        lib.oracle_probe_linear.argtypes = [_u16p, _u16p, ctypes.c_int32]
-        lib.oracle_probe_linear.restype = ctypes.c_double
-        lib.oracle_probe_mlp.argtypes = [_u16p, _u16p, _f32p, _u16p, ctypes.c_float,
-                                         ctypes.c_int32, ctypes.c_int32]
-        lib.oracle_probe_mlp.restype = ctypes.c_double
-        lib.oracle_switch.argtypes = [ctypes.c_int32, ctypes.c_int32, ctypes.c_int32,
-                                      ctypes.c_double, ctypes.c_float, ctypes.c_int32,
-                                      ctypes.c_int32, _i32p, ctypes.c_int32, _i32p, _i32p]
-        lib.oracle_switch.restype = ctypes.c_int32
-        lib.oracle_verify_row.argtypes = [_i32p, _i32p, ctypes.c_int32, _i32p, ctypes.c_int32,
-                                          _i32p, _i32p]
-        lib.oracle_verify_row.restype = ctypes.c_int32
-        lib.oracle_step_rows.argtypes = [
-            _i32p, _i32p, ctypes.c_int32, ctypes.c_int32, ctypes.c_int32,  # ctx lens b0 b1 cap
-            _u16p, ctypes.c_int32, _u16p, ctypes.c_int32,                   # hidden d probe_w kind
-            ctypes.c_int32, _f32p, ctypes.c_float,                          # H1 b1 b2
-            ctypes.c_int32, ctypes.c_int32, ctypes.c_int32, ctypes.c_int32,  # k n_min n_max kappa
-            ctypes.c_float,                                                 # logit_tau
-            _i32p, _i32p, _i32p, _f64p, _i32p, _i32p]
-        lib.oracle_step_rows.restype = None
-        lib.oracle_verify_rows.argtypes = [_i32p, _i32p, ctypes.c_int32, ctypes.c_int32,
-                                           ctypes.c_int32, ctypes.c_int32, _i32p, _i32p, _i32p,
-                                           _i32p, _i32p]
-        lib.oracle_verify_rows.restype = None
-        _lib = lib
-        return lib
+        if _lib is None:
+            _lib = configure(ctypes.CDLL(build()))
+        return _lib
+
+
+def use_library(lib):
+    """Routes this module's functions to `lib` (a configured oracle library); returns the previous
+    one.  Used by the tests that plant mistakes in a copy of the oracle."""
+    global _lib
+    with _lock:
+        old, _lib = _lib, lib
+        return old
 
 
 def _ptr(a: np.ndarray, ctype):
