@@ -101,9 +101,10 @@ struct alignas(16) Slot {
 __global__ void __launch_bounds__(kStepThreads) step_kernel(const StepArgs a) {
     extern __shared__ __align__(128) int32_t tiles[];  // stages x (kHalo + tile + kFwd)
     __shared__ __align__(8) uint64_t bars[kMaxStages];
+    __shared__ __align__(8) uint64_t tail_bar;                 // the old tail's small copy
     __shared__ __align__(8) uint64_t s_done;                   // leader: completes when every slot landed
     __shared__ int32_t s_suf[SWITCHSD_NMAX];
-    __shared__ int32_t s_old[kHalo];                           // the kHalo tokens before the old end
+    __shared__ __align__(16) int32_t s_tail[kHalo + 8];        // x[tail_lo .. L_old), tail_lo = roundown4(L_old - kHalo)
     __shared__ int32_t s_app[SWITCHSD_KMAX + 1];               // tokens appended by the verification
     __shared__ int32_t s_ver[3];                               // accepted, new length, verify status
     __shared__ unsigned long long s_wkey[kStepWarps];
@@ -123,6 +124,7 @@ __global__ void __launch_bounds__(kStepThreads) step_kernel(const StepArgs a) {
 
     if (tid == 0) {
         for (int s = 0; s < a.stages; ++s) mbar_init(&bars[s], 1);
+        mbar_init(&tail_bar, 1);
         if (rank == 0) {
             mbar_init(&s_done, 1);
             mbar_arrive_expect_tx(&s_done, slot_bytes * C);
@@ -132,35 +134,13 @@ __global__ void __launch_bounds__(kStepThreads) step_kernel(const StepArgs a) {
     pdl_wait();     // everything below may read what the preceding kernel wrote
     pdl_trigger();  // the next kernel may start launching
 
-    // Loads whose addresses do not depend on the row length go out first, in one round trip.
-    // Lane i of warp 1 holds draft[i], draft[i+32], target[i], target[i+32] and (lane 0) target[64].
-    int32_t pv_n = 0, d_lo = 0, d_hi = 0, t_lo = 0, t_hi = 0, t_top = 0;
-    if (verifying && warp == 1) {
-        const int32_t *dr = a.pv_draft + size_t(b) * a.k;
-        const int32_t *tg = a.pv_target + size_t(b) * (a.k + 1);
-        pv_n = a.pv_len[b];
-        if (lane < a.k) d_lo = dr[lane];
-        if (lane + 32 < a.k) d_hi = dr[lane + 32];
-        if (lane <= a.k) t_lo = tg[lane];
-        if (lane + 32 <= a.k) t_hi = tg[lane + 32];
-        if (lane == 0 && a.k >= 64) t_top = tg[64];
-    }
-    float zp = 0.f;
-    if (a.z_pre == nullptr) {
-        // the linear probe partial over this CTA's 1/C slice
-        const int nv = a.d >> 3;
-        const int per = (nv + int(C) - 1) / int(C);
-        const int v0 = int(rank) * per, v1 = min(nv, v0 + per);
-        const uint4 *h4 = reinterpret_cast<const uint4 *>(a.hidden + size_t(b) * size_t(a.d));
-        const uint4 *w4 = reinterpret_cast<const uint4 *>(a.probe_w);
-        for (int v = v0 + tid; v < v1; v += kStepThreads) zp = dot8_bf16(__ldg(w4 + v), __ldg(h4 + v), zp);
-    }
-
+    // Warp roles until the suffix is known.  Warp 0 reads the row length and issues the copies at
+    // once: first the old tail (for the suffix), then the tiles.  Warp 1 verifies the previous draft.
+    // Warps 2.. load this CTA's slice of the probe operands into registers and use them only after the
+    // scan, so no wait on them delays it.  Every thread arrives on the cluster barrier (release) after
+    // reading ctx_lens[b]: once the leader has waited on it, it may publish the new length.
     int32_t *row = a.ctx + size_t(b) * size_t(a.cap);
     const int32_t L_old = a.lens[b];
-    // Cluster barrier arrival, released after the row length is read: once a CTA has waited on it,
-    // every CTA of the cluster is running, has initialised its barriers and has read ctx_lens[b].
-    cluster_arrive_release();
     const bool len_ok = (L_old >= 1 && L_old <= a.cap);
     // Split on the old length; the last CTA also covers every end the append can add.
     const int32_t E_split = len_ok ? L_old - 1 : 0;
@@ -170,6 +150,8 @@ __global__ void __launch_bounds__(kStepThreads) step_kernel(const StepArgs a) {
     const int32_t e_lo = min(E_split, int32_t(rank) * chunk);
     const int32_t e_hi = rank + 1 == C ? E_max : min(E_split, e_lo + chunk);
     const int32_t ntiles = (e_hi - e_lo + a.tile - 1) / a.tile;
+    const int32_t tail_lo = max(0, (L_old - kHalo) & ~3);
+    const int32_t tail_hi = len_ok ? (L_old + 3) & ~3 : tail_lo;  // <= cap since cap % 4 == 0
 
     // Stage tile t: tokens [max(0, t0 - kHalo), min(roundup4(t1 + kFwd), cap)) land so that token p
     // sits at stage[kHalo + p - t0].  cap % 4 == 0 keeps every bound 16-byte aligned.
@@ -183,12 +165,30 @@ __global__ void __launch_bounds__(kStepThreads) step_kernel(const StepArgs a) {
         mbar_arrive_expect_tx(&bars[s], bytes);
         bulk_g2s(tiles + s * stage_ints + (kHalo + lo - t0), row + lo, bytes, &bars[s]);
     };
-    if (tid == 0) {
-        for (int t = 0; t < min(ntiles, a.stages); ++t) issue(t);
+    uint4 pw[2], ph[2];  // probe operands (warps 2..), consumed after the scan
+    int npv = 0;
+    int v_rest = 0, v_end = 0;  // probe words past the two held in registers, loaded after the scan
+    if (warp == 0) {
+        if (lane == 0) {
+            const uint32_t tb = uint32_t(tail_hi - tail_lo) * 4u;
+            mbar_arrive_expect_tx(&tail_bar, tb);
+            if (tb > 0) bulk_g2s(s_tail, row + tail_lo, tb, &tail_bar);
+            for (int t = 0; t < min(ntiles, a.stages); ++t) issue(t);
+        }
+        cluster_arrive_release();
     } else if (warp == 1) {
-        // Verification of the previous draft (every CTA of the row computes the same result).
+        // Verification of the previous draft (every CTA of the row computes the same result).  Lane i
+        // reads draft[i], draft[i+32], target[i], target[i+32] and (lane 0) target[64].
         int32_t acc = -1, L = L_old, vst = len_ok ? SWITCHSD_ROW_OK : SWITCHSD_ROW_BAD_LEN;
         if (verifying && len_ok) {
+            const int32_t *dr = a.pv_draft + size_t(b) * a.k;
+            const int32_t *tg = a.pv_target + size_t(b) * (a.k + 1);
+            const int32_t pv_n = a.pv_len[b];
+            const int32_t d_lo = lane < a.k ? dr[lane] : 0;
+            const int32_t d_hi = lane + 32 < a.k ? dr[lane + 32] : 0;
+            const int32_t t_lo = lane <= a.k ? tg[lane] : 0;
+            const int32_t t_hi = lane + 32 <= a.k ? tg[lane + 32] : 0;
+            const int32_t t_top = (lane == 0 && a.k >= 64) ? tg[64] : 0;
             if (pv_n < 0 || pv_n > a.k) {
                 vst = SWITCHSD_ROW_BAD_LEN;
             } else {
@@ -214,34 +214,43 @@ __global__ void __launch_bounds__(kStepThreads) step_kernel(const StepArgs a) {
             s_ver[1] = L;
             s_ver[2] = vst;
         }
-    } else if (warp == 2) {
-        const int32_t p = L_old - kHalo + lane;
-        if (lane < kHalo) s_old[lane] = (len_ok && p >= 0) ? row[p] : 0;
-    }
-    zp = warp_sum_f32(zp);
-    if (lane == 0) s_wz[warp] = zp;
-    __syncthreads();  // verification, old tail and probe partials are visible
-
-    // Every CTA has started and read ctx_lens[b] once this returns; it waits while the copies fly.
-    cluster_wait_acquire();
-    const int32_t acc = s_ver[0], L = s_ver[1];
-    const int32_t E = len_ok ? L - 1 : 0;  // candidate ends after the append: [0, E)
-    if (rank == 0 && verifying) {
-        // The leader publishes the append; the other CTAs only patch their staged copies.
-        for (int i = tid; i <= acc; i += kStepThreads) row[L_old + i] = s_app[i];
-        if (tid == 0 && len_ok) {
-            a.lens[b] = L;
-            a.out_accept[b] = acc;
+        cluster_arrive_release();
+    } else {
+        cluster_arrive_release();
+        if (a.z_pre == nullptr) {
+            const int nv = a.d >> 3;
+            const int per = (nv + int(C) - 1) / int(C);
+            const int v0 = int(rank) * per, v1 = min(nv, v0 + per);
+            const uint4 *h4 = reinterpret_cast<const uint4 *>(a.hidden + size_t(b) * size_t(a.d));
+            const uint4 *w4 = reinterpret_cast<const uint4 *>(a.probe_w);
+            int v = v0 + tid - 2 * kWarp;
+            for (; v < v1 && npv < 2; v += kStepThreads - 2 * kWarp, ++npv) {
+                pw[npv] = __ldg(w4 + v);
+                ph[npv] = __ldg(h4 + v);
+            }
+            v_rest = v;
+            v_end = v1;
         }
     }
-    if (tid < SWITCHSD_NMAX) {
-        const int32_t p = L - 1 - tid;  // suffix position; p >= L_old - kHalo since L >= L_old
-        s_suf[tid] = p < 0 ? 0 : (p >= L_old ? s_app[p - L_old] : s_old[p - (L_old - kHalo)]);
+    // Warps 0 and 1 meet (named barrier 1, 64 threads): the suffix needs the old tail and the append.
+    if (warp < 2) {
+        asm volatile("bar.sync 1, 64;\n" ::: "memory");
+        if (warp == 0) {
+            const bool tail_in = tail_hi == tail_lo || mbar_wait(&tail_bar, 0);
+            const int32_t L = s_ver[1];
+            const int32_t p = L - 1 - lane;  // suffix position; p >= L_old - kHalo since L >= L_old
+            int32_t v = 0;
+            if (p >= L_old)
+                v = s_app[p - L_old];
+            else if (len_ok && p >= 0 && tail_in)
+                v = s_tail[p - tail_lo];
+            s_suf[lane] = v;
+        }
     }
-    float cta_z = 0.f;
-    if (warp == 0) cta_z = warp_sum_f32(lane < kStepWarps ? s_wz[lane] : 0.f);
-    __syncthreads();
+    __syncthreads();  // suffix and verification visible
 
+    const int32_t acc = s_ver[0], L = s_ver[1];
+    const int32_t E = len_ok ? L - 1 : 0;  // candidate ends after the append: [0, E)
     const int32_t s0 = s_suf[0];
     const int32_t n_max = a.n_max, n_min = a.n_min;
     unsigned long long best = 0;  // CTA-uniform; real keys have m >= n_min >= 1, so 0 = no match
@@ -328,6 +337,31 @@ __global__ void __launch_bounds__(kStepThreads) step_kernel(const StepArgs a) {
         // Give the copies still in flight a second bounded wait before the CTA's memory goes away.
         if (tid == 0)
             for (int u = 0; u < min(ntiles, a.stages); ++u) (void)mbar_wait(&bars[u], 0u);
+    }
+
+    // The probe slice (operands loaded long ago), then the CTA's partial in a fixed order.
+    float zp = 0.f;
+    for (int i = 0; i < npv; ++i) zp = dot8_bf16(pw[i], ph[i], zp);
+    if (v_rest < v_end) {
+        const uint4 *h4 = reinterpret_cast<const uint4 *>(a.hidden + size_t(b) * size_t(a.d));
+        const uint4 *w4 = reinterpret_cast<const uint4 *>(a.probe_w);
+        for (int v = v_rest; v < v_end; v += kStepThreads - 2 * kWarp) zp = dot8_bf16(__ldg(w4 + v), __ldg(h4 + v), zp);
+    }
+    zp = warp_sum_f32(zp);
+    if (lane == 0) s_wz[warp] = zp;
+    __syncthreads();
+    float cta_z = 0.f;
+    if (warp == 0) cta_z = warp_sum_f32(lane < kStepWarps ? s_wz[lane] : 0.f);
+
+    // Every CTA has started and read ctx_lens[b] once this returns (they all arrived long ago).
+    cluster_wait_acquire();
+    if (rank == 0 && verifying) {
+        // The leader publishes the append; the other CTAs only patched their staged copies.
+        for (int i = tid; i <= acc; i += kStepThreads) row[L_old + i] = s_app[i];
+        if (tid == 0 && len_ok) {
+            a.lens[b] = L;
+            a.out_accept[b] = acc;
+        }
     }
 
     // Ship this CTA's message to the leader: asynchronous DSMEM stores that complete on its barrier.
