@@ -65,6 +65,8 @@ def parse_args(argv=None):
                     help="budget of the CPU-baseline sample")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-prefetch", action="store_true",
+                    help="read the context only after the preceding kernel is done (params.prefetch = 0)")
     return ap.parse_args(argv)
 
 
@@ -246,8 +248,9 @@ def cpu_baseline(wl: synth.Workload, budget_s: float) -> dict:
                       f"verify timed, single thread; the host target stand-in is not timed)"}
 
 
-def config_of(wl: synth.Workload, world: int, split: int, search: str = "scan") -> dict:
-    return {"workload": wl.name, "search": search, "B": wl.B, "L0": wl.L0, "V": wl.V, "d": wl.d, "k": wl.k,
+def config_of(wl: synth.Workload, world: int, split: int, search: str = "scan",
+              prefetch: bool = True) -> dict:
+    return {"workload": wl.name, "search": search, "prefetch": bool(prefetch and search == "scan"), "B": wl.B, "L0": wl.L0, "V": wl.V, "d": wl.d, "k": wl.k,
             "n_min": wl.n_min, "n_max": wl.n_max, "kappa": wl.kappa_eff, "tau": wl.tau,
             "probe": "linear" if wl.probe_kind == 0 else f"mlp{wl.d}x{wl.probe_hidden}",
             "global_batch": wl.B * world, "seq_len": wl.L0, "parallelism": f"replicas{world}",
@@ -272,7 +275,7 @@ def run_reference(args, world, rank):
             "ms_per_step": secs / steps * 1e3, "higher_is_better": True, "scaling": "weak",
             "vs_baseline": None, "dtype": "int32 (search/verify), f64 (probe)", "data": "synthetic",
             "impl": "reference",
-            "config": config_of(base, world, args.split, args.search),
+            "config": config_of(base, world, args.split, args.search, not args.no_prefetch),
             "cpu_baseline": {"value": value, "unit": UNIT, "cores": 1, "kind": "oracle",
                              "sample": f"{wl.name}: rows 0..{R - 1}, {args.warmup} untimed + "
                                        f"{steps} timed steps, single thread"},
@@ -298,7 +301,7 @@ class ReplicaLoop:
     switchsd_verify_step on batch i (its rows only); then one target stand-in covers all R*B rows."""
 
     def __init__(self, wl, R, cap, ctx1, lens1, pw, future1, hidden, split, dev, stream,
-                 search="scan"):
+                 search="scan", prefetch=True):
         import ctypes
         import torch
         from paper_2609_20186_gb300 import binding as bd, bf16_tensor
@@ -332,6 +335,9 @@ class ReplicaLoop:
         p.probe_kind, p.probe_hidden, p.b1, p.b2, p.split = wl.probe_kind, wl.probe_hidden, None, 0.0, split
         p.out_match_n = p.out_match_end = p.status = None
         p.stream = sp
+        # The kernel before each launch is another batch's launch, the target stand-in or a copy:
+        # none writes this batch's rows, so the context copies may start before it finishes.
+        p.prefetch = int(prefetch)
         # one workspace per batch, so consecutive launches never share one
         probe = bd.switchsd_params()
         probe.B, probe.probe_kind, probe.probe_hidden = B, wl.probe_kind, wl.probe_hidden
@@ -441,7 +447,7 @@ def run_ours(args, world, rank, local):
     hidden = bf16_tensor(hidden_host, dev)
     cs = torch.cuda.Stream(dev)
     loop = ReplicaLoop(wl, R, cap, ctx1, lens1, pw, future1, hidden, args.split, dev, cs,
-                       search=args.search)
+                       search=args.search, prefetch=not args.no_prefetch)
     ctx_bytes_all = R * B * cap * 4
 
     with torch.cuda.stream(cs):
@@ -530,7 +536,7 @@ def run_ours(args, world, rank, local):
 
     e2e = None
     if not args.no_e2e:
-        e2e = run_e2e(base, dev, W, K, args.split, world)
+        e2e = run_e2e(base, dev, W, K, args.split, world, prefetch=not args.no_prefetch)
 
     if rank != 0:
         return
@@ -539,7 +545,7 @@ def run_ours(args, world, rank, local):
         "ms_per_step": ms_per_step, "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "dtype": "int32 (search/verify), bf16 in / fp32 accumulate (probe)",
         "data": "synthetic",
-        "config": dict(config_of(base, world, args.split, args.search), replicas=R,
+        "config": dict(config_of(base, world, args.split, args.search, not args.no_prefetch), replicas=R,
                        l2=f"inputs larger than L2: {R} independent batches of B={B} "
                           f"({ctx_bytes_all / 2**20:.0f} MiB of contexts vs {l2 / 2**20:.0f} MiB L2), "
                           f"launch i reads batch i mod {R}"),
@@ -602,7 +608,7 @@ def cold_latency(loop, dev, cs, step_base, l2) -> dict:
             "note": "includes the ~2.2 us event-pair and ~2.2 us stream launch overhead of this GPU"}
 
 
-def run_e2e(base, dev, W, K, split, world):
+def run_e2e(base, dev, W, K, split, world, prefetch=True):
     """The same loop through the public API with host buffers, one batch: per step, H2D of the
     hidden states from pinned memory, switchsd_verify_step + target stand-in, D2H of mode / draft
     length / draft / accepted length, host sync."""
@@ -615,7 +621,7 @@ def run_e2e(base, dev, W, K, split, world):
     sess = Session(ctx, lens, wl.probe_weights(), k=k, n_min=wl.n_min, n_max=wl.n_max,
                    kappa=wl.kappa, logit_tau=wl.logit_tau, probe_kind=wl.probe_kind,
                    probe_hidden=wl.probe_hidden, future=wl.future(), harness=wl.harness_params(),
-                   split=split, d=d, device=dev)
+                   split=split, d=d, device=dev, prefetch=prefetch)  # an H2D copy precedes each call
     host_h = torch.empty(W + K, B, d, dtype=torch.int16).pin_memory()
     for t in range(W + K):
         host_h[t].copy_(torch.from_numpy(wl.hidden(t).view(np.int16)))

@@ -41,7 +41,7 @@
 extern "C" {
 #endif
 
-#define SWITCHSD_ABI_VERSION 1
+#define SWITCHSD_ABI_VERSION 2
 
 #define SWITCHSD_NMAX 32 /* largest supported n_max */
 #define SWITCHSD_KMAX 64 /* largest supported draft length k */
@@ -98,6 +98,18 @@ typedef struct switchsd_index switchsd_index;
  *                position e* of its most recent earlier occurrence (0 / -1 when none); may be NULL
  *   status       optional device int32[B] per-row status (SWITCHSD_ROW_*); may be NULL
  *   stream       cudaStream_t as void*
+ *   prefetch     0: the call reads nothing before the kernel that precedes it on the stream is done.
+ *                1: the rescan may read ctx_lens and ctx_tokens[b][0, ctx_lens[b]) before that preceding
+ *                kernel finishes (programmatic dependent launch), so the context copies overlap its tail.
+ *                The caller promises that (a) the kernel immediately before this call on the stream
+ *                writes neither these tokens nor these lengths, and (b) if that kernel was itself
+ *                launched with programmatic stream serialization, it waits for its own predecessors
+ *                (griddepcontrol.wait) before it lets dependents start -- every kernel of this library
+ *                does, and a kernel launched without that attribute always does.  The previous
+ *                writer of the rows is then complete when the copies start.  A copy or memset just
+ *                before the call is always safe.  The previous draft, target, hidden state, probe
+ *                weights and workspace are still read after the wait.  The index search ignores it.
+ *                Any other value is SWITCHSD_ERR_ARG.
  */
 typedef struct {
     int32_t B, cap, d, k, n_min, n_max, kappa;
@@ -114,6 +126,7 @@ typedef struct {
     int32_t *out_match_end;
     int32_t *status;
     void *stream;
+    int32_t prefetch;
 } switchsd_params;
 
 /*

@@ -19,6 +19,7 @@ PROBE_LINEAR, PROBE_MLP = 0, 1
 OK, ERR_ARG, ERR_SHAPE, ERR_CUDA = 0, -1, -2, -3
 ROW_OK, ROW_CAPACITY, ROW_BAD_LEN, ROW_TIMEOUT = 0, 1, 2, 3
 NMAX, KMAX = 32, 64
+ABI_VERSION = 2  # SWITCHSD_ABI_VERSION this binding marshals for
 
 _c_i32p = ctypes.c_void_p
 
@@ -36,6 +37,7 @@ class switchsd_params(ctypes.Structure):
         ("out_match_n", ctypes.c_void_p), ("out_match_end", ctypes.c_void_p),
         ("status", ctypes.c_void_p),
         ("stream", ctypes.c_void_p),
+        ("prefetch", ctypes.c_int32),
     ]
 
 
@@ -102,6 +104,8 @@ def load(path: str | None = None):
             fn = getattr(lib, name)
             fn.restype = res
             fn.argtypes = args
+        if lib.switchsd_abi_version() != ABI_VERSION:
+            raise RuntimeError(f"{p} has ABI {lib.switchsd_abi_version()}, the binding wants {ABI_VERSION}: rebuild it")
         _lib = lib
         return lib
 
@@ -146,7 +150,7 @@ def switchsd_step(ctx_tokens, ctx_lens, hidden, probe_w, out_draft, out_len, out
                   k: int, n_min: int, n_max: int, kappa: int = 0, logit_tau: float = 0.0,
                   probe_kind: int = PROBE_LINEAR, probe_hidden: int = 0, b1=None, b2: float = 0.0,
                   split: int = 0, out_match_n=None, out_match_end=None, status=None,
-                  workspace=None, stream=None) -> None:
+                  workspace=None, stream=None, prefetch: bool = False) -> None:
     """switchsd_step of include/switchsd.h on torch tensors (see the header for semantics).
 
     ctx_tokens int32 [B, cap]; ctx_lens int32 [B]; hidden bf16 [B, d]; probe_w bf16 (w[d] or
@@ -166,6 +170,7 @@ def switchsd_step(ctx_tokens, ctx_lens, hidden, probe_w, out_draft, out_len, out
     p.out_match_end = _dev(out_match_end, torch.int32, "out_match_end", (B,))
     p.status = _dev(status, torch.int32, "status", (B,))
     p.stream = _stream_ptr(stream)
+    p.prefetch = int(prefetch)
     nw = d if probe_kind == PROBE_LINEAR else probe_hidden * d + probe_hidden
     ws = _attach_workspace(p, workspace, ctx_tokens.device)  # noqa: F841 (kept alive for the call)
     code = load().switchsd_step(
@@ -237,7 +242,7 @@ def switchsd_verify_step(draft, target_argmax, draft_len, out_accept, ctx_tokens
                          n_max: int, kappa: int = 0, logit_tau: float = 0.0,
                          probe_kind: int = PROBE_LINEAR, probe_hidden: int = 0, b1=None,
                          b2: float = 0.0, split: int = 0, out_match_n=None, out_match_end=None,
-                         status=None, workspace=None, stream=None) -> None:
+                         status=None, workspace=None, stream=None, prefetch: bool = False) -> None:
     """switchsd_verify_step of include/switchsd.h: verification of the previous draft, then the next
     step, in one launch."""
     B, cap = ctx_tokens.shape
@@ -254,6 +259,7 @@ def switchsd_verify_step(draft, target_argmax, draft_len, out_accept, ctx_tokens
     p.out_match_end = _dev(out_match_end, torch.int32, "out_match_end", (B,))
     p.status = _dev(status, torch.int32, "status", (B,))
     p.stream = _stream_ptr(stream)
+    p.prefetch = int(prefetch)
     nw = d if probe_kind == PROBE_LINEAR else probe_hidden * d + probe_hidden
     ws = _attach_workspace(p, workspace, ctx_tokens.device)  # noqa: F841 (kept alive for the call)
     code = load().switchsd_verify_step(

@@ -50,6 +50,7 @@ constexpr int kMaxStages = 6;          // staged tiles in flight per CTA (bounde
 constexpr size_t kStageSmemBudget = 200 * 1024;
 constexpr int kMaxSplit = 16;
 constexpr unsigned long long kTimeoutBit = 1ull << 62;
+constexpr int kProbeStage = 256;      // probe words (8 bf16) of w and of h staged per CTA; the rest is read directly
 
 static_assert(kHalo >= SWITCHSD_NMAX && kHalo % 4 == 0, "halo must cover the longest n-gram");
 static_assert(kFwd % 4 == 0 && kTileMax % 4 == 0, "stages must stay 16-byte aligned");
@@ -67,6 +68,7 @@ struct StepArgs {
     const int32_t *pv_len;
     int32_t *out_accept;
     int32_t B, cap, d, k, n_min, n_max, kappa, tile, stages;
+    int32_t prefetch;        // 1: the length read and the context copies may precede the grid-dependency wait
     float logit_tau;
     int32_t *out_draft, *out_len, *out_mode;
     float *out_score;
@@ -102,6 +104,7 @@ __global__ void __launch_bounds__(kStepThreads) step_kernel(const StepArgs a) {
     extern __shared__ __align__(128) int32_t tiles[];  // stages x (kHalo + tile + kFwd)
     __shared__ __align__(8) uint64_t bars[kMaxStages];
     __shared__ __align__(8) uint64_t tail_bar;                 // the old tail's small copy
+    __shared__ __align__(8) uint64_t probe_bar;                // this CTA's slices of w and h
     __shared__ __align__(8) uint64_t s_done;                   // leader: completes when every slot landed
     __shared__ int32_t s_suf[SWITCHSD_NMAX];
     __shared__ __align__(16) int32_t s_tail[kHalo + 8];        // x[tail_lo .. L_old), tail_lo = roundown4(L_old - kHalo)
@@ -110,6 +113,7 @@ __global__ void __launch_bounds__(kStepThreads) step_kernel(const StepArgs a) {
     __shared__ unsigned long long s_wkey[kStepWarps];
     __shared__ float s_wz[kStepWarps];
     __shared__ __align__(16) int32_t s_mine[SWITCHSD_KMAX];    // continuation of this CTA's best match
+    __shared__ __align__(16) uint4 s_pw[kProbeStage], s_ph[kProbeStage];
     __shared__ Slot s_slot[kMaxSplit];                         // leader: one message per CTA
     __shared__ int32_t s_out[2];                               // leader: winner rank, draft length
 
@@ -125,14 +129,19 @@ __global__ void __launch_bounds__(kStepThreads) step_kernel(const StepArgs a) {
     if (tid == 0) {
         for (int s = 0; s < a.stages; ++s) mbar_init(&bars[s], 1);
         mbar_init(&tail_bar, 1);
+        mbar_init(&probe_bar, 1);
         if (rank == 0) {
             mbar_init(&s_done, 1);
             mbar_arrive_expect_tx(&s_done, slot_bytes * C);
         }
         fence_mbar_init();
     }
-    pdl_wait();     // everything below may read what the preceding kernel wrote
-    pdl_trigger();  // the next kernel may start launching
+    // Without prefetch every read below waits for the preceding kernel.  With it, the row length and
+    // the context copies go first: the caller guarantees that the kernel immediately before this one
+    // does not write them, and the kernels before that one are complete once it runs (each waits on
+    // its own predecessors before it lets this one start).  The L2-coherent load keeps a stale L1 line
+    // from an earlier grid out of the length.
+    if (!a.prefetch) pdl_wait();
 
     // Warp roles until the suffix is known.  Warp 0 reads the row length and issues the copies at
     // once: first the old tail (for the suffix), then the tiles.  Warp 1 verifies the previous draft.
@@ -140,7 +149,7 @@ __global__ void __launch_bounds__(kStepThreads) step_kernel(const StepArgs a) {
     // scan, so no wait on them delays it.  Every thread arrives on the cluster barrier (release) after
     // reading ctx_lens[b]: once the leader has waited on it, it may publish the new length.
     int32_t *row = a.ctx + size_t(b) * size_t(a.cap);
-    const int32_t L_old = a.lens[b];
+    const int32_t L_old = __ldcg(a.lens + b);
     const bool len_ok = (L_old >= 1 && L_old <= a.cap);
     // Split on the old length; the last CTA also covers every end the append can add.
     const int32_t E_split = len_ok ? L_old - 1 : 0;
@@ -163,18 +172,31 @@ __global__ void __launch_bounds__(kStepThreads) step_kernel(const StepArgs a) {
         const int32_t hi = min((t1 + kFwd + 3) & ~3, a.cap);
         const uint32_t bytes = uint32_t(hi - lo) * 4u;
         mbar_arrive_expect_tx(&bars[s], bytes);
-        bulk_g2s(tiles + s * stage_ints + (kHalo + lo - t0), row + lo, bytes, &bars[s]);
+        bulk_g2s_hint(tiles + s * stage_ints + (kHalo + lo - t0), row + lo, bytes, &bars[s], l2_evict_first_policy());
     };
-    uint4 pw[2], ph[2];  // probe operands (warps 2..), consumed after the scan
-    int npv = 0;
-    int v_rest = 0, v_end = 0;  // probe words past the two held in registers, loaded after the scan
+    // This CTA's slice of the linear probe: words [v0, v1) of 8 bf16.  The first kProbeStage of them
+    // are staged by two bulk copies issued after the wait and used after the scan.
+    int v0 = 0, v1 = 0;
+    if (a.z_pre == nullptr) {
+        const int nv = a.d >> 3;
+        const int per = (nv + int(C) - 1) / int(C);
+        v0 = min(nv, int(rank) * per);
+        v1 = min(nv, v0 + per);
+    }
+    const int v_staged = min(v1 - v0, kProbeStage);
+    const uint4 *h4 = reinterpret_cast<const uint4 *>(a.hidden + size_t(b) * size_t(a.d));
+    const uint4 *w4 = reinterpret_cast<const uint4 *>(a.probe_w);
     if (warp == 0) {
         if (lane == 0) {
             const uint32_t tb = uint32_t(tail_hi - tail_lo) * 4u;
             mbar_arrive_expect_tx(&tail_bar, tb);
-            if (tb > 0) bulk_g2s(s_tail, row + tail_lo, tb, &tail_bar);
+            if (tb > 0) bulk_g2s_hint(s_tail, row + tail_lo, tb, &tail_bar, l2_evict_first_policy());
             for (int t = 0; t < min(ntiles, a.stages); ++t) issue(t);
         }
+    }
+    if (a.prefetch) pdl_wait();  // the previous draft, target, hidden state and probe come after this
+    pdl_trigger();               // the next kernel may start launching
+    if (warp == 0) {
         cluster_arrive_release();
     } else if (warp == 1) {
         // Verification of the previous draft (every CTA of the row computes the same result).  Lane i
@@ -216,21 +238,15 @@ __global__ void __launch_bounds__(kStepThreads) step_kernel(const StepArgs a) {
         }
         cluster_arrive_release();
     } else {
-        cluster_arrive_release();
-        if (a.z_pre == nullptr) {
-            const int nv = a.d >> 3;
-            const int per = (nv + int(C) - 1) / int(C);
-            const int v0 = int(rank) * per, v1 = min(nv, v0 + per);
-            const uint4 *h4 = reinterpret_cast<const uint4 *>(a.hidden + size_t(b) * size_t(a.d));
-            const uint4 *w4 = reinterpret_cast<const uint4 *>(a.probe_w);
-            int v = v0 + tid - 2 * kWarp;
-            for (; v < v1 && npv < 2; v += kStepThreads - 2 * kWarp, ++npv) {
-                pw[npv] = __ldg(w4 + v);
-                ph[npv] = __ldg(h4 + v);
+        if (warp == 2 && lane == 0) {
+            const uint32_t pb = uint32_t(v_staged) * 16u;
+            mbar_arrive_expect_tx(&probe_bar, 2u * pb);
+            if (pb > 0) {
+                bulk_g2s(s_pw, w4 + v0, pb, &probe_bar);
+                bulk_g2s(s_ph, h4 + v0, pb, &probe_bar);
             }
-            v_rest = v;
-            v_end = v1;
         }
+        cluster_arrive_release();
     }
     // Warps 0 and 1 meet (named barrier 1, 64 threads): the suffix needs the old tail and the append.
     if (warp < 2) {
@@ -251,8 +267,12 @@ __global__ void __launch_bounds__(kStepThreads) step_kernel(const StepArgs a) {
 
     const int32_t acc = s_ver[0], L = s_ver[1];
     const int32_t E = len_ok ? L - 1 : 0;  // candidate ends after the append: [0, E)
-    const int32_t s0 = s_suf[0];
+    const int32_t s0 = s_suf[0], s1 = s_suf[1];
     const int32_t n_max = a.n_max, n_min = a.n_min;
+    // With n_min >= 2 a candidate must match the last two tokens, so the filter tests both (exact:
+    // the back-compare then starts at m = 2).  m0 is the length the filter has already checked.
+    const bool pair = n_min >= 2;
+    const int32_t m0 = pair ? 2 : 1;
     unsigned long long best = 0;  // CTA-uniform; real keys have m >= n_min >= 1, so 0 = no match
     bool bad = false;             // CTA-uniform: a copy did not land in time
     for (int t = 0; t < ntiles && !bad; ++t) {
@@ -276,7 +296,9 @@ __global__ void __launch_bounds__(kStepThreads) step_kernel(const StepArgs a) {
         if (landed) {
             const int32_t n4 = (t1 - t0 + 3) >> 2;
             const int4 *g4 = reinterpret_cast<const int4 *>(stage + kHalo);
-            for (int32_t g0 = tid; g0 < n4; g0 += 4 * kStepThreads) {
+            // The bound is warp-uniform (g0 - lane is the warp's first word) so the shuffle below always
+            // has the whole warp; lanes past the end read zeros and their ends fail e < t1.
+            for (int32_t g0 = tid; g0 - lane < n4; g0 += 4 * kStepThreads) {
                 int4 v[4];
 #pragma unroll
                 for (int u = 0; u < 4; ++u) {
@@ -285,15 +307,25 @@ __global__ void __launch_bounds__(kStepThreads) step_kernel(const StepArgs a) {
                 }
 #pragma unroll
                 for (int u = 0; u < 4; ++u) {
-                    const int32_t e4 = t0 + 4 * (g0 + u * kStepThreads);
+                    const int32_t g = g0 + u * kStepThreads;
+                    const int32_t e4 = t0 + 4 * g;
                     unsigned hits = unsigned(v[u].x == s0) | (unsigned(v[u].y == s0) << 1) |
                                     (unsigned(v[u].z == s0) << 2) | (unsigned(v[u].w == s0) << 3);
+                    if (pair) {
+                        // x[e4 - 1] is the last token of the previous word (lane - 1, or staged memory
+                        // for lane 0; at e4 = 0 that slot is unset, but e = 0 cannot hold a 2-gram).
+                        int32_t prev = __shfl_up_sync(kFull, v[u].w, 1);
+                        if (lane == 0) prev = g < n4 ? stage[kHalo + 4 * g - 1] : 0;
+                        hits &= unsigned(prev == s1) | (unsigned(v[u].x == s1) << 1) |
+                                (unsigned(v[u].y == s1) << 2) | (unsigned(v[u].z == s1) << 3);
+                    }
                     while (hits) {
                         const int32_t e = e4 + __ffs(hits) - 1;
                         hits &= hits - 1;
                         if (e >= t1) break;
                         const int32_t lim = min(n_max, e + 1);
-                        int32_t m = 1;
+                        if (lim < m0) continue;
+                        int32_t m = m0;
                         while (m < lim && stage[off + e - m] == s_suf[m]) ++m;
                         if (m >= n_min) {
                             const unsigned long long key =
@@ -339,13 +371,15 @@ __global__ void __launch_bounds__(kStepThreads) step_kernel(const StepArgs a) {
             for (int u = 0; u < min(ntiles, a.stages); ++u) (void)mbar_wait(&bars[u], 0u);
     }
 
-    // The probe slice (operands loaded long ago), then the CTA's partial in a fixed order.
+    // The probe slice (staged during the scan), then the CTA's partial in a fixed order.
     float zp = 0.f;
-    for (int i = 0; i < npv; ++i) zp = dot8_bf16(pw[i], ph[i], zp);
-    if (v_rest < v_end) {
-        const uint4 *h4 = reinterpret_cast<const uint4 *>(a.hidden + size_t(b) * size_t(a.d));
-        const uint4 *w4 = reinterpret_cast<const uint4 *>(a.probe_w);
-        for (int v = v_rest; v < v_end; v += kStepThreads - 2 * kWarp) zp = dot8_bf16(__ldg(w4 + v), __ldg(h4 + v), zp);
+    const bool probe_in = mbar_wait(&probe_bar, 0);
+    if (probe_in)
+        for (int i = tid; i < v_staged; i += kStepThreads) zp = dot8_bf16(s_pw[i], s_ph[i], zp);
+    for (int v = v0 + v_staged + tid; v < v1; v += kStepThreads) zp = dot8_bf16(__ldg(w4 + v), __ldg(h4 + v), zp);
+    if (!probe_in && tid == 0) {
+        best = kTimeoutBit;
+        (void)mbar_wait(&probe_bar, 0);  // a second bounded wait before the CTA's memory goes away
     }
     zp = warp_sum_f32(zp);
     if (lane == 0) s_wz[warp] = zp;
@@ -481,6 +515,7 @@ static int step_entry(int32_t *ctx_tokens, int32_t *ctx_lens, const uint16_t *hi
     if (p->n_min < 1 || p->n_max > SWITCHSD_NMAX || p->n_min > p->n_max) return SWITCHSD_ERR_SHAPE;
     if (p->split != 0 && p->split != 1 && p->split != 2 && p->split != 4 && p->split != 8 && p->split != 16)
         return SWITCHSD_ERR_SHAPE;
+    if (p->prefetch != 0 && p->prefetch != 1) return SWITCHSD_ERR_ARG;
     if (p->probe_kind == SWITCHSD_PROBE_MLP) {
         if (!mlp_shape_ok(p->d, p->probe_hidden)) return SWITCHSD_ERR_SHAPE;
         if (!p->workspace || !aligned16(p->workspace) ||
@@ -514,6 +549,7 @@ static int step_entry(int32_t *ctx_tokens, int32_t *ctx_lens, const uint16_t *hi
     args.out_match_n = p->out_match_n;
     args.out_match_end = p->out_match_end;
     args.status = p->status;
+    args.prefetch = p->prefetch;
 
     const int split = p->split > 0 ? p->split : choose_split(p->B, p->cap);
     // Tile: the largest CTA range (the last CTA may also cover a k + 1 token append), in one stage

@@ -33,7 +33,8 @@ class Session:
                  n_min: int, n_max: int, kappa: int = 0, logit_tau: float = 0.0,
                  probe_kind: int = bd.PROBE_LINEAR, probe_hidden: int = 0, future=None,
                  harness: dict | None = None, split: int = 0, d: int | None = None,
-                 use_index: bool = False, device="cuda", stream: torch.cuda.Stream | None = None):
+                 use_index: bool = False, device="cuda", stream: torch.cuda.Stream | None = None,
+                 prefetch: bool = False):
         self.lib = bd.load()
         self.device = torch.device(device)
         if self.device.type == "cuda" and self.device.index is None:
@@ -91,6 +92,7 @@ class Session:
             p.out_match_end = self.match_end.data_ptr() if debug else None
             p.status = self.status.data_ptr() if debug else None
             p.stream = sp
+            p.prefetch = int(prefetch)
             return p
         self._p_dbg, self._p_fast = params(True), params(False)
         self._step_head = (self.ctx.data_ptr(), self.lens.data_ptr())

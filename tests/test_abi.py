@@ -50,7 +50,7 @@ def test_every_declared_symbol_is_exported(lib):
 
 def test_abi_version_and_strerror(lib):
     from paper_2609_20186_gb300 import binding as bd
-    assert bd.abi_version() == 1
+    assert bd.abi_version() == 2
     for code in (0, -1, -2, -3, 1, 2, 3):
         assert bd.strerror(code) != "unknown code"
     assert bd.strerror(12345) == "unknown code"
@@ -90,6 +90,8 @@ def test_step_validation(lib):
     assert _step(lib, _params(n_min=5, n_max=4)) == bd.ERR_SHAPE
     assert _step(lib, _params(n_max=33)) == bd.ERR_SHAPE
     assert _step(lib, _params(split=3)) == bd.ERR_SHAPE
+    assert _step(lib, _params(prefetch=2)) == bd.ERR_ARG
+    assert _step(lib, _params(prefetch=-1)) == bd.ERR_ARG
     assert _step(lib, _params(probe_kind=1, probe_hidden=0)) == bd.ERR_SHAPE
     # the two-layer probe needs its workspace
     assert _step(lib, _params(probe_kind=1, probe_hidden=256)) == bd.ERR_ARG

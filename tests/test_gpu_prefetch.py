@@ -1,0 +1,63 @@
+"""params.prefetch: the context copies start before the preceding kernel finishes.
+
+The serving order is verify_step(t) -> target -> verify_step(t+1), launched back to back with no host
+synchronisation, so each call's context copies overlap the target stand-in's kernel while the rows
+were written by the call before it.  With and without prefetch the whole run must give identical
+outputs (the same kernels in the same order, so bit-identical, the probe logits included) and
+identical contexts; the no-prefetch path is itself held to the oracle by test_gpu_parity.py.
+"""
+import numpy as np
+import pytest
+
+import synth
+
+pytestmark = pytest.mark.gpu
+
+W = synth.WORKLOADS
+KEYS = ("draft", "len", "mode", "score", "match_n", "match_end", "status", "accept")
+
+
+def _chain(wl, prefetch: bool, steps: int, record_every: int):
+    import torch
+    from paper_2609_20186_gb300 import Session, bf16_tensor
+
+    ctx, lens = wl.contexts()
+    sess = Session(ctx, lens, wl.probe_weights(), k=wl.k, n_min=wl.n_min, n_max=wl.n_max,
+                   kappa=wl.kappa, logit_tau=wl.logit_tau, probe_kind=wl.probe_kind,
+                   probe_hidden=wl.probe_hidden, future=wl.future(), harness=wl.harness_params(),
+                   d=wl.d, prefetch=prefetch)
+    hidden = bf16_tensor(np.stack([wl.hidden(t) for t in range(steps)]), sess.device)
+    torch.cuda.synchronize()
+    rec = {}
+    for t in range(steps):
+        if t == 0:
+            sess.step(hidden[0])
+        else:
+            sess.verify_step(hidden[t])
+        if t % record_every == 0:  # recorded on the device; the other steps chain kernel to kernel
+            rec[t] = {key: getattr(sess, key).clone() for key in KEYS}
+        sess.harness(t)
+    sess.verify()
+    torch.cuda.synchronize()
+    out = {t: {key: v.cpu().numpy() for key, v in r.items()} for t, r in rec.items()}
+    return out, sess.ctx.cpu().numpy(), sess.lens.cpu().numpy()
+
+
+@pytest.mark.parametrize("name,steps", [("zipf_32k", 40), ("code_16k", 24), ("mixed_128k", 24),
+                                        ("uniform_8k", 40)])
+def test_prefetch_matches_back_to_back(name, steps):
+    wl = W[name].scaled(steps=steps)
+    a, a_ctx, a_lens = _chain(wl, False, steps, record_every=3)
+    b, b_ctx, b_lens = _chain(wl, True, steps, record_every=3)
+    assert np.array_equal(a_lens, b_lens)
+    assert (a_lens > wl.L0).all()  # every row grew: the chain really appended
+    assert np.array_equal(a_ctx, b_ctx)
+    for t in a:
+        for key in KEYS:
+            if key == "draft":
+                for r in range(wl.B):
+                    n = int(a[t]["len"][r])
+                    assert np.array_equal(a[t]["draft"][r, :n], b[t]["draft"][r, :n]), (t, r)
+            else:
+                assert np.array_equal(a[t][key], b[t][key]), (name, t, key)
+
