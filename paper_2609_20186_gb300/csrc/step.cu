@@ -136,6 +136,7 @@ __global__ void __launch_bounds__(kStepThreads) step_kernel(const StepArgs a) {
         }
         fence_mbar_init();
     }
+    __syncthreads();  // the barriers are initialised before any other thread arms or waits on one
     // Without prefetch every read below waits for the preceding kernel.  With it, the row length and
     // the context copies go first: the caller guarantees that the kernel immediately before this one
     // does not write them, and the kernels before that one are complete once it runs (each waits on
