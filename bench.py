@@ -66,7 +66,7 @@ def parse_args(argv=None):
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-prefetch", action="store_true",
-                    help="read the context only after the preceding kernel is done (params.prefetch = 0)")
+                    help="read nothing before the preceding kernel is done (params.prefetch = 0)")
     return ap.parse_args(argv)
 
 
@@ -336,8 +336,9 @@ class ReplicaLoop:
         p.out_match_n = p.out_match_end = p.status = None
         p.stream = sp
         # The kernel before each launch is another batch's launch, the target stand-in or a copy:
-        # none writes this batch's rows, so the context copies may start before it finishes.
-        p.prefetch = int(prefetch)
+        # none writes this batch's rows or hidden states (generated once, never written), so their
+        # copies may start before it finishes.
+        p.prefetch = (bd.PREFETCH_CONTEXT | bd.PREFETCH_PROBE) if prefetch else 0
         # one workspace per batch, so consecutive launches never share one
         probe = bd.switchsd_params()
         probe.B, probe.probe_kind, probe.probe_hidden = B, wl.probe_kind, wl.probe_hidden
@@ -613,7 +614,7 @@ def run_e2e(base, dev, W, K, split, world, prefetch=True):
     hidden states from pinned memory, switchsd_verify_step + target stand-in, D2H of mode / draft
     length / draft / accepted length, host sync."""
     import torch
-    from paper_2609_20186_gb300 import Session
+    from paper_2609_20186_gb300 import Session, binding
 
     wl = base.scaled(steps=W + K)
     B, d, k = wl.B, wl.d, wl.k
@@ -621,7 +622,8 @@ def run_e2e(base, dev, W, K, split, world, prefetch=True):
     sess = Session(ctx, lens, wl.probe_weights(), k=k, n_min=wl.n_min, n_max=wl.n_max,
                    kappa=wl.kappa, logit_tau=wl.logit_tau, probe_kind=wl.probe_kind,
                    probe_hidden=wl.probe_hidden, future=wl.future(), harness=wl.harness_params(),
-                   split=split, d=d, device=dev, prefetch=prefetch)  # an H2D copy precedes each call
+                   split=split, d=d, device=dev,  # an H2D copy precedes each call
+                   prefetch=(binding.PREFETCH_CONTEXT | binding.PREFETCH_PROBE) if prefetch else 0)
     host_h = torch.empty(W + K, B, d, dtype=torch.int16).pin_memory()
     for t in range(W + K):
         host_h[t].copy_(torch.from_numpy(wl.hidden(t).view(np.int16)))

@@ -67,6 +67,10 @@ extern "C" {
 #define SWITCHSD_ROW_BAD_LEN 2  /* ctx_lens[b] outside [1, cap] or draft_len[b] outside [0, k] */
 #define SWITCHSD_ROW_TIMEOUT 3  /* an on-chip copy did not complete within its wait limit */
 
+/* switchsd_params.prefetch bits. */
+#define SWITCHSD_PREFETCH_CONTEXT 1
+#define SWITCHSD_PREFETCH_PROBE 2
+
 /* Incremental n-gram index (switchsd_index_create); opaque. */
 typedef struct switchsd_index switchsd_index;
 
@@ -98,18 +102,22 @@ typedef struct switchsd_index switchsd_index;
  *                position e* of its most recent earlier occurrence (0 / -1 when none); may be NULL
  *   status       optional device int32[B] per-row status (SWITCHSD_ROW_*); may be NULL
  *   stream       cudaStream_t as void*
- *   prefetch     0: the call reads nothing before the kernel that precedes it on the stream is done.
- *                1: the rescan may read ctx_lens and ctx_tokens[b][0, ctx_lens[b]) before that preceding
- *                kernel finishes (programmatic dependent launch), so the context copies overlap its tail.
- *                The caller promises that (a) the kernel immediately before this call on the stream
- *                writes neither these tokens nor these lengths, and (b) if that kernel was itself
+ *   prefetch     0, or a set of SWITCHSD_PREFETCH_* bits naming inputs that the rescan may start to read
+ *                before the kernel that precedes the call on the stream has finished (programmatic
+ *                dependent launch), so that their copies overlap that kernel's tail:
+ *                  SWITCHSD_PREFETCH_CONTEXT  ctx_lens and ctx_tokens[b][0, ctx_lens[b])
+ *                  SWITCHSD_PREFETCH_PROBE    hidden and the linear probe's weights
+ *                For every bit set the caller promises that (a) the kernel immediately before this
+ *                call on the stream does not write those inputs, and (b) if that kernel was itself
  *                launched with programmatic stream serialization, it waits for its own predecessors
  *                (griddepcontrol.wait) before it lets dependents start -- every kernel of this library
- *                does, and a kernel launched without that attribute always does.  The previous
- *                writer of the rows is then complete when the copies start.  A copy or memset just
- *                before the call is always safe.  The previous draft, target, hidden state, probe
- *                weights and workspace are still read after the wait.  The index search ignores it.
- *                Any other value is SWITCHSD_ERR_ARG.
+ *                does, and a kernel launched without that attribute always does.  The earlier writer
+ *                of those inputs is then complete when the copies start.  A copy or memset just before
+ *                the call is always safe.  In a serving loop the target's last kernel (its argmax)
+ *                writes neither the context nor the hidden state.  The previous draft, its length
+ *                and the target argmax are always read after the wait.  The index search ignores the
+ *                field and the two-layer probe ignores SWITCHSD_PREFETCH_PROBE.  Other bits are
+ *                SWITCHSD_ERR_ARG.
  */
 typedef struct {
     int32_t B, cap, d, k, n_min, n_max, kappa;

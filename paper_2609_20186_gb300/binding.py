@@ -20,6 +20,7 @@ OK, ERR_ARG, ERR_SHAPE, ERR_CUDA = 0, -1, -2, -3
 ROW_OK, ROW_CAPACITY, ROW_BAD_LEN, ROW_TIMEOUT = 0, 1, 2, 3
 NMAX, KMAX = 32, 64
 ABI_VERSION = 2  # SWITCHSD_ABI_VERSION this binding marshals for
+PREFETCH_CONTEXT, PREFETCH_PROBE = 1, 2  # switchsd_params.prefetch bits
 
 _c_i32p = ctypes.c_void_p
 
@@ -150,7 +151,7 @@ def switchsd_step(ctx_tokens, ctx_lens, hidden, probe_w, out_draft, out_len, out
                   k: int, n_min: int, n_max: int, kappa: int = 0, logit_tau: float = 0.0,
                   probe_kind: int = PROBE_LINEAR, probe_hidden: int = 0, b1=None, b2: float = 0.0,
                   split: int = 0, out_match_n=None, out_match_end=None, status=None,
-                  workspace=None, stream=None, prefetch: bool = False) -> None:
+                  workspace=None, stream=None, prefetch: int = 0) -> None:
     """switchsd_step of include/switchsd.h on torch tensors (see the header for semantics).
 
     ctx_tokens int32 [B, cap]; ctx_lens int32 [B]; hidden bf16 [B, d]; probe_w bf16 (w[d] or
@@ -170,7 +171,7 @@ def switchsd_step(ctx_tokens, ctx_lens, hidden, probe_w, out_draft, out_len, out
     p.out_match_end = _dev(out_match_end, torch.int32, "out_match_end", (B,))
     p.status = _dev(status, torch.int32, "status", (B,))
     p.stream = _stream_ptr(stream)
-    p.prefetch = int(prefetch)
+    p.prefetch = int(prefetch)  # PREFETCH_* bits (see the header for the caller's guarantee)
     nw = d if probe_kind == PROBE_LINEAR else probe_hidden * d + probe_hidden
     ws = _attach_workspace(p, workspace, ctx_tokens.device)  # noqa: F841 (kept alive for the call)
     code = load().switchsd_step(
@@ -242,7 +243,7 @@ def switchsd_verify_step(draft, target_argmax, draft_len, out_accept, ctx_tokens
                          n_max: int, kappa: int = 0, logit_tau: float = 0.0,
                          probe_kind: int = PROBE_LINEAR, probe_hidden: int = 0, b1=None,
                          b2: float = 0.0, split: int = 0, out_match_n=None, out_match_end=None,
-                         status=None, workspace=None, stream=None, prefetch: bool = False) -> None:
+                         status=None, workspace=None, stream=None, prefetch: int = 0) -> None:
     """switchsd_verify_step of include/switchsd.h: verification of the previous draft, then the next
     step, in one launch."""
     B, cap = ctx_tokens.shape
@@ -259,7 +260,7 @@ def switchsd_verify_step(draft, target_argmax, draft_len, out_accept, ctx_tokens
     p.out_match_end = _dev(out_match_end, torch.int32, "out_match_end", (B,))
     p.status = _dev(status, torch.int32, "status", (B,))
     p.stream = _stream_ptr(stream)
-    p.prefetch = int(prefetch)
+    p.prefetch = int(prefetch)  # PREFETCH_* bits (see the header for the caller's guarantee)
     nw = d if probe_kind == PROBE_LINEAR else probe_hidden * d + probe_hidden
     ws = _attach_workspace(p, workspace, ctx_tokens.device)  # noqa: F841 (kept alive for the call)
     code = load().switchsd_verify_step(

@@ -68,7 +68,7 @@ struct StepArgs {
     const int32_t *pv_len;
     int32_t *out_accept;
     int32_t B, cap, d, k, n_min, n_max, kappa, tile, stages;
-    int32_t prefetch;        // 1: the length read and the context copies may precede the grid-dependency wait
+    int32_t prefetch;        // SWITCHSD_PREFETCH_* bits: reads that may precede the grid-dependency wait
     float logit_tau;
     int32_t *out_draft, *out_len, *out_mode;
     float *out_score;
@@ -137,12 +137,35 @@ __global__ void __launch_bounds__(kStepThreads) step_kernel(const StepArgs a) {
         fence_mbar_init();
     }
     __syncthreads();  // the barriers are initialised before any other thread arms or waits on one
-    // Without prefetch every read below waits for the preceding kernel.  With it, the row length and
-    // the context copies go first: the caller guarantees that the kernel immediately before this one
-    // does not write them, and the kernels before that one are complete once it runs (each waits on
-    // its own predecessors before it lets this one start).  The L2-coherent load keeps a stale L1 line
-    // from an earlier grid out of the length.
-    if (!a.prefetch) pdl_wait();
+    // Reads named by a prefetch bit go before the grid-dependency wait: the caller guarantees that
+    // the kernel immediately before this one does not write them, and the kernels before that one are
+    // complete once it runs (each waits on its own predecessors before it lets this one start).  The
+    // L2-coherent load keeps a stale L1 line from an earlier grid out of the length.
+    const bool pf_ctx = (a.prefetch & SWITCHSD_PREFETCH_CONTEXT) != 0;
+    const bool pf_probe = (a.prefetch & SWITCHSD_PREFETCH_PROBE) != 0;
+
+    // This CTA's slice of the linear probe: words [v0, v1) of 8 bf16.  The first kProbeStage of them
+    // are staged by two bulk copies (issued by thread 64) and used after the scan.
+    int v0 = 0, v1 = 0;
+    if (a.z_pre == nullptr) {
+        const int nv = a.d >> 3;
+        const int per = (nv + int(C) - 1) / int(C);
+        v0 = min(nv, int(rank) * per);
+        v1 = min(nv, v0 + per);
+    }
+    const int v_staged = min(v1 - v0, kProbeStage);
+    const uint4 *h4 = reinterpret_cast<const uint4 *>(a.hidden + size_t(b) * size_t(a.d));
+    const uint4 *w4 = reinterpret_cast<const uint4 *>(a.probe_w);
+    auto issue_probe = [&]() {
+        const uint32_t pb = uint32_t(v_staged) * 16u;
+        mbar_arrive_expect_tx(&probe_bar, 2u * pb);
+        if (pb > 0) {
+            bulk_g2s(s_pw, w4 + v0, pb, &probe_bar);
+            bulk_g2s(s_ph, h4 + v0, pb, &probe_bar);
+        }
+    };
+    if (pf_probe && tid == 2 * kWarp) issue_probe();
+    if (!pf_ctx) pdl_wait();
 
     // Warp roles until the suffix is known.  Warp 0 reads the row length and issues the copies at
     // once: first the old tail (for the suffix), then the tiles.  Warp 1 verifies the previous draft.
@@ -175,18 +198,6 @@ __global__ void __launch_bounds__(kStepThreads) step_kernel(const StepArgs a) {
         mbar_arrive_expect_tx(&bars[s], bytes);
         bulk_g2s_hint(tiles + s * stage_ints + (kHalo + lo - t0), row + lo, bytes, &bars[s], l2_evict_first_policy());
     };
-    // This CTA's slice of the linear probe: words [v0, v1) of 8 bf16.  The first kProbeStage of them
-    // are staged by two bulk copies issued after the wait and used after the scan.
-    int v0 = 0, v1 = 0;
-    if (a.z_pre == nullptr) {
-        const int nv = a.d >> 3;
-        const int per = (nv + int(C) - 1) / int(C);
-        v0 = min(nv, int(rank) * per);
-        v1 = min(nv, v0 + per);
-    }
-    const int v_staged = min(v1 - v0, kProbeStage);
-    const uint4 *h4 = reinterpret_cast<const uint4 *>(a.hidden + size_t(b) * size_t(a.d));
-    const uint4 *w4 = reinterpret_cast<const uint4 *>(a.probe_w);
     if (warp == 0) {
         if (lane == 0) {
             const uint32_t tb = uint32_t(tail_hi - tail_lo) * 4u;
@@ -195,8 +206,8 @@ __global__ void __launch_bounds__(kStepThreads) step_kernel(const StepArgs a) {
             for (int t = 0; t < min(ntiles, a.stages); ++t) issue(t);
         }
     }
-    if (a.prefetch) pdl_wait();  // the previous draft, target, hidden state and probe come after this
-    pdl_trigger();               // the next kernel may start launching
+    if (pf_ctx) pdl_wait();  // the previous draft and the target (and all that no bit names) come after this
+    pdl_trigger();           // the next kernel may start launching
     if (warp == 0) {
         cluster_arrive_release();
     } else if (warp == 1) {
@@ -239,14 +250,7 @@ __global__ void __launch_bounds__(kStepThreads) step_kernel(const StepArgs a) {
         }
         cluster_arrive_release();
     } else {
-        if (warp == 2 && lane == 0) {
-            const uint32_t pb = uint32_t(v_staged) * 16u;
-            mbar_arrive_expect_tx(&probe_bar, 2u * pb);
-            if (pb > 0) {
-                bulk_g2s(s_pw, w4 + v0, pb, &probe_bar);
-                bulk_g2s(s_ph, h4 + v0, pb, &probe_bar);
-            }
-        }
+        if (!pf_probe && tid == 2 * kWarp) issue_probe();
         cluster_arrive_release();
     }
     // Warps 0 and 1 meet (named barrier 1, 64 threads): the suffix needs the old tail and the append.
@@ -297,8 +301,8 @@ __global__ void __launch_bounds__(kStepThreads) step_kernel(const StepArgs a) {
         if (landed) {
             const int32_t n4 = (t1 - t0 + 3) >> 2;
             const int4 *g4 = reinterpret_cast<const int4 *>(stage + kHalo);
-            // The bound is warp-uniform (g0 - lane is the warp's first word) so the shuffle below always
-            // has the whole warp; lanes past the end read zeros and their ends fail e < t1.
+            // The bound is warp-uniform (g0 - lane is the warp's first word); lanes past the end read
+            // zeros and their ends fail e < t1.
             for (int32_t g0 = tid; g0 - lane < n4; g0 += 4 * kStepThreads) {
                 int4 v[4];
 #pragma unroll
@@ -312,13 +316,13 @@ __global__ void __launch_bounds__(kStepThreads) step_kernel(const StepArgs a) {
                     const int32_t e4 = t0 + 4 * g;
                     unsigned hits = unsigned(v[u].x == s0) | (unsigned(v[u].y == s0) << 1) |
                                     (unsigned(v[u].z == s0) << 2) | (unsigned(v[u].w == s0) << 3);
-                    if (pair) {
-                        // x[e4 - 1] is the last token of the previous word (lane - 1, or staged memory
-                        // for lane 0; at e4 = 0 that slot is unset, but e = 0 cannot hold a 2-gram).
-                        int32_t prev = __shfl_up_sync(kFull, v[u].w, 1);
-                        if (lane == 0) prev = g < n4 ? stage[kHalo + 4 * g - 1] : 0;
-                        hits &= unsigned(prev == s1) | (unsigned(v[u].x == s1) << 1) |
-                                (unsigned(v[u].y == s1) << 2) | (unsigned(v[u].z == s1) << 3);
+                    if (pair && hits != 0u) {
+                        // x[e - 1] sits in this word for three of the four ends; for the first it is
+                        // the staged token before the word (unset at e4 = 0, where no 2-gram ends).
+                        unsigned pm = (unsigned(v[u].x == s1) << 1) | (unsigned(v[u].y == s1) << 2) |
+                                      (unsigned(v[u].z == s1) << 3);
+                        if ((hits & 1u) != 0u && g < n4) pm |= unsigned(stage[kHalo + 4 * g - 1] == s1);
+                        hits &= pm;
                     }
                     while (hits) {
                         const int32_t e = e4 + __ffs(hits) - 1;
@@ -414,23 +418,23 @@ __global__ void __launch_bounds__(kStepThreads) step_kernel(const StepArgs a) {
     }
     if (rank != 0) return;
 
-    if (tid == 0) {
-        // Bounded wait for every CTA's message (C x slot_bytes of transaction).
-        const bool all_in = mbar_wait(&s_done, 0);
-        unsigned long long key = all_in ? 0ull : kTimeoutBit;
-        uint32_t win = 0;
-        float z = 0.f;
-        for (uint32_t r = 0; r < C && all_in; ++r) {
-            if (s_slot[r].key > key) {
-                key = s_slot[r].key;
-                win = r;
-            }
-            z += s_slot[r].z;
+    if (warp == 0) {
+        // Bounded wait for every CTA's message (C x slot_bytes of transaction); lane r reads CTA r's.
+        // The largest key wins (CTAs tie only at 0, no match: their ends differ), and the probe
+        // partials are summed by a fixed shuffle tree, so the result is the same on every run.
+        const bool all_in = __all_sync(kFull, mbar_wait(&s_done, 0));
+        unsigned long long k_r = 0ull;
+        float z_r = 0.f;
+        if (all_in && uint32_t(lane) < C) {
+            k_r = s_slot[lane].key;
+            z_r = s_slot[lane].z;
         }
-        if (a.z_pre != nullptr) {
-            z = a.b2;
-            for (int n = 0; n < a.z_tiles; ++n) z += a.z_pre[size_t(n) * a.B + b];
-        }
+        if (a.z_pre != nullptr) z_r = lane < a.z_tiles ? a.z_pre[size_t(lane) * a.B + b] : 0.f;
+        const unsigned long long key = all_in ? warp_max_u64(k_r) : kTimeoutBit;
+        const unsigned at = __ballot_sync(kFull, uint32_t(lane) < C && k_r == key);
+        const uint32_t win = at != 0u ? uint32_t(__ffs(at) - 1) : 0u;
+        float z = warp_sum_f32(z_r);
+        if (a.z_pre != nullptr) z += a.b2;
         const bool timeout = (key & kTimeoutBit) != 0;
         const bool hit = len_ok && !timeout && key != 0;
         const int32_t n = hit ? int32_t(key >> 32) : 0;
@@ -439,18 +443,20 @@ __global__ void __launch_bounds__(kStepThreads) step_kernel(const StepArgs a) {
         int32_t mode = SWITCHSD_MODE_NO_REP;
         if (hit) mode = (n >= kappa && z >= a.logit_tau) ? SWITCHSD_MODE_COPY : SWITCHSD_MODE_REP_NO_COPY;
         const int32_t len = mode == SWITCHSD_MODE_COPY ? min(a.k, L - 1 - e) : 0;
-        s_out[0] = int32_t(win);
-        s_out[1] = len;
-        a.out_mode[b] = mode;
-        a.out_len[b] = len;
-        a.out_score[b] = z;
-        if (a.out_match_n) a.out_match_n[b] = n;
-        if (a.out_match_end) a.out_match_end[b] = e;
-        if (verifying && !len_ok) a.out_accept[b] = -1;
-        if (a.status) {
-            int32_t st = s_ver[2];
-            if (st == SWITCHSD_ROW_OK && timeout) st = SWITCHSD_ROW_TIMEOUT;
-            a.status[b] = st;
+        if (lane == 0) {
+            s_out[0] = int32_t(win);
+            s_out[1] = len;
+            a.out_mode[b] = mode;
+            a.out_len[b] = len;
+            a.out_score[b] = z;
+            if (a.out_match_n) a.out_match_n[b] = n;
+            if (a.out_match_end) a.out_match_end[b] = e;
+            if (verifying && !len_ok) a.out_accept[b] = -1;
+            if (a.status) {
+                int32_t st = s_ver[2];
+                if (st == SWITCHSD_ROW_OK && timeout) st = SWITCHSD_ROW_TIMEOUT;
+                a.status[b] = st;
+            }
         }
     }
     __syncthreads();
@@ -516,7 +522,7 @@ static int step_entry(int32_t *ctx_tokens, int32_t *ctx_lens, const uint16_t *hi
     if (p->n_min < 1 || p->n_max > SWITCHSD_NMAX || p->n_min > p->n_max) return SWITCHSD_ERR_SHAPE;
     if (p->split != 0 && p->split != 1 && p->split != 2 && p->split != 4 && p->split != 8 && p->split != 16)
         return SWITCHSD_ERR_SHAPE;
-    if (p->prefetch != 0 && p->prefetch != 1) return SWITCHSD_ERR_ARG;
+    if ((p->prefetch & ~(SWITCHSD_PREFETCH_CONTEXT | SWITCHSD_PREFETCH_PROBE)) != 0) return SWITCHSD_ERR_ARG;
     if (p->probe_kind == SWITCHSD_PROBE_MLP) {
         if (!mlp_shape_ok(p->d, p->probe_hidden)) return SWITCHSD_ERR_SHAPE;
         if (!p->workspace || !aligned16(p->workspace) ||

@@ -34,7 +34,7 @@ class Session:
                  probe_kind: int = bd.PROBE_LINEAR, probe_hidden: int = 0, future=None,
                  harness: dict | None = None, split: int = 0, d: int | None = None,
                  use_index: bool = False, device="cuda", stream: torch.cuda.Stream | None = None,
-                 prefetch: bool = False):
+                 prefetch: int = 0):
         self.lib = bd.load()
         self.device = torch.device(device)
         if self.device.type == "cuda" and self.device.index is None:

@@ -90,7 +90,7 @@ def test_step_validation(lib):
     assert _step(lib, _params(n_min=5, n_max=4)) == bd.ERR_SHAPE
     assert _step(lib, _params(n_max=33)) == bd.ERR_SHAPE
     assert _step(lib, _params(split=3)) == bd.ERR_SHAPE
-    assert _step(lib, _params(prefetch=2)) == bd.ERR_ARG
+    assert _step(lib, _params(prefetch=4)) == bd.ERR_ARG
     assert _step(lib, _params(prefetch=-1)) == bd.ERR_ARG
     assert _step(lib, _params(probe_kind=1, probe_hidden=0)) == bd.ERR_SHAPE
     # the two-layer probe needs its workspace

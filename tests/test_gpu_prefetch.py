@@ -1,8 +1,8 @@
-"""params.prefetch: the context copies start before the preceding kernel finishes.
+"""params.prefetch: the context and probe copies start before the preceding kernel finishes.
 
 The serving order is verify_step(t) -> target -> verify_step(t+1), launched back to back with no host
 synchronisation, so each call's context copies overlap the target stand-in's kernel while the rows
-were written by the call before it.  With and without prefetch the whole run must give identical
+were written by the call before it (the hidden states are uploaded once, before the chain).  With and without prefetch the whole run must give identical
 outputs (the same kernels in the same order, so bit-identical, the probe logits included) and
 identical contexts; the no-prefetch path is itself held to the oracle by test_gpu_parity.py.
 """
@@ -17,7 +17,7 @@ W = synth.WORKLOADS
 KEYS = ("draft", "len", "mode", "score", "match_n", "match_end", "status", "accept")
 
 
-def _chain(wl, prefetch: bool, steps: int, record_every: int):
+def _chain(wl, prefetch: int, steps: int, record_every: int):
     import torch
     from paper_2609_20186_gb300 import Session, bf16_tensor
 
@@ -47,8 +47,9 @@ def _chain(wl, prefetch: bool, steps: int, record_every: int):
                                         ("uniform_8k", 40)])
 def test_prefetch_matches_back_to_back(name, steps):
     wl = W[name].scaled(steps=steps)
-    a, a_ctx, a_lens = _chain(wl, False, steps, record_every=3)
-    b, b_ctx, b_lens = _chain(wl, True, steps, record_every=3)
+    from paper_2609_20186_gb300 import binding as bd
+    a, a_ctx, a_lens = _chain(wl, 0, steps, record_every=3)
+    b, b_ctx, b_lens = _chain(wl, bd.PREFETCH_CONTEXT | bd.PREFETCH_PROBE, steps, record_every=3)
     assert np.array_equal(a_lens, b_lens)
     assert (a_lens > wl.L0).all()  # every row grew: the chain really appended
     assert np.array_equal(a_ctx, b_ctx)
