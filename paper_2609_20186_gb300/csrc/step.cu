@@ -109,7 +109,8 @@ __global__ void __launch_bounds__(kStepThreads) step_kernel(const StepArgs a) {
     __shared__ int32_t s_suf[SWITCHSD_NMAX];
     __shared__ __align__(16) int32_t s_tail[kHalo + 8];        // x[tail_lo .. L_old), tail_lo = roundown4(L_old - kHalo)
     __shared__ int32_t s_app[SWITCHSD_KMAX + 1];               // tokens appended by the verification
-    __shared__ int32_t s_ver[3];                               // accepted, new length, verify status
+    __shared__ int32_t s_ver[4];                               // accepted, new length, verify status, tail landed
+    __shared__ int32_t s_split[4];                             // warp 0's split: old length, e_lo, e_hi, tiles
     __shared__ unsigned long long s_wkey[kStepWarps];
     __shared__ float s_wz[kStepWarps];
     __shared__ __align__(16) int32_t s_mine[SWITCHSD_KMAX];    // continuation of this CTA's best match
@@ -169,22 +170,29 @@ __global__ void __launch_bounds__(kStepThreads) step_kernel(const StepArgs a) {
 
     // Warp roles until the suffix is known.  Warp 0 reads the row length and issues the copies at
     // once: first the old tail (for the suffix), then the tiles.  Warp 1 verifies the previous draft.
-    // Warps 2.. load this CTA's slice of the probe operands into registers and use them only after the
-    // scan, so no wait on them delays it.  Every thread arrives on the cluster barrier (release) after
-    // reading ctx_lens[b]: once the leader has waited on it, it may publish the new length.
+    // Warps 2.. start the probe copies (unless they went before the wait) and take the length from
+    // shared memory after the CTA barrier.  The leader publishes the new length once every CTA has
+    // arrived on the cluster barrier, so the two warps that read ctx_lens[b] arrive with release
+    // semantics (their read is ordered before the leader's write); the others arrive relaxed (the
+    // leader's barrier initialisation is published by its own mbarrier-init fence).
     int32_t *row = a.ctx + size_t(b) * size_t(a.cap);
-    const int32_t L_old = __ldcg(a.lens + b);
-    const bool len_ok = (L_old >= 1 && L_old <= a.cap);
-    // Split on the old length; the last CTA also covers every end the append can add.
-    const int32_t E_split = len_ok ? L_old - 1 : 0;
-    const int32_t E_max = len_ok ? (verifying ? min(L_old + a.k + 1, a.cap) : L_old) - 1 : 0;
-    int32_t chunk = (E_split + int32_t(C) - 1) / int32_t(C);
-    chunk = (chunk + 3) & ~3;
-    const int32_t e_lo = min(E_split, int32_t(rank) * chunk);
-    const int32_t e_hi = rank + 1 == C ? E_max : min(E_split, e_lo + chunk);
-    const int32_t ntiles = (e_hi - e_lo + a.tile - 1) / a.tile;
-    const int32_t tail_lo = max(0, (L_old - kHalo) & ~3);
-    const int32_t tail_hi = len_ok ? (L_old + 3) & ~3 : tail_lo;  // <= cap since cap % 4 == 0
+    int32_t L_old = 0, e_lo = 0, e_hi = 0, ntiles = 0, tail_lo = 0, tail_hi = 0;
+    bool len_ok = false;
+    auto set_split = [&](int32_t L0) {
+        // Split on the old length; the last CTA also covers every end the append can add.
+        L_old = L0;
+        len_ok = (L_old >= 1 && L_old <= a.cap);
+        const int32_t E_split = len_ok ? L_old - 1 : 0;
+        const int32_t E_max = len_ok ? (verifying ? min(L_old + a.k + 1, a.cap) : L_old) - 1 : 0;
+        int32_t chunk = (E_split + int32_t(C) - 1) / int32_t(C);
+        chunk = (chunk + 3) & ~3;
+        e_lo = min(E_split, int32_t(rank) * chunk);
+        e_hi = rank + 1 == C ? E_max : min(E_split, e_lo + chunk);
+        ntiles = (e_hi - e_lo + a.tile - 1) / a.tile;
+        tail_lo = max(0, (L_old - kHalo) & ~3);
+        tail_hi = len_ok ? (L_old + 3) & ~3 : tail_lo;  // <= cap since cap % 4 == 0
+    };
+    if (warp < 2) set_split(__ldcg(a.lens + b));
 
     // Stage tile t: tokens [max(0, t0 - kHalo), min(roundup4(t1 + kFwd), cap)) land so that token p
     // sits at stage[kHalo + p - t0].  cap % 4 == 0 keeps every bound 16-byte aligned.
@@ -204,6 +212,10 @@ __global__ void __launch_bounds__(kStepThreads) step_kernel(const StepArgs a) {
             mbar_arrive_expect_tx(&tail_bar, tb);
             if (tb > 0) bulk_g2s_hint(s_tail, row + tail_lo, tb, &tail_bar, l2_evict_first_policy());
             for (int t = 0; t < min(ntiles, a.stages); ++t) issue(t);
+            s_split[0] = L_old;
+            s_split[1] = e_lo;
+            s_split[2] = e_hi;
+            s_split[3] = ntiles;
         }
     }
     if (pf_ctx) pdl_wait();  // the previous draft and the target (and all that no bit names) come after this
@@ -251,7 +263,7 @@ __global__ void __launch_bounds__(kStepThreads) step_kernel(const StepArgs a) {
         cluster_arrive_release();
     } else {
         if (!pf_probe && tid == 2 * kWarp) issue_probe();
-        cluster_arrive_release();
+        cluster_arrive_relaxed();
     }
     // Warps 0 and 1 meet (named barrier 1, 64 threads): the suffix needs the old tail and the append.
     if (warp < 2) {
@@ -266,9 +278,19 @@ __global__ void __launch_bounds__(kStepThreads) step_kernel(const StepArgs a) {
             else if (len_ok && p >= 0 && tail_in)
                 v = s_tail[p - tail_lo];
             s_suf[lane] = v;
+            if (lane == 0) s_ver[3] = tail_in;
         }
     }
-    __syncthreads();  // suffix and verification visible
+    __syncthreads();  // suffix, verification and old length visible
+    if (warp >= 2) {
+        L_old = s_split[0];
+        e_lo = s_split[1];
+        e_hi = s_split[2];
+        ntiles = s_split[3];
+        len_ok = (L_old >= 1 && L_old <= a.cap);
+        tail_lo = max(0, (L_old - kHalo) & ~3);
+        tail_hi = len_ok ? (L_old + 3) & ~3 : tail_lo;
+    }
 
     const int32_t acc = s_ver[0], L = s_ver[1];
     const int32_t E = len_ok ? L - 1 : 0;  // candidate ends after the append: [0, E)
@@ -279,7 +301,7 @@ __global__ void __launch_bounds__(kStepThreads) step_kernel(const StepArgs a) {
     const bool pair = n_min >= 2;
     const int32_t m0 = pair ? 2 : 1;
     unsigned long long best = 0;  // CTA-uniform; real keys have m >= n_min >= 1, so 0 = no match
-    bool bad = false;             // CTA-uniform: a copy did not land in time
+    bool bad = s_ver[3] == 0;     // CTA-uniform: a copy did not land in time
     for (int t = 0; t < ntiles && !bad; ++t) {
         const int s = t % a.stages;
         const bool landed = mbar_wait(&bars[s], uint32_t(t / a.stages) & 1u);
@@ -372,8 +394,10 @@ __global__ void __launch_bounds__(kStepThreads) step_kernel(const StepArgs a) {
     if (bad) {
         best = kTimeoutBit;
         // Give the copies still in flight a second bounded wait before the CTA's memory goes away.
-        if (tid == 0)
+        if (tid == 0) {
             for (int u = 0; u < min(ntiles, a.stages); ++u) (void)mbar_wait(&bars[u], 0u);
+            (void)mbar_wait(&tail_bar, 0u);
+        }
     }
 
     // The probe slice (staged during the scan), then the CTA's partial in a fixed order.
