@@ -91,6 +91,13 @@ def configure(lib):
                                        ctypes.c_int32, ctypes.c_int32, _i32p, _i32p, _i32p,
                                        _i32p, _i32p]
     lib.oracle_verify_rows.restype = None
+    lib.oracle_verify_sampled_row.argtypes = [_i32p, _i32p, ctypes.c_int32, _i32p, ctypes.c_int32,
+                                              _f32p, _f32p, _f32p, _i32p, _i32p]
+    lib.oracle_verify_sampled_row.restype = ctypes.c_int32
+    lib.oracle_verify_sampled_rows.argtypes = [_i32p, _i32p, ctypes.c_int32, ctypes.c_int32,
+                                               ctypes.c_int32, ctypes.c_int32, _i32p, _i32p, _f32p,
+                                               _f32p, _f32p, _i32p, _i32p, _i32p]
+    lib.oracle_verify_sampled_rows.restype = None
     return lib
 
 
@@ -192,6 +199,26 @@ def verify_row(row: np.ndarray, L: int, cap: int, draft, target):
     return Lc.value, acc.value, st
 
 
+def verify_sampled_row(row: np.ndarray, L: int, cap: int, draft, p, u, resample, q=None):
+    """Verification at T > 0 (App. A) + append on one row buffer (modified in place): draft token i
+    is accepted iff float32(u[i] * q[i]) < p[i] (q = None: a copy draft, q = 1); resample has
+    len(draft) + 1 entries.  Returns (new_L, accept, status)."""
+    assert row.dtype == np.int32 and row.flags.c_contiguous and row.shape[0] >= cap
+    d = _c(draft, np.int32)
+    n = d.shape[0]
+    pa, ua = _c(p, np.float32), _c(u, np.float32)
+    qa = None if q is None else _c(q, np.float32)
+    r = _c(resample, np.int32)
+    assert pa.shape[0] >= n and ua.shape[0] >= n and r.shape[0] >= n + 1
+    assert qa is None or qa.shape[0] >= n
+    Lc = ctypes.c_int32(L)
+    acc = ctypes.c_int32()
+    st = _load().oracle_verify_sampled_row(_ptr(row, _i32p), ctypes.byref(Lc), cap, _ptr(d, _i32p), n,
+                                           _ptr(pa, _f32p), None if qa is None else _ptr(qa, _f32p),
+                                           _ptr(ua, _f32p), _ptr(r, _i32p), ctypes.byref(acc))
+    return Lc.value, acc.value, st
+
+
 # ---------------------------------------------------------------------------------------------
 # Batched functions (ABI layouts), used by the parity tests and the CPU baseline
 # ---------------------------------------------------------------------------------------------
@@ -253,4 +280,33 @@ def verify(ctx: np.ndarray, lens: np.ndarray, draft: np.ndarray, draft_len: np.n
     lib.oracle_verify_rows(_ptr(ctx, _i32p), _ptr(lens, _i32p), b0, bend, cap, k,
                            _ptr(draft, _i32p), _ptr(draft_len, _i32p), _ptr(target, _i32p),
                            _ptr(acc, _i32p), _ptr(st, _i32p))
+    return acc, st
+
+
+def verify_sampled(ctx: np.ndarray, lens: np.ndarray, draft: np.ndarray, draft_len: np.ndarray,
+                   p: np.ndarray, u: np.ndarray, resample: np.ndarray, q: np.ndarray | None = None,
+                   rows: tuple[int, int] | None = None):
+    """Verification at T > 0 + append on rows [b0, b1) (all by default); ctx and lens are updated in
+    place.  p, u, q float32 [B, k] (q None: every draft is a copy draft), resample int32 [B, k + 1].
+    Returns (accept [B], status [B])."""
+    lib = _load()
+    assert ctx.dtype == np.int32 and ctx.flags.c_contiguous
+    assert lens.dtype == np.int32 and lens.flags.c_contiguous
+    B, cap = ctx.shape
+    draft = _c(draft, np.int32)
+    k = draft.shape[1]
+    draft_len = _c(draft_len, np.int32)
+    p, u = _c(p, np.float32), _c(u, np.float32)
+    assert p.shape == (B, k) and u.shape == (B, k)
+    qa = None if q is None else _c(q, np.float32)
+    assert qa is None or qa.shape == (B, k)
+    resample = _c(resample, np.int32)
+    assert resample.shape == (B, k + 1)
+    acc = np.zeros(B, np.int32)
+    st = np.zeros(B, np.int32)
+    b0, bend = rows if rows is not None else (0, B)
+    lib.oracle_verify_sampled_rows(_ptr(ctx, _i32p), _ptr(lens, _i32p), b0, bend, cap, k,
+                                   _ptr(draft, _i32p), _ptr(draft_len, _i32p), _ptr(p, _f32p),
+                                   None if qa is None else _ptr(qa, _f32p), _ptr(u, _f32p),
+                                   _ptr(resample, _i32p), _ptr(acc, _i32p), _ptr(st, _i32p))
     return acc, st

@@ -193,3 +193,49 @@ void oracle_verify_rows(int32_t *ctx, int32_t *lens, int32_t b0, int32_t b1, int
         if (status != NULL) status[b] = st;
     }
 }
+
+/*
+ * Verification at temperature T > 0 (App. A runs SwitchSD with sampling; the acceptance rule is the
+ * speculative-sampling rule of the works §2 builds on).  Draft token i was proposed with drafter
+ * probability q[i] (q == NULL: a copy draft, which is deterministic, so q = 1) and has target
+ * probability p[i] at its position.  It is accepted iff u[i] * q[i] < p[i] -- the event
+ * u < min(1, p/q) for u uniform in [0, 1) -- with the product rounded to binary32 and compared in
+ * binary32 (the kernel's precision; float arithmetic here is binary32).  The first rejection, at a,
+ * ends the block: the appended token there is resample[a], the caller's draw from the residual
+ * distribution max(0, p - q) renormalised; after len acceptances resample[len] is the bonus draw from
+ * the target.  The append and the capacity rule are those of oracle_verify_row.
+ */
+int32_t oracle_verify_sampled_row(int32_t *row, int32_t *L, int32_t cap, const int32_t *draft, int32_t len,
+                                  const float *p, const float *q, const float *u, const int32_t *resample,
+                                  int32_t *accept)
+{
+    int32_t a = 0;
+    while (a < len) {
+        float qa = (q != NULL) ? q[a] : 1.0f;
+        float prod = u[a] * qa;
+        if (!(prod < p[a])) break;
+        ++a;
+    }
+    if (*L + a + 1 > cap) {
+        *accept = -1;
+        return ORACLE_ROW_CAPACITY;
+    }
+    for (int32_t i = 0; i < a; ++i) row[*L + i] = draft[i];
+    row[*L + a] = resample[a];
+    *L += a + 1;
+    *accept = a;
+    return ORACLE_ROW_OK;
+}
+
+void oracle_verify_sampled_rows(int32_t *ctx, int32_t *lens, int32_t b0, int32_t b1, int32_t cap, int32_t k,
+                                const int32_t *draft, const int32_t *draft_len, const float *p, const float *q,
+                                const float *u, const int32_t *resample, int32_t *out_accept, int32_t *status)
+{
+    for (int32_t b = b0; b < b1; ++b) {
+        int32_t st = oracle_verify_sampled_row(ctx + (int64_t)b * cap, &lens[b], cap, draft + (int64_t)b * k,
+                                               draft_len[b], p + (int64_t)b * k,
+                                               q != NULL ? q + (int64_t)b * k : NULL, u + (int64_t)b * k,
+                                               resample + (int64_t)b * (k + 1), &out_accept[b]);
+        if (status != NULL) status[b] = st;
+    }
+}

@@ -47,6 +47,11 @@ MUTANTS = {
     "verify: accepts one past the mismatch": ("while (a < len && draft[a] == target[a]) ++a;",
                                               "while (a < len && draft[a] == target[a]) ++a;\n"
                                               "    if (a < len) ++a;"),
+    "sampled: accepts a tie": ("if (!(prod < p[a])) break;", "if (!(prod <= p[a])) break;"),
+    "sampled: ignores q": ("float qa = (q != NULL) ? q[a] : 1.0f;", "float qa = 1.0f;"),
+    "sampled: inverts the ratio": ("float prod = u[a] * qa;\n        if (!(prod < p[a])) break;",
+                                   "float prod = u[a] * p[a];\n        if (!(prod < qa)) break;"),
+    "sampled: wrong resample": ("row[*L + a] = resample[a];", "row[*L + a] = resample[a > 0 ? a - 1 : 0];"),
 }
 
 
@@ -110,6 +115,18 @@ def battery() -> list:
     row = np.zeros(6, np.int32)
     row[:4] = [1, 2, 3, 4]
     check("verify fits exactly", oracle.verify_row(row, 4, 6, [5, 9], [5, 6, 7]) == (6, 1, 0))
+    # sampled verification hand cases (test_oracle_sampled.py)
+    row = np.zeros(16, np.int32)
+    row[:3] = [1, 2, 3]
+    check("sampled partial", oracle.verify_sampled_row(row, 3, 16, [4, 5, 6], [0.6, 0.4, 0.9], [0.5] * 3,
+                                                       [7, 8, 9, 10]) == (5, 1, 0) and row[4] == 8)
+    row = np.zeros(8, np.int32)
+    check("sampled tie", oracle.verify_sampled_row(row, 1, 8, [4], [0.5], [0.5], [7, 9])[1] == 0)
+    row = np.zeros(8, np.int32)
+    check("sampled q", oracle.verify_sampled_row(row, 1, 8, [4, 5], [0.3, 0.3], [0.5, 0.7], [7, 8, 9],
+                                                 q=[0.5, 0.5])[1] == 1)
+    row = np.zeros(8, np.int32)
+    check("sampled low p", oracle.verify_sampled_row(row, 1, 8, [4], [0.2], [0.5], [7, 9], q=[1.0])[1] == 0)
     return failed
 
 
