@@ -341,7 +341,7 @@ class ReplicaLoop:
         p.prefetch = (bd.PREFETCH_CONTEXT | bd.PREFETCH_PROBE) if prefetch else 0
         # one workspace per batch, so consecutive launches never share one
         probe = bd.switchsd_params()
-        probe.B, probe.probe_kind, probe.probe_hidden = B, wl.probe_kind, wl.probe_hidden
+        probe.B, probe.d, probe.probe_kind, probe.probe_hidden = B, wl.d, wl.probe_kind, wl.probe_hidden
         ws = max(256, int(self.lib.switchsd_workspace_bytes(ctypes.byref(probe))))
         self.workspace = torch.empty(R, ws, dtype=torch.uint8, device=dev)
         self.params = []

@@ -92,8 +92,8 @@ typedef struct switchsd_index switchsd_index;
  *   split        CTAs per row (1, 2, 4, 8 or 16); 0 lets the library choose
  *   workspace, workspace_bytes   device scratch for the two-layer probe: at least
  *                switchsd_workspace_bytes(params) bytes, 16-byte aligned, caller-owned; may be NULL for
- *                the linear probe.  It holds the probe's per-tile partial logits between its two kernels,
- *                so calls sharing one workspace must not overlap on the GPU
+ *                the linear probe.  It holds the first layer's split-K partial sums between the probe's
+ *                kernel and the step kernel, so calls sharing one workspace must not overlap on the GPU
  *   index        NULL: search by rescanning the context.  Else an index from switchsd_index_create for
  *                the same B, cap, n_min and n_max, kept current by switchsd_index_build and by the
  *                verification entry points given the same index; the search then walks its chains
@@ -116,8 +116,8 @@ typedef struct switchsd_index switchsd_index;
  *                the call is always safe.  In a serving loop the target's last kernel (its argmax)
  *                writes neither the context nor the hidden state.  The previous draft, its length
  *                and the target argmax are always read after the wait.  The index search ignores the
- *                field and the two-layer probe ignores SWITCHSD_PREFETCH_PROBE.  Other bits are
- *                SWITCHSD_ERR_ARG.
+ *                field; with the two-layer probe SWITCHSD_PREFETCH_PROBE lets the probe kernel's copies
+ *                of the hidden states and W1 start early.  Other bits are SWITCHSD_ERR_ARG.
  */
 typedef struct {
     int32_t B, cap, d, k, n_min, n_max, kappa;
@@ -224,8 +224,10 @@ int switchsd_verify_step(const int32_t *draft, const int32_t *target_argmax, con
 
 /*
  * Bytes of device workspace switchsd_step / switchsd_verify_step need for `params` (0 for the linear
- * probe; for the two-layer probe, one float per row and 64-unit tile of the hidden layer, rounded up to
- * 256 bytes).  Reads B, probe_kind and probe_hidden only.
+ * probe; for the two-layer probe, S x B x H1p floats rounded up to 256 bytes, where S is the first
+ * layer's split of d -- the largest power of two <= 16 with at least two 64-element chunks of d per
+ * part, 16 for d >= 2048 -- and H1p is probe_hidden rounded up to 64).  Reads B, d, probe_kind and
+ * probe_hidden only.
  */
 size_t switchsd_workspace_bytes(const switchsd_params *params);
 
@@ -234,12 +236,12 @@ size_t switchsd_workspace_bytes(const switchsd_params *params);
  * a convenience of the library.  Some callers cannot hand the library a workspace at call time (an
  * inference server that gives all of the GPU's memory to its own pool when it starts, or a host program
  * with no CUDA allocator of its own); this entry point takes the same arguments as switchsd_step, ignores
- * params->workspace and uses a fixed 256 KiB array compiled into the library instead.  It allocates
+ * params->workspace and uses a fixed 16 MiB array compiled into the library instead.  It allocates
  * nothing (no cudaMalloc, no cudaFree).
  *
- *   Limit: the two-layer probe needs B * ceil(probe_hidden / 64) <= 65,536 (for example B <= 16,384
- *   with 256 hidden units); larger requests return SWITCHSD_ERR_SHAPE.  The linear probe has no limit
- *   beyond switchsd_step's.
+ *   Limit: the two-layer probe needs switchsd_workspace_bytes(params) <= 16 MiB (S x B x H1p <= 4 Mi
+ *   floats: for example B <= 1,024 with d >= 2048 and 256 hidden units); larger requests return
+ *   SWITCHSD_ERR_SHAPE.  The linear probe has no limit beyond switchsd_step's.
  *   Set-up: the first call on each device looks up the array's device address (cudaGetSymbolAddress,
  *   with that device current); make that first call before any stream capture.
  *   Sharing: every call on a device uses the same array, and the array keeps whatever the last call

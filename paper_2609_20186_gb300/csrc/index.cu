@@ -17,6 +17,7 @@
 #include <new>
 
 #include "common.cuh"
+#include "index.cuh"
 #include "mlp.cuh"
 
 struct switchsd_index {
@@ -45,8 +46,10 @@ __device__ __forceinline__ uint32_t gram_hash(int n, Tok tok, int log2_buckets) 
 struct IndexArgs {
     int32_t *ctx, *lens;
     const uint16_t *hidden, *probe_w;
-    const float *z_pre;  // two-layer probe partial logits, else null
-    int32_t z_tiles;
+    const float *z1_part;  // two-layer probe: split-K partial sums of W1 h [mlp_S][B][H1p], else null
+    const float *b1;       // two-layer probe: first-layer biases (null = zero) and output weights
+    const uint16_t *w2;
+    int32_t mlp_S, H1, H1p;
     float b2;
     const int32_t *pv_draft, *pv_target, *pv_len;  // verification inputs (null: no verification)
     int32_t *out_accept;
@@ -177,9 +180,17 @@ __global__ void __launch_bounds__(kIdxMaxWarps * kWarp) index_kernel(const Index
     }
     if (lane == 0 && warp < kIdxMaxWarps) s_found[warp] = found;
 
-    // Probe partial over the whole hidden vector (linear probe).
+    // Probe partial over the whole hidden vector (linear probe), or over every unit of the two-layer
+    // probe: the S split-K partial sums in order, then b1, ReLU and w2.
     float zp = 0.f;
-    if (a.z_pre == nullptr) {
+    if (a.z1_part != nullptr) {
+        for (int u = tid; u < a.H1; u += blockDim.x) {
+            float z1 = 0.f;
+            for (int s = 0; s < a.mlp_S; ++s) z1 += a.z1_part[(size_t(s) * a.B + size_t(b)) * a.H1p + u];
+            const float bias = a.b1 ? a.b1[u] : 0.f;
+            zp = fmaf(bf16_lo(uint32_t(a.w2[u])), fmaxf(z1 + bias, 0.f), zp);
+        }
+    } else {
         const uint4 *h4 = reinterpret_cast<const uint4 *>(a.hidden + size_t(b) * a.d);
         const uint4 *w4 = reinterpret_cast<const uint4 *>(a.probe_w);
         for (int v = tid; v < (a.d >> 3); v += blockDim.x) {
@@ -200,12 +211,8 @@ __global__ void __launch_bounds__(kIdxMaxWarps * kWarp) index_kernel(const Index
 
     if (tid == 0) {
         float z = 0.f;
-        if (a.z_pre != nullptr) {
-            z = a.b2;
-            for (int t = 0; t < a.z_tiles; ++t) z += a.z_pre[size_t(t) * a.B + b];
-        } else {
-            for (int w = 0; w < nwarps; ++w) z += s_wz[w];
-        }
+        for (int w = 0; w < nwarps; ++w) z += s_wz[w];
+        if (a.z1_part != nullptr) z += a.b2;
         int32_t nstar = 0, estar = -1;
         for (int w = a.n_max - a.n_min; w >= 0; --w)
             if (s_found[w] >= 0) {
@@ -277,18 +284,23 @@ int index_n_min(const switchsd_index *idx) { return idx->n_min; }
 int index_n_max(const switchsd_index *idx) { return idx->n_max; }
 
 int index_launch(switchsd_index *idx, int32_t *ctx, int32_t *lens, const uint16_t *hidden, const uint16_t *probe_w,
-                 const float *z_pre, int z_tiles, float b2, const int32_t *pv_draft, const int32_t *pv_target,
-                 const int32_t *pv_len, int32_t *out_accept, int32_t *out_draft, int32_t *out_len, int32_t *out_mode,
-                 float *out_score, int32_t *out_match_n, int32_t *out_match_end, int32_t *status, int B, int cap,
-                 int d, int k, int n_min, int n_max, int kappa, float logit_tau, bool stepping, cudaStream_t stream) {
+                 const float *z1_part, const float *b1, const uint16_t *w2, int mlp_S, int H1, int H1p, float b2,
+                 const int32_t *pv_draft, const int32_t *pv_target, const int32_t *pv_len, int32_t *out_accept,
+                 int32_t *out_draft, int32_t *out_len, int32_t *out_mode, float *out_score, int32_t *out_match_n,
+                 int32_t *out_match_end, int32_t *status, int B, int cap, int d, int k, int n_min, int n_max, int kappa,
+                 float logit_tau, bool stepping, cudaStream_t stream) {
     if (idx->B != B || idx->cap != cap || idx->n_min != n_min || idx->n_max != n_max) return SWITCHSD_ERR_SHAPE;
     IndexArgs a;
     a.ctx = ctx;
     a.lens = lens;
     a.hidden = hidden;
     a.probe_w = probe_w;
-    a.z_pre = z_pre;
-    a.z_tiles = z_tiles;
+    a.z1_part = z1_part;
+    a.b1 = b1;
+    a.w2 = w2;
+    a.mlp_S = mlp_S;
+    a.H1 = H1;
+    a.H1p = H1p;
     a.b2 = b2;
     a.pv_draft = pv_draft;
     a.pv_target = pv_target;

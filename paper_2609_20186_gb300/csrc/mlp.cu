@@ -1,16 +1,14 @@
-// mlp.cu -- the two-layer copy-intent probe z = w2 . ReLU(W1 h + b1) + b2 on the tensor cores.
+// mlp.cu -- first layer of the two-layer copy-intent probe z = w2 . ReLU(W1 h + b1) + b2, on the tensor cores.
 //
 // The paper's probe is linear (Eq. 3); this two-layer form is an extension used with probe_kind
 // SWITCHSD_PROBE_MLP.  Its first layer is a real contraction, Z1[B, H1] = H[B, d] . W1[H1, d]^T, so it
-// runs on tcgen05: each thread-block cluster of S CTAs owns one 128-row x 64-unit tile of Z1 and
-// splits K = d between its CTAs.  A CTA stages its K chunks of H and W1 in shared memory with TMA
-// (128-byte swizzle, zero fill past the tensor edges), one thread issues tcgen05.mma (bf16 x bf16,
-// fp32 accumulators in 64 TMEM columns), and the four warps read their 32 rows back with tcgen05.ld.
-// After a cluster barrier (every CTA's MMAs complete) the S partial tiles are reduce-scattered across
-// the cluster with st.async into the freed operand areas (CTA r owns 64/S columns); the owner adds
-// b1, applies ReLU, weights by w2 and sums its columns; the leader adds the S owners' sums in a fixed
-// order and writes the tile's partial logit zpart[n_tile][b] to the caller's workspace.  The step kernel adds the n_tile partials (fixed order) and b2.  Deterministic: every sum
-// has a fixed order.
+// runs on tcgen05.  K = d is split S ways: CTA (s, n, m) stages its K chunks of H rows [128 m, +128) and
+// W1 units [64 n, +64) in shared memory with TMA (128-byte swizzle, zero fill past the tensor edges), one
+// thread issues tcgen05.mma (bf16 x bf16, fp32 accumulators in 64 TMEM columns), the four warps read
+// their 32 rows back with tcgen05.ld and store them as the split-K partial sums
+//     part[s][b][u]  (fp32, s < S, b < B, u < H1p = H1 rounded up to 64; units >= H1 hold zeros).
+// The step kernel that follows adds the S partials of its row in order, then b1, ReLU, w2 and b2: every
+// sum has a fixed order, so the result is deterministic.  No cluster and no cross-CTA exchange here.
 #include <cudaTypedefs.h>
 
 #include "common.cuh"
@@ -24,9 +22,8 @@ constexpr int kMlpKc = 64;             // K elements per staged chunk: one 128-b
 constexpr int kMlpThreads = 128;       // four warps: one per 32 TMEM lanes
 constexpr uint32_t kAChunk = kMlpM * kMlpKc * 2;    // 16 KB
 constexpr uint32_t kBChunk = kMlpN * kMlpKc * 2;    // 8 KB
-constexpr uint32_t kRecvBytes = kMlpM * kMlpN * 4;  // 32 KB: the columns a CTA owns, from every CTA
 constexpr uint32_t kTmemCols = 64;
-static_assert(kMaxMlpChunks * (kAChunk + kBChunk) + 1024 + 16 * 128 * 4 + 64 <= 227 * 1024,
+static_assert(kMaxMlpChunks * (kAChunk + kBChunk) + 1024 + 64 <= 227 * 1024,
               "operands, alignment slack and static shared memory must fit one CTA");
 
 // Instruction descriptor of tcgen05.mma kind::f16: D fp32, A and B bf16, both K-major, M = 128, N = 64.
@@ -34,10 +31,8 @@ constexpr uint32_t kIdesc = (1u << 4) | (1u << 7) | (1u << 10) | (uint32_t(kMlpN
                             (uint32_t(kMlpM >> 4) << 24);
 
 struct MlpArgs {
-    const float *b1;
-    const uint16_t *w2;
-    float *zpart;  // [NT][B]
-    int32_t B, d, H1, nchunks;
+    float *part;   // [S][B][H1p]
+    int32_t B, H1p, nchunks, prefetch;
 };
 
 // Shared-memory matrix descriptor: K-major, 128-byte swizzle, 8-row groups 1024 bytes apart.
@@ -52,12 +47,6 @@ __device__ __forceinline__ void tma_load_2d(void *dst, const CUtensorMap *map, i
             smem_addr(dst)),
         "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(smem_addr(bar))
         : "memory");
-}
-
-__device__ __forceinline__ void st_async_f32(uint32_t cluster_addr, float v, uint32_t cluster_mbar) {
-    asm volatile("st.async.shared::cluster.mbarrier::complete_tx::bytes.b32 [%0], %1, [%2];\n" ::"r"(cluster_addr),
-                 "r"(__float_as_uint(v)), "r"(cluster_mbar)
-                 : "memory");
 }
 
 __device__ __forceinline__ void tmem_ld32(uint32_t taddr, float *v) {
@@ -78,36 +67,34 @@ __global__ void __launch_bounds__(kMlpThreads) mlp_tc_kernel(const __grid_consta
                                                              const __grid_constant__ CUtensorMap tm_w,
                                                              const MlpArgs a) {
     extern __shared__ uint8_t smem_raw[];
-    __shared__ __align__(8) uint64_t tma_bar, mma_bar, red_bar, fin_bar;
+    __shared__ __align__(8) uint64_t tma_bar, mma_bar;
     __shared__ uint32_t s_tmem;
-    __shared__ float s_fin[kMaxMlpSplit][kMlpM];  // leader: every owner's per-row sum
 
     const int tid = threadIdx.x, warp = tid >> 5;
-    const uint32_t rank = cluster_ctarank();
-    const uint32_t S = cluster_nctarank();
+    const int S = int(gridDim.x), ks = blockIdx.x;
     const int n_tile = blockIdx.y, m0 = blockIdx.z * kMlpM, n0 = n_tile * kMlpN;
-    const int W = kMlpN / int(S);  // columns owned by each CTA
-    const int per = (a.nchunks + int(S) - 1) / int(S);
-    const int c0 = int(rank) * per;
+    const int per = (a.nchunks + S - 1) / S;
+    const int c0 = ks * per;
     const int nck = max(0, min(a.nchunks, c0 + per) - c0);
     // 1024-byte aligned operand area (the swizzle atom): A chunks, then B chunks.
     uint8_t *base = smem_raw + ((1024u - (smem_addr(smem_raw) & 1023u)) & 1023u);
     uint8_t *opA = base;
     uint8_t *opB = base + size_t(per) * kAChunk;
-    // The reduce-scatter lands on the operand area: it is written only after every CTA of the cluster
-    // has finished its MMAs (cluster barrier below).
-    float *recv = reinterpret_cast<float *>(base);  // [S][128][W]
+    auto issue_loads = [&]() {
+        mbar_arrive_expect_tx(&tma_bar, uint32_t(nck) * (kAChunk + kBChunk));
+        for (int c = 0; c < nck; ++c) {
+            tma_load_2d(opA + size_t(c) * kAChunk, &tm_h, (c0 + c) * kMlpKc, m0, &tma_bar);
+            tma_load_2d(opB + size_t(c) * kBChunk, &tm_w, (c0 + c) * kMlpKc, n0, &tma_bar);
+        }
+    };
 
     if (tid == 0) {
         mbar_init(&tma_bar, 1);
         mbar_init(&mma_bar, 1);
-        mbar_init(&red_bar, 1);
-        mbar_arrive_expect_tx(&red_bar, kRecvBytes);
-        if (rank == 0) {
-            mbar_init(&fin_bar, 1);
-            mbar_arrive_expect_tx(&fin_bar, S * kMlpM * 4u);
-        }
         fence_mbar_init();
+        // With the probe prefetch bit the caller guarantees that the preceding kernel writes neither
+        // the hidden states nor W1, so their copies may start before the grid-dependency wait.
+        if (a.prefetch && nck > 0) issue_loads();
     }
     if (warp == 0) {
         asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;\n" ::"r"(smem_addr(&s_tmem)),
@@ -115,16 +102,9 @@ __global__ void __launch_bounds__(kMlpThreads) mlp_tc_kernel(const __grid_consta
                      : "memory");
         asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;\n" ::: "memory");
     }
-    pdl_wait();
+    pdl_wait();     // the partial sums below overwrite what an earlier step kernel may still read
     pdl_trigger();
-
-    if (tid == 0 && nck > 0) {
-        mbar_arrive_expect_tx(&tma_bar, uint32_t(nck) * (kAChunk + kBChunk));
-        for (int c = 0; c < nck; ++c) {
-            tma_load_2d(opA + size_t(c) * kAChunk, &tm_h, (c0 + c) * kMlpKc, m0, &tma_bar);
-            tma_load_2d(opB + size_t(c) * kBChunk, &tm_w, (c0 + c) * kMlpKc, n0, &tma_bar);
-        }
-    }
+    if (tid == 0 && !a.prefetch && nck > 0) issue_loads();
     asm volatile("tcgen05.fence::before_thread_sync;\n" ::: "memory");
     __syncthreads();
     asm volatile("tcgen05.fence::after_thread_sync;\n" ::: "memory");
@@ -163,7 +143,8 @@ __global__ void __launch_bounds__(kMlpThreads) mlp_tc_kernel(const __grid_consta
     asm volatile("tcgen05.fence::after_thread_sync;\n" ::: "memory");
     ok = __syncthreads_and(ok && mma_done);
 
-    // Row tid of the tile: its 64 accumulators (zero when this CTA had no K chunk).
+    // Row tid of the tile: its 64 accumulators (zero when this CTA had no K chunk; NaN when a copy or
+    // the MMAs did not complete in time, so the row's logit shows the failure).
     float v[kMlpN];
     if (nck > 0 && ok) {
         const uint32_t taddr = tmem + (uint32_t(warp * 32) << 16);
@@ -171,47 +152,14 @@ __global__ void __launch_bounds__(kMlpThreads) mlp_tc_kernel(const __grid_consta
         tmem_ld32(taddr + 32, v + 32);
         asm volatile("tcgen05.wait::ld.sync.aligned;\n" ::: "memory");
     } else {
+        const float fill = ok ? 0.f : __int_as_float(0x7fc00000);
 #pragma unroll
-        for (int i = 0; i < kMlpN; ++i) v[i] = 0.f;
+        for (int i = 0; i < kMlpN; ++i) v[i] = fill;
     }
-
-    // Once every CTA has arrived, all MMAs of the cluster are complete (operand areas free) and every
-    // barrier is initialised: the reduce-scatter may start.
-    cluster_arrive_release();
-    cluster_wait_acquire();
-    // Reduce-scatter: columns [o W, (o+1) W) go to CTA o, into its recv[rank][tid][0..W).
-    for (int o = 0; o < int(S); ++o) {
-        const uint32_t mb = map_to_rank(&red_bar, uint32_t(o));
-        for (int q = 0; q < W; q += 4) {
-            const int col = o * W + q;
-            uint4 u;
-            u.x = __float_as_uint(v[col]);
-            u.y = __float_as_uint(v[col + 1]);
-            u.z = __float_as_uint(v[col + 2]);
-            u.w = __float_as_uint(v[col + 3]);
-            st_async_v4(map_to_rank(&recv[(size_t(rank) * kMlpM + tid) * W + q], uint32_t(o)), u, mb);
-        }
-    }
-    // Owner: add the S partials in order, then b1, ReLU and w2 over the owned columns.
-    const bool got = mbar_wait(&red_bar, 0);
-    float zt = 0.f;
-    for (int c = 0; c < W; ++c) {
-        float sum = 0.f;
-        for (uint32_t src = 0; src < S; ++src) sum += recv[(size_t(src) * kMlpM + tid) * W + c];
-        const int u = n0 + int(rank) * W + c;
-        if (u < a.H1) {
-            const float pre = sum + (a.b1 ? a.b1[u] : 0.f);
-            zt = fmaf(bf16_lo(uint32_t(a.w2[u])), fmaxf(pre, 0.f), zt);
-        }
-    }
-    if (!(got && ok)) zt = __int_as_float(0x7fc00000);  // NaN marks a tile that did not complete
-    st_async_f32(map_to_rank(&s_fin[rank][tid], 0), zt, map_to_rank(&fin_bar, 0));
-    if (rank == 0) {
-        const bool all_in = mbar_wait(&fin_bar, 0);
-        float z = 0.f;
-        for (uint32_t src = 0; src < S; ++src) z += s_fin[src][tid];
-        if (!all_in) z = __int_as_float(0x7fc00000);
-        if (m0 + tid < a.B) a.zpart[size_t(n_tile) * a.B + m0 + tid] = z;
+    if (m0 + tid < a.B) {
+        float4 *dst = reinterpret_cast<float4 *>(a.part + (size_t(ks) * a.B + size_t(m0 + tid)) * a.H1p + n0);
+#pragma unroll
+        for (int q = 0; q < kMlpN / 4; ++q) dst[q] = make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
     }
     asm volatile("tcgen05.fence::before_thread_sync;\n" ::: "memory");
     __syncthreads();
@@ -261,39 +209,35 @@ bool mlp_shape_ok(int d, int H1) {
     return (nchunks + s - 1) / s <= kMaxMlpChunks && H1 >= 1 && H1 <= kMaxMlpHidden && d >= 8 && d % 8 == 0;
 }
 
-int mlp_tiles_n(int H1) { return (H1 + kMlpN - 1) / kMlpN; }
+int mlp_hidden_padded(int H1) { return (H1 + kMlpN - 1) / kMlpN * kMlpN; }
 
-cudaError_t launch_mlp_tc(const uint16_t *hidden, const uint16_t *W1, const uint16_t *w2, const float *b1, float *zpart,
-                          int B, int d, int H1, cudaStream_t stream) {
+cudaError_t launch_mlp_tc(const uint16_t *hidden, const uint16_t *W1, float *part, int B, int d, int H1,
+                          bool prefetch, cudaStream_t stream) {
     CUtensorMap tm_h, tm_w;
     if (!encode_rows(&tm_h, hidden, B, d, kMlpM) || !encode_rows(&tm_w, W1, H1, d, kMlpN))
         return cudaErrorInvalidValue;
     const int nchunks = (d + kMlpKc - 1) / kMlpKc;
     const int S = mlp_split(d);
     const int per = (nchunks + S - 1) / S;
-    const size_t ops = size_t(per) * (kAChunk + kBChunk);
-    const size_t smem = 1024 + (ops > kRecvBytes ? ops : size_t(kRecvBytes));
+    const size_t smem = 1024 + size_t(per) * (kAChunk + kBChunk);
     static bool attr_done[64] = {false};
     int dev = 0;
     cudaGetDevice(&dev);
     if (dev >= 0 && dev < 64 && !attr_done[dev]) {
-        cudaError_t e = cudaFuncSetAttribute(mlp_tc_kernel, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
-        if (e != cudaSuccess) return e;
-        e = cudaFuncSetAttribute(mlp_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                 int(1024 + size_t(kMaxMlpChunks) * (kAChunk + kBChunk)));
+        const cudaError_t e = cudaFuncSetAttribute(mlp_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                                   int(1024 + size_t(kMaxMlpChunks) * (kAChunk + kBChunk)));
         if (e != cudaSuccess) return e;
         attr_done[dev] = true;
     }
     MlpArgs a;
-    a.b1 = b1;
-    a.w2 = w2;
-    a.zpart = zpart;
+    a.part = part;
     a.B = B;
-    a.d = d;
-    a.H1 = H1;
+    a.H1p = mlp_hidden_padded(H1);
     a.nchunks = nchunks;
-    const dim3 grid(unsigned(S), unsigned(mlp_tiles_n(H1)), unsigned((B + kMlpM - 1) / kMlpM));
-    return launch_pdl(mlp_tc_kernel, grid, dim3(kMlpThreads), smem, stream, unsigned(S), tm_h, tm_w, a);
+    a.prefetch = prefetch ? 1 : 0;
+    const dim3 grid(unsigned(S), unsigned(a.H1p / kMlpN), unsigned((B + kMlpM - 1) / kMlpM));
+    // An explicit one-CTA cluster: the copies and the MMA commit address shared::cluster.
+    return launch_pdl(mlp_tc_kernel, grid, dim3(kMlpThreads), smem, stream, 1u, tm_h, tm_w, a);
 }
 
 }  // namespace switchsd

@@ -6,19 +6,20 @@
 
 namespace switchsd {
 
-constexpr int kMaxMlpSplit = 16;    // CTAs per cluster splitting K
+constexpr int kMaxMlpSplit = 16;    // CTAs splitting K
 constexpr int kMaxMlpChunks = 8;    // 64-element K chunks staged per CTA: d <= 16 * 8 * 64 = 8192
 constexpr int kMaxMlpHidden = 1024; // H1: at most 16 tiles of 64 units
 
-// K split (cluster size) used for hidden size d.
+// K split used for hidden size d: the partial sums per (row, unit).
 int mlp_split(int d);
 // Whether (d, H1) is within the kernel's limits.
 bool mlp_shape_ok(int d, int H1);
-// Number of 64-unit tiles of the hidden layer: the partial logits per row written to the workspace.
-int mlp_tiles_n(int H1);
-// zpart [mlp_tiles_n(H1)][B] <- per-tile partial logits (without b2).  Launched with programmatic
-// stream serialization.
-cudaError_t launch_mlp_tc(const uint16_t *hidden, const uint16_t *W1, const uint16_t *w2, const float *b1, float *zpart,
-                          int B, int d, int H1, cudaStream_t stream);
+// H1 rounded up to the 64-unit tile: the row stride of the partial sums.
+int mlp_hidden_padded(int H1);
+// part [mlp_split(d)][B][mlp_hidden_padded(H1)] <- split-K partial sums of W1 h (fp32; units >= H1 are
+// zero).  Launched with programmatic stream serialization; prefetch: the hidden states and W1 may be
+// read before the preceding kernel finishes (the caller's guarantee, SWITCHSD_PREFETCH_PROBE).
+cudaError_t launch_mlp_tc(const uint16_t *hidden, const uint16_t *W1, float *part, int B, int d, int H1,
+                          bool prefetch, cudaStream_t stream);
 
 }  // namespace switchsd

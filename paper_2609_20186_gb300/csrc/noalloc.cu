@@ -1,12 +1,12 @@
 // noalloc.cu -- switchsd_step_static_workspace: switchsd_step for callers that cannot allocate.
 //
-// switchsd_step with the two-layer probe needs device scratch between its two kernels (the per-tile
-// partial logits), which the caller normally passes in params->workspace.  Some callers cannot hand
+// switchsd_step with the two-layer probe needs device scratch between its two kernels (the first
+// layer's split-K partial sums), which the caller normally passes in params->workspace.  Some callers cannot hand
 // the library device memory at call time: an inference server that gives all of the GPU's memory to
 // its own pool when it starts, or a host program with no CUDA allocator of its own.  This entry point
 // serves them from a fixed array compiled into the library instead, and allocates nothing.
 //
-// The array is a file-scope __device__ variable: every GPU that loads the library holds it (256 KiB)
+// The array is a file-scope __device__ variable: every GPU that loads the library holds it (16 MiB)
 // until the process exits.  Host code cannot use the variable's name as a device address, so the
 // first call on each device asks the runtime for the array's address (cudaGetSymbolAddress) with that
 // device current, and every later call on the device reuses it.
@@ -16,8 +16,8 @@
 
 namespace {
 
-// Two-layer probe scratch: one float per row and 64-unit tile of the hidden layer.
-constexpr size_t kStaticWorkspaceFloats = 65536;
+// Two-layer probe scratch: S x B x H1p floats (switchsd_workspace_bytes).
+constexpr size_t kStaticWorkspaceFloats = size_t(4) << 20;  // 16 MiB
 static __device__ __align__(256) float g_static_workspace[kStaticWorkspaceFloats];
 
 constexpr int kMaxDevices = 64;
@@ -45,7 +45,7 @@ extern "C" int switchsd_step_static_workspace(const int32_t *ctx_tokens, const i
                                               int32_t *out_len, int32_t *out_mode, float *out_score) {
     if (params == nullptr) return SWITCHSD_ERR_ARG;
     const size_t need = switchsd_workspace_bytes(params);
-    if (need > sizeof(g_static_workspace)) return SWITCHSD_ERR_SHAPE;  // B * ceil(H1 / 64) > 65,536
+    if (need > sizeof(g_static_workspace)) return SWITCHSD_ERR_SHAPE;  // S(d) * B * H1p > 4 Mi floats
     switchsd_params p = *params;
     if (need > 0) {
         void *ws = static_workspace_address();

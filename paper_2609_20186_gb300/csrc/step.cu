@@ -31,15 +31,11 @@
 // them in a fixed order, applies the switch and writes the winner's draft.  No global scratch, no
 // atomics, no global re-read of the context.
 #include "common.cuh"
+#include "index.cuh"
 #include "mlp.cuh"
 
 namespace switchsd {
 
-int index_launch(switchsd_index *idx, int32_t *ctx, int32_t *lens, const uint16_t *hidden, const uint16_t *probe_w,
-                 const float *z_pre, int z_tiles, float b2, const int32_t *pv_draft, const int32_t *pv_target,
-                 const int32_t *pv_len, int32_t *out_accept, int32_t *out_draft, int32_t *out_len, int32_t *out_mode,
-                 float *out_score, int32_t *out_match_n, int32_t *out_match_end, int32_t *status, int B, int cap,
-                 int d, int k, int n_min, int n_max, int kappa, float logit_tau, bool stepping, cudaStream_t stream);
 
 constexpr int kStepThreads = 256;
 constexpr int kStepWarps = kStepThreads / kWarp;
@@ -60,8 +56,10 @@ struct StepArgs {
     int32_t *lens;           // read; written when verifying
     const uint16_t *hidden;
     const uint16_t *probe_w;
-    const float *z_pre;      // two-layer probe: per-tile partial logits [z_tiles][B] (workspace), else null
-    int32_t z_tiles;
+    const float *z1_part;    // two-layer probe: split-K partial sums of W1 h [mlp_S][B][H1p] (workspace), else null
+    const float *b1;         // two-layer probe: first-layer biases [H1] (null = zero) and output weights [H1]
+    const uint16_t *w2;
+    int32_t mlp_S, H1, H1p;
     float b2;
     const int32_t *pv_draft; // previous draft [B, k] / target [B, k+1] / draft length [B]; null = no verify
     const int32_t *pv_target;
@@ -114,7 +112,7 @@ __global__ void __launch_bounds__(kStepThreads) step_kernel(const StepArgs a) {
     __shared__ unsigned long long s_wkey[kStepWarps];
     __shared__ float s_wz[kStepWarps];
     __shared__ __align__(16) int32_t s_mine[SWITCHSD_KMAX];    // continuation of this CTA's best match
-    __shared__ __align__(16) uint4 s_pw[kProbeStage], s_ph[kProbeStage];
+    __shared__ __align__(16) uint4 s_probe[2 * kProbeStage];   // linear: w then h slices; two-layer: partial sums
     __shared__ Slot s_slot[kMaxSplit];                         // leader: one message per CTA
     __shared__ int32_t s_out[2];                               // leader: winner rank, draft length
 
@@ -145,27 +143,48 @@ __global__ void __launch_bounds__(kStepThreads) step_kernel(const StepArgs a) {
     const bool pf_ctx = (a.prefetch & SWITCHSD_PREFETCH_CONTEXT) != 0;
     const bool pf_probe = (a.prefetch & SWITCHSD_PREFETCH_PROBE) != 0;
 
-    // This CTA's slice of the linear probe: words [v0, v1) of 8 bf16.  The first kProbeStage of them
-    // are staged by two bulk copies (issued by thread 64) and used after the scan.
-    int v0 = 0, v1 = 0;
-    if (a.z_pre == nullptr) {
+    // Linear probe: this CTA's slice is words [v0, v1) of 8 bf16; the first kProbeStage of them are
+    // staged by two bulk copies (issued by thread 64) and used after the scan.  Two-layer probe: this
+    // CTA finishes units [u0, u1) of the row -- the S split-K partial sums of each unit, staged the
+    // same way when they fit (m_staged), then b1, ReLU and w2.
+    uint4 *s_pw = s_probe, *s_ph = s_probe + kProbeStage;
+    const bool mlp = a.z1_part != nullptr;
+    int v0 = 0, v1 = 0, u0 = 0, u1 = 0, ucnt4 = 0;
+    bool m_staged = false;
+    if (!mlp) {
         const int nv = a.d >> 3;
         const int per = (nv + int(C) - 1) / int(C);
         v0 = min(nv, int(rank) * per);
         v1 = min(nv, v0 + per);
+    } else {
+        const int per = ((a.H1 + int(C) - 1) / int(C) + 3) & ~3;
+        u0 = min(a.H1, int(rank) * per);
+        u1 = min(a.H1, u0 + per);
+        ucnt4 = (u1 - u0 + 3) & ~3;  // units staged per partial (H1p >= u0 + ucnt4: rows are padded to 64)
+        m_staged = a.mlp_S * ucnt4 <= 2 * kProbeStage * 4;
     }
     const int v_staged = min(v1 - v0, kProbeStage);
     const uint4 *h4 = reinterpret_cast<const uint4 *>(a.hidden + size_t(b) * size_t(a.d));
     const uint4 *w4 = reinterpret_cast<const uint4 *>(a.probe_w);
     auto issue_probe = [&]() {
-        const uint32_t pb = uint32_t(v_staged) * 16u;
-        mbar_arrive_expect_tx(&probe_bar, 2u * pb);
-        if (pb > 0) {
-            bulk_g2s(s_pw, w4 + v0, pb, &probe_bar);
-            bulk_g2s(s_ph, h4 + v0, pb, &probe_bar);
+        if (!mlp) {
+            const uint32_t pb = uint32_t(v_staged) * 16u;
+            mbar_arrive_expect_tx(&probe_bar, 2u * pb);
+            if (pb > 0) {
+                bulk_g2s(s_pw, w4 + v0, pb, &probe_bar);
+                bulk_g2s(s_ph, h4 + v0, pb, &probe_bar);
+            }
+        } else {
+            const uint32_t pb = m_staged ? uint32_t(ucnt4) * 4u : 0u;
+            mbar_arrive_expect_tx(&probe_bar, uint32_t(a.mlp_S) * pb);
+            float *dst = reinterpret_cast<float *>(s_probe);
+            if (pb > 0)
+                for (int s = 0; s < a.mlp_S; ++s)
+                    bulk_g2s(dst + s * ucnt4, a.z1_part + (size_t(s) * a.B + size_t(b)) * a.H1p + u0, pb, &probe_bar);
         }
     };
-    if (pf_probe && tid == 2 * kWarp) issue_probe();
+    // The partial sums come from the kernel just before this one: never staged before the wait.
+    if (pf_probe && !mlp && tid == 2 * kWarp) issue_probe();
     if (!pf_ctx) pdl_wait();
 
     // Warp roles until the suffix is known.  Warp 0 reads the row length and issues the copies at
@@ -220,6 +239,11 @@ __global__ void __launch_bounds__(kStepThreads) step_kernel(const StepArgs a) {
     }
     if (pf_ctx) pdl_wait();  // the previous draft and the target (and all that no bit names) come after this
     pdl_trigger();           // the next kernel may start launching
+    float m_b1 = 0.f, m_w2 = 0.f;  // two-layer probe: this thread's first unit, loaded while the copies fly
+    if (mlp && tid < u1 - u0) {
+        m_b1 = a.b1 ? a.b1[u0 + tid] : 0.f;
+        m_w2 = bf16_lo(uint32_t(a.w2[u0 + tid]));
+    }
     if (warp == 0) {
         cluster_arrive_release();
     } else if (warp == 1) {
@@ -262,7 +286,7 @@ __global__ void __launch_bounds__(kStepThreads) step_kernel(const StepArgs a) {
         }
         cluster_arrive_release();
     } else {
-        if (!pf_probe && tid == 2 * kWarp) issue_probe();
+        if ((!pf_probe || mlp) && tid == 2 * kWarp) issue_probe();
         cluster_arrive_relaxed();
     }
     // Warps 0 and 1 meet (named barrier 1, 64 threads): the suffix needs the old tail and the append.
@@ -403,9 +427,25 @@ __global__ void __launch_bounds__(kStepThreads) step_kernel(const StepArgs a) {
     // The probe slice (staged during the scan), then the CTA's partial in a fixed order.
     float zp = 0.f;
     const bool probe_in = mbar_wait(&probe_bar, 0);
-    if (probe_in)
-        for (int i = tid; i < v_staged; i += kStepThreads) zp = dot8_bf16(s_pw[i], s_ph[i], zp);
-    for (int v = v0 + v_staged + tid; v < v1; v += kStepThreads) zp = dot8_bf16(__ldg(w4 + v), __ldg(h4 + v), zp);
+    if (!mlp) {
+        if (probe_in)
+            for (int i = tid; i < v_staged; i += kStepThreads) zp = dot8_bf16(s_pw[i], s_ph[i], zp);
+        for (int v = v0 + v_staged + tid; v < v1; v += kStepThreads)
+            zp = dot8_bf16(__ldg(w4 + v), __ldg(h4 + v), zp);
+    } else {
+        const float *sp = reinterpret_cast<const float *>(s_probe);
+        for (int j = tid; j < u1 - u0; j += kStepThreads) {
+            float z1 = 0.f;  // the S partial sums in order
+            if (m_staged) {
+                for (int s = 0; s < a.mlp_S; ++s) z1 += sp[s * ucnt4 + j];
+            } else {
+                for (int s = 0; s < a.mlp_S; ++s) z1 += a.z1_part[(size_t(s) * a.B + size_t(b)) * a.H1p + u0 + j];
+            }
+            const float bias = j < kStepThreads ? m_b1 : (a.b1 ? a.b1[u0 + j] : 0.f);
+            const float w2 = j < kStepThreads ? m_w2 : bf16_lo(uint32_t(a.w2[u0 + j]));
+            zp = fmaf(w2, fmaxf(z1 + bias, 0.f), zp);
+        }
+    }
     if (!probe_in && tid == 0) {
         best = kTimeoutBit;
         (void)mbar_wait(&probe_bar, 0);  // a second bounded wait before the CTA's memory goes away
@@ -453,12 +493,11 @@ __global__ void __launch_bounds__(kStepThreads) step_kernel(const StepArgs a) {
             k_r = s_slot[lane].key;
             z_r = s_slot[lane].z;
         }
-        if (a.z_pre != nullptr) z_r = lane < a.z_tiles ? a.z_pre[size_t(lane) * a.B + b] : 0.f;
         const unsigned long long key = all_in ? warp_max_u64(k_r) : kTimeoutBit;
         const unsigned at = __ballot_sync(kFull, uint32_t(lane) < C && k_r == key);
         const uint32_t win = at != 0u ? uint32_t(__ffs(at) - 1) : 0u;
         float z = warp_sum_f32(z_r);
-        if (a.z_pre != nullptr) z += a.b2;
+        if (mlp) z += a.b2;
         const bool timeout = (key & kTimeoutBit) != 0;
         const bool hit = len_ok && !timeout && key != 0;
         const int32_t n = hit ? int32_t(key >> 32) : 0;
@@ -560,7 +599,10 @@ static int step_entry(int32_t *ctx_tokens, int32_t *ctx_lens, const uint16_t *hi
     args.lens = ctx_lens;
     args.hidden = hidden;
     args.probe_w = probe_w;
-    args.z_pre = nullptr;
+    args.z1_part = nullptr;
+    args.b1 = nullptr;
+    args.w2 = nullptr;
+    args.mlp_S = args.H1 = args.H1p = 0;
     args.pv_draft = pv_draft;
     args.pv_target = pv_target;
     args.pv_len = pv_len;
@@ -599,21 +641,24 @@ static int step_entry(int32_t *ctx_tokens, int32_t *ctx_lens, const uint16_t *hi
         if (args.stages < 2) args.stages = 2;
     }
 
-    args.z_tiles = 0;
     args.b2 = p->b2;
     if (p->probe_kind == SWITCHSD_PROBE_MLP) {
-        float *zpart = static_cast<float *>(p->workspace);
-        if (launch_mlp_tc(hidden, probe_w, probe_w + size_t(p->probe_hidden) * size_t(p->d), p->b1, zpart, p->B, p->d,
-                          p->probe_hidden, stream) != cudaSuccess)
+        float *part = static_cast<float *>(p->workspace);
+        if (launch_mlp_tc(hidden, probe_w, part, p->B, p->d, p->probe_hidden,
+                          (p->prefetch & SWITCHSD_PREFETCH_PROBE) != 0, stream) != cudaSuccess)
             return SWITCHSD_ERR_CUDA;
-        args.z_pre = zpart;
-        args.z_tiles = mlp_tiles_n(p->probe_hidden);
+        args.z1_part = part;
+        args.b1 = p->b1;
+        args.w2 = probe_w + size_t(p->probe_hidden) * size_t(p->d);
+        args.mlp_S = mlp_split(p->d);
+        args.H1 = p->probe_hidden;
+        args.H1p = mlp_hidden_padded(p->probe_hidden);
     }
     if (p->index != nullptr)
-        return index_launch(p->index, ctx_tokens, ctx_lens, hidden, probe_w, args.z_pre, args.z_tiles, args.b2, pv_draft,
-                            pv_target, pv_len, out_accept, out_draft, out_len, out_mode, out_score, p->out_match_n,
-                            p->out_match_end, p->status, p->B, p->cap, p->d, p->k, p->n_min, p->n_max, p->kappa,
-                            p->logit_tau, true, stream);
+        return index_launch(p->index, ctx_tokens, ctx_lens, hidden, probe_w, args.z1_part, args.b1, args.w2, args.mlp_S,
+                            args.H1, args.H1p, args.b2, pv_draft, pv_target, pv_len, out_accept, out_draft, out_len,
+                            out_mode, out_score, p->out_match_n, p->out_match_end, p->status, p->B, p->cap, p->d, p->k,
+                            p->n_min, p->n_max, p->kappa, p->logit_tau, true, stream);
     if (launch_step(args, split, stream) != cudaSuccess) return SWITCHSD_ERR_CUDA;
     return SWITCHSD_OK;
 }
@@ -624,8 +669,10 @@ using namespace switchsd;
 
 extern "C" size_t switchsd_workspace_bytes(const switchsd_params *p) {
     if (!p || p->probe_kind != SWITCHSD_PROBE_MLP || p->B < 1) return 0;
-    const int tiles = mlp_tiles_n(p->probe_hidden < 1 ? 1 : p->probe_hidden);
-    return (size_t(tiles) * size_t(p->B) * sizeof(float) + 255) / 256 * 256;
+    const int H1 = p->probe_hidden < 1 ? 1 : p->probe_hidden;
+    const int d = p->d < 8 ? 8 : p->d;
+    const size_t floats = size_t(mlp_split(d)) * size_t(p->B) * size_t(mlp_hidden_padded(H1));
+    return (floats * sizeof(float) + 255) / 256 * 256;
 }
 
 extern "C" int switchsd_step(const int32_t *ctx_tokens, const int32_t *ctx_lens, const uint16_t *hidden,

@@ -6,17 +6,10 @@
 // draft[0..a) and target[a] at ctx[L..L+a] and lane 0 publishes L + a + 1.  The work is O(B k)
 // bytes: latency-bound by design.
 #include "common.cuh"
+#include "index.cuh"
 
 namespace switchsd {
 
-int index_launch(switchsd_index *idx, int32_t *ctx, int32_t *lens, const uint16_t *hidden, const uint16_t *probe_w,
-                 const float *z_pre, int z_tiles, float b2, const int32_t *pv_draft, const int32_t *pv_target,
-                 const int32_t *pv_len, int32_t *out_accept, int32_t *out_draft, int32_t *out_len, int32_t *out_mode,
-                 float *out_score, int32_t *out_match_n, int32_t *out_match_end, int32_t *status, int B, int cap,
-                 int d, int k, int n_min, int n_max, int kappa, float logit_tau, bool stepping, cudaStream_t stream);
-
-int index_n_min(const switchsd_index *idx);
-int index_n_max(const switchsd_index *idx);
 
 constexpr int kVerifyThreads = 256;
 
@@ -86,7 +79,8 @@ extern "C" int switchsd_verify(const int32_t *draft, const int32_t *target_argma
         return SWITCHSD_ERR_SHAPE;
     if (vp->index != nullptr) {
         // verification with insertion of the appended positions into the index (no step)
-        return index_launch(vp->index, vp->ctx_tokens, vp->ctx_lens, nullptr, nullptr, nullptr, 0, 0.f, draft,
+        return index_launch(vp->index, vp->ctx_tokens, vp->ctx_lens, nullptr, nullptr, nullptr, nullptr, nullptr, 0,
+                            0, 0, 0.f, draft,
                             target_argmax, vp->draft_len, out_accept, nullptr, nullptr, nullptr, nullptr, nullptr,
                             nullptr, vp->status, vp->B, vp->cap, 8, vp->k, index_n_min(vp->index),
                             index_n_max(vp->index), 0, 0.f, false, static_cast<cudaStream_t>(vp->stream));

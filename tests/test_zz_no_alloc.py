@@ -69,7 +69,7 @@ def test_static_workspace_matches_caller_workspace():
 
     lib = bd.load()
     B, d, H1, cap, k = 300, 4096, 200, 640, 8
-    ws = torch.empty(bd.switchsd_workspace_bytes(B, bd.PROBE_MLP, H1), dtype=torch.uint8, device="cuda")
+    ws = torch.empty(bd.switchsd_workspace_bytes(B, bd.PROBE_MLP, H1, d), dtype=torch.uint8, device="cuda")
     for seed in (11, 12):                       # two calls in a row on the shared static array
         prob = _problem(seed, B, d, H1, cap, k)
         ref = _run(lib, "switchsd_step", prob, B, d, H1, k, workspace=ws)
@@ -89,7 +89,7 @@ def test_static_workspace_rejects_requests_beyond_its_size():
     lib = bd.load()
     p = bd.switchsd_params()
     p.B, p.cap, p.d, p.k, p.n_min, p.n_max = 16385, 64, 4096, 8, 2, 6
-    p.probe_kind, p.probe_hidden = bd.PROBE_MLP, 256       # 16,385 rows x 4 tiles > 65,536
+    p.probe_kind, p.probe_hidden = bd.PROBE_MLP, 256       # 16 x 16,385 rows x 256 units > 4 Mi floats
     fake = 0x10000
     code = lib.switchsd_step_static_workspace(fake, fake, fake, fake, ctypes.byref(p), fake, fake, fake,
                                               fake)
