@@ -365,6 +365,7 @@ class ReplicaLoop:
         hp.B, hp.k, hp.V, hp.L0 = N, k, h["V"], h["L0"]
         hp.n_future = self.future.shape[1]
         hp.gamma, hp.step, hp.seed, hp.thr_neural = h["gamma"], 0, h["seed"], h["thr_neural"]
+        hp.p_hit, hp.p_miss, hp.q_neural = h["p_hit"], h["p_miss"], h["q_neural"]
         hp.stream = sp
         self.hp = hp
         e32, e16 = 4, 2

@@ -201,6 +201,31 @@ int switchsd_verify(const int32_t *draft, const int32_t *target_argmax, int32_t 
                     const switchsd_verify_params *vp);
 
 /*
+ * Verification and append at temperature T > 0 (App. A runs SwitchSD with sampling; the acceptance
+ * rule is the speculative-sampling rule of the works §2 builds on).  Draft token i is accepted iff
+ * u[i] * q[i] < p[i], the product rounded to binary32 and compared in binary32: the event
+ * u < min(1, p / q) for u uniform in [0, 1).  A copy draft is deterministic (q = 1), so a copied token
+ * is accepted with the target's probability of it.
+ *
+ *   draft      int32 [B, k]: the draft that was verified (copy or neural)
+ *   p_draft    float [B, k]: the target's probability of draft[i] at its position
+ *   q_draft    float [B, k]: the drafter's probability of draft[i], or NULL when every row holds a copy
+ *              draft (q = 1); a copy row among neural rows passes 1.0 entries
+ *   u          float [B, k]: uniform draws in [0, 1), one per draft position (the caller's random numbers)
+ *   resample   int32 [B, k+1]: entry a is the token appended after a acceptances: for a < len the
+ *              caller's draw from the residual distribution max(0, p - q) renormalised at that position,
+ *              for a = len its draw from the target after the full draft
+ *   out_accept int32 [B]: a, the accepted length
+ *
+ * The row's context receives draft[0..a) then resample[a]; ctx_lens grows by a+1; capacity, status and
+ * bad lengths as switchsd_verify.  With p one-hot (T -> 0) and resample = the argmax this is
+ * switchsd_verify.  vp->index must be NULL (SWITCHSD_ERR_ARG otherwise): the index keeps to the greedy
+ * verification.
+ */
+int switchsd_verify_sampled(const int32_t *draft, const float *p_draft, const float *q_draft, const float *u,
+                            const int32_t *resample, int32_t *out_accept, const switchsd_verify_params *vp);
+
+/*
  * One controller iteration in one launch (§3.3 "Overall Framework": after every verification step the
  * controller decides the next draft, Fig. 1): greedy verification and append of the previous draft,
  * exactly as switchsd_verify, then switchsd_step on the extended context.  The result equals

@@ -40,11 +40,28 @@ typedef struct {
     uint64_t seed;
     uint64_t thr_neural; /* threshold on a 32-bit word; 1 << 32 means always */
     void *stream;
+    float p_hit, p_miss; /* sampled: target probability of a draft token equal to / different from the stream */
+    float q_neural;      /* sampled: the neural drafter's probability of its token (copy drafts: 1) */
 } switchsd_harness_params;
 
 int switchsd_harness_target(const int32_t *ctx_lens, const int32_t *mode, const int32_t *draft,
                             const int32_t *draft_len, const int32_t *future, int32_t *vdraft,
                             int32_t *vlen, int32_t *target, const switchsd_harness_params *hp);
+
+/*
+ * The stand-in at temperature T > 0, feeding switchsd_verify_sampled.  vdraft / vlen as above; with
+ * g[i] = future[L - L0 + i] and key(slot) = the harness key of (seed, row, step, slot):
+ *   p[b][i]        p_hit if vdraft[i] == g[i] else p_miss (i < vlen; 0 beyond)
+ *   q[b][i]        1 for a copy row, q_neural for a neural row (i < vlen; 1 beyond)
+ *   u[b][i]        (key(4 i + 2) >> 40) * 2^-24, for every i < k (exact in binary32)
+ *   resample[b][i] i < vlen: g[i], or when g[i] == vdraft[i] the token (key(4 i + 3) >> 32) mod V (plus
+ *                  one mod V if that equals vdraft[i]) -- the residual excludes the rejected token;
+ *                  i = vlen: g[vlen] (the bonus draw); 0 beyond.
+ * p, q, u are float [B, k]; resample int32 [B, k+1].
+ */
+int switchsd_harness_sampled(const int32_t *ctx_lens, const int32_t *mode, const int32_t *draft,
+                             const int32_t *draft_len, const int32_t *future, int32_t *vdraft, int32_t *vlen,
+                             float *p, float *q, float *u, int32_t *resample, const switchsd_harness_params *hp);
 
 #ifdef __cplusplus
 }

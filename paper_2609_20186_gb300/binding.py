@@ -57,6 +57,7 @@ class switchsd_harness_params(ctypes.Structure):
         ("n_future", ctypes.c_int32), ("gamma", ctypes.c_int32), ("step", ctypes.c_int32),
         ("seed", ctypes.c_uint64), ("thr_neural", ctypes.c_uint64),
         ("stream", ctypes.c_void_p),
+        ("p_hit", ctypes.c_float), ("p_miss", ctypes.c_float), ("q_neural", ctypes.c_float),
     ]
 
 
@@ -69,6 +70,8 @@ _SIGNATURES = {
                       + [ctypes.c_void_p] * 4),
     "switchsd_verify": (ctypes.c_int, [ctypes.c_void_p] * 3
                         + [ctypes.POINTER(switchsd_verify_params)]),
+    "switchsd_verify_sampled": (ctypes.c_int, [ctypes.c_void_p] * 6
+                                + [ctypes.POINTER(switchsd_verify_params)]),
     "switchsd_verify_step": (ctypes.c_int, [ctypes.c_void_p] * 8 + [ctypes.POINTER(switchsd_params)]
                              + [ctypes.c_void_p] * 4),
     "switchsd_step_static_workspace": (ctypes.c_int, [ctypes.c_void_p] * 4
@@ -83,6 +86,8 @@ _SIGNATURES = {
     "switchsd_abi_version": (ctypes.c_int, []),
     "switchsd_harness_target": (ctypes.c_int, [ctypes.c_void_p] * 8
                                 + [ctypes.POINTER(switchsd_harness_params)]),
+    "switchsd_harness_sampled": (ctypes.c_int, [ctypes.c_void_p] * 11
+                                 + [ctypes.POINTER(switchsd_harness_params)]),
 }
 
 
@@ -292,6 +297,27 @@ def switchsd_verify(draft, target_argmax, out_accept, *, draft_len, ctx_tokens, 
     _check(code, "switchsd_verify")
 
 
+def switchsd_verify_sampled(draft, p_draft, u, resample, out_accept, *, draft_len, ctx_tokens, ctx_lens,
+                            q_draft=None, status=None, stream=None) -> None:
+    """switchsd_verify_sampled of include/switchsd.h on torch tensors: draft int32 [B, k], p_draft /
+    q_draft (None: copy drafts) / u float32 [B, k], resample int32 [B, k + 1]."""
+    B, cap = ctx_tokens.shape
+    k = draft.shape[1]
+    vp = switchsd_verify_params()
+    vp.B, vp.cap, vp.k = B, cap, k
+    vp.draft_len = _dev(draft_len, torch.int32, "draft_len", (B,))
+    vp.ctx_tokens = _dev(ctx_tokens, torch.int32, "ctx_tokens")
+    vp.ctx_lens = _dev(ctx_lens, torch.int32, "ctx_lens", (B,))
+    vp.status = _dev(status, torch.int32, "status", (B,))
+    vp.stream = _stream_ptr(stream)
+    code = load().switchsd_verify_sampled(
+        _dev(draft, torch.int32, "draft", (B, k)), _dev(p_draft, torch.float32, "p_draft", (B, k)),
+        _dev(q_draft, torch.float32, "q_draft", (B, k)), _dev(u, torch.float32, "u", (B, k)),
+        _dev(resample, torch.int32, "resample", (B, k + 1)), _dev(out_accept, torch.int32, "out_accept", (B,)),
+        ctypes.byref(vp))
+    _check(code, "switchsd_verify_sampled")
+
+
 def switchsd_harness_target(ctx_lens, mode, draft, draft_len, future, vdraft, vlen, target, *,
                             seed: int, V: int, L0: int, gamma: int, thr_neural: int, step: int,
                             stream=None) -> None:
@@ -310,3 +336,25 @@ def switchsd_harness_target(ctx_lens, mode, draft, draft_len, future, vdraft, vl
         _dev(vlen, torch.int32, "vlen", (B,)), _dev(target, torch.int32, "target", (B, k + 1)),
         ctypes.byref(hp))
     _check(code, "switchsd_harness_target")
+
+
+def switchsd_harness_sampled(ctx_lens, mode, draft, draft_len, future, vdraft, vlen, p, q, u, resample, *,
+                             seed: int, V: int, L0: int, gamma: int, thr_neural: int, step: int,
+                             p_hit: float, p_miss: float, q_neural: float, stream=None) -> None:
+    """switchsd_harness_sampled of include/switchsd_harness.h (the stand-in at T > 0)."""
+    B, k = draft.shape
+    hp = switchsd_harness_params()
+    hp.B, hp.k, hp.V, hp.L0 = B, k, V, L0
+    hp.n_future = future.shape[1]
+    hp.gamma, hp.step = gamma, step
+    hp.seed, hp.thr_neural = seed, thr_neural
+    hp.p_hit, hp.p_miss, hp.q_neural = p_hit, p_miss, q_neural
+    hp.stream = _stream_ptr(stream)
+    code = load().switchsd_harness_sampled(
+        _dev(ctx_lens, torch.int32, "ctx_lens", (B,)), _dev(mode, torch.int32, "mode", (B,)),
+        _dev(draft, torch.int32, "draft", (B, k)), _dev(draft_len, torch.int32, "draft_len", (B,)),
+        _dev(future, torch.int32, "future"), _dev(vdraft, torch.int32, "vdraft", (B, k)),
+        _dev(vlen, torch.int32, "vlen", (B,)), _dev(p, torch.float32, "p", (B, k)),
+        _dev(q, torch.float32, "q", (B, k)), _dev(u, torch.float32, "u", (B, k)),
+        _dev(resample, torch.int32, "resample", (B, k + 1)), ctypes.byref(hp))
+    _check(code, "switchsd_harness_sampled")

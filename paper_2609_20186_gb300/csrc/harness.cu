@@ -12,7 +12,8 @@ constexpr int kHarnessThreads = 256;
 
 struct HarnessArgs {
     const int32_t *lens, *mode, *draft, *draft_len, *future;
-    int32_t *vdraft, *vlen, *target;
+    int32_t *vdraft, *vlen, *target;  // target: the greedy tokens, or (sampled) the resample tokens
+    float *pp, *qq, *uu;              // sampled only
     switchsd_harness_params p;
 };
 
@@ -28,6 +29,7 @@ __device__ __forceinline__ int32_t token_of(uint64_t r, int32_t V) {
     return int32_t((r >> 32) % uint64_t(V));
 }
 
+template <bool kSampled>
 __global__ void __launch_bounds__(kHarnessThreads) harness_kernel(const HarnessArgs a) {
     const int lane = threadIdx.x & 31;
     const int b = (blockIdx.x * kHarnessThreads + threadIdx.x) >> 5;
@@ -44,7 +46,7 @@ __global__ void __launch_bounds__(kHarnessThreads) harness_kernel(const HarnessA
     for (int i = lane; i <= k; i += kWarp) {
         const int64_t pos = int64_t(L) - p.L0 + i;
         const int32_t g = (pos >= 0 && pos < p.n_future) ? a.future[size_t(b) * p.n_future + pos] : 0;
-        a.target[size_t(b) * (k + 1) + i] = g;
+        if (!kSampled) a.target[size_t(b) * (k + 1) + i] = g;
         if (i < k) {
             int32_t d = 0;
             if (i < len) {
@@ -62,7 +64,24 @@ __global__ void __launch_bounds__(kHarnessThreads) harness_kernel(const HarnessA
                 }
             }
             a.vdraft[size_t(b) * k + i] = d;
+            if (kSampled) {
+                const size_t o = size_t(b) * k + i;
+                const uint64_t slot = 4ull * uint64_t(i);
+                a.pp[o] = i < len ? (d == g ? p.p_hit : p.p_miss) : 0.f;
+                a.qq[o] = (i < len && !copy) ? p.q_neural : 1.f;
+                a.uu[o] = float(uint32_t(splitmix64(row_key ^ (slot + 2)) >> 40)) * 5.9604644775390625e-8f;  // 2^-24
+                int32_t r = 0;
+                if (i < len) {
+                    r = g;
+                    if (g == d) {
+                        r = token_of(splitmix64(row_key ^ (slot + 3)), p.V);
+                        if (r == d) r = (r + 1) % p.V;
+                    }
+                }
+                a.target[size_t(b) * (k + 1) + i] = r;
+            }
         }
+        if (kSampled && i >= len) a.target[size_t(b) * (k + 1) + i] = i == len ? g : 0;
     }
     if (lane == 0) a.vlen[b] = len;
 }
@@ -88,9 +107,39 @@ extern "C" int switchsd_harness_target(const int32_t *ctx_lens, const int32_t *m
     a.vdraft = vdraft;
     a.vlen = vlen;
     a.target = target;
+    a.pp = a.qq = a.uu = nullptr;
     a.p = *hp;
     const int wpb = kHarnessThreads / kWarp;
-    const cudaError_t e = launch_pdl(harness_kernel, dim3((hp->B + wpb - 1) / wpb), dim3(kHarnessThreads), 0,
-                                     static_cast<cudaStream_t>(hp->stream), 0u, a);
+    const cudaError_t e = launch_pdl(harness_kernel<false>, dim3((hp->B + wpb - 1) / wpb), dim3(kHarnessThreads),
+                                     0, static_cast<cudaStream_t>(hp->stream), 0u, a);
+    return e == cudaSuccess ? SWITCHSD_OK : SWITCHSD_ERR_CUDA;
+}
+
+extern "C" int switchsd_harness_sampled(const int32_t *ctx_lens, const int32_t *mode, const int32_t *draft,
+                                        const int32_t *draft_len, const int32_t *future, int32_t *vdraft,
+                                        int32_t *vlen, float *p, float *q, float *u, int32_t *resample,
+                                        const switchsd_harness_params *hp) {
+    if (!hp || !ctx_lens || !mode || !draft || !draft_len || !vdraft || !vlen || !p || !q || !u || !resample)
+        return SWITCHSD_ERR_ARG;
+    if (hp->n_future > 0 && !future) return SWITCHSD_ERR_ARG;
+    if (hp->B < 1 || hp->k < 1 || hp->k > SWITCHSD_KMAX || hp->V < 2 || hp->n_future < 0 || hp->gamma < 0 ||
+        hp->gamma > hp->k)
+        return SWITCHSD_ERR_SHAPE;
+    HarnessArgs a;
+    a.lens = ctx_lens;
+    a.mode = mode;
+    a.draft = draft;
+    a.draft_len = draft_len;
+    a.future = future;
+    a.vdraft = vdraft;
+    a.vlen = vlen;
+    a.target = resample;
+    a.pp = p;
+    a.qq = q;
+    a.uu = u;
+    a.p = *hp;
+    const int wpb = kHarnessThreads / kWarp;
+    const cudaError_t e = launch_pdl(harness_kernel<true>, dim3((hp->B + wpb - 1) / wpb), dim3(kHarnessThreads),
+                                     0, static_cast<cudaStream_t>(hp->stream), 0u, a);
     return e == cudaSuccess ? SWITCHSD_OK : SWITCHSD_ERR_CUDA;
 }

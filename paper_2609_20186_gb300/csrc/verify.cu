@@ -1,10 +1,13 @@
 // verify.cu -- switchsd_verify: greedy verification and append (§3.3 "Parallel Verification",
-// temperature 0 as in App. A).
+// temperature 0 as in the main experiments), and switchsd_verify_sampled: the same at temperature
+// T > 0 (App. A) with the speculative-sampling acceptance rule.
 //
-// One warp per row.  Lanes compare draft[i] with the target's greedy token 32 indices at a time; the
-// first set bit of the ballot of mismatches is the accepted length a.  Lanes then append
-// draft[0..a) and target[a] at ctx[L..L+a] and lane 0 publishes L + a + 1.  The work is O(B k)
-// bytes: latency-bound by design.
+// One warp per row.  Lanes test 32 draft indices at a time -- greedy: draft[i] differs from the
+// target's greedy token; sampled: u[i] * q[i] is not below p[i] (the product rounded to binary32, q = 1
+// for a copy draft) -- and the first set bit of the ballot of rejections is the accepted length a.
+// Lanes then append draft[0..a) and the target's token at a (greedy: its argmax; sampled: the caller's
+// residual or bonus draw) at ctx[L..L+a] and lane 0 publishes L + a + 1.  The work is O(B k) bytes:
+// latency-bound by design.
 #include "common.cuh"
 #include "index.cuh"
 
@@ -15,7 +18,8 @@ constexpr int kVerifyThreads = 256;
 
 struct VerifyArgs {
     const int32_t *draft;
-    const int32_t *target;
+    const int32_t *target;   // greedy: target argmax [B, k+1]; sampled: the residual / bonus draws [B, k+1]
+    const float *p, *q, *u;  // sampled only: target and drafter probabilities (q null: 1) and uniforms [B, k]
     const int32_t *draft_len;
     int32_t *ctx;
     int32_t *lens;
@@ -24,6 +28,7 @@ struct VerifyArgs {
     int32_t B, cap, k;
 };
 
+template <bool kSampled>
 __global__ void __launch_bounds__(kVerifyThreads) verify_kernel(const VerifyArgs a) {
     const int lane = threadIdx.x & 31;
     const int b = (blockIdx.x * kVerifyThreads + threadIdx.x) >> 5;
@@ -44,7 +49,16 @@ __global__ void __launch_bounds__(kVerifyThreads) verify_kernel(const VerifyArgs
     int32_t acc = len;
     for (int base = 0; base < len; base += kWarp) {
         const int i = base + lane;
-        const bool mismatch = i < len && dr[i] != tg[i];
+        bool mismatch = false;
+        if (i < len) {
+            if constexpr (kSampled) {
+                const size_t o = size_t(b) * a.k + i;
+                const float q = a.q ? a.q[o] : 1.f;
+                mismatch = !(__fmul_rn(a.u[o], q) < a.p[o]);
+            } else {
+                mismatch = dr[i] != tg[i];
+            }
+        }
         const unsigned m = __ballot_sync(kFull, mismatch);
         if (m) {
             acc = base + __ffs(m) - 1;
@@ -88,6 +102,7 @@ extern "C" int switchsd_verify(const int32_t *draft, const int32_t *target_argma
     VerifyArgs a;
     a.draft = draft;
     a.target = target_argmax;
+    a.p = a.q = a.u = nullptr;
     a.draft_len = vp->draft_len;
     a.ctx = vp->ctx_tokens;
     a.lens = vp->ctx_lens;
@@ -98,7 +113,37 @@ extern "C" int switchsd_verify(const int32_t *draft, const int32_t *target_argma
     a.k = vp->k;
     const int warps_per_block = kVerifyThreads / kWarp;
     const int blocks = (vp->B + warps_per_block - 1) / warps_per_block;
-    const cudaError_t e = launch_pdl(verify_kernel, dim3(blocks), dim3(kVerifyThreads), 0,
+    const cudaError_t e = launch_pdl(verify_kernel<false>, dim3(blocks), dim3(kVerifyThreads), 0,
+                                     static_cast<cudaStream_t>(vp->stream), 0u, a);
+    return e == cudaSuccess ? SWITCHSD_OK : SWITCHSD_ERR_CUDA;
+}
+
+extern "C" int switchsd_verify_sampled(const int32_t *draft, const float *p_draft, const float *q_draft,
+                                       const float *u, const int32_t *resample, int32_t *out_accept,
+                                       const switchsd_verify_params *vp) {
+    if (!vp || !draft || !p_draft || !u || !resample || !out_accept || !vp->draft_len || !vp->ctx_tokens ||
+        !vp->ctx_lens)
+        return SWITCHSD_ERR_ARG;
+    if (vp->index != nullptr) return SWITCHSD_ERR_ARG;  // the index keeps to the greedy verification
+    if (vp->B < 1 || vp->cap < 4 || (vp->cap & 3) != 0 || vp->k < 1 || vp->k > SWITCHSD_KMAX)
+        return SWITCHSD_ERR_SHAPE;
+    VerifyArgs a;
+    a.draft = draft;
+    a.target = resample;
+    a.p = p_draft;
+    a.q = q_draft;
+    a.u = u;
+    a.draft_len = vp->draft_len;
+    a.ctx = vp->ctx_tokens;
+    a.lens = vp->ctx_lens;
+    a.out_accept = out_accept;
+    a.status = vp->status;
+    a.B = vp->B;
+    a.cap = vp->cap;
+    a.k = vp->k;
+    const int warps_per_block = kVerifyThreads / kWarp;
+    const int blocks = (vp->B + warps_per_block - 1) / warps_per_block;
+    const cudaError_t e = launch_pdl(verify_kernel<true>, dim3(blocks), dim3(kVerifyThreads), 0,
                                      static_cast<cudaStream_t>(vp->stream), 0u, a);
     return e == cudaSuccess ? SWITCHSD_OK : SWITCHSD_ERR_CUDA;
 }

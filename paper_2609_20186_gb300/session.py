@@ -122,6 +122,9 @@ class Session:
             hp.n_future = self.future.shape[1]
             hp.gamma, hp.step = harness["gamma"], 0
             hp.seed, hp.thr_neural = harness["seed"], harness["thr_neural"]
+            hp.p_hit = harness.get("p_hit", 0.9)
+            hp.p_miss = harness.get("p_miss", 0.05)
+            hp.q_neural = harness.get("q_neural", 0.8)
             hp.stream = sp
             self._hp = hp
             self._harness_args = (self.lens.data_ptr(), self.mode.data_ptr(), self.draft.data_ptr(),
@@ -129,6 +132,12 @@ class Session:
                                   self.future.data_ptr() if self.future.numel() else None,
                                   self.vdraft.data_ptr(), self.vlen.data_ptr(),
                                   self.target.data_ptr())
+        # sampled verification (T > 0): target / drafter probabilities and uniforms of the last draft;
+        # self.target then holds the residual and bonus draws
+        f32 = dict(dtype=torch.float32, device=dev)
+        self.vp = torch.zeros(B, k, **f32)
+        self.vq = torch.ones(B, k, **f32)
+        self.vu = torch.zeros(B, k, **f32)
 
     # --- the three calls ---------------------------------------------------------------------
     def _check_hidden(self, hidden: torch.Tensor) -> None:
@@ -169,6 +178,24 @@ class Session:
                                         ctypes.byref(self._vp_dbg if debug else self._vp_fast))
         if code != bd.OK:
             raise RuntimeError(f"switchsd_verify failed: {code} ({bd.strerror(code)})")
+
+    def harness_sampled(self, t: int) -> None:
+        """The target stand-in at T > 0: vdraft / vlen, vp / vq / vu and the resample tokens in target."""
+        self._hp.step = t
+        a = self._harness_args
+        code = self.lib.switchsd_harness_sampled(*a[:7], self.vp.data_ptr(), self.vq.data_ptr(),
+                                                 self.vu.data_ptr(), a[7], ctypes.byref(self._hp))
+        if code != bd.OK:
+            raise RuntimeError(f"switchsd_harness_sampled failed: {code} ({bd.strerror(code)})")
+
+    def verify_sampled(self, debug: bool = True) -> None:
+        """switchsd_verify_sampled of the last harness draft (no index)."""
+        vp = self._vp_dbg if debug else self._vp_fast
+        code = self.lib.switchsd_verify_sampled(self.vdraft.data_ptr(), self.vp.data_ptr(), self.vq.data_ptr(),
+                                                self.vu.data_ptr(), self.target.data_ptr(), self.accept.data_ptr(),
+                                                ctypes.byref(vp))
+        if code != bd.OK:
+            raise RuntimeError(f"switchsd_verify_sampled failed: {code} ({bd.strerror(code)})")
 
     def iterate(self, hidden: torch.Tensor, t: int, debug: bool = True) -> None:
         self.step(hidden, debug)

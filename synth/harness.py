@@ -12,7 +12,8 @@ occasional edits).  Then, for a row of current length L:
   with probability ``p_neural`` (a seeded coin), else a seeded token different from it.
 
 Randomness comes from ``harness_key(seed, row, step, 4 * i + slot)`` (slot 0: the neural coin, low
-32 bits; slot 1: the replacement token, a token being (word >> 32) mod V).  The CUDA harness kernel
+32 bits; slot 1: the replacement token, a token being (word >> 32) mod V; slots 2 and 3 feed the
+sampled stand-in below).  The CUDA harness kernel
 implements the same chain, so both sides produce identical drafts and targets for identical inputs.
 No controller arithmetic happens here.
 """
@@ -66,3 +67,45 @@ def harness_targets(params: dict, step: int, ctx_lens: np.ndarray, mode: np.ndar
             vdraft[b, :ln] = np.where(coin < thr, gg, alt).astype(np.int32)
         vlen[b] = ln
     return vdraft, vlen, target
+
+
+def harness_sampled(params: dict, step: int, ctx_lens: np.ndarray, mode: np.ndarray,
+                    draft: np.ndarray, draft_len: np.ndarray, future: np.ndarray, rows=None):
+    """The stand-in at temperature T > 0 (the inputs of the sampled verification).  Returns
+    (vdraft [B, k], vlen [B], p [B, k], q [B, k], u [B, k], resample [B, k+1]); with g = the target
+    stream at the draft positions:
+
+    - p[i] = p_hit where vdraft[i] == g[i], else p_miss (i < vlen; 0 beyond);
+    - q[i] = 1 for a copy row, q_neural for a neural row (i < vlen; 1 beyond);
+    - u[i] = (key(4 i + 2) >> 40) * 2^-24 for every i < k (exact in binary32);
+    - resample[i] = g[i] for i < vlen, except where g[i] == vdraft[i]: then the token of key(4 i + 3),
+      plus one mod V if that equals vdraft[i] (the residual excludes the rejected token);
+      resample[vlen] = g[vlen]; 0 beyond.
+    """
+    B, k = draft.shape
+    V = params["V"]
+    seed = params["seed"]
+    p_hit, p_miss = np.float32(params["p_hit"]), np.float32(params["p_miss"])
+    q_neural = np.float32(params["q_neural"])
+    vdraft, vlen, g = harness_targets(params, step, ctx_lens, mode, draft, draft_len, future, rows)
+    p = np.zeros((B, k), np.float32)
+    q = np.ones((B, k), np.float32)
+    u = np.zeros((B, k), np.float32)
+    resample = np.zeros((B, k + 1), np.int32)
+    idx = range(B) if rows is None else rows
+    slots = 4 * np.arange(k, dtype=np.uint64)
+    for b in idx:
+        b = int(b)
+        ln = int(vlen[b])
+        d = vdraft[b, :ln].astype(np.int64)
+        gg = g[b, :ln].astype(np.int64)
+        p[b, :ln] = np.where(d == gg, p_hit, p_miss)
+        if int(mode[b]) != MODE_COPY:
+            q[b, :ln] = q_neural
+        word = harness_key(seed, b, step, slots + np.uint64(2))
+        u[b] = ((word >> np.uint64(40)).astype(np.float64) * 2.0 ** -24).astype(np.float32)
+        alt = _token(harness_key(seed, b, step, slots[:ln] + np.uint64(3)), V)
+        alt = np.where(alt == d, (alt + 1) % V, alt)
+        resample[b, :ln] = np.where(gg == d, alt, gg).astype(np.int32)
+        resample[b, ln] = g[b, ln]
+    return vdraft, vlen, p, q, u, resample

@@ -65,6 +65,9 @@ class Workload:
     p_in: float = 0.9              # per-token survival of a planted future copy (else an edit)
     p_neural: float = 0.75         # per-token agreement of the neural draft with the target
     gamma: int = 6                 # neural draft length (the drafter's lookahead, Table 3)
+    p_hit: float = 0.9             # sampled stand-in: target probability of a draft token on the stream
+    p_miss: float = 0.05           # ... and of one off it (the configs' "p=0.9 inside / 0.05 outside")
+    q_neural: float = 0.8          # ... the neural drafter's probability of its own token
     variant: str = ""              # planted workload: copy | nocopy | norep
 
     @property
@@ -164,6 +167,9 @@ class Workload:
             "L0": self.L0,
             "gamma": min(self.gamma, self.k),
             "thr_neural": _prob_to_thr(self.p_neural),
+            "p_hit": self.p_hit,
+            "p_miss": self.p_miss,
+            "q_neural": self.q_neural,
         }
 
     def expected_planted(self) -> dict:

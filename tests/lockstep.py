@@ -18,9 +18,9 @@ import synth
 SCORE_TOL = 1e-3
 
 
-def oracle_trace(wl: synth.Workload, rows, steps: int, ctx=None, lens=None):
+def oracle_trace(wl: synth.Workload, rows, steps: int, ctx=None, lens=None, sampled: bool = False):
     """Runs the oracle loop on the given rows; returns a list (per step) of dicts of per-row arrays
-    plus the final ctx / lens."""
+    plus the final ctx / lens.  sampled: verification at T > 0 with the sampled stand-in."""
     if ctx is None:
         ctx, lens = wl.contexts()
     ctx = ctx.copy()
@@ -42,12 +42,19 @@ def oracle_trace(wl: synth.Workload, rows, steps: int, ctx=None, lens=None):
             else:
                 for key in out:
                     out[key][b] = o[key][b]
-        vd, vl, tg = synth.harness_targets(hp, t, lens, out["mode"], out["draft"], out["len"],
-                                           future, rows=rows)
+        if sampled:
+            vd, vl, pp, qq, uu, rs = synth.harness_sampled(hp, t, lens, out["mode"], out["draft"],
+                                                           out["len"], future, rows=rows)
+        else:
+            vd, vl, tg = synth.harness_targets(hp, t, lens, out["mode"], out["draft"], out["len"],
+                                               future, rows=rows)
         acc = np.zeros(wl.B, np.int32)
         st = np.zeros(wl.B, np.int32)
         for b in rows:
-            a, s = oracle.verify(ctx, lens, vd, vl, tg, rows=(b, b + 1))
+            if sampled:
+                a, s = oracle.verify_sampled(ctx, lens, vd, vl, pp, uu, rs, q=qq, rows=(b, b + 1))
+            else:
+                a, s = oracle.verify(ctx, lens, vd, vl, tg, rows=(b, b + 1))
             acc[b], st[b] = a[b], s[b]
         out["accept"] = acc
         out["vstatus"] = st
@@ -57,12 +64,14 @@ def oracle_trace(wl: synth.Workload, rows, steps: int, ctx=None, lens=None):
 
 
 def gpu_trace(wl: synth.Workload, steps: int, split: int = 0, ctx=None, lens=None, device="cuda",
-              fused: bool = False, use_index: bool = False):
+              fused: bool = False, use_index: bool = False, sampled: bool = False):
     """Runs the GPU loop on all rows; returns the per-step host copies of every output.
 
     fused=False: switchsd_step, target stand-in, switchsd_verify per iteration.
     fused=True:  switchsd_verify_step (verification of iteration t-1, then step t) and the target
-                 stand-in per iteration; the last draft is verified by switchsd_verify."""
+                 stand-in per iteration; the last draft is verified by switchsd_verify.
+    sampled=True (not fused): the sampled stand-in and switchsd_verify_sampled (T > 0)."""
+    assert not (sampled and (fused or use_index))
     import torch
     from paper_2609_20186_gb300 import Session, bf16_tensor
 
@@ -85,8 +94,16 @@ def gpu_trace(wl: synth.Workload, steps: int, split: int = 0, ctx=None, lens=Non
         else:
             sess.step(hidden)
         out = sess.step_outputs()
-        sess.harness(t)
-        if not fused or t == steps - 1:
+        if sampled:
+            sess.harness_sampled(t)
+        else:
+            sess.harness(t)
+        if sampled:
+            sess.verify_sampled()
+            out["accept"] = sess.accept.cpu().numpy()
+            out["vstatus"] = sess.vstatus.cpu().numpy()
+            out["lens_after"] = sess.lens.cpu().numpy()
+        elif not fused or t == steps - 1:
             sess.verify()
             out["accept"] = sess.accept.cpu().numpy()
             out["vstatus"] = sess.vstatus.cpu().numpy()

@@ -118,6 +118,27 @@ def test_verify_validation(lib):
     assert lib.switchsd_verify(FAKE, FAKE, FAKE, ctypes.byref(vp)) == bd.ERR_ARG
 
 
+def test_verify_sampled_validation(lib):
+    from paper_2609_20186_gb300 import binding as bd
+    vp = bd.switchsd_verify_params()
+    vp.B, vp.cap, vp.k = 4, 64, 8
+    vp.draft_len = vp.ctx_tokens = vp.ctx_lens = FAKE
+    f = FAKE
+    assert lib.switchsd_verify_sampled(f, f, None, f, f, f, None) == bd.ERR_ARG
+    assert lib.switchsd_verify_sampled(f, None, None, f, f, f, ctypes.byref(vp)) == bd.ERR_ARG  # no p
+    assert lib.switchsd_verify_sampled(f, f, None, None, f, f, ctypes.byref(vp)) == bd.ERR_ARG  # no u
+    vp.index = FAKE                                  # the index keeps to greedy verification
+    assert lib.switchsd_verify_sampled(f, f, None, f, f, f, ctypes.byref(vp)) == bd.ERR_ARG
+    vp.index = None
+    vp.k = 65
+    assert lib.switchsd_verify_sampled(f, f, None, f, f, f, ctypes.byref(vp)) == bd.ERR_SHAPE
+    hp = bd.switchsd_harness_params()
+    hp.B, hp.k, hp.V, hp.gamma = 4, 8, 100, 6
+    assert lib.switchsd_harness_sampled(f, f, f, f, None, f, f, None, f, f, f, ctypes.byref(hp)) == bd.ERR_ARG
+    hp.gamma = 9
+    assert lib.switchsd_harness_sampled(f, f, f, f, None, f, f, f, f, f, f, ctypes.byref(hp)) == bd.ERR_SHAPE
+
+
 def test_binding_rejects_cpu_tensors(lib):
     import torch
     from paper_2609_20186_gb300 import binding as bd
