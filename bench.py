@@ -65,6 +65,8 @@ def parse_args(argv=None):
                     help="budget of the CPU-baseline sample")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--verify", default="greedy", choices=["greedy", "sampled"],
+                    help="verification at temperature 0 (greedy) or T > 0 (sampled: App. A)")
     ap.add_argument("--no-prefetch", action="store_true",
                     help="read nothing before the preceding kernel is done (params.prefetch = 0)")
     return ap.parse_args(argv)
@@ -208,7 +210,7 @@ def profiled_traffic(workload: str) -> float | None:
 # CPU oracle timing (baseline and reference arm)
 # ------------------------------------------------------------------------------------------------
 def time_oracle(wl: synth.Workload, budget_s: float, max_steps: int, rows: int | None = None,
-                warmup: int = 0):
+                warmup: int = 0, sampled: bool = False):
     """Runs the oracle loop (oracle step, host target stand-in, oracle verify) on rows [0, R):
     ``warmup`` untimed steps, then up to max_steps timed steps or until budget_s of oracle time is
     spent.  Returns (seq*steps, seconds, timed_steps, R).  Only the oracle's calls are timed."""
@@ -227,10 +229,16 @@ def time_oracle(wl: synth.Workload, budget_s: float, max_steps: int, rows: int |
                           logit_tau=wl.logit_tau, probe_kind=wl.probe_kind,
                           probe_hidden=wl.probe_hidden, rows=(0, R))
         dt = time.perf_counter() - t0
-        vd, vl, tg = synth.harness_targets(hp, t, lens, out["mode"], out["draft"], out["len"],
-                                           future, rows=range(R))
-        t0 = time.perf_counter()
-        oracle.verify(ctx, lens, vd, vl, tg, rows=(0, R))
+        if sampled:
+            vd, vl, pp, qq, uu, rs = synth.harness_sampled(hp, t, lens, out["mode"], out["draft"],
+                                                           out["len"], future, rows=range(R))
+            t0 = time.perf_counter()
+            oracle.verify_sampled(ctx, lens, vd, vl, pp, uu, rs, q=qq, rows=(0, R))
+        else:
+            vd, vl, tg = synth.harness_targets(hp, t, lens, out["mode"], out["draft"], out["len"],
+                                               future, rows=range(R))
+            t0 = time.perf_counter()
+            oracle.verify(ctx, lens, vd, vl, tg, rows=(0, R))
         dt += time.perf_counter() - t0
         if t < warmup:
             continue
@@ -241,16 +249,17 @@ def time_oracle(wl: synth.Workload, budget_s: float, max_steps: int, rows: int |
     return R * done, spent, done, R
 
 
-def cpu_baseline(wl: synth.Workload, budget_s: float) -> dict:
-    units, secs, steps, R = time_oracle(wl, budget_s, wl.steps)
+def cpu_baseline(wl: synth.Workload, budget_s: float, sampled: bool = False) -> dict:
+    units, secs, steps, R = time_oracle(wl, budget_s, wl.steps, sampled=sampled)
     return {"value": units / secs, "unit": UNIT, "cores": 1, "kind": "oracle",
             "sample": f"{wl.name}: rows 0..{R - 1}, first {steps} controller steps (oracle step + "
                       f"verify timed, single thread; the host target stand-in is not timed)"}
 
 
 def config_of(wl: synth.Workload, world: int, split: int, search: str = "scan",
-              prefetch: bool = True) -> dict:
-    return {"workload": wl.name, "search": search, "prefetch": bool(prefetch and search == "scan"), "B": wl.B, "L0": wl.L0, "V": wl.V, "d": wl.d, "k": wl.k,
+              prefetch: bool = True, verify: str = "greedy") -> dict:
+    return {"workload": wl.name, "search": search, "verify": verify,
+            "prefetch": bool(prefetch and search == "scan"), "B": wl.B, "L0": wl.L0, "V": wl.V, "d": wl.d, "k": wl.k,
             "n_min": wl.n_min, "n_max": wl.n_max, "kappa": wl.kappa_eff, "tau": wl.tau,
             "probe": "linear" if wl.probe_kind == 0 else f"mlp{wl.d}x{wl.probe_hidden}",
             "global_batch": wl.B * world, "seq_len": wl.L0, "parallelism": f"replicas{world}",
@@ -268,14 +277,15 @@ def run_reference(args, world, rank):
     base = synth.get_workload(args.workload)
     wl = base.scaled(steps=args.warmup + args.steps)
     R = wl.B if wl.B <= 64 else 16
-    units, secs, steps, R = time_oracle(wl, float("inf"), args.steps, rows=R, warmup=args.warmup)
+    units, secs, steps, R = time_oracle(wl, float("inf"), args.steps, rows=R, warmup=args.warmup,
+                                        sampled=args.verify == "sampled")
     value = units / secs
     line = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
             "steps": args.steps, "warmup": args.warmup,
             "ms_per_step": secs / steps * 1e3, "higher_is_better": True, "scaling": "weak",
             "vs_baseline": None, "dtype": "int32 (search/verify), f64 (probe)", "data": "synthetic",
             "impl": "reference",
-            "config": config_of(base, world, args.split, args.search, not args.no_prefetch),
+            "config": config_of(base, world, args.split, args.search, not args.no_prefetch, args.verify),
             "cpu_baseline": {"value": value, "unit": UNIT, "cores": 1, "kind": "oracle",
                              "sample": f"{wl.name}: rows 0..{R - 1}, {args.warmup} untimed + "
                                        f"{steps} timed steps, single thread"},
@@ -301,7 +311,7 @@ class ReplicaLoop:
     switchsd_verify_step on batch i (its rows only); then one target stand-in covers all R*B rows."""
 
     def __init__(self, wl, R, cap, ctx1, lens1, pw, future1, hidden, split, dev, stream,
-                 search="scan", prefetch=True):
+                 search="scan", prefetch=True, sampled=False):
         import ctypes
         import torch
         from paper_2609_20186_gb300 import binding as bd, bf16_tensor
@@ -309,6 +319,7 @@ class ReplicaLoop:
         self.bd, self.ct = bd, ctypes
         self.lib = bd.load()
         self.R, self.B, self.k, self.cap = R, wl.B, wl.k, cap
+        self.sampled = sampled  # verification at T > 0 (the sampled stand-in and rule)
         B, k = wl.B, wl.k
         ctx = np.zeros((B, cap), np.int32)
         ctx[:, : ctx1.shape[1]] = ctx1[:, : min(cap, ctx1.shape[1])]
@@ -369,10 +380,16 @@ class ReplicaLoop:
         hp.stream = sp
         self.hp = hp
         e32, e16 = 4, 2
+        f32 = dict(dtype=torch.float32, device=dev)
+        self.vp = torch.zeros(N, k, **f32)
+        self.vq = torch.ones(N, k, **f32)
+        self.vu = torch.zeros(N, k, **f32)
         self.rows = []
         for r in range(R):
             o = r * B
             self.rows.append(dict(
+                vp=self.vp.data_ptr() + o * k * e32, vq=self.vq.data_ptr() + o * k * e32,
+                vu=self.vu.data_ptr() + o * k * e32,
                 vdraft=self.vdraft.data_ptr() + o * k * e32, target=self.target.data_ptr() + o * (k + 1) * e32,
                 vlen=self.vlen.data_ptr() + o * e32, accept=self.accept.data_ptr() + o * e32,
                 ctx=self.ctx.data_ptr() + o * cap * e32, lens=self.lens.data_ptr() + o * e32,
@@ -387,6 +404,11 @@ class ReplicaLoop:
             code = self.lib.switchsd_step(c["ctx"], c["lens"], hid, self.probe_w.data_ptr(),
                                           self.ct.byref(self.params[r]), c["draft"], c["len"], c["mode"],
                                           c["score"])
+        elif self.sampled:
+            code = self.lib.switchsd_verify_sampled_step(
+                c["vdraft"], c["vp"], c["vq"], c["vu"], c["target"], c["vlen"], c["accept"], c["ctx"], c["lens"],
+                hid, self.probe_w.data_ptr(), self.ct.byref(self.params[r]), c["draft"], c["len"], c["mode"],
+                c["score"])
         else:
             code = self.lib.switchsd_verify_step(c["vdraft"], c["target"], c["vlen"], c["accept"], c["ctx"],
                                                  c["lens"], hid, self.probe_w.data_ptr(),
@@ -397,10 +419,16 @@ class ReplicaLoop:
 
     def harness(self, q: int):
         self.hp.step = q
-        code = self.lib.switchsd_harness_target(
-            self.lens.data_ptr(), self.mode.data_ptr(), self.draft.data_ptr(), self.len.data_ptr(),
-            self.future.data_ptr(), self.vdraft.data_ptr(), self.vlen.data_ptr(), self.target.data_ptr(),
-            self.ct.byref(self.hp))
+        if self.sampled:
+            code = self.lib.switchsd_harness_sampled(
+                self.lens.data_ptr(), self.mode.data_ptr(), self.draft.data_ptr(), self.len.data_ptr(),
+                self.future.data_ptr(), self.vdraft.data_ptr(), self.vlen.data_ptr(), self.vp.data_ptr(),
+                self.vq.data_ptr(), self.vu.data_ptr(), self.target.data_ptr(), self.ct.byref(self.hp))
+        else:
+            code = self.lib.switchsd_harness_target(
+                self.lens.data_ptr(), self.mode.data_ptr(), self.draft.data_ptr(), self.len.data_ptr(),
+                self.future.data_ptr(), self.vdraft.data_ptr(), self.vlen.data_ptr(), self.target.data_ptr(),
+                self.ct.byref(self.hp))
         if code != 0:
             raise RuntimeError(f"harness failed: {code}")
 
@@ -416,6 +444,8 @@ def run_ours(args, world, rank, local):
 
     if not torch.cuda.is_available():
         raise SystemExit("bench.py needs a CUDA device (the controller has no CPU path)")
+    if args.verify == "sampled" and args.search == "index":
+        raise SystemExit("--verify sampled runs the rescan (the index keeps to greedy verification)")
     torch.cuda.set_device(local)
     dev = torch.device("cuda", local)
     binding.load()
@@ -430,7 +460,7 @@ def run_ours(args, world, rank, local):
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         import oracle
         oracle.build()
-        cpu = cpu_baseline(base, args.cpu_seconds)
+        cpu = cpu_baseline(base, args.cpu_seconds, sampled=args.verify == "sampled")
 
     # Replica batches: enough of them that the timed loop reads every batch from HBM.
     R = choose_replicas(B * (base.L0 + 1024) * 4, l2, K)
@@ -449,7 +479,7 @@ def run_ours(args, world, rank, local):
     hidden = bf16_tensor(hidden_host, dev)
     cs = torch.cuda.Stream(dev)
     loop = ReplicaLoop(wl, R, cap, ctx1, lens1, pw, future1, hidden, args.split, dev, cs,
-                       search=args.search, prefetch=not args.no_prefetch)
+                       search=args.search, prefetch=not args.no_prefetch, sampled=args.verify == "sampled")
     ctx_bytes_all = R * B * cap * 4
 
     with torch.cuda.stream(cs):
@@ -512,7 +542,8 @@ def run_ours(args, world, rank, local):
         n_this = min(R, K - j * R)
         grow = (Lh[j + 1] - Lh[j])[:n_this]                # a + 1 per row
         ctx_read = 4 * Lh[j + 1][:n_this].sum(axis=1)
-        verify_rw = 8 * B + 16 * grow.sum(axis=1)          # lens r/w, draft + target read, append
+        # lens r/w; per tested position the draft and target (sampled: also p, q, u) read, the append
+        verify_rw = 8 * B + (28 if args.verify == "sampled" else 16) * grow.sum(axis=1)
         outputs = 12 * B + 4 * B * k                       # mode, len, score, draft (bound)
         if args.search == "index":
             # index path: per row the context tail, and per n one head read and one candidate
@@ -538,7 +569,8 @@ def run_ours(args, world, rank, local):
 
     e2e = None
     if not args.no_e2e:
-        e2e = run_e2e(base, dev, W, K, args.split, world, prefetch=not args.no_prefetch)
+        e2e = run_e2e(base, dev, W, K, args.split, world, prefetch=not args.no_prefetch,
+                      sampled=args.verify == "sampled")
 
     if rank != 0:
         return
@@ -547,7 +579,8 @@ def run_ours(args, world, rank, local):
         "ms_per_step": ms_per_step, "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "dtype": "int32 (search/verify), bf16 in / fp32 accumulate (probe)",
         "data": "synthetic",
-        "config": dict(config_of(base, world, args.split, args.search, not args.no_prefetch), replicas=R,
+        "config": dict(config_of(base, world, args.split, args.search, not args.no_prefetch, args.verify),
+                       replicas=R,
                        l2=f"inputs larger than L2: {R} independent batches of B={B} "
                           f"({ctx_bytes_all / 2**20:.0f} MiB of contexts vs {l2 / 2**20:.0f} MiB L2), "
                           f"launch i reads batch i mod {R}"),
@@ -610,7 +643,7 @@ def cold_latency(loop, dev, cs, step_base, l2) -> dict:
             "note": "includes the ~2.2 us event-pair and ~2.2 us stream launch overhead of this GPU"}
 
 
-def run_e2e(base, dev, W, K, split, world, prefetch=True):
+def run_e2e(base, dev, W, K, split, world, prefetch=True, sampled=False):
     """The same loop through the public API with host buffers, one batch: per step, H2D of the
     hidden states from pinned memory, switchsd_verify_step + target stand-in, D2H of mode / draft
     length / draft / accepted length, host sync."""
@@ -639,9 +672,14 @@ def run_e2e(base, dev, W, K, split, world, prefetch=True):
         dev_h.view(torch.int16).copy_(host_h[t], non_blocking=True)
         if t == 0:
             sess.step(dev_h, debug=False)
+        elif sampled:
+            sess.verify_sampled_step(dev_h, debug=False)
         else:
             sess.verify_step(dev_h, debug=False)
-        sess.harness(t)
+        if sampled:
+            sess.harness_sampled(t)
+        else:
+            sess.harness(t)
         out_mode.copy_(sess.mode, non_blocking=True)
         out_len.copy_(sess.len, non_blocking=True)
         out_draft.copy_(sess.draft, non_blocking=True)

@@ -248,6 +248,18 @@ int switchsd_verify_step(const int32_t *draft, const int32_t *target_argmax, con
                          int32_t *out_mode, float *out_score);
 
 /*
+ * switchsd_verify_step at temperature T > 0: the sampled verification and append of the previous draft,
+ * exactly as switchsd_verify_sampled (same arguments: draft, p_draft, q_draft or NULL, u, resample,
+ * draft_len), then switchsd_step on the extended context, in one launch.  params->index must be NULL
+ * (SWITCHSD_ERR_ARG otherwise).  Statuses as switchsd_verify_step.
+ */
+int switchsd_verify_sampled_step(const int32_t *draft, const float *p_draft, const float *q_draft, const float *u,
+                                 const int32_t *resample, const int32_t *draft_len, int32_t *out_accept,
+                                 int32_t *ctx_tokens, int32_t *ctx_lens, const uint16_t *hidden,
+                                 const uint16_t *probe_w, const switchsd_params *params, int32_t *out_draft,
+                                 int32_t *out_len, int32_t *out_mode, float *out_score);
+
+/*
  * Bytes of device workspace switchsd_step / switchsd_verify_step need for `params` (0 for the linear
  * probe; for the two-layer probe, S x B x H1p floats rounded up to 256 bytes, where S is the first
  * layer's split of d -- the largest power of two <= 16 with at least two 64-element chunks of d per

@@ -74,6 +74,8 @@ _SIGNATURES = {
                                 + [ctypes.POINTER(switchsd_verify_params)]),
     "switchsd_verify_step": (ctypes.c_int, [ctypes.c_void_p] * 8 + [ctypes.POINTER(switchsd_params)]
                              + [ctypes.c_void_p] * 4),
+    "switchsd_verify_sampled_step": (ctypes.c_int, [ctypes.c_void_p] * 11 + [ctypes.POINTER(switchsd_params)]
+                                     + [ctypes.c_void_p] * 4),
     "switchsd_step_static_workspace": (ctypes.c_int, [ctypes.c_void_p] * 4
                                        + [ctypes.POINTER(switchsd_params)] + [ctypes.c_void_p] * 4),
     "switchsd_index_create": (ctypes.c_int, [ctypes.POINTER(switchsd_params),

@@ -64,6 +64,8 @@ struct StepArgs {
     const int32_t *pv_draft; // previous draft [B, k] / target [B, k+1] / draft length [B]; null = no verify
     const int32_t *pv_target;
     const int32_t *pv_len;
+    const float *pv_p, *pv_q, *pv_u;  // sampled verification (T > 0): null = greedy; pv_target then holds
+                                      // the residual / bonus draws and pv_q may be null (copy drafts)
     int32_t *out_accept;
     int32_t B, cap, d, k, n_min, n_max, kappa, tile, stages;
     int32_t prefetch;        // SWITCHSD_PREFETCH_* bits: reads that may precede the grid-dependency wait
@@ -262,8 +264,19 @@ __global__ void __launch_bounds__(kStepThreads) step_kernel(const StepArgs a) {
             if (pv_n < 0 || pv_n > a.k) {
                 vst = SWITCHSD_ROW_BAD_LEN;
             } else {
-                const unsigned m_lo = __ballot_sync(kFull, lane < pv_n && d_lo != t_lo);
-                const unsigned m_hi = __ballot_sync(kFull, lane + 32 < pv_n && d_hi != t_hi);
+                // greedy: a draft token is rejected when it differs from the target's; sampled: when
+                // u * q (binary32) is not below p
+                bool rej_lo = lane < pv_n && d_lo != t_lo, rej_hi = lane + 32 < pv_n && d_hi != t_hi;
+                if (a.pv_p != nullptr) {
+                    const size_t o = size_t(b) * a.k;
+                    rej_lo = lane < pv_n &&
+                             !(__fmul_rn(a.pv_u[o + lane], a.pv_q ? a.pv_q[o + lane] : 1.f) < a.pv_p[o + lane]);
+                    rej_hi = lane + 32 < pv_n && !(__fmul_rn(a.pv_u[o + lane + 32],
+                                                            a.pv_q ? a.pv_q[o + lane + 32] : 1.f) <
+                                                   a.pv_p[o + lane + 32]);
+                }
+                const unsigned m_lo = __ballot_sync(kFull, rej_lo);
+                const unsigned m_hi = __ballot_sync(kFull, rej_hi);
                 acc = m_lo ? __ffs(m_lo) - 1 : (m_hi ? 32 + __ffs(m_hi) - 1 : pv_n);
                 if (L_old + acc + 1 > a.cap) {
                     vst = SWITCHSD_ROW_CAPACITY;
@@ -573,7 +586,8 @@ static cudaError_t launch_step(const StepArgs &args, int split, cudaStream_t str
 static int step_entry(int32_t *ctx_tokens, int32_t *ctx_lens, const uint16_t *hidden, const uint16_t *probe_w,
                       const switchsd_params *p, const int32_t *pv_draft, const int32_t *pv_target,
                       const int32_t *pv_len, int32_t *out_accept, int32_t *out_draft, int32_t *out_len,
-                      int32_t *out_mode, float *out_score) {
+                      int32_t *out_mode, float *out_score, const float *pv_p = nullptr,
+                      const float *pv_q = nullptr, const float *pv_u = nullptr) {
     if (!p || !ctx_tokens || !ctx_lens || !hidden || !probe_w || !out_draft || !out_len || !out_mode ||
         !out_score)
         return SWITCHSD_ERR_ARG;
@@ -606,6 +620,9 @@ static int step_entry(int32_t *ctx_tokens, int32_t *ctx_lens, const uint16_t *hi
     args.pv_draft = pv_draft;
     args.pv_target = pv_target;
     args.pv_len = pv_len;
+    args.pv_p = pv_p;
+    args.pv_q = pv_q;
+    args.pv_u = pv_u;
     args.out_accept = out_accept;
     args.B = p->B;
     args.cap = p->cap;
@@ -689,4 +706,16 @@ extern "C" int switchsd_verify_step(const int32_t *draft, const int32_t *target_
     if (!draft || !target_argmax || !draft_len || !out_accept) return SWITCHSD_ERR_ARG;
     return step_entry(ctx_tokens, ctx_lens, hidden, probe_w, p, draft, target_argmax, draft_len, out_accept,
                       out_draft, out_len, out_mode, out_score);
+}
+
+extern "C" int switchsd_verify_sampled_step(const int32_t *draft, const float *p_draft, const float *q_draft,
+                                            const float *u, const int32_t *resample, const int32_t *draft_len,
+                                            int32_t *out_accept, int32_t *ctx_tokens, int32_t *ctx_lens,
+                                            const uint16_t *hidden, const uint16_t *probe_w,
+                                            const switchsd_params *p, int32_t *out_draft, int32_t *out_len,
+                                            int32_t *out_mode, float *out_score) {
+    if (!draft || !p_draft || !u || !resample || !draft_len || !out_accept) return SWITCHSD_ERR_ARG;
+    if (p && p->index != nullptr) return SWITCHSD_ERR_ARG;  // the index keeps to greedy verification
+    return step_entry(ctx_tokens, ctx_lens, hidden, probe_w, p, draft, resample, draft_len, out_accept, out_draft,
+                      out_len, out_mode, out_score, p_draft, q_draft, u);
 }

@@ -179,6 +179,17 @@ class Session:
         if code != bd.OK:
             raise RuntimeError(f"switchsd_verify failed: {code} ({bd.strerror(code)})")
 
+    def verify_sampled_step(self, hidden: torch.Tensor, debug: bool = True) -> None:
+        """Sampled verification (T > 0) of the last sampled-harness draft and the next step, fused."""
+        self._check_hidden(hidden)
+        p = self._p_dbg if debug else self._p_fast
+        code = self.lib.switchsd_verify_sampled_step(
+            self.vdraft.data_ptr(), self.vp.data_ptr(), self.vq.data_ptr(), self.vu.data_ptr(),
+            self.target.data_ptr(), self.vlen.data_ptr(), self.accept.data_ptr(), self.ctx.data_ptr(),
+            self.lens.data_ptr(), hidden.data_ptr(), *self._step_tail, ctypes.byref(p), *self._step_outs)
+        if code != bd.OK:
+            raise RuntimeError(f"switchsd_verify_sampled_step failed: {code} ({bd.strerror(code)})")
+
     def harness_sampled(self, t: int) -> None:
         """The target stand-in at T > 0: vdraft / vlen, vp / vq / vu and the resample tokens in target."""
         self._hp.step = t

@@ -70,8 +70,8 @@ def gpu_trace(wl: synth.Workload, steps: int, split: int = 0, ctx=None, lens=Non
     fused=False: switchsd_step, target stand-in, switchsd_verify per iteration.
     fused=True:  switchsd_verify_step (verification of iteration t-1, then step t) and the target
                  stand-in per iteration; the last draft is verified by switchsd_verify.
-    sampled=True (not fused): the sampled stand-in and switchsd_verify_sampled (T > 0)."""
-    assert not (sampled and (fused or use_index))
+    sampled=True: the sampled stand-in and switchsd_verify_sampled / switchsd_verify_sampled_step (T > 0)."""
+    assert not (sampled and use_index)
     import torch
     from paper_2609_20186_gb300 import Session, bf16_tensor
 
@@ -85,7 +85,10 @@ def gpu_trace(wl: synth.Workload, steps: int, split: int = 0, ctx=None, lens=Non
     for t in range(steps):
         hidden = bf16_tensor(wl.hidden(t), sess.device)
         if fused and t > 0:
-            sess.verify_step(hidden)
+            if sampled:
+                sess.verify_sampled_step(hidden)
+            else:
+                sess.verify_step(hidden)
             prev = trace[-1]
             st = sess.status.cpu().numpy()
             prev["accept"] = sess.accept.cpu().numpy()
@@ -98,13 +101,11 @@ def gpu_trace(wl: synth.Workload, steps: int, split: int = 0, ctx=None, lens=Non
             sess.harness_sampled(t)
         else:
             sess.harness(t)
-        if sampled:
-            sess.verify_sampled()
-            out["accept"] = sess.accept.cpu().numpy()
-            out["vstatus"] = sess.vstatus.cpu().numpy()
-            out["lens_after"] = sess.lens.cpu().numpy()
-        elif not fused or t == steps - 1:
-            sess.verify()
+        if not fused or t == steps - 1:
+            if sampled:
+                sess.verify_sampled()
+            else:
+                sess.verify()
             out["accept"] = sess.accept.cpu().numpy()
             out["vstatus"] = sess.vstatus.cpu().numpy()
             out["lens_after"] = sess.lens.cpu().numpy()

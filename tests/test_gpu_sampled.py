@@ -1,7 +1,7 @@
 """Verification at temperature T > 0 (App. A): the CUDA path vs the oracle, through the C ABI.
 
-The loop is step -> sampled stand-in -> switchsd_verify_sampled on both sides from the same seeded
-inputs; accepted lengths, appended contexts and everything the step produces must match the oracle
+The loop is step -> sampled stand-in -> switchsd_verify_sampled (or the fused
+switchsd_verify_sampled_step) on both sides from the same seeded inputs; accepted lengths, appended contexts and everything the step produces must match the oracle
 bit for bit (the acceptance test is taken in binary32 on both sides), the probe logit within 1e-3.
 """
 import numpy as np
@@ -23,12 +23,13 @@ SMALL = {
 }
 
 
+@pytest.mark.parametrize("fused", [False, True], ids=["separate", "fused"])
 @pytest.mark.parametrize("name", list(SMALL))
-def test_sampled_lockstep(name):
+def test_sampled_lockstep(name, fused):
     wl = SMALL[name]
     rows = range(wl.B)
     o_trace, o_ctx, _ = lockstep.oracle_trace(wl, rows, wl.steps, sampled=True)
-    g_trace, g_ctx, _ = lockstep.gpu_trace(wl, wl.steps, sampled=True)
+    g_trace, g_ctx, _ = lockstep.gpu_trace(wl, wl.steps, sampled=True, fused=fused)
     flips, stats = lockstep.compare(wl, o_trace, g_trace, rows, o_ctx, g_ctx)
     assert stats["checked"] > 0
     # the sampled rule accepted something and rejected something over the run
@@ -118,7 +119,7 @@ def test_full_size_sampled_rows():
     """zipf_32k in the benchmark's shape: every row runs on the GPU at T > 0; the oracle replays a sample
     of rows over every step (rows are independent, so a replayed row is exact)."""
     wl = W["zipf_32k"].scaled(steps=16)
-    g_trace, g_ctx, _ = lockstep.gpu_trace(wl, wl.steps, sampled=True)
+    g_trace, g_ctx, _ = lockstep.gpu_trace(wl, wl.steps, sampled=True, fused=True)
     rows = [0, 17, 40, 63]
     o_trace, o_ctx, _ = lockstep.oracle_trace(wl, rows, wl.steps, sampled=True)
     flips, stats = lockstep.compare(wl, o_trace, g_trace, rows, o_ctx, g_ctx)
