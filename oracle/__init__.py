@@ -98,6 +98,10 @@ def configure(lib):
                                                ctypes.c_int32, ctypes.c_int32, _i32p, _i32p, _f32p,
                                                _f32p, _f32p, _i32p, _i32p, _i32p]
     lib.oracle_verify_sampled_rows.restype = None
+    lib.oracle_window_repeats.argtypes = [_i32p, ctypes.c_int32, ctypes.c_int32, ctypes.c_int32]
+    lib.oracle_window_repeats.restype = ctypes.c_int32
+    lib.oracle_copy_labels.argtypes = [_i32p, ctypes.c_int32, ctypes.c_int32, ctypes.POINTER(ctypes.c_uint8)]
+    lib.oracle_copy_labels.restype = None
     return lib
 
 
@@ -310,3 +314,18 @@ def verify_sampled(ctx: np.ndarray, lens: np.ndarray, draft: np.ndarray, draft_l
                                    None if qa is None else _ptr(qa, _f32p), _ptr(u, _f32p),
                                    _ptr(resample, _i32p), _ptr(acc, _i32p), _ptr(st, _i32p))
     return acc, st
+
+
+def window_repeats(x, n: int, s: int) -> bool:
+    """Whether the n-token window of x starting at s also starts at an earlier position (§3.2)."""
+    xa = _c(x, np.int32)
+    return bool(_load().oracle_window_repeats(_ptr(xa, _i32p), xa.shape[0], n, s))
+
+
+def copy_labels(x, n: int = 5) -> np.ndarray:
+    """Copy-mode labels (§3.2) of the sequence x: uint8 [len(x)], 1 where the position lies in an
+    n-token window that also occurs starting earlier."""
+    xa = _c(x, np.int32)
+    y = np.zeros(xa.shape[0], np.uint8)
+    _load().oracle_copy_labels(_ptr(xa, _i32p), xa.shape[0], n, y.ctypes.data_as(ctypes.POINTER(ctypes.c_uint8)))
+    return y

@@ -239,3 +239,33 @@ void oracle_verify_sampled_rows(int32_t *ctx, int32_t *lens, int32_t b0, int32_t
         if (status != NULL) status[b] = st;
     }
 }
+
+/*
+ * Copy-mode label of a position (§3.2, "Problem Formulation"): position j is a copy-mode instance
+ * (Y = 1) when it belongs to a verbatim sequence of at least n_train tokens that appears earlier in the
+ * context (the paper sets n_train = 5).  Read as: some window x[s .. s+n-1] with s <= j <= s+n-1 also
+ * occurs starting at an earlier position s' < s (the two occurrences may overlap, as in the search).
+ * A longer verbatim sequence contains such a window around every one of its positions, so windows of
+ * exactly n cover the definition.
+ *
+ * oracle_window_repeats: whether the window starting at s has an earlier occurrence (0 when the window
+ * does not fit).  oracle_copy_labels: y[j] for every j < L, by the definition above, O(L^2 n).
+ */
+int32_t oracle_window_repeats(const int32_t *x, int32_t L, int32_t n, int32_t s)
+{
+    if (n < 1 || s < 0 || s + n > L) return 0;
+    for (int32_t s2 = 0; s2 < s; ++s2) {
+        int32_t i = 0;
+        while (i < n && x[s2 + i] == x[s + i]) ++i;
+        if (i == n) return 1;
+    }
+    return 0;
+}
+
+void oracle_copy_labels(const int32_t *x, int32_t L, int32_t n, uint8_t *y)
+{
+    for (int32_t j = 0; j < L; ++j) y[j] = 0;
+    for (int32_t s = 0; s + n <= L; ++s)
+        if (oracle_window_repeats(x, L, n, s))
+            for (int32_t j = s; j < s + n; ++j) y[j] = 1;
+}

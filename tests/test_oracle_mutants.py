@@ -52,6 +52,10 @@ MUTANTS = {
     "sampled: inverts the ratio": ("float prod = u[a] * qa;\n        if (!(prod < p[a])) break;",
                                    "float prod = u[a] * p[a];\n        if (!(prod < qa)) break;"),
     "sampled: wrong resample": ("row[*L + a] = resample[a];", "row[*L + a] = resample[a > 0 ? a - 1 : 0];"),
+    "labels: counts the window itself": ("for (int32_t s2 = 0; s2 < s; ++s2) {", "for (int32_t s2 = 0; s2 <= s; ++s2) {"),
+    "labels: labels the window start only": ("for (int32_t j = s; j < s + n; ++j) y[j] = 1;", "y[s] = 1;"),
+    "labels: last window skipped": ("for (int32_t s = 0; s + n <= L; ++s)", "for (int32_t s = 0; s + n < L; ++s)"),
+    "labels: one token short": ("while (i < n && x[s2 + i] == x[s + i]) ++i;", "while (i < n - 1 && x[s2 + i] == x[s + i]) ++i;"),
 }
 
 
@@ -127,6 +131,10 @@ def battery() -> list:
                                                  q=[0.5, 0.5])[1] == 1)
     row = np.zeros(8, np.int32)
     check("sampled low p", oracle.verify_sampled_row(row, 1, 8, [4], [0.2], [0.5], [7, 9], q=[1.0])[1] == 0)
+    # copy-mode labels (test_oracle_labels.py)
+    check("labels repeat", oracle.copy_labels([1, 2, 3, 4, 5, 9, 1, 2, 3, 4, 5], 5).tolist() == [0] * 6 + [1] * 5)
+    check("labels unique", oracle.copy_labels([1, 2, 3, 4, 5, 6], 5).sum() == 0)
+    check("labels short", oracle.copy_labels([1, 2, 3, 4, 8, 1, 2, 3, 4], 5).sum() == 0)
     return failed
 
 
