@@ -321,6 +321,25 @@ void switchsd_index_destroy(switchsd_index *index);
 /* Human-readable text of a host return code or a row status (static storage, never NULL). */
 const char *switchsd_strerror(int code);
 
+/*
+ * Copy-mode labels (§3.2, "Problem Formulation"): the probe's training labels.  Position j of row b is
+ * labelled 1 when it lies in a window of n consecutive tokens that also occurs starting at an earlier
+ * position of the row (the paper uses n = n_train = 5); every other position 0.  The same exact token
+ * comparisons as the search, over every position instead of the current one.
+ *
+ *   ctx_tokens  device int32 [B, cap], ctx_lens device int32 [B] (a length outside [0, cap] labels
+ *               nothing)
+ *   n           1..SWITCHSD_NMAX
+ *   out_labels  device uint8 [B, cap]: 0 / 1 for j < ctx_lens[b], 0 beyond
+ *   workspace   device scratch of at least switchsd_labels_workspace_bytes(B, cap) bytes, 4-byte
+ *               aligned, caller-owned (a first-occurrence table per row; calls sharing it must not
+ *               overlap on the GPU)
+ *   stream      cudaStream_t as void*
+ */
+size_t switchsd_labels_workspace_bytes(int32_t B, int32_t cap);
+int switchsd_copy_labels(const int32_t *ctx_tokens, const int32_t *ctx_lens, int32_t B, int32_t cap, int32_t n,
+                         uint8_t *out_labels, void *workspace, size_t workspace_bytes, void *stream);
+
 /* SWITCHSD_ABI_VERSION of the loaded library. */
 int switchsd_abi_version(void);
 

@@ -86,6 +86,10 @@ _SIGNATURES = {
     "switchsd_strerror": (ctypes.c_char_p, [ctypes.c_int]),
     "switchsd_workspace_bytes": (ctypes.c_size_t, [ctypes.POINTER(switchsd_params)]),
     "switchsd_abi_version": (ctypes.c_int, []),
+    "switchsd_labels_workspace_bytes": (ctypes.c_size_t, [ctypes.c_int32, ctypes.c_int32]),
+    "switchsd_copy_labels": (ctypes.c_int, [ctypes.c_void_p, ctypes.c_void_p, ctypes.c_int32, ctypes.c_int32,
+                                            ctypes.c_int32, ctypes.c_void_p, ctypes.c_void_p, ctypes.c_size_t,
+                                            ctypes.c_void_p]),
     "switchsd_harness_target": (ctypes.c_int, [ctypes.c_void_p] * 8
                                 + [ctypes.POINTER(switchsd_harness_params)]),
     "switchsd_harness_sampled": (ctypes.c_int, [ctypes.c_void_p] * 11
@@ -360,3 +364,17 @@ def switchsd_harness_sampled(ctx_lens, mode, draft, draft_len, future, vdraft, v
         _dev(q, torch.float32, "q", (B, k)), _dev(u, torch.float32, "u", (B, k)),
         _dev(resample, torch.int32, "resample", (B, k + 1)), ctypes.byref(hp))
     _check(code, "switchsd_harness_sampled")
+
+
+def switchsd_copy_labels(ctx_tokens, ctx_lens, out_labels, *, n: int = 5, workspace=None, stream=None) -> None:
+    """switchsd_copy_labels of include/switchsd.h (§3.2 copy-mode labels): ctx_tokens int32 [B, cap],
+    ctx_lens int32 [B], out_labels uint8 [B, cap].  Allocates the workspace from torch when none is given."""
+    B, cap = ctx_tokens.shape
+    need = int(load().switchsd_labels_workspace_bytes(B, cap))
+    if workspace is None:
+        workspace = torch.empty(need, dtype=torch.uint8, device=ctx_tokens.device)
+    code = load().switchsd_copy_labels(
+        _dev(ctx_tokens, torch.int32, "ctx_tokens"), _dev(ctx_lens, torch.int32, "ctx_lens", (B,)), B, cap, n,
+        _dev(out_labels, torch.uint8, "out_labels", (B, cap)), _dev(workspace, torch.uint8, "workspace"),
+        workspace.numel(), _stream_ptr(stream))
+    _check(code, "switchsd_copy_labels")

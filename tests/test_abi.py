@@ -139,6 +139,21 @@ def test_verify_sampled_validation(lib):
     assert lib.switchsd_harness_sampled(f, f, f, f, None, f, f, f, f, f, f, ctypes.byref(hp)) == bd.ERR_SHAPE
 
 
+def test_labels_validation(lib):
+    from paper_2609_20186_gb300 import binding as bd
+    need = lib.switchsd_labels_workspace_bytes(4, 1000)
+    assert need >= 4 * 2000 * 4                          # a table of >= 2 cap slots per row
+    assert lib.switchsd_labels_workspace_bytes(0, 1000) == 0
+    f = FAKE
+    assert lib.switchsd_copy_labels(None, f, 4, 1000, 5, f, f, need, None) == bd.ERR_ARG
+    assert lib.switchsd_copy_labels(f, f, 4, 1000, 5, f, None, need, None) == bd.ERR_ARG
+    assert lib.switchsd_copy_labels(f, f, 4, 1000, 5, f, f + 2, need, None) == bd.ERR_ARG   # misaligned
+    assert lib.switchsd_copy_labels(f, f, 4, 1000, 5, f, f, need - 1, None) == bd.ERR_ARG  # too small
+    assert lib.switchsd_copy_labels(f, f, 4, 1000, 0, f, f, need, None) == bd.ERR_SHAPE
+    assert lib.switchsd_copy_labels(f, f, 4, 1000, 33, f, f, need, None) == bd.ERR_SHAPE
+    assert lib.switchsd_copy_labels(f, f, 0, 1000, 5, f, f, need, None) == bd.ERR_SHAPE
+
+
 def test_binding_rejects_cpu_tensors(lib):
     import torch
     from paper_2609_20186_gb300 import binding as bd
