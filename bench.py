@@ -65,6 +65,8 @@ def parse_args(argv=None):
                     help="budget of the CPU-baseline sample")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--task", default="step", choices=["step", "labels"],
+                    help="step: the controller step (the headline); labels: copy-mode labels (§3.2)")
     ap.add_argument("--verify", default="greedy", choices=["greedy", "sampled"],
                     help="verification at temperature 0 (greedy) or T > 0 (sampled: App. A)")
     ap.add_argument("--no-prefetch", action="store_true",
@@ -700,12 +702,114 @@ def run_e2e(base, dev, W, K, split, world, prefetch=True, sampled=False):
                     "stand-in, D2H of mode/len/draft/accept, host sync; L2 not flushed"}
 
 
+LABEL_METRIC = "copy-mode labels/sec (positions, §3.2, n_train=5); achieved HBM GB/s vs peak"
+LABEL_UNIT = "positions/s"
+
+
+def label_cpu_baseline(wl: synth.Workload, budget_s: float) -> dict:
+    """The oracle's labels (plain O(L^2 n) definition) on whole rows of the workload until budget_s."""
+    import oracle
+    oracle.build()
+    ctx, lens = wl.contexts()
+    done, spent = 0, 0.0
+    for b in range(wl.B):
+        t0 = time.perf_counter()
+        oracle.copy_labels(ctx[b, : int(lens[b])], 5)
+        spent += time.perf_counter() - t0
+        done += int(lens[b])
+        if spent >= budget_s:
+            break
+    return {"value": done / spent, "unit": LABEL_UNIT, "cores": 1, "kind": "oracle",
+            "sample": f"{wl.name}: oracle copy_labels on whole rows, {done} positions (single thread)"}
+
+
+def run_labels(args, world, rank, local):
+    """--task labels: switchsd_copy_labels over R replica batches of the workload's contexts (inputs
+    larger than L2), K calls in a CUDA graph; value = labelled positions per second."""
+    import torch
+    from paper_2609_20186_gb300 import binding as bd
+
+    if not torch.cuda.is_available():
+        raise SystemExit("bench.py needs a CUDA device (the controller has no CPU path)")
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    lib = bd.load()
+    wl = synth.get_workload(args.workload)
+    W, K = args.warmup, args.steps
+    props = torch.cuda.get_device_properties(dev)
+    l2 = int(getattr(props, "L2_cache_size", 128 << 20))
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        cpu = label_cpu_baseline(wl, args.cpu_seconds)
+    ctx1, lens1 = wl.contexts()
+    B, cap = ctx1.shape
+    R = choose_replicas(B * cap * 4, l2, max(K, 1))
+    ctx = torch.from_numpy(np.tile(ctx1, (R, 1))).to(dev)
+    lens = torch.from_numpy(np.tile(lens1, R)).to(dev)
+    labels = torch.zeros(R * B, cap, dtype=torch.uint8, device=dev)
+    ws_bytes = int(lib.switchsd_labels_workspace_bytes(B, cap))
+    ws = torch.empty(R, ws_bytes, dtype=torch.uint8, device=dev)
+    cs = torch.cuda.Stream(dev)
+    sp = cs.cuda_stream
+
+    def call(i):
+        r = i % R
+        code = lib.switchsd_copy_labels(ctx.data_ptr() + r * B * cap * 4, lens.data_ptr() + r * B * 4, B, cap, 5,
+                                        labels.data_ptr() + r * B * cap, ws[r].data_ptr(), ws_bytes, sp)
+        if code != 0:
+            raise RuntimeError(f"switchsd_copy_labels failed: {code}")
+
+    with torch.cuda.stream(cs):
+        for i in range(max(W, 3)):
+            call(i)
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, stream=cs):
+            for i in range(K):
+                call(i)
+        g.replay()
+        cs.synchronize()
+        barrier(world)
+        sampler = ClockSampler(_gpu_uuid(props))
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        torch.cuda.synchronize()
+        e0.record(cs)
+        g.replay()
+        e1.record(cs)
+        e1.synchronize()
+        torch.cuda.synchronize()
+        clocks = sampler.stop()
+    ms = e0.elapsed_time(e1)
+    secs = reduce_max(ms / 1e3, world)
+    positions = float(lens1.sum()) * K
+    value = replica_throughput(positions, secs, world)
+    T = ws_bytes // (4 * B)
+    bytes_per_call = float(lens1.sum()) * 4 + B * cap + B * T * 4    # context, labels, table clear
+    achieved = bytes_per_call / (secs / K) / 1e9
+    peaks = measured_peaks()
+    if rank == 0:
+        line = {"metric": LABEL_METRIC, "value": value, "unit": LABEL_UNIT, "n_gpus": world, "steps": K,
+                "warmup": W, "ms_per_step": secs * 1e3 / K, "higher_is_better": True, "scaling": "weak",
+                "vs_baseline": None, "dtype": "int32 tokens, uint8 labels", "data": "synthetic",
+                "config": {"workload": wl.name, "task": "labels", "B": B, "cap": cap, "n_train": 5,
+                           "global_batch": B * world, "seq_len": wl.L0, "parallelism": f"replicas{world}",
+                           "replicas": R,
+                           "l2": f"inputs larger than L2: {R} batches of B={B} ({R * B * cap * 4 >> 20} MiB)"},
+                "roofline": {"kernel": "switchsd_copy_labels", "bound": "hbm", "achieved": achieved,
+                             "peak": peaks["hbm_gbs"], "unit": "GB/s", "frac": achieved / peaks["hbm_gbs"],
+                             "traffic": None, "algorithmic_bytes_per_launch": bytes_per_call,
+                             "peak_source": f"{peaks['source']} hbm_gbs (copy)"},
+                "gpu_launches": 2 * K, "clocks": clocks, "cpu_baseline": cpu}
+        print(json.dumps(line), flush=True)
+
+
 def main(argv=None):
     args = parse_args(argv)
     world, rank, local = dist_init(args.gpus)
     try:
         if args.impl == "reference":
             run_reference(args, world, rank)
+        elif args.task == "labels":
+            run_labels(args, world, rank, local)
         else:
             run_ours(args, world, rank, local)
     finally:
