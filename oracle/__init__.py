@@ -102,6 +102,23 @@ def configure(lib):
     lib.oracle_window_repeats.restype = ctypes.c_int32
     lib.oracle_copy_labels.argtypes = [_i32p, ctypes.c_int32, ctypes.c_int32, ctypes.POINTER(ctypes.c_uint8)]
     lib.oracle_copy_labels.restype = None
+    lib.oracle_candidates.argtypes = [_i32p, ctypes.c_int32, ctypes.c_int32, ctypes.c_int32, ctypes.c_int32,
+                                      ctypes.c_double, ctypes.c_float, ctypes.c_int32, ctypes.c_int32, _i32p,
+                                      _i32p, _i32p, _i32p]
+    lib.oracle_candidates.restype = ctypes.c_int32
+    lib.oracle_verify_candidates_row.argtypes = [_i32p, _i32p, ctypes.c_int32, _i32p, _i32p, ctypes.c_int32,
+                                                 ctypes.c_int32, _i32p, _i32p, _i32p]
+    lib.oracle_verify_candidates_row.restype = ctypes.c_int32
+    lib.oracle_step_candidates_rows.argtypes = [
+        _i32p, _i32p, ctypes.c_int32, ctypes.c_int32, ctypes.c_int32,
+        _u16p, ctypes.c_int32, _u16p, ctypes.c_int32, ctypes.c_int32, _f32p, ctypes.c_float,
+        ctypes.c_int32, ctypes.c_int32, ctypes.c_int32, ctypes.c_int32, ctypes.c_int32, ctypes.c_float,
+        _i32p, _i32p, _i32p, _i32p, _f64p, _i32p, _i32p, _i32p]
+    lib.oracle_step_candidates_rows.restype = None
+    lib.oracle_verify_candidates_rows.argtypes = [_i32p, _i32p, ctypes.c_int32, ctypes.c_int32, ctypes.c_int32,
+                                                  ctypes.c_int32, ctypes.c_int32, _i32p, _i32p, _i32p, _i32p,
+                                                  _i32p, _i32p, _i32p]
+    lib.oracle_verify_candidates_rows.restype = None
     return lib
 
 
@@ -329,3 +346,85 @@ def copy_labels(x, n: int = 5) -> np.ndarray:
     y = np.zeros(xa.shape[0], np.uint8)
     _load().oracle_copy_labels(_ptr(xa, _i32p), xa.shape[0], n, y.ctypes.data_as(ctypes.POINTER(ctypes.c_uint8)))
     return y
+
+
+def candidates(x, *, n_min: int, n_max: int, kappa: int, z: float, logit_tau: float, W: int, D: int):
+    """Copy candidates of one context (§3.3): returns (mode, [candidate token lists], [candidate ends])
+    -- ends only for a copy row."""
+    xa = _c(x, np.int32)
+    L = xa.shape[0]
+    cand = np.zeros((W, D), np.int32)
+    clen = np.zeros(W, np.int32)
+    ends = np.zeros(max(W, 1), np.int32)
+    nc = ctypes.c_int32()
+    mode = _load().oracle_candidates(_ptr(xa, _i32p), L, n_min, n_max, kappa, float(z), float(logit_tau), W, D,
+                                     _ptr(cand, _i32p), _ptr(clen, _i32p), ctypes.byref(nc), _ptr(ends, _i32p))
+    n = nc.value
+    return mode, [cand[w, : clen[w]].tolist() for w in range(n)], ends[:n].tolist()
+
+
+def verify_candidates_row(row: np.ndarray, L: int, cap: int, cands, target):
+    """Verification of W candidates (§3.3) on one row buffer (modified in place): cands a list of token
+    lists (empty list = no candidate), target [W][D+1] (D = the longest candidate slot).
+    Returns (new_L, accept, choice, status)."""
+    W = max(len(cands), 1)
+    D = max([len(c) for c in cands] + [np.asarray(target).shape[1] - 1])
+    cand = np.zeros((W, D), np.int32)
+    clen = np.zeros(W, np.int32)
+    for w, c in enumerate(cands):
+        cand[w, : len(c)] = c
+        clen[w] = len(c)
+    t = np.zeros((W, D + 1), np.int32)
+    ta = np.asarray(target, np.int32)
+    t[: ta.shape[0], : ta.shape[1]] = ta
+    Lc, acc, ch = ctypes.c_int32(L), ctypes.c_int32(), ctypes.c_int32()
+    st = _load().oracle_verify_candidates_row(_ptr(row, _i32p), ctypes.byref(Lc), cap, _ptr(cand, _i32p),
+                                              _ptr(clen, _i32p), len(cands), D, _ptr(t, _i32p), ctypes.byref(acc),
+                                              ctypes.byref(ch))
+    return Lc.value, acc.value, ch.value, st
+
+
+def step_candidates(ctx: np.ndarray, lens: np.ndarray, hidden_bits: np.ndarray, probe_w_bits: np.ndarray, *,
+                    W: int, D: int, n_min: int, n_max: int, kappa: int = 0, logit_tau: float = 0.0,
+                    probe_kind: int = 0, probe_hidden: int = 0, b1=None, b2: float = 0.0,
+                    rows: tuple[int, int] | None = None) -> dict:
+    """The candidate step on rows [b0, b1): cand [B, W, D], cand_len [B, W], ncand, mode, score, match_n,
+    match_end (numpy, rows outside the range zero)."""
+    lib = _load()
+    B, cap = ctx.shape
+    lens = _c(lens, np.int32)
+    hidden = _c(hidden_bits, np.uint16)
+    d = hidden.shape[1]
+    pw = _c(probe_w_bits, np.uint16).reshape(-1)
+    b1a = None if b1 is None else _c(b1, np.float32)
+    b0, bend = rows if rows is not None else (0, B)
+    out = {"cand": np.zeros((B, W, D), np.int32), "cand_len": np.zeros((B, W), np.int32),
+           "ncand": np.zeros(B, np.int32), "mode": np.zeros(B, np.int32), "score": np.zeros(B, np.float64),
+           "match_n": np.zeros(B, np.int32), "match_end": np.full(B, -1, np.int32)}
+    scratch = np.zeros(max(W, 1), np.int32)
+    lib.oracle_step_candidates_rows(_ptr(ctx, _i32p), _ptr(lens, _i32p), b0, bend, cap, _ptr(hidden, _u16p), d,
+                                    _ptr(pw, _u16p), probe_kind, probe_hidden,
+                                    None if b1a is None else _ptr(b1a, _f32p), float(b2), W, D, n_min, n_max,
+                                    kappa, float(logit_tau), _ptr(out["cand"], _i32p), _ptr(out["cand_len"], _i32p),
+                                    _ptr(out["ncand"], _i32p), _ptr(out["mode"], _i32p), _ptr(out["score"], _f64p),
+                                    _ptr(out["match_n"], _i32p), _ptr(out["match_end"], _i32p),
+                                    _ptr(scratch, _i32p))
+    return out
+
+
+def verify_candidates(ctx: np.ndarray, lens: np.ndarray, cand: np.ndarray, cand_len: np.ndarray,
+                      ncand: np.ndarray, target: np.ndarray, rows: tuple[int, int] | None = None):
+    """Verification of the candidates on rows [b0, b1); ctx / lens updated in place.  cand [B, W, D],
+    cand_len [B, W], ncand [B], target [B, W, D+1].  Returns (accept, choice, status) [B]."""
+    lib = _load()
+    B, cap = ctx.shape
+    cand = _c(cand, np.int32)
+    W, D = cand.shape[1], cand.shape[2]
+    cand_len, ncand, target = _c(cand_len, np.int32), _c(ncand, np.int32), _c(target, np.int32)
+    assert target.shape == (B, W, D + 1)
+    acc, ch, st = np.zeros(B, np.int32), np.zeros(B, np.int32), np.zeros(B, np.int32)
+    b0, bend = rows if rows is not None else (0, B)
+    lib.oracle_verify_candidates_rows(_ptr(ctx, _i32p), _ptr(lens, _i32p), b0, bend, cap, W, D, _ptr(cand, _i32p),
+                                      _ptr(cand_len, _i32p), _ptr(ncand, _i32p), _ptr(target, _i32p),
+                                      _ptr(acc, _i32p), _ptr(ch, _i32p), _ptr(st, _i32p))
+    return acc, ch, st

@@ -269,3 +269,118 @@ void oracle_copy_labels(const int32_t *x, int32_t L, int32_t n, uint8_t *y)
         if (oracle_window_repeats(x, L, n, s))
             for (int32_t j = s; j < s + n; ++j) y[j] = 1;
 }
+
+/*
+ * Copy candidates, W of them (§3.3 "Copy-Based Speculative Generation": up to W candidate continuations
+ * of length D retrieved from the context and ranked by recency; App. D uses W = 10, D = 20).  Reading:
+ * the candidates are the W most recent ends e <= L-2 at which the kappa-gram ending at the current
+ * token also ends -- the common suffix of x[..e] and x[..L-1] is at least kappa tokens long (the gate
+ * of the decision rule) -- listed from the most recent; candidate w continues with
+ * x[e_w+1 .. e_w+len_w], len_w = min(D, L-1-e_w).  The mode follows the decision rule as in
+ * oracle_switch: no repetition when no n_min-gram of the suffix occurs earlier, copy when a candidate
+ * exists and the logit reaches logit_tau (compared in binary32), repetition without copy otherwise.
+ * Candidates are written only for a copy row (ncand = 0 otherwise).  Returns the mode.
+ */
+int32_t oracle_candidates(const int32_t *x, int32_t L, int32_t n_min, int32_t n_max, int32_t kappa, double z,
+                          float logit_tau, int32_t W, int32_t D, int32_t *cand, int32_t *cand_len, int32_t *ncand,
+                          int32_t *cand_end)
+{
+    int32_t has_match = 0, n = 0;
+    for (int32_t e = L - 2; e >= 0; --e) {
+        /* common suffix of x[..e] and x[..L-1], at most n_max tokens */
+        int32_t m = 0;
+        while (m < n_max && m <= e && x[e - m] == x[L - 1 - m]) ++m;
+        if (m >= n_min) has_match = 1;
+        if (m >= kappa && n < W) cand_end[n++] = e;
+    }
+    *ncand = 0;
+    if (!has_match) return ORACLE_MODE_NO_REP;
+    if (n == 0 || !((float)z >= logit_tau)) return ORACLE_MODE_REP_NO_COPY;
+    for (int32_t w = 0; w < n; ++w) {
+        int32_t avail = L - 1 - cand_end[w];
+        int32_t len = avail < D ? avail : D;
+        cand_len[w] = len;
+        for (int32_t i = 0; i < len; ++i) cand[(int64_t)w * D + i] = x[cand_end[w] + 1 + i];
+    }
+    *ncand = n;
+    return ORACLE_MODE_COPY;
+}
+
+/*
+ * Verification of W candidates (§3.3 "Parallel Verification with Block-Triangular Attention": the
+ * target checks every candidate in one pass and the longest validated continuation is kept).  target
+ * holds, per candidate w, the target's greedy token after each prefix of candidate w (D + 1 entries).
+ * a_w = the leading tokens of candidate w equal to target[w]; the kept candidate is the one with the
+ * largest a_w, the most recent (lowest w) on a tie; its a tokens and then target[w][a] are appended.
+ * ncand = 0 counts as one empty candidate (only target[0][0] is appended).  Capacity as
+ * oracle_verify_row.
+ */
+int32_t oracle_verify_candidates_row(int32_t *row, int32_t *L, int32_t cap, const int32_t *cand,
+                                     const int32_t *cand_len, int32_t ncand, int32_t D, const int32_t *target,
+                                     int32_t *accept, int32_t *choice)
+{
+    int32_t best = 0, a_best = -1;
+    int32_t nc = ncand > 0 ? ncand : 1;
+    for (int32_t w = 0; w < nc; ++w) {
+        int32_t len = ncand > 0 ? cand_len[w] : 0;
+        int32_t a = 0;
+        while (a < len && cand[(int64_t)w * D + a] == target[(int64_t)w * (D + 1) + a]) ++a;
+        if (a > a_best) {
+            a_best = a;
+            best = w;
+        }
+    }
+    *choice = best;
+    if (*L + a_best + 1 > cap) {
+        *accept = -1;
+        return ORACLE_ROW_CAPACITY;
+    }
+    for (int32_t i = 0; i < a_best; ++i) row[*L + i] = cand[(int64_t)best * D + i];
+    row[*L + a_best] = target[(int64_t)best * (D + 1) + a_best];
+    *L += a_best + 1;
+    *accept = a_best;
+    return ORACLE_ROW_OK;
+}
+
+/* The candidate step on rows [b0, b1): the search's match (as oracle_step_rows), the probe, and the
+ * candidates and mode of oracle_candidates.  out_cand [B][W][D], out_cand_len [B][W], the rest [B]. */
+void oracle_step_candidates_rows(const int32_t *ctx, const int32_t *lens, int32_t b0, int32_t b1, int32_t cap,
+                                 const uint16_t *hidden, int32_t d, const uint16_t *probe_w, int32_t probe_kind,
+                                 int32_t H1, const float *b1v, float b2, int32_t W, int32_t D, int32_t n_min,
+                                 int32_t n_max, int32_t kappa, float logit_tau, int32_t *out_cand,
+                                 int32_t *out_cand_len, int32_t *out_ncand, int32_t *out_mode, double *out_score,
+                                 int32_t *out_n, int32_t *out_e, int32_t *scratch_ends)
+{
+    if (kappa <= 0) kappa = n_min;
+    for (int32_t b = b0; b < b1; ++b) {
+        const int32_t *x = ctx + (int64_t)b * cap;
+        int32_t L = lens[b];
+        int32_t n_star, e_star;
+        oracle_longest_suffix_match(x, L, n_min, n_max, &n_star, &e_star);
+        const uint16_t *h = hidden + (int64_t)b * d;
+        double z;
+        if (probe_kind == 0)
+            z = oracle_probe_linear(h, probe_w, d);
+        else
+            z = oracle_probe_mlp(h, probe_w, b1v, probe_w + (int64_t)H1 * d, b2, d, H1);
+        out_mode[b] = oracle_candidates(x, L, n_min, n_max, kappa, z, logit_tau, W, D,
+                                        out_cand + (int64_t)b * W * D, out_cand_len + (int64_t)b * W,
+                                        &out_ncand[b], scratch_ends);
+        out_score[b] = z;
+        out_n[b] = n_star;
+        out_e[b] = e_star;
+    }
+}
+
+void oracle_verify_candidates_rows(int32_t *ctx, int32_t *lens, int32_t b0, int32_t b1, int32_t cap, int32_t W,
+                                   int32_t D, const int32_t *cand, const int32_t *cand_len, const int32_t *ncand,
+                                   const int32_t *target, int32_t *out_accept, int32_t *out_choice, int32_t *status)
+{
+    for (int32_t b = b0; b < b1; ++b) {
+        int32_t st = oracle_verify_candidates_row(ctx + (int64_t)b * cap, &lens[b], cap, cand + (int64_t)b * W * D,
+                                                  cand_len + (int64_t)b * W, ncand[b], D,
+                                                  target + (int64_t)b * W * (D + 1), &out_accept[b],
+                                                  &out_choice[b]);
+        if (status != NULL) status[b] = st;
+    }
+}

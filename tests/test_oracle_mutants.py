@@ -56,6 +56,12 @@ MUTANTS = {
     "labels: labels the window start only": ("for (int32_t j = s; j < s + n; ++j) y[j] = 1;", "y[s] = 1;"),
     "labels: last window skipped": ("for (int32_t s = 0; s + n <= L; ++s)", "for (int32_t s = 0; s + n < L; ++s)"),
     "labels: one token short": ("while (i < n && x[s2 + i] == x[s + i]) ++i;", "while (i < n - 1 && x[s2 + i] == x[s + i]) ++i;"),
+    "candidates: oldest first": ("    for (int32_t e = L - 2; e >= 0; --e) {\n        /* common suffix",
+                                 "    for (int32_t e = 0; e <= L - 2; ++e) {\n        /* common suffix"),
+    "candidates: n_min gate": ("if (m >= kappa && n < W) cand_end[n++] = e;", "if (m >= n_min && n < W) cand_end[n++] = e;"),
+    "candidates: latest on a tie": ("        if (a > a_best) {", "        if (a >= a_best) {"),
+    "candidates: first candidate's bonus": ("row[*L + a_best] = target[(int64_t)best * (D + 1) + a_best];",
+                                            "row[*L + a_best] = target[a_best];"),
 }
 
 
@@ -135,6 +141,20 @@ def battery() -> list:
     check("labels repeat", oracle.copy_labels([1, 2, 3, 4, 5, 9, 1, 2, 3, 4, 5], 5).tolist() == [0] * 6 + [1] * 5)
     check("labels unique", oracle.copy_labels([1, 2, 3, 4, 5, 6], 5).sum() == 0)
     check("labels short", oracle.copy_labels([1, 2, 3, 4, 8, 1, 2, 3, 4], 5).sum() == 0)
+    # candidates (test_oracle_candidates.py)
+    x = np.array([1, 2, 3, 9, 1, 2, 3, 8, 1, 2, 3], np.int32)
+    check("candidates order", oracle.candidates(x, n_min=2, n_max=4, kappa=3, z=1.0, logit_tau=0.0, W=4, D=3)
+          == (1, [[8, 1, 2], [9, 1, 2]], [6, 2]))
+    y = np.array([5, 2, 3, 9, 1, 2, 3], np.int32)
+    check("candidates gate", oracle.candidates(y, n_min=2, n_max=4, kappa=3, z=1.0, logit_tau=0.0, W=4, D=3)[0] == 2)
+    row = np.zeros(32, np.int32)
+    check("candidates choose", oracle.verify_candidates_row(row, 1, 32, [[4, 5], [4, 6]], [[4, 9, 0], [4, 8, 0]])
+          == (3, 1, 0, 0))
+    row = np.zeros(32, np.int32)
+    row[:3] = [1, 2, 3]
+    check("candidates bonus", oracle.verify_candidates_row(row, 3, 32, [[4, 5, 6], [4, 7, 8, 9]],
+                                                           [[4, 0, 0, 0, 0], [4, 7, 8, 1, 0]]) == (7, 3, 1, 0)
+          and row[6] == 1)
     return failed
 
 
