@@ -321,6 +321,62 @@ void switchsd_index_destroy(switchsd_index *index);
 /* Human-readable text of a host return code or a row status (static storage, never NULL). */
 const char *switchsd_strerror(int code);
 
+#define SWITCHSD_WMAX 16 /* largest number of copy candidates W */
+
+/*
+ * The step with W copy candidates (§3.3 "Copy-Based Speculative Generation": up to W continuations of
+ * length D retrieved from the context, ranked by recency; App. D uses W = 10, D = 20).  The candidates
+ * are the W most recent ends e <= L-2 at which the kappa-gram ending at the current token recurs (the
+ * common suffix is at least kappa = params->kappa, or n_min when <= 0, tokens long), most recent first;
+ * candidate w continues with x[e_w+1 .. e_w+len_w], len_w = min(D, L-1-e_w).  The mode: no repetition
+ * when no n_min-gram of the suffix recurs, copy when a candidate exists and z >= logit_tau, repetition
+ * without copy otherwise.  Everything else as switchsd_step (params->k is only the bound of the staged
+ * look-ahead and must be >= 1; params->index must be NULL).
+ *
+ *   W, D          1..SWITCHSD_WMAX, 1..SWITCHSD_KMAX
+ *   out_cand      device int32 [B, W, D]: candidate w's tokens in [b][w][0, len_w)
+ *   out_cand_len  device int32 [B, W]: len_w for w < ncand
+ *   out_ncand     device int32 [B]: candidates of a copy row (0 for the other modes)
+ *   out_mode, out_score   as switchsd_step (out_match_n / out_match_end / status from params as well)
+ */
+int switchsd_step_candidates(const int32_t *ctx_tokens, const int32_t *ctx_lens, const uint16_t *hidden,
+                             const uint16_t *probe_w, const switchsd_params *params, int32_t W, int32_t D,
+                             int32_t *out_cand, int32_t *out_cand_len, int32_t *out_ncand, int32_t *out_mode,
+                             float *out_score);
+
+/*
+ * Parameters of switchsd_verify_candidates.
+ *
+ *   B, cap        as switchsd_verify_params;  W, D  the candidate slots (as switchsd_step_candidates)
+ *   cand_len      device int32 [B, W], ncand device int32 [B] (a neural row passes its draft as the one
+ *                 candidate; ncand = 0 counts as one empty candidate)
+ *   ctx_tokens, ctx_lens, status, stream   as switchsd_verify_params
+ */
+typedef struct {
+    int32_t B, cap, W, D;
+    const int32_t *cand_len;
+    const int32_t *ncand;
+    int32_t *ctx_tokens;
+    int32_t *ctx_lens;
+    int32_t *status;
+    void *stream;
+} switchsd_candidates_verify_params;
+
+/*
+ * Verification of the W candidates of each row (§3.3 "Parallel Verification with Block-Triangular
+ * Attention": one target pass checks every candidate, and the longest validated continuation is kept).
+ *
+ *   cand        device int32 [B, W, D]
+ *   target      device int32 [B, W, D+1]: the target's greedy token after each prefix of candidate w
+ *   out_accept  device int32 [B]: the kept candidate's accepted length a (-1: capacity / bad lengths)
+ *   out_choice  device int32 [B]: the kept candidate (the longest accepted, the lowest index on a tie)
+ *
+ * The row receives the kept candidate's a tokens, then its target token at a; ctx_lens grows by a+1.
+ * Capacity and bad lengths as switchsd_verify.
+ */
+int switchsd_verify_candidates(const int32_t *cand, const int32_t *target, int32_t *out_accept, int32_t *out_choice,
+                               const switchsd_candidates_verify_params *vp);
+
 /*
  * Copy-mode labels (§3.2, "Problem Formulation"): the probe's training labels.  Position j of row b is
  * labelled 1 when it lies in a window of n consecutive tokens that also occurs starting at an earlier

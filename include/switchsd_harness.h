@@ -63,6 +63,19 @@ int switchsd_harness_sampled(const int32_t *ctx_lens, const int32_t *mode, const
                              const int32_t *draft_len, const int32_t *future, int32_t *vdraft, int32_t *vlen,
                              float *p, float *q, float *u, int32_t *resample, const switchsd_harness_params *hp);
 
+/*
+ * The stand-in for switchsd_verify_candidates.  A copy row's candidates (cand [B, W, D], cand_len
+ * [B, W], ncand [B] from switchsd_step_candidates) are passed on; a neural row gets min(gamma, D)
+ * neural tokens (the law of switchsd_harness_target) as its one candidate.  target[b][w][i] is the
+ * stream's token at position L + i for every kept candidate (the target's greedy token after any prefix
+ * the verification can accept), 0 for unused slots.  Outputs vcand [B, W, D], vlen [B, W], vn [B],
+ * target [B, W, D+1].
+ */
+int switchsd_harness_candidates(const int32_t *ctx_lens, const int32_t *mode, const int32_t *cand,
+                                const int32_t *cand_len, const int32_t *ncand, const int32_t *future, int32_t W,
+                                int32_t D, int32_t *vcand, int32_t *vlen, int32_t *vn, int32_t *target,
+                                const switchsd_harness_params *hp);
+
 #ifdef __cplusplus
 }
 #endif

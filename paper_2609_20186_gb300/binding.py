@@ -51,6 +51,14 @@ class switchsd_verify_params(ctypes.Structure):
     ]
 
 
+class switchsd_candidates_verify_params(ctypes.Structure):
+    _fields_ = [
+        ("B", ctypes.c_int32), ("cap", ctypes.c_int32), ("W", ctypes.c_int32), ("D", ctypes.c_int32),
+        ("cand_len", ctypes.c_void_p), ("ncand", ctypes.c_void_p), ("ctx_tokens", ctypes.c_void_p),
+        ("ctx_lens", ctypes.c_void_p), ("status", ctypes.c_void_p), ("stream", ctypes.c_void_p),
+    ]
+
+
 class switchsd_harness_params(ctypes.Structure):
     _fields_ = [
         ("B", ctypes.c_int32), ("k", ctypes.c_int32), ("V", ctypes.c_int32), ("L0", ctypes.c_int32),
@@ -86,6 +94,13 @@ _SIGNATURES = {
     "switchsd_strerror": (ctypes.c_char_p, [ctypes.c_int]),
     "switchsd_workspace_bytes": (ctypes.c_size_t, [ctypes.POINTER(switchsd_params)]),
     "switchsd_abi_version": (ctypes.c_int, []),
+    "switchsd_step_candidates": (ctypes.c_int, [ctypes.c_void_p] * 4 + [ctypes.POINTER(switchsd_params),
+                                                                        ctypes.c_int32, ctypes.c_int32]
+                                 + [ctypes.c_void_p] * 5),
+    "switchsd_verify_candidates": (ctypes.c_int, [ctypes.c_void_p] * 4
+                                   + [ctypes.POINTER(switchsd_candidates_verify_params)]),
+    "switchsd_harness_candidates": (ctypes.c_int, [ctypes.c_void_p] * 6 + [ctypes.c_int32, ctypes.c_int32]
+                                    + [ctypes.c_void_p] * 4 + [ctypes.POINTER(switchsd_harness_params)]),
     "switchsd_labels_workspace_bytes": (ctypes.c_size_t, [ctypes.c_int32, ctypes.c_int32]),
     "switchsd_copy_labels": (ctypes.c_int, [ctypes.c_void_p, ctypes.c_void_p, ctypes.c_int32, ctypes.c_int32,
                                             ctypes.c_int32, ctypes.c_void_p, ctypes.c_void_p, ctypes.c_size_t,

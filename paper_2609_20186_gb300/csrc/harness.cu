@@ -143,3 +143,96 @@ extern "C" int switchsd_harness_sampled(const int32_t *ctx_lens, const int32_t *
                                      0, static_cast<cudaStream_t>(hp->stream), 0u, a);
     return e == cudaSuccess ? SWITCHSD_OK : SWITCHSD_ERR_CUDA;
 }
+
+// ------------------------------------------------------------------------------------------------
+// The stand-in for switchsd_verify_candidates: a copy row's W candidates are verified against the
+// target stream (target[w][i] = the stream's token at position L + i for every candidate w: the target's
+// greedy token after any prefix the verification can accept); a neural row holds its neural draft as the
+// one candidate.  One warp per row.
+// ------------------------------------------------------------------------------------------------
+namespace switchsd {
+
+struct CandHarnessArgs {
+    const int32_t *lens, *mode, *cand, *cand_len, *ncand, *future;
+    int32_t *vcand, *vlen, *vn, *target;
+    int32_t W, D;
+    switchsd_harness_params p;
+};
+
+__global__ void __launch_bounds__(kHarnessThreads) harness_candidates_kernel(const CandHarnessArgs a) {
+    const int lane = threadIdx.x & 31;
+    const int b = (blockIdx.x * kHarnessThreads + threadIdx.x) >> 5;
+    const switchsd_harness_params &p = a.p;
+    pdl_wait();
+    pdl_trigger();
+    if (b >= p.B) return;
+    const bool copy = a.mode[b] == SWITCHSD_MODE_COPY;
+    int n = copy ? a.ncand[b] : 1;
+    n = n < 0 ? 0 : (n > a.W ? a.W : n);
+    const int gamma = p.gamma < a.D ? p.gamma : a.D;
+    const int32_t L = a.lens[b];
+    const uint64_t row_key = splitmix64(splitmix64(splitmix64(p.seed) ^ uint64_t(b)) ^ uint64_t(p.step));
+    for (int i = lane; i <= a.D; i += kWarp) {
+        const int64_t pos = int64_t(L) - p.L0 + i;
+        const int32_t g = (pos >= 0 && pos < p.n_future) ? a.future[size_t(b) * p.n_future + pos] : 0;
+        for (int w = 0; w < a.W; ++w) {
+            const size_t o = size_t(b) * a.W + w;
+            a.target[o * (a.D + 1) + i] = w < n ? g : 0;
+            if (i < a.D) {
+                int32_t d = 0;
+                if (w < n) {
+                    if (copy) {
+                        d = i < a.cand_len[o] ? a.cand[o * a.D + i] : 0;
+                    } else if (i < gamma) {
+                        const uint64_t slot = 4ull * uint64_t(i);
+                        const uint64_t coin = splitmix64(row_key ^ slot) & 0xffffffffull;
+                        if (coin < p.thr_neural) {
+                            d = g;
+                        } else {
+                            d = token_of(splitmix64(row_key ^ (slot + 1)), p.V);
+                            if (d == g) d = (d + 1) % p.V;
+                        }
+                    }
+                }
+                a.vcand[o * a.D + i] = d;
+            }
+        }
+    }
+    if (lane < a.W) {
+        const size_t o = size_t(b) * a.W + lane;
+        a.vlen[o] = lane < n ? (copy ? a.cand_len[o] : gamma) : 0;
+    }
+    if (lane == 0) a.vn[b] = n;
+}
+
+}  // namespace switchsd
+
+extern "C" int switchsd_harness_candidates(const int32_t *ctx_lens, const int32_t *mode, const int32_t *cand,
+                                           const int32_t *cand_len, const int32_t *ncand, const int32_t *future,
+                                           int32_t W, int32_t D, int32_t *vcand, int32_t *vlen, int32_t *vn,
+                                           int32_t *target, const switchsd_harness_params *hp) {
+    if (!hp || !ctx_lens || !mode || !cand || !cand_len || !ncand || !vcand || !vlen || !vn || !target)
+        return SWITCHSD_ERR_ARG;
+    if (hp->n_future > 0 && !future) return SWITCHSD_ERR_ARG;
+    if (hp->B < 1 || W < 1 || W > SWITCHSD_WMAX || D < 1 || D > SWITCHSD_KMAX || hp->V < 2 || hp->n_future < 0 ||
+        hp->gamma < 0)
+        return SWITCHSD_ERR_SHAPE;
+    CandHarnessArgs a;
+    a.lens = ctx_lens;
+    a.mode = mode;
+    a.cand = cand;
+    a.cand_len = cand_len;
+    a.ncand = ncand;
+    a.future = future;
+    a.vcand = vcand;
+    a.vlen = vlen;
+    a.vn = vn;
+    a.target = target;
+    a.W = W;
+    a.D = D;
+    a.p = *hp;
+    const int wpb = kHarnessThreads / kWarp;
+    const cudaError_t e = launch_pdl(harness_candidates_kernel, dim3((hp->B + wpb - 1) / wpb), dim3(kHarnessThreads),
+                                     0, static_cast<cudaStream_t>(hp->stream), 0u, a);
+    return e == cudaSuccess ? SWITCHSD_OK : SWITCHSD_ERR_CUDA;
+}

@@ -46,6 +46,7 @@ constexpr int kMaxStages = 6;          // staged tiles in flight per CTA (bounde
 constexpr size_t kStageSmemBudget = 200 * 1024;
 constexpr int kMaxSplit = 16;
 constexpr unsigned long long kTimeoutBit = 1ull << 62;
+constexpr int kMaxCand = SWITCHSD_WMAX; // candidate mode: largest W
 constexpr int kProbeStage = 256;      // probe words (8 bf16) of w and of h staged per CTA; the rest is read directly
 
 static_assert(kHalo >= SWITCHSD_NMAX && kHalo % 4 == 0, "halo must cover the longest n-gram");
@@ -73,6 +74,8 @@ struct StepArgs {
     int32_t *out_draft, *out_len, *out_mode;
     float *out_score;
     int32_t *out_match_n, *out_match_end, *status;
+    int32_t W, D, bm_words;   // candidate mode: W candidates of up to D tokens; bitmap words per CTA
+    int32_t *out_cand, *out_cand_len, *out_ncand;
 };
 
 __device__ __forceinline__ float dot8_bf16(uint4 w, uint4 h, float acc) {
@@ -96,10 +99,14 @@ __device__ __forceinline__ void st_cluster_i32(uint32_t addr, int32_t v) {
 struct alignas(16) Slot {
     unsigned long long key;
     float z;
-    int32_t pad;
-    int32_t cand[SWITCHSD_KMAX];
+    int32_t count;             // candidate mode: candidate ends that follow
+    int32_t cand[SWITCHSD_KMAX];  // the candidate draft, or (candidate mode) candidate ends, most recent first
 };
 
+// kCand: the candidate mode of switchsd_step_candidates -- besides the longest match, every end whose
+// common suffix reaches kappa is marked in a per-CTA bitmap; the CTA ships its kMaxCand most recent
+// marks and the leader keeps the W most recent of the row.
+template <bool kCand>
 __global__ void __launch_bounds__(kStepThreads) step_kernel(const StepArgs a) {
     extern __shared__ __align__(128) int32_t tiles[];  // stages x (kHalo + tile + kFwd)
     __shared__ __align__(8) uint64_t bars[kMaxStages];
@@ -117,6 +124,8 @@ __global__ void __launch_bounds__(kStepThreads) step_kernel(const StepArgs a) {
     __shared__ __align__(16) uint4 s_probe[2 * kProbeStage];   // linear: w then h slices; two-layer: partial sums
     __shared__ Slot s_slot[kMaxSplit];                         // leader: one message per CTA
     __shared__ int32_t s_out[2];                               // leader: winner rank, draft length
+    __shared__ __align__(16) int32_t s_cand[kMaxCand];         // candidate mode: this CTA's / the row's ends
+    __shared__ int32_t s_ncand;
 
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     const uint32_t rank = cluster_ctarank();
@@ -124,7 +133,7 @@ __global__ void __launch_bounds__(kStepThreads) step_kernel(const StepArgs a) {
     const int b = blockIdx.y;
     const int stage_ints = kHalo + a.tile + kFwd;
     const bool verifying = a.pv_len != nullptr;
-    const int kwords = (a.k + 3) >> 2;                          // 16-byte words of a candidate
+    const int kwords = kCand ? (a.W + 3) >> 2 : (a.k + 3) >> 2;  // 16-byte words of a message's payload
     const uint32_t slot_bytes = 16u * uint32_t(1 + kwords);
 
     if (tid == 0) {
@@ -300,6 +309,10 @@ __global__ void __launch_bounds__(kStepThreads) step_kernel(const StepArgs a) {
         cluster_arrive_release();
     } else {
         if ((!pf_probe || mlp) && tid == 2 * kWarp) issue_probe();
+        if (kCand) {
+            uint32_t *bm = reinterpret_cast<uint32_t *>(tiles + a.stages * stage_ints);
+            for (int i = tid - 2 * kWarp; i < a.bm_words; i += kStepThreads - 2 * kWarp) bm[i] = 0u;
+        }
         cluster_arrive_relaxed();
     }
     // Warps 0 and 1 meet (named barrier 1, 64 threads): the suffix needs the old tail and the append.
@@ -337,6 +350,7 @@ __global__ void __launch_bounds__(kStepThreads) step_kernel(const StepArgs a) {
     // the back-compare then starts at m = 2).  m0 is the length the filter has already checked.
     const bool pair = n_min >= 2;
     const int32_t m0 = pair ? 2 : 1;
+    const int32_t kappa_c = a.kappa > 0 ? a.kappa : n_min;  // candidate mode: the gate length
     unsigned long long best = 0;  // CTA-uniform; real keys have m >= n_min >= 1, so 0 = no match
     bool bad = s_ver[3] == 0;     // CTA-uniform: a copy did not land in time
     for (int t = 0; t < ntiles && !bad; ++t) {
@@ -396,6 +410,10 @@ __global__ void __launch_bounds__(kStepThreads) step_kernel(const StepArgs a) {
                                 (static_cast<unsigned long long>(m) << 32) | uint32_t(e);
                             mine = key > mine ? key : mine;
                         }
+                        if (kCand && m >= kappa_c) {
+                            uint32_t *bm = reinterpret_cast<uint32_t *>(tiles + a.stages * stage_ints);
+                            atomicOr(&bm[(e - e_lo) >> 5], 1u << ((e - e_lo) & 31));
+                        }
                     }
                 }
             }
@@ -410,7 +428,7 @@ __global__ void __launch_bounds__(kStepThreads) step_kernel(const StepArgs a) {
         for (int w = 0; w < kStepWarps; ++w) tile_best = s_wkey[w] > tile_best ? s_wkey[w] : tile_best;
         if (!bad && tile_best > best) {
             best = tile_best;
-            if (tid >= 1 && tid <= kwords) {
+            if (!kCand && tid >= 1 && tid <= kwords) {
                 const int32_t e = int32_t(best & 0xffffffffu);
                 const int32_t len = min(a.k, L - 1 - e);
 #pragma unroll
@@ -465,6 +483,32 @@ __global__ void __launch_bounds__(kStepThreads) step_kernel(const StepArgs a) {
     }
     zp = warp_sum_f32(zp);
     if (lane == 0) s_wz[warp] = zp;
+    if (kCand && warp == 0) {
+        // The CTA's most recent marked ends: 32 bitmap words per pass from the top; lane i holds word
+        // top - i, and a prefix sum of the popcounts ranks its bits after those of higher words.
+        const uint32_t *bm = reinterpret_cast<const uint32_t *>(tiles + a.stages * stage_ints);
+        int found = 0;
+        for (int top = a.bm_words - 1; top >= 0 && found < a.W; top -= kWarp) {
+            const int idx = top - lane;
+            const uint32_t wd = (idx >= 0 && !bad) ? bm[idx] : 0u;
+            const int c = __popc(wd);
+            int incl = c;
+#pragma unroll
+            for (int o = 1; o < kWarp; o <<= 1) {
+                const int t = __shfl_up_sync(kFull, incl, o);
+                if (lane >= o) incl += t;
+            }
+            int r = found + incl - c;
+            uint32_t w2 = wd;
+            while (w2 != 0u && r < a.W) {
+                const int bit = 31 - __clz(w2);
+                w2 &= ~(1u << bit);
+                s_cand[r++] = e_lo + idx * 32 + bit;
+            }
+            found += __shfl_sync(kFull, incl, kWarp - 1);
+        }
+        if (lane == 0) s_ncand = found < a.W ? found : a.W;
+    }
     __syncthreads();
     float cta_z = 0.f;
     if (warp == 0) cta_z = warp_sum_f32(lane < kStepWarps ? s_wz[lane] : 0.f);
@@ -487,10 +531,11 @@ __global__ void __launch_bounds__(kStepThreads) step_kernel(const StepArgs a) {
         h.x = uint32_t(best & 0xffffffffu);
         h.y = uint32_t(best >> 32);
         h.z = __float_as_uint(cta_z);
-        h.w = 0u;
+        h.w = kCand ? uint32_t(s_ncand) : 0u;
         st_async_v4(map_to_rank(&s_slot[rank], 0), h, done_addr);
     } else if (tid <= kwords) {
-        const uint4 v = *reinterpret_cast<const uint4 *>(&s_mine[4 * (tid - 1)]);
+        const uint4 v = kCand ? *reinterpret_cast<const uint4 *>(&s_cand[4 * (tid - 1)])
+                              : *reinterpret_cast<const uint4 *>(&s_mine[4 * (tid - 1)]);
         st_async_v4(map_to_rank(&s_slot[rank].cand[4 * (tid - 1)], 0), v, done_addr);
     }
     if (rank != 0) return;
@@ -516,14 +561,26 @@ __global__ void __launch_bounds__(kStepThreads) step_kernel(const StepArgs a) {
         const int32_t n = hit ? int32_t(key >> 32) : 0;
         const int32_t e = hit ? int32_t(key & 0xffffffffu) : -1;
         const int32_t kappa = a.kappa > 0 ? a.kappa : a.n_min;
+        int32_t ncand = 0;  // candidate mode: the row's candidates, merged from the most recent CTA down
+        if (kCand) {
+            if (lane == 0 && hit) {
+                for (int r = int(C) - 1; r >= 0 && ncand < a.W; --r) {
+                    const int c = s_slot[r].count;
+                    for (int i = 0; i < c && ncand < a.W; ++i) s_cand[ncand++] = s_slot[r].cand[i];
+                }
+            }
+            ncand = __shfl_sync(kFull, ncand, 0);
+        }
+        const bool gate = kCand ? ncand > 0 : n >= kappa;
         int32_t mode = SWITCHSD_MODE_NO_REP;
-        if (hit) mode = (n >= kappa && z >= a.logit_tau) ? SWITCHSD_MODE_COPY : SWITCHSD_MODE_REP_NO_COPY;
-        const int32_t len = mode == SWITCHSD_MODE_COPY ? min(a.k, L - 1 - e) : 0;
+        if (hit) mode = (gate && z >= a.logit_tau) ? SWITCHSD_MODE_COPY : SWITCHSD_MODE_REP_NO_COPY;
+        const int32_t len = (!kCand && mode == SWITCHSD_MODE_COPY) ? min(a.k, L - 1 - e) : 0;
         if (lane == 0) {
             s_out[0] = int32_t(win);
             s_out[1] = len;
+            if (kCand) s_ncand = mode == SWITCHSD_MODE_COPY ? ncand : 0;
             a.out_mode[b] = mode;
-            a.out_len[b] = len;
+            if (!kCand) a.out_len[b] = len;
             a.out_score[b] = z;
             if (a.out_match_n) a.out_match_n[b] = n;
             if (a.out_match_end) a.out_match_end[b] = e;
@@ -536,6 +593,19 @@ __global__ void __launch_bounds__(kStepThreads) step_kernel(const StepArgs a) {
         }
     }
     __syncthreads();
+    if (kCand) {
+        // The candidates' continuations, read from the row (the context is not modified in this mode).
+        const int nc = s_ncand;
+        if (tid == 0) a.out_ncand[b] = nc;
+        for (int t = tid; t < nc * a.D; t += kStepThreads) {
+            const int w = t / a.D, i = t - w * a.D;
+            const int32_t ew = s_cand[w];
+            const int32_t lw = min(a.D, L - 1 - ew);
+            if (i == 0) a.out_cand_len[size_t(b) * a.W + w] = lw;
+            if (i < lw) a.out_cand[(size_t(b) * a.W + w) * a.D + i] = row[ew + 1 + i];
+        }
+        return;
+    }
     const int32_t win = s_out[0], len = s_out[1];
     for (int i = tid; i < len; i += kStepThreads) a.out_draft[size_t(b) * a.k + i] = s_slot[win].cand[i];
 }
@@ -566,31 +636,43 @@ static int choose_split(int B, int cap) {
     return c;
 }
 
+template <bool kCand>
 static cudaError_t launch_step(const StepArgs &args, int split, cudaStream_t stream) {
     static bool attr_done[64] = {false};
     int dev = 0;
     cudaGetDevice(&dev);
     if (dev >= 0 && dev < 64 && !attr_done[dev]) {
-        cudaError_t e = cudaFuncSetAttribute(step_kernel, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
+        cudaError_t e = cudaFuncSetAttribute(step_kernel<kCand>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
         if (e != cudaSuccess) return e;
-        e = cudaFuncSetAttribute(step_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, int(kStageSmemBudget));
+        e = cudaFuncSetAttribute(step_kernel<kCand>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 int(kStageSmemBudget));
         if (e != cudaSuccess) return e;
         attr_done[dev] = true;
     }
-    const size_t smem = size_t(args.stages) * (kHalo + args.tile + kFwd) * sizeof(int32_t);
-    return launch_pdl(step_kernel, dim3(unsigned(split), unsigned(args.B), 1), dim3(kStepThreads, 1, 1), smem,
-                      stream, unsigned(split), args);
+    const size_t smem = size_t(args.stages) * (kHalo + args.tile + kFwd) * sizeof(int32_t) +
+                        (kCand ? size_t(args.bm_words) * sizeof(uint32_t) : 0);
+    return launch_pdl(step_kernel<kCand>, dim3(unsigned(split), unsigned(args.B), 1), dim3(kStepThreads, 1, 1),
+                      smem, stream, unsigned(split), args);
 }
+
+// Candidate-mode outputs of switchsd_step_candidates.
+struct CandSpec {
+    int32_t W, D;
+    int32_t *cand, *cand_len, *ncand;
+};
 
 // Shared validation and launch of switchsd_step / switchsd_verify_step.
 static int step_entry(int32_t *ctx_tokens, int32_t *ctx_lens, const uint16_t *hidden, const uint16_t *probe_w,
                       const switchsd_params *p, const int32_t *pv_draft, const int32_t *pv_target,
                       const int32_t *pv_len, int32_t *out_accept, int32_t *out_draft, int32_t *out_len,
                       int32_t *out_mode, float *out_score, const float *pv_p = nullptr,
-                      const float *pv_q = nullptr, const float *pv_u = nullptr) {
-    if (!p || !ctx_tokens || !ctx_lens || !hidden || !probe_w || !out_draft || !out_len || !out_mode ||
-        !out_score)
-        return SWITCHSD_ERR_ARG;
+                      const float *pv_q = nullptr, const float *pv_u = nullptr, const CandSpec *cs = nullptr) {
+    if (!p || !ctx_tokens || !ctx_lens || !hidden || !probe_w || !out_mode || !out_score) return SWITCHSD_ERR_ARG;
+    if (cs == nullptr && (!out_draft || !out_len)) return SWITCHSD_ERR_ARG;
+    if (cs != nullptr) {
+        if (!cs->cand || !cs->cand_len || !cs->ncand || p->index != nullptr) return SWITCHSD_ERR_ARG;
+        if (cs->W < 1 || cs->W > kMaxCand || cs->D < 1 || cs->D > SWITCHSD_KMAX) return SWITCHSD_ERR_SHAPE;
+    }
     if (!aligned16(ctx_tokens) || !aligned16(hidden) || !aligned16(probe_w)) return SWITCHSD_ERR_ARG;
     if (p->probe_kind != SWITCHSD_PROBE_LINEAR && p->probe_kind != SWITCHSD_PROBE_MLP) return SWITCHSD_ERR_ARG;
     if (p->B < 1 || p->B > 65535 || p->cap < 4 || (p->cap & 3) != 0) return SWITCHSD_ERR_SHAPE;
@@ -646,13 +728,21 @@ static int step_entry(int32_t *ctx_tokens, int32_t *ctx_lens, const uint16_t *hi
     // when it fits, else a ring of kTileMax stages, as many as the range needs up to kMaxStages and
     // the shared-memory budget.
     const int64_t range = ((int64_t(p->cap) - 1 + split - 1) / split + 3) / 4 * 4 + p->k + 1;
+    // candidate mode: a bit per end of the CTA's range, after the stages
+    args.W = cs ? cs->W : 0;
+    args.D = cs ? cs->D : 0;
+    args.bm_words = cs ? int32_t((range + 31) / 32) : 0;
+    args.out_cand = cs ? cs->cand : nullptr;
+    args.out_cand_len = cs ? cs->cand_len : nullptr;
+    args.out_ncand = cs ? cs->ncand : nullptr;
+    const size_t budget = kStageSmemBudget - size_t(args.bm_words) * sizeof(uint32_t);
     if (range <= kTileMax) {
         args.tile = int32_t((range + 3) / 4 * 4);
         args.stages = 1;
     } else {
         args.tile = kTileMax;
         const int64_t need = (range + kTileMax - 1) / kTileMax;
-        const int64_t fit = int64_t(kStageSmemBudget / ((kHalo + kTileMax + kFwd) * sizeof(int32_t)));
+        const int64_t fit = int64_t(budget / ((kHalo + kTileMax + kFwd) * sizeof(int32_t)));
         args.stages = int32_t(need < fit ? need : fit);
         if (args.stages > kMaxStages) args.stages = kMaxStages;
         if (args.stages < 2) args.stages = 2;
@@ -676,7 +766,8 @@ static int step_entry(int32_t *ctx_tokens, int32_t *ctx_lens, const uint16_t *hi
                             args.H1, args.H1p, args.b2, pv_draft, pv_target, pv_len, out_accept, out_draft, out_len,
                             out_mode, out_score, p->out_match_n, p->out_match_end, p->status, p->B, p->cap, p->d, p->k,
                             p->n_min, p->n_max, p->kappa, p->logit_tau, true, stream);
-    if (launch_step(args, split, stream) != cudaSuccess) return SWITCHSD_ERR_CUDA;
+    const cudaError_t e = cs ? launch_step<true>(args, split, stream) : launch_step<false>(args, split, stream);
+    if (e != cudaSuccess) return SWITCHSD_ERR_CUDA;
     return SWITCHSD_OK;
 }
 
@@ -706,6 +797,16 @@ extern "C" int switchsd_verify_step(const int32_t *draft, const int32_t *target_
     if (!draft || !target_argmax || !draft_len || !out_accept) return SWITCHSD_ERR_ARG;
     return step_entry(ctx_tokens, ctx_lens, hidden, probe_w, p, draft, target_argmax, draft_len, out_accept,
                       out_draft, out_len, out_mode, out_score);
+}
+
+extern "C" int switchsd_step_candidates(const int32_t *ctx_tokens, const int32_t *ctx_lens, const uint16_t *hidden,
+                                        const uint16_t *probe_w, const switchsd_params *p, int32_t W, int32_t D,
+                                        int32_t *out_cand, int32_t *out_cand_len, int32_t *out_ncand,
+                                        int32_t *out_mode, float *out_score) {
+    const CandSpec cs{W, D, out_cand, out_cand_len, out_ncand};
+    return step_entry(const_cast<int32_t *>(ctx_tokens), const_cast<int32_t *>(ctx_lens), hidden, probe_w, p,
+                      nullptr, nullptr, nullptr, nullptr, nullptr, nullptr, out_mode, out_score, nullptr, nullptr,
+                      nullptr, &cs);
 }
 
 extern "C" int switchsd_verify_sampled_step(const int32_t *draft, const float *p_draft, const float *q_draft,

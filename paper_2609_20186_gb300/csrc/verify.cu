@@ -147,3 +147,109 @@ extern "C" int switchsd_verify_sampled(const int32_t *draft, const float *p_draf
                                      static_cast<cudaStream_t>(vp->stream), 0u, a);
     return e == cudaSuccess ? SWITCHSD_OK : SWITCHSD_ERR_CUDA;
 }
+
+// ------------------------------------------------------------------------------------------------
+// switchsd_verify_candidates: the W copy candidates of a row verified at once (§3.3 "Parallel
+// Verification with Block-Triangular Attention": the target checks every candidate in one pass and
+// the longest validated continuation is kept).  One warp per row; per candidate a ballot gives its
+// accepted length, the longest is kept (the most recent, lowest index, on a tie) and appended with the
+// target's token after it.
+// ------------------------------------------------------------------------------------------------
+namespace switchsd {
+
+struct CandVerifyArgs {
+    const int32_t *cand, *cand_len, *ncand, *target;
+    int32_t *ctx, *lens, *out_accept, *out_choice, *status;
+    int32_t B, cap, W, D;
+};
+
+__global__ void __launch_bounds__(kVerifyThreads) verify_candidates_kernel(const CandVerifyArgs a) {
+    const int lane = threadIdx.x & 31;
+    const int b = (blockIdx.x * kVerifyThreads + threadIdx.x) >> 5;
+    pdl_wait();
+    pdl_trigger();
+    if (b >= a.B) return;
+    const int32_t L = a.lens[b];
+    const int32_t nc = a.ncand[b];
+    bool bad = L < 1 || L > a.cap || nc < 0 || nc > a.W;
+    for (int w = 0; w < nc && !bad; ++w) {
+        const int32_t len = a.cand_len[size_t(b) * a.W + w];
+        bad = len < 0 || len > a.D;
+    }
+    if (bad) {
+        if (lane == 0) {
+            a.out_accept[b] = -1;
+            a.out_choice[b] = 0;
+            if (a.status) a.status[b] = SWITCHSD_ROW_BAD_LEN;
+        }
+        return;
+    }
+    int32_t best = -1, best_w = 0;
+    for (int w = 0; w < (nc > 0 ? nc : 1); ++w) {  // no candidate: one empty one
+        const int32_t len = nc > 0 ? a.cand_len[size_t(b) * a.W + w] : 0;
+        const int32_t *c = a.cand + (size_t(b) * a.W + w) * a.D;
+        const int32_t *t = a.target + (size_t(b) * a.W + w) * (a.D + 1);
+        int32_t acc = len;
+        for (int base = 0; base < len; base += kWarp) {
+            const int i = base + lane;
+            const unsigned m = __ballot_sync(kFull, i < len && c[i] != t[i]);
+            if (m) {
+                acc = base + __ffs(m) - 1;
+                break;
+            }
+        }
+        if (acc > best) {
+            best = acc;
+            best_w = w;
+        }
+    }
+    if (L + best + 1 > a.cap) {
+        if (lane == 0) {
+            a.out_accept[b] = -1;
+            a.out_choice[b] = best_w;
+            if (a.status) a.status[b] = SWITCHSD_ROW_CAPACITY;
+        }
+        return;
+    }
+    const int32_t *c = a.cand + (size_t(b) * a.W + best_w) * a.D;
+    const int32_t *t = a.target + (size_t(b) * a.W + best_w) * (a.D + 1);
+    int32_t *row = a.ctx + size_t(b) * size_t(a.cap) + L;
+    for (int i = lane; i <= best; i += kWarp) row[i] = i < best ? c[i] : t[best];
+    if (lane == 0) {
+        a.lens[b] = L + best + 1;
+        a.out_accept[b] = best;
+        a.out_choice[b] = best_w;
+        if (a.status) a.status[b] = SWITCHSD_ROW_OK;
+    }
+}
+
+}  // namespace switchsd
+
+extern "C" int switchsd_verify_candidates(const int32_t *cand, const int32_t *target, int32_t *out_accept,
+                                          int32_t *out_choice, const switchsd_candidates_verify_params *vp) {
+    if (!vp || !cand || !target || !out_accept || !out_choice || !vp->cand_len || !vp->ncand || !vp->ctx_tokens ||
+        !vp->ctx_lens)
+        return SWITCHSD_ERR_ARG;
+    if (vp->B < 1 || vp->cap < 4 || (vp->cap & 3) != 0 || vp->W < 1 || vp->W > SWITCHSD_WMAX || vp->D < 1 ||
+        vp->D > SWITCHSD_KMAX)
+        return SWITCHSD_ERR_SHAPE;
+    CandVerifyArgs a;
+    a.cand = cand;
+    a.cand_len = vp->cand_len;
+    a.ncand = vp->ncand;
+    a.target = target;
+    a.ctx = vp->ctx_tokens;
+    a.lens = vp->ctx_lens;
+    a.out_accept = out_accept;
+    a.out_choice = out_choice;
+    a.status = vp->status;
+    a.B = vp->B;
+    a.cap = vp->cap;
+    a.W = vp->W;
+    a.D = vp->D;
+    const int warps_per_block = kVerifyThreads / kWarp;
+    const int blocks = (vp->B + warps_per_block - 1) / warps_per_block;
+    const cudaError_t e = launch_pdl(verify_candidates_kernel, dim3(blocks), dim3(kVerifyThreads), 0,
+                                     static_cast<cudaStream_t>(vp->stream), 0u, a);
+    return e == cudaSuccess ? SWITCHSD_OK : SWITCHSD_ERR_CUDA;
+}

@@ -7,4 +7,4 @@ n-gram search, no probe evaluation, no switch and no verification.
 """
 from .rng import splitmix64, harness_key, bf16_bits_from_f32, f32_from_bf16_bits  # noqa: F401
 from .workloads import WORKLOADS, Workload, get_workload  # noqa: F401
-from .harness import harness_targets, harness_sampled  # noqa: F401
+from .harness import harness_targets, harness_sampled, harness_candidates  # noqa: F401

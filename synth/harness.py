@@ -109,3 +109,46 @@ def harness_sampled(params: dict, step: int, ctx_lens: np.ndarray, mode: np.ndar
         resample[b, :ln] = np.where(gg == d, alt, gg).astype(np.int32)
         resample[b, ln] = g[b, ln]
     return vdraft, vlen, p, q, u, resample
+
+
+def harness_candidates(params: dict, step: int, ctx_lens: np.ndarray, mode: np.ndarray, cand: np.ndarray,
+                       cand_len: np.ndarray, ncand: np.ndarray, future: np.ndarray, rows=None):
+    """The stand-in for the verification of W copy candidates.  Returns (vcand [B, W, D], vlen [B, W],
+    vn [B], target [B, W, D+1]): a copy row passes its candidates on; any other row gets
+    min(gamma, D) neural tokens (the law of harness_targets) as its one candidate; target[b][w] is the
+    target stream at the row's next D+1 positions for every kept candidate (the target's greedy token
+    after any prefix the verification can accept), 0 for unused slots."""
+    B, W, D = cand.shape
+    V, L0, seed = params["V"], params["L0"], params["seed"]
+    gamma = min(params["gamma"], D)
+    thr = np.uint64(params["thr_neural"])
+    nfut = future.shape[1]
+    vcand = np.zeros((B, W, D), np.int32)
+    vlen = np.zeros((B, W), np.int32)
+    vn = np.zeros(B, np.int32)
+    target = np.zeros((B, W, D + 1), np.int32)
+    idx = range(B) if rows is None else rows
+    i = np.arange(D + 1, dtype=np.int64)
+    for b in idx:
+        b = int(b)
+        pos = int(ctx_lens[b]) - L0 + i
+        ok = (pos >= 0) & (pos < nfut)
+        g = np.where(ok, future[b, np.clip(pos, 0, max(nfut - 1, 0))] if nfut else 0, 0).astype(np.int64)
+        if int(mode[b]) == MODE_COPY:
+            n = min(max(int(ncand[b]), 0), W)
+            for w in range(n):
+                ln = int(cand_len[b, w])
+                vcand[b, w, :ln] = cand[b, w, :ln]
+                vlen[b, w] = ln
+        else:
+            n = 1
+            slots = 4 * np.arange(gamma, dtype=np.uint64)
+            coin = harness_key(seed, b, step, slots) & np.uint64(0xFFFFFFFF)
+            alt = _token(harness_key(seed, b, step, slots + np.uint64(1)), V)
+            gg = g[:gamma]
+            alt = np.where(alt == gg, (alt + 1) % V, alt)
+            vcand[b, 0, :gamma] = np.where(coin < thr, gg, alt).astype(np.int32)
+            vlen[b, 0] = gamma
+        vn[b] = n
+        target[b, :n] = g.astype(np.int32)
+    return vcand, vlen, vn, target
