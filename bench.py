@@ -65,6 +65,9 @@ def parse_args(argv=None):
                     help="budget of the CPU-baseline sample")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--candidates", type=int, default=0,
+                    help="W > 0: the step with W copy candidates (§3.3, App. D; the paper's W = 10)")
+    ap.add_argument("--cand-len", type=int, default=20, help="D, the candidate length (the paper's 20)")
     ap.add_argument("--task", default="step", choices=["step", "labels"],
                     help="step: the controller step (the headline); labels: copy-mode labels (§3.2)")
     ap.add_argument("--verify", default="greedy", choices=["greedy", "sampled"],
@@ -212,7 +215,7 @@ def profiled_traffic(workload: str) -> float | None:
 # CPU oracle timing (baseline and reference arm)
 # ------------------------------------------------------------------------------------------------
 def time_oracle(wl: synth.Workload, budget_s: float, max_steps: int, rows: int | None = None,
-                warmup: int = 0, sampled: bool = False):
+                warmup: int = 0, sampled: bool = False, cand: tuple[int, int] | None = None):
     """Runs the oracle loop (oracle step, host target stand-in, oracle verify) on rows [0, R):
     ``warmup`` untimed steps, then up to max_steps timed steps or until budget_s of oracle time is
     spent.  Returns (seq*steps, seconds, timed_steps, R).  Only the oracle's calls are timed."""
@@ -226,6 +229,24 @@ def time_oracle(wl: synth.Workload, budget_s: float, max_steps: int, rows: int |
     done = 0
     for t in range(warmup + max_steps):
         h = wl.hidden(t)
+        if cand is not None:
+            Wc, Dc = cand
+            t0 = time.perf_counter()
+            out = oracle.step_candidates(ctx, lens, h, pw, W=Wc, D=Dc, n_min=wl.n_min, n_max=wl.n_max,
+                                         kappa=wl.kappa, logit_tau=wl.logit_tau, probe_kind=wl.probe_kind,
+                                         probe_hidden=wl.probe_hidden, rows=(0, R))
+            dt = time.perf_counter() - t0
+            vc, vl, vn, tg = synth.harness_candidates(hp, t, lens, out["mode"], out["cand"], out["cand_len"],
+                                                      out["ncand"], future, rows=range(R))
+            t0 = time.perf_counter()
+            oracle.verify_candidates(ctx, lens, vc, vl, vn, tg, rows=(0, R))
+            dt += time.perf_counter() - t0
+            if t >= warmup:
+                spent += dt
+                done += 1
+                if spent >= budget_s:
+                    break
+            continue
         t0 = time.perf_counter()
         out = oracle.step(ctx, lens, h, pw, k=wl.k, n_min=wl.n_min, n_max=wl.n_max, kappa=wl.kappa,
                           logit_tau=wl.logit_tau, probe_kind=wl.probe_kind,
@@ -251,16 +272,17 @@ def time_oracle(wl: synth.Workload, budget_s: float, max_steps: int, rows: int |
     return R * done, spent, done, R
 
 
-def cpu_baseline(wl: synth.Workload, budget_s: float, sampled: bool = False) -> dict:
-    units, secs, steps, R = time_oracle(wl, budget_s, wl.steps, sampled=sampled)
+def cpu_baseline(wl: synth.Workload, budget_s: float, sampled: bool = False, cand=None) -> dict:
+    units, secs, steps, R = time_oracle(wl, budget_s, wl.steps, sampled=sampled, cand=cand)
     return {"value": units / secs, "unit": UNIT, "cores": 1, "kind": "oracle",
             "sample": f"{wl.name}: rows 0..{R - 1}, first {steps} controller steps (oracle step + "
                       f"verify timed, single thread; the host target stand-in is not timed)"}
 
 
 def config_of(wl: synth.Workload, world: int, split: int, search: str = "scan",
-              prefetch: bool = True, verify: str = "greedy") -> dict:
+              prefetch: bool = True, verify: str = "greedy", candidates: int = 0, cand_len: int = 0) -> dict:
     return {"workload": wl.name, "search": search, "verify": verify,
+            "candidates": ({"W": candidates, "D": cand_len} if candidates > 0 else None),
             "prefetch": bool(prefetch and search == "scan"), "B": wl.B, "L0": wl.L0, "V": wl.V, "d": wl.d, "k": wl.k,
             "n_min": wl.n_min, "n_max": wl.n_max, "kappa": wl.kappa_eff, "tau": wl.tau,
             "probe": "linear" if wl.probe_kind == 0 else f"mlp{wl.d}x{wl.probe_hidden}",
@@ -280,14 +302,16 @@ def run_reference(args, world, rank):
     wl = base.scaled(steps=args.warmup + args.steps)
     R = wl.B if wl.B <= 64 else 16
     units, secs, steps, R = time_oracle(wl, float("inf"), args.steps, rows=R, warmup=args.warmup,
-                                        sampled=args.verify == "sampled")
+                                        sampled=args.verify == "sampled",
+                                        cand=(args.candidates, args.cand_len) if args.candidates > 0 else None)
     value = units / secs
     line = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
             "steps": args.steps, "warmup": args.warmup,
             "ms_per_step": secs / steps * 1e3, "higher_is_better": True, "scaling": "weak",
             "vs_baseline": None, "dtype": "int32 (search/verify), f64 (probe)", "data": "synthetic",
             "impl": "reference",
-            "config": config_of(base, world, args.split, args.search, not args.no_prefetch, args.verify),
+            "config": config_of(base, world, args.split, args.search, not args.no_prefetch, args.verify,
+                                 args.candidates, args.cand_len),
             "cpu_baseline": {"value": value, "unit": UNIT, "cores": 1, "kind": "oracle",
                              "sample": f"{wl.name}: rows 0..{R - 1}, {args.warmup} untimed + "
                                        f"{steps} timed steps, single thread"},
@@ -313,7 +337,7 @@ class ReplicaLoop:
     switchsd_verify_step on batch i (its rows only); then one target stand-in covers all R*B rows."""
 
     def __init__(self, wl, R, cap, ctx1, lens1, pw, future1, hidden, split, dev, stream,
-                 search="scan", prefetch=True, sampled=False):
+                 search="scan", prefetch=True, sampled=False, cand_w=0, cand_d=20):
         import ctypes
         import torch
         from paper_2609_20186_gb300 import binding as bd, bf16_tensor
@@ -322,6 +346,7 @@ class ReplicaLoop:
         self.lib = bd.load()
         self.R, self.B, self.k, self.cap = R, wl.B, wl.k, cap
         self.sampled = sampled  # verification at T > 0 (the sampled stand-in and rule)
+        self.cw, self.cd = cand_w, cand_d  # W copy candidates of D tokens (0: the single-draft step)
         B, k = wl.B, wl.k
         ctx = np.zeros((B, cap), np.int32)
         ctx[:, : ctx1.shape[1]] = ctx1[:, : min(cap, ctx1.shape[1])]
@@ -382,6 +407,22 @@ class ReplicaLoop:
         hp.stream = sp
         self.hp = hp
         e32, e16 = 4, 2
+        Wc, Dc = max(cand_w, 1), cand_d
+        self.cand, self.clen = torch.zeros(N, Wc, Dc, **i32), torch.zeros(N, Wc, **i32)
+        self.ncand = torch.zeros(N, **i32)
+        self.vcand, self.vclen = torch.zeros(N, Wc, Dc, **i32), torch.zeros(N, Wc, **i32)
+        self.vn, self.ctarget = torch.zeros(N, **i32), torch.zeros(N, Wc, Dc + 1, **i32)
+        self.choice = torch.zeros(N, **i32)
+        self.cvps = []
+        for r in range(R):
+            v = bd.switchsd_candidates_verify_params()
+            v.B, v.cap, v.W, v.D = B, cap, Wc, Dc
+            v.cand_len = self.vclen.data_ptr() + r * B * Wc * 4
+            v.ncand = self.vn.data_ptr() + r * B * 4
+            v.ctx_tokens = self.ctx.data_ptr() + r * B * cap * 4
+            v.ctx_lens = self.lens.data_ptr() + r * B * 4
+            v.status, v.stream = None, sp
+            self.cvps.append(v)
         f32 = dict(dtype=torch.float32, device=dev)
         self.vp = torch.zeros(N, k, **f32)
         self.vq = torch.ones(N, k, **f32)
@@ -402,7 +443,19 @@ class ReplicaLoop:
     def launch(self, r: int, step_index: int, first: bool):
         c = self.rows[r]
         hid = self.hidden.data_ptr() + step_index * self.hstride
-        if first:
+        if self.cw > 0:
+            B, Wc, Dc, o = self.B, self.cw, self.cd, r * self.B
+            if not first:
+                code = self.lib.switchsd_verify_candidates(
+                    self.vcand.data_ptr() + o * Wc * Dc * 4, self.ctarget.data_ptr() + o * Wc * (Dc + 1) * 4,
+                    c["accept"], self.choice.data_ptr() + o * 4, self.ct.byref(self.cvps[r]))
+                if code != 0:
+                    raise RuntimeError(f"switchsd_verify_candidates failed: {code}")
+            code = self.lib.switchsd_step_candidates(
+                c["ctx"], c["lens"], hid, self.probe_w.data_ptr(), self.ct.byref(self.params[r]), Wc, Dc,
+                self.cand.data_ptr() + o * Wc * Dc * 4, self.clen.data_ptr() + o * Wc * 4,
+                self.ncand.data_ptr() + o * 4, c["mode"], c["score"])
+        elif first:
             code = self.lib.switchsd_step(c["ctx"], c["lens"], hid, self.probe_w.data_ptr(),
                                           self.ct.byref(self.params[r]), c["draft"], c["len"], c["mode"],
                                           c["score"])
@@ -421,7 +474,12 @@ class ReplicaLoop:
 
     def harness(self, q: int):
         self.hp.step = q
-        if self.sampled:
+        if self.cw > 0:
+            code = self.lib.switchsd_harness_candidates(
+                self.lens.data_ptr(), self.mode.data_ptr(), self.cand.data_ptr(), self.clen.data_ptr(),
+                self.ncand.data_ptr(), self.future.data_ptr(), self.cw, self.cd, self.vcand.data_ptr(),
+                self.vclen.data_ptr(), self.vn.data_ptr(), self.ctarget.data_ptr(), self.ct.byref(self.hp))
+        elif self.sampled:
             code = self.lib.switchsd_harness_sampled(
                 self.lens.data_ptr(), self.mode.data_ptr(), self.draft.data_ptr(), self.len.data_ptr(),
                 self.future.data_ptr(), self.vdraft.data_ptr(), self.vlen.data_ptr(), self.vp.data_ptr(),
@@ -448,6 +506,8 @@ def run_ours(args, world, rank, local):
         raise SystemExit("bench.py needs a CUDA device (the controller has no CPU path)")
     if args.verify == "sampled" and args.search == "index":
         raise SystemExit("--verify sampled runs the rescan (the index keeps to greedy verification)")
+    if args.candidates > 0 and (args.search == "index" or args.verify == "sampled"):
+        raise SystemExit("--candidates runs the rescan with greedy verification")
     torch.cuda.set_device(local)
     dev = torch.device("cuda", local)
     binding.load()
@@ -462,7 +522,8 @@ def run_ours(args, world, rank, local):
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         import oracle
         oracle.build()
-        cpu = cpu_baseline(base, args.cpu_seconds, sampled=args.verify == "sampled")
+        cpu = cpu_baseline(base, args.cpu_seconds, sampled=args.verify == "sampled",
+                           cand=(args.candidates, args.cand_len) if args.candidates > 0 else None)
 
     # Replica batches: enough of them that the timed loop reads every batch from HBM.
     R = choose_replicas(B * (base.L0 + 1024) * 4, l2, K)
@@ -481,7 +542,8 @@ def run_ours(args, world, rank, local):
     hidden = bf16_tensor(hidden_host, dev)
     cs = torch.cuda.Stream(dev)
     loop = ReplicaLoop(wl, R, cap, ctx1, lens1, pw, future1, hidden, args.split, dev, cs,
-                       search=args.search, prefetch=not args.no_prefetch, sampled=args.verify == "sampled")
+                       search=args.search, prefetch=not args.no_prefetch, sampled=args.verify == "sampled",
+                       cand_w=args.candidates, cand_d=args.cand_len)
     ctx_bytes_all = R * B * cap * 4
 
     with torch.cuda.stream(cs):
@@ -547,6 +609,12 @@ def run_ours(args, world, rank, local):
         # lens r/w; per tested position the draft and target (sampled: also p, q, u) read, the append
         verify_rw = 8 * B + (28 if args.verify == "sampled" else 16) * grow.sum(axis=1)
         outputs = 12 * B + 4 * B * k                       # mode, len, score, draft (bound)
+        if args.candidates > 0:
+            # the W candidates and the target's tokens for each are read by the verification; the
+            # candidates, their lengths and count written by the step (bounds)
+            Wc, Dc = args.candidates, args.cand_len
+            verify_rw = 8 * B + 4 * B * Wc * (2 * Dc + 2) + 4 * grow.sum(axis=1)
+            outputs = 12 * B + 4 * B * Wc * (Dc + 1)
         if args.search == "index":
             # index path: per row the context tail, and per n one head read and one candidate
             # compare (at least), plus one head and chain write per appended position
@@ -570,7 +638,7 @@ def run_ours(args, world, rank, local):
     cold = cold_latency(loop, dev, cs, warm_rounds + rounds, l2)
 
     e2e = None
-    if not args.no_e2e:
+    if not args.no_e2e and args.candidates == 0:  # the public-API loop covers the single-draft step
         e2e = run_e2e(base, dev, W, K, args.split, world, prefetch=not args.no_prefetch,
                       sampled=args.verify == "sampled")
 
@@ -581,7 +649,8 @@ def run_ours(args, world, rank, local):
         "ms_per_step": ms_per_step, "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "dtype": "int32 (search/verify), bf16 in / fp32 accumulate (probe)",
         "data": "synthetic",
-        "config": dict(config_of(base, world, args.split, args.search, not args.no_prefetch, args.verify),
+        "config": dict(config_of(base, world, args.split, args.search, not args.no_prefetch, args.verify,
+                                 args.candidates, args.cand_len),
                        replicas=R,
                        l2=f"inputs larger than L2: {R} independent batches of B={B} "
                           f"({ctx_bytes_all / 2**20:.0f} MiB of contexts vs {l2 / 2**20:.0f} MiB L2), "
@@ -598,8 +667,8 @@ def run_ours(args, world, rank, local):
         "controller": {"cold_single_launch_us": cold, "search": args.search,
                        "scan_equivalent_gbs": float(4 * Lh[1:].sum(axis=2).mean() / per_launch_s / 1e9),
                        "mean_context_tokens": float(Lh[1:].mean()),
-                       "launches_per_step": 1 if wl.probe_kind == 0 else 2},
-        "gpu_launches": K * (1 if wl.probe_kind == 0 else 2) + rounds,
+                       "launches_per_step": (1 if wl.probe_kind == 0 else 2) + (args.candidates > 0)},
+        "gpu_launches": K * ((1 if wl.probe_kind == 0 else 2) + (args.candidates > 0)) + rounds,
         "gpu_launches_note": "switchsd_verify_step launches (plus the two-layer probe kernel when "
                              "used) and one target stand-in launch per round, all in one CUDA graph",
         "clocks": clocks,
