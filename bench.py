@@ -445,16 +445,17 @@ class ReplicaLoop:
         hid = self.hidden.data_ptr() + step_index * self.hstride
         if self.cw > 0:
             B, Wc, Dc, o = self.B, self.cw, self.cd, r * self.B
-            if not first:
-                code = self.lib.switchsd_verify_candidates(
+            outs = (self.cand.data_ptr() + o * Wc * Dc * 4, self.clen.data_ptr() + o * Wc * 4,
+                    self.ncand.data_ptr() + o * 4, c["mode"], c["score"])
+            if first:
+                code = self.lib.switchsd_step_candidates(c["ctx"], c["lens"], hid, self.probe_w.data_ptr(),
+                                                         self.ct.byref(self.params[r]), Wc, Dc, *outs)
+            else:  # verification of the previous candidates and the next step, fused
+                code = self.lib.switchsd_verify_candidates_step(
                     self.vcand.data_ptr() + o * Wc * Dc * 4, self.ctarget.data_ptr() + o * Wc * (Dc + 1) * 4,
-                    c["accept"], self.choice.data_ptr() + o * 4, self.ct.byref(self.cvps[r]))
-                if code != 0:
-                    raise RuntimeError(f"switchsd_verify_candidates failed: {code}")
-            code = self.lib.switchsd_step_candidates(
-                c["ctx"], c["lens"], hid, self.probe_w.data_ptr(), self.ct.byref(self.params[r]), Wc, Dc,
-                self.cand.data_ptr() + o * Wc * Dc * 4, self.clen.data_ptr() + o * Wc * 4,
-                self.ncand.data_ptr() + o * 4, c["mode"], c["score"])
+                    self.vclen.data_ptr() + o * Wc * 4, self.vn.data_ptr() + o * 4, c["accept"],
+                    self.choice.data_ptr() + o * 4, c["ctx"], c["lens"], hid, self.probe_w.data_ptr(),
+                    self.ct.byref(self.params[r]), Wc, Dc, *outs)
         elif first:
             code = self.lib.switchsd_step(c["ctx"], c["lens"], hid, self.probe_w.data_ptr(),
                                           self.ct.byref(self.params[r]), c["draft"], c["len"], c["mode"],
@@ -667,8 +668,8 @@ def run_ours(args, world, rank, local):
         "controller": {"cold_single_launch_us": cold, "search": args.search,
                        "scan_equivalent_gbs": float(4 * Lh[1:].sum(axis=2).mean() / per_launch_s / 1e9),
                        "mean_context_tokens": float(Lh[1:].mean()),
-                       "launches_per_step": (1 if wl.probe_kind == 0 else 2) + (args.candidates > 0)},
-        "gpu_launches": K * ((1 if wl.probe_kind == 0 else 2) + (args.candidates > 0)) + rounds,
+                       "launches_per_step": 1 if wl.probe_kind == 0 else 2},
+        "gpu_launches": K * (1 if wl.probe_kind == 0 else 2) + rounds,
         "gpu_launches_note": "switchsd_verify_step launches (plus the two-layer probe kernel when "
                              "used) and one target stand-in launch per round, all in one CUDA graph",
         "clocks": clocks,

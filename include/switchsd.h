@@ -378,6 +378,21 @@ int switchsd_verify_candidates(const int32_t *cand, const int32_t *target, int32
                                const switchsd_candidates_verify_params *vp);
 
 /*
+ * switchsd_verify_candidates then switchsd_step_candidates in one launch (§3.3 "Overall Framework"):
+ * the previous iteration's W candidates (cand [B, W, D], target [B, W, D+1], cand_len [B, W], ncand
+ * [B], as switchsd_verify_candidates) are verified and the kept one appended, then the next
+ * candidates are searched on the extended context.  out_accept / out_choice as
+ * switchsd_verify_candidates; the other arguments as switchsd_step_candidates (the verified and the new
+ * candidate buffers must not alias).  params->status: as switchsd_verify_step.
+ */
+int switchsd_verify_candidates_step(const int32_t *cand, const int32_t *target, const int32_t *cand_len,
+                                    const int32_t *ncand, int32_t *out_accept, int32_t *out_choice,
+                                    int32_t *ctx_tokens, int32_t *ctx_lens, const uint16_t *hidden,
+                                    const uint16_t *probe_w, const switchsd_params *params, int32_t W, int32_t D,
+                                    int32_t *out_cand, int32_t *out_cand_len, int32_t *out_ncand, int32_t *out_mode,
+                                    float *out_score);
+
+/*
  * Copy-mode labels (§3.2, "Problem Formulation"): the probe's training labels.  Position j of row b is
  * labelled 1 when it lies in a window of n consecutive tokens that also occurs starting at an earlier
  * position of the row (the paper uses n = n_train = 5); every other position 0.  The same exact token

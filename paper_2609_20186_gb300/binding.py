@@ -99,6 +99,9 @@ _SIGNATURES = {
                                  + [ctypes.c_void_p] * 5),
     "switchsd_verify_candidates": (ctypes.c_int, [ctypes.c_void_p] * 4
                                    + [ctypes.POINTER(switchsd_candidates_verify_params)]),
+    "switchsd_verify_candidates_step": (ctypes.c_int, [ctypes.c_void_p] * 10 + [ctypes.POINTER(switchsd_params),
+                                                                             ctypes.c_int32, ctypes.c_int32]
+                                        + [ctypes.c_void_p] * 5),
     "switchsd_harness_candidates": (ctypes.c_int, [ctypes.c_void_p] * 6 + [ctypes.c_int32, ctypes.c_int32]
                                     + [ctypes.c_void_p] * 4 + [ctypes.POINTER(switchsd_harness_params)]),
     "switchsd_labels_workspace_bytes": (ctypes.c_size_t, [ctypes.c_int32, ctypes.c_int32]),

@@ -76,6 +76,9 @@ struct StepArgs {
     int32_t *out_match_n, *out_match_end, *status;
     int32_t W, D, bm_words;   // candidate mode: W candidates of up to D tokens; bitmap words per CTA
     int32_t *out_cand, *out_cand_len, *out_ncand;
+    const int32_t *pv_cand_len;  // candidate mode, verifying: the previous candidates' lengths [B, W]
+                                 // (pv_draft [B, W, D], pv_target [B, W, D+1], pv_len = their count [B])
+    int32_t *out_choice;         // ... and the kept candidate [B]
 };
 
 __device__ __forceinline__ float dot8_bf16(uint4 w, uint4 h, float acc) {
@@ -126,6 +129,7 @@ __global__ void __launch_bounds__(kStepThreads) step_kernel(const StepArgs a) {
     __shared__ int32_t s_out[2];                               // leader: winner rank, draft length
     __shared__ __align__(16) int32_t s_cand[kMaxCand];         // candidate mode: this CTA's / the row's ends
     __shared__ int32_t s_ncand;
+    __shared__ int32_t s_choice;                               // candidate verification: the kept candidate
 
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     const uint32_t rank = cluster_ctarank();
@@ -261,7 +265,48 @@ __global__ void __launch_bounds__(kStepThreads) step_kernel(const StepArgs a) {
         // Verification of the previous draft (every CTA of the row computes the same result).  Lane i
         // reads draft[i], draft[i+32], target[i], target[i+32] and (lane 0) target[64].
         int32_t acc = -1, L = L_old, vst = len_ok ? SWITCHSD_ROW_OK : SWITCHSD_ROW_BAD_LEN;
-        if (verifying && len_ok) {
+        if (kCand && verifying && len_ok) {
+            // The W previous candidates verified at once (§3.3): lane i tests positions i and i + 32
+            // of every candidate; the longest accepted one is kept (the lowest index on a tie).  Every
+            // slot's tokens are loaded without waiting for its length, so the loads go out together.
+            const int32_t nc = a.pv_len[b];
+            int32_t best = -1, best_w = 0;
+            bool badlen = nc < 0 || nc > a.W;
+            const int ncx = badlen ? 0 : (nc > 0 ? nc : 1);
+#pragma unroll
+            for (int w = 0; w < kMaxCand; ++w) {
+                if (w < ncx) {
+                    const size_t o = size_t(b) * a.W + w;
+                    const int32_t *c = a.pv_draft + o * a.D;
+                    const int32_t *t = a.pv_target + o * (a.D + 1);
+                    const int32_t c_lo = lane < a.D ? c[lane] : 0, c_hi = lane + 32 < a.D ? c[lane + 32] : 0;
+                    const int32_t t_lo = lane < a.D ? t[lane] : 0, t_hi = lane + 32 < a.D ? t[lane + 32] : 0;
+                    const int32_t len = nc > 0 ? a.pv_cand_len[o] : 0;
+                    badlen |= len < 0 || len > a.D;
+                    const unsigned m_lo = __ballot_sync(kFull, lane < len && c_lo != t_lo);
+                    const unsigned m_hi = __ballot_sync(kFull, lane + 32 < len && c_hi != t_hi);
+                    const int32_t acc_w = m_lo ? __ffs(m_lo) - 1 : (m_hi ? 32 + __ffs(m_hi) - 1 : len);
+                    if (acc_w > best) {
+                        best = acc_w;
+                        best_w = w;
+                    }
+                }
+            }
+            if (badlen) {
+                vst = SWITCHSD_ROW_BAD_LEN;
+            } else if (L_old + best + 1 > a.cap) {
+                vst = SWITCHSD_ROW_CAPACITY;
+            } else {
+                const size_t o = size_t(b) * a.W + best_w;
+                const int32_t *c = a.pv_draft + o * a.D;
+                if (lane < best) s_app[lane] = c[lane];
+                if (lane + 32 < best) s_app[lane + 32] = c[lane + 32];
+                if (lane == 0) s_app[best] = a.pv_target[o * (a.D + 1) + best];
+                acc = best;
+                L = L_old + best + 1;
+            }
+            if (lane == 0) s_choice = best_w;
+        } else if (verifying && len_ok) {
             const int32_t *dr = a.pv_draft + size_t(b) * a.k;
             const int32_t *tg = a.pv_target + size_t(b) * (a.k + 1);
             const int32_t pv_n = a.pv_len[b];
@@ -585,6 +630,7 @@ __global__ void __launch_bounds__(kStepThreads) step_kernel(const StepArgs a) {
             if (a.out_match_n) a.out_match_n[b] = n;
             if (a.out_match_end) a.out_match_end[b] = e;
             if (verifying && !len_ok) a.out_accept[b] = -1;
+            if (kCand && verifying && a.out_choice) a.out_choice[b] = len_ok ? s_choice : 0;
             if (a.status) {
                 int32_t st = s_ver[2];
                 if (st == SWITCHSD_ROW_OK && timeout) st = SWITCHSD_ROW_TIMEOUT;
@@ -659,6 +705,8 @@ static cudaError_t launch_step(const StepArgs &args, int split, cudaStream_t str
 struct CandSpec {
     int32_t W, D;
     int32_t *cand, *cand_len, *ncand;
+    const int32_t *pv_cand_len;  // fused verification of the previous candidates (null: none)
+    int32_t *out_choice;
 };
 
 // Shared validation and launch of switchsd_step / switchsd_verify_step.
@@ -709,7 +757,8 @@ static int step_entry(int32_t *ctx_tokens, int32_t *ctx_lens, const uint16_t *hi
     args.B = p->B;
     args.cap = p->cap;
     args.d = p->d;
-    args.k = p->k;
+    // candidate mode: a verified candidate appends up to D + 1 tokens, so the staged look-ahead covers D
+    args.k = cs ? (p->k > cs->D ? p->k : cs->D) : p->k;
     args.n_min = p->n_min;
     args.n_max = p->n_max;
     args.kappa = p->kappa;
@@ -727,7 +776,7 @@ static int step_entry(int32_t *ctx_tokens, int32_t *ctx_lens, const uint16_t *hi
     // Tile: the largest CTA range (the last CTA may also cover a k + 1 token append), in one stage
     // when it fits, else a ring of kTileMax stages, as many as the range needs up to kMaxStages and
     // the shared-memory budget.
-    const int64_t range = ((int64_t(p->cap) - 1 + split - 1) / split + 3) / 4 * 4 + p->k + 1;
+    const int64_t range = ((int64_t(p->cap) - 1 + split - 1) / split + 3) / 4 * 4 + args.k + 1;
     // candidate mode: a bit per end of the CTA's range, after the stages
     args.W = cs ? cs->W : 0;
     args.D = cs ? cs->D : 0;
@@ -735,6 +784,8 @@ static int step_entry(int32_t *ctx_tokens, int32_t *ctx_lens, const uint16_t *hi
     args.out_cand = cs ? cs->cand : nullptr;
     args.out_cand_len = cs ? cs->cand_len : nullptr;
     args.out_ncand = cs ? cs->ncand : nullptr;
+    args.pv_cand_len = cs ? cs->pv_cand_len : nullptr;
+    args.out_choice = cs ? cs->out_choice : nullptr;
     const size_t budget = kStageSmemBudget - size_t(args.bm_words) * sizeof(uint32_t);
     if (range <= kTileMax) {
         args.tile = int32_t((range + 3) / 4 * 4);
@@ -803,10 +854,22 @@ extern "C" int switchsd_step_candidates(const int32_t *ctx_tokens, const int32_t
                                         const uint16_t *probe_w, const switchsd_params *p, int32_t W, int32_t D,
                                         int32_t *out_cand, int32_t *out_cand_len, int32_t *out_ncand,
                                         int32_t *out_mode, float *out_score) {
-    const CandSpec cs{W, D, out_cand, out_cand_len, out_ncand};
+    const CandSpec cs{W, D, out_cand, out_cand_len, out_ncand, nullptr, nullptr};
     return step_entry(const_cast<int32_t *>(ctx_tokens), const_cast<int32_t *>(ctx_lens), hidden, probe_w, p,
                       nullptr, nullptr, nullptr, nullptr, nullptr, nullptr, out_mode, out_score, nullptr, nullptr,
                       nullptr, &cs);
+}
+
+extern "C" int switchsd_verify_candidates_step(const int32_t *cand, const int32_t *target, const int32_t *cand_len,
+                                               const int32_t *ncand, int32_t *out_accept, int32_t *out_choice,
+                                               int32_t *ctx_tokens, int32_t *ctx_lens, const uint16_t *hidden,
+                                               const uint16_t *probe_w, const switchsd_params *p, int32_t W,
+                                               int32_t D, int32_t *out_cand, int32_t *out_cand_len,
+                                               int32_t *out_ncand, int32_t *out_mode, float *out_score) {
+    if (!cand || !target || !cand_len || !ncand || !out_accept || !out_choice) return SWITCHSD_ERR_ARG;
+    const CandSpec cs{W, D, out_cand, out_cand_len, out_ncand, cand_len, out_choice};
+    return step_entry(ctx_tokens, ctx_lens, hidden, probe_w, p, cand, target, ncand, out_accept, nullptr, nullptr,
+                      out_mode, out_score, nullptr, nullptr, nullptr, &cs);
 }
 
 extern "C" int switchsd_verify_sampled_step(const int32_t *draft, const float *p_draft, const float *q_draft,

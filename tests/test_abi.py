@@ -48,6 +48,14 @@ def test_every_declared_symbol_is_exported(lib):
         assert hasattr(lib, name)
 
 
+def test_binding_declares_every_function():
+    """Every function of include/*.h has a ctypes signature in the binding (an undeclared one would
+    pass 64-bit device pointers through ctypes' default int conversion)."""
+    from paper_2609_20186_gb300 import binding as bd
+    missing = sorted(set(declared_functions()) - set(bd._SIGNATURES))
+    assert missing == []
+
+
 def test_abi_version_and_strerror(lib):
     from paper_2609_20186_gb300 import binding as bd
     assert bd.abi_version() == 2

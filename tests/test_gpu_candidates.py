@@ -55,7 +55,9 @@ def oracle_loop(wl, rows, steps, Wc, D):
     return trace, ctx
 
 
-def gpu_loop(wl, steps, Wc, D, split=0):
+def gpu_loop(wl, steps, Wc, D, split=0, fused=False):
+    """fused: switchsd_verify_candidates_step verifies iteration t-1's candidates and searches step t's in
+    one launch; the last iteration's candidates are verified by switchsd_verify_candidates."""
     import torch
     from paper_2609_20186_gb300 import binding as bd, bf16_tensor
     lib = bd.load()
@@ -95,9 +97,18 @@ def gpu_loop(wl, steps, Wc, D, split=0):
     trace = []
     for t in range(steps):
         hid = bf16_tensor(wl.hidden(t), dev)
-        assert lib.switchsd_step_candidates(c.data_ptr(), ln.data_ptr(), hid.data_ptr(), pw.data_ptr(),
-                                            ctypes.byref(p), Wc, D, cand.data_ptr(), clen.data_ptr(),
-                                            ncand.data_ptr(), mode.data_ptr(), score.data_ptr()) == 0
+        if fused and t > 0:
+            assert lib.switchsd_verify_candidates_step(
+                vc.data_ptr(), tg.data_ptr(), vl.data_ptr(), vn.data_ptr(), acc.data_ptr(), ch.data_ptr(),
+                c.data_ptr(), ln.data_ptr(), hid.data_ptr(), pw.data_ptr(), ctypes.byref(p), Wc, D, cand.data_ptr(),
+                clen.data_ptr(), ncand.data_ptr(), mode.data_ptr(), score.data_ptr()) == 0
+            s_ = st.cpu().numpy()
+            trace[-1].update(accept=acc.cpu().numpy(), choice=ch.cpu().numpy(), lens_after=ln.cpu().numpy(),
+                             vstatus=np.where((s_ == 1) | (s_ == 2), s_, 0))
+        else:
+            assert lib.switchsd_step_candidates(c.data_ptr(), ln.data_ptr(), hid.data_ptr(), pw.data_ptr(),
+                                                ctypes.byref(p), Wc, D, cand.data_ptr(), clen.data_ptr(),
+                                                ncand.data_ptr(), mode.data_ptr(), score.data_ptr()) == 0
         out = {"cand": cand.cpu().numpy(), "cand_len": clen.cpu().numpy(), "ncand": ncand.cpu().numpy(),
                "mode": mode.cpu().numpy(), "score": score.cpu().numpy(), "match_n": mn.cpu().numpy(),
                "match_end": me.cpu().numpy(), "status": st.cpu().numpy()}
@@ -105,10 +116,11 @@ def gpu_loop(wl, steps, Wc, D, split=0):
         assert lib.switchsd_harness_candidates(ln.data_ptr(), mode.data_ptr(), cand.data_ptr(), clen.data_ptr(),
                                                ncand.data_ptr(), fut.data_ptr(), Wc, D, vc.data_ptr(), vl.data_ptr(),
                                                vn.data_ptr(), tg.data_ptr(), ctypes.byref(hp)) == 0
-        assert lib.switchsd_verify_candidates(vc.data_ptr(), tg.data_ptr(), acc.data_ptr(), ch.data_ptr(),
-                                              ctypes.byref(vp)) == 0
-        out.update(accept=acc.cpu().numpy(), choice=ch.cpu().numpy(), lens_after=ln.cpu().numpy(),
-                   vstatus=vst.cpu().numpy())
+        if not fused or t == steps - 1:
+            assert lib.switchsd_verify_candidates(vc.data_ptr(), tg.data_ptr(), acc.data_ptr(), ch.data_ptr(),
+                                                  ctypes.byref(vp)) == 0
+            out.update(accept=acc.cpu().numpy(), choice=ch.cpu().numpy(), lens_after=ln.cpu().numpy(),
+                       vstatus=vst.cpu().numpy())
         trace.append(out)
     torch.cuda.synchronize()
     return trace, c.cpu().numpy()
@@ -143,13 +155,14 @@ def compare(wl, o_trace, g_trace, rows, o_ctx, g_ctx):
     return checked, copies
 
 
+@pytest.mark.parametrize("fused", [False, True], ids=["separate", "fused"])
 @pytest.mark.parametrize("Wc,D", [(10, 20), (3, 8), (16, 64), (1, 4)])
 @pytest.mark.parametrize("name", list(SMALL))
-def test_candidates_lockstep(name, Wc, D):
+def test_candidates_lockstep(name, Wc, D, fused):
     wl = SMALL[name]
     rows = range(wl.B)
     o_trace, o_ctx = oracle_loop(wl, rows, wl.steps, Wc, D)
-    g_trace, g_ctx = gpu_loop(wl, wl.steps, Wc, D)
+    g_trace, g_ctx = gpu_loop(wl, wl.steps, Wc, D, fused=fused)
     checked, copies = compare(wl, o_trace, g_trace, rows, o_ctx, g_ctx)
     assert checked > 0
 
@@ -175,7 +188,7 @@ def test_candidates_multi_stage_ring():
 
 def test_candidates_full_size_sampled_rows():
     wl = W["zipf_32k"].scaled(steps=8)
-    g_trace, g_ctx = gpu_loop(wl, wl.steps, 10, 20)
+    g_trace, g_ctx = gpu_loop(wl, wl.steps, 10, 20, fused=True)
     rows = [0, 21, 42, 63]
     o_trace, o_ctx = oracle_loop(wl, rows, wl.steps, 10, 20)
     checked, copies = compare(wl, o_trace, g_trace, rows, o_ctx, g_ctx)
