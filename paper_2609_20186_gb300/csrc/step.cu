@@ -428,6 +428,13 @@ __global__ void __launch_bounds__(kStepThreads) step_kernel(const StepArgs a) {
                     const int32_t g = g0 + u * kStepThreads;
                     v[u] = g < n4 ? g4[g] : make_int4(0, 0, 0, 0);
                 }
+                // One predicate for the four words first: most words hold no first-token hit, and the
+                // bit masks are only built for those that do.
+                bool any = false;
+#pragma unroll
+                for (int u = 0; u < 4; ++u)
+                    any |= (v[u].x == s0) | (v[u].y == s0) | (v[u].z == s0) | (v[u].w == s0);
+                if (!any) continue;
 #pragma unroll
                 for (int u = 0; u < 4; ++u) {
                     const int32_t g = g0 + u * kStepThreads;
@@ -637,10 +644,14 @@ __global__ void __launch_bounds__(kStepThreads) step_kernel(const StepArgs a) {
                 a.status[b] = st;
             }
         }
+        // The copy draft from the winner's message (every lane knows win and len).
+        if (!kCand)
+            for (int i = lane; i < len; i += kWarp) a.out_draft[size_t(b) * a.k + i] = s_slot[win].cand[i];
     }
-    __syncthreads();
     if (kCand) {
-        // The candidates' continuations, read from the row (the context is not modified in this mode).
+        __syncthreads();
+        // The candidates' continuations, read from the row (the leader's append, if any, is visible
+        // to its threads after the barrier).
         const int nc = s_ncand;
         if (tid == 0) a.out_ncand[b] = nc;
         for (int t = tid; t < nc * a.D; t += kStepThreads) {
@@ -650,10 +661,7 @@ __global__ void __launch_bounds__(kStepThreads) step_kernel(const StepArgs a) {
             if (i == 0) a.out_cand_len[size_t(b) * a.W + w] = lw;
             if (i < lw) a.out_cand[(size_t(b) * a.W + w) * a.D + i] = row[ew + 1 + i];
         }
-        return;
     }
-    const int32_t win = s_out[0], len = s_out[1];
-    for (int i = tid; i < len; i += kStepThreads) a.out_draft[size_t(b) * a.k + i] = s_slot[win].cand[i];
 }
 
 // ------------------------------------------------------------------------------------------------
