@@ -41,7 +41,7 @@
 extern "C" {
 #endif
 
-#define SWITCHSD_ABI_VERSION 2
+#define SWITCHSD_ABI_VERSION 3
 
 #define SWITCHSD_NMAX 32 /* largest supported n_max */
 #define SWITCHSD_KMAX 64 /* largest supported draft length k */
@@ -118,6 +118,13 @@ typedef struct switchsd_index switchsd_index;
  *                and the target argmax are always read after the wait.  The index search ignores the
  *                field; with the two-layer probe SWITCHSD_PREFETCH_PROBE lets the probe kernel's copies
  *                of the hidden states and W1 start early.  Other bits are SWITCHSD_ERR_ARG.
+ *   hidden_rows  0 or 1: hidden is [B, d], the state the probe reads for each row.  k + 1 (the fused
+ *                switchsd_verify_step and switchsd_verify_sampled_step only, linear probe, no index):
+ *                hidden is the target's verification output [B, k+1, d] and the probe reads row a_b of
+ *                each row b -- the state that produced the appended token t[a_b], the most recent one the
+ *                target computed -- or row 0 when nothing was appended (capacity, bad lengths).  The
+ *                probe's copies then wait for the verification; SWITCHSD_PREFETCH_PROBE is ignored.
+ *                Any other value is SWITCHSD_ERR_ARG.
  */
 typedef struct {
     int32_t B, cap, d, k, n_min, n_max, kappa;
@@ -135,6 +142,7 @@ typedef struct {
     int32_t *status;
     void *stream;
     int32_t prefetch;
+    int32_t hidden_rows;
 } switchsd_params;
 
 /*

@@ -70,6 +70,7 @@ struct StepArgs {
     int32_t *out_accept;
     int32_t B, cap, d, k, n_min, n_max, kappa, tile, stages;
     int32_t prefetch;        // SWITCHSD_PREFETCH_* bits: reads that may precede the grid-dependency wait
+    int32_t hidden_rows;     // > 1: hidden is [B, hidden_rows, d] and the probe reads row a_b (verifying)
     float logit_tau;
     int32_t *out_draft, *out_len, *out_mode;
     float *out_score;
@@ -179,7 +180,10 @@ __global__ void __launch_bounds__(kStepThreads) step_kernel(const StepArgs a) {
         m_staged = a.mlp_S * ucnt4 <= 2 * kProbeStage * 4;
     }
     const int v_staged = min(v1 - v0, kProbeStage);
-    const uint4 *h4 = reinterpret_cast<const uint4 *>(a.hidden + size_t(b) * size_t(a.d));
+    // gather: the probe reads the row a_b of the target's [B, k+1, d] output, known after the verification
+    const bool gather = verifying && a.hidden_rows > 1;
+    const uint4 *h4 = reinterpret_cast<const uint4 *>(a.hidden + size_t(b) * size_t(gather ? a.hidden_rows : 1) *
+                                                                  size_t(a.d));
     const uint4 *w4 = reinterpret_cast<const uint4 *>(a.probe_w);
     auto issue_probe = [&]() {
         if (!mlp) {
@@ -199,7 +203,7 @@ __global__ void __launch_bounds__(kStepThreads) step_kernel(const StepArgs a) {
         }
     };
     // The partial sums come from the kernel just before this one: never staged before the wait.
-    if (pf_probe && !mlp && tid == 2 * kWarp) issue_probe();
+    if (pf_probe && !mlp && !gather && tid == 2 * kWarp) issue_probe();
     if (!pf_ctx) pdl_wait();
 
     // Warp roles until the suffix is known.  Warp 0 reads the row length and issues the copies at
@@ -350,10 +354,14 @@ __global__ void __launch_bounds__(kStepThreads) step_kernel(const StepArgs a) {
             s_ver[0] = acc;
             s_ver[1] = L;
             s_ver[2] = vst;
+            if (gather) {  // the probe's slice of hidden row a_b (row 0 when nothing was appended)
+                h4 += size_t(acc > 0 ? acc : 0) * size_t(a.d >> 3);
+                issue_probe();
+            }
         }
         cluster_arrive_release();
     } else {
-        if ((!pf_probe || mlp) && tid == 2 * kWarp) issue_probe();
+        if ((!pf_probe || mlp) && !gather && tid == 2 * kWarp) issue_probe();
         if (kCand) {
             uint32_t *bm = reinterpret_cast<uint32_t *>(tiles + a.stages * stage_ints);
             for (int i = tid - 2 * kWarp; i < a.bm_words; i += kStepThreads - 2 * kWarp) bm[i] = 0u;
@@ -389,6 +397,7 @@ __global__ void __launch_bounds__(kStepThreads) step_kernel(const StepArgs a) {
 
     const int32_t acc = s_ver[0], L = s_ver[1];
     const int32_t E = len_ok ? L - 1 : 0;  // candidate ends after the append: [0, E)
+    if (gather && !(warp == 1 && lane == 0)) h4 += size_t(acc > 0 ? acc : 0) * size_t(a.d >> 3);
     const int32_t s0 = s_suf[0], s1 = s_suf[1];
     const int32_t n_max = a.n_max, n_min = a.n_min;
     // With n_min >= 2 a candidate must match the last two tokens, so the filter tests both (exact:
@@ -738,6 +747,12 @@ static int step_entry(int32_t *ctx_tokens, int32_t *ctx_lens, const uint16_t *hi
     if (p->split != 0 && p->split != 1 && p->split != 2 && p->split != 4 && p->split != 8 && p->split != 16)
         return SWITCHSD_ERR_SHAPE;
     if ((p->prefetch & ~(SWITCHSD_PREFETCH_CONTEXT | SWITCHSD_PREFETCH_PROBE)) != 0) return SWITCHSD_ERR_ARG;
+    // hidden_rows: 0 / 1, or k + 1 for the fused greedy / sampled verification with the linear probe
+    if (p->hidden_rows != 0 && p->hidden_rows != 1) {
+        if (p->hidden_rows != p->k + 1 || pv_len == nullptr || cs != nullptr || p->index != nullptr ||
+            p->probe_kind != SWITCHSD_PROBE_LINEAR)
+            return SWITCHSD_ERR_ARG;
+    }
     if (p->probe_kind == SWITCHSD_PROBE_MLP) {
         if (!mlp_shape_ok(p->d, p->probe_hidden)) return SWITCHSD_ERR_SHAPE;
         if (!p->workspace || !aligned16(p->workspace) ||
@@ -779,6 +794,7 @@ static int step_entry(int32_t *ctx_tokens, int32_t *ctx_lens, const uint16_t *hi
     args.out_match_end = p->out_match_end;
     args.status = p->status;
     args.prefetch = p->prefetch;
+    args.hidden_rows = p->hidden_rows > 1 ? p->hidden_rows : 1;
 
     const int split = p->split > 0 ? p->split : choose_split(p->B, p->cap);
     // Tile: the largest CTA range (the last CTA may also cover a k + 1 token append), in one stage

@@ -34,8 +34,9 @@ class Session:
                  probe_kind: int = bd.PROBE_LINEAR, probe_hidden: int = 0, future=None,
                  harness: dict | None = None, split: int = 0, d: int | None = None,
                  use_index: bool = False, device="cuda", stream: torch.cuda.Stream | None = None,
-                 prefetch: int = 0):
+                 prefetch: int = 0, hidden_rows: int = 0):
         self.lib = bd.load()
+        self.hidden_rows = int(hidden_rows)
         self.device = torch.device(device)
         if self.device.type == "cuda" and self.device.index is None:
             self.device = torch.device("cuda", torch.cuda.current_device())
@@ -93,6 +94,7 @@ class Session:
             p.status = self.status.data_ptr() if debug else None
             p.stream = sp
             p.prefetch = int(prefetch)
+            p.hidden_rows = int(hidden_rows)  # k + 1: verify_step reads row a_b of a [B, k+1, d] hidden
             return p
         self._p_dbg, self._p_fast = params(True), params(False)
         self._step_head = (self.ctx.data_ptr(), self.lens.data_ptr())
@@ -140,26 +142,33 @@ class Session:
         self.vu = torch.zeros(B, k, **f32)
 
     # --- the three calls ---------------------------------------------------------------------
-    def _check_hidden(self, hidden: torch.Tensor) -> None:
+    def _check_hidden(self, hidden: torch.Tensor, rows: int = 1) -> None:
+        """hidden: bf16 [B, d], or [B, rows, d] when rows > 1 (the fused verification's gather)."""
+        shape_ok = hidden.shape[0] == self.B and (
+            (rows <= 1 and hidden.dim() == 2) or (rows > 1 and hidden.dim() == 3 and hidden.shape[1] == rows))
         if (hidden.dtype != torch.bfloat16 or hidden.device != self.device
-                or not hidden.is_contiguous() or hidden.shape[0] != self.B
-                or (self.d is not None and hidden.shape[1] != self.d)):
-            raise ValueError("hidden must be a contiguous bf16 [B, d] tensor on the session device")
+                or not hidden.is_contiguous() or not shape_ok
+                or (self.d is not None and hidden.shape[-1] != self.d)):
+            raise ValueError("hidden must be a contiguous bf16 [B, d] (or [B, k+1, d]) tensor on the session device")
         if self.d is None:
             self._p_dbg.d = self._p_fast.d = hidden.shape[1]
             self.d = hidden.shape[1]
 
     def step(self, hidden: torch.Tensor, debug: bool = True) -> None:
+        """switchsd_step (no verification): hidden is [B, d] whatever hidden_rows is."""
         self._check_hidden(hidden)
         p = self._p_dbg if debug else self._p_fast
+        rows, p.hidden_rows = p.hidden_rows, 0
         code = self.lib.switchsd_step(*self._step_head, hidden.data_ptr(), *self._step_tail,
                                       ctypes.byref(p), *self._step_outs)
+        p.hidden_rows = rows
         if code != bd.OK:
             raise RuntimeError(f"switchsd_step failed: {code} ({bd.strerror(code)})")
 
     def verify_step(self, hidden: torch.Tensor, debug: bool = True) -> None:
-        """Verification of the last harness draft (vdraft / target / vlen) and the next step, fused."""
-        self._check_hidden(hidden)
+        """Verification of the last harness draft (vdraft / target / vlen) and the next step, fused.
+        With hidden_rows = k + 1, hidden is the target's [B, k+1, d] output and row a_b is probed."""
+        self._check_hidden(hidden, self.hidden_rows)
         p = self._p_dbg if debug else self._p_fast
         code = self.lib.switchsd_verify_step(*self._vs_head, self.ctx.data_ptr(), self.lens.data_ptr(),
                                              hidden.data_ptr(), *self._step_tail, ctypes.byref(p),
@@ -181,7 +190,7 @@ class Session:
 
     def verify_sampled_step(self, hidden: torch.Tensor, debug: bool = True) -> None:
         """Sampled verification (T > 0) of the last sampled-harness draft and the next step, fused."""
-        self._check_hidden(hidden)
+        self._check_hidden(hidden, self.hidden_rows)
         p = self._p_dbg if debug else self._p_fast
         code = self.lib.switchsd_verify_sampled_step(
             self.vdraft.data_ptr(), self.vp.data_ptr(), self.vq.data_ptr(), self.vu.data_ptr(),
