@@ -231,6 +231,12 @@ __global__ void __launch_bounds__(kStepThreads) step_kernel(const StepArgs a) {
         tail_hi = len_ok ? (L_old + 3) & ~3 : tail_lo;  // <= cap since cap % 4 == 0
     };
     if (warp < 2) set_split(__ldcg(a.lens + b));
+    // Every thread arrives now, before issuing any copy or load: only the length read has to precede
+    // the leader's write of the new length.
+    if (warp < 2)
+        cluster_arrive_release();
+    else
+        cluster_arrive_relaxed();
 
     // Stage tile t: tokens [max(0, t0 - kHalo), min(roundup4(t1 + kFwd), cap)) land so that token p
     // sits at stage[kHalo + p - t0].  cap % 4 == 0 keeps every bound 16-byte aligned.
@@ -263,9 +269,7 @@ __global__ void __launch_bounds__(kStepThreads) step_kernel(const StepArgs a) {
         m_b1 = a.b1 ? a.b1[u0 + tid] : 0.f;
         m_w2 = bf16_lo(uint32_t(a.w2[u0 + tid]));
     }
-    if (warp == 0) {
-        cluster_arrive_release();
-    } else if (warp == 1) {
+    if (warp == 1) {
         // Verification of the previous draft (every CTA of the row computes the same result).  Lane i
         // reads draft[i], draft[i+32], target[i], target[i+32] and (lane 0) target[64].
         int32_t acc = -1, L = L_old, vst = len_ok ? SWITCHSD_ROW_OK : SWITCHSD_ROW_BAD_LEN;
@@ -359,14 +363,12 @@ __global__ void __launch_bounds__(kStepThreads) step_kernel(const StepArgs a) {
                 issue_probe();
             }
         }
-        cluster_arrive_release();
-    } else {
+    } else if (warp >= 2) {
         if ((!pf_probe || mlp) && !gather && tid == 2 * kWarp) issue_probe();
         if (kCand) {
             uint32_t *bm = reinterpret_cast<uint32_t *>(tiles + a.stages * stage_ints);
             for (int i = tid - 2 * kWarp; i < a.bm_words; i += kStepThreads - 2 * kWarp) bm[i] = 0u;
         }
-        cluster_arrive_relaxed();
     }
     // Warps 0 and 1 meet (named barrier 1, 64 threads): the suffix needs the old tail and the append.
     if (warp < 2) {
