@@ -41,6 +41,14 @@ __device__ __forceinline__ void mbar_arrive_expect_tx(uint64_t *bar, uint32_t by
                  : "memory");
 }
 
+// The same for a barrier that only counts an asynchronous copy's bytes: the arriving thread publishes
+// nothing through it, so the arrive needs no release ordering.
+__device__ __forceinline__ void mbar_expect_tx_relaxed(uint64_t *bar, uint32_t bytes) {
+    asm volatile("mbarrier.arrive.expect_tx.relaxed.cta.shared::cta.b64 _, [%0], %1;\n" ::"r"(smem_addr(bar)),
+                 "r"(bytes)
+                 : "memory");
+}
+
 // Bounded wait for phase `parity` of the barrier to complete.  Returns false on timeout.
 __device__ __forceinline__ bool mbar_wait(uint64_t *bar, uint32_t parity) {
     const uint32_t addr = smem_addr(bar);

@@ -188,14 +188,14 @@ __global__ void __launch_bounds__(kStepThreads) step_kernel(const StepArgs a) {
     auto issue_probe = [&]() {
         if (!mlp) {
             const uint32_t pb = uint32_t(v_staged) * 16u;
-            mbar_arrive_expect_tx(&probe_bar, 2u * pb);
+            mbar_expect_tx_relaxed(&probe_bar, 2u * pb);
             if (pb > 0) {
                 bulk_g2s(s_pw, w4 + v0, pb, &probe_bar);
                 bulk_g2s(s_ph, h4 + v0, pb, &probe_bar);
             }
         } else {
             const uint32_t pb = m_staged ? uint32_t(ucnt4) * 4u : 0u;
-            mbar_arrive_expect_tx(&probe_bar, uint32_t(a.mlp_S) * pb);
+            mbar_expect_tx_relaxed(&probe_bar, uint32_t(a.mlp_S) * pb);
             float *dst = reinterpret_cast<float *>(s_probe);
             if (pb > 0)
                 for (int s = 0; s < a.mlp_S; ++s)
@@ -247,13 +247,13 @@ __global__ void __launch_bounds__(kStepThreads) step_kernel(const StepArgs a) {
         const int32_t lo = max(0, t0 - kHalo);
         const int32_t hi = min((t1 + kFwd + 3) & ~3, a.cap);
         const uint32_t bytes = uint32_t(hi - lo) * 4u;
-        mbar_arrive_expect_tx(&bars[s], bytes);
+        mbar_expect_tx_relaxed(&bars[s], bytes);
         bulk_g2s_hint(tiles + s * stage_ints + (kHalo + lo - t0), row + lo, bytes, &bars[s], l2_evict_first_policy());
     };
     if (warp == 0) {
         if (lane == 0) {
             const uint32_t tb = uint32_t(tail_hi - tail_lo) * 4u;
-            mbar_arrive_expect_tx(&tail_bar, tb);
+            mbar_expect_tx_relaxed(&tail_bar, tb);
             if (tb > 0) bulk_g2s_hint(s_tail, row + tail_lo, tb, &tail_bar, l2_evict_first_policy());
             for (int t = 0; t < min(ntiles, a.stages); ++t) issue(t);
             s_split[0] = L_old;
