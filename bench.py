@@ -734,10 +734,7 @@ def run_e2e(base, dev, W, K, split, world, prefetch=True, sampled=False):
     for t in range(W + K):
         host_h[t].copy_(torch.from_numpy(wl.hidden(t).view(np.int16)))
     dev_h = torch.empty(B, d, dtype=torch.bfloat16, device=dev)
-    out_mode = torch.empty(B, dtype=torch.int32).pin_memory()
-    out_len = torch.empty(B, dtype=torch.int32).pin_memory()
-    out_draft = torch.empty(B, k, dtype=torch.int32).pin_memory()
-    out_acc = torch.empty(B, dtype=torch.int32).pin_memory()
+    host_out = torch.empty(B * (k + 3), dtype=torch.int32).pin_memory()  # mode, len, accept, draft
     stream = torch.cuda.current_stream()
 
     def one(t):
@@ -752,10 +749,7 @@ def run_e2e(base, dev, W, K, split, world, prefetch=True, sampled=False):
             sess.harness_sampled(t)
         else:
             sess.harness(t)
-        out_mode.copy_(sess.mode, non_blocking=True)
-        out_len.copy_(sess.len, non_blocking=True)
-        out_draft.copy_(sess.draft, non_blocking=True)
-        out_acc.copy_(sess.accept, non_blocking=True)
+        sess.outputs_to(host_out)  # one D2H copy of mode, draft length, accepted length and draft
         stream.synchronize()
 
     for t in range(W):

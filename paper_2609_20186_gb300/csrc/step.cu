@@ -131,6 +131,7 @@ __global__ void __launch_bounds__(kStepThreads) step_kernel(const StepArgs a) {
     __shared__ __align__(16) int32_t s_cand[kMaxCand];         // candidate mode: this CTA's / the row's ends
     __shared__ int32_t s_ncand;
     __shared__ int32_t s_choice;                               // candidate verification: the kept candidate
+    __shared__ int32_t s_probe_late;                           // early probe: its copies did not land in time
 
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     const uint32_t rank = cluster_ctarank();
@@ -145,6 +146,7 @@ __global__ void __launch_bounds__(kStepThreads) step_kernel(const StepArgs a) {
         for (int s = 0; s < a.stages; ++s) mbar_init(&bars[s], 1);
         mbar_init(&tail_bar, 1);
         mbar_init(&probe_bar, 1);
+        s_probe_late = 0;
         if (rank == 0) {
             mbar_init(&s_done, 1);
             mbar_arrive_expect_tx(&s_done, slot_bytes * C);
@@ -261,6 +263,23 @@ __global__ void __launch_bounds__(kStepThreads) step_kernel(const StepArgs a) {
             s_split[2] = e_hi;
             s_split[3] = ntiles;
         }
+    }
+    // A prefetched linear probe is finished before the wait by warps 2.. (idle until then): its slice was
+    // copied at the very start and nothing the preceding kernel writes enters it.
+    const bool early_probe = pf_probe && !mlp && !gather;
+    if (early_probe && warp >= 2) {
+        float zp = 0.f;
+        const bool in = mbar_wait(&probe_bar, 0);
+        if (in)
+            for (int i = tid - 2 * kWarp; i < v_staged; i += kStepThreads - 2 * kWarp)
+                zp = dot8_bf16(s_pw[i], s_ph[i], zp);
+        for (int v = v0 + v_staged + tid - 2 * kWarp; v < v1; v += kStepThreads - 2 * kWarp)
+            zp = dot8_bf16(__ldg(w4 + v), __ldg(h4 + v), zp);
+        zp = warp_sum_f32(zp);
+        if (lane == 0) s_wz[warp] = zp;
+        if (!in && lane == 0) s_probe_late = 1;  // benign race: every writer stores 1
+    } else if (early_probe && lane == 0) {
+        s_wz[warp] = 0.f;  // warps 0 and 1 hold no share of the early probe
     }
     if (pf_ctx) pdl_wait();  // the previous draft and the target (and all that no bit names) come after this
     pdl_trigger();           // the next kernel may start launching
@@ -518,10 +537,12 @@ __global__ void __launch_bounds__(kStepThreads) step_kernel(const StepArgs a) {
         }
     }
 
-    // The probe slice (staged during the scan), then the CTA's partial in a fixed order.
+    // The probe slice (staged during the scan) unless it was finished before the wait, then the CTA's
+    // partial in a fixed order.
     float zp = 0.f;
-    const bool probe_in = mbar_wait(&probe_bar, 0);
-    if (!mlp) {
+    const bool probe_in = early_probe ? s_probe_late == 0 : mbar_wait(&probe_bar, 0);
+    if (early_probe) {
+    } else if (!mlp) {
         if (probe_in)
             for (int i = tid; i < v_staged; i += kStepThreads) zp = dot8_bf16(s_pw[i], s_ph[i], zp);
         for (int v = v0 + v_staged + tid; v < v1; v += kStepThreads)
@@ -544,8 +565,10 @@ __global__ void __launch_bounds__(kStepThreads) step_kernel(const StepArgs a) {
         best = kTimeoutBit;
         (void)mbar_wait(&probe_bar, 0);  // a second bounded wait before the CTA's memory goes away
     }
-    zp = warp_sum_f32(zp);
-    if (lane == 0) s_wz[warp] = zp;
+    if (!early_probe) {
+        zp = warp_sum_f32(zp);
+        if (lane == 0) s_wz[warp] = zp;
+    }
     if (kCand && warp == 0) {
         // The CTA's most recent marked ends: 32 bitmap words per pass from the top; lane i holds word
         // top - i, and a prefix sum of the popcounts ranks its bits after those of higher words.

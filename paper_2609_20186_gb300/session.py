@@ -48,9 +48,13 @@ class Session:
         self.probe_w = bf16_tensor(probe_w_bits.reshape(-1), dev)
         B = self.B
         i32 = dict(dtype=torch.int32, device=dev)
-        self.draft = torch.zeros(B, k, **i32)
-        self.len = torch.zeros(B, **i32)
-        self.mode = torch.zeros(B, **i32)
+        # The per-step results a caller reads back live in one buffer, so one copy brings them to the
+        # host (outputs_to): mode [B], draft length [B], accepted length [B], draft [B, k].
+        self.results = torch.zeros(B * (k + 3), **i32)
+        self.mode = self.results[0:B]
+        self.len = self.results[B:2 * B]
+        self.accept = self.results[2 * B:3 * B]
+        self.draft = self.results[3 * B:].view(B, k)
         self.score = torch.zeros(B, dtype=torch.float32, device=dev)
         self.match_n = torch.zeros(B, **i32)
         self.match_end = torch.zeros(B, **i32)
@@ -58,7 +62,6 @@ class Session:
         self.vdraft = torch.zeros(B, k, **i32)
         self.vlen = torch.zeros(B, **i32)
         self.target = torch.zeros(B, k + 1, **i32)
-        self.accept = torch.zeros(B, **i32)
         self.vstatus = torch.zeros(B, **i32)
         fut = future if future is not None else np.zeros((B, 0), np.int32)
         self.future = torch.from_numpy(np.ascontiguousarray(fut, np.int32)).to(dev)
@@ -221,6 +224,14 @@ class Session:
         self.step(hidden, debug)
         self.harness(t)
         self.verify(debug)
+
+    def outputs_to(self, host: torch.Tensor) -> dict:
+        """One asynchronous device-to-host copy of mode, draft length, accepted length and draft into
+        `host` (pinned int32 [B * (k + 3)]); returns views of it.  Synchronise the stream before use."""
+        host.copy_(self.results, non_blocking=True)
+        B, k = self.B, self.k
+        return {"mode": host[0:B], "len": host[B:2 * B], "accept": host[2 * B:3 * B],
+                "draft": host[3 * B:].view(B, k)}
 
     # --- host views ------------------------------------------------------------------------------
     def step_outputs(self) -> dict:
