@@ -377,6 +377,8 @@ class ReplicaLoop:
         # none writes this batch's rows or hidden states (generated once, never written), so their
         # copies may start before it finishes.
         p.prefetch = (bd.PREFETCH_CONTEXT | bd.PREFETCH_PROBE) if prefetch else 0
+        # params.len_bound (split on a bound, copies before the length read) measured no faster here
+        p.len_bound = 0
         # one workspace per batch, so consecutive launches never share one
         probe = bd.switchsd_params()
         probe.B, probe.d, probe.probe_kind, probe.probe_hidden = B, wl.d, wl.probe_kind, wl.probe_hidden

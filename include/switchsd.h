@@ -41,7 +41,7 @@
 extern "C" {
 #endif
 
-#define SWITCHSD_ABI_VERSION 3
+#define SWITCHSD_ABI_VERSION 4
 
 #define SWITCHSD_NMAX 32 /* largest supported n_max */
 #define SWITCHSD_KMAX 64 /* largest supported draft length k */
@@ -125,6 +125,12 @@ typedef struct switchsd_index switchsd_index;
  *                target computed -- or row 0 when nothing was appended (capacity, bad lengths).  The
  *                probe's copies then wait for the verification; SWITCHSD_PREFETCH_PROBE is ignored.
  *                Any other value is SWITCHSD_ERR_ARG.
+ *   len_bound    0, or an upper bound on every ctx_lens[b] before the call's append (<= cap).  The rescan
+ *                then splits each row's ends between its CTAs on the bound instead of on the row's
+ *                length, so the context copies leave before the length is read; a row longer than the
+ *                bound gets SWITCHSD_ROW_BAD_LEN.  cap is always a valid bound; a bound far above the
+ *                lengths leaves CTAs idle and copies bytes past the rows' ends.  The index search
+ *                ignores it.  Outside [0, cap]: SWITCHSD_ERR_ARG.
  */
 typedef struct {
     int32_t B, cap, d, k, n_min, n_max, kappa;
@@ -143,6 +149,7 @@ typedef struct {
     void *stream;
     int32_t prefetch;
     int32_t hidden_rows;
+    int32_t len_bound;
 } switchsd_params;
 
 /*

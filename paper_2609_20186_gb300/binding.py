@@ -19,7 +19,7 @@ PROBE_LINEAR, PROBE_MLP = 0, 1
 OK, ERR_ARG, ERR_SHAPE, ERR_CUDA = 0, -1, -2, -3
 ROW_OK, ROW_CAPACITY, ROW_BAD_LEN, ROW_TIMEOUT = 0, 1, 2, 3
 NMAX, KMAX = 32, 64
-ABI_VERSION = 3  # SWITCHSD_ABI_VERSION this binding marshals for
+ABI_VERSION = 4  # SWITCHSD_ABI_VERSION this binding marshals for
 PREFETCH_CONTEXT, PREFETCH_PROBE = 1, 2  # switchsd_params.prefetch bits
 
 _c_i32p = ctypes.c_void_p
@@ -40,6 +40,7 @@ class switchsd_params(ctypes.Structure):
         ("stream", ctypes.c_void_p),
         ("prefetch", ctypes.c_int32),
         ("hidden_rows", ctypes.c_int32),
+        ("len_bound", ctypes.c_int32),
     ]
 
 

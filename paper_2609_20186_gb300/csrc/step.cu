@@ -71,6 +71,7 @@ struct StepArgs {
     int32_t B, cap, d, k, n_min, n_max, kappa, tile, stages;
     int32_t prefetch;        // SWITCHSD_PREFETCH_* bits: reads that may precede the grid-dependency wait
     int32_t hidden_rows;     // > 1: hidden is [B, hidden_rows, d] and the probe reads row a_b (verifying)
+    int32_t len_bound;       // > 0: every row's length is at most this; the ranges are split on it
     float logit_tau;
     int32_t *out_draft, *out_len, *out_mode;
     float *out_score;
@@ -232,14 +233,6 @@ __global__ void __launch_bounds__(kStepThreads) step_kernel(const StepArgs a) {
         tail_lo = max(0, (L_old - kHalo) & ~3);
         tail_hi = len_ok ? (L_old + 3) & ~3 : tail_lo;  // <= cap since cap % 4 == 0
     };
-    if (warp < 2) set_split(__ldcg(a.lens + b));
-    // Every thread arrives now, before issuing any copy or load: only the length read has to precede
-    // the leader's write of the new length.
-    if (warp < 2)
-        cluster_arrive_release();
-    else
-        cluster_arrive_relaxed();
-
     // Stage tile t: tokens [max(0, t0 - kHalo), min(roundup4(t1 + kFwd), cap)) land so that token p
     // sits at stage[kHalo + p - t0].  cap % 4 == 0 keeps every bound 16-byte aligned.
     auto issue = [&](int t) {
@@ -252,12 +245,37 @@ __global__ void __launch_bounds__(kStepThreads) step_kernel(const StepArgs a) {
         mbar_expect_tx_relaxed(&bars[s], bytes);
         bulk_g2s_hint(tiles + s * stage_ints + (kHalo + lo - t0), row + lo, bytes, &bars[s], l2_evict_first_policy());
     };
+    // With a length bound the ranges are split on the bound, so the tile copies leave before the row
+    // length is read; the length then gives the tail, the verification and the end of the scan (a row
+    // longer than the bound is a bad length).
+    const bool bounded = a.len_bound > 0;
+    if (warp < 2) {
+        if (bounded) {
+            set_split(a.len_bound);
+            if (warp == 0 && lane == 0)
+                for (int t = 0; t < min(ntiles, a.stages); ++t) issue(t);
+            L_old = __ldcg(a.lens + b);
+            len_ok = L_old >= 1 && L_old <= a.len_bound && L_old <= a.cap;
+            tail_lo = max(0, (L_old - kHalo) & ~3);
+            tail_hi = len_ok ? (L_old + 3) & ~3 : tail_lo;
+        } else {
+            set_split(__ldcg(a.lens + b));
+        }
+    }
+    // Every thread arrives now, before issuing anything else: only the length read has to precede
+    // the leader's write of the new length.
+    if (warp < 2)
+        cluster_arrive_release();
+    else
+        cluster_arrive_relaxed();
+
     if (warp == 0) {
         if (lane == 0) {
             const uint32_t tb = uint32_t(tail_hi - tail_lo) * 4u;
             mbar_expect_tx_relaxed(&tail_bar, tb);
             if (tb > 0) bulk_g2s_hint(s_tail, row + tail_lo, tb, &tail_bar, l2_evict_first_policy());
-            for (int t = 0; t < min(ntiles, a.stages); ++t) issue(t);
+            if (!bounded)
+                for (int t = 0; t < min(ntiles, a.stages); ++t) issue(t);
             s_split[0] = L_old;
             s_split[1] = e_lo;
             s_split[2] = e_hi;
@@ -411,7 +429,7 @@ __global__ void __launch_bounds__(kStepThreads) step_kernel(const StepArgs a) {
         e_lo = s_split[1];
         e_hi = s_split[2];
         ntiles = s_split[3];
-        len_ok = (L_old >= 1 && L_old <= a.cap);
+        len_ok = (L_old >= 1 && L_old <= (a.len_bound > 0 ? min(a.len_bound, a.cap) : a.cap));
         tail_lo = max(0, (L_old - kHalo) & ~3);
         tail_hi = len_ok ? (L_old + 3) & ~3 : tail_lo;
     }
@@ -772,6 +790,7 @@ static int step_entry(int32_t *ctx_tokens, int32_t *ctx_lens, const uint16_t *hi
     if (p->split != 0 && p->split != 1 && p->split != 2 && p->split != 4 && p->split != 8 && p->split != 16)
         return SWITCHSD_ERR_SHAPE;
     if ((p->prefetch & ~(SWITCHSD_PREFETCH_CONTEXT | SWITCHSD_PREFETCH_PROBE)) != 0) return SWITCHSD_ERR_ARG;
+    if (p->len_bound < 0 || p->len_bound > p->cap) return SWITCHSD_ERR_ARG;
     // hidden_rows: 0 / 1, or k + 1 for the fused greedy / sampled verification with the linear probe
     if (p->hidden_rows != 0 && p->hidden_rows != 1) {
         if (p->hidden_rows != p->k + 1 || pv_len == nullptr || cs != nullptr || p->index != nullptr ||
@@ -820,6 +839,7 @@ static int step_entry(int32_t *ctx_tokens, int32_t *ctx_lens, const uint16_t *hi
     args.status = p->status;
     args.prefetch = p->prefetch;
     args.hidden_rows = p->hidden_rows > 1 ? p->hidden_rows : 1;
+    args.len_bound = p->len_bound;
 
     const int split = p->split > 0 ? p->split : choose_split(p->B, p->cap);
     // Tile: the largest CTA range (the last CTA may also cover a k + 1 token append), in one stage

@@ -34,7 +34,7 @@ class Session:
                  probe_kind: int = bd.PROBE_LINEAR, probe_hidden: int = 0, future=None,
                  harness: dict | None = None, split: int = 0, d: int | None = None,
                  use_index: bool = False, device="cuda", stream: torch.cuda.Stream | None = None,
-                 prefetch: int = 0, hidden_rows: int = 0):
+                 prefetch: int = 0, hidden_rows: int = 0, len_bound: int = 0):
         self.lib = bd.load()
         self.hidden_rows = int(hidden_rows)
         self.device = torch.device(device)
@@ -98,6 +98,7 @@ class Session:
             p.stream = sp
             p.prefetch = int(prefetch)
             p.hidden_rows = int(hidden_rows)  # k + 1: verify_step reads row a_b of a [B, k+1, d] hidden
+            p.len_bound = int(len_bound)      # > 0: split on this bound, copies before the length read
             return p
         self._p_dbg, self._p_fast = params(True), params(False)
         self._step_head = (self.ctx.data_ptr(), self.lens.data_ptr())

@@ -58,7 +58,7 @@ def test_binding_declares_every_function():
 
 def test_abi_version_and_strerror(lib):
     from paper_2609_20186_gb300 import binding as bd
-    assert bd.abi_version() == 3
+    assert bd.abi_version() == 4
     for code in (0, -1, -2, -3, 1, 2, 3):
         assert bd.strerror(code) != "unknown code"
     assert bd.strerror(12345) == "unknown code"
@@ -100,6 +100,8 @@ def test_step_validation(lib):
     assert _step(lib, _params(split=3)) == bd.ERR_SHAPE
     assert _step(lib, _params(prefetch=4)) == bd.ERR_ARG
     assert _step(lib, _params(hidden_rows=9)) == bd.ERR_ARG   # k + 1 rows only with a verification
+    assert _step(lib, _params(len_bound=65)) == bd.ERR_ARG    # above cap
+    assert _step(lib, _params(len_bound=-1)) == bd.ERR_ARG
     assert _step(lib, _params(prefetch=-1)) == bd.ERR_ARG
     assert _step(lib, _params(probe_kind=1, probe_hidden=0)) == bd.ERR_SHAPE
     # the two-layer probe needs its workspace

@@ -17,7 +17,7 @@ W = synth.WORKLOADS
 KEYS = ("draft", "len", "mode", "score", "match_n", "match_end", "status", "accept")
 
 
-def _chain(wl, prefetch: int, steps: int, record_every: int):
+def _chain(wl, prefetch: int, steps: int, record_every: int, len_bound: int = 0):
     import torch
     from paper_2609_20186_gb300 import Session, bf16_tensor
 
@@ -25,7 +25,7 @@ def _chain(wl, prefetch: int, steps: int, record_every: int):
     sess = Session(ctx, lens, wl.probe_weights(), k=wl.k, n_min=wl.n_min, n_max=wl.n_max,
                    kappa=wl.kappa, logit_tau=wl.logit_tau, probe_kind=wl.probe_kind,
                    probe_hidden=wl.probe_hidden, future=wl.future(), harness=wl.harness_params(),
-                   d=wl.d, prefetch=prefetch)
+                   d=wl.d, prefetch=prefetch, len_bound=len_bound)
     hidden = bf16_tensor(np.stack([wl.hidden(t) for t in range(steps)]), sess.device)
     torch.cuda.synchronize()
     rec = {}
@@ -62,3 +62,39 @@ def test_prefetch_matches_back_to_back(name, steps):
             else:
                 assert np.array_equal(a[t][key], b[t][key]), (name, t, key)
 
+
+@pytest.mark.parametrize("name,steps", [("zipf_32k", 40), ("uniform_8k", 40), ("mixed_128k", 24),
+                                        ("code_16k", 16)])
+def test_length_bound_matches(name, steps):
+    """params.len_bound = cap splits every row's ends on cap (copies before the length read): the run
+    must be bit-identical to the plain one, rows far from full (uniform_8k) included."""
+    from paper_2609_20186_gb300 import binding as bd
+    wl = W[name].scaled(steps=steps)
+    cap = wl.contexts()[0].shape[1]
+    a, a_ctx, a_lens = _chain(wl, 0, steps, record_every=4)
+    b, b_ctx, b_lens = _chain(wl, bd.PREFETCH_CONTEXT | bd.PREFETCH_PROBE, steps, record_every=4, len_bound=cap)
+    assert np.array_equal(a_lens, b_lens) and np.array_equal(a_ctx, b_ctx)
+    for t in a:
+        for key in KEYS:
+            if key != "draft":
+                assert np.array_equal(a[t][key], b[t][key]), (name, t, key)
+
+
+def test_length_above_bound_is_bad_length():
+    import torch
+    from paper_2609_20186_gb300 import Session, bf16_tensor
+    wl = W["uniform_8k"].scaled(B=6, L0=2000, steps=2)
+    ctx, lens = wl.contexts()
+    lens[:] = [1990, 2000, 2001, 2005, 1, 1500]
+    sess = Session(ctx, lens, wl.probe_weights(), k=wl.k, n_min=wl.n_min, n_max=wl.n_max, kappa=wl.kappa,
+                   logit_tau=wl.logit_tau, d=wl.d, len_bound=2000)
+    sess.step(bf16_tensor(wl.hidden(0), sess.device))
+    torch.cuda.synchronize()
+    st = sess.status.cpu().numpy()
+    assert st.tolist() == [0, 0, 2, 2, 0, 0]
+    ref = Session(ctx, lens, wl.probe_weights(), k=wl.k, n_min=wl.n_min, n_max=wl.n_max, kappa=wl.kappa,
+                  logit_tau=wl.logit_tau, d=wl.d)
+    ref.step(bf16_tensor(wl.hidden(0), ref.device))
+    torch.cuda.synchronize()
+    for r in (0, 1, 4, 5):                         # rows within the bound: the plain step's results
+        assert sess.mode.cpu()[r] == ref.mode.cpu()[r] and sess.match_end.cpu()[r] == ref.match_end.cpu()[r]
