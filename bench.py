@@ -214,69 +214,108 @@ def profiled_traffic(workload: str) -> float | None:
 # ------------------------------------------------------------------------------------------------
 # CPU oracle timing (baseline and reference arm)
 # ------------------------------------------------------------------------------------------------
+def host_threads() -> int:
+    try:
+        return max(1, len(os.sched_getaffinity(0)))
+    except AttributeError:
+        return max(1, os.cpu_count() or 1)
+
+
 def time_oracle(wl: synth.Workload, budget_s: float, max_steps: int, rows: int | None = None,
-                warmup: int = 0, sampled: bool = False, cand: tuple[int, int] | None = None):
+                warmup: int = 0, sampled: bool = False, cand: tuple[int, int] | None = None,
+                threads: int = 1):
     """Runs the oracle loop (oracle step, host target stand-in, oracle verify) on rows [0, R):
     ``warmup`` untimed steps, then up to max_steps timed steps or until budget_s of oracle time is
-    spent.  Returns (seq*steps, seconds, timed_steps, R).  Only the oracle's calls are timed."""
+    spent.  Returns (seq*steps, seconds, timed_steps, R).  Only the oracle's calls are timed.
+
+    threads > 1 runs each oracle call as that many concurrent calls on contiguous ranges of rows (rows
+    are independent; the oracle's C calls release the interpreter lock), the oracle itself unchanged."""
     import oracle
+    from concurrent.futures import ThreadPoolExecutor
     R = wl.B if rows is None else min(rows, wl.B)
     ctx, lens = wl.contexts()
     future = wl.future()
     pw = wl.probe_weights()
     hp = wl.harness_params()
+    nt = max(1, min(threads, R))
+    chunks = [(R * i // nt, R * (i + 1) // nt) for i in range(nt)]
+    pool = ThreadPoolExecutor(nt) if nt > 1 else None
+
+    def over_rows(fn):
+        """fn(b0, b1) -> dict or tuple of [B] arrays filled on rows [b0, b1); merged over the chunks."""
+        if pool is None:
+            return fn(0, R)
+        parts = list(pool.map(lambda c: fn(*c), chunks))
+        first = parts[0]
+        if isinstance(first, dict):
+            for (b0, b1), part in zip(chunks[1:], parts[1:]):
+                for key in first:
+                    first[key][b0:b1] = part[key][b0:b1]
+            return first
+        for (b0, b1), part in zip(chunks[1:], parts[1:]):
+            for x, y in zip(first, part):
+                x[b0:b1] = y[b0:b1]
+        return first
+
     spent = 0.0
     done = 0
-    for t in range(warmup + max_steps):
-        h = wl.hidden(t)
-        if cand is not None:
-            Wc, Dc = cand
-            t0 = time.perf_counter()
-            out = oracle.step_candidates(ctx, lens, h, pw, W=Wc, D=Dc, n_min=wl.n_min, n_max=wl.n_max,
-                                         kappa=wl.kappa, logit_tau=wl.logit_tau, probe_kind=wl.probe_kind,
-                                         probe_hidden=wl.probe_hidden, rows=(0, R))
-            dt = time.perf_counter() - t0
-            vc, vl, vn, tg = synth.harness_candidates(hp, t, lens, out["mode"], out["cand"], out["cand_len"],
-                                                      out["ncand"], future, rows=range(R))
-            t0 = time.perf_counter()
-            oracle.verify_candidates(ctx, lens, vc, vl, vn, tg, rows=(0, R))
-            dt += time.perf_counter() - t0
-            if t >= warmup:
-                spent += dt
-                done += 1
-                if spent >= budget_s:
-                    break
-            continue
-        t0 = time.perf_counter()
-        out = oracle.step(ctx, lens, h, pw, k=wl.k, n_min=wl.n_min, n_max=wl.n_max, kappa=wl.kappa,
-                          logit_tau=wl.logit_tau, probe_kind=wl.probe_kind,
-                          probe_hidden=wl.probe_hidden, rows=(0, R))
-        dt = time.perf_counter() - t0
-        if sampled:
-            vd, vl, pp, qq, uu, rs = synth.harness_sampled(hp, t, lens, out["mode"], out["draft"],
-                                                           out["len"], future, rows=range(R))
-            t0 = time.perf_counter()
-            oracle.verify_sampled(ctx, lens, vd, vl, pp, uu, rs, q=qq, rows=(0, R))
-        else:
-            vd, vl, tg = synth.harness_targets(hp, t, lens, out["mode"], out["draft"], out["len"],
-                                               future, rows=range(R))
-            t0 = time.perf_counter()
-            oracle.verify(ctx, lens, vd, vl, tg, rows=(0, R))
-        dt += time.perf_counter() - t0
-        if t < warmup:
-            continue
-        spent += dt
-        done += 1
-        if spent >= budget_s:
-            break
+    try:
+        for t in range(warmup + max_steps):
+            h = wl.hidden(t)
+            if cand is not None:
+                Wc, Dc = cand
+                t0 = time.perf_counter()
+                out = over_rows(lambda b0, b1: oracle.step_candidates(
+                    ctx, lens, h, pw, W=Wc, D=Dc, n_min=wl.n_min, n_max=wl.n_max, kappa=wl.kappa,
+                    logit_tau=wl.logit_tau, probe_kind=wl.probe_kind, probe_hidden=wl.probe_hidden,
+                    rows=(b0, b1)))
+                dt = time.perf_counter() - t0
+                vc, vl, vn, tg = synth.harness_candidates(hp, t, lens, out["mode"], out["cand"],
+                                                          out["cand_len"], out["ncand"], future, rows=range(R))
+                t0 = time.perf_counter()
+                over_rows(lambda b0, b1: oracle.verify_candidates(ctx, lens, vc, vl, vn, tg, rows=(b0, b1)))
+                dt += time.perf_counter() - t0
+            else:
+                t0 = time.perf_counter()
+                out = over_rows(lambda b0, b1: oracle.step(
+                    ctx, lens, h, pw, k=wl.k, n_min=wl.n_min, n_max=wl.n_max, kappa=wl.kappa,
+                    logit_tau=wl.logit_tau, probe_kind=wl.probe_kind, probe_hidden=wl.probe_hidden,
+                    rows=(b0, b1)))
+                dt = time.perf_counter() - t0
+                if sampled:
+                    vd, vl, pp, qq, uu, rs = synth.harness_sampled(hp, t, lens, out["mode"], out["draft"],
+                                                                   out["len"], future, rows=range(R))
+                    t0 = time.perf_counter()
+                    over_rows(lambda b0, b1: oracle.verify_sampled(ctx, lens, vd, vl, pp, uu, rs, q=qq,
+                                                                   rows=(b0, b1)))
+                else:
+                    vd, vl, tg = synth.harness_targets(hp, t, lens, out["mode"], out["draft"], out["len"],
+                                                       future, rows=range(R))
+                    t0 = time.perf_counter()
+                    over_rows(lambda b0, b1: oracle.verify(ctx, lens, vd, vl, tg, rows=(b0, b1)))
+                dt += time.perf_counter() - t0
+            if t < warmup:
+                continue
+            spent += dt
+            done += 1
+            if spent >= budget_s:
+                break
+    finally:
+        if pool is not None:
+            pool.shutdown()
     return R * done, spent, done, R
 
 
 def cpu_baseline(wl: synth.Workload, budget_s: float, sampled: bool = False, cand=None) -> dict:
-    units, secs, steps, R = time_oracle(wl, budget_s, wl.steps, sampled=sampled, cand=cand)
-    return {"value": units / secs, "unit": UNIT, "cores": 1, "kind": "oracle",
+    """The oracle on all host cores (rows split over threads), with a single-thread run beside it."""
+    nt = host_threads()
+    units, secs, steps, R = time_oracle(wl, budget_s, wl.steps, sampled=sampled, cand=cand, threads=nt)
+    u1, s1, steps1, _ = time_oracle(wl, budget_s / 3, wl.steps, sampled=sampled, cand=cand, threads=1)
+    return {"value": units / secs, "unit": UNIT, "cores": min(nt, R), "kind": "oracle",
+            "single_thread_value": u1 / s1,
             "sample": f"{wl.name}: rows 0..{R - 1}, first {steps} controller steps (oracle step + "
-                      f"verify timed, single thread; the host target stand-in is not timed)"}
+                      f"verify timed over {min(nt, R)} threads, each a contiguous range of rows; the host "
+                      f"target stand-in is not timed); single thread: first {steps1} steps"}
 
 
 def config_of(wl: synth.Workload, world: int, split: int, search: str = "scan",
@@ -292,8 +331,8 @@ def config_of(wl: synth.Workload, world: int, split: int, search: str = "scan",
 
 
 def run_reference(args, world, rank):
-    """The reference arm: the CPU oracle on this host, W untimed + K timed steps of the workload on
-    a bounded sample of rows (all rows when B <= 64, else the first 16)."""
+    """The reference arm: the CPU oracle on this host's cores, W untimed + K timed steps of the workload
+    on a bounded sample of rows (all rows when B <= 64, else the first 16)."""
     if rank != 0:
         return
     import oracle
@@ -301,9 +340,11 @@ def run_reference(args, world, rank):
     base = synth.get_workload(args.workload)
     wl = base.scaled(steps=args.warmup + args.steps)
     R = wl.B if wl.B <= 64 else 16
+    nt = host_threads()
     units, secs, steps, R = time_oracle(wl, float("inf"), args.steps, rows=R, warmup=args.warmup,
                                         sampled=args.verify == "sampled",
-                                        cand=(args.candidates, args.cand_len) if args.candidates > 0 else None)
+                                        cand=(args.candidates, args.cand_len) if args.candidates > 0 else None,
+                                        threads=nt)
     value = units / secs
     line = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
             "steps": args.steps, "warmup": args.warmup,
@@ -312,9 +353,9 @@ def run_reference(args, world, rank):
             "impl": "reference",
             "config": config_of(base, world, args.split, args.search, not args.no_prefetch, args.verify,
                                  args.candidates, args.cand_len),
-            "cpu_baseline": {"value": value, "unit": UNIT, "cores": 1, "kind": "oracle",
+            "cpu_baseline": {"value": value, "unit": UNIT, "cores": min(nt, R), "kind": "oracle",
                              "sample": f"{wl.name}: rows 0..{R - 1}, {args.warmup} untimed + "
-                                       f"{steps} timed steps, single thread"},
+                                       f"{steps} timed steps, rows split over {min(nt, R)} threads"},
             "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0,
                     "d2h_bytes_per_step": 0}}
     print(json.dumps(line), flush=True)
@@ -640,6 +681,12 @@ def run_ours(args, world, rank, local):
     # cold single-launch latency: L2 flushed, one event-bracketed fused launch on batch 0
     cold = cold_latency(loop, dev, cs, warm_rounds + rounds, l2)
 
+    ceiling = None
+    if args.search == "scan":
+        ceiling = read_ceiling(loop, d, K, warm_rounds * R, not args.no_prefetch, cs)
+        ceiling["frac"] = ceiling["achieved"] / peaks["hbm_gbs"]
+        ceiling["step_time_ratio"] = ceiling["launch_us"] / (per_launch_s * 1e6)
+
     e2e = None
     if not args.no_e2e and args.candidates == 0:  # the public-API loop covers the single-draft step
         e2e = run_e2e(base, dev, W, K, args.split, world, prefetch=not args.no_prefetch,
@@ -666,7 +713,9 @@ def run_ours(args, world, rank, local):
                      "launch_us": per_launch_s * 1e6,
                      "duration": "timed region / K launches (the region also holds one target "
                                  "stand-in launch and one 4 KB length snapshot per round)",
-                     "peak_source": peaks["source"] + " hbm_gbs (copy)"},
+                     "peak_source": peaks["source"] + " hbm_gbs (copy)",
+                     "frac_nominal": achieved / NOMINAL_HBM_GBS,
+                     "size_matched_ceiling": ceiling},
         "controller": {"cold_single_launch_us": cold, "search": args.search,
                        "scan_equivalent_gbs": float(4 * Lh[1:].sum(axis=2).mean() / per_launch_s / 1e9),
                        "mean_context_tokens": float(Lh[1:].mean()),
@@ -682,6 +731,7 @@ def run_ours(args, world, rank, local):
 
 
 COLD_STEPS = 32
+NOMINAL_HBM_GBS = 7900.0  # HBM3e nominal of this GPU
 CLOCK_WINDOW_S = 0.4
 
 
@@ -717,10 +767,57 @@ def cold_latency(loop, dev, cs, step_base, l2) -> dict:
             "note": "includes the ~2.2 us event-pair and ~2.2 us stream launch overhead of this GPU"}
 
 
+def read_ceiling(loop, d: int, K: int, step_base: int, prefetch: bool, cs) -> dict:
+    """The size-matched ceiling: switchsd_harness_read -- a plain read of each launch's contexts and
+    hidden states and nothing else -- in the timed graph's launch order (K launches, launch i on batch
+    i mod R, programmatic dependent launch), best of a few CTA splits per row."""
+    import torch
+    R, B, cap = loop.R, loop.B, loop.cap
+    nh = loop.hidden.shape[0]
+    out = torch.empty(R, B * 32, dtype=torch.int32, device=loop.lens.device)
+    L = loop.lens.cpu().numpy().astype(np.int64).reshape(R, B)
+    per_batch = 16 * ((L + 3) // 4).sum(axis=1) + 2 * B * d
+    nbytes = float(np.mean([per_batch[i % R] for i in range(K)]))
+
+    def enqueue(split):
+        for i in range(K):
+            r = i % R
+            code = loop.lib.switchsd_harness_read(
+                loop.rows[r]["ctx"], loop.rows[r]["lens"], B, cap,
+                loop.hidden.data_ptr() + ((step_base + i) % nh) * loop.hstride, d, split, int(prefetch),
+                out[r].data_ptr(), cs.cuda_stream)
+            if code != 0:
+                raise RuntimeError(f"switchsd_harness_read failed: {code}")
+
+    best = None
+    for split in (4, 8, 16, 32):
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.stream(cs):
+            enqueue(split)                                  # eager warm-up
+            with torch.cuda.graph(g, stream=cs):
+                enqueue(split)
+            g.replay()
+            cs.synchronize()
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record(cs)
+            g.replay()
+            e1.record(cs)
+            e1.synchronize()
+        us = e0.elapsed_time(e1) * 1e3 / K
+        if best is None or us < best[0]:
+            best = (us, split)
+    us, split = best
+    return {"kernel": "switchsd_harness_read", "launch_us": us, "achieved": nbytes / us / 1e3,
+            "bytes_per_launch": nbytes, "split": split, "prefetch": bool(prefetch),
+            "note": "plain 16-byte loads of every launch's context tokens and hidden states, same graph, "
+                    "launch order and inputs larger than L2; best of splits 4, 8, 16, 32"}
+
+
 def run_e2e(base, dev, W, K, split, world, prefetch=True, sampled=False):
-    """The same loop through the public API with host buffers, one batch: per step, H2D of the
-    hidden states from pinned memory, switchsd_verify_step + target stand-in, D2H of mode / draft
-    length / draft / accepted length, host sync."""
+    """The same loop through the public API with host buffers, one batch.  Per step (greedy): the
+    target stand-in for the previous draft, then one switchsd_verify_step_host call -- pinned H2D of
+    this step's hidden states, the fused launch, one D2H of mode / draft length / accepted length /
+    draft, host sync.  Sampled: the same copies and launches as separate calls."""
     import torch
     from paper_2609_20186_gb300 import Session, binding
 
@@ -740,22 +837,22 @@ def run_e2e(base, dev, W, K, split, world, prefetch=True, sampled=False):
     stream = torch.cuda.current_stream()
 
     def one(t):
-        dev_h.view(torch.int16).copy_(host_h[t], non_blocking=True)
         if t == 0:
-            sess.step(dev_h, debug=False)
-        elif sampled:
-            sess.verify_sampled_step(dev_h, debug=False)
-        else:
-            sess.verify_step(dev_h, debug=False)
+            sess.step_host(host_h[0], dev_h, host_out)
+            return
         if sampled:
-            sess.harness_sampled(t)
-        else:
-            sess.harness(t)
-        sess.outputs_to(host_out)  # one D2H copy of mode, draft length, accepted length and draft
-        stream.synchronize()
+            sess.harness_sampled(t - 1)
+            dev_h.view(torch.int16).copy_(host_h[t], non_blocking=True)
+            sess.verify_sampled_step(dev_h, debug=False)
+            sess.outputs_to(host_out)  # one D2H copy of mode, draft length, accepted length and draft
+            stream.synchronize()
+            return
+        sess.harness(t - 1)            # the target's tokens for the previous draft
+        sess.verify_step_host(host_h[t], dev_h, host_out)
 
     for t in range(W):
         one(t)
+    torch.cuda.synchronize()
     barrier(world)
     t0 = time.perf_counter()
     for i in range(K):
@@ -764,8 +861,11 @@ def run_e2e(base, dev, W, K, split, world, prefetch=True, sampled=False):
     value = replica_throughput(B * K, secs, world)
     return {"value": value, "unit": UNIT, "h2d_bytes_per_step": B * d * 2,
             "d2h_bytes_per_step": B * (k + 3) * 4,
-            "note": "one batch; per step: pinned H2D of hidden, switchsd_verify_step + target "
-                    "stand-in, D2H of mode/len/draft/accept, host sync; L2 not flushed"}
+            "note": ("one batch; per step: target stand-in, then " +
+                     ("pinned H2D of hidden, switchsd_verify_sampled_step, D2H of mode/len/accept/draft, "
+                      "host sync" if sampled else
+                      "one switchsd_verify_step_host call (pinned H2D of hidden, fused launch, one D2H of "
+                      "mode/len/accept/draft, host sync)") + "; L2 not flushed")}
 
 
 LABEL_METRIC = "copy-mode labels/sec (positions, §3.2, n_train=5); achieved HBM GB/s vs peak"

@@ -29,7 +29,8 @@
  *     optional per-row `status` array (SWITCHSD_ROW_*); the kernels never trap.
  *   - Token ids are opaque int32 values: only equality is used.
  *   - bf16 values are passed as their 16-bit patterns (uint16_t), the upper half of an IEEE binary32.
- *   - All calls may be captured into a CUDA graph: they allocate nothing and synchronise nothing.
+ *   - All calls may be captured into a CUDA graph: they allocate nothing and synchronise nothing
+ *     (the host-staged entries switchsd_step_host / switchsd_verify_step_host synchronise when asked).
  */
 #ifndef SWITCHSD_H_
 #define SWITCHSD_H_
@@ -41,7 +42,7 @@
 extern "C" {
 #endif
 
-#define SWITCHSD_ABI_VERSION 4
+#define SWITCHSD_ABI_VERSION 5
 
 #define SWITCHSD_NMAX 32 /* largest supported n_max */
 #define SWITCHSD_KMAX 64 /* largest supported draft length k */
@@ -273,6 +274,40 @@ int switchsd_verify_sampled_step(const int32_t *draft, const float *p_draft, con
                                  int32_t *ctx_tokens, int32_t *ctx_lens, const uint16_t *hidden,
                                  const uint16_t *probe_w, const switchsd_params *params, int32_t *out_draft,
                                  int32_t *out_len, int32_t *out_mode, float *out_score);
+
+/*
+ * Host staging around one step: switchsd_step / switchsd_verify_step for inputs that arrive in host
+ * memory and results read back on the host, in one call.  Before the step, in_bytes are copied from
+ * in_host to in_dev (device; typically the hidden states the step then reads); after it, out_bytes
+ * from out_dev (device; typically one buffer holding the step's mode, draft length, accepted length
+ * and draft) to out_host.  Both copies are cudaMemcpyAsync on params->stream, ordered with the step's
+ * launch; host buffers should be pinned for the copies to be asynchronous.  A zero byte count skips
+ * that copy.  synchronize != 0: the call returns after the stream has drained, so out_host holds the
+ * results; 0: everything is queued on the stream and the call returns at once.
+ */
+typedef struct {
+    const void *in_host;
+    void *in_dev;
+    size_t in_bytes;
+    const void *out_dev;
+    void *out_host;
+    size_t out_bytes;
+    int32_t synchronize;
+} switchsd_host_io;
+
+/* switchsd_step between the two copies of `io`.  Returns SWITCHSD_ERR_ARG for a NULL io or params or a
+ * NULL pointer of a copy with a nonzero byte count, SWITCHSD_ERR_CUDA when a copy or the
+ * synchronisation fails, else switchsd_step's code (a step that fails validation queues no copy back). */
+int switchsd_step_host(const switchsd_host_io *io, const int32_t *ctx_tokens, const int32_t *ctx_lens,
+                       const uint16_t *hidden, const uint16_t *probe_w, const switchsd_params *params,
+                       int32_t *out_draft, int32_t *out_len, int32_t *out_mode, float *out_score);
+
+/* switchsd_verify_step between the two copies of `io`; codes as switchsd_step_host. */
+int switchsd_verify_step_host(const switchsd_host_io *io, const int32_t *draft, const int32_t *target_argmax,
+                              const int32_t *draft_len, int32_t *out_accept, int32_t *ctx_tokens,
+                              int32_t *ctx_lens, const uint16_t *hidden, const uint16_t *probe_w,
+                              const switchsd_params *params, int32_t *out_draft, int32_t *out_len,
+                              int32_t *out_mode, float *out_score);
 
 /*
  * Bytes of device workspace switchsd_step / switchsd_verify_step need for `params` (0 for the linear

@@ -76,6 +76,24 @@ int switchsd_harness_candidates(const int32_t *ctx_lens, const int32_t *mode, co
                                 int32_t D, int32_t *vcand, int32_t *vlen, int32_t *vn, int32_t *target,
                                 const switchsd_harness_params *hp);
 
+/*
+ * Not a stand-in: the size-matched read ceiling that benchmarks set beside the step kernel.  Reads
+ * what one step reads -- the first ctx_lens[b] tokens of every row (rounded up to whole 16-byte
+ * words) and the hidden states -- and nothing else: grid (split, B) of 256-thread CTAs, CTA (c, b)
+ * taking the c-th of `split` equal runs of row b's context words and of its d bf16 hidden values,
+ * 16-byte loads four in flight per thread, xor-folded into out[b * split + c] so no load is dead.
+ * prefetch != 0 issues the loads before the kernel's grid-dependency wait (as the step kernel does
+ * under SWITCHSD_PREFETCH_CONTEXT | SWITCHSD_PREFETCH_PROBE), else after it; launched with
+ * programmatic stream serialization like every kernel of the library.
+ * ctx_tokens int32 [B, cap] (16-byte aligned, cap a multiple of 4), ctx_lens int32 [B] (a length
+ * outside [0, cap] reads nothing), hidden bf16 bits [B, d] (16-byte aligned, d a multiple of 8),
+ * out uint32 [B * split]; split in [1, 1024].  Returns SWITCHSD_OK, SWITCHSD_ERR_ARG (NULL or
+ * misaligned pointer), SWITCHSD_ERR_SHAPE or SWITCHSD_ERR_CUDA.
+ */
+int switchsd_harness_read(const int32_t *ctx_tokens, const int32_t *ctx_lens, int32_t B, int32_t cap,
+                          const uint16_t *hidden, int32_t d, int32_t split, int32_t prefetch, uint32_t *out,
+                          void *stream);
+
 #ifdef __cplusplus
 }
 #endif

@@ -19,7 +19,7 @@ PROBE_LINEAR, PROBE_MLP = 0, 1
 OK, ERR_ARG, ERR_SHAPE, ERR_CUDA = 0, -1, -2, -3
 ROW_OK, ROW_CAPACITY, ROW_BAD_LEN, ROW_TIMEOUT = 0, 1, 2, 3
 NMAX, KMAX = 32, 64
-ABI_VERSION = 4  # SWITCHSD_ABI_VERSION this binding marshals for
+ABI_VERSION = 5  # SWITCHSD_ABI_VERSION this binding marshals for
 PREFETCH_CONTEXT, PREFETCH_PROBE = 1, 2  # switchsd_params.prefetch bits
 
 _c_i32p = ctypes.c_void_p
@@ -61,6 +61,14 @@ class switchsd_candidates_verify_params(ctypes.Structure):
     ]
 
 
+class switchsd_host_io(ctypes.Structure):
+    _fields_ = [
+        ("in_host", ctypes.c_void_p), ("in_dev", ctypes.c_void_p), ("in_bytes", ctypes.c_size_t),
+        ("out_dev", ctypes.c_void_p), ("out_host", ctypes.c_void_p), ("out_bytes", ctypes.c_size_t),
+        ("synchronize", ctypes.c_int32),
+    ]
+
+
 class switchsd_harness_params(ctypes.Structure):
     _fields_ = [
         ("B", ctypes.c_int32), ("k", ctypes.c_int32), ("V", ctypes.c_int32), ("L0", ctypes.c_int32),
@@ -86,6 +94,13 @@ _SIGNATURES = {
                              + [ctypes.c_void_p] * 4),
     "switchsd_verify_sampled_step": (ctypes.c_int, [ctypes.c_void_p] * 11 + [ctypes.POINTER(switchsd_params)]
                                      + [ctypes.c_void_p] * 4),
+    "switchsd_step_host": (ctypes.c_int, [ctypes.POINTER(switchsd_host_io)] + [ctypes.c_void_p] * 4
+                           + [ctypes.POINTER(switchsd_params)] + [ctypes.c_void_p] * 4),
+    "switchsd_verify_step_host": (ctypes.c_int, [ctypes.POINTER(switchsd_host_io)] + [ctypes.c_void_p] * 8
+                                  + [ctypes.POINTER(switchsd_params)] + [ctypes.c_void_p] * 4),
+    "switchsd_harness_read": (ctypes.c_int, [ctypes.c_void_p, ctypes.c_void_p, ctypes.c_int32, ctypes.c_int32,
+                                             ctypes.c_void_p, ctypes.c_int32, ctypes.c_int32, ctypes.c_int32,
+                                             ctypes.c_void_p, ctypes.c_void_p]),
     "switchsd_step_static_workspace": (ctypes.c_int, [ctypes.c_void_p] * 4
                                        + [ctypes.POINTER(switchsd_params)] + [ctypes.c_void_p] * 4),
     "switchsd_index_create": (ctypes.c_int, [ctypes.POINTER(switchsd_params),

@@ -236,3 +236,95 @@ extern "C" int switchsd_harness_candidates(const int32_t *ctx_lens, const int32_
                                      0, static_cast<cudaStream_t>(hp->stream), 0u, a);
     return e == cudaSuccess ? SWITCHSD_OK : SWITCHSD_ERR_CUDA;
 }
+
+// ------------------------------------------------------------------------------------------------
+// switchsd_harness_read: a plain read of what one step reads, the size-matched ceiling for the step
+// kernel.  Grid (split, B): CTA (c, b) reads the c-th of `split` equal runs of the 16-byte words that
+// hold row b's first ctx_lens[b] tokens, and the c-th run of row b's hidden states, with 16-byte
+// non-coherent loads, four in flight per thread; the words are xor-folded into out[b * split + c] so
+// no load is dead.  prefetch != 0 issues the loads before the grid-dependency wait (the step kernel's
+// SWITCHSD_PREFETCH_CONTEXT / _PROBE order), else after it.
+// ------------------------------------------------------------------------------------------------
+namespace switchsd {
+
+constexpr int kReadThreads = 256;
+
+struct ReadArgs {
+    const int32_t *ctx, *lens;
+    const uint16_t *hidden;
+    uint32_t *out;
+    int32_t B, cap, d, split, prefetch;
+};
+
+__device__ __forceinline__ uint32_t fold_ld(const uint4 *p) {
+    uint4 v;
+    asm volatile("ld.global.nc.L1::no_allocate.v4.u32 {%0, %1, %2, %3}, [%4];\n"
+                 : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
+                 : "l"(p));
+    return v.x ^ v.y ^ v.z ^ v.w;
+}
+
+// xor of the 16-byte words [w0, w1) of `base` taken by this thread (stride kReadThreads)
+__device__ __forceinline__ uint32_t fold_run(const uint4 *base, int32_t w0, int32_t w1) {
+    uint32_t acc = 0;
+    int32_t w = w0 + int32_t(threadIdx.x);
+    for (; w + 3 * kReadThreads < w1; w += 4 * kReadThreads) {
+        const uint32_t a0 = fold_ld(base + w), a1 = fold_ld(base + w + kReadThreads);
+        const uint32_t a2 = fold_ld(base + w + 2 * kReadThreads), a3 = fold_ld(base + w + 3 * kReadThreads);
+        acc ^= a0 ^ a1 ^ a2 ^ a3;
+    }
+    for (; w < w1; w += kReadThreads) acc ^= fold_ld(base + w);
+    return acc;
+}
+
+__global__ void __launch_bounds__(kReadThreads) read_kernel(const ReadArgs a) {
+    __shared__ uint32_t s_fold[kReadThreads / kWarp];
+    const int b = blockIdx.y, c = blockIdx.x;
+    if (!a.prefetch) pdl_wait();
+    int32_t L = a.lens[b];
+    L = (L >= 0 && L <= a.cap) ? L : 0;
+    const int32_t nw = (L + 3) / 4;  // cap is a multiple of 4: the last word stays inside the row
+    const int32_t per = (nw + a.split - 1) / a.split;
+    const int32_t w0 = min(nw, c * per), w1 = min(nw, w0 + per);
+    uint32_t acc = fold_run(reinterpret_cast<const uint4 *>(a.ctx + size_t(b) * size_t(a.cap)), w0, w1);
+    const int32_t hw = a.d / 8;
+    const int32_t hper = (hw + a.split - 1) / a.split;
+    const int32_t h0 = min(hw, c * hper), h1 = min(hw, h0 + hper);
+    acc ^= fold_run(reinterpret_cast<const uint4 *>(a.hidden + size_t(b) * size_t(a.d)), h0, h1);
+    if (a.prefetch) pdl_wait();
+    pdl_trigger();
+    for (int o = kWarp / 2; o > 0; o >>= 1) acc ^= __shfl_xor_sync(0xffffffffu, acc, o);
+    if ((threadIdx.x & (kWarp - 1)) == 0) s_fold[threadIdx.x / kWarp] = acc;
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        uint32_t r = 0;
+        for (int i = 0; i < kReadThreads / kWarp; ++i) r ^= s_fold[i];
+        a.out[size_t(b) * size_t(a.split) + c] = r;
+    }
+}
+
+}  // namespace switchsd
+
+extern "C" int switchsd_harness_read(const int32_t *ctx_tokens, const int32_t *ctx_lens, int32_t B, int32_t cap,
+                                     const uint16_t *hidden, int32_t d, int32_t split, int32_t prefetch,
+                                     uint32_t *out, void *stream) {
+    if (!ctx_tokens || !ctx_lens || !hidden || !out) return SWITCHSD_ERR_ARG;
+    if ((reinterpret_cast<uintptr_t>(ctx_tokens) & 15) != 0 || (reinterpret_cast<uintptr_t>(hidden) & 15) != 0 ||
+        (reinterpret_cast<uintptr_t>(out) & 3) != 0)
+        return SWITCHSD_ERR_ARG;
+    if (B < 1 || B > 65535 || cap < 4 || cap % 4 != 0 || d < 8 || d % 8 != 0 || split < 1 || split > 1024)
+        return SWITCHSD_ERR_SHAPE;
+    ReadArgs a;
+    a.ctx = ctx_tokens;
+    a.lens = ctx_lens;
+    a.hidden = hidden;
+    a.out = out;
+    a.B = B;
+    a.cap = cap;
+    a.d = d;
+    a.split = split;
+    a.prefetch = prefetch != 0;
+    const cudaError_t e = launch_pdl(read_kernel, dim3(unsigned(split), unsigned(B)), dim3(kReadThreads), 0,
+                                     static_cast<cudaStream_t>(stream), 0u, a);
+    return e == cudaSuccess ? SWITCHSD_OK : SWITCHSD_ERR_CUDA;
+}

@@ -7,6 +7,10 @@ one decoding iteration as three library calls on one stream:
     switchsd_harness_target  (stand-in for the neural drafter and the target forward)
     switchsd_verify          (controller: greedy verification and append)
 
+For inputs that arrive in host memory and decisions read back on the host, ``step_host`` and
+``verify_step_host`` make the host-to-device copy, the step and one device-to-host copy of every
+per-row result in a single library call (switchsd_step_host / switchsd_verify_step_host).
+
 Inputs arrive as numpy arrays (token ids int32, bf16 values as uint16 bit patterns) and are copied to
 the device once.  The buffers are checked once at construction; each call then passes the cached
 argument list straight to the C function, so the per-call host cost is one foreign call.  Nothing
@@ -144,6 +148,7 @@ class Session:
         self.vp = torch.zeros(B, k, **f32)
         self.vq = torch.ones(B, k, **f32)
         self.vu = torch.zeros(B, k, **f32)
+        self._io = bd.switchsd_host_io()  # host_io of the host-staged calls, refilled per call
 
     # --- the three calls ---------------------------------------------------------------------
     def _check_hidden(self, hidden: torch.Tensor, rows: int = 1) -> None:
@@ -230,9 +235,59 @@ class Session:
         """One asynchronous device-to-host copy of mode, draft length, accepted length and draft into
         `host` (pinned int32 [B * (k + 3)]); returns views of it.  Synchronise the stream before use."""
         host.copy_(self.results, non_blocking=True)
+        return self._host_views(host)
+
+    # --- host-staged calls (inputs and results in host memory) ------------------------------------
+    def _host_io(self, hidden_host: torch.Tensor, hidden: torch.Tensor, results_host: torch.Tensor,
+                 synchronize: bool):
+        if (hidden_host.device.type != "cpu" or not hidden_host.is_contiguous()
+                or hidden_host.numel() * hidden_host.element_size() != hidden.numel() * hidden.element_size()):
+            raise ValueError("hidden_host must be a contiguous host tensor with the bytes of hidden")
+        if (results_host.device.type != "cpu" or results_host.dtype != torch.int32
+                or not results_host.is_contiguous() or results_host.numel() != self.results.numel()):
+            raise ValueError("results_host must be a contiguous host int32 tensor of B * (k + 3) entries")
+        io = self._io
+        io.in_host, io.in_dev = hidden_host.data_ptr(), hidden.data_ptr()
+        io.in_bytes = hidden.numel() * hidden.element_size()
+        io.out_dev, io.out_host = self.results.data_ptr(), results_host.data_ptr()
+        io.out_bytes = self.results.numel() * 4
+        io.synchronize = int(bool(synchronize))
+        return io
+
+    def _host_views(self, host: torch.Tensor) -> dict:
         B, k = self.B, self.k
         return {"mode": host[0:B], "len": host[B:2 * B], "accept": host[2 * B:3 * B],
                 "draft": host[3 * B:].view(B, k)}
+
+    def step_host(self, hidden_host: torch.Tensor, hidden: torch.Tensor, results_host: torch.Tensor,
+                  debug: bool = False, synchronize: bool = True) -> dict:
+        """switchsd_step_host: the bytes of hidden_host (host, pinned) are copied into `hidden` (the
+        device [B, d] buffer the step reads), the step runs, and mode / draft length / accepted length /
+        draft come back into results_host (host int32 [B * (k + 3)], pinned) in one copy -- one library
+        call.  With synchronize the call returns when results_host is filled.  Returns its views."""
+        self._check_hidden(hidden)
+        io = self._host_io(hidden_host, hidden, results_host, synchronize)
+        p = self._p_dbg if debug else self._p_fast
+        rows, p.hidden_rows = p.hidden_rows, 0
+        code = self.lib.switchsd_step_host(ctypes.byref(io), *self._step_head, hidden.data_ptr(), *self._step_tail,
+                                           ctypes.byref(p), *self._step_outs)
+        p.hidden_rows = rows
+        if code != bd.OK:
+            raise RuntimeError(f"switchsd_step_host failed: {code} ({bd.strerror(code)})")
+        return self._host_views(results_host)
+
+    def verify_step_host(self, hidden_host: torch.Tensor, hidden: torch.Tensor, results_host: torch.Tensor,
+                         debug: bool = False, synchronize: bool = True) -> dict:
+        """switchsd_verify_step_host: verify_step between the copies of step_host, in one library call."""
+        self._check_hidden(hidden, self.hidden_rows)
+        io = self._host_io(hidden_host, hidden, results_host, synchronize)
+        p = self._p_dbg if debug else self._p_fast
+        code = self.lib.switchsd_verify_step_host(ctypes.byref(io), *self._vs_head, self.ctx.data_ptr(),
+                                                  self.lens.data_ptr(), hidden.data_ptr(), *self._step_tail,
+                                                  ctypes.byref(p), *self._step_outs)
+        if code != bd.OK:
+            raise RuntimeError(f"switchsd_verify_step_host failed: {code} ({bd.strerror(code)})")
+        return self._host_views(results_host)
 
     # --- host views ------------------------------------------------------------------------------
     def step_outputs(self) -> dict:

@@ -58,7 +58,7 @@ def test_binding_declares_every_function():
 
 def test_abi_version_and_strerror(lib):
     from paper_2609_20186_gb300 import binding as bd
-    assert bd.abi_version() == 4
+    assert bd.abi_version() == 5
     for code in (0, -1, -2, -3, 1, 2, 3):
         assert bd.strerror(code) != "unknown code"
     assert bd.strerror(12345) == "unknown code"
@@ -163,6 +163,39 @@ def test_labels_validation(lib):
     assert lib.switchsd_copy_labels(f, f, 4, 1000, 0, f, f, need, None) == bd.ERR_SHAPE
     assert lib.switchsd_copy_labels(f, f, 4, 1000, 33, f, f, need, None) == bd.ERR_SHAPE
     assert lib.switchsd_copy_labels(f, f, 0, 1000, 5, f, f, need, None) == bd.ERR_SHAPE
+
+
+def test_host_staged_validation(lib):
+    """switchsd_step_host / switchsd_verify_step_host reject a bad io before any copy, and pass a bad
+    step on unchanged (no byte counts: nothing is queued before the step's own validation)."""
+    from paper_2609_20186_gb300 import binding as bd
+    f = FAKE
+    io = bd.switchsd_host_io()
+    p = _params()
+    assert lib.switchsd_step_host(None, f, f, f, f, ctypes.byref(p), f, f, f, f) == bd.ERR_ARG
+    assert lib.switchsd_step_host(ctypes.byref(io), f, f, f, f, None, f, f, f, f) == bd.ERR_ARG
+    io.in_bytes = 64                                     # a copy with no buffers
+    assert lib.switchsd_step_host(ctypes.byref(io), f, f, f, f, ctypes.byref(p), f, f, f, f) == bd.ERR_ARG
+    io.in_bytes, io.out_bytes = 0, 64
+    assert lib.switchsd_verify_step_host(ctypes.byref(io), f, f, f, f, f, f, f, f, ctypes.byref(p),
+                                         f, f, f, f) == bd.ERR_ARG
+    io.out_bytes = 0
+    bad = _params(B=0)
+    assert lib.switchsd_step_host(ctypes.byref(io), f, f, f, f, ctypes.byref(bad), f, f, f, f) == bd.ERR_SHAPE
+    assert lib.switchsd_verify_step_host(ctypes.byref(io), f, f, f, f, f, f, f, f, ctypes.byref(bad),
+                                         f, f, f, f) == bd.ERR_SHAPE
+
+
+def test_read_ceiling_validation(lib):
+    from paper_2609_20186_gb300 import binding as bd
+    f = FAKE
+    assert lib.switchsd_harness_read(None, f, 4, 64, f, 16, 8, 1, f, None) == bd.ERR_ARG
+    assert lib.switchsd_harness_read(f + 4, f, 4, 64, f, 16, 8, 1, f, None) == bd.ERR_ARG   # misaligned
+    assert lib.switchsd_harness_read(f, f, 4, 64, f + 2, 16, 8, 1, f, None) == bd.ERR_ARG
+    assert lib.switchsd_harness_read(f, f, 4, 66, f, 16, 8, 1, f, None) == bd.ERR_SHAPE     # cap % 4
+    assert lib.switchsd_harness_read(f, f, 4, 64, f, 12, 8, 1, f, None) == bd.ERR_SHAPE     # d % 8
+    assert lib.switchsd_harness_read(f, f, 4, 64, f, 16, 0, 1, f, None) == bd.ERR_SHAPE     # split
+    assert lib.switchsd_harness_read(f, f, 0, 64, f, 16, 8, 1, f, None) == bd.ERR_SHAPE
 
 
 def test_binding_rejects_cpu_tensors(lib):

@@ -1,0 +1,90 @@
+"""The host-staged entry points and the read ceiling on the GPU, through the C ABI.
+
+switchsd_step_host / switchsd_verify_step_host must give exactly what the device-buffer calls give
+(same contexts, outputs and accepted lengths, step after step) with the hidden states taken from host
+memory and the results delivered to host memory.  switchsd_harness_read must fold exactly the words it
+is documented to read (checked against numpy)."""
+import numpy as np
+import pytest
+
+import synth
+
+pytestmark = pytest.mark.gpu
+
+
+def _session(wl, prefetch):
+    from paper_2609_20186_gb300 import Session, binding
+    ctx, lens = wl.contexts()
+    return Session(ctx, lens, wl.probe_weights(), k=wl.k, n_min=wl.n_min, n_max=wl.n_max, kappa=wl.kappa,
+                   logit_tau=wl.logit_tau, probe_kind=wl.probe_kind, probe_hidden=wl.probe_hidden,
+                   future=wl.future(), harness=wl.harness_params(), d=wl.d,
+                   prefetch=(binding.PREFETCH_CONTEXT | binding.PREFETCH_PROBE) if prefetch else 0)
+
+
+@pytest.mark.parametrize("name", ["zipf_32k", "code_16k"])
+@pytest.mark.parametrize("prefetch", [False, True])
+def test_host_staged_matches_device_calls(name, prefetch):
+    import torch
+    from paper_2609_20186_gb300 import bf16_tensor
+    wl = synth.WORKLOADS[name].scaled(B=8, L0=6001, steps=10)
+    a, b = _session(wl, prefetch), _session(wl, prefetch)
+    B, d, k = wl.B, wl.d, wl.k
+    dev_h = torch.empty(B, d, dtype=torch.bfloat16, device="cuda")
+    host_h = torch.empty(B, d, dtype=torch.int16).pin_memory()
+    host_out = torch.empty(B * (k + 3), dtype=torch.int32).pin_memory()
+    for t in range(wl.steps):
+        hid = wl.hidden(t)
+        host_h.copy_(torch.from_numpy(hid.view(np.int16)))
+        if t == 0:
+            a.step(bf16_tensor(hid, "cuda"), debug=False)
+            got = b.step_host(host_h, dev_h, host_out)
+        else:
+            a.harness(t - 1)
+            b.harness(t - 1)
+            a.verify_step(bf16_tensor(hid, "cuda"), debug=False)
+            got = b.verify_step_host(host_h, dev_h, host_out)
+        torch.cuda.synchronize()
+        want = a.results.cpu().numpy()
+        assert np.array_equal(host_out.numpy(), want), (name, t)
+        assert np.array_equal(got["draft"].numpy(), want[3 * B:].reshape(B, k))
+        assert np.array_equal(a.lens.cpu().numpy(), b.lens.cpu().numpy()), (name, t)
+        assert np.array_equal(a.score.cpu().numpy(), b.score.cpu().numpy()), (name, t)
+    assert np.array_equal(a.ctx.cpu().numpy(), b.ctx.cpu().numpy())
+
+
+def test_host_staged_without_sync_then_stream_sync():
+    import torch
+    wl = synth.WORKLOADS["uniform_8k"].scaled(B=4, L0=3000, steps=3)
+    s = _session(wl, False)
+    B, d, k = wl.B, wl.d, wl.k
+    dev_h = torch.empty(B, d, dtype=torch.bfloat16, device="cuda")
+    host_h = torch.from_numpy(wl.hidden(0).view(np.int16)).pin_memory()
+    host_out = torch.full((B * (k + 3),), -7, dtype=torch.int32).pin_memory()
+    s.step_host(host_h, dev_h, host_out, synchronize=False)
+    torch.cuda.current_stream().synchronize()
+    assert np.array_equal(host_out.numpy(), s.results.cpu().numpy())
+
+
+@pytest.mark.parametrize("prefetch", [0, 1])
+@pytest.mark.parametrize("split", [1, 3, 8, 32])
+def test_read_ceiling_folds_what_it_reads(split, prefetch):
+    import torch
+    from paper_2609_20186_gb300 import binding as bd
+    lib = bd.load()
+    rng = np.random.default_rng(5)
+    B, cap, d = 5, 4100, 136
+    ctx = rng.integers(-2**31, 2**31 - 1, size=(B, cap), dtype=np.int64).astype(np.int32)
+    lens = np.array([0, 1, 4099, 4100, 1234], np.int32)
+    hid = rng.integers(0, 2**16, size=(B, d), dtype=np.int64).astype(np.uint16)
+    c, ln = torch.from_numpy(ctx).cuda(), torch.from_numpy(lens).cuda()
+    h = torch.from_numpy(hid.view(np.int16)).cuda()
+    out = torch.full((B * split,), 0x5A5A, dtype=torch.int32, device="cuda")
+    s = torch.cuda.current_stream().cuda_stream
+    assert lib.switchsd_harness_read(c.data_ptr(), ln.data_ptr(), B, cap, h.data_ptr(), d, split, prefetch,
+                                     out.data_ptr(), s) == 0
+    got = out.cpu().numpy().view(np.uint32).reshape(B, split)
+    for b in range(B):
+        words = 4 * ((int(lens[b]) + 3) // 4)   # whole 16-byte words covering the first L tokens
+        want = np.bitwise_xor.reduce(ctx[b, :words].view(np.uint32)) if words else np.uint32(0)
+        want ^= np.bitwise_xor.reduce(hid[b].view(np.uint32))
+        assert np.bitwise_xor.reduce(got[b]) == want, b
