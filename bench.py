@@ -815,9 +815,10 @@ def read_ceiling(loop, d: int, K: int, step_base: int, prefetch: bool, cs) -> di
 
 def run_e2e(base, dev, W, K, split, world, prefetch=True, sampled=False):
     """The same loop through the public API with host buffers, one batch.  Per step (greedy): the
-    target stand-in for the previous draft, then one switchsd_verify_step_host call -- pinned H2D of
-    this step's hidden states, the fused launch, one D2H of mode / draft length / accepted length /
-    draft, host sync.  Sampled: the same copies and launches as separate calls."""
+    target stand-in for the previous draft, then one replay of a switchsd_plan of
+    switchsd_verify_step_host -- pinned H2D of this step's hidden states, the fused launch, one D2H of
+    mode / draft length / accepted length / draft -- and a host sync.  Sampled: the same copies and
+    launches as separate stream-ordered calls."""
     import torch
     from paper_2609_20186_gb300 import Session, binding
 
@@ -835,6 +836,8 @@ def run_e2e(base, dev, W, K, split, world, prefetch=True, sampled=False):
     dev_h = torch.empty(B, d, dtype=torch.bfloat16, device=dev)
     host_out = torch.empty(B * (k + 3), dtype=torch.int32).pin_memory()  # mode, len, accept, draft
     stream = torch.cuda.current_stream()
+    # switchsd_plan: the host-staged fused step (switchsd_verify_step_host) recorded once as a graph
+    plan = None if sampled else sess.host_plan(host_h[1], dev_h, host_out, verify=True)
 
     def one(t):
         if t == 0:
@@ -848,7 +851,7 @@ def run_e2e(base, dev, W, K, split, world, prefetch=True, sampled=False):
             stream.synchronize()
             return
         sess.harness(t - 1)            # the target's tokens for the previous draft
-        sess.verify_step_host(host_h[t], dev_h, host_out)
+        plan.run(host_h[t])            # H2D of this step's hidden states, the fused launch, D2H, sync
 
     for t in range(W):
         one(t)
@@ -864,8 +867,9 @@ def run_e2e(base, dev, W, K, split, world, prefetch=True, sampled=False):
             "note": ("one batch; per step: target stand-in, then " +
                      ("pinned H2D of hidden, switchsd_verify_sampled_step, D2H of mode/len/accept/draft, "
                       "host sync" if sampled else
-                      "one switchsd_verify_step_host call (pinned H2D of hidden, fused launch, one D2H of "
-                      "mode/len/accept/draft, host sync)") + "; L2 not flushed")}
+                      "one switchsd_plan_run call replaying switchsd_verify_step_host recorded as a CUDA "
+                      "graph (pinned H2D of hidden, fused launch, one D2H of mode/len/accept/draft), host "
+                      "sync") + "; L2 not flushed")}
 
 
 LABEL_METRIC = "copy-mode labels/sec (positions, §3.2, n_train=5); achieved HBM GB/s vs peak"

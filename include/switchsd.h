@@ -280,9 +280,11 @@ int switchsd_verify_sampled_step(const int32_t *draft, const float *p_draft, con
  * memory and results read back on the host, in one call.  Before the step, in_bytes are copied from
  * in_host to in_dev (device; typically the hidden states the step then reads); after it, out_bytes
  * from out_dev (device; typically one buffer holding the step's mode, draft length, accepted length
- * and draft) to out_host.  Both copies are cudaMemcpyAsync on params->stream, ordered with the step's
- * launch; host buffers should be pinned for the copies to be asynchronous.  A zero byte count skips
- * that copy.  synchronize != 0: the call returns after the stream has drained, so out_host holds the
+ * and draft) to out_host.  Both copies run on params->stream, ordered with the step: for page-locked
+ * host memory mapped into the device's address space (any pinned allocation under unified addressing)
+ * as a small kernel that reads or writes the host buffer through its device address, otherwise as
+ * cudaMemcpyAsync.  After an input copy by kernel the step keeps a SWITCHSD_PREFETCH_* bit only if
+ * the copied range misses the inputs that bit covers.  A zero byte count skips that copy.  synchronize != 0: the call returns after the stream has drained, so out_host holds the
  * results; 0: everything is queued on the stream and the call returns at once.
  */
 typedef struct {
@@ -308,6 +310,49 @@ int switchsd_verify_step_host(const switchsd_host_io *io, const int32_t *draft, 
                               int32_t *ctx_lens, const uint16_t *hidden, const uint16_t *probe_w,
                               const switchsd_params *params, int32_t *out_draft, int32_t *out_len,
                               int32_t *out_mode, float *out_score);
+
+/*
+ * The arguments of one switchsd_verify_step call (draft, target_argmax and draft_len all set), or of
+ * one switchsd_step call (all three NULL; out_accept is then unused), for switchsd_plan_create.
+ */
+typedef struct {
+    const int32_t *draft, *target_argmax, *draft_len;
+    int32_t *out_accept;
+    int32_t *ctx_tokens, *ctx_lens;
+    const uint16_t *hidden, *probe_w;
+    const switchsd_params *params;
+    int32_t *out_draft, *out_len, *out_mode;
+    float *out_score;
+} switchsd_step_args;
+
+/* A host-staged step recorded once as a CUDA graph (opaque). */
+typedef struct switchsd_plan switchsd_plan;
+
+/*
+ * Records what switchsd_verify_step_host (or switchsd_step_host) does with `args` and `io` -- the H2D
+ * copy, the step's launch(es), the D2H copy -- into a CUDA graph, by stream capture on a private
+ * stream; nothing runs.  io->synchronize is ignored (switchsd_plan_run takes it).  The recorded
+ * launches hold the device pointers and the parameter values, so *args and *args->params may be freed
+ * after the call; replays launch on args->params->stream.  The caller keeps every buffer alive and, for
+ * the two-layer probe, the workspace unshared while the plan can run.  Returns SWITCHSD_ERR_ARG (NULL out, args, params or io, a partial set of verification
+ * buffers, a copy without buffers), SWITCHSD_ERR_CUDA (capture or instantiation failed), or the step's
+ * own validation code; *out is then NULL.
+ */
+int switchsd_plan_create(const switchsd_step_args *args, const switchsd_host_io *io, switchsd_plan **out);
+
+/*
+ * Replays the plan on its stream.  in_host / out_host: the host ends of the two copies for this
+ * replay (NULL: the ones of the last replay, first those of io at creation); the device ends and byte
+ * counts are fixed, and a copy recorded as a kernel (pinned buffer at creation) takes pinned buffers
+ * only.  synchronize != 0: returns after the stream has drained.  Equivalent to the switchsd_*_host
+ * call it recorded.  SWITCHSD_ERR_ARG for a NULL plan or a pageable buffer where a pinned one was
+ * recorded, SWITCHSD_ERR_CUDA if a copy could not be retargeted or the launch or synchronisation
+ * failed.
+ */
+int switchsd_plan_run(switchsd_plan *plan, const void *in_host, void *out_host, int32_t synchronize);
+
+/* Frees the plan's graph (NULL is ignored).  The plan must not be running. */
+void switchsd_plan_destroy(switchsd_plan *plan);
 
 /*
  * Bytes of device workspace switchsd_step / switchsd_verify_step need for `params` (0 for the linear

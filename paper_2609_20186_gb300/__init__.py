@@ -12,4 +12,4 @@ from .binding import (  # noqa: F401
     switchsd_verify_params, switchsd_harness_params, NgramIndex, load, strerror, abi_version,
     MODE_NO_REP, MODE_COPY, MODE_REP_NO_COPY, PROBE_LINEAR, PROBE_MLP,
 )
-from .session import Session, bf16_tensor  # noqa: F401
+from .session import HostPlan, Session, bf16_tensor  # noqa: F401

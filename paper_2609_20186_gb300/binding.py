@@ -69,6 +69,17 @@ class switchsd_host_io(ctypes.Structure):
     ]
 
 
+class switchsd_step_args(ctypes.Structure):
+    _fields_ = [
+        ("draft", ctypes.c_void_p), ("target_argmax", ctypes.c_void_p), ("draft_len", ctypes.c_void_p),
+        ("out_accept", ctypes.c_void_p), ("ctx_tokens", ctypes.c_void_p), ("ctx_lens", ctypes.c_void_p),
+        ("hidden", ctypes.c_void_p), ("probe_w", ctypes.c_void_p),
+        ("params", ctypes.POINTER(switchsd_params)),
+        ("out_draft", ctypes.c_void_p), ("out_len", ctypes.c_void_p), ("out_mode", ctypes.c_void_p),
+        ("out_score", ctypes.c_void_p),
+    ]
+
+
 class switchsd_harness_params(ctypes.Structure):
     _fields_ = [
         ("B", ctypes.c_int32), ("k", ctypes.c_int32), ("V", ctypes.c_int32), ("L0", ctypes.c_int32),
@@ -101,6 +112,10 @@ _SIGNATURES = {
     "switchsd_harness_read": (ctypes.c_int, [ctypes.c_void_p, ctypes.c_void_p, ctypes.c_int32, ctypes.c_int32,
                                              ctypes.c_void_p, ctypes.c_int32, ctypes.c_int32, ctypes.c_int32,
                                              ctypes.c_void_p, ctypes.c_void_p]),
+    "switchsd_plan_create": (ctypes.c_int, [ctypes.POINTER(switchsd_step_args), ctypes.POINTER(switchsd_host_io),
+                                            ctypes.POINTER(ctypes.c_void_p)]),
+    "switchsd_plan_run": (ctypes.c_int, [ctypes.c_void_p, ctypes.c_void_p, ctypes.c_void_p, ctypes.c_int32]),
+    "switchsd_plan_destroy": (None, [ctypes.c_void_p]),
     "switchsd_step_static_workspace": (ctypes.c_int, [ctypes.c_void_p] * 4
                                        + [ctypes.POINTER(switchsd_params)] + [ctypes.c_void_p] * 4),
     "switchsd_index_create": (ctypes.c_int, [ctypes.POINTER(switchsd_params),

@@ -289,9 +289,76 @@ class Session:
             raise RuntimeError(f"switchsd_verify_step_host failed: {code} ({bd.strerror(code)})")
         return self._host_views(results_host)
 
+    def host_plan(self, hidden_host: torch.Tensor, hidden: torch.Tensor, results_host: torch.Tensor,
+                  verify: bool = True, debug: bool = False) -> "HostPlan":
+        """switchsd_plan_create: what verify_step_host (verify=True) or step_host does with these buffers,
+        recorded once as a CUDA graph; HostPlan.run replays it with this step's host buffers."""
+        self._check_hidden(hidden, self.hidden_rows if verify else 1)
+        io = bd.switchsd_host_io.from_buffer_copy(self._host_io(hidden_host, hidden, results_host, False))
+        p = bd.switchsd_params.from_buffer_copy(self._p_dbg if debug else self._p_fast)
+        if not verify:
+            p.hidden_rows = 0
+        a = bd.switchsd_step_args()
+        if verify:
+            a.draft, a.target_argmax, a.draft_len, a.out_accept = self._vs_head
+        a.ctx_tokens, a.ctx_lens = self._step_head
+        a.hidden, a.probe_w = hidden.data_ptr(), self.probe_w.data_ptr()
+        a.params = ctypes.pointer(p)
+        a.out_draft, a.out_len, a.out_mode, a.out_score = self._step_outs
+        h = ctypes.c_void_p()
+        code = self.lib.switchsd_plan_create(ctypes.byref(a), ctypes.byref(io), ctypes.byref(h))
+        if code != bd.OK:
+            raise RuntimeError(f"switchsd_plan_create failed: {code} ({bd.strerror(code)})")
+        return HostPlan(self, h, io.in_bytes, (hidden_host, hidden, results_host))
+
     # --- host views ------------------------------------------------------------------------------
     def step_outputs(self) -> dict:
         return {"draft": self.draft.cpu().numpy(), "len": self.len.cpu().numpy(),
                 "mode": self.mode.cpu().numpy(), "score": self.score.cpu().numpy(),
                 "match_n": self.match_n.cpu().numpy(), "match_end": self.match_end.cpu().numpy(),
                 "status": self.status.cpu().numpy()}
+
+
+class HostPlan:
+    """A recorded host-staged step (switchsd_plan) of a Session.  run() replays it: H2D of this step's
+    hidden states from host memory, the step, one D2H of the results, and (by default) a host wait."""
+
+    def __init__(self, session: Session, handle: ctypes.c_void_p, in_bytes: int, keep):
+        self.session, self.handle, self.in_bytes = session, handle, in_bytes
+        self._keep = keep  # the buffers recorded at creation stay alive with the plan
+
+    def run(self, hidden_host: torch.Tensor | None = None, results_host: torch.Tensor | None = None,
+            synchronize: bool = True) -> None:
+        """hidden_host: host tensor with the hidden states' bytes (pinned; None: the last one);
+        results_host: pinned host int32 [B * (k + 3)] (None: the last one).  After a synchronised run
+        (or a stream synchronisation) ``results()`` holds this replay's results."""
+        if self.handle is None:
+            raise RuntimeError("the plan was closed")
+        hp = rp = None
+        if hidden_host is not None:
+            if hidden_host.device.type != "cpu" or hidden_host.numel() * hidden_host.element_size() != self.in_bytes:
+                raise ValueError("hidden_host must be a host tensor with the bytes of the recorded hidden states")
+            hp = hidden_host.data_ptr()
+        if results_host is not None:
+            if results_host.device.type != "cpu" or results_host.numel() != self.session.results.numel():
+                raise ValueError("results_host must be a host int32 tensor of B * (k + 3) entries")
+            rp = results_host.data_ptr()
+            self._keep = self._keep[:2] + (results_host,)
+        code = self.session.lib.switchsd_plan_run(self.handle, hp, rp, int(bool(synchronize)))
+        if code != bd.OK:
+            raise RuntimeError(f"switchsd_plan_run failed: {code} ({bd.strerror(code)})")
+
+    def results(self) -> dict:
+        """Views (mode, len, accept, draft) of the host buffer the last replay wrote."""
+        return self.session._host_views(self._keep[2])
+
+    def close(self) -> None:
+        if self.handle is not None:
+            self.session.lib.switchsd_plan_destroy(self.handle)
+            self.handle = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass

@@ -186,6 +186,33 @@ def test_host_staged_validation(lib):
                                          f, f, f, f) == bd.ERR_SHAPE
 
 
+def test_plan_validation(lib):
+    """switchsd_plan_create / _run / _destroy reject bad arguments before any CUDA call."""
+    from paper_2609_20186_gb300 import binding as bd
+    f = FAKE
+    io = bd.switchsd_host_io()
+    p = _params()
+    a = bd.switchsd_step_args()
+    a.ctx_tokens = a.ctx_lens = a.hidden = a.probe_w = f
+    a.out_draft = a.out_len = a.out_mode = a.out_score = f
+    a.params = ctypes.pointer(p)
+    h = ctypes.c_void_p(12345)
+    assert lib.switchsd_plan_create(ctypes.byref(a), ctypes.byref(io), None) == bd.ERR_ARG
+    assert lib.switchsd_plan_create(None, ctypes.byref(io), ctypes.byref(h)) == bd.ERR_ARG
+    assert h.value is None                               # *out is cleared on failure
+    assert lib.switchsd_plan_create(ctypes.byref(a), None, ctypes.byref(h)) == bd.ERR_ARG
+    a.draft = f                                          # a partial set of verification buffers
+    assert lib.switchsd_plan_create(ctypes.byref(a), ctypes.byref(io), ctypes.byref(h)) == bd.ERR_ARG
+    a.draft = None
+    io.in_bytes = 16                                     # a copy without buffers
+    assert lib.switchsd_plan_create(ctypes.byref(a), ctypes.byref(io), ctypes.byref(h)) == bd.ERR_ARG
+    a.params = None
+    io.in_bytes = 0
+    assert lib.switchsd_plan_create(ctypes.byref(a), ctypes.byref(io), ctypes.byref(h)) == bd.ERR_ARG
+    assert lib.switchsd_plan_run(None, None, None, 1) == bd.ERR_ARG
+    lib.switchsd_plan_destroy(None)
+
+
 def test_read_ceiling_validation(lib):
     from paper_2609_20186_gb300 import binding as bd
     f = FAKE

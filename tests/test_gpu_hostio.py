@@ -1,8 +1,8 @@
 """The host-staged entry points and the read ceiling on the GPU, through the C ABI.
 
-switchsd_step_host / switchsd_verify_step_host must give exactly what the device-buffer calls give
-(same contexts, outputs and accepted lengths, step after step) with the hidden states taken from host
-memory and the results delivered to host memory.  switchsd_harness_read must fold exactly the words it
+switchsd_step_host / switchsd_verify_step_host, and switchsd_plan replays of them, must give exactly
+what the device-buffer calls give (same contexts, outputs and accepted lengths, step after step) with
+the hidden states taken from host memory and the results delivered to host memory.  switchsd_harness_read must fold exactly the words it
 is documented to read (checked against numpy)."""
 import numpy as np
 import pytest
@@ -88,3 +88,73 @@ def test_read_ceiling_folds_what_it_reads(split, prefetch):
         want = np.bitwise_xor.reduce(ctx[b, :words].view(np.uint32)) if words else np.uint32(0)
         want ^= np.bitwise_xor.reduce(hid[b].view(np.uint32))
         assert np.bitwise_xor.reduce(got[b]) == want, b
+
+
+@pytest.mark.parametrize("name", ["zipf_32k", "code_16k"])
+@pytest.mark.parametrize("prefetch", [False, True])
+def test_plan_replays_match_device_calls(name, prefetch):
+    """Replays alternate between two host hidden buffers and two host result buffers, so the recorded
+    copies are retargeted on every replay."""
+    import torch
+    from paper_2609_20186_gb300 import bf16_tensor
+    wl = synth.WORKLOADS[name].scaled(B=8, L0=6001, steps=12)
+    a, b = _session(wl, prefetch), _session(wl, prefetch)
+    B, d, k = wl.B, wl.d, wl.k
+    dev_h = torch.empty(B, d, dtype=torch.bfloat16, device="cuda")
+    host_h = [torch.empty(B, d, dtype=torch.int16).pin_memory() for _ in range(2)]
+    host_out = [torch.empty(B * (k + 3), dtype=torch.int32).pin_memory() for _ in range(2)]
+    first = b.host_plan(host_h[0], dev_h, host_out[0], verify=False)
+    plan = b.host_plan(host_h[1], dev_h, host_out[1], verify=True)
+    for t in range(wl.steps):
+        hid = wl.hidden(t)
+        hh, ho = host_h[t % 2], host_out[(t // 2) % 2]
+        hh.copy_(torch.from_numpy(hid.view(np.int16)))
+        if t == 0:
+            a.step(bf16_tensor(hid, "cuda"), debug=False)
+            first.run(hh, ho)
+            got = first.results()
+        else:
+            a.harness(t - 1)
+            b.harness(t - 1)
+            a.verify_step(bf16_tensor(hid, "cuda"), debug=False)
+            plan.run(hh, ho)
+            got = plan.results()
+        torch.cuda.synchronize()
+        want = a.results.cpu().numpy()
+        assert np.array_equal(ho.numpy(), want), (name, t)
+        assert np.array_equal(got["mode"].numpy(), want[:B])
+        assert np.array_equal(a.lens.cpu().numpy(), b.lens.cpu().numpy()), (name, t)
+        assert np.array_equal(a.score.cpu().numpy(), b.score.cpu().numpy()), (name, t)
+    assert np.array_equal(a.ctx.cpu().numpy(), b.ctx.cpu().numpy())
+    first.close()
+    plan.close()
+    plan.close()  # idempotent
+
+
+@pytest.mark.parametrize("pinned", [False, True])
+def test_host_staged_pageable_and_pinned(pinned):
+    """Pageable host buffers take the copy engine, pinned ones the copy kernels: same results."""
+    import torch
+    from paper_2609_20186_gb300 import bf16_tensor
+    wl = synth.WORKLOADS["zipf_32k"].scaled(B=4, L0=5003, steps=5)
+    a, b = _session(wl, True), _session(wl, True)
+    B, d, k = wl.B, wl.d, wl.k
+    dev_h = torch.empty(B, d, dtype=torch.bfloat16, device="cuda")
+    host_h = torch.empty(B, d, dtype=torch.int16)
+    host_out = torch.empty(B * (k + 3), dtype=torch.int32)
+    if pinned:
+        host_h, host_out = host_h.pin_memory(), host_out.pin_memory()
+    for t in range(wl.steps):
+        hid = wl.hidden(t)
+        host_h.copy_(torch.from_numpy(hid.view(np.int16)))
+        if t == 0:
+            a.step(bf16_tensor(hid, "cuda"), debug=False)
+            b.step_host(host_h, dev_h, host_out)
+        else:
+            a.harness(t - 1)
+            b.harness(t - 1)
+            a.verify_step(bf16_tensor(hid, "cuda"), debug=False)
+            b.verify_step_host(host_h, dev_h, host_out)
+        torch.cuda.synchronize()
+        assert np.array_equal(host_out.numpy(), a.results.cpu().numpy()), t
+    assert np.array_equal(a.ctx.cpu().numpy(), b.ctx.cpu().numpy())
