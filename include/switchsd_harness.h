@@ -81,9 +81,10 @@ int switchsd_harness_candidates(const int32_t *ctx_lens, const int32_t *mode, co
  * what one step reads -- the first ctx_lens[b] tokens of every row (rounded up to whole 16-byte
  * words) and the hidden states -- and nothing else: grid (split, B) of 256-thread CTAs, CTA (c, b)
  * taking the c-th of `split` equal runs of row b's context words and of its d bf16 hidden values,
- * 16-byte loads four in flight per thread, xor-folded into out[b * split + c] so no load is dead.
- * prefetch != 0 issues the loads before the kernel's grid-dependency wait (as the step kernel does
- * under SWITCHSD_PREFETCH_CONTEXT | SWITCHSD_PREFETCH_PROBE), else after it; launched with
+ * copied into shared memory by bulk (TMA) copies in chunks of up to 64 KB and xor-folded into
+ * out[b * split + c] so no byte is left unread (~0u if a copy did not complete in time).  prefetch
+ * != 0 issues the first chunk's copies before the kernel's grid-dependency wait (as the step kernel
+ * does under SWITCHSD_PREFETCH_CONTEXT | SWITCHSD_PREFETCH_PROBE), else after it; launched with
  * programmatic stream serialization like every kernel of the library.
  * ctx_tokens int32 [B, cap] (16-byte aligned, cap a multiple of 4), ctx_lens int32 [B] (a length
  * outside [0, cap] reads nothing), hidden bf16 bits [B, d] (16-byte aligned, d a multiple of 8),

@@ -239,15 +239,18 @@ extern "C" int switchsd_harness_candidates(const int32_t *ctx_lens, const int32_
 
 // ------------------------------------------------------------------------------------------------
 // switchsd_harness_read: a plain read of what one step reads, the size-matched ceiling for the step
-// kernel.  Grid (split, B): CTA (c, b) reads the c-th of `split` equal runs of the 16-byte words that
-// hold row b's first ctx_lens[b] tokens, and the c-th run of row b's hidden states, with 16-byte
-// non-coherent loads, four in flight per thread; the words are xor-folded into out[b * split + c] so
-// no load is dead.  prefetch != 0 issues the loads before the grid-dependency wait (the step kernel's
-// SWITCHSD_PREFETCH_CONTEXT / _PROBE order), else after it.
+// kernel.  Grid (split, B): CTA (c, b) takes the c-th of `split` equal runs of the 16-byte words that
+// hold row b's first ctx_lens[b] tokens, then the c-th run of row b's hidden states, copies them into
+// shared memory with bulk (TMA) copies in chunks of up to 64 KB, and xor-folds every word it received
+// into out[b * split + c], so no byte is left unread.  prefetch != 0 issues the first chunk's copies
+// before the grid-dependency wait (the step kernel's SWITCHSD_PREFETCH_CONTEXT / _PROBE order), else
+// after it.  Bulk copies into shared memory read faster than 16-byte loads from every thread on this
+// workload's sizes, so this is the faster of the two plain reads.
 // ------------------------------------------------------------------------------------------------
 namespace switchsd {
 
 constexpr int kReadThreads = 256;
+constexpr int32_t kReadChunkWords = 4096;  // 16-byte words per chunk: 64 KB of shared memory
 
 struct ReadArgs {
     const int32_t *ctx, *lens;
@@ -256,50 +259,65 @@ struct ReadArgs {
     int32_t B, cap, d, split, prefetch;
 };
 
-__device__ __forceinline__ uint32_t fold_ld(const uint4 *p) {
-    uint4 v;
-    asm volatile("ld.global.nc.L1::no_allocate.v4.u32 {%0, %1, %2, %3}, [%4];\n"
-                 : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
-                 : "l"(p));
-    return v.x ^ v.y ^ v.z ^ v.w;
-}
-
-// xor of the 16-byte words [w0, w1) of `base` taken by this thread (stride kReadThreads)
-__device__ __forceinline__ uint32_t fold_run(const uint4 *base, int32_t w0, int32_t w1) {
-    uint32_t acc = 0;
-    int32_t w = w0 + int32_t(threadIdx.x);
-    for (; w + 3 * kReadThreads < w1; w += 4 * kReadThreads) {
-        const uint32_t a0 = fold_ld(base + w), a1 = fold_ld(base + w + kReadThreads);
-        const uint32_t a2 = fold_ld(base + w + 2 * kReadThreads), a3 = fold_ld(base + w + 3 * kReadThreads);
-        acc ^= a0 ^ a1 ^ a2 ^ a3;
-    }
-    for (; w < w1; w += kReadThreads) acc ^= fold_ld(base + w);
-    return acc;
-}
-
 __global__ void __launch_bounds__(kReadThreads) read_kernel(const ReadArgs a) {
+    extern __shared__ __align__(128) uint4 s_chunk[];
+    __shared__ uint64_t s_bar;
     __shared__ uint32_t s_fold[kReadThreads / kWarp];
     const int b = blockIdx.y, c = blockIdx.x;
+    if (threadIdx.x == 0) {
+        mbar_init(&s_bar, 1);
+        fence_mbar_init();
+    }
+    __syncthreads();
     if (!a.prefetch) pdl_wait();
     int32_t L = a.lens[b];
     L = (L >= 0 && L <= a.cap) ? L : 0;
     const int32_t nw = (L + 3) / 4;  // cap is a multiple of 4: the last word stays inside the row
     const int32_t per = (nw + a.split - 1) / a.split;
     const int32_t w0 = min(nw, c * per), w1 = min(nw, w0 + per);
-    uint32_t acc = fold_run(reinterpret_cast<const uint4 *>(a.ctx + size_t(b) * size_t(a.cap)), w0, w1);
     const int32_t hw = a.d / 8;
     const int32_t hper = (hw + a.split - 1) / a.split;
     const int32_t h0 = min(hw, c * hper), h1 = min(hw, h0 + hper);
-    acc ^= fold_run(reinterpret_cast<const uint4 *>(a.hidden + size_t(b) * size_t(a.d)), h0, h1);
+    const uint4 *row = reinterpret_cast<const uint4 *>(a.ctx + size_t(b) * size_t(a.cap)) + w0;
+    const uint4 *hrow = reinterpret_cast<const uint4 *>(a.hidden + size_t(b) * size_t(a.d)) + h0;
+    // the CTA's words: context [0, nctx) then hidden [nctx, total), in chunks of kReadChunkWords
+    const int32_t nctx = w1 - w0, total = nctx + (h1 - h0);
+    const int32_t nchunks = (total + kReadChunkWords - 1) / kReadChunkWords;
+    auto issue = [&](int32_t i) {  // thread 0: chunk i's copies, completing on s_bar
+        const int32_t v0 = i * kReadChunkWords, v1 = min(total, v0 + kReadChunkWords);
+        const int32_t c0 = min(v0, nctx), c1 = min(v1, nctx);
+        const int32_t g0 = max(v0, nctx) - nctx, g1 = max(v1, nctx) - nctx;
+        mbar_arrive_expect_tx(&s_bar, uint32_t(v1 - v0) * 16u);
+        if (c1 > c0) bulk_g2s(s_chunk, row + c0, uint32_t(c1 - c0) * 16u, &s_bar);
+        if (g1 > g0) bulk_g2s(s_chunk + (c1 - c0), hrow + g0, uint32_t(g1 - g0) * 16u, &s_bar);
+    };
+    if (threadIdx.x == 0 && nchunks > 0) issue(0);
     if (a.prefetch) pdl_wait();
     pdl_trigger();
+    uint32_t acc = 0;
+    bool bad = false;
+    for (int32_t i = 0; i < nchunks; ++i) {
+        const bool arrived = mbar_wait(&s_bar, uint32_t(i & 1));
+        if (!__syncthreads_and(arrived)) {  // a copy did not complete in time: leave after waiting once more
+            bad = true;
+            if (threadIdx.x == 0) mbar_wait(&s_bar, uint32_t(i & 1));
+            break;
+        }
+        const int32_t n = min(total, (i + 1) * kReadChunkWords) - i * kReadChunkWords;
+        for (int32_t j = threadIdx.x; j < n; j += kReadThreads) {
+            const uint4 v = s_chunk[j];
+            acc ^= v.x ^ v.y ^ v.z ^ v.w;
+        }
+        __syncthreads();  // the buffer is read before the next chunk overwrites it
+        if (threadIdx.x == 0 && i + 1 < nchunks) issue(i + 1);
+    }
     for (int o = kWarp / 2; o > 0; o >>= 1) acc ^= __shfl_xor_sync(0xffffffffu, acc, o);
     if ((threadIdx.x & (kWarp - 1)) == 0) s_fold[threadIdx.x / kWarp] = acc;
     __syncthreads();
     if (threadIdx.x == 0) {
         uint32_t r = 0;
         for (int i = 0; i < kReadThreads / kWarp; ++i) r ^= s_fold[i];
-        a.out[size_t(b) * size_t(a.split) + c] = r;
+        a.out[size_t(b) * size_t(a.split) + c] = bad ? ~0u : r;
     }
 }
 
@@ -314,6 +332,18 @@ extern "C" int switchsd_harness_read(const int32_t *ctx_tokens, const int32_t *c
         return SWITCHSD_ERR_ARG;
     if (B < 1 || B > 65535 || cap < 4 || cap % 4 != 0 || d < 8 || d % 8 != 0 || split < 1 || split > 1024)
         return SWITCHSD_ERR_SHAPE;
+    static bool attr_done[64] = {false};
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess) return SWITCHSD_ERR_CUDA;
+    if (dev >= 0 && dev < 64 && !attr_done[dev]) {
+        if (cudaFuncSetAttribute(read_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 int(kReadChunkWords * 16)) != cudaSuccess)
+            return SWITCHSD_ERR_CUDA;
+        attr_done[dev] = true;
+    }
+    // shared memory: the largest chunk any CTA can have
+    const int64_t words = (int64_t(cap / 4) + split - 1) / split + (int64_t(d / 8) + split - 1) / split;
+    const size_t smem = size_t(words < kReadChunkWords ? words : kReadChunkWords) * 16;
     ReadArgs a;
     a.ctx = ctx_tokens;
     a.lens = ctx_lens;
@@ -324,7 +354,8 @@ extern "C" int switchsd_harness_read(const int32_t *ctx_tokens, const int32_t *c
     a.d = d;
     a.split = split;
     a.prefetch = prefetch != 0;
-    const cudaError_t e = launch_pdl(read_kernel, dim3(unsigned(split), unsigned(B)), dim3(kReadThreads), 0,
-                                     static_cast<cudaStream_t>(stream), 0u, a);
+    // an explicit cluster of one CTA, as for every kernel here that issues bulk copies
+    const cudaError_t e = launch_pdl(read_kernel, dim3(unsigned(split), unsigned(B)), dim3(kReadThreads), smem,
+                                     static_cast<cudaStream_t>(stream), 1u, a);
     return e == cudaSuccess ? SWITCHSD_OK : SWITCHSD_ERR_CUDA;
 }
