@@ -120,11 +120,13 @@ typedef struct switchsd_index switchsd_index;
  *                field; with the two-layer probe SWITCHSD_PREFETCH_PROBE lets the probe kernel's copies
  *                of the hidden states and W1 start early.  Other bits are SWITCHSD_ERR_ARG.
  *   hidden_rows  0 or 1: hidden is [B, d], the state the probe reads for each row.  k + 1 (the fused
- *                switchsd_verify_step and switchsd_verify_sampled_step only, linear probe, no index):
- *                hidden is the target's verification output [B, k+1, d] and the probe reads row a_b of
- *                each row b -- the state that produced the appended token t[a_b], the most recent one the
- *                target computed -- or row 0 when nothing was appended (capacity, bad lengths).  The
- *                probe's copies then wait for the verification; SWITCHSD_PREFETCH_PROBE is ignored.
+ *                switchsd_verify_step and switchsd_verify_sampled_step only, no index): hidden is the
+ *                target's verification output [B, k+1, d] and the probe reads row a_b of each row b --
+ *                the state that produced the appended token t[a_b], the most recent one the target
+ *                computed -- or row 0 when nothing was appended (capacity, bad lengths).  The probe's
+ *                copies then wait for the verification; SWITCHSD_PREFETCH_PROBE is ignored.  With the
+ *                two-layer probe a gather kernel first copies each row's a_b state (by the same
+ *                acceptance rule) into the workspace, which switchsd_workspace_bytes then sizes for it.
  *                Any other value is SWITCHSD_ERR_ARG.
  *   len_bound    0, or an upper bound on every ctx_lens[b] before the call's append (<= cap).  The rescan
  *                then splits each row's ends between its CTAs on the bound instead of on the row's
@@ -358,8 +360,9 @@ void switchsd_plan_destroy(switchsd_plan *plan);
  * Bytes of device workspace switchsd_step / switchsd_verify_step need for `params` (0 for the linear
  * probe; for the two-layer probe, S x B x H1p floats rounded up to 256 bytes, where S is the first
  * layer's split of d -- the largest power of two <= 16 with at least two 64-element chunks of d per
- * part, 16 for d >= 2048 -- and H1p is probe_hidden rounded up to 64).  Reads B, d, probe_kind and
- * probe_hidden only.
+ * part, 16 for d >= 2048 -- and H1p is probe_hidden rounded up to 64; with hidden_rows > 1, B x d bf16
+ * more, rounded up to 256 bytes, for the gathered states).  Reads B, d, probe_kind, probe_hidden and
+ * hidden_rows only.
  */
 size_t switchsd_workspace_bytes(const switchsd_params *params);
 

@@ -243,10 +243,11 @@ def switchsd_step(ctx_tokens, ctx_lens, hidden, probe_w, out_draft, out_len, out
     _check(code, "switchsd_step")
 
 
-def switchsd_workspace_bytes(B: int, probe_kind: int = PROBE_LINEAR, probe_hidden: int = 0, d: int = 0) -> int:
+def switchsd_workspace_bytes(B: int, probe_kind: int = PROBE_LINEAR, probe_hidden: int = 0, d: int = 0,
+                             hidden_rows: int = 0) -> int:
     """switchsd_workspace_bytes of include/switchsd.h for a batch of B rows of hidden size d."""
     p = switchsd_params()
-    p.B, p.d, p.probe_kind, p.probe_hidden = B, d, probe_kind, probe_hidden
+    p.B, p.d, p.probe_kind, p.probe_hidden, p.hidden_rows = B, d, probe_kind, probe_hidden, hidden_rows
     return int(load().switchsd_workspace_bytes(ctypes.byref(p)))
 
 

@@ -769,6 +769,73 @@ struct CandSpec {
     int32_t *out_choice;
 };
 
+// ------------------------------------------------------------------------------------------------
+// hidden_rows = k + 1 with the two-layer probe.  The probe's tensor-core kernel runs before the step
+// kernel, so the state it reads -- row a_b of each row's [k+1, d] block -- is gathered first, by a
+// kernel that takes the accepted length a_b by the verification's own rule (the step kernel then
+// verifies again and must agree): greedy, the first draft position whose token differs from the
+// target's; sampled, the first whose u * q (binary32) is not below p; a_b = draft_len when none.
+// Row 0 when nothing is appended: a bad length (ctx_lens outside [1, cap], or above len_bound when set;
+// draft_len outside [0, k]) or an append that does not fit in cap.
+// ------------------------------------------------------------------------------------------------
+constexpr int kGatherThreads = 256;
+
+struct GatherArgs {
+    const uint16_t *hidden;  // [B, k + 1, d]
+    uint16_t *out;           // [B, d]
+    const int32_t *lens, *pv_draft, *pv_target, *pv_len;
+    const float *pv_p, *pv_q, *pv_u;  // sampled verification, else NULL
+    int32_t cap, d, k, len_bound;
+};
+
+__global__ void __launch_bounds__(kGatherThreads) gather_rows_kernel(const GatherArgs g) {
+    __shared__ int32_t s_row;
+    const int b = blockIdx.x;
+    pdl_wait();  // the verification inputs come from the preceding kernels
+    pdl_trigger();
+    if (threadIdx.x < kWarp) {
+        const int lane = threadIdx.x;
+        const int32_t L_old = g.lens[b];
+        const bool len_ok = L_old >= 1 && L_old <= (g.len_bound > 0 ? min(g.len_bound, g.cap) : g.cap);
+        int32_t acc = -1;
+        if (len_ok) {
+            const int32_t *dr = g.pv_draft + size_t(b) * g.k;
+            const int32_t *tg = g.pv_target + size_t(b) * (g.k + 1);
+            const int32_t pv_n = g.pv_len[b];
+            if (pv_n >= 0 && pv_n <= g.k) {
+                bool rej_lo, rej_hi;
+                if (g.pv_p != nullptr) {
+                    const size_t o = size_t(b) * g.k;
+                    rej_lo = lane < pv_n && !(__fmul_rn(g.pv_u[o + lane], g.pv_q ? g.pv_q[o + lane] : 1.f) <
+                                              g.pv_p[o + lane]);
+                    rej_hi = lane + 32 < pv_n && !(__fmul_rn(g.pv_u[o + lane + 32],
+                                                             g.pv_q ? g.pv_q[o + lane + 32] : 1.f) <
+                                                   g.pv_p[o + lane + 32]);
+                } else {
+                    rej_lo = lane < pv_n && dr[lane] != tg[lane];
+                    rej_hi = lane + 32 < pv_n && dr[lane + 32] != tg[lane + 32];
+                }
+                const unsigned m_lo = __ballot_sync(kFull, rej_lo);
+                const unsigned m_hi = __ballot_sync(kFull, rej_hi);
+                acc = m_lo ? __ffs(m_lo) - 1 : (m_hi ? 32 + __ffs(m_hi) - 1 : pv_n);
+                if (L_old + acc + 1 > g.cap) acc = -1;
+            }
+        }
+        if (lane == 0) s_row = acc > 0 ? acc : 0;
+    }
+    __syncthreads();
+    const uint4 *src = reinterpret_cast<const uint4 *>(g.hidden + (size_t(b) * size_t(g.k + 1) + size_t(s_row)) *
+                                                                      size_t(g.d));
+    uint4 *dst = reinterpret_cast<uint4 *>(g.out + size_t(b) * size_t(g.d));
+    for (int i = threadIdx.x; i < (g.d >> 3); i += kGatherThreads) dst[i] = src[i];
+}
+
+// Bytes of the two-layer probe's split-K partial sums in the workspace (the gathered states follow).
+static size_t mlp_part_bytes(int B, int d, int H1) {
+    const size_t floats = size_t(mlp_split(d)) * size_t(B) * size_t(mlp_hidden_padded(H1));
+    return (floats * sizeof(float) + 255) / 256 * 256;
+}
+
 // Shared validation and launch of switchsd_step / switchsd_verify_step.
 static int step_entry(int32_t *ctx_tokens, int32_t *ctx_lens, const uint16_t *hidden, const uint16_t *probe_w,
                       const switchsd_params *p, const int32_t *pv_draft, const int32_t *pv_target,
@@ -791,10 +858,9 @@ static int step_entry(int32_t *ctx_tokens, int32_t *ctx_lens, const uint16_t *hi
         return SWITCHSD_ERR_SHAPE;
     if ((p->prefetch & ~(SWITCHSD_PREFETCH_CONTEXT | SWITCHSD_PREFETCH_PROBE)) != 0) return SWITCHSD_ERR_ARG;
     if (p->len_bound < 0 || p->len_bound > p->cap) return SWITCHSD_ERR_ARG;
-    // hidden_rows: 0 / 1, or k + 1 for the fused greedy / sampled verification with the linear probe
+    // hidden_rows: 0 / 1, or k + 1 for the fused greedy / sampled verification (rescan, one draft)
     if (p->hidden_rows != 0 && p->hidden_rows != 1) {
-        if (p->hidden_rows != p->k + 1 || pv_len == nullptr || cs != nullptr || p->index != nullptr ||
-            p->probe_kind != SWITCHSD_PROBE_LINEAR)
+        if (p->hidden_rows != p->k + 1 || pv_len == nullptr || cs != nullptr || p->index != nullptr)
             return SWITCHSD_ERR_ARG;
     }
     if (p->probe_kind == SWITCHSD_PROBE_MLP) {
@@ -871,8 +937,32 @@ static int step_entry(int32_t *ctx_tokens, int32_t *ctx_lens, const uint16_t *hi
     args.b2 = p->b2;
     if (p->probe_kind == SWITCHSD_PROBE_MLP) {
         float *part = static_cast<float *>(p->workspace);
-        if (launch_mlp_tc(hidden, probe_w, part, p->B, p->d, p->probe_hidden,
-                          (p->prefetch & SWITCHSD_PREFETCH_PROBE) != 0, stream) != cudaSuccess)
+        const uint16_t *probe_in = hidden;
+        bool probe_pf = (p->prefetch & SWITCHSD_PREFETCH_PROBE) != 0;
+        if (args.hidden_rows > 1) {  // gather row a_b of each row first; the step kernel reads no state
+            GatherArgs g;
+            g.hidden = hidden;
+            g.out = reinterpret_cast<uint16_t *>(static_cast<char *>(p->workspace) +
+                                                 mlp_part_bytes(p->B, p->d, p->probe_hidden));
+            g.lens = ctx_lens;
+            g.pv_draft = pv_draft;
+            g.pv_target = pv_target;
+            g.pv_len = pv_len;
+            g.pv_p = pv_p;
+            g.pv_q = pv_q;
+            g.pv_u = pv_u;
+            g.cap = p->cap;
+            g.d = p->d;
+            g.k = p->k;
+            g.len_bound = p->len_bound;
+            if (launch_pdl(gather_rows_kernel, dim3(unsigned(p->B)), dim3(kGatherThreads), 0, stream, 0u, g) !=
+                cudaSuccess)
+                return SWITCHSD_ERR_CUDA;
+            probe_in = g.out;
+            probe_pf = false;  // the probe kernel's input was just written by the gather
+            args.hidden_rows = 1;
+        }
+        if (launch_mlp_tc(probe_in, probe_w, part, p->B, p->d, p->probe_hidden, probe_pf, stream) != cudaSuccess)
             return SWITCHSD_ERR_CUDA;
         args.z1_part = part;
         args.b1 = p->b1;
@@ -899,8 +989,9 @@ extern "C" size_t switchsd_workspace_bytes(const switchsd_params *p) {
     if (!p || p->probe_kind != SWITCHSD_PROBE_MLP || p->B < 1) return 0;
     const int H1 = p->probe_hidden < 1 ? 1 : p->probe_hidden;
     const int d = p->d < 8 ? 8 : p->d;
-    const size_t floats = size_t(mlp_split(d)) * size_t(p->B) * size_t(mlp_hidden_padded(H1));
-    return (floats * sizeof(float) + 255) / 256 * 256;
+    size_t bytes = mlp_part_bytes(p->B, d, H1);
+    if (p->hidden_rows > 1) bytes += (size_t(p->B) * size_t(d) * sizeof(uint16_t) + 255) / 256 * 256;
+    return bytes;
 }
 
 extern "C" int switchsd_step(const int32_t *ctx_tokens, const int32_t *ctx_lens, const uint16_t *hidden,

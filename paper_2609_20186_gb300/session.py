@@ -78,6 +78,7 @@ class Session:
         # workspace of the two-layer probe (none for the linear probe)
         probe = bd.switchsd_params()
         probe.B, probe.d, probe.probe_kind, probe.probe_hidden = B, d or 0, probe_kind, probe_hidden
+        probe.hidden_rows = int(hidden_rows)  # k + 1 with the two-layer probe: room for the gathered rows
         ws_bytes = int(self.lib.switchsd_workspace_bytes(ctypes.byref(probe)))
         self.workspace = torch.empty(max(ws_bytes, 256), dtype=torch.uint8, device=dev)
 

@@ -112,6 +112,13 @@ def test_step_validation(lib):
     assert _step(lib, _params(probe_kind=1, probe_hidden=256, workspace=FAKE,
                               workspace_bytes=need - 1)) == bd.ERR_ARG
     assert _step(lib, _params(probe_kind=1, probe_hidden=256, d=8200)) == bd.ERR_SHAPE
+    # hidden_rows = k + 1 with the two-layer probe: the workspace also holds B x d gathered bf16 states
+    grown = bd.switchsd_workspace_bytes(4, 1, 256, 16, hidden_rows=9)
+    assert grown == bd.switchsd_workspace_bytes(4, 1, 256, 16) + 256
+    assert bd.switchsd_workspace_bytes(4, 0, 0, 16, hidden_rows=9) == 0
+    f = FAKE
+    q = _params(probe_kind=1, probe_hidden=256, hidden_rows=9, workspace=FAKE, workspace_bytes=grown - 1)
+    assert lib.switchsd_verify_step(f, f, f, f, f, f, f, f, ctypes.byref(q), f, f, f, f) == bd.ERR_ARG
 
 
 def test_verify_validation(lib):

@@ -1,5 +1,7 @@
 """The fused verification reading the probe's state from the target's [B, k+1, d] output (params
-.hidden_rows = k + 1): row a_b of each row, row 0 when nothing was appended.
+.hidden_rows = k + 1): row a_b of each row, row 0 when nothing was appended.  The code workload runs the
+two-layer probe (its rows gathered by a separate kernel before the tensor-core probe kernel), with a
+batch of 130 rows spanning two 128-row tiles of that kernel.
 
 The oracle side gathers the same row on the host from its own accepted lengths and runs the oracle step
 on the gathered [B, d] states; everything must match as in the other lockstep tests (a wrong row changes
@@ -51,8 +53,8 @@ def _gpu(wl, steps, sampled):
     from paper_2609_20186_gb300 import Session, bf16_tensor
     ctx, lens = wl.contexts()
     sess = Session(ctx, lens, wl.probe_weights(), k=wl.k, n_min=wl.n_min, n_max=wl.n_max, kappa=wl.kappa,
-                   logit_tau=wl.logit_tau, future=wl.future(), harness=wl.harness_params(), d=wl.d,
-                   hidden_rows=wl.k + 1)
+                   logit_tau=wl.logit_tau, probe_kind=wl.probe_kind, probe_hidden=wl.probe_hidden,
+                   future=wl.future(), harness=wl.harness_params(), d=wl.d, hidden_rows=wl.k + 1)
     trace = []
     for t in range(steps):
         ha = bf16_tensor(_hidden_all(wl, t), sess.device)
@@ -76,7 +78,8 @@ def _gpu(wl, steps, sampled):
 
 @pytest.mark.parametrize("sampled", [False, True], ids=["greedy", "sampled"])
 @pytest.mark.parametrize("name,B,L0,steps", [("uniform_8k", 8, 3000, 16), ("zipf_32k", 8, 9001, 16),
-                                             ("mixed_128k", 4, 20003, 10)])
+                                             ("mixed_128k", 4, 20003, 10), ("code_16k", 8, 5000, 12),
+                                             ("code_16k", 130, 3001, 6)])
 def test_gather_lockstep(name, B, L0, steps, sampled):
     wl = W[name].scaled(name=f"{name}_gather", B=B, L0=L0, steps=steps)
     o_trace, o_ctx = _oracle(wl, steps, sampled)
