@@ -548,8 +548,6 @@ def run_ours(args, world, rank, local):
 
     if not torch.cuda.is_available():
         raise SystemExit("bench.py needs a CUDA device (the controller has no CPU path)")
-    if args.verify == "sampled" and args.search == "index":
-        raise SystemExit("--verify sampled runs the rescan (the index keeps to greedy verification)")
     if args.candidates > 0 and (args.search == "index" or args.verify == "sampled"):
         raise SystemExit("--candidates runs the rescan with greedy verification")
     torch.cuda.set_device(local)

@@ -120,7 +120,7 @@ typedef struct switchsd_index switchsd_index;
  *                field; with the two-layer probe SWITCHSD_PREFETCH_PROBE lets the probe kernel's copies
  *                of the hidden states and W1 start early.  Other bits are SWITCHSD_ERR_ARG.
  *   hidden_rows  0 or 1: hidden is [B, d], the state the probe reads for each row.  k + 1 (the fused
- *                switchsd_verify_step and switchsd_verify_sampled_step only, no index): hidden is the
+ *                switchsd_verify_step and switchsd_verify_sampled_step only): hidden is the
  *                target's verification output [B, k+1, d] and the probe reads row a_b of each row b --
  *                the state that produced the appended token t[a_b], the most recent one the target
  *                computed -- or row 0 when nothing was appended (capacity, bad lengths).  The probe's
@@ -237,8 +237,8 @@ int switchsd_verify(const int32_t *draft, const int32_t *target_argmax, int32_t 
  *
  * The row's context receives draft[0..a) then resample[a]; ctx_lens grows by a+1; capacity, status and
  * bad lengths as switchsd_verify.  With p one-hot (T -> 0) and resample = the argmax this is
- * switchsd_verify.  vp->index must be NULL (SWITCHSD_ERR_ARG otherwise): the index keeps to the greedy
- * verification.
+ * switchsd_verify.  With vp->index the index kernel applies the same rule and inserts the appended
+ * positions, as for switchsd_verify.
  */
 int switchsd_verify_sampled(const int32_t *draft, const float *p_draft, const float *q_draft, const float *u,
                             const int32_t *resample, int32_t *out_accept, const switchsd_verify_params *vp);
@@ -268,8 +268,8 @@ int switchsd_verify_step(const int32_t *draft, const int32_t *target_argmax, con
 /*
  * switchsd_verify_step at temperature T > 0: the sampled verification and append of the previous draft,
  * exactly as switchsd_verify_sampled (same arguments: draft, p_draft, q_draft or NULL, u, resample,
- * draft_len), then switchsd_step on the extended context, in one launch.  params->index must be NULL
- * (SWITCHSD_ERR_ARG otherwise).  Statuses as switchsd_verify_step.
+ * draft_len), then switchsd_step on the extended context, in one launch (with params->index, in the
+ * index kernel).  Statuses as switchsd_verify_step.
  */
 int switchsd_verify_sampled_step(const int32_t *draft, const float *p_draft, const float *q_draft, const float *u,
                                  const int32_t *resample, const int32_t *draft_len, int32_t *out_accept,

@@ -52,6 +52,8 @@ struct IndexArgs {
     int32_t mlp_S, H1, H1p;
     float b2;
     const int32_t *pv_draft, *pv_target, *pv_len;  // verification inputs (null: no verification)
+    const float *pv_p, *pv_q, *pv_u;               // sampled verification (null p: greedy)
+    int32_t hidden_rows;                           // > 1: the probe reads row a_b of [B, hidden_rows, d]
     int32_t *out_accept;
     int32_t *out_draft, *out_len, *out_mode;
     float *out_score;
@@ -95,7 +97,18 @@ __global__ void __launch_bounds__(kIdxMaxWarps * kWarp) index_kernel(const Index
                 acc = n;
                 for (int base = 0; base < n; base += kWarp) {
                     const int i = base + lane;
-                    const unsigned m = __ballot_sync(kFull, i < n && dr[i] != tg[i]);
+                    // greedy: a draft token is rejected when it differs from the target's; sampled: when
+                    // u * q (binary32) is not below p
+                    bool rej = false;
+                    if (i < n) {
+                        if (a.pv_p != nullptr) {
+                            const size_t o = size_t(b) * a.k + i;
+                            rej = !(__fmul_rn(a.pv_u[o], a.pv_q ? a.pv_q[o] : 1.f) < a.pv_p[o]);
+                        } else {
+                            rej = dr[i] != tg[i];
+                        }
+                    }
+                    const unsigned m = __ballot_sync(kFull, rej);
                     if (m) {
                         acc = base + __ffs(m) - 1;
                         break;
@@ -191,7 +204,9 @@ __global__ void __launch_bounds__(kIdxMaxWarps * kWarp) index_kernel(const Index
             zp = fmaf(bf16_lo(uint32_t(a.w2[u])), fmaxf(z1 + bias, 0.f), zp);
         }
     } else {
-        const uint4 *h4 = reinterpret_cast<const uint4 *>(a.hidden + size_t(b) * a.d);
+        const int32_t hrow = a.hidden_rows > 1 && s_ver[0] > 0 ? s_ver[0] : 0;  // row a_b when gathering
+        const uint4 *h4 = reinterpret_cast<const uint4 *>(
+            a.hidden + (size_t(b) * size_t(a.hidden_rows > 1 ? a.hidden_rows : 1) + size_t(hrow)) * a.d);
         const uint4 *w4 = reinterpret_cast<const uint4 *>(a.probe_w);
         for (int v = tid; v < (a.d >> 3); v += blockDim.x) {
             const uint4 w = __ldg(w4 + v), h = __ldg(h4 + v);
@@ -288,9 +303,14 @@ int index_launch(switchsd_index *idx, int32_t *ctx, int32_t *lens, const uint16_
                  const int32_t *pv_draft, const int32_t *pv_target, const int32_t *pv_len, int32_t *out_accept,
                  int32_t *out_draft, int32_t *out_len, int32_t *out_mode, float *out_score, int32_t *out_match_n,
                  int32_t *out_match_end, int32_t *status, int B, int cap, int d, int k, int n_min, int n_max, int kappa,
-                 float logit_tau, bool stepping, cudaStream_t stream) {
+                 float logit_tau, bool stepping, cudaStream_t stream, const float *pv_p, const float *pv_q,
+                 const float *pv_u, int hidden_rows) {
     if (idx->B != B || idx->cap != cap || idx->n_min != n_min || idx->n_max != n_max) return SWITCHSD_ERR_SHAPE;
     IndexArgs a;
+    a.pv_p = pv_p;
+    a.pv_q = pv_q;
+    a.pv_u = pv_u;
+    a.hidden_rows = hidden_rows;
     a.ctx = ctx;
     a.lens = lens;
     a.hidden = hidden;

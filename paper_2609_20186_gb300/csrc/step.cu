@@ -858,10 +858,9 @@ static int step_entry(int32_t *ctx_tokens, int32_t *ctx_lens, const uint16_t *hi
         return SWITCHSD_ERR_SHAPE;
     if ((p->prefetch & ~(SWITCHSD_PREFETCH_CONTEXT | SWITCHSD_PREFETCH_PROBE)) != 0) return SWITCHSD_ERR_ARG;
     if (p->len_bound < 0 || p->len_bound > p->cap) return SWITCHSD_ERR_ARG;
-    // hidden_rows: 0 / 1, or k + 1 for the fused greedy / sampled verification (rescan, one draft)
+    // hidden_rows: 0 / 1, or k + 1 for the fused greedy / sampled verification of one draft
     if (p->hidden_rows != 0 && p->hidden_rows != 1) {
-        if (p->hidden_rows != p->k + 1 || pv_len == nullptr || cs != nullptr || p->index != nullptr)
-            return SWITCHSD_ERR_ARG;
+        if (p->hidden_rows != p->k + 1 || pv_len == nullptr || cs != nullptr) return SWITCHSD_ERR_ARG;
     }
     if (p->probe_kind == SWITCHSD_PROBE_MLP) {
         if (!mlp_shape_ok(p->d, p->probe_hidden)) return SWITCHSD_ERR_SHAPE;
@@ -954,7 +953,7 @@ static int step_entry(int32_t *ctx_tokens, int32_t *ctx_lens, const uint16_t *hi
             g.cap = p->cap;
             g.d = p->d;
             g.k = p->k;
-            g.len_bound = p->len_bound;
+            g.len_bound = p->index != nullptr ? 0 : p->len_bound;  // the index ignores the bound
             if (launch_pdl(gather_rows_kernel, dim3(unsigned(p->B)), dim3(kGatherThreads), 0, stream, 0u, g) !=
                 cudaSuccess)
                 return SWITCHSD_ERR_CUDA;
@@ -975,7 +974,8 @@ static int step_entry(int32_t *ctx_tokens, int32_t *ctx_lens, const uint16_t *hi
         return index_launch(p->index, ctx_tokens, ctx_lens, hidden, probe_w, args.z1_part, args.b1, args.w2, args.mlp_S,
                             args.H1, args.H1p, args.b2, pv_draft, pv_target, pv_len, out_accept, out_draft, out_len,
                             out_mode, out_score, p->out_match_n, p->out_match_end, p->status, p->B, p->cap, p->d, p->k,
-                            p->n_min, p->n_max, p->kappa, p->logit_tau, true, stream);
+                            p->n_min, p->n_max, p->kappa, p->logit_tau, true, stream, pv_p, pv_q, pv_u,
+                            args.hidden_rows);
     const cudaError_t e = cs ? launch_step<true>(args, split, stream) : launch_step<false>(args, split, stream);
     if (e != cudaSuccess) return SWITCHSD_ERR_CUDA;
     return SWITCHSD_OK;
@@ -1039,7 +1039,6 @@ extern "C" int switchsd_verify_sampled_step(const int32_t *draft, const float *p
                                             const switchsd_params *p, int32_t *out_draft, int32_t *out_len,
                                             int32_t *out_mode, float *out_score) {
     if (!draft || !p_draft || !u || !resample || !draft_len || !out_accept) return SWITCHSD_ERR_ARG;
-    if (p && p->index != nullptr) return SWITCHSD_ERR_ARG;  // the index keeps to greedy verification
     return step_entry(ctx_tokens, ctx_lens, hidden, probe_w, p, draft, resample, draft_len, out_accept, out_draft,
                       out_len, out_mode, out_score, p_draft, q_draft, u);
 }

@@ -124,9 +124,16 @@ extern "C" int switchsd_verify_sampled(const int32_t *draft, const float *p_draf
     if (!vp || !draft || !p_draft || !u || !resample || !out_accept || !vp->draft_len || !vp->ctx_tokens ||
         !vp->ctx_lens)
         return SWITCHSD_ERR_ARG;
-    if (vp->index != nullptr) return SWITCHSD_ERR_ARG;  // the index keeps to the greedy verification
     if (vp->B < 1 || vp->cap < 4 || (vp->cap & 3) != 0 || vp->k < 1 || vp->k > SWITCHSD_KMAX)
         return SWITCHSD_ERR_SHAPE;
+    if (vp->index != nullptr) {
+        // the same rule in the index kernel, which also inserts the appended positions (no step)
+        return index_launch(vp->index, vp->ctx_tokens, vp->ctx_lens, nullptr, nullptr, nullptr, nullptr, nullptr, 0,
+                            0, 0, 0.f, draft, resample, vp->draft_len, out_accept, nullptr, nullptr, nullptr, nullptr,
+                            nullptr, nullptr, vp->status, vp->B, vp->cap, 8, vp->k, index_n_min(vp->index),
+                            index_n_max(vp->index), 0, 0.f, false, static_cast<cudaStream_t>(vp->stream), p_draft,
+                            q_draft, u);
+    }
     VerifyArgs a;
     a.draft = draft;
     a.target = resample;

@@ -71,7 +71,6 @@ def gpu_trace(wl: synth.Workload, steps: int, split: int = 0, ctx=None, lens=Non
     fused=True:  switchsd_verify_step (verification of iteration t-1, then step t) and the target
                  stand-in per iteration; the last draft is verified by switchsd_verify.
     sampled=True: the sampled stand-in and switchsd_verify_sampled / switchsd_verify_sampled_step (T > 0)."""
-    assert not (sampled and use_index)
     import torch
     from paper_2609_20186_gb300 import Session, bf16_tensor
 

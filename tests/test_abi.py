@@ -145,9 +145,6 @@ def test_verify_sampled_validation(lib):
     assert lib.switchsd_verify_sampled(f, f, None, f, f, f, None) == bd.ERR_ARG
     assert lib.switchsd_verify_sampled(f, None, None, f, f, f, ctypes.byref(vp)) == bd.ERR_ARG  # no p
     assert lib.switchsd_verify_sampled(f, f, None, None, f, f, ctypes.byref(vp)) == bd.ERR_ARG  # no u
-    vp.index = FAKE                                  # the index keeps to greedy verification
-    assert lib.switchsd_verify_sampled(f, f, None, f, f, f, ctypes.byref(vp)) == bd.ERR_ARG
-    vp.index = None
     vp.k = 65
     assert lib.switchsd_verify_sampled(f, f, None, f, f, f, ctypes.byref(vp)) == bd.ERR_SHAPE
     hp = bd.switchsd_harness_params()

@@ -48,13 +48,14 @@ def _oracle(wl, steps, sampled):
     return trace, ctx
 
 
-def _gpu(wl, steps, sampled):
+def _gpu(wl, steps, sampled, use_index=False):
     import torch
     from paper_2609_20186_gb300 import Session, bf16_tensor
     ctx, lens = wl.contexts()
     sess = Session(ctx, lens, wl.probe_weights(), k=wl.k, n_min=wl.n_min, n_max=wl.n_max, kappa=wl.kappa,
                    logit_tau=wl.logit_tau, probe_kind=wl.probe_kind, probe_hidden=wl.probe_hidden,
-                   future=wl.future(), harness=wl.harness_params(), d=wl.d, hidden_rows=wl.k + 1)
+                   future=wl.future(), harness=wl.harness_params(), d=wl.d, hidden_rows=wl.k + 1,
+                   use_index=use_index)
     trace = []
     for t in range(steps):
         ha = bf16_tensor(_hidden_all(wl, t), sess.device)
@@ -88,3 +89,14 @@ def test_gather_lockstep(name, B, L0, steps, sampled):
     assert stats["checked"] > 0
     # the accepted lengths vary, so rows other than 0 were read
     assert any((t["accept"] > 0).any() for t in o_trace)
+
+
+@pytest.mark.parametrize("sampled", [False, True], ids=["greedy", "sampled"])
+@pytest.mark.parametrize("name,B,L0,steps", [("zipf_32k", 8, 9001, 12), ("code_16k", 8, 5000, 10)])
+def test_gather_index_lockstep(name, B, L0, steps, sampled):
+    """The same with the incremental index: its kernel verifies, inserts and probes row a_b."""
+    wl = W[name].scaled(name=f"{name}_gather_index", B=B, L0=L0, steps=steps)
+    o_trace, o_ctx = _oracle(wl, steps, sampled)
+    g_trace, g_ctx = _gpu(wl, steps, sampled, use_index=True)
+    flips, stats = lockstep.compare(wl, o_trace, g_trace, range(wl.B), o_ctx, g_ctx)
+    assert stats["checked"] > 0

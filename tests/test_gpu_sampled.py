@@ -37,6 +37,18 @@ def test_sampled_lockstep(name, fused):
     assert acc.max() > 0 and (acc == 0).any()
 
 
+@pytest.mark.parametrize("fused", [False, True], ids=["separate", "fused"])
+@pytest.mark.parametrize("name", ["zipf_small", "code_small", "mixed_small"])
+def test_sampled_index_lockstep(name, fused):
+    """The incremental index with the sampled rule: verification and inserts in the index kernel."""
+    wl = SMALL[name]
+    rows = range(wl.B)
+    o_trace, o_ctx, _ = lockstep.oracle_trace(wl, rows, wl.steps, sampled=True)
+    g_trace, g_ctx, _ = lockstep.gpu_trace(wl, wl.steps, sampled=True, fused=fused, use_index=True)
+    flips, stats = lockstep.compare(wl, o_trace, g_trace, rows, o_ctx, g_ctx)
+    assert stats["checked"] > 0
+
+
 def test_device_sampled_harness_matches_host():
     import torch
     from paper_2609_20186_gb300 import binding as bd
