@@ -501,8 +501,8 @@ int switchsd_verify_candidates_step(const int32_t *cand, const int32_t *target, 
  *   n           1..SWITCHSD_NMAX
  *   out_labels  device uint8 [B, cap]: 0 / 1 for j < ctx_lens[b], 0 beyond
  *   workspace   device scratch of at least switchsd_labels_workspace_bytes(B, cap) bytes, 4-byte
- *               aligned, caller-owned (a first-occurrence table per row; calls sharing it must not
- *               overlap on the GPU)
+ *               aligned, caller-owned (a first-occurrence table per row and the table slot of every
+ *               window start; calls sharing it must not overlap on the GPU)
  *   stream      cudaStream_t as void*
  */
 size_t switchsd_labels_workspace_bytes(int32_t B, int32_t cap);

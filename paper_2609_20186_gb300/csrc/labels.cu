@@ -7,8 +7,8 @@
 //   insert  thread per window start s: hash the n tokens, probe linearly; an empty slot is claimed with
 //           atomicCAS, a slot whose window holds the same tokens takes atomicMin(slot, s).  Every slot
 //           then holds the smallest start among the windows with its tokens -- the same value whatever
-//           order the inserts ran in.
-//   label   CTA per 256 positions: for the window starts s in [j0 - n + 1, j0 + 256) it finds the slot
+//           order the inserts ran in.  The slot of s is recorded in where[s].
+//   label   CTA per 256 positions: for the window starts s in [j0 - n + 1, j0 + 256) it reads the slot
 //           of s and marks s when the slot's smallest start is below s (the window repeats); position
 //           j is then the OR of the marks of the n windows that cover it.
 //
@@ -23,6 +23,7 @@ constexpr int kLabelThreads = 256;
 struct LabelArgs {
     const int32_t *ctx, *lens;
     int32_t *table;     // [B][T]
+    int32_t *where;     // [B][cap]: the slot of each window start
     uint8_t *labels;    // [B][cap]
     int32_t B, cap, n;
     uint32_t tmask;     // T - 1
@@ -57,15 +58,18 @@ __global__ void __launch_bounds__(kLabelThreads) label_insert_kernel(const Label
     if (s + a.n > L) return;
     const int32_t *x = a.ctx + size_t(b) * size_t(a.cap);
     int32_t *tab = a.table + size_t(b) * (size_t(a.tmask) + 1);
+    int32_t *where = a.where + size_t(b) * size_t(a.cap);
     uint32_t h = window_hash(x + s, a.n, a.tmask);
     for (uint32_t probe = 0; probe <= a.tmask; ++probe, h = (h + 1) & a.tmask) {
-        int32_t v = tab[h];
+        // Claim the slot if empty; otherwise the CAS returns its start (one round trip either way).
+        const int32_t v = atomicCAS(&tab[h], -1, s);
         if (v < 0) {
-            v = atomicCAS(&tab[h], -1, s);
-            if (v < 0) return;  // claimed the empty slot
+            where[s] = int32_t(h);
+            return;
         }
         if (same_window(x + v, x + s, a.n)) {
             atomicMin(&tab[h], s);
+            where[s] = int32_t(h);
             return;
         }
     }
@@ -78,22 +82,15 @@ __global__ void __launch_bounds__(kLabelThreads) label_mark_kernel(const LabelAr
     pdl_wait();
     pdl_trigger();
     const int32_t L = row_length(a, b);
-    const int32_t *x = a.ctx + size_t(b) * size_t(a.cap);
     const int32_t *tab = a.table + size_t(b) * (size_t(a.tmask) + 1);
+    const int32_t *where = a.where + size_t(b) * size_t(a.cap);
     const int32_t first = j0 - a.n + 1;
     for (int t = threadIdx.x; t < kLabelThreads + a.n - 1; t += kLabelThreads) {
         const int32_t s = first + t;
         uint8_t rep = 0;
         if (s >= 0 && s + a.n <= L) {
-            uint32_t h = window_hash(x + s, a.n, a.tmask);
-            for (uint32_t probe = 0; probe <= a.tmask; ++probe, h = (h + 1) & a.tmask) {
-                const int32_t v = tab[h];
-                if (v < 0) break;  // not reached: every window was inserted
-                if (same_window(x + v, x + s, a.n)) {
-                    rep = v < s;
-                    break;
-                }
-            }
+            const int32_t h = where[s];  // written by the insert of s
+            rep = h >= 0 && uint32_t(h) <= a.tmask && tab[h] < s;
         }
         s_rep[t] = rep;
     }
@@ -118,7 +115,7 @@ using namespace switchsd;
 
 extern "C" size_t switchsd_labels_workspace_bytes(int32_t B, int32_t cap) {
     if (B < 1 || cap < 1) return 0;
-    return size_t(B) * size_t(table_slots(cap)) * sizeof(int32_t);
+    return size_t(B) * (size_t(table_slots(cap)) + size_t(cap)) * sizeof(int32_t);
 }
 
 extern "C" int switchsd_copy_labels(const int32_t *ctx_tokens, const int32_t *ctx_lens, int32_t B, int32_t cap,
@@ -135,6 +132,7 @@ extern "C" int switchsd_copy_labels(const int32_t *ctx_tokens, const int32_t *ct
     a.ctx = ctx_tokens;
     a.lens = ctx_lens;
     a.table = static_cast<int32_t *>(workspace);
+    a.where = a.table + size_t(B) * T;
     a.labels = out_labels;
     a.B = B;
     a.cap = cap;
