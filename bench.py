@@ -950,10 +950,7 @@ def run_labels(args, world, rank, local):
     secs = reduce_max(ms / 1e3, world)
     positions = float(lens1.sum()) * K
     value = replica_throughput(positions, secs, world)
-    T = 16                                                             # table slots per row (the library's rule)
-    while T < 2 * cap:
-        T *= 2
-    bytes_per_call = float(lens1.sum()) * 4 + B * cap + B * T * 4    # context, labels, table clear
+    bytes_per_call = float(lens1.sum()) * 4 + B * cap                # context read, labels written
     achieved = bytes_per_call / (secs / K) / 1e9
     peaks = measured_peaks()
     if rank == 0:
