@@ -93,20 +93,19 @@ def test_full_size_sampled_positions():
 
 
 @pytest.mark.parametrize("n", [1, 5])
-def test_long_runs_take_the_fallback(n):
-    """Rows whose equal windows overflow one partition's list (runs, short periods, a 2-token alphabet)
-    take the global-table fallback; rows beside them in the batch the main path.  Every position is
-    compared with the oracle either way."""
+def test_long_runs_and_short_periods(n):
+    """Rows where thousands of windows are equal (one run, period 2, a 2-token alphabet: every insert
+    lands on a few table slots) beside ordinary rows in one batch; every position against the oracle."""
     rng = np.random.default_rng(77 + n)
     B, cap = 6, 12000
     ctx = np.zeros((B, cap), np.int32)
     ctx[0] = 7                                          # one run: every window equal
     ctx[1] = np.tile([3, 9], cap // 2)                  # period 2
     ctx[2] = rng.integers(0, 2, cap)                    # two-letter alphabet: few distinct windows
-    ctx[3] = rng.integers(0, 100000, cap)               # main path
+    ctx[3] = rng.integers(0, 100000, cap)               # distinct windows
     ctx[4, :6000] = 5                                   # half a run, then distinct tokens
     ctx[4, 6000:] = rng.integers(0, 100000, cap - 6000)
-    ctx[5] = np.minimum(rng.zipf(1.3, cap), 50000)      # main path
+    ctx[5] = np.minimum(rng.zipf(1.3, cap), 50000)      # Zipf ids
     lens = np.array([cap, cap - 1, cap, cap, cap - 3, 9001], np.int32)
     got = _labels(ctx, lens, n)
     for b in range(B):
