@@ -465,6 +465,7 @@ class ReplicaLoop:
             v.ctx_tokens = self.ctx.data_ptr() + r * B * cap * 4
             v.ctx_lens = self.lens.data_ptr() + r * B * 4
             v.status, v.stream = None, sp
+            v.index = self.indexes[r].handle if self.indexes else None
             self.cvps.append(v)
         f32 = dict(dtype=torch.float32, device=dev)
         self.vp = torch.zeros(N, k, **f32)
@@ -548,8 +549,8 @@ def run_ours(args, world, rank, local):
 
     if not torch.cuda.is_available():
         raise SystemExit("bench.py needs a CUDA device (the controller has no CPU path)")
-    if args.candidates > 0 and (args.search == "index" or args.verify == "sampled"):
-        raise SystemExit("--candidates runs the rescan with greedy verification")
+    if args.candidates > 0 and args.verify == "sampled":
+        raise SystemExit("--candidates runs with greedy verification")
     torch.cuda.set_device(local)
     dev = torch.device("cuda", local)
     binding.load()

@@ -42,7 +42,7 @@
 extern "C" {
 #endif
 
-#define SWITCHSD_ABI_VERSION 5
+#define SWITCHSD_ABI_VERSION 6
 
 #define SWITCHSD_NMAX 32 /* largest supported n_max */
 #define SWITCHSD_KMAX 64 /* largest supported draft length k */
@@ -429,7 +429,9 @@ const char *switchsd_strerror(int code);
  * candidate w continues with x[e_w+1 .. e_w+len_w], len_w = min(D, L-1-e_w).  The mode: no repetition
  * when no n_min-gram of the suffix recurs, copy when a candidate exists and z >= logit_tau, repetition
  * without copy otherwise.  Everything else as switchsd_step (params->k is only the bound of the staged
- * look-ahead and must be >= 1; params->index must be NULL).
+ * look-ahead and must be >= 1).  With params->index the index kernel lists the ends from its chain of
+ * the kappa-gram, so kappa (or n_min when <= 0) must be at least the index's n_min
+ * (SWITCHSD_ERR_SHAPE otherwise); a kappa above n_max gives no candidate, as for the rescan.
  *
  *   W, D          1..SWITCHSD_WMAX, 1..SWITCHSD_KMAX
  *   out_cand      device int32 [B, W, D]: candidate w's tokens in [b][w][0, len_w)
@@ -448,7 +450,8 @@ int switchsd_step_candidates(const int32_t *ctx_tokens, const int32_t *ctx_lens,
  *   B, cap        as switchsd_verify_params;  W, D  the candidate slots (as switchsd_step_candidates)
  *   cand_len      device int32 [B, W], ncand device int32 [B] (a neural row passes its draft as the one
  *                 candidate; ncand = 0 counts as one empty candidate)
- *   ctx_tokens, ctx_lens, status, stream   as switchsd_verify_params
+ *   ctx_tokens, ctx_lens, status, stream, index   as switchsd_verify_params (with an index the index
+ *                 kernel verifies, appends and inserts the appended positions)
  */
 typedef struct {
     int32_t B, cap, W, D;
@@ -458,6 +461,7 @@ typedef struct {
     int32_t *ctx_lens;
     int32_t *status;
     void *stream;
+    switchsd_index *index;  /* NULL, or the index kept current by the append (as switchsd_verify_params) */
 } switchsd_candidates_verify_params;
 
 /*

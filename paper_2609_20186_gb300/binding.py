@@ -19,7 +19,7 @@ PROBE_LINEAR, PROBE_MLP = 0, 1
 OK, ERR_ARG, ERR_SHAPE, ERR_CUDA = 0, -1, -2, -3
 ROW_OK, ROW_CAPACITY, ROW_BAD_LEN, ROW_TIMEOUT = 0, 1, 2, 3
 NMAX, KMAX = 32, 64
-ABI_VERSION = 5  # SWITCHSD_ABI_VERSION this binding marshals for
+ABI_VERSION = 6  # SWITCHSD_ABI_VERSION this binding marshals for
 PREFETCH_CONTEXT, PREFETCH_PROBE = 1, 2  # switchsd_params.prefetch bits
 
 _c_i32p = ctypes.c_void_p
@@ -58,6 +58,7 @@ class switchsd_candidates_verify_params(ctypes.Structure):
         ("B", ctypes.c_int32), ("cap", ctypes.c_int32), ("W", ctypes.c_int32), ("D", ctypes.c_int32),
         ("cand_len", ctypes.c_void_p), ("ncand", ctypes.c_void_p), ("ctx_tokens", ctypes.c_void_p),
         ("ctx_lens", ctypes.c_void_p), ("status", ctypes.c_void_p), ("stream", ctypes.c_void_p),
+        ("index", ctypes.c_void_p),
     ]
 
 

@@ -14,6 +14,10 @@
 //   insertion of the appended end positions (all lanes at once; positions of one run that fall into
 //   the same bucket are linked through __match_any_sync, so one read of the old heads suffices);
 //   the lookup, the probe and the switch / copy draft (as switchsd_step), when stepping.
+// Candidate mode (W > 0, as switchsd_step_candidates / switchsd_verify_candidates): the previous W
+// candidates are verified and the longest accepted one appended; the warp of n = kappa walks its
+// chain on past the first match and lists the W most recent ends whose kappa-gram equals the
+// suffix's -- exactly the ends whose common suffix with the current one reaches kappa.
 #include <new>
 
 #include "common.cuh"
@@ -61,6 +65,11 @@ struct IndexArgs {
     int32_t *heads, *prev;
     int32_t B, cap, d, k, n_min, n_max, kappa, log2_buckets, stepping;
     float logit_tau;
+    // candidate mode (W > 0): W candidates of up to D tokens; pv_draft / pv_target / pv_len then hold
+    // the previous candidates [B][W][D], their targets [B][W][D+1] and counts [B]
+    int32_t W, D;
+    const int32_t *pv_cand_len;  // [B][W]
+    int32_t *out_choice, *out_cand, *out_cand_len, *out_ncand;
 };
 
 __global__ void __launch_bounds__(kIdxMaxWarps * kWarp) index_kernel(const IndexArgs a) {
@@ -69,6 +78,8 @@ __global__ void __launch_bounds__(kIdxMaxWarps * kWarp) index_kernel(const Index
     __shared__ int32_t s_found[kIdxMaxWarps];
     __shared__ float s_wz[kIdxMaxWarps];
     __shared__ int32_t s_out[3];
+    __shared__ int32_t s_cend[SWITCHSD_WMAX];  // candidate mode: the listed ends, most recent first
+    __shared__ int32_t s_ncf, s_choice;
 
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     const int nwarps = blockDim.x >> 5;
@@ -77,6 +88,7 @@ __global__ void __launch_bounds__(kIdxMaxWarps * kWarp) index_kernel(const Index
     pdl_wait();
     pdl_trigger();
 
+    if (tid == 0) s_ncf = 0;
     int32_t *row = a.ctx + size_t(b) * a.cap;
     const int32_t L_old = a.lens[b];
     const bool len_ok = L_old >= 1 && L_old <= a.cap;
@@ -87,7 +99,48 @@ __global__ void __launch_bounds__(kIdxMaxWarps * kWarp) index_kernel(const Index
     }
     if (warp == 0) {
         int32_t acc = -1, L = L_old, vst = len_ok ? SWITCHSD_ROW_OK : SWITCHSD_ROW_BAD_LEN;
-        if (verifying && len_ok) {
+        int32_t choice = 0;
+        if (verifying && len_ok && a.W > 0) {
+            // The previous W candidates: lane i tests positions i and i + 32 of each; the longest
+            // accepted one is kept (the lowest index on a tie).  ncand = 0 is one empty candidate.
+            const int32_t nc = a.pv_len[b];
+            bool badlen = nc < 0 || nc > a.W;
+            const int ncx = badlen ? 0 : (nc > 0 ? nc : 1);
+            int32_t best = -1;
+            for (int w = 0; w < ncx; ++w) {
+                const size_t o = size_t(b) * a.W + w;
+                const int32_t *c = a.pv_draft + o * a.D;
+                const int32_t *t = a.pv_target + o * (a.D + 1);
+                const int32_t c_lo = lane < a.D ? c[lane] : 0, c_hi = lane + 32 < a.D ? c[lane + 32] : 0;
+                const int32_t t_lo = lane < a.D ? t[lane] : 0, t_hi = lane + 32 < a.D ? t[lane + 32] : 0;
+                const int32_t len = nc > 0 ? a.pv_cand_len[o] : 0;
+                badlen |= len < 0 || len > a.D;
+                const unsigned m_lo = __ballot_sync(kFull, lane < len && c_lo != t_lo);
+                const unsigned m_hi = __ballot_sync(kFull, lane + 32 < len && c_hi != t_hi);
+                const int32_t acc_w = m_lo ? __ffs(m_lo) - 1 : (m_hi ? 32 + __ffs(m_hi) - 1 : len);
+                if (acc_w > best) {
+                    best = acc_w;
+                    choice = w;
+                }
+            }
+            if (badlen) {
+                vst = SWITCHSD_ROW_BAD_LEN;
+                choice = 0;
+            } else if (L_old + best + 1 > a.cap) {
+                vst = SWITCHSD_ROW_CAPACITY;
+            } else {
+                const size_t o = size_t(b) * a.W + choice;
+                const int32_t *c = a.pv_draft + o * a.D;
+                const int32_t tb = a.pv_target[o * (a.D + 1) + best];
+                for (int i = lane; i <= best; i += kWarp) {
+                    const int32_t t = i < best ? c[i] : tb;
+                    s_tail[SWITCHSD_NMAX + i] = t;
+                    row[L_old + i] = t;
+                }
+                acc = best;
+                L = L_old + best + 1;
+            }
+        } else if (verifying && len_ok) {
             const int32_t n = a.pv_len[b];
             if (n < 0 || n > a.k) {
                 vst = SWITCHSD_ROW_BAD_LEN;
@@ -137,6 +190,7 @@ __global__ void __launch_bounds__(kIdxMaxWarps * kWarp) index_kernel(const Index
             } else if (verifying) {
                 a.out_accept[b] = -1;
             }
+            if (verifying && a.W > 0 && a.out_choice) a.out_choice[b] = choice;
             if (!a.stepping && a.status) a.status[b] = vst;
         }
     }
@@ -172,8 +226,11 @@ __global__ void __launch_bounds__(kIdxMaxWarps * kWarp) index_kernel(const Index
     }
     if (!a.stepping) return;
 
-    // Lookup: the most recent earlier occurrence of the suffix n-gram, if any.
-    int32_t found = -1;
+    // Lookup: the most recent earlier occurrence of the suffix n-gram, if any.  Candidate mode: the
+    // warp of n = kappa lists the W most recent.
+    const int32_t kappa_c = a.kappa > 0 ? a.kappa : a.n_min;
+    const bool collect = a.W > 0 && has_n && n == kappa_c;
+    int32_t found = -1, nfound = 0;
     if (has_n && len_ok && L >= n + 1) {
         const uint32_t bucket = gram_hash(n, [&](int i) { return tail_tok(L - 1 - i); }, a.log2_buckets);
         const int32_t mine = lane < n ? tail_tok(L - 1 - lane) : 0;
@@ -182,16 +239,19 @@ __global__ void __launch_bounds__(kIdxMaxWarps * kWarp) index_kernel(const Index
         // unbuilt index from reading outside its tables.
         for (int32_t hops = 0; e >= 0 && e < a.cap && hops < a.cap; ++hops) {
             if (e <= L - 2 && e >= n - 1) {
-                const bool eq = lane >= n || row[e - lane] == mine;
+                const bool eq = lane >= n || (e - lane >= L_old ? tail_tok(e - lane) : row[e - lane]) == mine;
                 if (__all_sync(kFull, eq)) {
-                    found = e;
-                    break;
+                    if (found < 0) found = e;
+                    if (!collect) break;
+                    if (lane == 0) s_cend[nfound] = e;
+                    if (++nfound >= a.W) break;
                 }
             }
             e = prev[e];
         }
     }
     if (lane == 0 && warp < kIdxMaxWarps) s_found[warp] = found;
+    if (collect && lane == 0) s_ncf = nfound;
 
     // Probe partial over the whole hidden vector (linear probe), or over every unit of the two-layer
     // probe: the S split-K partial sums in order, then b1, ReLU and w2.
@@ -236,20 +296,35 @@ __global__ void __launch_bounds__(kIdxMaxWarps * kWarp) index_kernel(const Index
                 break;
             }
         const bool hit = len_ok && nstar > 0;
-        const int32_t kappa = a.kappa > 0 ? a.kappa : a.n_min;
+        const bool gate = a.W > 0 ? s_ncf > 0 : nstar >= kappa_c;
         int32_t mode = SWITCHSD_MODE_NO_REP;
-        if (hit) mode = (nstar >= kappa && z >= a.logit_tau) ? SWITCHSD_MODE_COPY : SWITCHSD_MODE_REP_NO_COPY;
-        const int32_t len = mode == SWITCHSD_MODE_COPY ? min(a.k, L - 1 - estar) : 0;
+        if (hit) mode = (gate && z >= a.logit_tau) ? SWITCHSD_MODE_COPY : SWITCHSD_MODE_REP_NO_COPY;
+        const int32_t len = (a.W == 0 && mode == SWITCHSD_MODE_COPY) ? min(a.k, L - 1 - estar) : 0;
         s_out[0] = estar;
         s_out[1] = len;
+        s_out[2] = mode == SWITCHSD_MODE_COPY ? s_ncf : 0;  // candidate mode: candidates written
         a.out_mode[b] = mode;
-        a.out_len[b] = len;
+        if (a.W == 0) a.out_len[b] = len;
+        else a.out_ncand[b] = s_out[2];
         a.out_score[b] = z;
         if (a.out_match_n) a.out_match_n[b] = nstar;
         if (a.out_match_end) a.out_match_end[b] = estar;
         if (a.status) a.status[b] = s_ver[2];
     }
     __syncthreads();
+    if (a.W > 0) {
+        // The candidates' continuations x[e_w+1 .. e_w+len_w], len_w = min(D, L-1-e_w).
+        const int32_t nc = s_out[2];
+        for (int t = tid; t < nc * a.D; t += blockDim.x) {
+            const int w = t / a.D, i = t - w * a.D;
+            const int32_t ew = s_cend[w];
+            const int32_t lw = min(a.D, L - 1 - ew);
+            const int32_t p = ew + 1 + i;
+            if (i == 0) a.out_cand_len[size_t(b) * a.W + w] = lw;
+            if (i < lw) a.out_cand[(size_t(b) * a.W + w) * a.D + i] = p >= L_old ? tail_tok(p) : row[p];
+        }
+        return;
+    }
     const int32_t e = s_out[0], len = s_out[1];
     // The copy draft x[e+1 .. e+len]: positions below L_old are in global memory, the rest in s_tail.
     for (int i = tid; i < len; i += blockDim.x) {
@@ -304,9 +379,19 @@ int index_launch(switchsd_index *idx, int32_t *ctx, int32_t *lens, const uint16_
                  int32_t *out_draft, int32_t *out_len, int32_t *out_mode, float *out_score, int32_t *out_match_n,
                  int32_t *out_match_end, int32_t *status, int B, int cap, int d, int k, int n_min, int n_max, int kappa,
                  float logit_tau, bool stepping, cudaStream_t stream, const float *pv_p, const float *pv_q,
-                 const float *pv_u, int hidden_rows) {
+                 const float *pv_u, int hidden_rows, const IndexCandidates *cand) {
     if (idx->B != B || idx->cap != cap || idx->n_min != n_min || idx->n_max != n_max) return SWITCHSD_ERR_SHAPE;
+    // Candidate mode lists the ends of the kappa-gram chain: kappa must be one of the index's n, or
+    // above n_max (no end can then reach it: no candidate, as for the rescan).
+    if (cand != nullptr && (kappa > 0 ? kappa : n_min) < n_min) return SWITCHSD_ERR_SHAPE;
     IndexArgs a;
+    a.W = cand ? cand->W : 0;
+    a.D = cand ? cand->D : 0;
+    a.pv_cand_len = cand ? cand->pv_cand_len : nullptr;
+    a.out_choice = cand ? cand->out_choice : nullptr;
+    a.out_cand = cand ? cand->out_cand : nullptr;
+    a.out_cand_len = cand ? cand->out_cand_len : nullptr;
+    a.out_ncand = cand ? cand->out_ncand : nullptr;
     a.pv_p = pv_p;
     a.pv_q = pv_q;
     a.pv_u = pv_u;

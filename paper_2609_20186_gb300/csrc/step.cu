@@ -845,7 +845,7 @@ static int step_entry(int32_t *ctx_tokens, int32_t *ctx_lens, const uint16_t *hi
     if (!p || !ctx_tokens || !ctx_lens || !hidden || !probe_w || !out_mode || !out_score) return SWITCHSD_ERR_ARG;
     if (cs == nullptr && (!out_draft || !out_len)) return SWITCHSD_ERR_ARG;
     if (cs != nullptr) {
-        if (!cs->cand || !cs->cand_len || !cs->ncand || p->index != nullptr) return SWITCHSD_ERR_ARG;
+        if (!cs->cand || !cs->cand_len || !cs->ncand) return SWITCHSD_ERR_ARG;
         if (cs->W < 1 || cs->W > kMaxCand || cs->D < 1 || cs->D > SWITCHSD_KMAX) return SWITCHSD_ERR_SHAPE;
     }
     if (!aligned16(ctx_tokens) || !aligned16(hidden) || !aligned16(probe_w)) return SWITCHSD_ERR_ARG;
@@ -970,12 +970,23 @@ static int step_entry(int32_t *ctx_tokens, int32_t *ctx_lens, const uint16_t *hi
         args.H1 = p->probe_hidden;
         args.H1p = mlp_hidden_padded(p->probe_hidden);
     }
-    if (p->index != nullptr)
+    if (p->index != nullptr) {
+        IndexCandidates ic;
+        if (cs != nullptr) {
+            ic.W = cs->W;
+            ic.D = cs->D;
+            ic.pv_cand_len = cs->pv_cand_len;
+            ic.out_choice = cs->out_choice;
+            ic.out_cand = cs->cand;
+            ic.out_cand_len = cs->cand_len;
+            ic.out_ncand = cs->ncand;
+        }
         return index_launch(p->index, ctx_tokens, ctx_lens, hidden, probe_w, args.z1_part, args.b1, args.w2, args.mlp_S,
                             args.H1, args.H1p, args.b2, pv_draft, pv_target, pv_len, out_accept, out_draft, out_len,
                             out_mode, out_score, p->out_match_n, p->out_match_end, p->status, p->B, p->cap, p->d, p->k,
                             p->n_min, p->n_max, p->kappa, p->logit_tau, true, stream, pv_p, pv_q, pv_u,
-                            args.hidden_rows);
+                            args.hidden_rows, cs != nullptr ? &ic : nullptr);
+    }
     const cudaError_t e = cs ? launch_step<true>(args, split, stream) : launch_step<false>(args, split, stream);
     if (e != cudaSuccess) return SWITCHSD_ERR_CUDA;
     return SWITCHSD_OK;

@@ -240,6 +240,20 @@ extern "C" int switchsd_verify_candidates(const int32_t *cand, const int32_t *ta
     if (vp->B < 1 || vp->cap < 4 || (vp->cap & 3) != 0 || vp->W < 1 || vp->W > SWITCHSD_WMAX || vp->D < 1 ||
         vp->D > SWITCHSD_KMAX)
         return SWITCHSD_ERR_SHAPE;
+    if (vp->index != nullptr) {
+        // the same rule in the index kernel, which also inserts the appended positions (no step)
+        IndexCandidates ic;
+        ic.W = vp->W;
+        ic.D = vp->D;
+        ic.pv_cand_len = vp->cand_len;
+        ic.out_choice = out_choice;
+        ic.out_cand = ic.out_cand_len = ic.out_ncand = nullptr;
+        return index_launch(vp->index, vp->ctx_tokens, vp->ctx_lens, nullptr, nullptr, nullptr, nullptr, nullptr, 0,
+                            0, 0, 0.f, cand, target, vp->ncand, out_accept, nullptr, nullptr, nullptr, nullptr,
+                            nullptr, nullptr, vp->status, vp->B, vp->cap, 8, vp->D, index_n_min(vp->index),
+                            index_n_max(vp->index), 0, 0.f, false, static_cast<cudaStream_t>(vp->stream), nullptr,
+                            nullptr, nullptr, 1, &ic);
+    }
     CandVerifyArgs a;
     a.cand = cand;
     a.cand_len = vp->cand_len;

@@ -58,7 +58,7 @@ def test_binding_declares_every_function():
 
 def test_abi_version_and_strerror(lib):
     from paper_2609_20186_gb300 import binding as bd
-    assert bd.abi_version() == 5
+    assert bd.abi_version() == 6
     for code in (0, -1, -2, -3, 1, 2, 3):
         assert bd.strerror(code) != "unknown code"
     assert bd.strerror(12345) == "unknown code"

@@ -55,9 +55,10 @@ def oracle_loop(wl, rows, steps, Wc, D):
     return trace, ctx
 
 
-def gpu_loop(wl, steps, Wc, D, split=0, fused=False):
+def gpu_loop(wl, steps, Wc, D, split=0, fused=False, use_index=False):
     """fused: switchsd_verify_candidates_step verifies iteration t-1's candidates and searches step t's in
-    one launch; the last iteration's candidates are verified by switchsd_verify_candidates."""
+    one launch; the last iteration's candidates are verified by switchsd_verify_candidates.  use_index:
+    the incremental n-gram index (built from the initial contexts) searches, verifies and inserts."""
     import torch
     from paper_2609_20186_gb300 import binding as bd, bf16_tensor
     lib = bd.load()
@@ -85,6 +86,11 @@ def gpu_loop(wl, steps, Wc, D, split=0, fused=False):
     p.workspace, p.workspace_bytes = ws.data_ptr(), ws.numel()
     p.out_match_n, p.out_match_end, p.status = mn.data_ptr(), me.data_ptr(), st.data_ptr()
     p.stream = torch.cuda.current_stream().cuda_stream
+    idx = None
+    if use_index:
+        idx = bd.NgramIndex(B, cap, wl.n_min, wl.n_max)
+        idx.build(c, ln)
+        p.index = idx.handle
     h = wl.harness_params()
     hp = bd.switchsd_harness_params()
     hp.B, hp.k, hp.V, hp.L0, hp.n_future = B, wl.k, h["V"], h["L0"], fut.shape[1]
@@ -94,6 +100,7 @@ def gpu_loop(wl, steps, Wc, D, split=0, fused=False):
     vp.B, vp.cap, vp.W, vp.D = B, cap, Wc, D
     vp.cand_len, vp.ncand, vp.ctx_tokens, vp.ctx_lens = vl.data_ptr(), vn.data_ptr(), c.data_ptr(), ln.data_ptr()
     vp.status, vp.stream = vst.data_ptr(), p.stream
+    vp.index = idx.handle if idx is not None else None
     trace = []
     for t in range(steps):
         hid = bf16_tensor(wl.hidden(t), dev)
@@ -123,6 +130,8 @@ def gpu_loop(wl, steps, Wc, D, split=0, fused=False):
                        vstatus=vst.cpu().numpy())
         trace.append(out)
     torch.cuda.synchronize()
+    if idx is not None:
+        idx.close()
     return trace, c.cpu().numpy()
 
 
@@ -193,3 +202,42 @@ def test_candidates_full_size_sampled_rows():
     o_trace, o_ctx = oracle_loop(wl, rows, wl.steps, 10, 20)
     checked, copies = compare(wl, o_trace, g_trace, rows, o_ctx, g_ctx)
     assert checked > 0
+
+
+@pytest.mark.parametrize("fused", [False, True], ids=["separate", "fused"])
+@pytest.mark.parametrize("Wc,D", [(10, 20), (16, 64), (1, 4)])
+@pytest.mark.parametrize("name", list(SMALL))
+def test_candidates_index_lockstep(name, Wc, D, fused):
+    """The index's candidate mode: the kappa-gram chain lists the ends, the index kernel verifies the
+    candidates and inserts the appended positions; everything as the rescan's lockstep."""
+    wl = SMALL[name]
+    rows = range(wl.B)
+    o_trace, o_ctx = oracle_loop(wl, rows, wl.steps, Wc, D)
+    g_trace, g_ctx = gpu_loop(wl, wl.steps, Wc, D, fused=fused, use_index=True)
+    checked, copies = compare(wl, o_trace, g_trace, rows, o_ctx, g_ctx)
+    assert checked > 0
+
+
+def test_candidates_index_kappa_below_n_min_is_rejected():
+    import ctypes
+    import torch
+    from paper_2609_20186_gb300 import binding as bd
+    lib = bd.load()
+    wl = SMALL["mixed_small"]  # n_min = 2
+    B, cap = 2, 64
+    idx = bd.NgramIndex(B, cap, 3, 8)
+    z = torch.zeros(B, cap, dtype=torch.int32, device="cuda")
+    ln = torch.full((B,), 10, dtype=torch.int32, device="cuda")
+    idx.build(z, ln)
+    p = bd.switchsd_params()
+    p.B, p.cap, p.d, p.k, p.n_min, p.n_max, p.kappa = B, cap, 8, 4, 3, 8, 2
+    p.index = idx.handle
+    p.stream = torch.cuda.current_stream().cuda_stream
+    h = torch.zeros(B, 8, dtype=torch.bfloat16, device="cuda")
+    o = torch.zeros(B, 4, 4, dtype=torch.int32, device="cuda")
+    v = torch.zeros(B, 4, dtype=torch.int32, device="cuda")
+    f = torch.zeros(B, dtype=torch.float32, device="cuda")
+    assert lib.switchsd_step_candidates(z.data_ptr(), ln.data_ptr(), h.data_ptr(), h.data_ptr(), ctypes.byref(p),
+                                        4, 4, o.data_ptr(), v.data_ptr(), v.data_ptr(), v.data_ptr(),
+                                        f.data_ptr()) == bd.ERR_SHAPE
+    idx.close()
