@@ -183,7 +183,7 @@ def measured_peaks() -> dict:
 def kernel_source_hash() -> str:
     h = hashlib.sha256()
     csrc = os.path.join(ROOT, "paper_2609_20186_gb300", "csrc")
-    for f in ("common.cuh", "step.cu"):
+    for f in ("common.cuh", "step.cuh", "step.cu"):
         with open(os.path.join(csrc, f), "rb") as fh:
             h.update(fh.read())
     return h.hexdigest()[:16]

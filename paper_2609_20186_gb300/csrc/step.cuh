@@ -1,0 +1,75 @@
+// step.cuh -- the step kernel's constants, arguments and launcher (step.cu), shared with the entry
+// points (step_api.cu).
+#pragma once
+
+#include "common.cuh"
+
+namespace switchsd {
+
+constexpr int kStepThreads = 256;
+constexpr int kStepWarps = kStepThreads / kWarp;
+constexpr int kTileMax = 8192;        // largest staged tile (candidate ends)
+constexpr int kHalo = 32;             // look-back staged before a tile: >= SWITCHSD_NMAX, multiple of 4
+constexpr int kFwd = SWITCHSD_KMAX;   // look-ahead staged after a tile: the longest copy draft
+constexpr int kMaxStages = 6;          // staged tiles in flight per CTA (bounded by shared memory)
+constexpr size_t kStageSmemBudget = 200 * 1024;
+constexpr int kMaxSplit = 16;
+constexpr unsigned long long kTimeoutBit = 1ull << 62;
+constexpr int kMaxCand = SWITCHSD_WMAX; // candidate mode: largest W
+constexpr int kProbeStage = 256;      // probe words (8 bf16) of w and of h staged per CTA; the rest is read directly
+
+static_assert(kHalo >= SWITCHSD_NMAX && kHalo % 4 == 0, "halo must cover the longest n-gram");
+static_assert(kFwd % 4 == 0 && kTileMax % 4 == 0, "stages must stay 16-byte aligned");
+
+struct StepArgs {
+    int32_t *ctx;            // read through TMA; written (append) by the leader when verifying
+    int32_t *lens;           // read; written when verifying
+    const uint16_t *hidden;
+    const uint16_t *probe_w;
+    const float *z1_part;    // two-layer probe: split-K partial sums of W1 h [mlp_S][B][H1p] (workspace), else null
+    const float *b1;         // two-layer probe: first-layer biases [H1] (null = zero) and output weights [H1]
+    const uint16_t *w2;
+    int32_t mlp_S, H1, H1p;
+    float b2;
+    const int32_t *pv_draft; // previous draft [B, k] / target [B, k+1] / draft length [B]; null = no verify
+    const int32_t *pv_target;
+    const int32_t *pv_len;
+    const float *pv_p, *pv_q, *pv_u;  // sampled verification (T > 0): null = greedy; pv_target then holds
+                                      // the residual / bonus draws and pv_q may be null (copy drafts)
+    int32_t *out_accept;
+    int32_t B, cap, d, k, n_min, n_max, kappa, tile, stages;
+    int32_t prefetch;        // SWITCHSD_PREFETCH_* bits: reads that may precede the grid-dependency wait
+    int32_t hidden_rows;     // > 1: hidden is [B, hidden_rows, d] and the probe reads row a_b (verifying)
+    int32_t len_bound;       // > 0: every row's length is at most this; the ranges are split on it
+    float logit_tau;
+    int32_t *out_draft, *out_len, *out_mode;
+    float *out_score;
+    int32_t *out_match_n, *out_match_end, *status;
+    int32_t W, D, bm_words;   // candidate mode: W candidates of up to D tokens; bitmap words per CTA
+    int32_t *out_cand, *out_cand_len, *out_ncand;
+    const int32_t *pv_cand_len;  // candidate mode, verifying: the previous candidates' lengths [B, W]
+                                 // (pv_draft [B, W, D], pv_target [B, W, D+1], pv_len = their count [B])
+    int32_t *out_choice;         // ... and the kept candidate [B]
+};
+
+__device__ __forceinline__ float dot8_bf16(uint4 w, uint4 h, float acc) {
+    acc = fmaf(bf16_lo(w.x), bf16_lo(h.x), acc);
+    acc = fmaf(bf16_hi(w.x), bf16_hi(h.x), acc);
+    acc = fmaf(bf16_lo(w.y), bf16_lo(h.y), acc);
+    acc = fmaf(bf16_hi(w.y), bf16_hi(h.y), acc);
+    acc = fmaf(bf16_lo(w.z), bf16_lo(h.z), acc);
+    acc = fmaf(bf16_hi(w.z), bf16_hi(h.z), acc);
+    acc = fmaf(bf16_lo(w.w), bf16_lo(h.w), acc);
+    acc = fmaf(bf16_hi(w.w), bf16_hi(h.w), acc);
+    return acc;
+}
+
+__device__ __forceinline__ void st_cluster_i32(uint32_t addr, int32_t v) {
+    asm volatile("st.shared::cluster.s32 [%0], %1;\n" ::"r"(addr), "r"(v) : "memory");
+}
+
+// Launches step_kernel<cand> on grid (split, B) as clusters of `split` CTAs, with the shared memory
+// that args.stages / args.tile / args.bm_words call for.
+cudaError_t launch_step_kernel(const StepArgs &args, bool cand, int split, cudaStream_t stream);
+
+}  // namespace switchsd
