@@ -66,6 +66,7 @@ __global__ void __launch_bounds__(kStepThreads) step_kernel(const StepArgs a) {
     __shared__ int32_t s_out[2];                               // leader: winner rank, draft length
     __shared__ __align__(16) int32_t s_cand[kMaxCand];         // candidate mode: this CTA's / the row's ends
     __shared__ int32_t s_ncand;
+    __shared__ int32_t s_wtot[kStepWarps];                     // candidate mode: marks per warp in a pass
     __shared__ int32_t s_choice;                               // candidate verification: the kept candidate
     __shared__ int32_t s_probe_late;                           // early probe: its copies did not land in time
 
@@ -255,13 +256,17 @@ __global__ void __launch_bounds__(kStepThreads) step_kernel(const StepArgs a) {
             const int ncx = badlen ? 0 : (nc > 0 ? nc : 1);
 #pragma unroll
             for (int w = 0; w < kMaxCand; ++w) {
-                if (w < ncx) {
+                // Slot 0 is read before the count arrives (every row uses it unless the count is bad),
+                // so a row with at most one candidate -- a neural draft -- waits for one round trip.
+                if (w == 0 || w < ncx) {
                     const size_t o = size_t(b) * a.W + w;
                     const int32_t *c = a.pv_draft + o * a.D;
                     const int32_t *t = a.pv_target + o * (a.D + 1);
                     const int32_t c_lo = lane < a.D ? c[lane] : 0, c_hi = lane + 32 < a.D ? c[lane + 32] : 0;
                     const int32_t t_lo = lane < a.D ? t[lane] : 0, t_hi = lane + 32 < a.D ? t[lane + 32] : 0;
-                    const int32_t len = nc > 0 ? a.pv_cand_len[o] : 0;
+                    const int32_t len_w = a.pv_cand_len[o];
+                    if (w >= ncx) break;  // warp-uniform: a bad count uses no slot
+                    const int32_t len = nc > 0 ? len_w : 0;
                     badlen |= len < 0 || len > a.D;
                     const unsigned m_lo = __ballot_sync(kFull, lane < len && c_lo != t_lo);
                     const unsigned m_hi = __ballot_sync(kFull, lane + 32 < len && c_hi != t_hi);
@@ -522,13 +527,14 @@ __global__ void __launch_bounds__(kStepThreads) step_kernel(const StepArgs a) {
         zp = warp_sum_f32(zp);
         if (lane == 0) s_wz[warp] = zp;
     }
-    if (kCand && warp == 0) {
-        // The CTA's most recent marked ends: 32 bitmap words per pass from the top; lane i holds word
-        // top - i, and a prefix sum of the popcounts ranks its bits after those of higher words.
+    if (kCand) {
+        // The CTA's most recent marked ends: kStepThreads bitmap words per pass from the top; thread t
+        // holds word top - t, and prefix sums of the popcounts (within the warp, then over the warps)
+        // rank its bits after those of higher words.  `found` is CTA-uniform.
         const uint32_t *bm = reinterpret_cast<const uint32_t *>(tiles + a.stages * stage_ints);
         int found = 0;
-        for (int top = a.bm_words - 1; top >= 0 && found < a.W; top -= kWarp) {
-            const int idx = top - lane;
+        for (int top = a.bm_words - 1; top >= 0 && found < a.W; top -= kStepThreads) {
+            const int idx = top - tid;
             const uint32_t wd = (idx >= 0 && !bad) ? bm[idx] : 0u;
             const int c = __popc(wd);
             int incl = c;
@@ -537,16 +543,25 @@ __global__ void __launch_bounds__(kStepThreads) step_kernel(const StepArgs a) {
                 const int t = __shfl_up_sync(kFull, incl, o);
                 if (lane >= o) incl += t;
             }
-            int r = found + incl - c;
+            if (lane == kWarp - 1) s_wtot[warp] = incl;
+            __syncthreads();
+            int before = found, total = 0;
+#pragma unroll
+            for (int w = 0; w < kStepWarps; ++w) {
+                before += w < warp ? s_wtot[w] : 0;
+                total += s_wtot[w];
+            }
+            int r = before + incl - c;
             uint32_t w2 = wd;
             while (w2 != 0u && r < a.W) {
                 const int bit = 31 - __clz(w2);
                 w2 &= ~(1u << bit);
                 s_cand[r++] = e_lo + idx * 32 + bit;
             }
-            found += __shfl_sync(kFull, incl, kWarp - 1);
+            found += total;
+            __syncthreads();  // s_wtot is rewritten by the next pass
         }
-        if (lane == 0) s_ncand = found < a.W ? found : a.W;
+        if (tid == 0) s_ncand = found < a.W ? found : a.W;
     }
     __syncthreads();
     float cta_z = 0.f;
@@ -602,13 +617,25 @@ __global__ void __launch_bounds__(kStepThreads) step_kernel(const StepArgs a) {
         const int32_t kappa = a.kappa > 0 ? a.kappa : a.n_min;
         int32_t ncand = 0;  // candidate mode: the row's candidates, merged from the most recent CTA down
         if (kCand) {
-            if (lane == 0 && hit) {
-                for (int r = int(C) - 1; r >= 0 && ncand < a.W; --r) {
-                    const int c = s_slot[r].count;
-                    for (int i = 0; i < c && ncand < a.W; ++i) s_cand[ncand++] = s_slot[r].cand[i];
-                }
+            // lane r holds CTA r's count; a suffix sum over the lanes places its ends after those of the
+            // more recent CTAs r+1 .. C-1; then lanes copy (CTA, end) pairs in parallel.
+            const int cnt = (hit && uint32_t(lane) < C) ? min(int(s_slot[lane].count), a.W) : 0;
+            int incl = cnt;
+#pragma unroll
+            for (int o = 1; o < kWarp; o <<= 1) {
+                const int t = __shfl_down_sync(kFull, incl, o);
+                if (lane + o < kWarp) incl += t;
             }
-            ncand = __shfl_sync(kFull, ncand, 0);
+            const int off = incl - cnt;
+            for (int j0 = 0; j0 < int(C) * kMaxCand; j0 += kWarp) {  // warp-uniform bound
+                const int j = j0 + lane;
+                const int r = min(j / kMaxCand, int(C) - 1), i = j - r * kMaxCand;
+                const int cnt_r = __shfl_sync(kFull, cnt, r);
+                const int off_r = __shfl_sync(kFull, off, r);
+                if (j < int(C) * kMaxCand && i < cnt_r && off_r + i < a.W) s_cand[off_r + i] = s_slot[r].cand[i];
+            }
+            __syncwarp();
+            ncand = min(__shfl_sync(kFull, incl, 0), a.W);
         }
         const bool gate = kCand ? ncand > 0 : n >= kappa;
         int32_t mode = SWITCHSD_MODE_NO_REP;
