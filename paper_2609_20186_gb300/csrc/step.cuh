@@ -8,7 +8,8 @@ namespace switchsd {
 
 constexpr int kStepThreads = 256;
 constexpr int kStepWarps = kStepThreads / kWarp;
-constexpr int kTileMax = 8192;        // largest staged tile (candidate ends)
+constexpr int kTileMax = 8192;        // tile of the ring of stages, for ranges above kSingleTileMax
+constexpr int kSingleTileMax = 16384; // a CTA range up to this many ends is staged by one copy
 constexpr int kHalo = 32;             // look-back staged before a tile: >= SWITCHSD_NMAX, multiple of 4
 constexpr int kFwd = SWITCHSD_KMAX;   // look-ahead staged after a tile: the longest copy draft
 constexpr int kMaxStages = 6;          // staged tiles in flight per CTA (bounded by shared memory)

@@ -183,8 +183,9 @@ static int step_entry(int32_t *ctx_tokens, int32_t *ctx_lens, const uint16_t *hi
 
     const int split = p->split > 0 ? p->split : choose_split(p->B, p->cap);
     // Tile: the largest CTA range (the last CTA may also cover a k + 1 token append), in one stage
-    // when it fits, else a ring of kTileMax stages, as many as the range needs up to kMaxStages and
-    // the shared-memory budget.
+    // up to kSingleTileMax ends (64 KB; one copy, and few enough bytes that a grid of two or four
+    // CTAs per SM stays resident in one wave), else a ring of kTileMax stages, as many as the range
+    // needs up to kMaxStages and the shared-memory budget.
     const int64_t range = ((int64_t(p->cap) - 1 + split - 1) / split + 3) / 4 * 4 + args.k + 1;
     // candidate mode: a bit per end of the CTA's range, after the stages
     args.W = cs ? cs->W : 0;
@@ -196,7 +197,7 @@ static int step_entry(int32_t *ctx_tokens, int32_t *ctx_lens, const uint16_t *hi
     args.pv_cand_len = cs ? cs->pv_cand_len : nullptr;
     args.out_choice = cs ? cs->out_choice : nullptr;
     const size_t budget = kStageSmemBudget - size_t(args.bm_words) * sizeof(uint32_t);
-    if (range <= kTileMax) {
+    if (range <= kSingleTileMax) {
         args.tile = int32_t((range + 3) / 4 * 4);
         args.stages = 1;
     } else {
