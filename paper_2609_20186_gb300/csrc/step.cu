@@ -501,10 +501,15 @@ __global__ void __launch_bounds__(kStepThreads) step_kernel(const StepArgs a) {
     const bool probe_in = early_probe ? s_probe_late == 0 : mbar_wait(&probe_bar, 0);
     if (early_probe) {
     } else if (!mlp) {
-        if (probe_in)
-            for (int i = tid; i < v_staged; i += kStepThreads) zp = dot8_bf16(s_pw[i], s_ph[i], zp);
-        for (int v = v0 + v_staged + tid; v < v1; v += kStepThreads)
-            zp = dot8_bf16(__ldg(w4 + v), __ldg(h4 + v), zp);
+        // The early probe's partition of the slice (warps 2-7, the same order), so the logit does not
+        // depend on whether the probe ran before or after the wait.
+        if (warp >= 2) {
+            if (probe_in)
+                for (int i = tid - 2 * kWarp; i < v_staged; i += kStepThreads - 2 * kWarp)
+                    zp = dot8_bf16(s_pw[i], s_ph[i], zp);
+            for (int v = v0 + v_staged + tid - 2 * kWarp; v < v1; v += kStepThreads - 2 * kWarp)
+                zp = dot8_bf16(__ldg(w4 + v), __ldg(h4 + v), zp);
+        }
     } else {
         const float *sp = reinterpret_cast<const float *>(s_probe);
         for (int j = tid; j < u1 - u0; j += kStepThreads) {

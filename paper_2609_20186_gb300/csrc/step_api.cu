@@ -27,12 +27,14 @@ static int sm_count_cached() {
 
 static bool aligned16(const void *p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 
-// CTAs per row: the smallest power of two giving at least two CTAs per SM over the batch, with at
-// least 1024 tokens of capacity per CTA, at most kMaxSplit.
+// CTAs per row: the largest power of two, at most kMaxSplit, that leaves every CTA at least 4096
+// candidate ends and keeps the grid within one wave of four CTAs per SM (the step kernel's register
+// limit); 1 at least.  Measured on this GPU, per-CTA ranges of 4K-9K ends in a single wave beat both
+// smaller ranges (more CTAs per row to reduce and ship) and a second wave.
 static int choose_split(int B, int cap) {
     const int sms = sm_count_cached() > 0 ? sm_count_cached() : 148;
     int c = 1;
-    while (c < kMaxSplit && int64_t(B) * c < 2ll * sms && cap / (2 * c) >= 1024) c *= 2;
+    while (c < kMaxSplit && cap / (2 * c) >= 4096 && int64_t(B) * (2 * c) <= 4ll * sms) c *= 2;
     return c;
 }
 
