@@ -322,7 +322,7 @@ def config_of(wl: synth.Workload, world: int, split: int, search: str = "scan",
               prefetch: bool = True, verify: str = "greedy", candidates: int = 0, cand_len: int = 0) -> dict:
     return {"workload": wl.name, "search": search, "verify": verify,
             "candidates": ({"W": candidates, "D": cand_len} if candidates > 0 else None),
-            "prefetch": bool(prefetch and search == "scan"), "B": wl.B, "L0": wl.L0, "V": wl.V, "d": wl.d, "k": wl.k,
+            "prefetch": bool(prefetch), "B": wl.B, "L0": wl.L0, "V": wl.V, "d": wl.d, "k": wl.k,
             "n_min": wl.n_min, "n_max": wl.n_max, "kappa": wl.kappa_eff, "tau": wl.tau,
             "probe": "linear" if wl.probe_kind == 0 else f"mlp{wl.d}x{wl.probe_hidden}",
             "global_batch": wl.B * world, "seq_len": wl.L0, "parallelism": f"replicas{world}",

@@ -116,9 +116,11 @@ typedef struct switchsd_index switchsd_index;
  *                of those inputs is then complete when the copies start.  A copy or memset just before
  *                the call is always safe.  In a serving loop the target's last kernel (its argmax)
  *                writes neither the context nor the hidden state.  The previous draft, its length
- *                and the target argmax are always read after the wait.  The index search ignores the
- *                field; with the two-layer probe SWITCHSD_PREFETCH_PROBE lets the probe kernel's copies
- *                of the hidden states and W1 start early.  Other bits are SWITCHSD_ERR_ARG.
+ *                and the target argmax are always read after the wait.  The index search reads the
+ *                row's length and tail (CONTEXT) and computes the linear probe (PROBE) before the wait;
+ *                its tables come after it.  With the two-layer probe SWITCHSD_PREFETCH_PROBE lets the
+ *                probe kernel's copies of the hidden states and W1 start early.  Other bits are
+ *                SWITCHSD_ERR_ARG.
  *   hidden_rows  0 or 1: hidden is [B, d], the state the probe reads for each row.  k + 1 (the fused
  *                switchsd_verify_step and switchsd_verify_sampled_step only): hidden is the
  *                target's verification output [B, k+1, d] and the probe reads row a_b of each row b --

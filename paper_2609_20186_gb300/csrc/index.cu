@@ -70,7 +70,29 @@ struct IndexArgs {
     int32_t W, D;
     const int32_t *pv_cand_len;  // [B][W]
     int32_t *out_choice, *out_cand, *out_cand_len, *out_ncand;
+    int32_t prefetch;  // SWITCHSD_PREFETCH_* bits: the inputs they name are read before the wait
 };
+
+// This thread's share of the linear probe's dot product over row b's hidden state (threads stride the
+// d/8 words; the same partition wherever it is computed, so the logit is the same).
+__device__ __forceinline__ float index_probe_partial(const IndexArgs &a, int b, int32_t hrow) {
+    const uint4 *h4 = reinterpret_cast<const uint4 *>(
+        a.hidden + (size_t(b) * size_t(a.hidden_rows > 1 ? a.hidden_rows : 1) + size_t(hrow)) * a.d);
+    const uint4 *w4 = reinterpret_cast<const uint4 *>(a.probe_w);
+    float zp = 0.f;
+    for (int v = threadIdx.x; v < (a.d >> 3); v += blockDim.x) {
+        const uint4 w = __ldg(w4 + v), h = __ldg(h4 + v);
+        zp = fmaf(bf16_lo(w.x), bf16_lo(h.x), zp);
+        zp = fmaf(bf16_hi(w.x), bf16_hi(h.x), zp);
+        zp = fmaf(bf16_lo(w.y), bf16_lo(h.y), zp);
+        zp = fmaf(bf16_hi(w.y), bf16_hi(h.y), zp);
+        zp = fmaf(bf16_lo(w.z), bf16_lo(h.z), zp);
+        zp = fmaf(bf16_hi(w.z), bf16_hi(h.z), zp);
+        zp = fmaf(bf16_lo(w.w), bf16_lo(h.w), zp);
+        zp = fmaf(bf16_hi(w.w), bf16_hi(h.w), zp);
+    }
+    return zp;
+}
 
 __global__ void __launch_bounds__(kIdxMaxWarps * kWarp) index_kernel(const IndexArgs a) {
     __shared__ int32_t s_tail[kIdxTail];     // x[L_old - NMAX .. L_old + KMAX]
@@ -79,14 +101,20 @@ __global__ void __launch_bounds__(kIdxMaxWarps * kWarp) index_kernel(const Index
     __shared__ float s_wz[kIdxMaxWarps];
     __shared__ int32_t s_out[3];
     __shared__ int32_t s_cend[SWITCHSD_WMAX];  // candidate mode: the listed ends, most recent first
-    __shared__ int32_t s_ncf, s_choice;
+    __shared__ int32_t s_ncf;
 
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     const int nwarps = blockDim.x >> 5;
     const int b = blockIdx.x;
     const bool verifying = a.pv_len != nullptr;
-    pdl_wait();
-    pdl_trigger();
+    // With the prefetch bits (the caller's promise that the preceding kernel writes neither) the row's
+    // length and tail, and the linear probe of row 0 of its state, are read before the wait.
+    const bool pf_ctx = (a.prefetch & SWITCHSD_PREFETCH_CONTEXT) != 0;
+    const bool pf_probe = (a.prefetch & SWITCHSD_PREFETCH_PROBE) != 0 && a.stepping && a.z1_part == nullptr &&
+                          a.hidden_rows <= 1;
+    float zp_early = 0.f;
+    if (pf_probe) zp_early = index_probe_partial(a, b, 0);
+    if (!pf_ctx) pdl_wait();
 
     if (tid == 0) s_ncf = 0;
     int32_t *row = a.ctx + size_t(b) * a.cap;
@@ -97,6 +125,8 @@ __global__ void __launch_bounds__(kIdxMaxWarps * kWarp) index_kernel(const Index
         const int32_t p = tail0 + i;
         s_tail[i] = (len_ok && p >= 0) ? row[p] : 0;
     }
+    if (pf_ctx) pdl_wait();  // the previous draft, the target and the index tables come after this
+    pdl_trigger();
     if (warp == 0) {
         int32_t acc = -1, L = L_old, vst = len_ok ? SWITCHSD_ROW_OK : SWITCHSD_ROW_BAD_LEN;
         int32_t choice = 0;
@@ -263,22 +293,11 @@ __global__ void __launch_bounds__(kIdxMaxWarps * kWarp) index_kernel(const Index
             const float bias = a.b1 ? a.b1[u] : 0.f;
             zp = fmaf(bf16_lo(uint32_t(a.w2[u])), fmaxf(z1 + bias, 0.f), zp);
         }
+    } else if (pf_probe) {
+        zp = zp_early;
     } else {
         const int32_t hrow = a.hidden_rows > 1 && s_ver[0] > 0 ? s_ver[0] : 0;  // row a_b when gathering
-        const uint4 *h4 = reinterpret_cast<const uint4 *>(
-            a.hidden + (size_t(b) * size_t(a.hidden_rows > 1 ? a.hidden_rows : 1) + size_t(hrow)) * a.d);
-        const uint4 *w4 = reinterpret_cast<const uint4 *>(a.probe_w);
-        for (int v = tid; v < (a.d >> 3); v += blockDim.x) {
-            const uint4 w = __ldg(w4 + v), h = __ldg(h4 + v);
-            zp = fmaf(bf16_lo(w.x), bf16_lo(h.x), zp);
-            zp = fmaf(bf16_hi(w.x), bf16_hi(h.x), zp);
-            zp = fmaf(bf16_lo(w.y), bf16_lo(h.y), zp);
-            zp = fmaf(bf16_hi(w.y), bf16_hi(h.y), zp);
-            zp = fmaf(bf16_lo(w.z), bf16_lo(h.z), zp);
-            zp = fmaf(bf16_hi(w.z), bf16_hi(h.z), zp);
-            zp = fmaf(bf16_lo(w.w), bf16_lo(h.w), zp);
-            zp = fmaf(bf16_hi(w.w), bf16_hi(h.w), zp);
-        }
+        zp = index_probe_partial(a, b, hrow);
     }
     zp = warp_sum_f32(zp);
     if (lane == 0) s_wz[warp] = zp;
@@ -379,7 +398,7 @@ int index_launch(switchsd_index *idx, int32_t *ctx, int32_t *lens, const uint16_
                  int32_t *out_draft, int32_t *out_len, int32_t *out_mode, float *out_score, int32_t *out_match_n,
                  int32_t *out_match_end, int32_t *status, int B, int cap, int d, int k, int n_min, int n_max, int kappa,
                  float logit_tau, bool stepping, cudaStream_t stream, const float *pv_p, const float *pv_q,
-                 const float *pv_u, int hidden_rows, const IndexCandidates *cand) {
+                 const float *pv_u, int hidden_rows, const IndexCandidates *cand, int prefetch) {
     if (idx->B != B || idx->cap != cap || idx->n_min != n_min || idx->n_max != n_max) return SWITCHSD_ERR_SHAPE;
     // Candidate mode lists the ends of the kappa-gram chain: kappa must be one of the index's n, or
     // above n_max (no end can then reach it: no candidate, as for the rescan).
@@ -392,6 +411,7 @@ int index_launch(switchsd_index *idx, int32_t *ctx, int32_t *lens, const uint16_
     a.out_cand = cand ? cand->out_cand : nullptr;
     a.out_cand_len = cand ? cand->out_cand_len : nullptr;
     a.out_ncand = cand ? cand->out_ncand : nullptr;
+    a.prefetch = prefetch;
     a.pv_p = pv_p;
     a.pv_q = pv_q;
     a.pv_u = pv_u;

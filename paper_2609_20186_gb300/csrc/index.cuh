@@ -23,7 +23,9 @@ struct IndexCandidates {
 // One launch of the index kernel on B rows: the verification of the previous draft (when pv_len is
 // not null; greedy, or sampled when pv_p is not null: accept while u * q < p in binary32, q null = 1),
 // the inserts of the appended tokens' n-grams and, when stepping, the lookup, probe, switch and copy
-// draft.  Linear probe: z1_part null; hidden_rows > 1: hidden is [B, hidden_rows, d] and the probe
+// draft.  prefetch: the SWITCHSD_PREFETCH_* bits of switchsd_params (the row's length and tail, and
+// the linear probe, are then read before the grid-dependency wait).  Linear probe: z1_part null;
+// hidden_rows > 1: hidden is [B, hidden_rows, d] and the probe
 // reads row a_b (row 0 when nothing was appended).  Two-layer probe: z1_part = the split-K partial
 // sums [mlp_S][B][H1p] of W1 h written by the kernel just before, b1 (may be null) and w2 the second
 // layer.  Returns a SWITCHSD_* code.
@@ -34,7 +36,7 @@ int index_launch(switchsd_index *idx, int32_t *ctx, int32_t *lens, const uint16_
                  int32_t *out_match_end, int32_t *status, int B, int cap, int d, int k, int n_min, int n_max, int kappa,
                  float logit_tau, bool stepping, cudaStream_t stream, const float *pv_p = nullptr,
                  const float *pv_q = nullptr, const float *pv_u = nullptr, int hidden_rows = 1,
-                 const IndexCandidates *cand = nullptr);
+                 const IndexCandidates *cand = nullptr, int prefetch = 0);
 
 int index_n_min(const switchsd_index *idx);
 int index_n_max(const switchsd_index *idx);

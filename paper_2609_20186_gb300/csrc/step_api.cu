@@ -263,7 +263,7 @@ static int step_entry(int32_t *ctx_tokens, int32_t *ctx_lens, const uint16_t *hi
                             args.H1, args.H1p, args.b2, pv_draft, pv_target, pv_len, out_accept, out_draft, out_len,
                             out_mode, out_score, p->out_match_n, p->out_match_end, p->status, p->B, p->cap, p->d, p->k,
                             p->n_min, p->n_max, p->kappa, p->logit_tau, true, stream, pv_p, pv_q, pv_u,
-                            args.hidden_rows, cs != nullptr ? &ic : nullptr);
+                            args.hidden_rows, cs != nullptr ? &ic : nullptr, p->prefetch);
     }
     const cudaError_t e = launch_step_kernel(args, cs != nullptr, split, stream);
     if (e != cudaSuccess) return SWITCHSD_ERR_CUDA;

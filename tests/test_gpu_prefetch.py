@@ -17,7 +17,7 @@ W = synth.WORKLOADS
 KEYS = ("draft", "len", "mode", "score", "match_n", "match_end", "status", "accept")
 
 
-def _chain(wl, prefetch: int, steps: int, record_every: int, len_bound: int = 0):
+def _chain(wl, prefetch: int, steps: int, record_every: int, len_bound: int = 0, use_index: bool = False):
     import torch
     from paper_2609_20186_gb300 import Session, bf16_tensor
 
@@ -25,7 +25,7 @@ def _chain(wl, prefetch: int, steps: int, record_every: int, len_bound: int = 0)
     sess = Session(ctx, lens, wl.probe_weights(), k=wl.k, n_min=wl.n_min, n_max=wl.n_max,
                    kappa=wl.kappa, logit_tau=wl.logit_tau, probe_kind=wl.probe_kind,
                    probe_hidden=wl.probe_hidden, future=wl.future(), harness=wl.harness_params(),
-                   d=wl.d, prefetch=prefetch, len_bound=len_bound)
+                   d=wl.d, prefetch=prefetch, len_bound=len_bound, use_index=use_index)
     hidden = bf16_tensor(np.stack([wl.hidden(t) for t in range(steps)]), sess.device)
     torch.cuda.synchronize()
     rec = {}
@@ -60,6 +60,22 @@ def test_prefetch_matches_back_to_back(name, steps):
                     n = int(a[t]["len"][r])
                     assert np.array_equal(a[t]["draft"][r, :n], b[t]["draft"][r, :n]), (t, r)
             else:
+                assert np.array_equal(a[t][key], b[t][key]), (name, t, key)
+
+
+@pytest.mark.parametrize("name,steps", [("zipf_32k", 40), ("mixed_128k", 24), ("code_16k", 16)])
+def test_prefetch_matches_back_to_back_index(name, steps):
+    """The same with the incremental index: its kernel reads the row's length and tail and computes the
+    linear probe before the wait."""
+    wl = W[name].scaled(steps=steps)
+    from paper_2609_20186_gb300 import binding as bd
+    a, a_ctx, a_lens = _chain(wl, 0, steps, record_every=3, use_index=True)
+    b, b_ctx, b_lens = _chain(wl, bd.PREFETCH_CONTEXT | bd.PREFETCH_PROBE, steps, record_every=3, use_index=True)
+    assert np.array_equal(a_lens, b_lens) and (a_lens > wl.L0).all()
+    assert np.array_equal(a_ctx, b_ctx)
+    for t in a:
+        for key in KEYS:
+            if key != "draft":
                 assert np.array_equal(a[t][key], b[t][key]), (name, t, key)
 
 
