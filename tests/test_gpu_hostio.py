@@ -12,12 +12,12 @@ import synth
 pytestmark = pytest.mark.gpu
 
 
-def _session(wl, prefetch):
+def _session(wl, prefetch, use_index=False):
     from paper_2609_20186_gb300 import Session, binding
     ctx, lens = wl.contexts()
     return Session(ctx, lens, wl.probe_weights(), k=wl.k, n_min=wl.n_min, n_max=wl.n_max, kappa=wl.kappa,
                    logit_tau=wl.logit_tau, probe_kind=wl.probe_kind, probe_hidden=wl.probe_hidden,
-                   future=wl.future(), harness=wl.harness_params(), d=wl.d,
+                   future=wl.future(), harness=wl.harness_params(), d=wl.d, use_index=use_index,
                    prefetch=(binding.PREFETCH_CONTEXT | binding.PREFETCH_PROBE) if prefetch else 0)
 
 
@@ -90,15 +90,16 @@ def test_read_ceiling_folds_what_it_reads(split, prefetch):
         assert np.bitwise_xor.reduce(got[b]) == want, b
 
 
+@pytest.mark.parametrize("use_index", [False, True], ids=["rescan", "index"])
 @pytest.mark.parametrize("name", ["zipf_32k", "code_16k"])
 @pytest.mark.parametrize("prefetch", [False, True])
-def test_plan_replays_match_device_calls(name, prefetch):
+def test_plan_replays_match_device_calls(name, prefetch, use_index):
     """Replays alternate between two host hidden buffers and two host result buffers, so the recorded
-    copies are retargeted on every replay."""
+    copies are retargeted on every replay.  With the index, the recorded graph holds the index kernel."""
     import torch
     from paper_2609_20186_gb300 import bf16_tensor
     wl = synth.WORKLOADS[name].scaled(B=8, L0=6001, steps=12)
-    a, b = _session(wl, prefetch), _session(wl, prefetch)
+    a, b = _session(wl, prefetch, use_index), _session(wl, prefetch, use_index)
     B, d, k = wl.B, wl.d, wl.k
     dev_h = torch.empty(B, d, dtype=torch.bfloat16, device="cuda")
     host_h = [torch.empty(B, d, dtype=torch.int16).pin_memory() for _ in range(2)]
