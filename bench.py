@@ -837,11 +837,10 @@ def read_ceiling(loop, d: int, K: int, step_base: int, prefetch: bool, cs) -> di
 
 
 def run_e2e(base, dev, W, K, split, world, prefetch=True, sampled=False):
-    """The same loop through the public API with host buffers, one batch.  Per step (greedy): the
-    target stand-in for the previous draft, then one replay of a switchsd_plan of
-    switchsd_verify_step_host -- pinned H2D of this step's hidden states, the fused launch, one D2H of
-    mode / draft length / accepted length / draft -- and a host sync.  Sampled: the same copies and
-    launches as separate stream-ordered calls."""
+    """The same loop through the public API with host buffers, one batch.  Per step: the target
+    stand-in for the previous draft, then one replay of a switchsd_plan of switchsd_verify_step_host
+    (or switchsd_verify_sampled_step_host) -- pinned H2D of this step's hidden states, the fused launch,
+    one D2H of mode / draft length / accepted length / draft -- and a host sync."""
     import torch
     from paper_2609_20186_gb300 import Session, binding
 
@@ -859,22 +858,19 @@ def run_e2e(base, dev, W, K, split, world, prefetch=True, sampled=False):
     dev_h = torch.empty(B, d, dtype=torch.bfloat16, device=dev)
     host_out = torch.empty(B * (k + 3), dtype=torch.int32).pin_memory()  # mode, len, accept, draft
     stream = torch.cuda.current_stream()
-    # switchsd_plan: the host-staged fused step (switchsd_verify_step_host) recorded once as a graph
-    plan = None if sampled else sess.host_plan(host_h[1], dev_h, host_out, verify=True)
+    # switchsd_plan: the host-staged fused step (switchsd_verify_step_host, or the sampled one) recorded
+    # once as a graph
+    plan = sess.host_plan(host_h[1], dev_h, host_out, verify=not sampled, sampled=sampled)
 
     def one(t):
         if t == 0:
             sess.step_host(host_h[0], dev_h, host_out)
             return
         if sampled:
-            sess.harness_sampled(t - 1)
-            dev_h.view(torch.int16).copy_(host_h[t], non_blocking=True)
-            sess.verify_sampled_step(dev_h, debug=False)
-            sess.outputs_to(host_out)  # one D2H copy of mode, draft length, accepted length and draft
-            stream.synchronize()
-            return
-        sess.harness(t - 1)            # the target's tokens for the previous draft
-        plan.run(host_h[t])            # H2D of this step's hidden states, the fused launch, D2H, sync
+            sess.harness_sampled(t - 1)  # the target's probabilities, uniforms and resample tokens
+        else:
+            sess.harness(t - 1)          # the target's tokens for the previous draft
+        plan.run(host_h[t])              # H2D of this step's hidden states, the fused launch, D2H, sync
 
     for t in range(W):
         one(t)
@@ -887,12 +883,10 @@ def run_e2e(base, dev, W, K, split, world, prefetch=True, sampled=False):
     value = replica_throughput(B * K, secs, world)
     return {"value": value, "unit": UNIT, "h2d_bytes_per_step": B * d * 2,
             "d2h_bytes_per_step": B * (k + 3) * 4,
-            "note": ("one batch; per step: target stand-in, then " +
-                     ("pinned H2D of hidden, switchsd_verify_sampled_step, D2H of mode/len/accept/draft, "
-                      "host sync" if sampled else
-                      "one switchsd_plan_run call replaying switchsd_verify_step_host recorded as a CUDA "
-                      "graph (pinned H2D of hidden, fused launch, one D2H of mode/len/accept/draft), host "
-                      "sync") + "; L2 not flushed")}
+            "note": ("one batch; per step: target stand-in, then one switchsd_plan_run call replaying "
+                     + ("switchsd_verify_sampled_step_host" if sampled else "switchsd_verify_step_host")
+                     + " recorded as a CUDA graph (pinned H2D of hidden, fused launch, one D2H of "
+                       "mode/len/accept/draft), host sync; L2 not flushed")}
 
 
 LABEL_METRIC = "copy-mode labels/sec (positions, §3.2, n_train=5); achieved HBM GB/s vs peak"

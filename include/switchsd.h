@@ -42,7 +42,7 @@
 extern "C" {
 #endif
 
-#define SWITCHSD_ABI_VERSION 6
+#define SWITCHSD_ABI_VERSION 7
 
 #define SWITCHSD_NMAX 32 /* largest supported n_max */
 #define SWITCHSD_KMAX 64 /* largest supported draft length k */
@@ -315,9 +315,19 @@ int switchsd_verify_step_host(const switchsd_host_io *io, const int32_t *draft, 
                               const switchsd_params *params, int32_t *out_draft, int32_t *out_len,
                               int32_t *out_mode, float *out_score);
 
+/* switchsd_verify_sampled_step between the two copies of `io`; codes as switchsd_step_host. */
+int switchsd_verify_sampled_step_host(const switchsd_host_io *io, const int32_t *draft, const float *p_draft,
+                                      const float *q_draft, const float *u, const int32_t *resample,
+                                      const int32_t *draft_len, int32_t *out_accept, int32_t *ctx_tokens,
+                                      int32_t *ctx_lens, const uint16_t *hidden, const uint16_t *probe_w,
+                                      const switchsd_params *params, int32_t *out_draft, int32_t *out_len,
+                                      int32_t *out_mode, float *out_score);
+
 /*
- * The arguments of one switchsd_verify_step call (draft, target_argmax and draft_len all set), or of
- * one switchsd_step call (all three NULL; out_accept is then unused), for switchsd_plan_create.
+ * The arguments of one switchsd_verify_step call (draft, target_argmax and draft_len all set), of one
+ * switchsd_verify_sampled_step call (p_draft and u set as well -- q_draft may stay NULL -- and
+ * target_argmax holding the resample tokens), or of one switchsd_step call (the verification buffers
+ * all NULL; out_accept is then unused), for switchsd_plan_create.
  */
 typedef struct {
     const int32_t *draft, *target_argmax, *draft_len;
@@ -327,6 +337,7 @@ typedef struct {
     const switchsd_params *params;
     int32_t *out_draft, *out_len, *out_mode;
     float *out_score;
+    const float *p_draft, *q_draft, *u;
 } switchsd_step_args;
 
 /* A host-staged step recorded once as a CUDA graph (opaque). */
@@ -338,9 +349,10 @@ typedef struct switchsd_plan switchsd_plan;
  * stream; nothing runs.  io->synchronize is ignored (switchsd_plan_run takes it).  The recorded
  * launches hold the device pointers and the parameter values, so *args and *args->params may be freed
  * after the call; replays launch on args->params->stream.  The caller keeps every buffer alive and, for
- * the two-layer probe, the workspace unshared while the plan can run.  Returns SWITCHSD_ERR_ARG (NULL out, args, params or io, a partial set of verification
- * buffers, a copy without buffers), SWITCHSD_ERR_CUDA (capture or instantiation failed), or the step's
- * own validation code; *out is then NULL.
+ * the two-layer probe, the workspace unshared while the plan can run.  Returns SWITCHSD_ERR_ARG (NULL
+ * out, args, params or io, a partial set of verification buffers, p_draft without u, a copy without
+ * buffers), SWITCHSD_ERR_CUDA (capture or instantiation failed), or the step's own validation code;
+ * *out is then NULL.
  */
 int switchsd_plan_create(const switchsd_step_args *args, const switchsd_host_io *io, switchsd_plan **out);
 

@@ -19,7 +19,7 @@ PROBE_LINEAR, PROBE_MLP = 0, 1
 OK, ERR_ARG, ERR_SHAPE, ERR_CUDA = 0, -1, -2, -3
 ROW_OK, ROW_CAPACITY, ROW_BAD_LEN, ROW_TIMEOUT = 0, 1, 2, 3
 NMAX, KMAX = 32, 64
-ABI_VERSION = 6  # SWITCHSD_ABI_VERSION this binding marshals for
+ABI_VERSION = 7  # SWITCHSD_ABI_VERSION this binding marshals for
 PREFETCH_CONTEXT, PREFETCH_PROBE = 1, 2  # switchsd_params.prefetch bits
 
 _c_i32p = ctypes.c_void_p
@@ -78,6 +78,7 @@ class switchsd_step_args(ctypes.Structure):
         ("params", ctypes.POINTER(switchsd_params)),
         ("out_draft", ctypes.c_void_p), ("out_len", ctypes.c_void_p), ("out_mode", ctypes.c_void_p),
         ("out_score", ctypes.c_void_p),
+        ("p_draft", ctypes.c_void_p), ("q_draft", ctypes.c_void_p), ("u", ctypes.c_void_p),
     ]
 
 
@@ -110,6 +111,8 @@ _SIGNATURES = {
                            + [ctypes.POINTER(switchsd_params)] + [ctypes.c_void_p] * 4),
     "switchsd_verify_step_host": (ctypes.c_int, [ctypes.POINTER(switchsd_host_io)] + [ctypes.c_void_p] * 8
                                   + [ctypes.POINTER(switchsd_params)] + [ctypes.c_void_p] * 4),
+    "switchsd_verify_sampled_step_host": (ctypes.c_int, [ctypes.POINTER(switchsd_host_io)] + [ctypes.c_void_p] * 11
+                                          + [ctypes.POINTER(switchsd_params)] + [ctypes.c_void_p] * 4),
     "switchsd_harness_read": (ctypes.c_int, [ctypes.c_void_p, ctypes.c_void_p, ctypes.c_int32, ctypes.c_int32,
                                              ctypes.c_void_p, ctypes.c_int32, ctypes.c_int32, ctypes.c_int32,
                                              ctypes.c_void_p, ctypes.c_void_p]),

@@ -164,6 +164,26 @@ extern "C" int switchsd_verify_step_host(const switchsd_host_io *io, const int32
     return stage_out(io, s);
 }
 
+extern "C" int switchsd_verify_sampled_step_host(const switchsd_host_io *io, const int32_t *draft,
+                                                 const float *p_draft, const float *q_draft, const float *u,
+                                                 const int32_t *resample, const int32_t *draft_len,
+                                                 int32_t *out_accept, int32_t *ctx_tokens, int32_t *ctx_lens,
+                                                 const uint16_t *hidden, const uint16_t *probe_w,
+                                                 const switchsd_params *params, int32_t *out_draft,
+                                                 int32_t *out_len, int32_t *out_mode, float *out_score) {
+    if (!io_ok(io) || params == nullptr) return SWITCHSD_ERR_ARG;
+    cudaStream_t s = static_cast<cudaStream_t>(params->stream);
+    bool by_kernel = false;
+    int code = stage_in(io, s, &by_kernel);
+    if (code != SWITCHSD_OK) return code;
+    const switchsd_params q = by_kernel ? after_copy_kernel(*params, io, ctx_tokens, ctx_lens, hidden, probe_w)
+                                        : *params;
+    code = switchsd_verify_sampled_step(draft, p_draft, q_draft, u, resample, draft_len, out_accept, ctx_tokens,
+                                        ctx_lens, hidden, probe_w, &q, out_draft, out_len, out_mode, out_score);
+    if (code != SWITCHSD_OK) return code;
+    return stage_out(io, s);
+}
+
 // ------------------------------------------------------------------------------------------------
 // switchsd_plan: the host-staged step recorded once as a CUDA graph and replayed per call.
 //
@@ -236,6 +256,8 @@ extern "C" int switchsd_plan_create(const switchsd_step_args *a, const switchsd_
     const bool verify = a->draft != nullptr || a->target_argmax != nullptr || a->draft_len != nullptr;
     if (verify && (a->draft == nullptr || a->target_argmax == nullptr || a->draft_len == nullptr))
         return SWITCHSD_ERR_ARG;
+    const bool sampled = a->p_draft != nullptr || a->u != nullptr || a->q_draft != nullptr;
+    if (sampled && (!verify || a->p_draft == nullptr || a->u == nullptr)) return SWITCHSD_ERR_ARG;
     switchsd_plan *p = new switchsd_plan;
     p->io = *io;
     p->io.synchronize = 0;
@@ -256,11 +278,15 @@ extern "C" int switchsd_plan_create(const switchsd_step_args *a, const switchsd_
                                          : *a->params;
         q.stream = cap;
         if (code == SWITCHSD_OK)
-            code = verify ? switchsd_verify_step(a->draft, a->target_argmax, a->draft_len, a->out_accept,
-                                                 a->ctx_tokens, a->ctx_lens, a->hidden, a->probe_w, &q, a->out_draft,
-                                                 a->out_len, a->out_mode, a->out_score)
-                          : switchsd_step(a->ctx_tokens, a->ctx_lens, a->hidden, a->probe_w, &q, a->out_draft,
-                                          a->out_len, a->out_mode, a->out_score);
+            code = sampled ? switchsd_verify_sampled_step(a->draft, a->p_draft, a->q_draft, a->u, a->target_argmax,
+                                                          a->draft_len, a->out_accept, a->ctx_tokens, a->ctx_lens,
+                                                          a->hidden, a->probe_w, &q, a->out_draft, a->out_len,
+                                                          a->out_mode, a->out_score)
+                   : verify ? switchsd_verify_step(a->draft, a->target_argmax, a->draft_len, a->out_accept,
+                                                   a->ctx_tokens, a->ctx_lens, a->hidden, a->probe_w, &q, a->out_draft,
+                                                   a->out_len, a->out_mode, a->out_score)
+                            : switchsd_step(a->ctx_tokens, a->ctx_lens, a->hidden, a->probe_w, &q, a->out_draft,
+                                            a->out_len, a->out_mode, a->out_score);
         p->out_kernel = p->io.out_bytes > 0 && mapped_address(p->io.out_host) != nullptr;
         if (code == SWITCHSD_OK) code = stage_out(&p->io, cap);  // synchronize is 0: queues the copy only
         cudaGraph_t g = nullptr;

@@ -291,17 +291,21 @@ class Session:
         return self._host_views(results_host)
 
     def host_plan(self, hidden_host: torch.Tensor, hidden: torch.Tensor, results_host: torch.Tensor,
-                  verify: bool = True, debug: bool = False) -> "HostPlan":
-        """switchsd_plan_create: what verify_step_host (verify=True) or step_host does with these buffers,
-        recorded once as a CUDA graph; HostPlan.run replays it with this step's host buffers."""
-        self._check_hidden(hidden, self.hidden_rows if verify else 1)
+                  verify: bool = True, debug: bool = False, sampled: bool = False) -> "HostPlan":
+        """switchsd_plan_create: what verify_step_host (verify=True), verify_sampled_step_host
+        (sampled=True: the sampled verification of vdraft with vp / vq / vu and the resample tokens in
+        target) or step_host does with these buffers, recorded once as a CUDA graph; HostPlan.run
+        replays it with this step's host buffers."""
+        self._check_hidden(hidden, self.hidden_rows if (verify or sampled) else 1)
         io = bd.switchsd_host_io.from_buffer_copy(self._host_io(hidden_host, hidden, results_host, False))
         p = bd.switchsd_params.from_buffer_copy(self._p_dbg if debug else self._p_fast)
-        if not verify:
+        if not (verify or sampled):
             p.hidden_rows = 0
         a = bd.switchsd_step_args()
-        if verify:
+        if verify or sampled:
             a.draft, a.target_argmax, a.draft_len, a.out_accept = self._vs_head
+        if sampled:
+            a.p_draft, a.q_draft, a.u = self.vp.data_ptr(), self.vq.data_ptr(), self.vu.data_ptr()
         a.ctx_tokens, a.ctx_lens = self._step_head
         a.hidden, a.probe_w = hidden.data_ptr(), self.probe_w.data_ptr()
         a.params = ctypes.pointer(p)
@@ -311,6 +315,20 @@ class Session:
         if code != bd.OK:
             raise RuntimeError(f"switchsd_plan_create failed: {code} ({bd.strerror(code)})")
         return HostPlan(self, h, io.in_bytes, (hidden_host, hidden, results_host))
+
+    def verify_sampled_step_host(self, hidden_host: torch.Tensor, hidden: torch.Tensor,
+                                 results_host: torch.Tensor, debug: bool = False, synchronize: bool = True) -> dict:
+        """switchsd_verify_sampled_step_host: verify_sampled_step between the copies of step_host."""
+        self._check_hidden(hidden, self.hidden_rows)
+        io = self._host_io(hidden_host, hidden, results_host, synchronize)
+        p = self._p_dbg if debug else self._p_fast
+        code = self.lib.switchsd_verify_sampled_step_host(
+            ctypes.byref(io), self.vdraft.data_ptr(), self.vp.data_ptr(), self.vq.data_ptr(), self.vu.data_ptr(),
+            self.target.data_ptr(), self.vlen.data_ptr(), self.accept.data_ptr(), self.ctx.data_ptr(),
+            self.lens.data_ptr(), hidden.data_ptr(), *self._step_tail, ctypes.byref(p), *self._step_outs)
+        if code != bd.OK:
+            raise RuntimeError(f"switchsd_verify_sampled_step_host failed: {code} ({bd.strerror(code)})")
+        return self._host_views(results_host)
 
     # --- host views ------------------------------------------------------------------------------
     def step_outputs(self) -> dict:

@@ -58,7 +58,7 @@ def test_binding_declares_every_function():
 
 def test_abi_version_and_strerror(lib):
     from paper_2609_20186_gb300 import binding as bd
-    assert bd.abi_version() == 6
+    assert bd.abi_version() == 7
     for code in (0, -1, -2, -3, 1, 2, 3):
         assert bd.strerror(code) != "unknown code"
     assert bd.strerror(12345) == "unknown code"
@@ -188,6 +188,10 @@ def test_host_staged_validation(lib):
     assert lib.switchsd_step_host(ctypes.byref(io), f, f, f, f, ctypes.byref(bad), f, f, f, f) == bd.ERR_SHAPE
     assert lib.switchsd_verify_step_host(ctypes.byref(io), f, f, f, f, f, f, f, f, ctypes.byref(bad),
                                          f, f, f, f) == bd.ERR_SHAPE
+    assert lib.switchsd_verify_sampled_step_host(None, f, f, None, f, f, f, f, f, f, f, f, ctypes.byref(p),
+                                                 f, f, f, f) == bd.ERR_ARG
+    assert lib.switchsd_verify_sampled_step_host(ctypes.byref(io), f, f, None, f, f, f, f, f, f, f, f,
+                                                 ctypes.byref(bad), f, f, f, f) == bd.ERR_SHAPE
 
 
 def test_plan_validation(lib):
@@ -210,6 +214,11 @@ def test_plan_validation(lib):
     a.draft = None
     io.in_bytes = 16                                     # a copy without buffers
     assert lib.switchsd_plan_create(ctypes.byref(a), ctypes.byref(io), ctypes.byref(h)) == bd.ERR_ARG
+    a.p_draft = f                                        # sampled arguments without a verification
+    assert lib.switchsd_plan_create(ctypes.byref(a), ctypes.byref(io), ctypes.byref(h)) == bd.ERR_ARG
+    a.draft = a.target_argmax = a.draft_len = a.out_accept = f   # ... or without the uniforms
+    assert lib.switchsd_plan_create(ctypes.byref(a), ctypes.byref(io), ctypes.byref(h)) == bd.ERR_ARG
+    a.p_draft = a.draft = a.target_argmax = a.draft_len = a.out_accept = None
     a.params = None
     io.in_bytes = 0
     assert lib.switchsd_plan_create(ctypes.byref(a), ctypes.byref(io), ctypes.byref(h)) == bd.ERR_ARG

@@ -159,3 +159,43 @@ def test_host_staged_pageable_and_pinned(pinned):
         torch.cuda.synchronize()
         assert np.array_equal(host_out.numpy(), a.results.cpu().numpy()), t
     assert np.array_equal(a.ctx.cpu().numpy(), b.ctx.cpu().numpy())
+
+
+@pytest.mark.parametrize("use_index", [False, True], ids=["rescan", "index"])
+def test_sampled_host_staged_and_plan_match_device_calls(use_index):
+    """The sampled fused step from host buffers: switchsd_verify_sampled_step_host on one session, a
+    plan of it on another, the device call on a third; all three agree step after step."""
+    import torch
+    from paper_2609_20186_gb300 import bf16_tensor
+    wl = synth.WORKLOADS["zipf_32k"].scaled(B=8, L0=6001, steps=10)
+    a, b, c = (_session(wl, True, use_index) for _ in range(3))
+    B, d, k = wl.B, wl.d, wl.k
+    dev_b = torch.empty(B, d, dtype=torch.bfloat16, device="cuda")
+    dev_c = torch.empty(B, d, dtype=torch.bfloat16, device="cuda")
+    host_h = [torch.empty(B, d, dtype=torch.int16).pin_memory() for _ in range(2)]
+    out_b = torch.empty(B * (k + 3), dtype=torch.int32).pin_memory()
+    out_c = torch.empty(B * (k + 3), dtype=torch.int32).pin_memory()
+    plan = c.host_plan(host_h[1], dev_c, out_c, verify=False, sampled=True)
+    for t in range(wl.steps):
+        hid = wl.hidden(t)
+        hh = host_h[t % 2]
+        hh.copy_(torch.from_numpy(hid.view(np.int16)))
+        if t == 0:
+            for s_, dh, ho in ((a, None, None), (b, dev_b, out_b), (c, dev_c, out_c)):
+                if dh is None:
+                    s_.step(bf16_tensor(hid, "cuda"), debug=False)
+                else:
+                    s_.step_host(hh, dh, ho)
+        else:
+            for s_ in (a, b, c):
+                s_.harness_sampled(t - 1)
+            a.verify_sampled_step(bf16_tensor(hid, "cuda"), debug=False)
+            b.verify_sampled_step_host(hh, dev_b, out_b)
+            plan.run(hh, out_c)
+        torch.cuda.synchronize()
+        want = a.results.cpu().numpy()
+        assert np.array_equal(out_b.numpy(), want), t
+        assert np.array_equal(out_c.numpy(), want), t
+    assert np.array_equal(a.ctx.cpu().numpy(), b.ctx.cpu().numpy())
+    assert np.array_equal(a.ctx.cpu().numpy(), c.ctx.cpu().numpy())
+    plan.close()
