@@ -73,6 +73,9 @@ __global__ void __launch_bounds__(kStepThreads) step_kernel(const StepArgs a) {
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     const uint32_t rank = cluster_ctarank();
     const uint32_t C = cluster_nctarank();
+    // The leader is the last CTA: its range holds the most recent ends, so the candidate mode finds
+    // most continuations in its own staged tile.
+    const uint32_t lead = C - 1;
     const int b = blockIdx.y;
     const int stage_ints = kHalo + a.tile + kFwd;
     const bool verifying = a.pv_len != nullptr;
@@ -84,7 +87,7 @@ __global__ void __launch_bounds__(kStepThreads) step_kernel(const StepArgs a) {
         mbar_init(&tail_bar, 1);
         mbar_init(&probe_bar, 1);
         s_probe_late = 0;
-        if (rank == 0) {
+        if (rank == lead) {
             mbar_init(&s_done, 1);
             mbar_arrive_expect_tx(&s_done, slot_bytes * C);
         }
@@ -574,7 +577,7 @@ __global__ void __launch_bounds__(kStepThreads) step_kernel(const StepArgs a) {
 
     // Every CTA has started and read ctx_lens[b] once this returns (they all arrived long ago).
     cluster_wait_acquire();
-    if (rank == 0 && verifying) {
+    if (rank == lead && verifying) {
         // The leader publishes the append; the other CTAs only patched their staged copies.
         for (int i = tid; i <= acc; i += kStepThreads) row[L_old + i] = s_app[i];
         if (tid == 0 && len_ok) {
@@ -584,20 +587,20 @@ __global__ void __launch_bounds__(kStepThreads) step_kernel(const StepArgs a) {
     }
 
     // Ship this CTA's message to the leader: asynchronous DSMEM stores that complete on its barrier.
-    const uint32_t done_addr = map_to_rank(&s_done, 0);
+    const uint32_t done_addr = map_to_rank(&s_done, lead);
     if (tid == 0) {
         uint4 h;
         h.x = uint32_t(best & 0xffffffffu);
         h.y = uint32_t(best >> 32);
         h.z = __float_as_uint(cta_z);
         h.w = kCand ? uint32_t(s_ncand) : 0u;
-        st_async_v4(map_to_rank(&s_slot[rank], 0), h, done_addr);
+        st_async_v4(map_to_rank(&s_slot[rank], lead), h, done_addr);
     } else if (tid <= kwords) {
         const uint4 v = kCand ? *reinterpret_cast<const uint4 *>(&s_cand[4 * (tid - 1)])
                               : *reinterpret_cast<const uint4 *>(&s_mine[4 * (tid - 1)]);
-        st_async_v4(map_to_rank(&s_slot[rank].cand[4 * (tid - 1)], 0), v, done_addr);
+        st_async_v4(map_to_rank(&s_slot[rank].cand[4 * (tid - 1)], lead), v, done_addr);
     }
-    if (rank != 0) return;
+    if (rank != lead) return;
 
     if (warp == 0) {
         // Bounded wait for every CTA's message (C x slot_bytes of transaction); lane r reads CTA r's.
@@ -669,16 +672,23 @@ __global__ void __launch_bounds__(kStepThreads) step_kernel(const StepArgs a) {
     }
     if (kCand) {
         __syncthreads();
-        // The candidates' continuations, read from the row (the leader's append, if any, is visible
-        // to its threads after the barrier).
+        // The candidates' continuations: from the leader's own staged tile for ends in its range (one
+        // stage: it holds the range, its look-ahead and the patched append), else from the row (the
+        // leader's append is visible to its threads after the barrier).
         const int nc = s_ncand;
         if (tid == 0) a.out_ncand[b] = nc;
+        const bool one_stage = ntiles == 1;
+        const int32_t off0 = kHalo - e_lo;  // tiles[off0 + p] = x[p] over the staged range
         for (int t = tid; t < nc * a.D; t += kStepThreads) {
             const int w = t / a.D, i = t - w * a.D;
             const int32_t ew = s_cand[w];
             const int32_t lw = min(a.D, L - 1 - ew);
             if (i == 0) a.out_cand_len[size_t(b) * a.W + w] = lw;
-            if (i < lw) a.out_cand[(size_t(b) * a.W + w) * a.D + i] = row[ew + 1 + i];
+            if (i < lw) {
+                const int32_t p = ew + 1 + i;
+                a.out_cand[(size_t(b) * a.W + w) * a.D + i] =
+                    (one_stage && ew >= e_lo && ew < e_hi) ? tiles[off0 + p] : row[p];
+            }
         }
     }
 }
