@@ -223,13 +223,14 @@ def host_threads() -> int:
 
 def time_oracle(wl: synth.Workload, budget_s: float, max_steps: int, rows: int | None = None,
                 warmup: int = 0, sampled: bool = False, cand: tuple[int, int] | None = None,
-                threads: int = 1):
+                threads: int = 1, state: dict | None = None):
     """Runs the oracle loop (oracle step, host target stand-in, oracle verify) on rows [0, R):
     ``warmup`` untimed steps, then up to max_steps timed steps or until budget_s of oracle time is
     spent.  Returns (seq*steps, seconds, timed_steps, R).  Only the oracle's calls are timed.
 
     threads > 1 runs each oracle call as that many concurrent calls on contiguous ranges of rows (rows
-    are independent; the oracle's C calls release the interpreter lock), the oracle itself unchanged."""
+    are independent; the oracle's C calls release the interpreter lock), the oracle itself unchanged.
+    state: if given, receives the final contexts and lengths."""
     import oracle
     from concurrent.futures import ThreadPoolExecutor
     R = wl.B if rows is None else min(rows, wl.B)
@@ -303,6 +304,8 @@ def time_oracle(wl: synth.Workload, budget_s: float, max_steps: int, rows: int |
     finally:
         if pool is not None:
             pool.shutdown()
+    if state is not None:
+        state.update(ctx=ctx, lens=lens)
     return R * done, spent, done, R
 
 

@@ -1,5 +1,6 @@
 """Host-side logic of bench.py: replica throughput over ranks (gloo, world size 2, CPU), replica
-count for the inputs-larger-than-L2 protocol, and the reference arm's JSON line."""
+count for the inputs-larger-than-L2 protocol, the CPU baseline's split of rows over threads, and the
+reference arm's JSON line."""
 import json
 import os
 import socket
@@ -70,3 +71,20 @@ def test_reference_arm_line():
     assert line["value"] > 0 and line["cpu_baseline"]["kind"] == "oracle"
     assert line["e2e"]["h2d_bytes_per_step"] == 0 and line["e2e"]["value"] == line["value"]
     assert line["config"]["workload"] == "uniform_8k"
+
+
+@pytest.mark.parametrize("mode", ["greedy", "sampled", "candidates"])
+def test_threaded_oracle_timing_computes_the_same(mode):
+    """The CPU baseline runs the oracle on contiguous row ranges in threads: the loop must leave the same
+    contexts and lengths as one thread (rows are independent)."""
+    sys.path.insert(0, ROOT)
+    import bench
+    import synth
+    wl = synth.get_workload("zipf_32k").scaled(B=12, L0=3001, steps=6)
+    kw = dict(sampled=mode == "sampled", cand=(4, 8) if mode == "candidates" else None)
+    one, many = {}, {}
+    u1, _, s1, _ = bench.time_oracle(wl, 1e9, 6, threads=1, state=one, **kw)
+    u4, _, s4, _ = bench.time_oracle(wl, 1e9, 6, threads=4, state=many, **kw)
+    assert (u1, s1) == (u4, s4) == (12 * 6, 6)
+    assert (one["lens"] > wl.L0).all()
+    assert (one["lens"] == many["lens"]).all() and (one["ctx"] == many["ctx"]).all()
