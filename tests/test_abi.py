@@ -238,6 +238,51 @@ def test_read_ceiling_validation(lib):
     assert lib.switchsd_harness_read(f, f, 0, 64, f, 16, 8, 1, f, None) == bd.ERR_SHAPE
 
 
+def test_candidates_index_static_validation(lib):
+    """The candidate, index and static-workspace entry points reject bad arguments before any CUDA call."""
+    from paper_2609_20186_gb300 import binding as bd
+    f = FAKE
+    p = _params()
+    # switchsd_step_candidates: W in 1..WMAX, D in 1..KMAX, every output given
+    cand = lambda W, D, outs=(f, f, f): lib.switchsd_step_candidates(f, f, f, f, ctypes.byref(p), W, D, *outs, f, f)
+    assert cand(0, 20) == bd.ERR_SHAPE
+    assert cand(17, 20) == bd.ERR_SHAPE                  # W above SWITCHSD_WMAX (16)
+    assert cand(10, 0) == bd.ERR_SHAPE
+    assert cand(10, 65) == bd.ERR_SHAPE
+    assert cand(10, 20, (None, f, f)) == bd.ERR_ARG
+    assert cand(10, 20, (f, f, None)) == bd.ERR_ARG
+    # the fused candidate verification needs its verification buffers
+    assert lib.switchsd_verify_candidates_step(None, f, f, f, f, f, f, f, f, f, ctypes.byref(p), 10, 20,
+                                               f, f, f, f, f) == bd.ERR_ARG
+    assert lib.switchsd_verify_candidates_step(f, f, f, f, f, None, f, f, f, f, ctypes.byref(p), 10, 20,
+                                               f, f, f, f, f) == bd.ERR_ARG
+    # switchsd_verify_candidates: pointers, then shapes
+    vp = bd.switchsd_candidates_verify_params()
+    vp.B, vp.cap, vp.W, vp.D = 4, 64, 10, 20
+    vp.cand_len = vp.ncand = vp.ctx_tokens = vp.ctx_lens = f
+    assert lib.switchsd_verify_candidates(f, f, f, f, None) == bd.ERR_ARG
+    assert lib.switchsd_verify_candidates(f, f, f, None, ctypes.byref(vp)) == bd.ERR_ARG
+    vp.W = 17
+    assert lib.switchsd_verify_candidates(f, f, f, f, ctypes.byref(vp)) == bd.ERR_SHAPE
+    vp.W, vp.cap = 10, 66
+    assert lib.switchsd_verify_candidates(f, f, f, f, ctypes.byref(vp)) == bd.ERR_SHAPE
+    # the fused verification needs its buffers too
+    assert lib.switchsd_verify_step(None, f, f, f, f, f, f, f, ctypes.byref(p), f, f, f, f) == bd.ERR_ARG
+    assert lib.switchsd_verify_step(f, f, f, None, f, f, f, f, ctypes.byref(p), f, f, f, f) == bd.ERR_ARG
+    # switchsd_index_create: shapes before any allocation
+    h = ctypes.c_void_p()
+    assert lib.switchsd_index_create(None, ctypes.byref(h)) == bd.ERR_ARG
+    for kw in (dict(B=0), dict(cap=66), dict(n_min=0), dict(n_min=5, n_max=4), dict(n_max=33)):
+        q = _params(**kw)
+        assert lib.switchsd_index_create(ctypes.byref(q), ctypes.byref(h)) == bd.ERR_SHAPE, kw
+        assert h.value is None
+    # switchsd_step_static_workspace: no params; a two-layer probe whose scratch exceeds the 16 MiB array
+    assert lib.switchsd_step_static_workspace(f, f, f, f, None, f, f, f, f) == bd.ERR_ARG
+    big = _params(probe_kind=1, probe_hidden=1024, d=8192, B=4096)
+    assert bd.switchsd_workspace_bytes(4096, 1, 1024, 8192) > 16 << 20
+    assert lib.switchsd_step_static_workspace(f, f, f, f, ctypes.byref(big), f, f, f, f) == bd.ERR_SHAPE
+
+
 def test_binding_rejects_cpu_tensors(lib):
     import torch
     from paper_2609_20186_gb300 import binding as bd
