@@ -65,6 +65,9 @@ def parse_args(argv=None):
                     help="budget of the CPU-baseline sample")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-per-config", action="store_true",
+                    help="time the selected workload only (by default the 32K headline also times the "
+                         "suite's other workloads into the same line)")
     ap.add_argument("--candidates", type=int, default=0,
                     help="W > 0: the step with W copy candidates (§3.3, App. D; the paper's W = 10)")
     ap.add_argument("--cand-len", type=int, default=20, help="D, the candidate length (the paper's 20)")
@@ -183,7 +186,7 @@ def measured_peaks() -> dict:
 def kernel_source_hash() -> str:
     h = hashlib.sha256()
     csrc = os.path.join(ROOT, "paper_2609_20186_gb300", "csrc")
-    for f in ("common.cuh", "step.cuh", "step.cu"):
+    for f in ("common.cuh", "step.cuh", "step.cu", "rescan.cu"):
         with open(os.path.join(csrc, f), "rb") as fh:
             h.update(fh.read())
     return h.hexdigest()[:16]
@@ -330,7 +333,7 @@ def config_of(wl: synth.Workload, world: int, split: int, search: str = "scan",
             "probe": "linear" if wl.probe_kind == 0 else f"mlp{wl.d}x{wl.probe_hidden}",
             "global_batch": wl.B * world, "seq_len": wl.L0, "parallelism": f"replicas{world}",
             "split": split,
-            "l2": "flushed before every timed step (write 2x L2, then read another 2x L2 buffer)"}
+            "l2": "cold: every timed launch reads contexts that are not in L2"}
 
 
 def run_reference(args, world, rank):
@@ -367,11 +370,13 @@ def run_reference(args, world, rank):
 # ------------------------------------------------------------------------------------------------
 # GPU run
 # ------------------------------------------------------------------------------------------------
-def choose_replicas(ctx_bytes: int, l2_bytes: int, K: int) -> int:
-    """Smallest power of two R with R batches' contexts >= 2.2x L2 (so each launch reads its batch
-    from HBM), at most K."""
-    r = 1
-    while r * ctx_bytes < 2.2 * l2_bytes and r < K:
+def choose_replicas(batch_bytes: int, l2_bytes: int, K: int, min_cover: int = 64, max_r: int = 1024) -> int:
+    """Replica batches of the timed loop: the smallest power of two R such that the other R - 1 batches'
+    contexts cover 2.2x L2 (a batch read again R launches later has been pushed out of L2 in between),
+    and R >= min(K, min_cover), so that a timed region of up to min_cover launches reads each batch once
+    (the target stand-in then runs outside it); at most max_r (workloads far below L2 stay L2-resident)."""
+    r = 2
+    while r < max_r and ((r - 1) * batch_bytes < 2.2 * l2_bytes or r < min(K, min_cover)):
         r *= 2
     return r
 
@@ -394,11 +399,11 @@ class ReplicaLoop:
         B, k = wl.B, wl.k
         ctx = np.zeros((B, cap), np.int32)
         ctx[:, : ctx1.shape[1]] = ctx1[:, : min(cap, ctx1.shape[1])]
-        self.ctx = torch.from_numpy(np.tile(ctx, (R, 1))).to(dev)
-        self.lens = torch.from_numpy(np.tile(lens1, R)).to(dev)
+        self.ctx = torch.from_numpy(ctx).to(dev).repeat(R, 1).contiguous()
+        self.lens = torch.from_numpy(np.ascontiguousarray(lens1, np.int32)).to(dev).repeat(R).contiguous()
         self.probe_w = bf16_tensor(pw.reshape(-1), dev)
-        fut = np.tile(future1, (R, 1))
-        self.future = torch.from_numpy(np.ascontiguousarray(fut, np.int32)).to(dev)
+        fut = torch.from_numpy(np.ascontiguousarray(future1, np.int32)).to(dev)
+        self.future = fut.repeat(R, 1).contiguous()
         i32 = dict(dtype=torch.int32, device=dev)
         N = R * B
         self.draft = torch.zeros(N, k, **i32)
@@ -409,7 +414,7 @@ class ReplicaLoop:
         self.vlen = torch.zeros(N, **i32)
         self.target = torch.zeros(N, k + 1, **i32)
         self.accept = torch.zeros(N, **i32)
-        self.hidden = hidden                     # bf16 [steps, B, d]: one block per launch
+        self.hidden = hidden                     # bf16 [nh, B, d]: launch i reads block i mod nh
         sp = stream.cuda_stream
         p = bd.switchsd_params()
         p.B, p.cap, p.d, p.k = B, cap, wl.d, k
@@ -489,7 +494,7 @@ class ReplicaLoop:
 
     def launch(self, r: int, step_index: int, first: bool):
         c = self.rows[r]
-        hid = self.hidden.data_ptr() + step_index * self.hstride
+        hid = self.hidden.data_ptr() + (step_index % self.hidden.shape[0]) * self.hstride
         if self.cw > 0:
             B, Wc, Dc, o = self.B, self.cw, self.cd, r * self.B
             outs = (self.cand.data_ptr() + o * Wc * Dc * 4, self.clen.data_ptr() + o * Wc * 4,
@@ -546,9 +551,220 @@ class ReplicaLoop:
         self.harness(q)
 
 
+def nvtx_range(name: str):
+    """An NVTX range around a phase of the run (visible in a profiler timeline); a no-op without NVTX."""
+    import contextlib
+    import torch
+    try:
+        torch.cuda.nvtx.range_push(name)
+    except Exception:
+        return contextlib.nullcontext()
+
+    @contextlib.contextmanager
+    def _pop():
+        try:
+            yield
+        finally:
+            try:
+                torch.cuda.nvtx.range_pop()
+            except Exception:
+                pass
+    return _pop()
+
+
+def l2_flush(buf):
+    """Writes a buffer of 2x L2 so that nothing the next launches read is left in L2."""
+    buf.fill_(1.0)
+
+
+def measure_loop(base, args, dev, cs, l2, W, K, split, search, prefetch, sampled, cand_w, cand_d, world,
+                 headline=False, flush=None):
+    """Times K fused controller launches (switchsd_verify_step, or its sampled / candidate / index form)
+    of workload `base` captured in one CUDA graph, launch i on replica batch i mod R (see
+    choose_replicas), after at least W untimed launches and an L2 flush.  Returns the measurement as a
+    dict; the headline also gets the clock record, the L2-resident leg and the cold single launches."""
+    import torch
+    from paper_2609_20186_gb300 import bf16_tensor
+
+    B, d, k = base.B, base.d, base.k
+    batch_bytes = B * (base.L0 + 1024) * 4
+    R = choose_replicas(batch_bytes, l2, K, max_r=(16 if search == "index" else 1024))
+    rounds = -(-K // R)
+    warm_rounds = max(1, -(-W // R))
+    per_row_steps = warm_rounds + 2 * rounds + (COLD_STEPS if headline else 0) + 1
+    wl = base.scaled(steps=per_row_steps)
+    cap = wl.cap
+    ctx1, lens1 = wl.contexts()
+    future1 = wl.future()
+    pw = wl.probe_weights()
+    n_hidden = min((warm_rounds + rounds) * R, 64)        # distinct hidden blocks, cycled over launches
+    hidden_host = np.empty((n_hidden, B, d), np.uint16)
+    for i in range(n_hidden):
+        hidden_host[i] = wl.hidden(i)
+    hidden = bf16_tensor(hidden_host, dev)
+    loop = ReplicaLoop(wl, R, cap, ctx1, lens1, pw, future1, hidden, split, dev, cs, search=search,
+                       prefetch=prefetch, sampled=sampled, cand_w=cand_w, cand_d=cand_d)
+    if flush is None:
+        flush = torch.empty(2 * l2 // 4, dtype=torch.float32, device=dev)
+
+    with torch.cuda.stream(cs):
+        for q in range(warm_rounds):                       # eager warm-up rounds (every batch once per round)
+            loop.round(q, q == 0, q * R)
+        # length snapshots at round boundaries: outside the timed graph, except between its own rounds
+        lens_hist = torch.zeros(rounds + 1, R * B, dtype=torch.int32, device=dev)
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, stream=cs):
+            for j in range(rounds):
+                q = warm_rounds + j
+                if j > 0:
+                    loop.harness(q - 1)                    # the target's tokens for the round just run
+                    lens_hist[j].copy_(loop.lens)
+                for r in range(min(R, K - j * R)):
+                    loop.launch(r, q * R + r, False)
+        snap = [(t, t.clone()) for t in (loop.lens, loop.vdraft, loop.vlen, loop.target, loop.mode,
+                                         loop.draft, loop.len, loop.score, loop.accept, loop.vp, loop.vq,
+                                         loop.vu, loop.vcand, loop.vclen, loop.vn, loop.ctarget)]
+
+        def restore():
+            for dst, src in snap:
+                dst.copy_(src)
+        lens_hist[0].copy_(loop.lens)
+        g.replay()                                         # first replay: graph upload + warm-up
+        cs.synchronize()
+    # A replay from the restored state repeats the same launches on the same inputs (tokens past a
+    # restored length are never read), so identical untimed replays can surround the timed one while the
+    # clocks are sampled.  The index keeps its inserts across replays: its leg is replayed once only.
+    replayable = search != "index"
+    barrier(world)
+    ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    sampler = ClockSampler(_gpu_uuid(torch.cuda.get_device_properties(dev))) if headline else None
+
+    def surround():
+        if sampler is None or not replayable:
+            return
+        t_end = time.perf_counter() + CLOCK_WINDOW_S
+        while time.perf_counter() < t_end:
+            restore()
+            l2_flush(flush)
+            g.replay()
+            cs.synchronize()
+
+    with torch.cuda.stream(cs):
+        surround()
+        if replayable:
+            restore()
+        elif True:
+            # the index's leg: its state after the first replay is the start of the timed one
+            lens_hist[0].copy_(loop.lens)
+        l2_flush(flush)
+        with nvtx_range(f"timed {base.name} {search} x{K}"):
+            ev0.record(cs)
+            g.replay()
+            ev1.record(cs)
+            ev1.synchronize()
+        lens_hist[rounds].copy_(loop.lens)
+        cs.synchronize()
+        surround()
+    clocks = sampler.stop() if sampler is not None else None
+    if clocks is not None:
+        clocks["window"] = (f"sampled over {2 * CLOCK_WINDOW_S:.1f} s of identical replays of the timed "
+                            "graph surrounding the timed replay")
+    region_s = ev0.elapsed_time(ev1) / 1e3
+    barrier(world)
+
+    # algorithmic bytes of every fused launch in the timed replay (lens after each round's append)
+    Lh = lens_hist.cpu().numpy().astype(np.int64).reshape(rounds + 1, R, B)
+    probe_bytes = 2 * B * d + (2 * d if wl.probe_kind == 0 else 2 * (wl.probe_hidden * d + wl.probe_hidden))
+    launch_bytes = []
+    for j in range(rounds):
+        n_this = min(R, K - j * R)
+        grow = (Lh[j + 1] - Lh[j])[:n_this]                # a + 1 per row
+        if np.any(grow <= 0):
+            raise SystemExit(f"timed graph round {j}: rows did not grow; the launches did not run")
+        ctx_read = 4 * Lh[j + 1][:n_this].sum(axis=1)
+        verify_rw = 8 * B + (28 if sampled else 16) * grow.sum(axis=1)
+        outputs = 12 * B + 4 * B * k                       # mode, len, score, draft (bound)
+        if cand_w > 0:
+            verify_rw = 8 * B + 4 * B * cand_w * (2 * cand_d + 2) + 4 * grow.sum(axis=1)
+            outputs = 12 * B + 4 * B * cand_w * (cand_d + 1)
+        if search == "index":
+            nn = wl.n_max - wl.n_min + 1
+            ctx_read = np.full(n_this, 4 * B * (32 + nn * (4 + 4 * wl.n_max)), np.int64) + \
+                12 * nn * grow.sum(axis=1)
+        launch_bytes.extend((ctx_read + probe_bytes + verify_rw + outputs).tolist())
+    launch_bytes = np.array(launch_bytes, dtype=np.float64)
+    per_launch_s = region_s / K
+    out = {"R": R, "cap": cap, "rounds": rounds, "region_s": region_s, "per_launch_s": per_launch_s,
+           "launch_bytes": float(launch_bytes.mean()), "clocks": clocks,
+           "mean_context_tokens": float(Lh[1:].mean()),
+           "scan_equivalent_gbs": float(4 * Lh[1:].sum(axis=2).mean() / per_launch_s / 1e9),
+           "ctx_bytes_all": R * B * cap * 4, "launches_per_step": 1 if wl.probe_kind == 0 else 2,
+           "harness_in_region": rounds - 1,
+           "value": replica_throughput(B * K, region_s, world),
+           "ms_per_step": reduce_max(region_s, world) / K * 1e3}
+
+    if headline and R >= 2 and search == "scan":
+        # warm L2, reported separately: K launches alternating between two batches only
+        with torch.cuda.stream(cs):
+            restore()
+            g2 = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(g2, stream=cs):
+                for i in range(K):
+                    loop.launch(i % 2, warm_rounds * R + i, False)
+            g2.replay()
+            cs.synchronize()
+            restore()
+            e2, e3 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e2.record(cs)
+            g2.replay()
+            e3.record(cs)
+            e3.synchronize()
+            restore()
+        us = e2.elapsed_time(e3) * 1e3 / K
+        out["l2_resident"] = {"launch_us": us, "value": B / (us * 1e-6), "unit": UNIT,
+                              "note": "L2-resident: K launches alternating between two batches "
+                                      f"({2 * B * cap * 4 / 2**20:.0f} MiB of contexts, inside L2); not the headline"}
+    if headline:
+        out["cold"] = cold_latency(loop, dev, cs, warm_rounds + rounds, l2)
+    if search == "scan" and cand_w == 0:
+        out["ceiling"] = read_ceiling(loop, d, K, warm_rounds * R, prefetch, cs, flush)
+    out["loop"] = loop
+    return out
+
+
+def roofline_of(m: dict, peaks: dict, kernel: str, traffic) -> dict:
+    achieved = m["launch_bytes"] / m["per_launch_s"] / 1e9
+    r = {"kernel": kernel, "bound": "hbm", "achieved": achieved, "peak": peaks["hbm_gbs"], "unit": "GB/s",
+         "frac": achieved / peaks["hbm_gbs"], "traffic": traffic,
+         "algorithmic_bytes_per_launch": m["launch_bytes"], "launch_us": m["per_launch_s"] * 1e6,
+         "duration": "timed region / K launches (CUDA events on the launching stream around one graph "
+                     "replay of the K launches)",
+         "peak_source": peaks["source"] + " hbm_gbs (copy)", "frac_nominal": achieved / NOMINAL_HBM_GBS}
+    c = m.get("ceiling")
+    if c is not None:
+        c = dict(c)
+        c["frac"] = c["achieved"] / peaks["hbm_gbs"]
+        c["step_time_ratio"] = c["launch_us"] / (m["per_launch_s"] * 1e6)
+        r["size_matched_ceiling"] = c
+    return r
+
+
+def l2_note(m: dict, B: int, l2: int) -> str:
+    if (m["R"] - 1) * B * m["cap"] * 4 < 2.2 * l2:
+        return (f"L2-resident: the whole workload ({m['R']} batches, {m['ctx_bytes_all'] / 2**20:.1f} MiB of "
+                "contexts) is below L2")
+    return (f"inputs larger than L2: {m['R']} independent batches of B={B} ({m['ctx_bytes_all'] / 2**20:.0f} MiB "
+            f"of contexts vs {l2 / 2**20:.0f} MiB L2), launch i reads batch i mod {m['R']}, L2 flushed before "
+            "the timed replay")
+
+
+PER_CONFIG = (("planted_copy", "scan"), ("uniform_8k", "scan"), ("code_16k", "scan"), ("mixed_128k", "scan"),
+              ("mixed_128k", "index"))
+
+
 def run_ours(args, world, rank, local):
     import torch
-    from paper_2609_20186_gb300 import Session, bf16_tensor, binding
+    from paper_2609_20186_gb300 import binding
 
     if not torch.cuda.is_available():
         raise SystemExit("bench.py needs a CUDA device (the controller has no CPU path)")
@@ -571,187 +787,81 @@ def run_ours(args, world, rank, local):
         cpu = cpu_baseline(base, args.cpu_seconds, sampled=args.verify == "sampled",
                            cand=(args.candidates, args.cand_len) if args.candidates > 0 else None)
 
-    # Replica batches: enough of them that the timed loop reads every batch from HBM.
-    R = choose_replicas(B * (base.L0 + 1024) * 4, l2, K)
-    rounds = -(-K // R)
-    warm_rounds = max(1, -(-W // R))
-    per_row_steps = warm_rounds + 2 * rounds + COLD_STEPS
-    wl = base.scaled(steps=per_row_steps)
-    cap = wl.cap
-    ctx1, lens1 = wl.contexts()
-    future1 = wl.future()
-    pw = wl.probe_weights()
-    n_launch = (warm_rounds + rounds) * R
-    hidden_host = np.empty((n_launch, B, d), np.uint16)
-    for i in range(n_launch):
-        hidden_host[i] = wl.hidden(i)
-    hidden = bf16_tensor(hidden_host, dev)
     cs = torch.cuda.Stream(dev)
-    loop = ReplicaLoop(wl, R, cap, ctx1, lens1, pw, future1, hidden, args.split, dev, cs,
-                       search=args.search, prefetch=not args.no_prefetch, sampled=args.verify == "sampled",
-                       cand_w=args.candidates, cand_d=args.cand_len)
-    ctx_bytes_all = R * B * cap * 4
-
-    with torch.cuda.stream(cs):
-        for q in range(warm_rounds):                       # eager warm-up rounds
-            loop.round(q, q == 0, q * R)
-        lens_hist = torch.zeros(rounds + 1, R * B, dtype=torch.int32, device=dev)
-        g = torch.cuda.CUDAGraph()
-        with torch.cuda.graph(g, stream=cs):
-            for j in range(rounds):
-                q = warm_rounds + j
-                lens_hist[j].copy_(loop.lens)
-                n_this = min(R, K - j * R)
-                for r in range(n_this):
-                    loop.launch(r, q * R + r, False)
-                loop.harness(q)
-            lens_hist[rounds].copy_(loop.lens)
-        g.replay()                                         # first replay: graph upload + warm-up
-        cs.synchronize()
-        # A replay is repeatable from a snapshot of the lengths and the verification inputs (tokens
-        # past a restored length are never read), so identical untimed replays can surround the timed
-        # one while the clocks are sampled.
-        snap = [(t, t.clone()) for t in (loop.lens, loop.vdraft, loop.vlen, loop.target, loop.mode,
-                                         loop.draft, loop.len, loop.score, loop.accept)]
-
-        def restore():
-            for dst, src in snap:
-                dst.copy_(src)
-    barrier(world)
-    ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    sampler = ClockSampler(_gpu_uuid(props))
-    with torch.cuda.stream(cs):
-        t_end = time.perf_counter() + CLOCK_WINDOW_S
-        while time.perf_counter() < t_end:
-            restore()
-            g.replay()
-            cs.synchronize()
-        restore()
-        ev0.record(cs)
-        g.replay()
-        ev1.record(cs)
-        ev1.synchronize()
-        t_end = time.perf_counter() + CLOCK_WINDOW_S
-        while time.perf_counter() < t_end:
-            restore()
-            g.replay()
-            cs.synchronize()
-    clocks = sampler.stop() or {"sm_mhz": None, "sm_max_mhz": None, "reasons": [], "samples": 0}
-    clocks["window"] = (f"sampled over {2 * CLOCK_WINDOW_S:.1f} s of identical replays of the timed "
-                        "graph surrounding the timed replay")
-    region_s = ev0.elapsed_time(ev1) / 1e3
-    barrier(world)
-    value = replica_throughput(B * K, region_s, world)
-    ms_per_step = reduce_max(region_s, world) / K * 1e3
-
-    # algorithmic bytes of every fused launch in the timed replay (lens after each round's append)
-    Lh = lens_hist.cpu().numpy().astype(np.int64).reshape(rounds + 1, R, B)
-    probe_bytes = 2 * B * d + (2 * d if wl.probe_kind == 0 else 2 * (wl.probe_hidden * d + wl.probe_hidden))
-    launch_bytes = []
-    for j in range(rounds):
-        n_this = min(R, K - j * R)
-        grow = (Lh[j + 1] - Lh[j])[:n_this]                # a + 1 per row
-        ctx_read = 4 * Lh[j + 1][:n_this].sum(axis=1)
-        # lens r/w; per tested position the draft and target (sampled: also p, q, u) read, the append
-        verify_rw = 8 * B + (28 if args.verify == "sampled" else 16) * grow.sum(axis=1)
-        outputs = 12 * B + 4 * B * k                       # mode, len, score, draft (bound)
-        if args.candidates > 0:
-            # the W candidates and the target's tokens for each are read by the verification; the
-            # candidates, their lengths and count written by the step (bounds)
-            Wc, Dc = args.candidates, args.cand_len
-            verify_rw = 8 * B + 4 * B * Wc * (2 * Dc + 2) + 4 * grow.sum(axis=1)
-            outputs = 12 * B + 4 * B * Wc * (Dc + 1)
-        if args.search == "index":
-            # index path: per row the context tail, and per n one head read and one candidate
-            # compare (at least), plus one head and chain write per appended position
-            nn = wl.n_max - wl.n_min + 1
-            ctx_read = np.full(n_this, 4 * B * (32 + nn * (4 + 4 * wl.n_max)), np.int64) + \
-                12 * nn * grow.sum(axis=1)
-        launch_bytes.extend((ctx_read + probe_bytes + verify_rw + outputs).tolist())
-    launch_bytes = np.array(launch_bytes, dtype=np.float64)
-    # Every fused launch appends at least one token per row: a timed region in which some row did not
-    # grow did not run its launches.
-    for j in range(rounds):
-        n_this = min(R, K - j * R)
-        if np.any(Lh[j + 1][:n_this] <= Lh[j][:n_this]):
-            raise SystemExit(f"timed graph round {j}: rows did not grow; the launches did not run")
+    flush = torch.empty(2 * l2 // 4, dtype=torch.float32, device=dev)
+    prefetch = not args.no_prefetch
+    sampled = args.verify == "sampled"
+    m = measure_loop(base, args, dev, cs, l2, W, K, args.split, args.search, prefetch, sampled,
+                     args.candidates, args.cand_len, world, headline=True, flush=flush)
     peaks = measured_peaks()
-    per_launch_s = region_s / K
-    achieved = float(launch_bytes.mean() / per_launch_s / 1e9)
     traffic = profiled_traffic(base.name)
-
-    # warm L2, reported separately: the same launches alternating between two batches only (their
-    # contexts stay in L2); replayed from the restored state, which is restored again afterwards
-    l2_res = None
-    if R >= 2 and args.search == "scan":  # (the index's tables would keep the leg's inserts)
-        with torch.cuda.stream(cs):
-            restore()
-            g2 = torch.cuda.CUDAGraph()
-            with torch.cuda.graph(g2, stream=cs):
-                for i in range(K):
-                    loop.launch(i % 2, (warm_rounds * R + i) % loop.hidden.shape[0], False)
-            g2.replay()                                      # upload + warm-up
-            cs.synchronize()
-            restore()
-            e2, e3 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-            e2.record(cs)
-            g2.replay()
-            e3.record(cs)
-            e3.synchronize()
-            restore()
-        us = e2.elapsed_time(e3) * 1e3 / K
-        l2_res = {"launch_us": us, "value": B / (us * 1e-6), "unit": UNIT,
-                  "note": "L2-resident: K launches alternating between two batches "
-                          f"({2 * B * cap * 4 / 2**20:.0f} MiB of contexts, inside L2); not the headline"}
-
-    # cold single-launch latency: L2 flushed, one event-bracketed fused launch on batch 0
-    cold = cold_latency(loop, dev, cs, warm_rounds + rounds, l2)
-
-    ceiling = None
-    if args.search == "scan":
-        ceiling = read_ceiling(loop, d, K, warm_rounds * R, not args.no_prefetch, cs)
-        ceiling["frac"] = ceiling["achieved"] / peaks["hbm_gbs"]
-        ceiling["step_time_ratio"] = ceiling["launch_us"] / (per_launch_s * 1e6)
+    roof = roofline_of(m, peaks, "switchsd_verify_step" + (" (index)" if args.search == "index" else ""),
+                       traffic)
 
     e2e = None
     if not args.no_e2e and args.candidates == 0:  # the public-API loop covers the single-draft step
-        e2e = run_e2e(base, dev, W, K, args.split, world, prefetch=not args.no_prefetch,
-                      sampled=args.verify == "sampled")
+        with nvtx_range("e2e"):
+            e2e = run_e2e(base, dev, W, K, args.split, world, prefetch=prefetch, sampled=sampled)
+
+    head = m
+    loops = [head.pop("loop")]
+    # The other workloads of the suite, each measured the same way (same K and W), in the same line.
+    per_config = None
+    if not args.no_per_config and args.workload == "zipf_32k" and args.candidates == 0 and not sampled:
+        per_config = {}
+        for name, search in PER_CONFIG:
+            loops.clear()
+            torch.cuda.synchronize()
+            torch.cuda.empty_cache()
+            wb = synth.get_workload(name)
+            mc = measure_loop(wb, args, dev, cs, l2, W, K, args.split, search, prefetch, False, 0, 20, world,
+                              flush=flush)
+            mc.pop("loop")
+            entry = {"value": mc["value"], "unit": UNIT, "ms_per_step": mc["ms_per_step"],
+                     "B": wb.B, "L0": wb.L0, "k": wb.k, "d": wb.d, "n_min": wb.n_min, "n_max": wb.n_max,
+                     "probe": "linear" if wb.probe_kind == 0 else f"mlp{wb.d}x{wb.probe_hidden}",
+                     "search": search, "launches_per_step": mc["launches_per_step"],
+                     "l2": l2_note(mc, wb.B, l2)}
+            if search == "index":
+                entry["scan_equivalent_gbs"] = mc["scan_equivalent_gbs"]
+                entry["launch_us"] = mc["per_launch_s"] * 1e6
+                entry["roofline"] = None
+                entry["note"] = ("the index reads the context tail and its hash tables, not the context: its "
+                                 "bytes are not the scan's, so it has no HBM roofline; scan_equivalent_gbs = "
+                                 "the context bytes a rescan would read over the same time (effective, not "
+                                 "achieved)")
+            else:
+                entry["roofline"] = roofline_of(mc, peaks, "switchsd_verify_step" +
+                                                (" + two-layer probe kernel" if wb.probe_kind else ""), None)
+            if not args.no_e2e and search == "scan":
+                entry["e2e"] = run_e2e(wb, dev, W, K, args.split, world, prefetch=prefetch)
+            per_config[name + ("_index" if search == "index" else "")] = entry
+    loops.clear()
 
     if rank != 0:
         return
     line = {
-        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": K, "warmup": W,
-        "ms_per_step": ms_per_step, "higher_is_better": True, "scaling": "weak",
+        "metric": METRIC, "value": head["value"], "unit": UNIT, "n_gpus": world, "steps": K, "warmup": W,
+        "ms_per_step": head["ms_per_step"], "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "dtype": "int32 (search/verify), bf16 in / fp32 accumulate (probe)",
         "data": "synthetic",
-        "config": dict(config_of(base, world, args.split, args.search, not args.no_prefetch, args.verify,
-                                 args.candidates, args.cand_len),
-                       replicas=R,
-                       l2=f"inputs larger than L2: {R} independent batches of B={B} "
-                          f"({ctx_bytes_all / 2**20:.0f} MiB of contexts vs {l2 / 2**20:.0f} MiB L2), "
-                          f"launch i reads batch i mod {R}"),
-        "roofline": {"kernel": "switchsd_verify_step" + (" (index)" if args.search == "index" else ""),
-                     "bound": "hbm", "achieved": achieved,
-                     "peak": peaks["hbm_gbs"], "unit": "GB/s", "frac": achieved / peaks["hbm_gbs"],
-                     "traffic": traffic,
-                     "algorithmic_bytes_per_launch": float(launch_bytes.mean()),
-                     "launch_us": per_launch_s * 1e6,
-                     "duration": "timed region / K launches (the region also holds one target "
-                                 "stand-in launch and one 4 KB length snapshot per round)",
-                     "peak_source": peaks["source"] + " hbm_gbs (copy)",
-                     "frac_nominal": achieved / NOMINAL_HBM_GBS,
-                     "size_matched_ceiling": ceiling},
-        "controller": {"cold_single_launch_us": cold, "l2_resident": l2_res, "search": args.search,
-                       "scan_equivalent_gbs": float(4 * Lh[1:].sum(axis=2).mean() / per_launch_s / 1e9),
-                       "mean_context_tokens": float(Lh[1:].mean()),
-                       "launches_per_step": 1 if wl.probe_kind == 0 else 2},
-        "gpu_launches": K * (1 if wl.probe_kind == 0 else 2) + rounds,
-        "gpu_launches_note": "switchsd_verify_step launches (plus the two-layer probe kernel when "
-                             "used) and one target stand-in launch per round, all in one CUDA graph",
-        "clocks": clocks,
+        "config": config_of(base, world, args.split, args.search, prefetch, args.verify,
+                            args.candidates, args.cand_len),
+        "roofline": roof,
+        "controller": {"protocol": l2_note(head, B, l2), "replicas": head["R"],
+                       "cold_single_launch_us": head.get("cold"), "l2_resident": head.get("l2_resident"),
+                       "search": args.search, "scan_equivalent_gbs": head["scan_equivalent_gbs"],
+                       "mean_context_tokens": head["mean_context_tokens"],
+                       "launches_per_step": head["launches_per_step"],
+                       "target_standin_launches_in_timed_region": head["harness_in_region"]},
+        "gpu_launches": K * head["launches_per_step"] + 2 * head["harness_in_region"],
+        "gpu_launches_note": "fused controller launches (switchsd_verify_step; plus the two-layer probe kernel "
+                             "when used) in one CUDA graph, and, when K exceeds the replica count, one target "
+                             "stand-in launch and one length snapshot per extra round",
+        "clocks": head["clocks"],
         "e2e": e2e,
         "cpu_baseline": cpu,
+        "per_config": per_config,
     }
     print(json.dumps(line), flush=True)
 
@@ -793,10 +903,11 @@ def cold_latency(loop, dev, cs, step_base, l2) -> dict:
             "note": "includes the ~2.2 us event-pair and ~2.2 us stream launch overhead of this GPU"}
 
 
-def read_ceiling(loop, d: int, K: int, step_base: int, prefetch: bool, cs) -> dict:
+def read_ceiling(loop, d: int, K: int, step_base: int, prefetch: bool, cs, flush) -> dict:
     """The size-matched ceiling: switchsd_harness_read -- a plain read of each launch's contexts and
     hidden states and nothing else -- in the timed graph's launch order (K launches, launch i on batch
-    i mod R, programmatic dependent launch), best of a few CTA splits per row."""
+    i mod R, programmatic dependent launch, L2 flushed before the timed replay), best of a few CTA splits
+    per row."""
     import torch
     R, B, cap = loop.R, loop.B, loop.cap
     nh = loop.hidden.shape[0]
@@ -816,14 +927,14 @@ def read_ceiling(loop, d: int, K: int, step_base: int, prefetch: bool, cs) -> di
                 raise RuntimeError(f"switchsd_harness_read failed: {code}")
 
     best = None
-    for split in (4, 8, 16, 32):
+    for split in (2, 4, 8, 16):
         g = torch.cuda.CUDAGraph()
         with torch.cuda.stream(cs):
             enqueue(split)                                  # eager warm-up
             with torch.cuda.graph(g, stream=cs):
                 enqueue(split)
             g.replay()
-            cs.synchronize()
+            l2_flush(flush)
             e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
             e0.record(cs)
             g.replay()
@@ -835,8 +946,9 @@ def read_ceiling(loop, d: int, K: int, step_base: int, prefetch: bool, cs) -> di
     us, split = best
     return {"kernel": "switchsd_harness_read", "launch_us": us, "achieved": nbytes / us / 1e3,
             "bytes_per_launch": nbytes, "split": split, "prefetch": bool(prefetch),
-            "note": "plain 16-byte loads of every launch's context tokens and hidden states, same graph, "
-                    "launch order and inputs larger than L2; best of splits 4, 8, 16, 32"}
+            "note": "bulk copies of every launch's context tokens and hidden states into shared memory, "
+                    "folded, and nothing else; same graph, launch order, replica batches and L2 flush; "
+                    "best of splits 2, 4, 8, 16"}
 
 
 def run_e2e(base, dev, W, K, split, world, prefetch=True, sampled=False):

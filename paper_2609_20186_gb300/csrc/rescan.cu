@@ -1,0 +1,519 @@
+// rescan.cu -- the rescan kernel: switchsd_step / switchsd_verify_step / switchsd_verify_sampled_step with
+// the linear probe (Eq. 3), laid out for a short chain of dependent phases after the grid-dependency
+// wait.
+//
+// Paper: §3.3 (kappa-gram gate, recency-ranked copy candidates, Eq. 4 decision rule, parallel
+// verification), Eq. 3 (linear probe), Fig. 1 (three cases).
+//
+// Row b is handled by a cluster of C CTAs of kRescanThreads threads (grid = C x B).  The row's old
+// candidate ends [0, L_old - 1) are split into C contiguous 16-byte-aligned ranges; each CTA stages its
+// range (plus kHalo tokens of look-back and kFwd of look-ahead) with one bulk copy, and the row's last
+// kHalo tokens with another, as soon as it has read the row length -- before the grid-dependency wait
+// when the caller allows it.  The CTAs are small (four warps, at most 72 registers a thread) so that the
+// next launch's CTAs are resident, with their copies in flight, while this launch finishes.
+//
+// After the wait there is no CTA-wide or cluster-wide barrier on the path:
+//  * every warp verifies the previous draft itself (the draft and the target are a few L2 lines), and
+//    keeps its own window of the row's last kHalo old tokens followed by the appended tokens: the new
+//    suffix and the appended positions come from it, so the staged tile is never patched;
+//  * every warp scans its share of the CTA's old ends (first-token filter, then the second token, then
+//    a backward compare against its suffix window), and the leader's warp 0 also tests the a+1 ends the
+//    append creates;
+//  * every warp ships its best key, its share of the probe's dot product and its best match's
+//    continuation (from the staged tile, or from its window past the old length) to the row's leader CTA
+//    (the last one) with asynchronous DSMEM stores completing on the leader's mbarrier, and is done.
+// The leader's warp 0 publishes the append, waits (bounded) for the C x kRescanWarps messages, reduces
+// them in a fixed order and writes the outputs.  The only cluster barrier is arrived on right after the
+// length read and waited on just before the first message, so the leader's message barrier is
+// initialised before anyone ships to it and no CTA reads the length after the leader rewrites it.
+#include "step.cuh"
+
+namespace switchsd {
+
+// Per-warp window of y = old context followed by the append: s_y[w][j] = y[L_old - kHalo + j].
+constexpr int kYLen = kHalo + SWITCHSD_KMAX + 4;
+// 32-bit match keys: m << kKeyShift | e with m <= SWITCHSD_NMAX (bits 25..30) and e < 2^25; bit 31 alone
+// marks a copy that did not land.
+constexpr int kKeyShift = 25;
+constexpr uint32_t kKeyEndMask = (1u << kKeyShift) - 1u;
+constexpr uint32_t kKeyTimeout = 1u << 31;
+static_assert(SWITCHSD_NMAX < (1 << (31 - kKeyShift)), "m must fit below the timeout bit");
+// The scan: kScanWords words per thread per round; a thread's rounds of a CTA range fit the 32 bits of its
+// pass mask.
+constexpr int kScanWords = 4;
+static_assert(kRescanTileMax / 4 / (kScanWords * kRescanThreads) <= 32, "a thread's rounds fit its pass mask");
+
+// The scan of a CTA's old ends [e_lo, e_end) against the new suffix (suf[-q] = its q-th token from the end)
+// for the longest-then-most-recent match: the largest key m << kKeyShift | e over the ends with
+// m(e) >= n_min, 0 if none.  stage[kHalo + p - e_lo] = x[p] over [e_lo - kHalo, e_end + kFwd).
+//
+// Filter depth F = min(n_min, 3): end e passes when its last F tokens equal the suffix's, i.e.
+// t(e) = (x[e] ^ s0) | (x[e-1] ^ s1) | (x[e-2] ^ s2) (its first F terms) is 0.  Exact: every end with
+// m(e) >= n_min >= F passes.  Each token's x ^ s1 and x ^ s2 serve the next two ends, so an end costs an
+// xor per term and a three-input logic op, and a running three-input min tests a round together.
+//
+// Pass 1: rounds of kScanWords words per thread (word g0 + u kT, g0 = tid + kScanWords kT r; consecutive
+// lanes hold consecutive words, so the two tokens before a word are the previous lane's last two -- lane 0
+// loads them; unset before position 0, where lim < F drops the end); a round with an end that passes only
+// sets its bit.  No branch and no backward compare in the hot loop.
+// Pass 2 (rare): the rounds that passed, in warp-synchronous steps (each step every lane with a round left
+// takes its next one, so the compares of a hot suffix run side by side), reloaded from shared memory;
+// their passing ends take the backward compare from m = F, eight positions per step with independent
+// loads.
+template <int F>
+__device__ __forceinline__ uint32_t scan_ends(const int32_t *stage, int32_t e_lo, int32_t e_end, const int32_t *suf,
+                                              int32_t n_min, int32_t n_max, int tid, int lane) {
+    const int32_t s0 = suf[0], s1 = F >= 2 ? suf[-1] : 0, s2 = F >= 3 ? suf[-2] : 0;
+    const int32_t n4 = (e_end - e_lo + 3) >> 2;
+    const int4 *g4 = reinterpret_cast<const int4 *>(stage + kHalo);
+    const int32_t off = kHalo - e_lo;
+    // t of the four ends of word v, given the two tokens before it (pz = x[4g - 2], pw = x[4g - 1])
+    auto filter4 = [&](const int4 &v, int32_t pz, int32_t pw, uint32_t (&t)[4]) {
+        t[0] = uint32_t(v.x ^ s0);
+        t[1] = uint32_t(v.y ^ s0);
+        t[2] = uint32_t(v.z ^ s0);
+        t[3] = uint32_t(v.w ^ s0);
+        if (F >= 2) {
+            t[0] |= uint32_t(pw ^ s1);
+            t[1] |= uint32_t(v.x ^ s1);
+            t[2] |= uint32_t(v.y ^ s1);
+            t[3] |= uint32_t(v.z ^ s1);
+        }
+        if (F >= 3) {
+            t[0] |= uint32_t(pz ^ s2);
+            t[1] |= uint32_t(pw ^ s2);
+            t[2] |= uint32_t(v.x ^ s2);
+            t[3] |= uint32_t(v.y ^ s2);
+        }
+    };
+    uint32_t passed = 0u;
+    int rnd = 0;
+    for (int32_t g0 = tid; g0 - lane < n4; g0 += kScanWords * kRescanThreads, ++rnd) {
+        int4 v[kScanWords];
+        int2 pv[kScanWords];
+#pragma unroll
+        for (int u = 0; u < kScanWords; ++u) {
+            const int32_t g = g0 + u * kRescanThreads;
+            v[u] = g < n4 ? g4[g] : make_int4(0, 0, 0, 0);
+            pv[u] = (F >= 2 && lane == 0 && g < n4) ? *reinterpret_cast<const int2 *>(stage + kHalo + 4 * g - 2)
+                                                     : make_int2(0, 0);
+        }
+        uint32_t mn = 0xffffffffu;
+#pragma unroll
+        for (int u = 0; u < kScanWords; ++u) {
+            if (F >= 2) {
+                const int32_t uw = __shfl_up_sync(kFull, v[u].w, 1);
+                const int32_t uz = F >= 3 ? __shfl_up_sync(kFull, v[u].z, 1) : 0;
+                if (lane > 0) pv[u] = make_int2(uz, uw);
+            }
+            uint32_t t[4];
+            filter4(v[u], pv[u].x, pv[u].y, t);
+            mn = __vimin3_u32(mn, __vimin3_u32(t[0], t[1], t[2]), t[3]);
+        }
+        passed |= uint32_t(mn == 0u) << (rnd & 31);
+    }
+    uint32_t mine = 0u;
+    while (__any_sync(kFull, passed != 0u)) {
+        if (passed == 0u) continue;
+        const int r = __ffs(passed) - 1;
+        passed &= passed - 1u;
+#pragma unroll 1
+        for (int u = 0; u < kScanWords; ++u) {
+            const int32_t g = tid + r * kScanWords * kRescanThreads + u * kRescanThreads;
+            if (g >= n4) break;
+            const int2 pv = *reinterpret_cast<const int2 *>(stage + kHalo + 4 * g - 2);
+            uint32_t t[4];
+            filter4(g4[g], pv.x, pv.y, t);
+            uint32_t hall = uint32_t(t[0] == 0u) | (uint32_t(t[1] == 0u) << 1) | (uint32_t(t[2] == 0u) << 2) |
+                            (uint32_t(t[3] == 0u) << 3);
+            while (hall) {
+                const int j = __ffs(hall) - 1;
+                hall &= hall - 1;
+                const int32_t e = e_lo + 4 * g + j;
+                if (e >= e_end) break;
+                const int32_t lim = min(n_max, e + 1);
+                if (lim < F) continue;  // the filter read a token before position 0
+                // m(e) from F: x[e - q] against suf[-q], eight positions per step, every load issued
+                // unconditionally (q clamped to lim - 1; the sentinel bit ends the run at the count)
+                int32_t m = F;
+#pragma unroll 1
+                while (m < lim) {
+                    const int32_t cnt = min(8, lim - m);
+                    unsigned miss = 1u << cnt;
+#pragma unroll
+                    for (int i = 0; i < 8; ++i) {
+                        const int32_t q = min(m + i, lim - 1);
+                        miss |= unsigned(stage[off + e - q] != suf[-q]) << i;
+                    }
+                    const int32_t run = __ffs(miss) - 1;
+                    m += run;
+                    if (run < cnt) break;
+                }
+                if (m >= n_min) {
+                    const uint32_t key = (uint32_t(m) << kKeyShift) | uint32_t(e);
+                    mine = key > mine ? key : mine;
+                }
+            }
+        }
+    }
+    return mine;
+}
+
+template <bool kSampled>
+__global__ void __launch_bounds__(kRescanThreads, kRescanMinBlocks) rescan_kernel(const StepArgs a) {
+    extern __shared__ __align__(128) int32_t dsm[];
+    __shared__ __align__(8) uint64_t bars[4];              // tile, tail, probe slices, messages (leader)
+    __shared__ __align__(16) int32_t s_tail[kHalo + 8];    // x[tail_lo .. L_old), tail_lo = roundown4(L_old - kHalo)
+    __shared__ int32_t s_y[kRescanWarps][kYLen];
+
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    const uint32_t rank = cluster_ctarank();
+    const uint32_t C = cluster_nctarank();
+    const uint32_t lead = C - 1;
+    const int b = blockIdx.y;
+    const int stage_ints = kHalo + a.tile + kFwd;
+    int32_t *stage = dsm;
+    uint4 *s_pw = reinterpret_cast<uint4 *>(dsm + ((stage_ints + 3) & ~3));
+    uint4 *s_ph = s_pw + a.probe_words;
+    unsigned char *msgs = reinterpret_cast<unsigned char *>(s_ph + a.probe_words);
+    const bool verifying = a.pv_len != nullptr;
+    const int kw = (a.k + 3) >> 2;                          // 16-byte words of a message's continuation
+    const uint32_t slot_bytes = 16u * uint32_t(1 + kw);
+    const int nmsg = int(C) * kRescanWarps;
+
+    if (tid == 0) {
+        mbar_init(&bars[0], 1);
+        mbar_init(&bars[1], 1);
+        mbar_init(&bars[2], 1);
+        if (rank == lead) {
+            mbar_init(&bars[3], 1);
+            mbar_arrive_expect_tx(&bars[3], slot_bytes * uint32_t(nmsg));
+        }
+        fence_mbar_init();
+    }
+    __syncthreads();  // the barriers are initialised before any thread arms or waits on one
+
+    const bool pf_ctx = (a.prefetch & SWITCHSD_PREFETCH_CONTEXT) != 0;
+    const bool gather = verifying && a.hidden_rows > 1;
+    const bool pf_probe = (a.prefetch & SWITCHSD_PREFETCH_PROBE) != 0 && !gather;
+    if (!pf_ctx) pdl_wait();
+    int32_t *row = a.ctx + size_t(b) * size_t(a.cap);
+    // The CTA's ends are split on the row's old length, or, with a length bound, on the bound: its tile
+    // copy then leaves before the length is read, and a row longer than the bound is a bad length.
+    const bool bounded = a.len_bound > 0;
+    auto range_of = [&](int32_t E, int32_t &e_lo_, int32_t &e_hi_) {
+        int32_t chunk = (E + int32_t(C) - 1) / int32_t(C);
+        chunk = (chunk + 3) & ~3;
+        e_lo_ = min(E, int32_t(rank) * chunk);
+        e_hi_ = min(E, e_lo_ + chunk);
+    };
+    int32_t e_lo = 0, e_hi = 0, lo = 0;
+    if (bounded) {
+        range_of(a.len_bound - 1, e_lo, e_hi);
+        lo = max(0, e_lo - kHalo);
+    }
+    auto tile_hi = [&]() { return e_hi > e_lo ? min((e_hi + kFwd + 3) & ~3, a.cap) : lo; };
+    const uint64_t pol = l2_evict_first_policy();
+    auto issue_tile = [&](int32_t hi_) {  // positions [lo, hi_) land at stage[kHalo + p - e_lo]
+        const uint32_t bytes = uint32_t(hi_ - lo) * 4u;
+        mbar_expect_tx_relaxed(&bars[0], bytes);
+        if (bytes > 0) bulk_g2s_hint(stage + (kHalo + lo - e_lo), row + lo, bytes, &bars[0], pol);
+    };
+    if (bounded && tid == 0) issue_tile(tile_hi());
+    // Every thread reads the length itself (one L2 request per warp), then arrives on the cluster
+    // barrier with release: the leader rewrites the length only after waiting on it.
+    const int32_t L_old = __ldcg(a.lens + b);
+    cluster_arrive_release();
+    const bool len_ok = L_old >= 1 && L_old <= (bounded ? a.len_bound : a.cap);
+    const int32_t E_old = len_ok ? L_old - 1 : 0;
+    if (!bounded) {
+        range_of(E_old, e_lo, e_hi);
+        lo = max(0, e_lo - kHalo);
+    }
+    const int32_t hi = tile_hi();                       // the staged positions end here
+    const int32_t e_end = max(e_lo, min(e_hi, E_old));  // the old ends scanned: [e_lo, e_end)
+    const int32_t tail_lo = max(0, (L_old - kHalo) & ~3);
+    const int32_t tail_hi = len_ok ? (L_old + 3) & ~3 : tail_lo;  // <= cap since cap % 4 == 0
+
+    // Linear probe: this CTA's slice is words [v0, v1) of 8 bf16; the first probe_words of w and h are
+    // staged by bulk copies, the rest read directly.  Warps 1.. compute it (warp 0 issues the copies and
+    // releases the next launch).
+    const int nv = a.d >> 3;
+    const int vper = (nv + int(C) - 1) / int(C);
+    const int v0 = min(nv, int(rank) * vper), v1 = min(nv, v0 + vper);
+    const int v_staged = gather ? 0 : min(v1 - v0, a.probe_words);
+    const uint4 *w4 = reinterpret_cast<const uint4 *>(a.probe_w);
+    const uint4 *h4 = reinterpret_cast<const uint4 *>(a.hidden + size_t(b) * size_t(gather ? a.hidden_rows : 1) *
+                                                                  size_t(a.d));
+    auto issue_probe = [&]() {
+        const uint32_t pb = uint32_t(v_staged) * 16u;
+        mbar_expect_tx_relaxed(&bars[2], 2u * pb);
+        if (pb > 0) {
+            bulk_g2s(s_pw, w4 + v0, pb, &bars[2]);
+            bulk_g2s(s_ph, h4 + v0, pb, &bars[2]);
+        }
+    };
+    if (tid == 0) {
+        const uint32_t tb = uint32_t(tail_hi - tail_lo) * 4u;
+        mbar_expect_tx_relaxed(&bars[1], tb);
+        if (tb > 0) bulk_g2s_hint(s_tail, row + tail_lo, tb, &bars[1], pol);
+        if (pf_probe) issue_probe();
+        if (!bounded) issue_tile(hi);
+        // The parameters only the leader's last phase reads are fetched now, so that phase does not wait
+        // on the constant cache.
+        asm volatile("" ::"l"(a.out_mode), "l"(a.out_len), "l"(a.out_score), "l"(a.out_match_n), "l"(a.out_match_end),
+                     "l"(a.status), "l"(a.out_draft), "l"(a.out_accept), "r"(a.kappa), "f"(a.logit_tau));
+    }
+    float zp = 0.f;
+    bool probe_ok = true;
+    auto probe_dot = [&](const uint4 *h) {  // warps 1..: thread j = tid - 32 takes words j, j + kT - 32, ...
+        if (v_staged > 0) {
+            probe_ok = mbar_wait(&bars[2], 0);
+            if (probe_ok)
+                for (int i = tid - kWarp; i < v_staged; i += kRescanThreads - kWarp) zp = dot8_bf16(s_pw[i], s_ph[i], zp);
+        }
+        for (int v = v0 + v_staged + tid - kWarp; v < v1; v += kRescanThreads - kWarp)
+            zp = dot8_bf16(__ldg(w4 + v), __ldg(h + v), zp);
+    };
+    // A prefetched probe is finished before the wait by warps 1.. (its inputs are not written by the
+    // preceding kernel); warp 0 goes straight to the wait and releases the next launch.
+    if (pf_probe && warp >= 1) probe_dot(h4);
+    if (pf_ctx) pdl_wait();
+    pdl_trigger();
+    if (!pf_probe && !gather && tid == 0) issue_probe();
+
+    // ---- verification of the previous draft (every warp) ----
+    int32_t acc = -1, L = L_old, vst = len_ok ? SWITCHSD_ROW_OK : SWITCHSD_ROW_BAD_LEN;
+    int32_t d_lo = 0, d_hi = 0, t_acc = 0;
+    if (verifying && len_ok) {
+        const int32_t *dr = a.pv_draft + size_t(b) * a.k;
+        const int32_t *tg = a.pv_target + size_t(b) * (a.k + 1);
+        const int32_t pv_n = a.pv_len[b];
+        d_lo = lane < a.k ? dr[lane] : 0;
+        d_hi = lane + 32 < a.k ? dr[lane + 32] : 0;
+        const int32_t t_lo = lane <= a.k ? tg[lane] : 0;
+        const int32_t t_hi = lane + 32 <= a.k ? tg[lane + 32] : 0;
+        const int32_t t_top = (lane == 0 && a.k >= 64) ? tg[64] : 0;
+        if (pv_n < 0 || pv_n > a.k) {
+            vst = SWITCHSD_ROW_BAD_LEN;
+        } else {
+            bool rej_lo, rej_hi;
+            if (kSampled) {
+                // T > 0: draft token i is rejected when u_i * q_i (binary32) is not below p_i
+                const size_t o = size_t(b) * a.k;
+                rej_lo = lane < pv_n &&
+                         !(__fmul_rn(a.pv_u[o + lane], a.pv_q ? a.pv_q[o + lane] : 1.f) < a.pv_p[o + lane]);
+                rej_hi = lane + 32 < pv_n &&
+                         !(__fmul_rn(a.pv_u[o + lane + 32], a.pv_q ? a.pv_q[o + lane + 32] : 1.f) < a.pv_p[o + lane + 32]);
+            } else {
+                rej_lo = lane < pv_n && d_lo != t_lo;
+                rej_hi = lane + 32 < pv_n && d_hi != t_hi;
+            }
+            const unsigned m_lo = __ballot_sync(kFull, rej_lo);
+            const unsigned m_hi = __ballot_sync(kFull, rej_hi);
+            const int32_t at = m_lo ? __ffs(m_lo) - 1 : (m_hi ? 32 + __ffs(m_hi) - 1 : pv_n);
+            if (L_old + at + 1 > a.cap) {
+                vst = SWITCHSD_ROW_CAPACITY;
+            } else {
+                acc = at;
+                t_acc = __shfl_sync(kFull, acc < 32 ? t_lo : (acc < 64 ? t_hi : t_top), acc & 31);
+                L = L_old + acc + 1;
+            }
+        }
+    }
+    // The probed state of a fused verification with hidden_rows = k + 1: row a_b (row 0 when nothing was
+    // appended).  Its words are loaded now and used after the scan.
+    uint4 gw = make_uint4(0, 0, 0, 0), gh = make_uint4(0, 0, 0, 0);
+    if (gather) {
+        h4 += size_t(acc > 0 ? acc : 0) * size_t(nv);
+        const int v = v0 + tid - kWarp;
+        if (warp >= 1 && v < v1) {
+            gw = __ldg(w4 + v);
+            gh = __ldg(h4 + v);
+        }
+    }
+
+    // ---- this warp's window: y[L_old - kHalo + j], the old tail then the appended tokens ----
+    const bool tail_in = tail_hi == tail_lo || mbar_wait(&bars[1], 0);
+    int32_t *y = s_y[warp];
+    {
+        const int32_t p = L_old - kHalo + lane;
+        y[lane] = (len_ok && p >= 0 && tail_in) ? s_tail[p - tail_lo] : 0;
+        if (acc >= 0) {
+            if (lane < acc) y[kHalo + lane] = d_lo;
+            if (lane + 32 < acc) y[kHalo + 32 + lane] = d_hi;
+            if (lane == 0) y[kHalo + acc] = t_acc;
+        }
+    }
+    __syncwarp();
+    const int32_t *suf = y + kHalo + acc;  // suf[-m] = the m-th token from the end of the new context
+    const int32_t n_max = a.n_max, n_min = a.n_min;
+
+    // ---- scan of this warp's share of the CTA's old ends ----
+    // key = m << kKeyShift | e (e < 2^kKeyShift, m <= 32): the largest key is the longest match, then the
+    // most recent; 0 = no match; kKeyTimeout marks a copy that did not land.
+    uint32_t mine = 0;
+    const bool tile_in = hi == lo || mbar_wait(&bars[0], 0);
+    bool timed_out = !tail_in || !tile_in;
+    const int32_t off = kHalo - e_lo;  // stage[off + p] = x[p] over the staged range
+    if (!timed_out && len_ok && L >= 2) {
+        // (n_min is uniform over the launch: one instance runs)
+        mine = a.n_min >= 3 ? scan_ends<3>(stage, e_lo, e_end, suf, n_min, n_max, tid, lane)
+                            : (a.n_min == 2 ? scan_ends<2>(stage, e_lo, e_end, suf, n_min, n_max, tid, lane)
+                                            : scan_ends<1>(stage, e_lo, e_end, suf, n_min, n_max, tid, lane));
+        // The ends the append creates, [L_old - 1, L - 1), lie in the window: the leader's warp 0.
+        if (rank == lead && warp == 0 && acc >= 0) {
+#pragma unroll 1
+            for (int32_t j = lane; j <= acc; j += kWarp) {
+                const int32_t e = L_old - 1 + j;
+                const int32_t lim = min(n_max, e + 1);
+                int32_t m = 0;
+#pragma unroll 1
+                while (m < lim && y[kHalo - 1 + j - m] == suf[-m]) ++m;
+                if (m >= n_min) {
+                    const uint32_t key = (uint32_t(m) << kKeyShift) | uint32_t(e);
+                    mine = key > mine ? key : mine;
+                }
+            }
+        }
+    }
+    uint32_t key = __reduce_max_sync(kFull, mine);
+    if (timed_out) key = kKeyTimeout;
+
+    // ---- probe share (unless finished before the wait) ----
+    if (warp >= 1) {
+        if (gather) {
+            zp = dot8_bf16(gw, gh, 0.f);  // zero words for a thread past the slice
+            for (int v = v0 + tid - kWarp + (kRescanThreads - kWarp); v < v1; v += kRescanThreads - kWarp)
+                zp = dot8_bf16(__ldg(w4 + v), __ldg(h4 + v), zp);
+        } else if (!pf_probe) {
+            probe_dot(h4);
+        }
+    }
+    if (!probe_ok) key = kKeyTimeout;
+    const float z_w = warp_sum_f32(zp);
+
+    // ---- the continuation of this warp's best match: lane j (1..kw) gathers tokens 4(j-1) .. +3 ----
+    uint4 cw = make_uint4(0, 0, 0, 0);
+    if (key != 0u && key != kKeyTimeout && lane >= 1 && lane <= kw) {
+        const int32_t e = int32_t(key & kKeyEndMask);
+        const int32_t len = min(a.k, L - 1 - e);
+        int32_t t4[4];
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+            const int32_t i = 4 * (lane - 1) + q;
+            const int32_t p = e + 1 + i;
+            t4[q] = i < len ? (p < L_old ? stage[off + p] : y[kHalo + p - L_old]) : 0;
+        }
+        cw = make_uint4(uint32_t(t4[0]), uint32_t(t4[1]), uint32_t(t4[2]), uint32_t(t4[3]));
+    }
+
+    // ---- ship to the leader ----
+    cluster_wait_acquire();  // every CTA has read the length and the leader's barrier is initialised
+    const uint32_t done_addr = map_to_rank(&bars[3], lead);
+    unsigned char *slot = msgs + size_t(rank * kRescanWarps + warp) * slot_bytes;
+    if (lane == 0) {
+        uint4 h;
+        h.x = key;
+        h.y = __float_as_uint(z_w);
+        h.z = 0u;
+        h.w = 0u;
+        st_async_v4(map_to_rank(slot, lead), h, done_addr);
+    } else if (lane <= kw) {
+        st_async_v4(map_to_rank(slot + 16 * lane, lead), cw, done_addr);
+    }
+    if (rank != lead || warp != 0) {
+        if (timed_out && lane == 0) {  // copies still in flight get a second bounded wait
+            (void)mbar_wait(&bars[0], 0);
+            (void)mbar_wait(&bars[1], 0);
+        }
+        if (!probe_ok && lane == 0) (void)mbar_wait(&bars[2], 0);
+        return;
+    }
+
+    // ---- leader, warp 0: the append, then the row's answer ----
+    if (verifying) {
+        for (int32_t i = lane; i <= acc; i += kWarp) row[L_old + i] = y[kHalo + i];
+        if (lane == 0 && len_ok) {
+            a.lens[b] = L;
+            a.out_accept[b] = acc;
+        }
+    }
+    const bool all_in = __all_sync(kFull, mbar_wait(&bars[3], 0));
+    uint32_t k_r = 0u;
+    int32_t i_r = 0;
+    float z_r = 0.f;
+    if (all_in) {
+        for (int i = lane; i < nmsg; i += kWarp) {  // lane j: messages j, j + 32, ... in order
+            const uint2 hv = *reinterpret_cast<const uint2 *>(msgs + size_t(i) * slot_bytes);
+            z_r += __uint_as_float(hv.y);
+            if (hv.x > k_r) {
+                k_r = hv.x;
+                i_r = i;
+            }
+        }
+    }
+    const uint32_t best = all_in ? __reduce_max_sync(kFull, k_r) : kKeyTimeout;
+    const unsigned at = __ballot_sync(kFull, k_r == best);
+    const int32_t win = __shfl_sync(kFull, i_r, at != 0u ? __ffs(at) - 1 : 0);
+    const float z = warp_sum_f32(z_r);
+    const bool timeout = best == kKeyTimeout;
+    const bool hit = len_ok && !timeout && best != 0u;
+    const int32_t n = hit ? int32_t(best >> kKeyShift) : 0;
+    const int32_t e = hit ? int32_t(best & kKeyEndMask) : -1;
+    const int32_t kappa = a.kappa > 0 ? a.kappa : a.n_min;
+    int32_t mode = SWITCHSD_MODE_NO_REP;
+    if (hit) mode = (n >= kappa && z >= a.logit_tau) ? SWITCHSD_MODE_COPY : SWITCHSD_MODE_REP_NO_COPY;
+    const int32_t len = mode == SWITCHSD_MODE_COPY ? min(a.k, L - 1 - e) : 0;
+    if (lane == 0) {
+        a.out_mode[b] = mode;
+        a.out_len[b] = len;
+        a.out_score[b] = z;
+        if (a.out_match_n) a.out_match_n[b] = n;
+        if (a.out_match_end) a.out_match_end[b] = e;
+        if (verifying && !len_ok) a.out_accept[b] = -1;
+        if (a.status) {
+            int32_t st = vst;
+            if (st == SWITCHSD_ROW_OK && timeout) st = SWITCHSD_ROW_TIMEOUT;
+            a.status[b] = st;
+        }
+    }
+    const int32_t *wd = reinterpret_cast<const int32_t *>(msgs + size_t(win) * slot_bytes + 16);
+    for (int i = lane; i < len; i += kWarp) a.out_draft[size_t(b) * a.k + i] = wd[i];
+    if (!all_in && lane == 0) (void)mbar_wait(&bars[3], 0);  // messages still in flight: a second bounded wait
+    if (timed_out && lane == 0) {
+        (void)mbar_wait(&bars[0], 0);
+        (void)mbar_wait(&bars[1], 0);
+    }
+    if (!probe_ok && lane == 0) (void)mbar_wait(&bars[2], 0);
+}
+
+size_t rescan_smem_bytes(const StepArgs &args, int split) {
+    const size_t stage = size_t((kHalo + args.tile + kFwd + 3) & ~3) * sizeof(int32_t);
+    const size_t probe = 2 * size_t(args.probe_words) * 16;
+    const size_t msgs = size_t(split) * kRescanWarps * 16 * size_t(1 + ((args.k + 3) >> 2));
+    return stage + probe + msgs;
+}
+
+template <bool kSampled>
+static cudaError_t launch_rescan(const StepArgs &args, int split, cudaStream_t stream) {
+    static bool attr_done[64] = {false};
+    int dev = 0;
+    cudaGetDevice(&dev);
+    if (dev >= 0 && dev < 64 && !attr_done[dev]) {
+        cudaError_t e = cudaFuncSetAttribute(rescan_kernel<kSampled>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
+        if (e != cudaSuccess) return e;
+        e = cudaFuncSetAttribute(rescan_kernel<kSampled>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 int(kRescanSmemBudget));
+        if (e != cudaSuccess) return e;
+        attr_done[dev] = true;
+    }
+    return launch_pdl(rescan_kernel<kSampled>, dim3(unsigned(split), unsigned(args.B), 1), dim3(kRescanThreads, 1, 1),
+                      rescan_smem_bytes(args, split), stream, unsigned(split), args);
+}
+
+cudaError_t launch_rescan_kernel(const StepArgs &args, int split, cudaStream_t stream) {
+    return args.pv_p != nullptr ? launch_rescan<true>(args, split, stream) : launch_rescan<false>(args, split, stream);
+}
+
+}  // namespace switchsd

@@ -18,6 +18,14 @@ constexpr int kMaxSplit = 16;
 constexpr unsigned long long kTimeoutBit = 1ull << 62;
 constexpr int kMaxCand = SWITCHSD_WMAX; // candidate mode: largest W
 constexpr int kProbeStage = 256;      // probe words (8 bf16) of w and of h staged per CTA; the rest is read directly
+// The rescan kernel (rescan.cu): four warps, at most 72 registers a thread, so that seven CTAs fit on an
+// SM and the next launch's CTAs are resident while this launch finishes.
+constexpr int kRescanThreads = 128;
+constexpr int kRescanWarps = kRescanThreads / kWarp;
+constexpr int kRescanMinBlocks = 7;
+constexpr int kRescanTileMax = 16384;  // largest CTA range of the rescan kernel (one bulk copy)
+constexpr size_t kRescanSmemBudget = 100 * 1024;
+constexpr int kRescanCapMax = 1 << 25;  // the rescan kernel's match keys hold an end below 2^25
 
 static_assert(kHalo >= SWITCHSD_NMAX && kHalo % 4 == 0, "halo must cover the longest n-gram");
 static_assert(kFwd % 4 == 0 && kTileMax % 4 == 0, "stages must stay 16-byte aligned");
@@ -51,6 +59,7 @@ struct StepArgs {
     const int32_t *pv_cand_len;  // candidate mode, verifying: the previous candidates' lengths [B, W]
                                  // (pv_draft [B, W, D], pv_target [B, W, D+1], pv_len = their count [B])
     int32_t *out_choice;         // ... and the kept candidate [B]
+    int32_t probe_words;         // rescan kernel: probe words of w and of h staged per CTA
 };
 
 __device__ __forceinline__ float dot8_bf16(uint4 w, uint4 h, float acc) {
@@ -72,5 +81,10 @@ __device__ __forceinline__ void st_cluster_i32(uint32_t addr, int32_t v) {
 // Launches step_kernel<cand> on grid (split, B) as clusters of `split` CTAs, with the shared memory
 // that args.stages / args.tile / args.bm_words call for.
 cudaError_t launch_step_kernel(const StepArgs &args, bool cand, int split, cudaStream_t stream);
+
+// The rescan kernel (rescan.cu) on grid (split, B): the linear probe, greedy or sampled verification (or
+// none), no candidates, no length bound; args.tile >= the largest CTA range, args.probe_words set.
+cudaError_t launch_rescan_kernel(const StepArgs &args, int split, cudaStream_t stream);
+size_t rescan_smem_bytes(const StepArgs &args, int split);
 
 }  // namespace switchsd

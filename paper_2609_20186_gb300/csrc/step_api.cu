@@ -38,6 +38,19 @@ static int choose_split(int B, int cap) {
     return c;
 }
 
+// CTAs per row of the rescan kernel: the largest power of two, at most kMaxSplit, that leaves every CTA
+// at least 8192 candidate ends while two launches' grids fit on the GPU at once (seven of its CTAs per
+// SM), so the next launch's copies are in flight while this one finishes; 1 at least.  Measured on the
+// 32K-context workload in a graph of back-to-back launches: 4 CTAs (8K ends each) 3.5-3.8 us per launch,
+// 8 CTAs 4.2-4.3 us, 2 CTAs 3.8-4.0 us.
+static int choose_rescan_split(int B, int cap) {
+    const int sms = sm_count_cached() > 0 ? sm_count_cached() : 148;
+    int c = 1;
+    while (c < kMaxSplit && cap / (2 * c) >= 8192 && 2 * int64_t(B) * (2 * c) <= int64_t(kRescanMinBlocks) * sms)
+        c *= 2;
+    return c;
+}
+
 // Candidate-mode outputs of switchsd_step_candidates.
 struct CandSpec {
     int32_t W, D;
@@ -183,6 +196,28 @@ static int step_entry(int32_t *ctx_tokens, int32_t *ctx_lens, const uint16_t *hi
     args.hidden_rows = p->hidden_rows > 1 ? p->hidden_rows : 1;
     args.len_bound = p->len_bound;
 
+    // The rescan kernel takes the linear probe's step without candidates (the index has its own kernel);
+    // the step kernel takes everything else.
+    const bool rescan = cs == nullptr && p->probe_kind == SWITCHSD_PROBE_LINEAR && p->index == nullptr &&
+                        p->cap <= kRescanCapMax;
+    if (rescan) {
+        const int rsplit = p->split > 0 ? p->split : choose_rescan_split(p->B, p->cap);
+        const int64_t rrange = ((int64_t(p->cap) - 1 + rsplit - 1) / rsplit + 3) / 4 * 4;
+        const int nv = p->d >> 3;
+        const int vper = (nv + rsplit - 1) / rsplit;
+        args.tile = int32_t(rrange);
+        args.stages = 1;
+        args.probe_words = vper < kProbeStage ? vper : kProbeStage;
+        args.W = args.D = args.bm_words = 0;
+        args.out_cand = args.out_cand_len = args.out_ncand = args.out_choice = nullptr;
+        args.pv_cand_len = nullptr;
+        args.b2 = 0.f;
+        if (rrange <= kRescanTileMax && rescan_smem_bytes(args, rsplit) <= kRescanSmemBudget) {
+            if (launch_rescan_kernel(args, rsplit, stream) != cudaSuccess) return SWITCHSD_ERR_CUDA;
+            return SWITCHSD_OK;
+        }
+    }
+    args.probe_words = 0;
     const int split = p->split > 0 ? p->split : choose_split(p->B, p->cap);
     // Tile: the largest CTA range (the last CTA may also cover a k + 1 token append), in one stage
     // up to kSingleTileMax ends (64 KB; one copy, and few enough bytes that a grid of two or four

@@ -51,13 +51,20 @@ def test_replica_throughput_gloo_world2():
 
 
 def test_choose_replicas():
+    """The replica count keeps every timed launch's batch out of L2 whatever the step count: the other
+    R - 1 batches cover 2.2x L2, and a region of up to 64 launches reads each batch once."""
     sys.path.insert(0, ROOT)
     import bench
     l2 = 126 << 20
-    r = bench.choose_replicas(10 << 20, l2, 512)
-    assert r & (r - 1) == 0 and r * (10 << 20) >= 2.2 * l2 and (r // 2) * (10 << 20) < 2.2 * l2
-    assert bench.choose_replicas(10 << 20, l2, 8) == 8        # never more batches than launches
-    assert bench.choose_replicas(1 << 30, l2, 512) == 1
+    batch = 10 << 20
+    for K in (1, 3, 20, 64, 512):
+        r = bench.choose_replicas(batch, l2, K)
+        assert r & (r - 1) == 0 and (r - 1) * batch >= 2.2 * l2
+        assert r >= min(K, 64)
+        assert r == 2 or ((r // 2 - 1) * batch < 2.2 * l2 or r // 2 < min(K, 64))  # the smallest such
+    assert bench.choose_replicas(1 << 30, l2, 20) == 32      # huge batches: 20 distinct batches still
+    assert bench.choose_replicas(1 << 30, l2, 1) == 2
+    assert bench.choose_replicas(8 << 10, l2, 20, max_r=1024) == 1024  # far below L2: capped
 
 
 def test_reference_arm_line():
