@@ -390,9 +390,12 @@ size_t switchsd_workspace_bytes(const switchsd_params *params);
  *
  *   Limit: the two-layer probe needs switchsd_workspace_bytes(params) <= 16 MiB (S x B x H1p <= 4 Mi
  *   floats: for example B <= 1,024 with d >= 2048 and 256 hidden units); larger requests return
- *   SWITCHSD_ERR_SHAPE.  The linear probe has no limit beyond switchsd_step's.
+ *   SWITCHSD_ERR_SHAPE.  The linear probe has no limit beyond switchsd_step's.  Like switchsd_step it
+ *   verifies nothing, so params->hidden_rows must be 0 or 1.
  *   Set-up: the first call on each device looks up the array's device address (cudaGetSymbolAddress,
- *   with that device current); make that first call before any stream capture.
+ *   with that device current) and keeps it; make that first call before any stream capture.  A device
+ *   reset (cudaDeviceReset) invalidates the kept address: do not call this entry point on a device after
+ *   resetting it in the same process.
  *   Sharing: every call on a device uses the same array, and the array keeps whatever the last call
  *   left there.  Nothing in it needs to start at zero (each call writes every entry it reads), but calls
  *   that overlap on the GPU race on it: issue them on one stream, or order them.

@@ -68,6 +68,25 @@ __device__ __forceinline__ bool mbar_wait(uint64_t *bar, uint32_t parity) {
     return false;
 }
 
+// mbar_wait with a caller's poll count (0: give up at once).
+__device__ __forceinline__ bool mbar_wait_polls(uint64_t *bar, uint32_t parity, uint32_t polls) {
+    const uint32_t addr = smem_addr(bar);
+    for (uint32_t it = 0; it < polls; ++it) {
+        uint32_t done;
+        asm volatile(
+            "{\n"
+            ".reg .pred p;\n"
+            "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n"
+            "selp.u32 %0, 1, 0, p;\n"
+            "}\n"
+            : "=r"(done)
+            : "r"(addr), "r"(parity)
+            : "memory");
+        if (done) return true;
+    }
+    return false;
+}
+
 // Bulk asynchronous copy global -> this CTA's shared memory, completing `bytes` of transaction on
 // `bar`.  dst, src 16-byte aligned; bytes a multiple of 16.
 __device__ __forceinline__ void bulk_g2s(void *dst, const void *src, uint32_t bytes, uint64_t *bar) {

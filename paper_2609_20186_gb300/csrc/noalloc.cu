@@ -9,7 +9,9 @@
 // The array is a file-scope __device__ variable: every GPU that loads the library holds it (16 MiB)
 // until the process exits.  Host code cannot use the variable's name as a device address, so the
 // first call on each device asks the runtime for the array's address (cudaGetSymbolAddress) with that
-// device current, and every later call on the device reuses it.
+// device current, and every later call on the device reuses it.  A device reset (cudaDeviceReset) ends
+// the context the address belongs to, so the cached address is not valid after one: a process that
+// resets a device must not call this entry point on it again.
 #include <mutex>
 
 #include "common.cuh"
@@ -31,7 +33,10 @@ void *static_workspace_address() {
     std::lock_guard<std::mutex> guard(g_lock);
     if (g_address[dev] == nullptr) {
         void *p = nullptr;
-        if (cudaGetSymbolAddress(&p, g_static_workspace) != cudaSuccess) return nullptr;
+        if (cudaGetSymbolAddress(&p, g_static_workspace) != cudaSuccess) {
+            (void)cudaGetLastError();  // leave no error behind for the caller's next runtime check
+            return nullptr;
+        }
         g_address[dev] = p;
     }
     return g_address[dev];

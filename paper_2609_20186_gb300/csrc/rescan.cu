@@ -439,7 +439,7 @@ __global__ void __launch_bounds__(kRescanThreads, kRescanMinBlocks) rescan_kerne
             a.out_accept[b] = acc;
         }
     }
-    const bool all_in = __all_sync(kFull, mbar_wait(&bars[3], 0));
+    const bool all_in = __all_sync(kFull, mbar_wait_polls(&bars[3], 0, a.msg_wait_polls));
     uint32_t k_r = 0u;
     int32_t i_r = 0;
     float z_r = 0.f;

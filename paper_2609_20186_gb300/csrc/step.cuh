@@ -60,6 +60,8 @@ struct StepArgs {
                                  // (pv_draft [B, W, D], pv_target [B, W, D+1], pv_len = their count [B])
     int32_t *out_choice;         // ... and the kept candidate [B]
     int32_t probe_words;         // rescan kernel: probe words of w and of h staged per CTA
+    uint32_t msg_wait_polls;     // rescan kernel: polls of the leader's wait for the messages (kWaitLimit
+                                 // normally; see msg_wait_polls() in step_api.cu)
 };
 
 __device__ __forceinline__ float dot8_bf16(uint4 w, uint4 h, float acc) {

@@ -3,6 +3,8 @@
 // switchsd_workspace_bytes.  Host-side validation, the choice of the split, the shared-memory tiling of
 // each CTA's range, the two-layer probe's kernels and the index's kernel; the step kernel itself is
 // in step.cu.
+#include <cstdlib>
+
 #include "common.cuh"
 #include "index.cuh"
 #include "mlp.cuh"
@@ -39,16 +41,31 @@ static int choose_split(int B, int cap) {
 }
 
 // CTAs per row of the rescan kernel: the largest power of two, at most kMaxSplit, that leaves every CTA
-// at least 8192 candidate ends while two launches' grids fit on the GPU at once (seven of its CTAs per
-// SM), so the next launch's copies are in flight while this one finishes; 1 at least.  Measured on the
-// 32K-context workload in a graph of back-to-back launches: 4 CTAs (8K ends each) 3.5-3.8 us per launch,
-// 8 CTAs 4.2-4.3 us, 2 CTAs 3.8-4.0 us.
+// at least 4096 candidate ends while two launches' grids fit on the GPU at once (seven of its CTAs per
+// SM), so the next launch's copies are in flight while this one finishes; 1 at least.  Measured in the
+// benchmark's launch graph: the 32K-context rows 8 CTAs 4.74 us per launch (4: 5.04, 16: 6.85), the 8K
+// rows 2 CTAs 3.41 us (4: 3.43, 1: 4.19), the 128K rows 16 CTAs 5.87 us (8: 8.59).
 static int choose_rescan_split(int B, int cap) {
     const int sms = sm_count_cached() > 0 ? sm_count_cached() : 148;
     int c = 1;
-    while (c < kMaxSplit && cap / (2 * c) >= 8192 && 2 * int64_t(B) * (2 * c) <= int64_t(kRescanMinBlocks) * sms)
+    while (c < kMaxSplit && cap / (2 * c) >= 4096 && 2 * int64_t(B) * (2 * c) <= int64_t(kRescanMinBlocks) * sms)
         c *= 2;
     return c;
+}
+
+// Polls of the rescan kernel's wait for the row's messages: kWaitLimit, or the value of the environment
+// variable SWITCHSD_DIAG_MESSAGE_WAIT_POLLS when it is set (read once per process).  A diagnostic of the
+// bounded-wait path: with 0 the leader gives up at once, reports SWITCHSD_ROW_TIMEOUT for every row, and
+// still waits (bounded, kWaitLimit) for the messages in flight before it exits.
+static uint32_t msg_wait_polls() {
+    static const uint32_t polls = [] {
+        const char *v = std::getenv("SWITCHSD_DIAG_MESSAGE_WAIT_POLLS");
+        if (v == nullptr || *v == '\0') return kWaitLimit;
+        char *end = nullptr;
+        const unsigned long n = std::strtoul(v, &end, 10);
+        return (end != nullptr && *end == '\0' && n <= kWaitLimit) ? uint32_t(n) : kWaitLimit;
+    }();
+    return polls;
 }
 
 // Candidate-mode outputs of switchsd_step_candidates.
@@ -208,6 +225,7 @@ static int step_entry(int32_t *ctx_tokens, int32_t *ctx_lens, const uint16_t *hi
         args.tile = int32_t(rrange);
         args.stages = 1;
         args.probe_words = vper < kProbeStage ? vper : kProbeStage;
+        args.msg_wait_polls = msg_wait_polls();
         args.W = args.D = args.bm_words = 0;
         args.out_cand = args.out_cand_len = args.out_ncand = args.out_choice = nullptr;
         args.pv_cand_len = nullptr;

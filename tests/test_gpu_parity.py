@@ -5,7 +5,8 @@ probe logits within 1e-3 absolute; no switch flip outside 1e-3 of the threshold 
 
 Small cases compare every row at every step and span several staged tiles with ragged tails; the
 full-size workloads run every row on the GPU in the launch configuration the benchmark uses, and the
-oracle replays a sample of rows (rows are independent, so a replayed row is exact).
+oracle replays every row of every step (its calls split over the host cores), 64 of the 256 rows for the
+two-layer-probe workload.
 """
 import numpy as np
 import pytest
@@ -77,19 +78,21 @@ def test_planted(variant):
         assert g["accept"][0] == exp["accept"] and g_lens[0] == wl.L0 + exp["accept"] + 1
 
 
-FULL_ROWS = {"uniform_8k": [0, 31, 63], "zipf_32k": [0, 29, 63], "code_16k": [0, 101, 255],
-             "mixed_128k": [0, 7, 15]}
+FULL_ROWS = {"uniform_8k": 64, "zipf_32k": 64, "code_16k": 64, "mixed_128k": 16}
 
 
 @pytest.mark.parametrize("name", list(FULL_ROWS))
-def test_full_size_sampled_rows(name):
-    """Full-size workload in the benchmark's launch configuration (fused verify + step)."""
+def test_full_size_every_row(name):
+    """Full-size workload in the benchmark's launch configuration (fused verify + step), every step:
+    every row (the first 64 of the code workload's 256) against the oracle."""
     wl = W[name]
-    rows = FULL_ROWS[name]
+    n = FULL_ROWS[name]
     g_trace, g_ctx, _ = lockstep.gpu_trace(wl, wl.steps, fused=True)
-    o_trace, o_ctx, _ = lockstep.oracle_trace(wl, rows, wl.steps)
+    o_trace, o_ctx, _ = lockstep.oracle_trace_rows(wl, n, wl.steps)
+    rows = range(n)
     flips, stats = lockstep.compare(wl, o_trace, g_trace, rows, o_ctx, g_ctx)
-    assert stats["checked"] >= (len(rows) - len(flips)) * 1
+    assert stats["checked"] >= (n - len(flips)) * wl.steps
+    assert len(flips) <= 2
     # every row of the batch stayed healthy on the GPU
     for t in g_trace:
         assert np.all(t["status"] == 0) and np.all(t["vstatus"] == 0)
@@ -289,4 +292,4 @@ def test_two_layer_probe_tensor_cores(B, d, H1, bias):
     got = out["score"].cpu().numpy()
     for b in range(B):
         ref = oracle.probe_mlp(h[b], W1, w2, b1=b1, b2=b2)
-        assert abs(got[b] - ref) <= 1e-3 * max(1.0, abs(ref)), (b, got[b], ref)
+        assert abs(got[b] - ref) <= 1e-3, (b, got[b], ref)
