@@ -646,6 +646,7 @@ def measure_loop(base, args, dev, cs, l2, W, K, split, search, prefetch, sampled
         while time.perf_counter() < t_end:
             restore()
             l2_flush(flush)
+            torch.cuda._sleep(SPIN_CYCLES)
             g.replay()
             cs.synchronize()
 
@@ -657,6 +658,8 @@ def measure_loop(base, args, dev, cs, l2, W, K, split, search, prefetch, sampled
             # the index's leg: its state after the first replay is the start of the timed one
             lens_hist[0].copy_(loop.lens)
         l2_flush(flush)
+        # a GPU spin long enough for the host to submit the graph, so the region starts with work queued
+        torch.cuda._sleep(SPIN_CYCLES)
         with nvtx_range(f"timed {base.name} {search} x{K}"):
             ev0.record(cs)
             g.replay()
@@ -935,6 +938,7 @@ def read_ceiling(loop, d: int, K: int, step_base: int, prefetch: bool, cs, flush
                 enqueue(split)
             g.replay()
             l2_flush(flush)
+            torch.cuda._sleep(SPIN_CYCLES)
             e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
             e0.record(cs)
             g.replay()

@@ -47,68 +47,53 @@ static_assert(kRescanTileMax / 4 / (kScanWords * kRescanThreads) <= 32, "a threa
 // for the longest-then-most-recent match: the largest key m << kKeyShift | e over the ends with
 // m(e) >= n_min, 0 if none.  stage[kHalo + p - e_lo] = x[p] over [e_lo - kHalo, e_end + kFwd).
 //
-// Filter depth F = min(n_min, 3): end e passes when its last F tokens equal the suffix's, i.e.
-// t(e) = (x[e] ^ s0) | (x[e-1] ^ s1) | (x[e-2] ^ s2) (its first F terms) is 0.  Exact: every end with
-// m(e) >= n_min >= F passes.  Each token's x ^ s1 and x ^ s2 serve the next two ends, so an end costs an
-// xor per term and a three-input logic op, and a running three-input min tests a round together.
+// Filter depth F = min(n_min, 3): end e can match only if its last F tokens equal the suffix's.  Pass 1
+// tests a hash of them, h(e) = x[e] + x[e-1] A + x[e-2] B (the first F terms, mod 2^32), against the
+// suffix's: equal tokens give equal hashes, so no end that matches is missed, and the few that collide
+// are dropped by pass 2's exact test.  Two multiply-adds per end and a running three-input min test a
+// round of sixteen ends; the shared-memory reads, not the arithmetic, set the pace.
 //
-// Pass 1: rounds of kScanWords words per thread (word g0 + u kT, g0 = tid + kScanWords kT r; consecutive
-// lanes hold consecutive words, so the two tokens before a word are the previous lane's last two -- lane 0
-// loads them; unset before position 0, where lim < F drops the end); a round with an end that passes only
-// sets its bit.  No branch and no backward compare in the hot loop.
+// Pass 1: rounds of kScanWords words per thread (word g0 + u kT, g0 = tid + kScanWords kT r: consecutive
+// lanes read consecutive words), each with the two tokens before it (unset before position 0, where
+// lim < F drops the end); a round with an end that passes only sets its bit.  No branch and no backward
+// compare in the hot loop.
 // Pass 2 (rare): the rounds that passed, in warp-synchronous steps (each step every lane with a round left
 // takes its next one, so the compares of a hot suffix run side by side), reloaded from shared memory;
-// their passing ends take the backward compare from m = F, eight positions per step with independent
-// loads.
+// their ends that pass the exact test (x[e-i] = suf[-i] for i < F) take the backward compare from m = F,
+// eight positions per step with independent loads.
+constexpr uint32_t kHashA = 0x9E3779B1u, kHashB = 0x85EBCA77u;  // odd multipliers
+
 template <int F>
 __device__ __forceinline__ uint32_t scan_ends(const int32_t *stage, int32_t e_lo, int32_t e_end, const int32_t *suf,
                                               int32_t n_min, int32_t n_max, int tid, int lane) {
     const int32_t s0 = suf[0], s1 = F >= 2 ? suf[-1] : 0, s2 = F >= 3 ? suf[-2] : 0;
+    const uint32_t hs = uint32_t(s0) + (F >= 2 ? uint32_t(s1) * kHashA : 0u) + (F >= 3 ? uint32_t(s2) * kHashB : 0u);
     const int32_t n4 = (e_end - e_lo + 3) >> 2;
     const int4 *g4 = reinterpret_cast<const int4 *>(stage + kHalo);
     const int32_t off = kHalo - e_lo;
-    // t of the four ends of word v, given the two tokens before it (pz = x[4g - 2], pw = x[4g - 1])
-    auto filter4 = [&](const int4 &v, int32_t pz, int32_t pw, uint32_t (&t)[4]) {
-        t[0] = uint32_t(v.x ^ s0);
-        t[1] = uint32_t(v.y ^ s0);
-        t[2] = uint32_t(v.z ^ s0);
-        t[3] = uint32_t(v.w ^ s0);
-        if (F >= 2) {
-            t[0] |= uint32_t(pw ^ s1);
-            t[1] |= uint32_t(v.x ^ s1);
-            t[2] |= uint32_t(v.y ^ s1);
-            t[3] |= uint32_t(v.z ^ s1);
-        }
-        if (F >= 3) {
-            t[0] |= uint32_t(pz ^ s2);
-            t[1] |= uint32_t(pw ^ s2);
-            t[2] |= uint32_t(v.x ^ s2);
-            t[3] |= uint32_t(v.y ^ s2);
-        }
+    auto hash = [&](int32_t x0, int32_t x1, int32_t x2) {  // x0 = x[e], x1 = x[e-1], x2 = x[e-2]
+        uint32_t h = uint32_t(x0);
+        if (F >= 2) h += uint32_t(x1) * kHashA;
+        if (F >= 3) h += uint32_t(x2) * kHashB;
+        return h ^ hs;
     };
     uint32_t passed = 0u;
     int rnd = 0;
     for (int32_t g0 = tid; g0 - lane < n4; g0 += kScanWords * kRescanThreads, ++rnd) {
         int4 v[kScanWords];
-        int2 pv[kScanWords];
+        int2 pv[kScanWords];  // x[4g - 2], x[4g - 1]
 #pragma unroll
         for (int u = 0; u < kScanWords; ++u) {
             const int32_t g = g0 + u * kRescanThreads;
             v[u] = g < n4 ? g4[g] : make_int4(0, 0, 0, 0);
-            pv[u] = (F >= 2 && lane == 0 && g < n4) ? *reinterpret_cast<const int2 *>(stage + kHalo + 4 * g - 2)
-                                                     : make_int2(0, 0);
+            pv[u] = (F >= 2 && g < n4) ? *reinterpret_cast<const int2 *>(stage + kHalo + 4 * g - 2) : make_int2(0, 0);
         }
         uint32_t mn = 0xffffffffu;
 #pragma unroll
         for (int u = 0; u < kScanWords; ++u) {
-            if (F >= 2) {
-                const int32_t uw = __shfl_up_sync(kFull, v[u].w, 1);
-                const int32_t uz = F >= 3 ? __shfl_up_sync(kFull, v[u].z, 1) : 0;
-                if (lane > 0) pv[u] = make_int2(uz, uw);
-            }
-            uint32_t t[4];
-            filter4(v[u], pv[u].x, pv[u].y, t);
-            mn = __vimin3_u32(mn, __vimin3_u32(t[0], t[1], t[2]), t[3]);
+            const uint32_t h0 = hash(v[u].x, pv[u].y, pv[u].x), h1 = hash(v[u].y, v[u].x, pv[u].y);
+            const uint32_t h2 = hash(v[u].z, v[u].y, v[u].x), h3 = hash(v[u].w, v[u].z, v[u].y);
+            mn = __vimin3_u32(mn, __vimin3_u32(h0, h1, h2), h3);
         }
         passed |= uint32_t(mn == 0u) << (rnd & 31);
     }
@@ -121,18 +106,25 @@ __device__ __forceinline__ uint32_t scan_ends(const int32_t *stage, int32_t e_lo
         for (int u = 0; u < kScanWords; ++u) {
             const int32_t g = tid + r * kScanWords * kRescanThreads + u * kRescanThreads;
             if (g >= n4) break;
+            const int4 v = g4[g];
             const int2 pv = *reinterpret_cast<const int2 *>(stage + kHalo + 4 * g - 2);
-            uint32_t t[4];
-            filter4(g4[g], pv.x, pv.y, t);
-            uint32_t hall = uint32_t(t[0] == 0u) | (uint32_t(t[1] == 0u) << 1) | (uint32_t(t[2] == 0u) << 2) |
-                            (uint32_t(t[3] == 0u) << 3);
+            // exact test of the last F tokens of each end
+            const int32_t x[6] = {pv.x, pv.y, v.x, v.y, v.z, v.w};
+            uint32_t hall = 0u;
+#pragma unroll
+            for (int j = 0; j < 4; ++j) {
+                bool ok = x[j + 2] == s0;
+                if (F >= 2) ok = ok && x[j + 1] == s1;
+                if (F >= 3) ok = ok && x[j] == s2;
+                hall |= uint32_t(ok) << j;
+            }
             while (hall) {
                 const int j = __ffs(hall) - 1;
                 hall &= hall - 1;
                 const int32_t e = e_lo + 4 * g + j;
                 if (e >= e_end) break;
                 const int32_t lim = min(n_max, e + 1);
-                if (lim < F) continue;  // the filter read a token before position 0
+                if (lim < F) continue;  // the test read a token before position 0
                 // m(e) from F: x[e - q] against suf[-q], eight positions per step, every load issued
                 // unconditionally (q clamped to lim - 1; the sentinel bit ends the run at the count)
                 int32_t m = F;
@@ -221,9 +213,12 @@ __global__ void __launch_bounds__(kRescanThreads, kRescanMinBlocks) rescan_kerne
     };
     if (bounded && tid == 0) issue_tile(tile_hi());
     // Every thread reads the length itself (one L2 request per warp), then arrives on the cluster
-    // barrier with release: the leader rewrites the length only after waiting on it.
+    // barrier.  The arrive is relaxed: the barrier only has to publish the leader's message barrier (its
+    // initialisation fence is a release), and each warp's read of the length is ordered before the leader
+    // rewrites it by the data itself -- the warp's message is computed from the length, and the leader
+    // rewrites it only after every message has landed.
     const int32_t L_old = __ldcg(a.lens + b);
-    cluster_arrive_release();
+    cluster_arrive_relaxed();
     const bool len_ok = L_old >= 1 && L_old <= (bounded ? a.len_bound : a.cap);
     const int32_t E_old = len_ok ? L_old - 1 : 0;
     if (!bounded) {
