@@ -706,6 +706,45 @@ def measure_loop(base, args, dev, cs, l2, W, K, split, search, prefetch, sampled
            "value": replica_throughput(B * K, region_s, world),
            "ms_per_step": reduce_max(region_s, world) / K * 1e3}
 
+    if headline and replayable:
+        # the controller's per-mode tallies of the timed launches (switchsd_params.counters): the same
+        # launches replayed from the restored state with the counters on, outside the timed region
+        from paper_2609_20186_gb300 import binding as bdm
+        ctr = torch.zeros(bdm.COUNTERS, dtype=torch.int64, device=dev)
+        saved = loop.params
+        loop.params = []
+        for q in saved:
+            q2 = bdm.switchsd_params.from_buffer_copy(q)
+            q2.counters = ctr.data_ptr()
+            loop.params.append(q2)
+        with torch.cuda.stream(cs):
+            restore()
+            gc = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(gc, stream=cs):
+                for j in range(rounds):
+                    q = warm_rounds + j
+                    if j > 0:
+                        loop.harness(q - 1)
+                    for r in range(min(R, K - j * R)):
+                        loop.launch(r, q * R + r, False)
+            restore()
+            ctr.zero_()
+            gc.replay()
+            cs.synchronize()
+            restore()
+        loop.params = saved
+        c = ctr.cpu().numpy()
+        steps_all = int(c[0] + c[1] + c[2])
+        out["modes"] = {
+            "steps": steps_all, "no_rep": int(c[0]), "copy": int(c[1]), "rep_no_copy": int(c[2]),
+            "copy_share": float(c[1]) / max(steps_all, 1),
+            "copy_drafts_verified": int(c[3]),
+            "mean_accept_copy": float(c[4]) / max(int(c[3]), 1),
+            "neural_drafts_verified": int(c[5]),
+            "mean_accept_neural": float(c[6]) / max(int(c[5]), 1),
+            "note": "device counters (switchsd_params.counters) over the timed launches, replayed from the "
+                    "same state: rows per mode chosen, and per drafter (the previous step's mode) the drafts "
+                    "verified and their mean accepted length; neural drafts are the target stand-in's"}
     if headline and R >= 2 and search == "scan":
         # warm L2, reported separately: K launches alternating between two batches only
         with torch.cuda.stream(cs):
@@ -856,7 +895,8 @@ def run_ours(args, world, rank, local):
                        "search": args.search, "scan_equivalent_gbs": head["scan_equivalent_gbs"],
                        "mean_context_tokens": head["mean_context_tokens"],
                        "launches_per_step": head["launches_per_step"],
-                       "target_standin_launches_in_timed_region": head["harness_in_region"]},
+                       "target_standin_launches_in_timed_region": head["harness_in_region"],
+                       "modes": head.get("modes")},
         "gpu_launches": K * head["launches_per_step"] + 2 * head["harness_in_region"],
         "gpu_launches_note": "fused controller launches (switchsd_verify_step; plus the two-layer probe kernel "
                              "when used) in one CUDA graph, and, when K exceeds the replica count, one target "
@@ -970,7 +1010,8 @@ def run_e2e(base, dev, W, K, split, world, prefetch=True, sampled=False):
                    kappa=wl.kappa, logit_tau=wl.logit_tau, probe_kind=wl.probe_kind,
                    probe_hidden=wl.probe_hidden, future=wl.future(), harness=wl.harness_params(),
                    split=split, d=d, device=dev,  # an H2D copy precedes each call
-                   prefetch=(binding.PREFETCH_CONTEXT | binding.PREFETCH_PROBE) if prefetch else 0)
+                   prefetch=(binding.PREFETCH_CONTEXT | binding.PREFETCH_PROBE) if prefetch else 0,
+                   counters=True)
     host_h = torch.empty(W + K, B, d, dtype=torch.int16).pin_memory()
     for t in range(W + K):
         host_h[t].copy_(torch.from_numpy(wl.hidden(t).view(np.int16)))
@@ -1000,7 +1041,16 @@ def run_e2e(base, dev, W, K, split, world, prefetch=True, sampled=False):
         one(W + i)
     secs = time.perf_counter() - t0
     value = replica_throughput(B * K, secs, world)
-    return {"value": value, "unit": UNIT, "h2d_bytes_per_step": B * d * 2,
+    c = sess.counters.cpu().numpy()
+    steps_all = int(c[0] + c[1] + c[2])
+    modes = {"steps": steps_all, "no_rep": int(c[0]), "copy": int(c[1]), "rep_no_copy": int(c[2]),
+             "copy_share": float(c[1]) / max(steps_all, 1),
+             "copy_drafts_verified": int(c[3]), "mean_accept_copy": float(c[4]) / max(int(c[3]), 1),
+             "neural_drafts_verified": int(c[5]), "mean_accept_neural": float(c[6]) / max(int(c[5]), 1),
+             "note": f"device counters (switchsd_params.counters) over the {W + K} steps of this loop on one "
+                     "batch: rows per mode chosen, and per drafter (the previous step's mode) the drafts "
+                     "verified and their mean accepted length; neural drafts are the target stand-in's"}
+    return {"value": value, "unit": UNIT, "h2d_bytes_per_step": B * d * 2, "modes": modes,
             "d2h_bytes_per_step": B * (k + 3) * 4,
             "note": ("one batch; per step: target stand-in, then one switchsd_plan_run call replaying "
                      + ("switchsd_verify_sampled_step_host" if sampled else "switchsd_verify_step_host")

@@ -42,7 +42,7 @@
 extern "C" {
 #endif
 
-#define SWITCHSD_ABI_VERSION 7
+#define SWITCHSD_ABI_VERSION 8
 
 #define SWITCHSD_NMAX 32 /* largest supported n_max */
 #define SWITCHSD_KMAX 64 /* largest supported draft length k */
@@ -71,6 +71,14 @@ extern "C" {
 /* switchsd_params.prefetch bits. */
 #define SWITCHSD_PREFETCH_CONTEXT 1
 #define SWITCHSD_PREFETCH_PROBE 2
+
+/* Slots of switchsd_params.counters. */
+#define SWITCHSD_CTR_STEPS 0           /* + mode: rows whose step chose that mode (3 slots) */
+#define SWITCHSD_CTR_COPY_DRAFTS 3     /* copy drafts verified */
+#define SWITCHSD_CTR_COPY_ACCEPTED 4   /* their accepted tokens */
+#define SWITCHSD_CTR_NEURAL_DRAFTS 5   /* other drafts verified */
+#define SWITCHSD_CTR_NEURAL_ACCEPTED 6 /* their accepted tokens */
+#define SWITCHSD_COUNTERS 7
 
 /* Incremental n-gram index (switchsd_index_create); opaque. */
 typedef struct switchsd_index switchsd_index;
@@ -136,6 +144,20 @@ typedef struct switchsd_index switchsd_index;
  *                bound gets SWITCHSD_ROW_BAD_LEN.  cap is always a valid bound; a bound far above the
  *                lengths leaves CTAs idle and copies bytes past the rows' ends.  The index search
  *                ignores it.  Outside [0, cap]: SWITCHSD_ERR_ARG.
+ *   counters     optional device uint64[SWITCHSD_COUNTERS], or NULL: the controller's per-mode tallies
+ *                (the paper's copy-iteration share and mean accepted length per drafter, §4 and Table
+ *                1), added to by every row of every call -- the caller zeroes them when it wants to
+ *                start counting:
+ *                  [SWITCHSD_CTR_STEPS + m]  rows whose step chose mode m (SWITCHSD_MODE_*)
+ *                  [SWITCHSD_CTR_COPY_DRAFTS], [SWITCHSD_CTR_COPY_ACCEPTED]  drafts verified whose
+ *                        previous step was COPY, and the tokens accepted of them
+ *                  [SWITCHSD_CTR_NEURAL_DRAFTS], [SWITCHSD_CTR_NEURAL_ACCEPTED]  the same for the
+ *                        other drafts (the neural drafter's)
+ *                The fused verifications take each row's previous mode from out_mode[b] as the call
+ *                finds it (the caller passes the same out_mode array every step; the call overwrites it
+ *                with the new mode).  Rows whose verification fails (bad length, capacity) add no draft.
+ *                Integer additions: the totals do not depend on the order of the rows.  The candidate
+ *                entry points ignore it.
  */
 typedef struct {
     int32_t B, cap, d, k, n_min, n_max, kappa;
@@ -155,6 +177,7 @@ typedef struct {
     int32_t prefetch;
     int32_t hidden_rows;
     int32_t len_bound;
+    uint64_t *counters;
 } switchsd_params;
 
 /*

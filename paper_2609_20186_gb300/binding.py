@@ -19,7 +19,7 @@ PROBE_LINEAR, PROBE_MLP = 0, 1
 OK, ERR_ARG, ERR_SHAPE, ERR_CUDA = 0, -1, -2, -3
 ROW_OK, ROW_CAPACITY, ROW_BAD_LEN, ROW_TIMEOUT = 0, 1, 2, 3
 NMAX, KMAX = 32, 64
-ABI_VERSION = 7  # SWITCHSD_ABI_VERSION this binding marshals for
+ABI_VERSION = 8  # SWITCHSD_ABI_VERSION this binding marshals for
 PREFETCH_CONTEXT, PREFETCH_PROBE = 1, 2  # switchsd_params.prefetch bits
 
 _c_i32p = ctypes.c_void_p
@@ -41,7 +41,12 @@ class switchsd_params(ctypes.Structure):
         ("prefetch", ctypes.c_int32),
         ("hidden_rows", ctypes.c_int32),
         ("len_bound", ctypes.c_int32),
+        ("counters", ctypes.c_void_p),
     ]
+
+
+# slots of switchsd_params.counters (include/switchsd.h)
+CTR_STEPS, CTR_COPY_DRAFTS, CTR_COPY_ACCEPTED, CTR_NEURAL_DRAFTS, CTR_NEURAL_ACCEPTED, COUNTERS = 0, 3, 4, 5, 6, 7
 
 
 class switchsd_verify_params(ctypes.Structure):

@@ -220,6 +220,18 @@ inline cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, s
     return cudaLaunchKernelEx(&cfg, kernel, std::forward<Args>(args)...);
 }
 
+// The per-mode tallies of switchsd_params.counters for one row: its step chose `mode`; when its
+// verification appended (acc >= 0) the draft it verified came from the previous step's mode `prev`.
+__device__ __forceinline__ void count_row(unsigned long long *ctr, int32_t mode, bool verified, int32_t prev,
+                                          int32_t acc) {
+    atomicAdd(&ctr[SWITCHSD_CTR_STEPS + mode], 1ull);
+    if (verified && acc >= 0) {
+        const int slot = prev == SWITCHSD_MODE_COPY ? SWITCHSD_CTR_COPY_DRAFTS : SWITCHSD_CTR_NEURAL_DRAFTS;
+        atomicAdd(&ctr[slot], 1ull);
+        atomicAdd(&ctr[slot + 1], static_cast<unsigned long long>(acc));
+    }
+}
+
 __device__ __forceinline__ float bf16_lo(uint32_t v) { return __uint_as_float(v << 16); }
 __device__ __forceinline__ float bf16_hi(uint32_t v) { return __uint_as_float(v & 0xffff0000u); }
 

@@ -71,6 +71,7 @@ struct IndexArgs {
     const int32_t *pv_cand_len;  // [B][W]
     int32_t *out_choice, *out_cand, *out_cand_len, *out_ncand;
     int32_t prefetch;  // SWITCHSD_PREFETCH_* bits: the inputs they name are read before the wait
+    unsigned long long *counters;  // optional per-mode tallies (switchsd_params.counters), else null
 };
 
 // This thread's share of the linear probe's dot product over row b's hidden state (threads stride the
@@ -322,6 +323,8 @@ __global__ void __launch_bounds__(kIdxMaxWarps * kWarp) index_kernel(const Index
         s_out[0] = estar;
         s_out[1] = len;
         s_out[2] = mode == SWITCHSD_MODE_COPY ? s_ncf : 0;  // candidate mode: candidates written
+        if (a.W == 0 && a.counters)  // out_mode still holds the previous step's mode
+            count_row(a.counters, mode, verifying, a.out_mode[b], s_ver[0]);
         a.out_mode[b] = mode;
         if (a.W == 0) a.out_len[b] = len;
         else a.out_ncand[b] = s_out[2];
@@ -398,7 +401,8 @@ int index_launch(switchsd_index *idx, int32_t *ctx, int32_t *lens, const uint16_
                  int32_t *out_draft, int32_t *out_len, int32_t *out_mode, float *out_score, int32_t *out_match_n,
                  int32_t *out_match_end, int32_t *status, int B, int cap, int d, int k, int n_min, int n_max, int kappa,
                  float logit_tau, bool stepping, cudaStream_t stream, const float *pv_p, const float *pv_q,
-                 const float *pv_u, int hidden_rows, const IndexCandidates *cand, int prefetch) {
+                 const float *pv_u, int hidden_rows, const IndexCandidates *cand, int prefetch,
+                 unsigned long long *counters) {
     if (idx->B != B || idx->cap != cap || idx->n_min != n_min || idx->n_max != n_max) return SWITCHSD_ERR_SHAPE;
     // Candidate mode lists the ends of the kappa-gram chain: kappa must be one of the index's n, or
     // above n_max (no end can then reach it: no candidate, as for the rescan).
@@ -412,6 +416,7 @@ int index_launch(switchsd_index *idx, int32_t *ctx, int32_t *lens, const uint16_
     a.out_cand_len = cand ? cand->out_cand_len : nullptr;
     a.out_ncand = cand ? cand->out_ncand : nullptr;
     a.prefetch = prefetch;
+    a.counters = stepping ? counters : nullptr;
     a.pv_p = pv_p;
     a.pv_q = pv_q;
     a.pv_u = pv_u;

@@ -36,7 +36,7 @@ int index_launch(switchsd_index *idx, int32_t *ctx, int32_t *lens, const uint16_
                  int32_t *out_match_end, int32_t *status, int B, int cap, int d, int k, int n_min, int n_max, int kappa,
                  float logit_tau, bool stepping, cudaStream_t stream, const float *pv_p = nullptr,
                  const float *pv_q = nullptr, const float *pv_u = nullptr, int hidden_rows = 1,
-                 const IndexCandidates *cand = nullptr, int prefetch = 0);
+                 const IndexCandidates *cand = nullptr, int prefetch = 0, unsigned long long *counters = nullptr);
 
 int index_n_min(const switchsd_index *idx);
 int index_n_max(const switchsd_index *idx);

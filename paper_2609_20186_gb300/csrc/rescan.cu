@@ -187,7 +187,10 @@ __global__ void __launch_bounds__(kRescanThreads, kRescanMinBlocks) rescan_kerne
 
     const bool pf_ctx = (a.prefetch & SWITCHSD_PREFETCH_CONTEXT) != 0;
     const bool gather = verifying && a.hidden_rows > 1;
-    const bool pf_probe = (a.prefetch & SWITCHSD_PREFETCH_PROBE) != 0 && !gather;
+    // Two-layer probe: the first layer's split-K partial sums come from the probe kernel just before this
+    // one (read after the wait); this CTA finishes units [u0, u1) (b1, ReLU, w2).
+    const bool mlp = a.z1_part != nullptr;
+    const bool pf_probe = (a.prefetch & SWITCHSD_PREFETCH_PROBE) != 0 && !gather && !mlp;
     if (!pf_ctx) pdl_wait();
     int32_t *row = a.ctx + size_t(b) * size_t(a.cap);
     // The CTA's ends are split on the row's old length, or, with a length bound, on the bound: its tile
@@ -236,7 +239,7 @@ __global__ void __launch_bounds__(kRescanThreads, kRescanMinBlocks) rescan_kerne
     const int nv = a.d >> 3;
     const int vper = (nv + int(C) - 1) / int(C);
     const int v0 = min(nv, int(rank) * vper), v1 = min(nv, v0 + vper);
-    const int v_staged = gather ? 0 : min(v1 - v0, a.probe_words);
+    const int v_staged = (gather || mlp) ? 0 : min(v1 - v0, a.probe_words);
     const uint4 *w4 = reinterpret_cast<const uint4 *>(a.probe_w);
     const uint4 *h4 = reinterpret_cast<const uint4 *>(a.hidden + size_t(b) * size_t(gather ? a.hidden_rows : 1) *
                                                                   size_t(a.d));
@@ -275,7 +278,7 @@ __global__ void __launch_bounds__(kRescanThreads, kRescanMinBlocks) rescan_kerne
     if (pf_probe && warp >= 1) probe_dot(h4);
     if (pf_ctx) pdl_wait();
     pdl_trigger();
-    if (!pf_probe && !gather && tid == 0) issue_probe();
+    if (!pf_probe && !gather && !mlp && tid == 0) issue_probe();
 
     // ---- verification of the previous draft (every warp) ----
     int32_t acc = -1, L = L_old, vst = len_ok ? SWITCHSD_ROW_OK : SWITCHSD_ROW_BAD_LEN;
@@ -377,7 +380,17 @@ __global__ void __launch_bounds__(kRescanThreads, kRescanMinBlocks) rescan_kerne
 
     // ---- probe share (unless finished before the wait) ----
     if (warp >= 1) {
-        if (gather) {
+        if (mlp) {
+            // units u0 + j, u0 + j + (kT - 32), ... for thread j = tid - 32: the S partial sums in order
+            const int uper = (a.H1 + int(C) - 1) / int(C);
+            const int u0 = min(a.H1, int(rank) * uper), u1 = min(a.H1, u0 + uper);
+            for (int u = u0 + tid - kWarp; u < u1; u += kRescanThreads - kWarp) {
+                float z1 = 0.f;
+                for (int sp = 0; sp < a.mlp_S; ++sp) z1 += a.z1_part[(size_t(sp) * a.B + size_t(b)) * a.H1p + u];
+                if (a.b1) z1 += a.b1[u];
+                zp = fmaf(bf16_lo(uint32_t(a.w2[u])), fmaxf(z1, 0.f), zp);
+            }
+        } else if (gather) {
             zp = dot8_bf16(gw, gh, 0.f);  // zero words for a thread past the slice
             for (int v = v0 + tid - kWarp + (kRescanThreads - kWarp); v < v1; v += kRescanThreads - kWarp)
                 zp = dot8_bf16(__ldg(w4 + v), __ldg(h4 + v), zp);
@@ -451,7 +464,7 @@ __global__ void __launch_bounds__(kRescanThreads, kRescanMinBlocks) rescan_kerne
     const uint32_t best = all_in ? __reduce_max_sync(kFull, k_r) : kKeyTimeout;
     const unsigned at = __ballot_sync(kFull, k_r == best);
     const int32_t win = __shfl_sync(kFull, i_r, at != 0u ? __ffs(at) - 1 : 0);
-    const float z = warp_sum_f32(z_r);
+    const float z = warp_sum_f32(z_r) + (mlp ? a.b2 : 0.f);
     const bool timeout = best == kKeyTimeout;
     const bool hit = len_ok && !timeout && best != 0u;
     const int32_t n = hit ? int32_t(best >> kKeyShift) : 0;
@@ -461,6 +474,7 @@ __global__ void __launch_bounds__(kRescanThreads, kRescanMinBlocks) rescan_kerne
     if (hit) mode = (n >= kappa && z >= a.logit_tau) ? SWITCHSD_MODE_COPY : SWITCHSD_MODE_REP_NO_COPY;
     const int32_t len = mode == SWITCHSD_MODE_COPY ? min(a.k, L - 1 - e) : 0;
     if (lane == 0) {
+        if (a.counters) count_row(a.counters, mode, verifying, a.out_mode[b], acc);  // out_mode: the previous mode
         a.out_mode[b] = mode;
         a.out_len[b] = len;
         a.out_score[b] = z;

@@ -653,6 +653,8 @@ __global__ void __launch_bounds__(kStepThreads) step_kernel(const StepArgs a) {
             s_out[0] = int32_t(win);
             s_out[1] = len;
             if (kCand) s_ncand = mode == SWITCHSD_MODE_COPY ? ncand : 0;
+            if (!kCand && a.counters)  // out_mode still holds the previous step's mode
+                count_row(a.counters, mode, verifying, a.out_mode[b], s_ver[0]);
             a.out_mode[b] = mode;
             if (!kCand) a.out_len[b] = len;
             a.out_score[b] = z;

@@ -60,6 +60,7 @@ struct StepArgs {
                                  // (pv_draft [B, W, D], pv_target [B, W, D+1], pv_len = their count [B])
     int32_t *out_choice;         // ... and the kept candidate [B]
     int32_t probe_words;         // rescan kernel: probe words of w and of h staged per CTA
+    unsigned long long *counters;  // optional per-mode tallies (switchsd_params.counters), else null
     uint32_t msg_wait_polls;     // rescan kernel: polls of the leader's wait for the messages (kWaitLimit
                                  // normally; see msg_wait_polls() in step_api.cu)
 };

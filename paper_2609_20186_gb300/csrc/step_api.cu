@@ -212,29 +212,9 @@ static int step_entry(int32_t *ctx_tokens, int32_t *ctx_lens, const uint16_t *hi
     args.prefetch = p->prefetch;
     args.hidden_rows = p->hidden_rows > 1 ? p->hidden_rows : 1;
     args.len_bound = p->len_bound;
+    args.counters = cs == nullptr ? reinterpret_cast<unsigned long long *>(p->counters) : nullptr;
+    args.msg_wait_polls = kWaitLimit;
 
-    // The rescan kernel takes the linear probe's step without candidates (the index has its own kernel);
-    // the step kernel takes everything else.
-    const bool rescan = cs == nullptr && p->probe_kind == SWITCHSD_PROBE_LINEAR && p->index == nullptr &&
-                        p->cap <= kRescanCapMax;
-    if (rescan) {
-        const int rsplit = p->split > 0 ? p->split : choose_rescan_split(p->B, p->cap);
-        const int64_t rrange = ((int64_t(p->cap) - 1 + rsplit - 1) / rsplit + 3) / 4 * 4;
-        const int nv = p->d >> 3;
-        const int vper = (nv + rsplit - 1) / rsplit;
-        args.tile = int32_t(rrange);
-        args.stages = 1;
-        args.probe_words = vper < kProbeStage ? vper : kProbeStage;
-        args.msg_wait_polls = msg_wait_polls();
-        args.W = args.D = args.bm_words = 0;
-        args.out_cand = args.out_cand_len = args.out_ncand = args.out_choice = nullptr;
-        args.pv_cand_len = nullptr;
-        args.b2 = 0.f;
-        if (rrange <= kRescanTileMax && rescan_smem_bytes(args, rsplit) <= kRescanSmemBudget) {
-            if (launch_rescan_kernel(args, rsplit, stream) != cudaSuccess) return SWITCHSD_ERR_CUDA;
-            return SWITCHSD_OK;
-        }
-    }
     args.probe_words = 0;
     const int split = p->split > 0 ? p->split : choose_split(p->B, p->cap);
     // Tile: the largest CTA range (the last CTA may also cover a k + 1 token append), in one stage
@@ -316,7 +296,28 @@ static int step_entry(int32_t *ctx_tokens, int32_t *ctx_lens, const uint16_t *hi
                             args.H1, args.H1p, args.b2, pv_draft, pv_target, pv_len, out_accept, out_draft, out_len,
                             out_mode, out_score, p->out_match_n, p->out_match_end, p->status, p->B, p->cap, p->d, p->k,
                             p->n_min, p->n_max, p->kappa, p->logit_tau, true, stream, pv_p, pv_q, pv_u,
-                            args.hidden_rows, cs != nullptr ? &ic : nullptr, p->prefetch);
+                            args.hidden_rows, cs != nullptr ? &ic : nullptr, p->prefetch, args.counters);
+    }
+    // The rescan kernel takes the step without candidates (linear probe, or the two-layer probe's finish
+    // after its kernel above); the step kernel takes the candidate mode.
+    const bool rescan = cs == nullptr && p->cap <= kRescanCapMax;
+    if (rescan) {
+        const int rsplit = p->split > 0 ? p->split : choose_rescan_split(p->B, p->cap);
+        const int64_t rrange = ((int64_t(p->cap) - 1 + rsplit - 1) / rsplit + 3) / 4 * 4;
+        const int nv = p->d >> 3;
+        const int vper = (nv + rsplit - 1) / rsplit;
+        StepArgs ra = args;
+        ra.tile = int32_t(rrange);
+        ra.stages = 1;
+        ra.probe_words = args.z1_part != nullptr ? 0 : (vper < kProbeStage ? vper : kProbeStage);
+        ra.msg_wait_polls = msg_wait_polls();
+        ra.W = ra.D = ra.bm_words = 0;
+        ra.out_cand = ra.out_cand_len = ra.out_ncand = ra.out_choice = nullptr;
+        ra.pv_cand_len = nullptr;
+        if (rrange <= kRescanTileMax && rescan_smem_bytes(ra, rsplit) <= kRescanSmemBudget) {
+            if (launch_rescan_kernel(ra, rsplit, stream) != cudaSuccess) return SWITCHSD_ERR_CUDA;
+            return SWITCHSD_OK;
+        }
     }
     const cudaError_t e = launch_step_kernel(args, cs != nullptr, split, stream);
     if (e != cudaSuccess) return SWITCHSD_ERR_CUDA;

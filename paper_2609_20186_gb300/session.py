@@ -38,7 +38,7 @@ class Session:
                  probe_kind: int = bd.PROBE_LINEAR, probe_hidden: int = 0, future=None,
                  harness: dict | None = None, split: int = 0, d: int | None = None,
                  use_index: bool = False, device="cuda", stream: torch.cuda.Stream | None = None,
-                 prefetch: int = 0, hidden_rows: int = 0, len_bound: int = 0):
+                 prefetch: int = 0, hidden_rows: int = 0, len_bound: int = 0, counters: bool = False):
         self.lib = bd.load()
         self.hidden_rows = int(hidden_rows)
         self.device = torch.device(device)
@@ -67,6 +67,8 @@ class Session:
         self.vlen = torch.zeros(B, **i32)
         self.target = torch.zeros(B, k + 1, **i32)
         self.vstatus = torch.zeros(B, **i32)
+        # per-mode tallies (switchsd_params.counters; uint64 on the device, int64 here), when asked for
+        self.counters = torch.zeros(bd.COUNTERS, dtype=torch.int64, device=dev) if counters else None
         fut = future if future is not None else np.zeros((B, 0), np.int32)
         self.future = torch.from_numpy(np.ascontiguousarray(fut, np.int32)).to(dev)
         self.stream = stream
@@ -104,6 +106,7 @@ class Session:
             p.prefetch = int(prefetch)
             p.hidden_rows = int(hidden_rows)  # k + 1: verify_step reads row a_b of a [B, k+1, d] hidden
             p.len_bound = int(len_bound)      # > 0: split on this bound, copies before the length read
+            p.counters = self.counters.data_ptr() if self.counters is not None else None
             return p
         self._p_dbg, self._p_fast = params(True), params(False)
         self._step_head = (self.ctx.data_ptr(), self.lens.data_ptr())

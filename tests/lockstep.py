@@ -110,13 +110,15 @@ def oracle_trace_rows(wl: synth.Workload, n_rows: int, steps: int, threads: int 
 
 
 def gpu_trace(wl: synth.Workload, steps: int, split: int = 0, ctx=None, lens=None, device="cuda",
-              fused: bool = False, use_index: bool = False, sampled: bool = False):
+              fused: bool = False, use_index: bool = False, sampled: bool = False, extras: dict | None = None):
     """Runs the GPU loop on all rows; returns the per-step host copies of every output.
 
     fused=False: switchsd_step, target stand-in, switchsd_verify per iteration.
     fused=True:  switchsd_verify_step (verification of iteration t-1, then step t) and the target
                  stand-in per iteration; the last draft is verified by switchsd_verify.
-    sampled=True: the sampled stand-in and switchsd_verify_sampled / switchsd_verify_sampled_step (T > 0)."""
+    sampled=True: the sampled stand-in and switchsd_verify_sampled / switchsd_verify_sampled_step (T > 0).
+    extras: if given, the run keeps the per-mode counters (switchsd_params.counters) and stores them
+    there under "counters" (host int64 array)."""
     import torch
     from paper_2609_20186_gb300 import Session, bf16_tensor
 
@@ -125,7 +127,7 @@ def gpu_trace(wl: synth.Workload, steps: int, split: int = 0, ctx=None, lens=Non
     sess = Session(ctx, lens, wl.probe_weights(), k=wl.k, n_min=wl.n_min, n_max=wl.n_max,
                    kappa=wl.kappa, logit_tau=wl.logit_tau, probe_kind=wl.probe_kind,
                    probe_hidden=wl.probe_hidden, future=wl.future(), harness=wl.harness_params(),
-                   split=split, d=wl.d, use_index=use_index, device=device)
+                   split=split, d=wl.d, use_index=use_index, device=device, counters=extras is not None)
     trace = []
     for t in range(steps):
         hidden = bf16_tensor(wl.hidden(t), sess.device)
@@ -156,6 +158,8 @@ def gpu_trace(wl: synth.Workload, steps: int, split: int = 0, ctx=None, lens=Non
             out["lens_after"] = sess.lens.cpu().numpy()
         trace.append(out)
     torch.cuda.synchronize()
+    if extras is not None:
+        extras["counters"] = sess.counters.cpu().numpy()
     return trace, sess.ctx.cpu().numpy(), sess.lens.cpu().numpy()
 
 

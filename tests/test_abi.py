@@ -58,7 +58,7 @@ def test_binding_declares_every_function():
 
 def test_abi_version_and_strerror(lib):
     from paper_2609_20186_gb300 import binding as bd
-    assert bd.abi_version() == 7
+    assert bd.abi_version() == 8
     for code in (0, -1, -2, -3, 1, 2, 3):
         assert bd.strerror(code) != "unknown code"
     assert bd.strerror(12345) == "unknown code"
@@ -291,3 +291,35 @@ def test_binding_rejects_cpu_tensors(lib):
         bd.switchsd_verify(t, torch.zeros(2, 9, dtype=torch.int32), torch.zeros(2, dtype=torch.int32),
                            draft_len=torch.zeros(2, dtype=torch.int32), ctx_tokens=t,
                            ctx_lens=torch.zeros(2, dtype=torch.int32))
+
+
+def test_params_layout_matches_the_header(tmp_path):
+    """The binding's ctypes structures have the C header's layout (size and every field's offset): a
+    program compiled against include/switchsd.h prints them."""
+    import ctypes
+    import shutil
+    import subprocess
+    from paper_2609_20186_gb300 import binding as bd
+
+    cc = shutil.which("gcc") or shutil.which("cc")
+    if cc is None:
+        pytest.skip("no C compiler")
+    structs = {"switchsd_params": bd.switchsd_params, "switchsd_verify_params": bd.switchsd_verify_params,
+               "switchsd_candidates_verify_params": bd.switchsd_candidates_verify_params}
+    lines = ['#include <stdio.h>', '#include <stddef.h>', '#include "switchsd.h"', "int main(void) {"]
+    for name, st in structs.items():
+        lines.append(f'  printf("{name} size %zu\\n", sizeof({name}));')
+        for field, _ in st._fields_:
+            lines.append(f'  printf("{name} {field} %zu\\n", offsetof({name}, {field}));')
+    lines += ["  return 0;", "}"]
+    src = tmp_path / "layout.c"
+    src.write_text("\n".join(lines) + "\n")
+    exe = tmp_path / "layout"
+    root = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+    subprocess.run([cc, "-std=c99", "-I", os.path.join(root, "include"), str(src), "-o", str(exe)], check=True)
+    out = subprocess.run([str(exe)], check=True, capture_output=True, text=True).stdout.splitlines()
+    got = {tuple(line.split()[:2]): int(line.split()[2]) for line in out}
+    for name, st in structs.items():
+        assert got[(name, "size")] == ctypes.sizeof(st), name
+        for field, _ in st._fields_:
+            assert got[(name, field)] == getattr(st, field).offset, (name, field)
