@@ -588,7 +588,7 @@ def measure_loop(base, args, dev, cs, l2, W, K, split, search, prefetch, sampled
 
     B, d, k = base.B, base.d, base.k
     batch_bytes = B * (base.L0 + 1024) * 4
-    R = choose_replicas(batch_bytes, l2, K, max_r=(16 if search == "index" else 1024))
+    R = choose_replicas(batch_bytes, l2, K, max_r=(32 if search == "index" else 1024))
     rounds = -(-K // R)
     warm_rounds = max(1, -(-W // R))
     per_row_steps = warm_rounds + 2 * rounds + (COLD_STEPS if headline else 0) + 1
