@@ -11,6 +11,8 @@
 // sum has a fixed order, so the result is deterministic.  No cluster and no cross-CTA exchange here.
 #include <cudaTypedefs.h>
 
+#include <algorithm>
+
 #include "common.cuh"
 #include "mlp.cuh"
 
@@ -25,6 +27,7 @@ constexpr uint32_t kBChunk = kMlpN * kMlpKc * 2;    // 8 KB
 constexpr uint32_t kTmemCols = 64;
 static_assert(kMaxMlpChunks * (kAChunk + kBChunk) + 1024 + 64 <= 227 * 1024,
               "operands, alignment slack and static shared memory must fit one CTA");
+static_assert(kMlpThreads == kMlpM && kMlpN == 64, "one thread per tile row; 16 chunks of 16 bytes per row");
 
 // Instruction descriptor of tcgen05.mma kind::f16: D fp32, A and B bf16, both K-major, M = 128, N = 64.
 constexpr uint32_t kIdesc = (1u << 4) | (1u << 7) | (1u << 10) | (uint32_t(kMlpN >> 3) << 17) |
@@ -33,6 +36,7 @@ constexpr uint32_t kIdesc = (1u << 4) | (1u << 7) | (1u << 10) | (uint32_t(kMlpN
 struct MlpArgs {
     float *part;   // [S][B][H1p]
     int32_t B, H1p, nchunks, prefetch;
+    int32_t stages;  // operand stages: chunk c goes to stage c % stages, refilled once its MMAs are done
 };
 
 // Shared-memory matrix descriptor: K-major, 128-byte swizzle, 8-row groups 1024 bytes apart.
@@ -67,34 +71,39 @@ __global__ void __launch_bounds__(kMlpThreads) mlp_tc_kernel(const __grid_consta
                                                              const __grid_constant__ CUtensorMap tm_w,
                                                              const MlpArgs a) {
     extern __shared__ uint8_t smem_raw[];
-    __shared__ __align__(8) uint64_t tma_bar, mma_bar;
+    __shared__ __align__(8) uint64_t full[kMaxMlpChunks], empty[kMaxMlpChunks], mma_bar;
     __shared__ uint32_t s_tmem;
 
-    const int tid = threadIdx.x, warp = tid >> 5;
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const int S = int(gridDim.x), ks = blockIdx.x;
     const int n_tile = blockIdx.y, m0 = blockIdx.z * kMlpM, n0 = n_tile * kMlpN;
     const int per = (a.nchunks + S - 1) / S;
     const int c0 = ks * per;
     const int nck = max(0, min(a.nchunks, c0 + per) - c0);
-    // 1024-byte aligned operand area (the swizzle atom): A chunks, then B chunks.
+    const int st = a.stages;  // 1 .. kMaxMlpChunks
+    // 1024-byte aligned operand stages (the swizzle atom): A chunks, then B chunks.
     uint8_t *base = smem_raw + ((1024u - (smem_addr(smem_raw) & 1023u)) & 1023u);
     uint8_t *opA = base;
-    uint8_t *opB = base + size_t(per) * kAChunk;
-    auto issue_loads = [&]() {
-        mbar_arrive_expect_tx(&tma_bar, uint32_t(nck) * (kAChunk + kBChunk));
-        for (int c = 0; c < nck; ++c) {
-            tma_load_2d(opA + size_t(c) * kAChunk, &tm_h, (c0 + c) * kMlpKc, m0, &tma_bar);
-            tma_load_2d(opB + size_t(c) * kBChunk, &tm_w, (c0 + c) * kMlpKc, n0, &tma_bar);
-        }
+    uint8_t *opB = base + size_t(st) * kAChunk;
+    auto issue = [&](int c) {  // chunk c of this CTA's K slice into stage c % st
+        const int sg = c % st;
+        mbar_arrive_expect_tx(&full[sg], kAChunk + kBChunk);
+        tma_load_2d(opA + size_t(sg) * kAChunk, &tm_h, (c0 + c) * kMlpKc, m0, &full[sg]);
+        tma_load_2d(opB + size_t(sg) * kBChunk, &tm_w, (c0 + c) * kMlpKc, n0, &full[sg]);
     };
+    const int first = min(nck, st);  // chunks issued up front
 
     if (tid == 0) {
-        mbar_init(&tma_bar, 1);
+        for (int i = 0; i < st; ++i) {
+            mbar_init(&full[i], 1);
+            mbar_init(&empty[i], 1);
+        }
         mbar_init(&mma_bar, 1);
         fence_mbar_init();
         // With the probe prefetch bit the caller guarantees that the preceding kernel writes neither
         // the hidden states nor W1, so their copies may start before the grid-dependency wait.
-        if (a.prefetch && nck > 0) issue_loads();
+        if (a.prefetch)
+            for (int c = 0; c < first; ++c) issue(c);
     }
     if (warp == 0) {
         asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;\n" ::"r"(smem_addr(&s_tmem)),
@@ -104,40 +113,65 @@ __global__ void __launch_bounds__(kMlpThreads) mlp_tc_kernel(const __grid_consta
     }
     pdl_wait();     // the partial sums below overwrite what an earlier step kernel may still read
     pdl_trigger();
-    if (tid == 0 && !a.prefetch && nck > 0) issue_loads();
+    if (tid == 0 && !a.prefetch)
+        for (int c = 0; c < first; ++c) issue(c);
     asm volatile("tcgen05.fence::before_thread_sync;\n" ::: "memory");
     __syncthreads();
     asm volatile("tcgen05.fence::after_thread_sync;\n" ::: "memory");
     const uint32_t tmem = s_tmem;
 
+    // One thread: wait for chunk c, issue its MMAs, commit them to the stage's empty barrier; a stage is
+    // refilled (chunk c + st) once those MMAs have read it.  ok = every copy and commit arrived in time.
     bool ok = true;
     if (tid == 0) {
-        if (nck > 0 && mbar_wait(&tma_bar, 0)) {
-            for (int c = 0; c < nck; ++c) {
-                const uint64_t da = sw128_desc(smem_addr(opA + size_t(c) * kAChunk));
-                const uint64_t db = sw128_desc(smem_addr(opB + size_t(c) * kBChunk));
-#pragma unroll
-                for (int j = 0; j < kMlpKc / 16; ++j) {
-                    const uint32_t acc = (c | j) != 0;
-                    // advance both descriptors by j * 32 bytes inside the swizzle row
-                    asm volatile(
-                        "{\n"
-                        ".reg .pred p;\n"
-                        "setp.ne.b32 p, %4, 0;\n"
-                        "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n"
-                        "}\n" ::"r"(tmem),
-                        "l"(da + uint64_t(2 * j)), "l"(db + uint64_t(2 * j)), "r"(kIdesc), "r"(acc)
-                        : "memory");
-                }
+        int landed = 0, issued = first;
+        for (int c = 0; c < nck; ++c) {
+            const int sg = c % st;
+            const uint32_t ph = uint32_t(c / st) & 1u;
+            if (!mbar_wait(&full[sg], ph)) {
+                ok = false;
+                break;
             }
+            landed = c + 1;
+            asm volatile("tcgen05.fence::after_thread_sync;\n" ::: "memory");
+            const uint64_t da = sw128_desc(smem_addr(opA + size_t(sg) * kAChunk));
+            const uint64_t db = sw128_desc(smem_addr(opB + size_t(sg) * kBChunk));
+#pragma unroll
+            for (int j = 0; j < kMlpKc / 16; ++j) {
+                const uint32_t acc = (c | j) != 0;
+                // advance both descriptors by j * 32 bytes inside the swizzle row
+                asm volatile(
+                    "{\n"
+                    ".reg .pred p;\n"
+                    "setp.ne.b32 p, %4, 0;\n"
+                    "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n"
+                    "}\n" ::"r"(tmem),
+                    "l"(da + uint64_t(2 * j)), "l"(db + uint64_t(2 * j)), "r"(kIdesc), "r"(acc)
+                    : "memory");
+            }
+            if (c + st < nck) {
+                asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];\n" ::"r"(
+                                 smem_addr(&empty[sg]))
+                             : "memory");
+                if (!mbar_wait(&empty[sg], ph)) {
+                    ok = false;
+                    break;
+                }
+                issue(c + st);
+                issued = c + st + 1;
+            }
+        }
+        if (landed > 0) {
+            // arrives once every MMA issued has completed (on the failure path too: they read the stages)
             asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];\n" ::"r"(
                              smem_addr(&mma_bar))
                          : "memory");
         } else {
-            // nothing to accumulate, or the copies did not land: release the waiters, flag the tile
-            if (nck > 0) ok = false;
+            // nothing to accumulate, or the first copy did not land: release the waiters
             asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];\n" ::"r"(smem_addr(&mma_bar)) : "memory");
         }
+        // copies issued but not waited for (a wait gave up): a second bounded wait before the stages go
+        for (int c = landed; c < issued; ++c) (void)mbar_wait(&full[c % st], uint32_t(c / st) & 1u);
     }
     const bool mma_done = mbar_wait(&mma_bar, 0);
     asm volatile("tcgen05.fence::after_thread_sync;\n" ::: "memory");
@@ -156,13 +190,23 @@ __global__ void __launch_bounds__(kMlpThreads) mlp_tc_kernel(const __grid_consta
 #pragma unroll
         for (int i = 0; i < kMlpN; ++i) v[i] = fill;
     }
-    if (m0 + tid < a.B) {
-        float4 *dst = reinterpret_cast<float4 *>(a.part + (size_t(ks) * a.B + size_t(m0 + tid)) * a.H1p + n0);
+    // The tile goes out through shared memory (the operand stages are free: every MMA has completed), so
+    // that each warp store writes two whole 256-byte rows instead of one 16-byte piece of 32 rows.  Row r
+    // keeps its 16-byte chunk q at position q ^ (r % 16): both the row-wise writes below and the reads
+    // across rows hit distinct banks.
+    float4 *tile = reinterpret_cast<float4 *>(base);  // [kMlpM rows][16 chunks]
 #pragma unroll
-        for (int q = 0; q < kMlpN / 4; ++q) dst[q] = make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
-    }
+    for (int q = 0; q < kMlpN / 4; ++q)
+        tile[tid * 16 + (q ^ (tid & 15))] = make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
     asm volatile("tcgen05.fence::before_thread_sync;\n" ::: "memory");
     __syncthreads();
+#pragma unroll 4
+    for (int i = 0; i < 16; ++i) {  // warp w writes rows 32 w .. 32 w + 31, two per store
+        const int r = warp * 32 + 2 * i + (lane >> 4), c = lane & 15;
+        if (m0 + r < a.B)
+            reinterpret_cast<float4 *>(a.part + (size_t(ks) * a.B + size_t(m0 + r)) * a.H1p + n0)[c] =
+                tile[r * 16 + (c ^ (r & 15))];
+    }
     if (warp == 0)
         asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;\n" ::"r"(tmem), "r"(kTmemCols) : "memory");
 }
@@ -212,14 +256,16 @@ bool mlp_shape_ok(int d, int H1) {
 int mlp_hidden_padded(int H1) { return (H1 + kMlpN - 1) / kMlpN * kMlpN; }
 
 cudaError_t launch_mlp_tc(const uint16_t *hidden, const uint16_t *W1, float *part, int B, int d, int H1,
-                          bool prefetch, cudaStream_t stream) {
+                          bool prefetch, cudaStream_t stream, int stages) {
     CUtensorMap tm_h, tm_w;
     if (!encode_rows(&tm_h, hidden, B, d, kMlpM) || !encode_rows(&tm_w, W1, H1, d, kMlpN))
         return cudaErrorInvalidValue;
     const int nchunks = (d + kMlpKc - 1) / kMlpKc;
     const int S = mlp_split(d);
     const int per = (nchunks + S - 1) / S;
-    const size_t smem = 1024 + size_t(per) * (kAChunk + kBChunk);
+    const int st = stages >= 1 && stages < per ? stages : per;
+    // the operand stages, which also hold the output tile (kMlpM x kMlpN fp32) once the MMAs are done
+    const size_t smem = 1024 + std::max(size_t(st) * (kAChunk + kBChunk), size_t(kMlpM) * kMlpN * 4);
     static bool attr_done[64] = {false};
     int dev = 0;
     cudaGetDevice(&dev);
@@ -235,6 +281,7 @@ cudaError_t launch_mlp_tc(const uint16_t *hidden, const uint16_t *W1, float *par
     a.H1p = mlp_hidden_padded(H1);
     a.nchunks = nchunks;
     a.prefetch = prefetch ? 1 : 0;
+    a.stages = st;
     const dim3 grid(unsigned(S), unsigned(a.H1p / kMlpN), unsigned((B + kMlpM - 1) / kMlpM));
     // An explicit one-CTA cluster: the copies and the MMA commit address shared::cluster.
     return launch_pdl(mlp_tc_kernel, grid, dim3(kMlpThreads), smem, stream, 1u, tm_h, tm_w, a);

@@ -26,6 +26,7 @@
 // them in a fixed order and writes the outputs.  The only cluster barrier is arrived on right after the
 // length read and waited on just before the first message, so the leader's message barrier is
 // initialised before anyone ships to it and no CTA reads the length after the leader rewrites it.
+#include "mlp.cuh"
 #include "step.cuh"
 
 namespace switchsd {
@@ -191,7 +192,12 @@ __global__ void __launch_bounds__(kRescanThreads, kRescanMinBlocks) rescan_kerne
     // one (read after the wait); this CTA finishes units [u0, u1) (b1, ReLU, w2).
     const bool mlp = a.z1_part != nullptr;
     const bool pf_probe = (a.prefetch & SWITCHSD_PREFETCH_PROBE) != 0 && !gather && !mlp;
-    if (!pf_ctx) pdl_wait();
+    // Two-layer probe: every input but the partial sums was written by kernels that completed before the
+    // first-layer kernel released this launch (it does so only after its own wait), so verification and
+    // scan run while it computes; warps 1.. wait just before reading the sums.  Reads before that wait
+    // go through L2 (bulk copies, ld.global.cg).
+    const bool late = mlp && a.wait_late != 0;
+    if (!pf_ctx && !late) pdl_wait();
     int32_t *row = a.ctx + size_t(b) * size_t(a.cap);
     // The CTA's ends are split on the row's old length, or, with a length bound, on the bound: its tile
     // copy then leaves before the length is read, and a row longer than the bound is a bad length.
@@ -276,7 +282,7 @@ __global__ void __launch_bounds__(kRescanThreads, kRescanMinBlocks) rescan_kerne
     // A prefetched probe is finished before the wait by warps 1.. (its inputs are not written by the
     // preceding kernel); warp 0 goes straight to the wait and releases the next launch.
     if (pf_probe && warp >= 1) probe_dot(h4);
-    if (pf_ctx) pdl_wait();
+    if (pf_ctx && !late) pdl_wait();
     pdl_trigger();
     if (!pf_probe && !gather && !mlp && tid == 0) issue_probe();
 
@@ -286,12 +292,12 @@ __global__ void __launch_bounds__(kRescanThreads, kRescanMinBlocks) rescan_kerne
     if (verifying && len_ok) {
         const int32_t *dr = a.pv_draft + size_t(b) * a.k;
         const int32_t *tg = a.pv_target + size_t(b) * (a.k + 1);
-        const int32_t pv_n = a.pv_len[b];
-        d_lo = lane < a.k ? dr[lane] : 0;
-        d_hi = lane + 32 < a.k ? dr[lane + 32] : 0;
-        const int32_t t_lo = lane <= a.k ? tg[lane] : 0;
-        const int32_t t_hi = lane + 32 <= a.k ? tg[lane + 32] : 0;
-        const int32_t t_top = (lane == 0 && a.k >= 64) ? tg[64] : 0;
+        const int32_t pv_n = __ldcg(a.pv_len + b);
+        d_lo = lane < a.k ? __ldcg(dr + lane) : 0;
+        d_hi = lane + 32 < a.k ? __ldcg(dr + lane + 32) : 0;
+        const int32_t t_lo = lane <= a.k ? __ldcg(tg + lane) : 0;
+        const int32_t t_hi = lane + 32 <= a.k ? __ldcg(tg + lane + 32) : 0;
+        const int32_t t_top = (lane == 0 && a.k >= 64) ? __ldcg(tg + 64) : 0;
         if (pv_n < 0 || pv_n > a.k) {
             vst = SWITCHSD_ROW_BAD_LEN;
         } else {
@@ -299,10 +305,11 @@ __global__ void __launch_bounds__(kRescanThreads, kRescanMinBlocks) rescan_kerne
             if (kSampled) {
                 // T > 0: draft token i is rejected when u_i * q_i (binary32) is not below p_i
                 const size_t o = size_t(b) * a.k;
-                rej_lo = lane < pv_n &&
-                         !(__fmul_rn(a.pv_u[o + lane], a.pv_q ? a.pv_q[o + lane] : 1.f) < a.pv_p[o + lane]);
+                rej_lo = lane < pv_n && !(__fmul_rn(__ldcg(a.pv_u + o + lane), a.pv_q ? __ldcg(a.pv_q + o + lane) : 1.f) <
+                                          __ldcg(a.pv_p + o + lane));
                 rej_hi = lane + 32 < pv_n &&
-                         !(__fmul_rn(a.pv_u[o + lane + 32], a.pv_q ? a.pv_q[o + lane + 32] : 1.f) < a.pv_p[o + lane + 32]);
+                         !(__fmul_rn(__ldcg(a.pv_u + o + lane + 32), a.pv_q ? __ldcg(a.pv_q + o + lane + 32) : 1.f) <
+                           __ldcg(a.pv_p + o + lane + 32));
             } else {
                 rej_lo = lane < pv_n && d_lo != t_lo;
                 rej_hi = lane + 32 < pv_n && d_hi != t_hi;
@@ -384,9 +391,17 @@ __global__ void __launch_bounds__(kRescanThreads, kRescanMinBlocks) rescan_kerne
             // units u0 + j, u0 + j + (kT - 32), ... for thread j = tid - 32: the S partial sums in order
             const int uper = (a.H1 + int(C) - 1) / int(C);
             const int u0 = min(a.H1, int(rank) * uper), u1 = min(a.H1, u0 + uper);
+            if (late) pdl_wait();
             for (int u = u0 + tid - kWarp; u < u1; u += kRescanThreads - kWarp) {
+                // every partial sum is loaded before the first add (independent L2 reads), then added in order
+                float pz[kMaxMlpSplit];
+#pragma unroll
+                for (int sp = 0; sp < kMaxMlpSplit; ++sp)
+                    pz[sp] = sp < a.mlp_S ? __ldcg(a.z1_part + (size_t(sp) * a.B + size_t(b)) * a.H1p + u) : 0.f;
                 float z1 = 0.f;
-                for (int sp = 0; sp < a.mlp_S; ++sp) z1 += a.z1_part[(size_t(sp) * a.B + size_t(b)) * a.H1p + u];
+#pragma unroll
+                for (int sp = 0; sp < kMaxMlpSplit; ++sp)
+                    if (sp < a.mlp_S) z1 += pz[sp];
                 if (a.b1) z1 += a.b1[u];
                 zp = fmaf(bf16_lo(uint32_t(a.w2[u])), fmaxf(z1, 0.f), zp);
             }

@@ -63,6 +63,9 @@ struct StepArgs {
     unsigned long long *counters;  // optional per-mode tallies (switchsd_params.counters), else null
     uint32_t msg_wait_polls;     // rescan kernel: polls of the leader's wait for the messages (kWaitLimit
                                  // normally; see msg_wait_polls() in step_api.cu)
+    int32_t wait_late;           // rescan kernel, two-layer probe: the kernel just before is the probe's
+                                 // first layer, which releases this launch only after its own wait; the
+                                 // grid-dependency wait then guards the partial sums alone
 };
 
 __device__ __forceinline__ float dot8_bf16(uint4 w, uint4 h, float acc) {

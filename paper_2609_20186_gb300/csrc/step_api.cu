@@ -214,6 +214,7 @@ static int step_entry(int32_t *ctx_tokens, int32_t *ctx_lens, const uint16_t *hi
     args.len_bound = p->len_bound;
     args.counters = cs == nullptr ? reinterpret_cast<unsigned long long *>(p->counters) : nullptr;
     args.msg_wait_polls = kWaitLimit;
+    args.wait_late = 0;
 
     args.probe_words = 0;
     const int split = p->split > 0 ? p->split : choose_split(p->B, p->cap);
@@ -245,7 +246,26 @@ static int step_entry(int32_t *ctx_tokens, int32_t *ctx_lens, const uint16_t *hi
     }
 
     args.b2 = p->b2;
-    if (p->probe_kind == SWITCHSD_PROBE_MLP) {
+    // The rescan kernel takes the step without candidates or index (linear probe, or the two-layer
+    // probe's finish after its first-layer kernel); the step kernel takes the rest.
+    const bool mlp_probe = p->probe_kind == SWITCHSD_PROBE_MLP;
+    const int rsplit = p->split > 0 ? p->split : choose_rescan_split(p->B, p->cap);
+    StepArgs ra = args;
+    bool rescan = false;
+    if (cs == nullptr && p->index == nullptr && p->cap <= kRescanCapMax) {
+        const int64_t rrange = ((int64_t(p->cap) - 1 + rsplit - 1) / rsplit + 3) / 4 * 4;
+        const int nv = p->d >> 3;
+        const int vper = (nv + rsplit - 1) / rsplit;
+        ra.tile = int32_t(rrange);
+        ra.stages = 1;
+        ra.probe_words = mlp_probe ? 0 : (vper < kProbeStage ? vper : kProbeStage);
+        ra.msg_wait_polls = msg_wait_polls();
+        ra.W = ra.D = ra.bm_words = 0;
+        ra.out_cand = ra.out_cand_len = ra.out_ncand = ra.out_choice = nullptr;
+        ra.pv_cand_len = nullptr;
+        rescan = rrange <= kRescanTileMax && rescan_smem_bytes(ra, rsplit) <= kRescanSmemBudget;
+    }
+    if (mlp_probe) {
         float *part = static_cast<float *>(p->workspace);
         const uint16_t *probe_in = hidden;
         bool probe_pf = (p->prefetch & SWITCHSD_PREFETCH_PROBE) != 0;
@@ -272,7 +292,10 @@ static int step_entry(int32_t *ctx_tokens, int32_t *ctx_lens, const uint16_t *hi
             probe_pf = false;  // the probe kernel's input was just written by the gather
             args.hidden_rows = 1;
         }
-        if (launch_mlp_tc(probe_in, probe_w, part, p->B, p->d, p->probe_hidden, probe_pf, stream) != cudaSuccess)
+        // Beside the rescan kernel the first layer stages two chunks at a time, so that every CTA of the
+        // rescan kernel fits on the GPU while it runs (that kernel verifies and scans meanwhile).
+        if (launch_mlp_tc(probe_in, probe_w, part, p->B, p->d, p->probe_hidden, probe_pf, stream,
+                          rescan ? kMlpStagesBeside : 0) != cudaSuccess)
             return SWITCHSD_ERR_CUDA;
         args.z1_part = part;
         args.b1 = p->b1;
@@ -298,26 +321,19 @@ static int step_entry(int32_t *ctx_tokens, int32_t *ctx_lens, const uint16_t *hi
                             p->n_min, p->n_max, p->kappa, p->logit_tau, true, stream, pv_p, pv_q, pv_u,
                             args.hidden_rows, cs != nullptr ? &ic : nullptr, p->prefetch, args.counters);
     }
-    // The rescan kernel takes the step without candidates (linear probe, or the two-layer probe's finish
-    // after its kernel above); the step kernel takes the candidate mode.
-    const bool rescan = cs == nullptr && p->cap <= kRescanCapMax;
     if (rescan) {
-        const int rsplit = p->split > 0 ? p->split : choose_rescan_split(p->B, p->cap);
-        const int64_t rrange = ((int64_t(p->cap) - 1 + rsplit - 1) / rsplit + 3) / 4 * 4;
-        const int nv = p->d >> 3;
-        const int vper = (nv + rsplit - 1) / rsplit;
-        StepArgs ra = args;
-        ra.tile = int32_t(rrange);
-        ra.stages = 1;
-        ra.probe_words = args.z1_part != nullptr ? 0 : (vper < kProbeStage ? vper : kProbeStage);
-        ra.msg_wait_polls = msg_wait_polls();
-        ra.W = ra.D = ra.bm_words = 0;
-        ra.out_cand = ra.out_cand_len = ra.out_ncand = ra.out_choice = nullptr;
-        ra.pv_cand_len = nullptr;
-        if (rrange <= kRescanTileMax && rescan_smem_bytes(ra, rsplit) <= kRescanSmemBudget) {
-            if (launch_rescan_kernel(ra, rsplit, stream) != cudaSuccess) return SWITCHSD_ERR_CUDA;
-            return SWITCHSD_OK;
-        }
+        ra.z1_part = args.z1_part;
+        ra.b1 = args.b1;
+        ra.w2 = args.w2;
+        ra.mlp_S = args.mlp_S;
+        ra.H1 = args.H1;
+        ra.H1p = args.H1p;
+        ra.hidden_rows = args.hidden_rows;
+        // the first-layer kernel launched just above waits for every earlier kernel before it releases
+        // this one, so only its own output, the partial sums, needs this launch's wait
+        ra.wait_late = args.z1_part != nullptr ? 1 : 0;
+        if (launch_rescan_kernel(ra, rsplit, stream) != cudaSuccess) return SWITCHSD_ERR_CUDA;
+        return SWITCHSD_OK;
     }
     const cudaError_t e = launch_step_kernel(args, cs != nullptr, split, stream);
     if (e != cudaSuccess) return SWITCHSD_ERR_CUDA;
