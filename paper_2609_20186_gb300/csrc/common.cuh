@@ -168,6 +168,20 @@ __device__ __forceinline__ void st_async_v4(uint32_t cluster_addr, uint4 v, uint
         : "memory");
 }
 
+// Bulk copy of `bytes` from this CTA's shared memory to another CTA's (cluster address), completing that
+// many bytes of transaction on the destination's mbarrier (cluster address).  Both addresses 16-byte
+// aligned, bytes a multiple of 16.  The source is read asynchronously: generic writes to it need
+// fence_proxy_async() first, and it stays untouched until bulk_wait_read() returns.
+__device__ __forceinline__ void bulk_s2c(uint32_t dst_cluster, const void *src, uint32_t bytes, uint32_t mbar_cluster) {
+    asm volatile(
+        "cp.async.bulk.shared::cluster.shared::cta.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];\n"
+        "cp.async.bulk.commit_group;\n" ::"r"(dst_cluster),
+        "r"(smem_addr(src)), "r"(bytes), "r"(mbar_cluster)
+        : "memory");
+}
+__device__ __forceinline__ void bulk_wait_read() { asm volatile("cp.async.bulk.wait_group.read 0;\n" ::: "memory"); }
+__device__ __forceinline__ void fence_proxy_async() { asm volatile("fence.proxy.async.shared::cta;\n" ::: "memory"); }
+
 // Remote arrive on an mbarrier in another CTA of the cluster (release, cluster scope).
 __device__ __forceinline__ void mbar_arrive_remote(uint32_t cluster_addr) {
     asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];\n" ::"r"(cluster_addr) : "memory");

@@ -64,9 +64,13 @@ static_assert(kRescanTileMax / 4 / (kScanWords * kRescanThreads) <= 32, "a threa
 // eight positions per step with independent loads.
 constexpr uint32_t kHashA = 0x9E3779B1u, kHashB = 0x85EBCA77u;  // odd multipliers
 
-template <int F>
+//
+// Candidate mode (kCand): every end whose common suffix reaches kappa_c is also marked in the CTA's bitmap
+// bm (bit e - e_lo; F <= kappa_c, so the filter passes every such end).
+template <int F, bool kCand>
 __device__ __forceinline__ uint32_t scan_ends(const int32_t *stage, int32_t e_lo, int32_t e_end, const int32_t *suf,
-                                              int32_t n_min, int32_t n_max, int tid, int lane) {
+                                              int32_t n_min, int32_t n_max, int tid, int lane,
+                                              uint32_t *bm = nullptr, int32_t kappa_c = 0) {
     const int32_t s0 = suf[0], s1 = F >= 2 ? suf[-1] : 0, s2 = F >= 3 ? suf[-2] : 0;
     const uint32_t hs = uint32_t(s0) + (F >= 2 ? uint32_t(s1) * kHashA : 0u) + (F >= 3 ? uint32_t(s2) * kHashB : 0u);
     const int32_t n4 = (e_end - e_lo + 3) >> 2;
@@ -146,18 +150,41 @@ __device__ __forceinline__ uint32_t scan_ends(const int32_t *stage, int32_t e_lo
                     const uint32_t key = (uint32_t(m) << kKeyShift) | uint32_t(e);
                     mine = key > mine ? key : mine;
                 }
+                if (kCand && m >= kappa_c) atomicOr(&bm[(e - e_lo) >> 5], 1u << ((e - e_lo) & 31));
             }
         }
     }
     return mine;
 }
 
-template <bool kSampled>
+constexpr int kVerifyLoads = 4;  // candidate verification: staging loads a thread has in flight at once
+
+// Candidate mode's shared memory beyond the single-draft layout: per CTA one candidate message of cslot
+// bytes -- a 16-byte header (count), the ends (W, most recent first), their continuations [W][D] -- the
+// leader receiving C of them and every CTA staging its own; a bitmap of the CTA's marked ends; the
+// verification's staging of the previous candidates (drafts [W][D], targets [W][D+1], lengths [W], count).
+struct CandLayout {
+    uint32_t cslot;  // bytes of a candidate message
+    int bm_words;    // bitmap words (a multiple of 4)
+    int v_ints;      // verification staging (a multiple of 4)
+};
+__host__ __device__ inline CandLayout cand_layout(int tile, int W, int D) {
+    CandLayout c;
+    c.cslot = 16u * uint32_t(1 + (W + 3) / 4 + (W * D + 3) / 4);
+    c.bm_words = ((tile + 31) / 32 + 3) & ~3;
+    c.v_ints = (W * D + W * (D + 1) + W + 1 + 3) & ~3;
+    return c;
+}
+
+template <bool kSampled, bool kCand>
 __global__ void __launch_bounds__(kRescanThreads, kRescanMinBlocks) rescan_kernel(const StepArgs a) {
     extern __shared__ __align__(128) int32_t dsm[];
     __shared__ __align__(8) uint64_t bars[4];              // tile, tail, probe slices, messages (leader)
     __shared__ __align__(16) int32_t s_tail[kHalo + 8];    // x[tail_lo .. L_old), tail_lo = roundown4(L_old - kHalo)
     __shared__ int32_t s_y[kRescanWarps][kYLen];
+    __shared__ int32_t s_sel[kMaxCand];                    // candidate mode: the CTA's selected ends / the
+                                                           // leader's merged candidates' sources
+    __shared__ int32_t s_wtot[kRescanWarps];               // candidate mode: marks per warp in a pass
 
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     const uint32_t rank = cluster_ctarank();
@@ -170,9 +197,16 @@ __global__ void __launch_bounds__(kRescanThreads, kRescanMinBlocks) rescan_kerne
     uint4 *s_ph = s_pw + a.probe_words;
     unsigned char *msgs = reinterpret_cast<unsigned char *>(s_ph + a.probe_words);
     const bool verifying = a.pv_len != nullptr;
-    const int kw = (a.k + 3) >> 2;                          // 16-byte words of a message's continuation
+    const int kw = kCand ? 0 : (a.k + 3) >> 2;             // 16-byte words of a message's continuation
     const uint32_t slot_bytes = 16u * uint32_t(1 + kw);
     const int nmsg = int(C) * kRescanWarps;
+    const CandLayout cl = cand_layout(kCand ? a.tile : 0, kCand ? a.W : 0, kCand ? a.D : 0);
+    unsigned char *cmsgs = msgs + size_t(nmsg) * slot_bytes;                  // [C][cslot] (leader)
+    unsigned char *cstage = cmsgs + size_t(C) * cl.cslot;                     // this CTA's message
+    uint32_t *bm = reinterpret_cast<uint32_t *>(cstage + cl.cslot);           // [bm_words]
+    int32_t *vc = reinterpret_cast<int32_t *>(bm + cl.bm_words);              // previous drafts [W][D]
+    int32_t *vt = vc + a.W * a.D;                                             // their targets [W][D+1]
+    int32_t *vl = vt + a.W * (a.D + 1);                                       // their lengths [W]
 
     if (tid == 0) {
         mbar_init(&bars[0], 1);
@@ -180,11 +214,13 @@ __global__ void __launch_bounds__(kRescanThreads, kRescanMinBlocks) rescan_kerne
         mbar_init(&bars[2], 1);
         if (rank == lead) {
             mbar_init(&bars[3], 1);
-            mbar_arrive_expect_tx(&bars[3], slot_bytes * uint32_t(nmsg));
+            mbar_arrive_expect_tx(&bars[3], slot_bytes * uint32_t(nmsg) + (kCand ? cl.cslot * C : 0u));
         }
         fence_mbar_init();
     }
-    __syncthreads();  // the barriers are initialised before any thread arms or waits on one
+    if (kCand)
+        for (int i = tid; i < cl.bm_words; i += kRescanThreads) bm[i] = 0u;
+    __syncthreads();  // the barriers are initialised (and the bitmap cleared) before any thread uses them
 
     const bool pf_ctx = (a.prefetch & SWITCHSD_PREFETCH_CONTEXT) != 0;
     const bool gather = verifying && a.hidden_rows > 1;
@@ -289,7 +325,63 @@ __global__ void __launch_bounds__(kRescanThreads, kRescanMinBlocks) rescan_kerne
     // ---- verification of the previous draft (every warp) ----
     int32_t acc = -1, L = L_old, vst = len_ok ? SWITCHSD_ROW_OK : SWITCHSD_ROW_BAD_LEN;
     int32_t d_lo = 0, d_hi = 0, t_acc = 0;
-    if (verifying && len_ok) {
+    int32_t choice = 0;  // candidate mode: the kept candidate
+    if (kCand && verifying) {
+        // The W previous candidates verified at once (§3.3): the CTA stages every slot's draft, target and
+        // length (one round of independent L2 reads, whatever the count), then each warp takes, per
+        // candidate, the first position where draft and target differ; the longest accepted candidate is
+        // kept, the lowest index on a tie.  A count of 0 (a neural draft) uses slot 0 with length 0.
+        const int W = a.W, D = a.D;
+        const size_t o = size_t(b) * size_t(W);
+        // one index space over drafts, targets, lengths and the count (vl[W]); each thread issues all of
+        // its loads before its first store, so they share one round trip
+        const int n_d = W * D, n_t = W * (D + 1), n_all = n_d + n_t + W + 1;
+        for (int base = tid; base < n_all; base += kVerifyLoads * kRescanThreads) {
+            int32_t v[kVerifyLoads];
+#pragma unroll
+            for (int u = 0; u < kVerifyLoads; ++u) {
+                const int i = base + u * kRescanThreads;
+                v[u] = 0;
+                if (i < n_d) v[u] = __ldcg(a.pv_draft + o * D + i);
+                else if (i < n_d + n_t) v[u] = __ldcg(a.pv_target + o * (D + 1) + (i - n_d));
+                else if (i < n_d + n_t + W) v[u] = __ldcg(a.pv_cand_len + o + (i - n_d - n_t));
+                else if (i < n_all) v[u] = __ldcg(a.pv_len + b);
+            }
+#pragma unroll
+            for (int u = 0; u < kVerifyLoads; ++u)
+                if (base + u * kRescanThreads < n_all) vc[base + u * kRescanThreads] = v[u];  // vc, vt, vl contiguous
+        }
+        __syncthreads();
+        const int32_t nc = vl[W];
+        if (len_ok) {
+            bool badlen = nc < 0 || nc > W;
+            const int ncx = badlen ? 0 : (nc > 0 ? nc : 1);
+            int32_t best = -1, best_w = 0;
+            for (int w = 0; w < ncx; ++w) {
+                const int32_t len = nc > 0 ? vl[w] : 0;
+                badlen |= len < 0 || len > D;
+                const int32_t lc = (len >= 0 && len <= D) ? len : 0;
+                const int32_t *cw_ = vc + w * D, *tw_ = vt + w * (D + 1);
+                const unsigned m_lo = __ballot_sync(kFull, lane < lc && cw_[lane] != tw_[lane]);
+                const unsigned m_hi = __ballot_sync(kFull, lane + 32 < lc && cw_[lane + 32] != tw_[lane + 32]);
+                const int32_t acc_w = m_lo ? __ffs(m_lo) - 1 : (m_hi ? 32 + __ffs(m_hi) - 1 : lc);
+                if (acc_w > best) {
+                    best = acc_w;
+                    best_w = w;
+                }
+            }
+            choice = best_w;
+            if (badlen) {
+                vst = SWITCHSD_ROW_BAD_LEN;
+            } else if (L_old + best + 1 > a.cap) {
+                vst = SWITCHSD_ROW_CAPACITY;
+            } else {
+                acc = best;
+                L = L_old + acc + 1;
+            }
+        }
+    }
+    if (!kCand && verifying && len_ok) {
         const int32_t *dr = a.pv_draft + size_t(b) * a.k;
         const int32_t *tg = a.pv_target + size_t(b) * (a.k + 1);
         const int32_t pv_n = __ldcg(a.pv_len + b);
@@ -345,9 +437,14 @@ __global__ void __launch_bounds__(kRescanThreads, kRescanMinBlocks) rescan_kerne
         const int32_t p = L_old - kHalo + lane;
         y[lane] = (len_ok && p >= 0 && tail_in) ? s_tail[p - tail_lo] : 0;
         if (acc >= 0) {
-            if (lane < acc) y[kHalo + lane] = d_lo;
-            if (lane + 32 < acc) y[kHalo + 32 + lane] = d_hi;
-            if (lane == 0) y[kHalo + acc] = t_acc;
+            if (kCand) {  // the kept candidate's accepted tokens, then its target's next token
+                for (int i = lane; i < acc; i += kWarp) y[kHalo + i] = vc[choice * a.D + i];
+                if (lane == 0) y[kHalo + acc] = vt[choice * (a.D + 1) + acc];
+            } else {
+                if (lane < acc) y[kHalo + lane] = d_lo;
+                if (lane + 32 < acc) y[kHalo + 32 + lane] = d_hi;
+                if (lane == 0) y[kHalo + acc] = t_acc;
+            }
         }
     }
     __syncwarp();
@@ -355,6 +452,8 @@ __global__ void __launch_bounds__(kRescanThreads, kRescanMinBlocks) rescan_kerne
     const int32_t n_max = a.n_max, n_min = a.n_min;
 
     // ---- scan of this warp's share of the CTA's old ends ----
+    const int32_t kappa_c = a.kappa > 0 ? a.kappa : a.n_min;  // candidate mode: the gate length
+    uint32_t new_c[3] = {0u, 0u, 0u};                         // candidate mode: appended ends (leader)
     // key = m << kKeyShift | e (e < 2^kKeyShift, m <= 32): the largest key is the longest match, then the
     // most recent; 0 = no match; kKeyTimeout marks a copy that did not land.
     uint32_t mine = 0;
@@ -362,12 +461,39 @@ __global__ void __launch_bounds__(kRescanThreads, kRescanMinBlocks) rescan_kerne
     bool timed_out = !tail_in || !tile_in;
     const int32_t off = kHalo - e_lo;  // stage[off + p] = x[p] over the staged range
     if (!timed_out && len_ok && L >= 2) {
-        // (n_min is uniform over the launch: one instance runs)
-        mine = a.n_min >= 3 ? scan_ends<3>(stage, e_lo, e_end, suf, n_min, n_max, tid, lane)
-                            : (a.n_min == 2 ? scan_ends<2>(stage, e_lo, e_end, suf, n_min, n_max, tid, lane)
-                                            : scan_ends<1>(stage, e_lo, e_end, suf, n_min, n_max, tid, lane));
-        // The ends the append creates, [L_old - 1, L - 1), lie in the window: the leader's warp 0.
-        if (rank == lead && warp == 0 && acc >= 0) {
+        // (n_min and kappa are uniform over the launch: one instance runs)
+        if constexpr (kCand) {
+            const int32_t fd = min(n_min, kappa_c);  // the filter may test no more than a candidate needs
+            mine = fd >= 3 ? scan_ends<3, true>(stage, e_lo, e_end, suf, n_min, n_max, tid, lane, bm, kappa_c)
+                           : (fd == 2 ? scan_ends<2, true>(stage, e_lo, e_end, suf, n_min, n_max, tid, lane, bm, kappa_c)
+                                      : scan_ends<1, true>(stage, e_lo, e_end, suf, n_min, n_max, tid, lane, bm, kappa_c));
+        } else {
+            mine = a.n_min >= 3 ? scan_ends<3, false>(stage, e_lo, e_end, suf, n_min, n_max, tid, lane)
+                                : (a.n_min == 2 ? scan_ends<2, false>(stage, e_lo, e_end, suf, n_min, n_max, tid, lane)
+                                                : scan_ends<1, false>(stage, e_lo, e_end, suf, n_min, n_max, tid, lane));
+        }
+        // The ends the append creates, [L_old - 1, L - 1), lie in the window: the leader's warp 0.  In
+        // candidate mode new_c[t] bit i marks end L_old - 1 + 32 t + i as a candidate (warp-uniform).
+        if (kCand && rank == lead && warp == 0 && acc >= 0) {
+#pragma unroll 1
+            for (int t = 0; 32 * t <= acc; ++t) {
+                const int32_t j = lane + 32 * t;
+                bool qual = false;
+                if (j <= acc) {
+                    const int32_t e = L_old - 1 + j;
+                    const int32_t lim = min(n_max, e + 1);
+                    int32_t m = 0;
+#pragma unroll 1
+                    while (m < lim && y[kHalo - 1 + j - m] == suf[-m]) ++m;
+                    if (m >= n_min) {
+                        const uint32_t key = (uint32_t(m) << kKeyShift) | uint32_t(e);
+                        mine = key > mine ? key : mine;
+                    }
+                    qual = m >= kappa_c;
+                }
+                new_c[t] = __ballot_sync(kFull, qual);
+            }
+        } else if (rank == lead && warp == 0 && acc >= 0) {
 #pragma unroll 1
             for (int32_t j = lane; j <= acc; j += kWarp) {
                 const int32_t e = L_old - 1 + j;
@@ -384,6 +510,69 @@ __global__ void __launch_bounds__(kRescanThreads, kRescanMinBlocks) rescan_kerne
     }
     uint32_t key = __reduce_max_sync(kFull, mine);
     if (timed_out) key = kKeyTimeout;
+
+    // ---- candidate mode: this CTA's W most recent marked ends and their continuations (warp 0) ----
+    if constexpr (kCand) {
+        __syncthreads();  // every warp's marks are in the bitmap
+        // Bitmap words from the top, kRescanThreads per pass: thread t holds word top - t; prefix sums of
+        // the popcounts (within the warp, then over the warps) rank its bits after those of higher words.
+        // `found` is CTA-uniform.
+        const int nwords = (e_end - e_lo + 31) >> 5;
+        int found = 0;
+        for (int top = nwords - 1; top >= 0 && found < a.W; top -= kRescanThreads) {
+            const int idx = top - tid;
+            const uint32_t wd = idx >= 0 ? bm[idx] : 0u;
+            const int c = __popc(wd);
+            int incl = c;
+#pragma unroll
+            for (int o_ = 1; o_ < kWarp; o_ <<= 1) {
+                const int t_ = __shfl_up_sync(kFull, incl, o_);
+                if (lane >= o_) incl += t_;
+            }
+            if (lane == kWarp - 1) s_wtot[warp] = incl;
+            __syncthreads();
+            int r = found, total = 0;
+#pragma unroll
+            for (int w = 0; w < kRescanWarps; ++w) {
+                r += w < warp ? s_wtot[w] : 0;
+                total += s_wtot[w];
+            }
+            r += incl - c;
+            uint32_t w2 = wd;
+            while (w2 != 0u && r < a.W) {
+                const int bit = 31 - __clz(w2);
+                w2 &= ~(1u << bit);
+                s_sel[r++] = e_lo + idx * 32 + bit;
+            }
+            found += total;
+            __syncthreads();  // s_wtot is rewritten by the next pass; s_sel is complete after the last
+        }
+        if (warp == 0) {
+            const int nsel = min(found, a.W);
+            // the message: header (count), the ends, then candidate w's D tokens at w D -- from the staged
+            // tile, or past the old length from this warp's window (an end e continues for
+            // min(D, L - 1 - e) tokens, all below L)
+            int32_t *ce = reinterpret_cast<int32_t *>(cstage + 16);
+            int32_t *ct = reinterpret_cast<int32_t *>(cstage + 16 + 16 * ((a.W + 3) / 4));
+            if (lane == 0) *reinterpret_cast<int4 *>(cstage) = make_int4(nsel, 0, 0, 0);
+            if (lane < nsel) ce[lane] = s_sel[lane];
+            const int dw = kWarp / a.D, di = kWarp - dw * a.D;  // (candidate, token) step of 32 slots
+            int w = lane / a.D, i = lane - w * a.D;
+            for (int t = lane; t < nsel * a.D; t += kWarp) {
+                const int32_t ew = s_sel[w];
+                const int32_t p = ew + 1 + i;
+                ct[t] = i < min(a.D, L - 1 - ew) ? (p < L_old ? stage[off + p] : y[kHalo + p - L_old]) : 0;
+                w += dw;
+                i += di;
+                if (i >= a.D) {
+                    i -= a.D;
+                    ++w;
+                }
+            }
+            fence_proxy_async();  // the bulk copy below reads the message through the async proxy
+            __syncwarp();
+        }
+    }
 
     // ---- probe share (unless finished before the wait) ----
     if (warp >= 1) {
@@ -445,7 +634,10 @@ __global__ void __launch_bounds__(kRescanThreads, kRescanMinBlocks) rescan_kerne
     } else if (lane <= kw) {
         st_async_v4(map_to_rank(slot + 16 * lane, lead), cw, done_addr);
     }
+    if (kCand && warp == 0 && lane == 0)  // this CTA's candidates, in one bulk copy
+        bulk_s2c(map_to_rank(cmsgs + size_t(rank) * cl.cslot, lead), cstage, cl.cslot, done_addr);
     if (rank != lead || warp != 0) {
+        if (kCand && warp == 0 && lane == 0) bulk_wait_read();  // the message has been read out
         if (timed_out && lane == 0) {  // copies still in flight get a second bounded wait
             (void)mbar_wait(&bars[0], 0);
             (void)mbar_wait(&bars[1], 0);
@@ -485,25 +677,114 @@ __global__ void __launch_bounds__(kRescanThreads, kRescanMinBlocks) rescan_kerne
     const int32_t n = hit ? int32_t(best >> kKeyShift) : 0;
     const int32_t e = hit ? int32_t(best & kKeyEndMask) : -1;
     const int32_t kappa = a.kappa > 0 ? a.kappa : a.n_min;
-    int32_t mode = SWITCHSD_MODE_NO_REP;
-    if (hit) mode = (n >= kappa && z >= a.logit_tau) ? SWITCHSD_MODE_COPY : SWITCHSD_MODE_REP_NO_COPY;
-    const int32_t len = mode == SWITCHSD_MODE_COPY ? min(a.k, L - 1 - e) : 0;
-    if (lane == 0) {
-        if (a.counters) count_row(a.counters, mode, verifying, a.out_mode[b], acc);  // out_mode: the previous mode
-        a.out_mode[b] = mode;
-        a.out_len[b] = len;
-        a.out_score[b] = z;
-        if (a.out_match_n) a.out_match_n[b] = n;
-        if (a.out_match_end) a.out_match_end[b] = e;
-        if (verifying && !len_ok) a.out_accept[b] = -1;
-        if (a.status) {
-            int32_t st = vst;
-            if (st == SWITCHSD_ROW_OK && timeout) st = SWITCHSD_ROW_TIMEOUT;
-            a.status[b] = st;
+    if constexpr (kCand) {
+        // The row's candidates, most recent first: the appended ends (highest first), then the CTAs' lists
+        // from the leader's (the most recent range) down to CTA 0's.  s_sel[w] is merged candidate w's
+        // source: -1 - j for the appended end L_old - 1 + j, else r kMaxCand + i for entry i of CTA r.
+        auto count_of = [&](int r) {
+            return min(*reinterpret_cast<const int32_t *>(cmsgs + size_t(r) * cl.cslot), a.W);
+        };
+        const int n_new = hit ? __popc(new_c[0]) + __popc(new_c[1]) + __popc(new_c[2]) : 0;
+        int total = n_new;
+        if (hit)
+            for (int r = 0; r < int(C); ++r) total += count_of(r);
+        const int ncand = min(total, a.W);
+        int32_t mode = SWITCHSD_MODE_NO_REP;
+        if (hit) mode = (ncand > 0 && z >= a.logit_tau) ? SWITCHSD_MODE_COPY : SWITCHSD_MODE_REP_NO_COPY;
+        const int nc = mode == SWITCHSD_MODE_COPY ? ncand : 0;
+        if (lane < nc) {
+            int src = 0;
+            if (lane < n_new) {
+                int k = lane, j = -1;
+                for (int t = 2; t >= 0 && j < 0; --t) {
+                    const int pc = __popc(new_c[t]);
+                    if (k < pc) {
+                        uint32_t mm = new_c[t];
+                        for (int q = 0; q < k; ++q) mm &= ~(1u << (31 - __clz(mm)));
+                        j = 32 * t + 31 - __clz(mm);
+                    } else {
+                        k -= pc;
+                    }
+                }
+                src = -1 - j;
+            } else {
+                int k = lane - n_new, r = int(C) - 1;
+                for (; r > 0; --r) {
+                    const int cr = count_of(r);
+                    if (k < cr) break;
+                    k -= cr;
+                }
+                src = r * kMaxCand + k;
+            }
+            s_sel[lane] = src;
         }
+        __syncwarp();
+        const int cwE = (a.W + 3) / 4;
+        auto cand_end = [&](int src) -> int32_t {
+            if (src < 0) return L_old - 2 - src;  // L_old - 1 + j with j = -1 - src
+            const int r = src / kMaxCand;
+            return reinterpret_cast<const int32_t *>(cmsgs + size_t(r) * cl.cslot + 16)[src - r * kMaxCand];
+        };
+        if (lane < nc) a.out_cand_len[size_t(b) * a.W + lane] = min(a.D, L - 1 - cand_end(s_sel[lane]));
+        const int dw = kWarp / a.D, di = kWarp - dw * a.D;  // (candidate, token) step of 32 slots
+        int w = lane / a.D, i = lane - w * a.D;
+        for (int t = lane; t < nc * a.D; t += kWarp, w += dw, i += di) {
+            if (i >= a.D) {
+                i -= a.D;
+                ++w;
+            }
+            const int src = s_sel[w];
+            const int32_t ew = cand_end(src);
+            if (i < min(a.D, L - 1 - ew)) {
+                int32_t tok;
+                if (src < 0) {
+                    tok = y[kHalo + ew + 1 + i - L_old];
+                } else {
+                    const int r = src / kMaxCand;
+                    tok = reinterpret_cast<const int32_t *>(cmsgs + size_t(r) * cl.cslot + 16 + 16 * cwE)
+                        [(src - r * kMaxCand) * a.D + i];
+                }
+                a.out_cand[(size_t(b) * a.W + w) * a.D + i] = tok;
+            }
+        }
+        if (lane == 0) {
+            a.out_mode[b] = mode;
+            a.out_score[b] = z;
+            a.out_ncand[b] = nc;
+            if (a.out_match_n) a.out_match_n[b] = n;
+            if (a.out_match_end) a.out_match_end[b] = e;
+            if (verifying && !len_ok) a.out_accept[b] = -1;
+            if (verifying && a.out_choice) a.out_choice[b] = len_ok ? choice : 0;
+            if (a.status) {
+                int32_t st = vst;
+                if (st == SWITCHSD_ROW_OK && timeout) st = SWITCHSD_ROW_TIMEOUT;
+                a.status[b] = st;
+            }
+            bulk_wait_read();  // the leader's own message has been read out
+        }
+        (void)win;
+    } else {
+        const int32_t kappa = a.kappa > 0 ? a.kappa : a.n_min;
+        int32_t mode = SWITCHSD_MODE_NO_REP;
+        if (hit) mode = (n >= kappa && z >= a.logit_tau) ? SWITCHSD_MODE_COPY : SWITCHSD_MODE_REP_NO_COPY;
+        const int32_t len = mode == SWITCHSD_MODE_COPY ? min(a.k, L - 1 - e) : 0;
+        if (lane == 0) {
+            if (a.counters) count_row(a.counters, mode, verifying, a.out_mode[b], acc);  // out_mode: the previous mode
+            a.out_mode[b] = mode;
+            a.out_len[b] = len;
+            a.out_score[b] = z;
+            if (a.out_match_n) a.out_match_n[b] = n;
+            if (a.out_match_end) a.out_match_end[b] = e;
+            if (verifying && !len_ok) a.out_accept[b] = -1;
+            if (a.status) {
+                int32_t st = vst;
+                if (st == SWITCHSD_ROW_OK && timeout) st = SWITCHSD_ROW_TIMEOUT;
+                a.status[b] = st;
+            }
+        }
+        const int32_t *wd = reinterpret_cast<const int32_t *>(msgs + size_t(win) * slot_bytes + 16);
+        for (int i = lane; i < len; i += kWarp) a.out_draft[size_t(b) * a.k + i] = wd[i];
     }
-    const int32_t *wd = reinterpret_cast<const int32_t *>(msgs + size_t(win) * slot_bytes + 16);
-    for (int i = lane; i < len; i += kWarp) a.out_draft[size_t(b) * a.k + i] = wd[i];
     if (!all_in && lane == 0) (void)mbar_wait(&bars[3], 0);  // messages still in flight: a second bounded wait
     if (timed_out && lane == 0) {
         (void)mbar_wait(&bars[0], 0);
@@ -513,31 +794,38 @@ __global__ void __launch_bounds__(kRescanThreads, kRescanMinBlocks) rescan_kerne
 }
 
 size_t rescan_smem_bytes(const StepArgs &args, int split) {
+    const bool cand = args.W > 0;
     const size_t stage = size_t((kHalo + args.tile + kFwd + 3) & ~3) * sizeof(int32_t);
     const size_t probe = 2 * size_t(args.probe_words) * 16;
-    const size_t msgs = size_t(split) * kRescanWarps * 16 * size_t(1 + ((args.k + 3) >> 2));
-    return stage + probe + msgs;
+    const size_t msgs = size_t(split) * kRescanWarps * 16 * size_t(1 + (cand ? 0 : ((args.k + 3) >> 2)));
+    if (!cand) return stage + probe + msgs;
+    const CandLayout c = cand_layout(args.tile, args.W, args.D);
+    return stage + probe + msgs + size_t(split + 1) * c.cslot + size_t(c.bm_words + c.v_ints) * sizeof(int32_t);
 }
 
-template <bool kSampled>
+template <bool kSampled, bool kCand>
 static cudaError_t launch_rescan(const StepArgs &args, int split, cudaStream_t stream) {
     static bool attr_done[64] = {false};
     int dev = 0;
     cudaGetDevice(&dev);
     if (dev >= 0 && dev < 64 && !attr_done[dev]) {
-        cudaError_t e = cudaFuncSetAttribute(rescan_kernel<kSampled>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
+        cudaError_t e = cudaFuncSetAttribute(rescan_kernel<kSampled, kCand>,
+                                             cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
         if (e != cudaSuccess) return e;
-        e = cudaFuncSetAttribute(rescan_kernel<kSampled>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+        e = cudaFuncSetAttribute(rescan_kernel<kSampled, kCand>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                  int(kRescanSmemBudget));
         if (e != cudaSuccess) return e;
         attr_done[dev] = true;
     }
-    return launch_pdl(rescan_kernel<kSampled>, dim3(unsigned(split), unsigned(args.B), 1), dim3(kRescanThreads, 1, 1),
-                      rescan_smem_bytes(args, split), stream, unsigned(split), args);
+    return launch_pdl(rescan_kernel<kSampled, kCand>, dim3(unsigned(split), unsigned(args.B), 1),
+                      dim3(kRescanThreads, 1, 1), rescan_smem_bytes(args, split), stream, unsigned(split), args);
 }
 
 cudaError_t launch_rescan_kernel(const StepArgs &args, int split, cudaStream_t stream) {
-    return args.pv_p != nullptr ? launch_rescan<true>(args, split, stream) : launch_rescan<false>(args, split, stream);
+    // candidate verification is greedy (the candidates' targets are compared token by token)
+    if (args.W > 0) return launch_rescan<false, true>(args, split, stream);
+    return args.pv_p != nullptr ? launch_rescan<true, false>(args, split, stream)
+                                : launch_rescan<false, false>(args, split, stream);
 }
 
 }  // namespace switchsd

@@ -382,11 +382,12 @@ __global__ void __launch_bounds__(kStepThreads) step_kernel(const StepArgs a) {
     if (gather && !(warp == 1 && lane == 0)) h4 += size_t(acc > 0 ? acc : 0) * size_t(a.d >> 3);
     const int32_t s0 = s_suf[0], s1 = s_suf[1];
     const int32_t n_max = a.n_max, n_min = a.n_min;
-    // With n_min >= 2 a candidate must match the last two tokens, so the filter tests both (exact:
-    // the back-compare then starts at m = 2).  m0 is the length the filter has already checked.
-    const bool pair = n_min >= 2;
-    const int32_t m0 = pair ? 2 : 1;
+    // With n_min >= 2 a match must cover the last two tokens, so the filter tests both (exact: the
+    // back-compare then starts at m = 2) -- unless, in candidate mode, a candidate needs only one
+    // (kappa = 1).  m0 is the length the filter has already checked.
     const int32_t kappa_c = a.kappa > 0 ? a.kappa : n_min;  // candidate mode: the gate length
+    const bool pair = n_min >= 2 && (!kCand || kappa_c >= 2);
+    const int32_t m0 = pair ? 2 : 1;
     unsigned long long best = 0;  // CTA-uniform; real keys have m >= n_min >= 1, so 0 = no match
     bool bad = s_ver[3] == 0;     // CTA-uniform: a copy did not land in time
     for (int t = 0; t < ntiles && !bad; ++t) {

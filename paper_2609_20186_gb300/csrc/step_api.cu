@@ -246,13 +246,14 @@ static int step_entry(int32_t *ctx_tokens, int32_t *ctx_lens, const uint16_t *hi
     }
 
     args.b2 = p->b2;
-    // The rescan kernel takes the step without candidates or index (linear probe, or the two-layer
-    // probe's finish after its first-layer kernel); the step kernel takes the rest.
+    // The rescan kernel takes the step without the index -- single draft or W candidates, linear probe or
+    // the two-layer probe's finish after its first-layer kernel -- when the row's range fits its shared
+    // memory; the step kernel takes the rest.
     const bool mlp_probe = p->probe_kind == SWITCHSD_PROBE_MLP;
     const int rsplit = p->split > 0 ? p->split : choose_rescan_split(p->B, p->cap);
     StepArgs ra = args;
     bool rescan = false;
-    if (cs == nullptr && p->index == nullptr && p->cap <= kRescanCapMax) {
+    if (p->index == nullptr && p->cap <= kRescanCapMax) {
         const int64_t rrange = ((int64_t(p->cap) - 1 + rsplit - 1) / rsplit + 3) / 4 * 4;
         const int nv = p->d >> 3;
         const int vper = (nv + rsplit - 1) / rsplit;
@@ -260,9 +261,12 @@ static int step_entry(int32_t *ctx_tokens, int32_t *ctx_lens, const uint16_t *hi
         ra.stages = 1;
         ra.probe_words = mlp_probe ? 0 : (vper < kProbeStage ? vper : kProbeStage);
         ra.msg_wait_polls = msg_wait_polls();
-        ra.W = ra.D = ra.bm_words = 0;
-        ra.out_cand = ra.out_cand_len = ra.out_ncand = ra.out_choice = nullptr;
-        ra.pv_cand_len = nullptr;
+        ra.bm_words = 0;  // the rescan kernel sizes its own bitmap from the tile
+        if (cs == nullptr) {
+            ra.W = ra.D = 0;
+            ra.out_cand = ra.out_cand_len = ra.out_ncand = ra.out_choice = nullptr;
+            ra.pv_cand_len = nullptr;
+        }
         rescan = rrange <= kRescanTileMax && rescan_smem_bytes(ra, rsplit) <= kRescanSmemBudget;
     }
     if (mlp_probe) {

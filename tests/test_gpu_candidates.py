@@ -176,6 +176,26 @@ def test_candidates_lockstep(name, Wc, D, fused):
     assert checked > 0
 
 
+KAPPA_LOW = {
+    "zipf_kappa2": W["zipf_32k"].scaled(name="zipf_kappa2", B=4, L0=20003, steps=8, kappa=2),
+    "code_kappa1": W["code_16k"].scaled(name="code_kappa1", B=4, L0=20003, steps=6, kappa=1),
+}
+
+
+@pytest.mark.parametrize("split", [0, 1], ids=["rescan_kernel", "step_kernel"])
+@pytest.mark.parametrize("name", list(KAPPA_LOW))
+def test_candidates_kappa_below_n_min(name, split):
+    """kappa below n_min on the scan path: a candidate needs only kappa tokens of common suffix, fewer
+    than a match that decides the mode, so the scan's filter must not test more than kappa tokens.  The
+    library's split takes the rescan kernel; one CTA over 20K-token rows takes the step kernel."""
+    wl = KAPPA_LOW[name]
+    rows = range(wl.B)
+    o_trace, o_ctx = oracle_loop(wl, rows, wl.steps, 10, 20)
+    g_trace, g_ctx = gpu_loop(wl, wl.steps, 10, 20, split=split, fused=True)
+    checked, copies = compare(wl, o_trace, g_trace, rows, o_ctx, g_ctx)
+    assert checked > 0 and copies > 0
+
+
 @pytest.mark.parametrize("split", [1, 2, 4, 8, 16])
 def test_candidates_split_invariance(split):
     wl = SMALL["zipf_small"]
