@@ -127,8 +127,13 @@ typedef struct switchsd_index switchsd_index;
  *                and the target argmax are always read after the wait.  The index search reads the
  *                row's length and tail (CONTEXT) and computes the linear probe (PROBE) before the wait;
  *                its tables come after it.  With the two-layer probe SWITCHSD_PREFETCH_PROBE lets the
- *                probe kernel's copies of the hidden states and W1 start early.  Other bits are
- *                SWITCHSD_ERR_ARG.
+ *                probe kernel's copies of the hidden states and W1 and its MMAs start early, and that
+ *                kernel then releases the call's step kernel at once (whose reads before its own wait
+ *                are still only those the bits name; its wait covers the probe kernel, whose stores
+ *                follow that kernel's wait).  A call's kernels write the workspace, the outputs and, when
+ *                verifying, the context and lengths; the call's last kernel may release the next kernel
+ *                on the stream before the first-layer probe kernel of the same call has finished, which
+ *                writes only the workspace.  Other bits are SWITCHSD_ERR_ARG.
  *   hidden_rows  0 or 1: hidden is [B, d], the state the probe reads for each row.  k + 1 (the fused
  *                switchsd_verify_step and switchsd_verify_sampled_step only): hidden is the
  *                target's verification output [B, k+1, d] and the probe reads row a_b of each row b --

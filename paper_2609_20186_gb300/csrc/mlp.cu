@@ -105,16 +105,22 @@ __global__ void __launch_bounds__(kMlpThreads) mlp_tc_kernel(const __grid_consta
         if (a.prefetch)
             for (int c = 0; c < first; ++c) issue(c);
     }
+    // With the prefetch bit this kernel reads nothing the preceding kernel writes, and the step kernel it
+    // releases reads before its own wait only what the caller's prefetch bits cover: both start at once.
+    // That kernel's wait covers this whole grid, whose stores follow this grid's own wait below.
+    if (a.prefetch) pdl_trigger();
     if (warp == 0) {
         asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;\n" ::"r"(smem_addr(&s_tmem)),
                      "r"(kTmemCols)
                      : "memory");
         asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;\n" ::: "memory");
     }
-    pdl_wait();     // the partial sums below overwrite what an earlier step kernel may still read
-    pdl_trigger();
-    if (tid == 0 && !a.prefetch)
-        for (int c = 0; c < first; ++c) issue(c);
+    if (!a.prefetch) {
+        pdl_wait();  // the operands may come from the preceding kernel
+        pdl_trigger();
+        if (tid == 0)
+            for (int c = 0; c < first; ++c) issue(c);
+    }
     asm volatile("tcgen05.fence::before_thread_sync;\n" ::: "memory");
     __syncthreads();
     asm volatile("tcgen05.fence::after_thread_sync;\n" ::: "memory");
@@ -194,6 +200,9 @@ __global__ void __launch_bounds__(kMlpThreads) mlp_tc_kernel(const __grid_consta
     // that each warp store writes two whole 256-byte rows instead of one 16-byte piece of 32 rows.  Row r
     // keeps its 16-byte chunk q at position q ^ (r % 16): both the row-wise writes below and the reads
     // across rows hit distinct banks.
+    // The partial sums overwrite what an earlier step kernel may still read: with the prefetch bit the
+    // copies and the MMAs above ran before the wait, the stores come after it.
+    if (a.prefetch) pdl_wait();
     float4 *tile = reinterpret_cast<float4 *>(base);  // [kMlpM rows][16 chunks]
 #pragma unroll
     for (int q = 0; q < kMlpN / 4; ++q)

@@ -19,7 +19,8 @@ bool mlp_shape_ok(int d, int H1);
 int mlp_hidden_padded(int H1);
 // part [mlp_split(d)][B][mlp_hidden_padded(H1)] <- split-K partial sums of W1 h (fp32; units >= H1 are
 // zero).  Launched with programmatic stream serialization; prefetch: the hidden states and W1 may be
-// read before the preceding kernel finishes (the caller's guarantee, SWITCHSD_PREFETCH_PROBE).  stages:
+// read (and the MMAs run) before the preceding kernel finishes (the caller's guarantee,
+// SWITCHSD_PREFETCH_PROBE), and the next kernel is released at once; the stores wait.  stages:
 // operand chunks staged at once per CTA (0 or >= the CTA's chunks: all of them; fewer leave shared memory
 // to a kernel that runs beside this one).
 cudaError_t launch_mlp_tc(const uint16_t *hidden, const uint16_t *W1, float *part, int B, int d, int H1,

@@ -269,6 +269,7 @@ static int step_entry(int32_t *ctx_tokens, int32_t *ctx_lens, const uint16_t *hi
         }
         rescan = rrange <= kRescanTileMax && rescan_smem_bytes(ra, rsplit) <= kRescanSmemBudget;
     }
+    bool mlp_early = false;  // the first-layer kernel releases the step kernel at its start
     if (mlp_probe) {
         float *part = static_cast<float *>(p->workspace);
         const uint16_t *probe_in = hidden;
@@ -302,6 +303,7 @@ static int step_entry(int32_t *ctx_tokens, int32_t *ctx_lens, const uint16_t *hi
                           rescan ? kMlpStagesBeside : 0) != cudaSuccess)
             return SWITCHSD_ERR_CUDA;
         args.z1_part = part;
+        mlp_early = probe_pf;
         args.b1 = p->b1;
         args.w2 = probe_w + size_t(p->probe_hidden) * size_t(p->d);
         args.mlp_S = mlp_split(p->d);
@@ -333,9 +335,11 @@ static int step_entry(int32_t *ctx_tokens, int32_t *ctx_lens, const uint16_t *hi
         ra.H1 = args.H1;
         ra.H1p = args.H1p;
         ra.hidden_rows = args.hidden_rows;
-        // the first-layer kernel launched just above waits for every earlier kernel before it releases
-        // this one, so only its own output, the partial sums, needs this launch's wait
-        ra.wait_late = args.z1_part != nullptr ? 1 : 0;
+        // Without the probe prefetch the first-layer kernel launched just above waits for every earlier
+        // kernel before it releases this one, so only its own output, the partial sums, needs this
+        // launch's wait.  With it, that kernel releases this one at its start: this launch then reads
+        // before its wait only what the caller's prefetch bits cover, and everything else after it.
+        ra.wait_late = (args.z1_part != nullptr && !mlp_early) ? 1 : 0;
         if (launch_rescan_kernel(ra, rsplit, stream) != cudaSuccess) return SWITCHSD_ERR_CUDA;
         return SWITCHSD_OK;
     }
