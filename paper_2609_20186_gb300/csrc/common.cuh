@@ -41,6 +41,12 @@ __device__ __forceinline__ void mbar_arrive_expect_tx(uint64_t *bar, uint32_t by
                  : "memory");
 }
 
+// A plain arrive (release at CTA scope): the arriving thread's earlier shared-memory writes are visible to a
+// thread that then observes the phase complete.
+__device__ __forceinline__ void mbar_arrive(uint64_t *bar) {
+    asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];\n" ::"r"(smem_addr(bar)) : "memory");
+}
+
 // The same for a barrier that only counts an asynchronous copy's bytes: the arriving thread publishes
 // nothing through it, so the arrive needs no release ordering.
 __device__ __forceinline__ void mbar_expect_tx_relaxed(uint64_t *bar, uint32_t bytes) {

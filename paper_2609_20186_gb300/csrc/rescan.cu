@@ -9,7 +9,7 @@
 // candidate ends [0, L_old - 1) are split into C contiguous 16-byte-aligned ranges; each CTA stages its
 // range (plus kHalo tokens of look-back and kFwd of look-ahead) with one bulk copy, and the row's last
 // kHalo tokens with another, as soon as it has read the row length -- before the grid-dependency wait
-// when the caller allows it.  The CTAs are small (four warps, at most 72 registers a thread) so that the
+// when the caller allows it.  The CTAs are small (four warps, at most 64 registers a thread) so that the
 // next launch's CTAs are resident, with their copies in flight, while this launch finishes.
 //
 // After the wait there is no CTA-wide or cluster-wide barrier on the path:
@@ -26,6 +26,8 @@
 // them in a fixed order and writes the outputs.  The only cluster barrier is arrived on right after the
 // length read and waited on just before the first message, so the leader's message barrier is
 // initialised before anyone ships to it and no CTA reads the length after the leader rewrites it.
+#include <mutex>
+
 #include "mlp.cuh"
 #include "step.cuh"
 
@@ -64,93 +66,163 @@ static_assert(kRescanTileMax / 4 / (kScanWords * kRescanThreads) <= 32, "a threa
 // eight positions per step with independent loads.
 constexpr uint32_t kHashA = 0x9E3779B1u, kHashB = 0x85EBCA77u;  // odd multipliers
 
+// The F-token hash of end e (x0 = x[e], x1 = x[e-1], x2 = x[e-2]; the first F terms, mod 2^32).
+template <int F>
+__device__ __forceinline__ uint32_t end_hash(int32_t x0, int32_t x1, int32_t x2) {
+    uint32_t h = uint32_t(x0);
+    if (F >= 2) h += uint32_t(x1) * kHashA;
+    if (F >= 3) h += uint32_t(x2) * kHashB;
+    return h;
+}
+// One byte of it for the pre-wait table (multiplicative: the top byte of an odd multiple).
+__device__ __forceinline__ uint32_t hash_byte(uint32_t h) { return (h * 0x2C1B3C6Du) >> 24; }
+// Nonzero iff some byte of v is zero (exact as a whole-word test).
+__device__ __forceinline__ uint32_t has_zero_byte(uint32_t v) { return (v - 0x01010101u) & ~v & 0x80808080u; }
+
+// Pre-wait hashing: hb[g] holds the hash bytes of the ends e_lo + 4g .. + 3 (byte j = end e_lo + 4g + j),
+// for the words g < n4 of this CTA's old ends; threads t, t + nt, ... of the caller take one word each.
+template <int F>
+__device__ __forceinline__ void hash_ends(const int32_t *stage, uint32_t *hb, int32_t n4, int t, int nt) {
+    const int4 *g4 = reinterpret_cast<const int4 *>(stage + kHalo);
+    for (int32_t g = t; g < n4; g += nt) {
+        const int4 v = g4[g];
+        const int2 pv = F >= 2 ? *reinterpret_cast<const int2 *>(stage + kHalo + 4 * g - 2) : make_int2(0, 0);
+        hb[g] = hash_byte(end_hash<F>(v.x, pv.y, pv.x)) | hash_byte(end_hash<F>(v.y, v.x, pv.y)) << 8 |
+                hash_byte(end_hash<F>(v.z, v.y, v.x)) << 16 | hash_byte(end_hash<F>(v.w, v.z, v.y)) << 24;
+    }
+}
+
 //
 // Candidate mode (kCand): every end whose common suffix reaches kappa_c is also marked in the CTA's bitmap
 // bm (bit e - e_lo; F <= kappa_c, so the filter passes every such end).
-template <int F, bool kCand>
+//
+// kPre: the hashes were taken before the grid-dependency wait (hash_ends into hb); pass 1 then compares
+// one byte per end against the suffix's (four ends a 4-byte load), and pass 2 takes only the ends whose
+// byte matches.  The byte filter passes every end that matches and about 1 in 256 of the others, which
+// the exact test drops.
+template <int F, bool kCand, bool kPre>
 __device__ __forceinline__ uint32_t scan_ends(const int32_t *stage, int32_t e_lo, int32_t e_end, const int32_t *suf,
                                               int32_t n_min, int32_t n_max, int tid, int lane,
-                                              uint32_t *bm = nullptr, int32_t kappa_c = 0) {
+                                              uint32_t *bm = nullptr, int32_t kappa_c = 0,
+                                              const uint32_t *hb = nullptr) {
     const int32_t s0 = suf[0], s1 = F >= 2 ? suf[-1] : 0, s2 = F >= 3 ? suf[-2] : 0;
-    const uint32_t hs = uint32_t(s0) + (F >= 2 ? uint32_t(s1) * kHashA : 0u) + (F >= 3 ? uint32_t(s2) * kHashB : 0u);
+    const uint32_t hs = end_hash<F>(s0, s1, s2);
+    const uint32_t hs4 = hash_byte(hs) * 0x01010101u;
     const int32_t n4 = (e_end - e_lo + 3) >> 2;
     const int4 *g4 = reinterpret_cast<const int4 *>(stage + kHalo);
     const int32_t off = kHalo - e_lo;
-    auto hash = [&](int32_t x0, int32_t x1, int32_t x2) {  // x0 = x[e], x1 = x[e-1], x2 = x[e-2]
-        uint32_t h = uint32_t(x0);
-        if (F >= 2) h += uint32_t(x1) * kHashA;
-        if (F >= 3) h += uint32_t(x2) * kHashB;
-        return h ^ hs;
-    };
     uint32_t passed = 0u;
     int rnd = 0;
-    for (int32_t g0 = tid; g0 - lane < n4; g0 += kScanWords * kRescanThreads, ++rnd) {
-        int4 v[kScanWords];
-        int2 pv[kScanWords];  // x[4g - 2], x[4g - 1]
+    if constexpr (kPre) {
+        for (int32_t g0 = tid; g0 - lane < n4; g0 += kScanWords * kRescanThreads, ++rnd) {
+            uint32_t z = 0u;
 #pragma unroll
-        for (int u = 0; u < kScanWords; ++u) {
-            const int32_t g = g0 + u * kRescanThreads;
-            v[u] = g < n4 ? g4[g] : make_int4(0, 0, 0, 0);
-            pv[u] = (F >= 2 && g < n4) ? *reinterpret_cast<const int2 *>(stage + kHalo + 4 * g - 2) : make_int2(0, 0);
+            for (int u = 0; u < kScanWords; ++u) {
+                const int32_t g = g0 + u * kRescanThreads;
+                z |= g < n4 ? has_zero_byte(hb[g] ^ hs4) : 0u;
+            }
+            passed |= uint32_t(z != 0u) << (rnd & 31);
         }
-        uint32_t mn = 0xffffffffu;
+    } else {
+        auto hash = [&](int32_t x0, int32_t x1, int32_t x2) { return end_hash<F>(x0, x1, x2) ^ hs; };
+        for (int32_t g0 = tid; g0 - lane < n4; g0 += kScanWords * kRescanThreads, ++rnd) {
+            int4 v[kScanWords];
+            int2 pv[kScanWords];  // x[4g - 2], x[4g - 1]
 #pragma unroll
-        for (int u = 0; u < kScanWords; ++u) {
-            const uint32_t h0 = hash(v[u].x, pv[u].y, pv[u].x), h1 = hash(v[u].y, v[u].x, pv[u].y);
-            const uint32_t h2 = hash(v[u].z, v[u].y, v[u].x), h3 = hash(v[u].w, v[u].z, v[u].y);
-            mn = __vimin3_u32(mn, __vimin3_u32(h0, h1, h2), h3);
+            for (int u = 0; u < kScanWords; ++u) {
+                const int32_t g = g0 + u * kRescanThreads;
+                v[u] = g < n4 ? g4[g] : make_int4(0, 0, 0, 0);
+                pv[u] = (F >= 2 && g < n4) ? *reinterpret_cast<const int2 *>(stage + kHalo + 4 * g - 2) : make_int2(0, 0);
+            }
+            uint32_t mn = 0xffffffffu;
+#pragma unroll
+            for (int u = 0; u < kScanWords; ++u) {
+                const uint32_t h0 = hash(v[u].x, pv[u].y, pv[u].x), h1 = hash(v[u].y, v[u].x, pv[u].y);
+                const uint32_t h2 = hash(v[u].z, v[u].y, v[u].x), h3 = hash(v[u].w, v[u].z, v[u].y);
+                mn = __vimin3_u32(mn, __vimin3_u32(h0, h1, h2), h3);
+            }
+            passed |= uint32_t(mn == 0u) << (rnd & 31);
         }
-        passed |= uint32_t(mn == 0u) << (rnd & 31);
     }
     uint32_t mine = 0u;
+    // m(e) from F for an end whose last F tokens match: x[e - q] against suf[-q], eight positions per step,
+    // every load issued unconditionally (q clamped to lim - 1; the sentinel bit ends the run at the count)
+    auto match_len = [&](int32_t e, int32_t lim) {
+        int32_t m = F;
+#pragma unroll 1
+        while (m < lim) {
+            const int32_t cnt = min(8, lim - m);
+            unsigned miss = 1u << cnt;
+#pragma unroll
+            for (int i = 0; i < 8; ++i) {
+                const int32_t q = min(m + i, lim - 1);
+                miss |= unsigned(stage[off + e - q] != suf[-q]) << i;
+            }
+            const int32_t run = __ffs(miss) - 1;
+            m += run;
+            if (run < cnt) break;
+        }
+        return m;
+    };
+    auto take = [&](int32_t e, int32_t m) {
+        if (m >= n_min) {
+            const uint32_t key = (uint32_t(m) << kKeyShift) | uint32_t(e);
+            mine = key > mine ? key : mine;
+        }
+        if (kCand && m >= kappa_c) atomicOr(&bm[(e - e_lo) >> 5], 1u << ((e - e_lo) & 31));
+    };
     while (__any_sync(kFull, passed != 0u)) {
         if (passed == 0u) continue;
         const int r = __ffs(passed) - 1;
         passed &= passed - 1u;
-#pragma unroll 1
-        for (int u = 0; u < kScanWords; ++u) {
-            const int32_t g = tid + r * kScanWords * kRescanThreads + u * kRescanThreads;
-            if (g >= n4) break;
-            const int4 v = g4[g];
-            const int2 pv = *reinterpret_cast<const int2 *>(stage + kHalo + 4 * g - 2);
-            // exact test of the last F tokens of each end
-            const int32_t x[6] = {pv.x, pv.y, v.x, v.y, v.z, v.w};
-            uint32_t hall = 0u;
+        if constexpr (kPre) {
+            // the round's ends whose hash byte matches: bit 4u + j for end j of word u
+            uint32_t cand = 0u;
 #pragma unroll
-            for (int j = 0; j < 4; ++j) {
-                bool ok = x[j + 2] == s0;
-                if (F >= 2) ok = ok && x[j + 1] == s1;
-                if (F >= 3) ok = ok && x[j] == s2;
-                hall |= uint32_t(ok) << j;
+            for (int u = 0; u < kScanWords; ++u) {
+                const int32_t g = tid + r * kScanWords * kRescanThreads + u * kRescanThreads;
+                const uint32_t eq = g < n4 ? __vcmpeq4(hb[g], hs4) : 0u;  // 0xff in each matching byte
+                cand |= ((eq & 1u) | (eq >> 7 & 2u) | (eq >> 14 & 4u) | (eq >> 21 & 8u)) << (4 * u);
             }
-            while (hall) {
-                const int j = __ffs(hall) - 1;
-                hall &= hall - 1;
-                const int32_t e = e_lo + 4 * g + j;
+            while (cand) {
+                const int i = __ffs(cand) - 1;
+                cand &= cand - 1u;
+                const int32_t g = tid + r * kScanWords * kRescanThreads + (i >> 2) * kRescanThreads;
+                const int32_t e = e_lo + 4 * g + (i & 3);
                 if (e >= e_end) break;
                 const int32_t lim = min(n_max, e + 1);
-                if (lim < F) continue;  // the test read a token before position 0
-                // m(e) from F: x[e - q] against suf[-q], eight positions per step, every load issued
-                // unconditionally (q clamped to lim - 1; the sentinel bit ends the run at the count)
-                int32_t m = F;
+                if (lim < F) continue;  // the hash read a token before position 0
+                bool ok = stage[off + e] == s0;
+                if (F >= 2) ok = ok && stage[off + e - 1] == s1;
+                if (F >= 3) ok = ok && stage[off + e - 2] == s2;
+                if (ok) take(e, match_len(e, lim));
+            }
+        } else {
 #pragma unroll 1
-                while (m < lim) {
-                    const int32_t cnt = min(8, lim - m);
-                    unsigned miss = 1u << cnt;
+            for (int u = 0; u < kScanWords; ++u) {
+                const int32_t g = tid + r * kScanWords * kRescanThreads + u * kRescanThreads;
+                if (g >= n4) break;
+                const int4 v = g4[g];
+                const int2 pv = *reinterpret_cast<const int2 *>(stage + kHalo + 4 * g - 2);
+                // exact test of the last F tokens of each end
+                const int32_t x[6] = {pv.x, pv.y, v.x, v.y, v.z, v.w};
+                uint32_t hall = 0u;
 #pragma unroll
-                    for (int i = 0; i < 8; ++i) {
-                        const int32_t q = min(m + i, lim - 1);
-                        miss |= unsigned(stage[off + e - q] != suf[-q]) << i;
-                    }
-                    const int32_t run = __ffs(miss) - 1;
-                    m += run;
-                    if (run < cnt) break;
+                for (int j = 0; j < 4; ++j) {
+                    bool ok = x[j + 2] == s0;
+                    if (F >= 2) ok = ok && x[j + 1] == s1;
+                    if (F >= 3) ok = ok && x[j] == s2;
+                    hall |= uint32_t(ok) << j;
                 }
-                if (m >= n_min) {
-                    const uint32_t key = (uint32_t(m) << kKeyShift) | uint32_t(e);
-                    mine = key > mine ? key : mine;
+                while (hall) {
+                    const int j = __ffs(hall) - 1;
+                    hall &= hall - 1;
+                    const int32_t e = e_lo + 4 * g + j;
+                    if (e >= e_end) break;
+                    const int32_t lim = min(n_max, e + 1);
+                    if (lim < F) continue;  // the test read a token before position 0
+                    take(e, match_len(e, lim));
                 }
-                if (kCand && m >= kappa_c) atomicOr(&bm[(e - e_lo) >> 5], 1u << ((e - e_lo) & 31));
             }
         }
     }
@@ -176,10 +248,13 @@ __host__ __device__ inline CandLayout cand_layout(int tile, int W, int D) {
     return c;
 }
 
-template <bool kSampled, bool kCand>
-__global__ void __launch_bounds__(kRescanThreads, kRescanMinBlocks) rescan_kernel(const StepArgs a) {
+// kPre: the pre-wait hash table (a.hash_words > 0); kMlp: the two-layer probe's finish (a.z1_part set).
+// Separate instances, so that each carries only its own scan and its own probe code and registers.
+template <bool kSampled, bool kCand, bool kPre, bool kMlp>
+__global__ void __launch_bounds__(kRescanThreads, kRescanLaunchBlocks) rescan_kernel(const StepArgs a) {
     extern __shared__ __align__(128) int32_t dsm[];
-    __shared__ __align__(8) uint64_t bars[4];              // tile, tail, probe slices, messages (leader)
+    __shared__ __align__(8) uint64_t bars[5];              // tile, tail, probe slices, messages (leader),
+                                                           // pre-wait hashes
     __shared__ __align__(16) int32_t s_tail[kHalo + 8];    // x[tail_lo .. L_old), tail_lo = roundown4(L_old - kHalo)
     __shared__ int32_t s_y[kRescanWarps][kYLen];
     __shared__ int32_t s_sel[kMaxCand];                    // candidate mode: the CTA's selected ends / the
@@ -193,7 +268,8 @@ __global__ void __launch_bounds__(kRescanThreads, kRescanMinBlocks) rescan_kerne
     const int b = blockIdx.y;
     const int stage_ints = kHalo + a.tile + kFwd;
     int32_t *stage = dsm;
-    uint4 *s_pw = reinterpret_cast<uint4 *>(dsm + ((stage_ints + 3) & ~3));
+    uint32_t *hb = reinterpret_cast<uint32_t *>(dsm + ((stage_ints + 3) & ~3));  // [hash_words]
+    uint4 *s_pw = reinterpret_cast<uint4 *>(hb + a.hash_words);
     uint4 *s_ph = s_pw + a.probe_words;
     unsigned char *msgs = reinterpret_cast<unsigned char *>(s_ph + a.probe_words);
     const bool verifying = a.pv_len != nullptr;
@@ -212,6 +288,7 @@ __global__ void __launch_bounds__(kRescanThreads, kRescanMinBlocks) rescan_kerne
         mbar_init(&bars[0], 1);
         mbar_init(&bars[1], 1);
         mbar_init(&bars[2], 1);
+        mbar_init(&bars[4], kRescanThreads - kWarp);
         if (rank == lead) {
             mbar_init(&bars[3], 1);
             mbar_arrive_expect_tx(&bars[3], slot_bytes * uint32_t(nmsg) + (kCand ? cl.cslot * C : 0u));
@@ -226,7 +303,7 @@ __global__ void __launch_bounds__(kRescanThreads, kRescanMinBlocks) rescan_kerne
     const bool gather = verifying && a.hidden_rows > 1;
     // Two-layer probe: the first layer's split-K partial sums come from the probe kernel just before this
     // one (read after the wait); this CTA finishes units [u0, u1) (b1, ReLU, w2).
-    const bool mlp = a.z1_part != nullptr;
+    constexpr bool mlp = kMlp;
     const bool pf_probe = (a.prefetch & SWITCHSD_PREFETCH_PROBE) != 0 && !gather && !mlp;
     // Two-layer probe: every input but the partial sums was written by kernels that completed before the
     // first-layer kernel released this launch (it does so only after its own wait), so verification and
@@ -318,9 +395,59 @@ __global__ void __launch_bounds__(kRescanThreads, kRescanMinBlocks) rescan_kerne
     // A prefetched probe is finished before the wait by warps 1.. (its inputs are not written by the
     // preceding kernel); warp 0 goes straight to the wait and releases the next launch.
     if (pf_probe && warp >= 1) probe_dot(h4);
+    // Warps 1.. hash this CTA's old ends once the tile has landed -- before the wait when the context is
+    // prefetched -- so that the scan after it compares one byte per end (scan_ends, kPre).
+    constexpr bool pre = kPre;
+    // the filter depth F (in candidate mode no deeper than the gate length kappa)
+    auto filter_depth = [&]() {
+        return min(kCand ? min(a.n_min, a.kappa > 0 ? a.kappa : a.n_min) : a.n_min, 3);
+    };
+    if (pre && warp >= 1) {
+        const int fdepth = filter_depth();
+        if (len_ok && (hi == lo || mbar_wait(&bars[0], 0))) {
+            const int32_t n4 = (e_end - e_lo + 3) >> 2;
+            if (fdepth >= 3) hash_ends<3>(stage, hb, n4, tid - kWarp, kRescanThreads - kWarp);
+            else if (fdepth == 2) hash_ends<2>(stage, hb, n4, tid - kWarp, kRescanThreads - kWarp);
+            else hash_ends<1>(stage, hb, n4, tid - kWarp, kRescanThreads - kWarp);
+        }
+        mbar_arrive(&bars[4]);  // every thread of warps 1.., whether or not it hashed
+    }
     if (pf_ctx && !late) pdl_wait();
     pdl_trigger();
     if (!pf_probe && !gather && !mlp && tid == 0) issue_probe();
+
+    // Two-layer probe: this CTA finishes units [u0m, u1m) (the S partial sums in order, b1, ReLU, w2);
+    // thread j = tid - 32 of warps 1.. takes units u0m + j, u0m + j + (kT - 32), ...  When this launch's
+    // wait already covers the first-layer kernel (not late), the first unit's partial sums are loaded
+    // now, so that their round trip overlaps the verification's; the sums are taken after it.
+    const int uper = mlp ? (a.H1 + int(C) - 1) / int(C) : 0;
+    const int u0m = min(a.H1, int(rank) * uper), u1m = min(a.H1, u0m + uper);
+    auto mlp_unit = [&](int u, const float *pz, float acc) {
+        float z1 = 0.f;
+#pragma unroll
+        for (int sp = 0; sp < kMaxMlpSplit; ++sp)
+            if (sp < a.mlp_S) z1 += pz[sp];
+        if (a.b1) z1 += a.b1[u];
+        return fmaf(bf16_lo(uint32_t(a.w2[u])), fmaxf(z1, 0.f), acc);
+    };
+    auto mlp_load = [&](int u, float *pz) {
+#pragma unroll
+        for (int sp = 0; sp < kMaxMlpSplit; ++sp)
+            pz[sp] = sp < a.mlp_S ? __ldcg(a.z1_part + (size_t(sp) * a.B + size_t(b)) * a.H1p + u) : 0.f;
+    };
+    // every partial sum of a unit is loaded before the first add (independent L2 reads), then added in
+    // order; the same threads and order either way, so the logit does not depend on when this runs
+    auto mlp_finish = [&](int from) {
+        for (int u = from; u < u1m; u += kRescanThreads - kWarp) {
+            float pz[kMaxMlpSplit];
+            mlp_load(u, pz);
+            zp = mlp_unit(u, pz, zp);
+        }
+    };
+    const bool mlp_early = mlp && !late && warp >= 1;
+    float pz0[kMaxMlpSplit];
+    const int u_first = u0m + tid - kWarp;
+    if (mlp_early && u_first < u1m) mlp_load(u_first, pz0);
 
     // ---- verification of the previous draft (every warp) ----
     int32_t acc = -1, L = L_old, vst = len_ok ? SWITCHSD_ROW_OK : SWITCHSD_ROW_BAD_LEN;
@@ -418,6 +545,10 @@ __global__ void __launch_bounds__(kRescanThreads, kRescanMinBlocks) rescan_kerne
             }
         }
     }
+    if (mlp_early && u_first < u1m) {
+        zp = mlp_unit(u_first, pz0, zp);
+        mlp_finish(u_first + (kRescanThreads - kWarp));
+    }
     // The probed state of a fused verification with hidden_rows = k + 1: row a_b (row 0 when nothing was
     // appended).  Its words are loaded now and used after the scan.
     uint4 gw = make_uint4(0, 0, 0, 0), gh = make_uint4(0, 0, 0, 0);
@@ -458,20 +589,17 @@ __global__ void __launch_bounds__(kRescanThreads, kRescanMinBlocks) rescan_kerne
     // most recent; 0 = no match; kKeyTimeout marks a copy that did not land.
     uint32_t mine = 0;
     const bool tile_in = hi == lo || mbar_wait(&bars[0], 0);
-    bool timed_out = !tail_in || !tile_in;
+    const bool hashed = !pre || mbar_wait(&bars[4], 0);
+    bool timed_out = !tail_in || !tile_in || !hashed;
     const int32_t off = kHalo - e_lo;  // stage[off + p] = x[p] over the staged range
     if (!timed_out && len_ok && L >= 2) {
         // (n_min and kappa are uniform over the launch: one instance runs)
-        if constexpr (kCand) {
-            const int32_t fd = min(n_min, kappa_c);  // the filter may test no more than a candidate needs
-            mine = fd >= 3 ? scan_ends<3, true>(stage, e_lo, e_end, suf, n_min, n_max, tid, lane, bm, kappa_c)
-                           : (fd == 2 ? scan_ends<2, true>(stage, e_lo, e_end, suf, n_min, n_max, tid, lane, bm, kappa_c)
-                                      : scan_ends<1, true>(stage, e_lo, e_end, suf, n_min, n_max, tid, lane, bm, kappa_c));
-        } else {
-            mine = a.n_min >= 3 ? scan_ends<3, false>(stage, e_lo, e_end, suf, n_min, n_max, tid, lane)
-                                : (a.n_min == 2 ? scan_ends<2, false>(stage, e_lo, e_end, suf, n_min, n_max, tid, lane)
-                                                : scan_ends<1, false>(stage, e_lo, e_end, suf, n_min, n_max, tid, lane));
-        }
+        // the filter depth may test no more than a candidate needs (fdepth <= kappa in candidate mode)
+        const int fdepth = filter_depth();
+        mine = fdepth >= 3 ? scan_ends<3, kCand, kPre>(stage, e_lo, e_end, suf, n_min, n_max, tid, lane, bm, kappa_c, hb)
+                           : (fdepth == 2
+                                  ? scan_ends<2, kCand, kPre>(stage, e_lo, e_end, suf, n_min, n_max, tid, lane, bm, kappa_c, hb)
+                                  : scan_ends<1, kCand, kPre>(stage, e_lo, e_end, suf, n_min, n_max, tid, lane, bm, kappa_c, hb));
         // The ends the append creates, [L_old - 1, L - 1), lie in the window: the leader's warp 0.  In
         // candidate mode new_c[t] bit i marks end L_old - 1 + 32 t + i as a candidate (warp-uniform).
         if (kCand && rank == lead && warp == 0 && acc >= 0) {
@@ -576,24 +704,11 @@ __global__ void __launch_bounds__(kRescanThreads, kRescanMinBlocks) rescan_kerne
 
     // ---- probe share (unless finished before the wait) ----
     if (warp >= 1) {
-        if (mlp) {
-            // units u0 + j, u0 + j + (kT - 32), ... for thread j = tid - 32: the S partial sums in order
-            const int uper = (a.H1 + int(C) - 1) / int(C);
-            const int u0 = min(a.H1, int(rank) * uper), u1 = min(a.H1, u0 + uper);
-            if (late) pdl_wait();
-            for (int u = u0 + tid - kWarp; u < u1; u += kRescanThreads - kWarp) {
-                // every partial sum is loaded before the first add (independent L2 reads), then added in order
-                float pz[kMaxMlpSplit];
-#pragma unroll
-                for (int sp = 0; sp < kMaxMlpSplit; ++sp)
-                    pz[sp] = sp < a.mlp_S ? __ldcg(a.z1_part + (size_t(sp) * a.B + size_t(b)) * a.H1p + u) : 0.f;
-                float z1 = 0.f;
-#pragma unroll
-                for (int sp = 0; sp < kMaxMlpSplit; ++sp)
-                    if (sp < a.mlp_S) z1 += pz[sp];
-                if (a.b1) z1 += a.b1[u];
-                zp = fmaf(bf16_lo(uint32_t(a.w2[u])), fmaxf(z1, 0.f), zp);
-            }
+        if (late) {  // the partial sums only now: this launch waits for the first-layer kernel here
+            pdl_wait();
+            mlp_finish(u0m + tid - kWarp);
+        } else if (mlp) {
+            // finished after the verification (mlp_early)
         } else if (gather) {
             zp = dot8_bf16(gw, gh, 0.f);  // zero words for a thread past the slice
             for (int v = v0 + tid - kWarp + (kRescanThreads - kWarp); v < v1; v += kRescanThreads - kWarp)
@@ -796,36 +911,119 @@ __global__ void __launch_bounds__(kRescanThreads, kRescanMinBlocks) rescan_kerne
 size_t rescan_smem_bytes(const StepArgs &args, int split) {
     const bool cand = args.W > 0;
     const size_t stage = size_t((kHalo + args.tile + kFwd + 3) & ~3) * sizeof(int32_t);
-    const size_t probe = 2 * size_t(args.probe_words) * 16;
+    const size_t probe = 2 * size_t(args.probe_words) * 16 + size_t(args.hash_words) * 4;
     const size_t msgs = size_t(split) * kRescanWarps * 16 * size_t(1 + (cand ? 0 : ((args.k + 3) >> 2)));
     if (!cand) return stage + probe + msgs;
     const CandLayout c = cand_layout(args.tile, args.W, args.D);
     return stage + probe + msgs + size_t(split + 1) * c.cslot + size_t(c.bm_words + c.v_ints) * sizeof(int32_t);
 }
 
-template <bool kSampled, bool kCand>
-static cudaError_t launch_rescan(const StepArgs &args, int split, cudaStream_t stream) {
+template <bool kSampled, bool kCand, bool kPre, bool kMlp>
+static cudaError_t rescan_attrs() {
     static bool attr_done[64] = {false};
     int dev = 0;
     cudaGetDevice(&dev);
     if (dev >= 0 && dev < 64 && !attr_done[dev]) {
-        cudaError_t e = cudaFuncSetAttribute(rescan_kernel<kSampled, kCand>,
+        cudaError_t e = cudaFuncSetAttribute(rescan_kernel<kSampled, kCand, kPre, kMlp>,
                                              cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
         if (e != cudaSuccess) return e;
-        e = cudaFuncSetAttribute(rescan_kernel<kSampled, kCand>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+        e = cudaFuncSetAttribute(rescan_kernel<kSampled, kCand, kPre, kMlp>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                  int(kRescanSmemBudget));
         if (e != cudaSuccess) return e;
         attr_done[dev] = true;
     }
-    return launch_pdl(rescan_kernel<kSampled, kCand>, dim3(unsigned(split), unsigned(args.B), 1),
+    return cudaSuccess;
+}
+
+template <bool kSampled, bool kCand, bool kPre, bool kMlp>
+static cudaError_t launch_rescan(const StepArgs &args, int split, cudaStream_t stream) {
+    const cudaError_t e = rescan_attrs<kSampled, kCand, kPre, kMlp>();
+    if (e != cudaSuccess) return e;
+    return launch_pdl(rescan_kernel<kSampled, kCand, kPre, kMlp>, dim3(unsigned(split), unsigned(args.B), 1),
                       dim3(kRescanThreads, 1, 1), rescan_smem_bytes(args, split), stream, unsigned(split), args);
+}
+
+// Resident CTAs per SM of an instance at a dynamic shared-memory size (cached: the occupancy calculator
+// runs once per instance, device and size).
+template <bool kSampled, bool kCand, bool kPre, bool kMlp>
+static cudaError_t rescan_per_sm(size_t smem, int &out) {
+    struct Entry {
+        int dev;
+        size_t smem;
+        int n;
+    };
+    static std::mutex mu;
+    static Entry cache[32];
+    static int used = 0;
+    int dev = 0;
+    cudaGetDevice(&dev);
+    {
+        std::lock_guard<std::mutex> lk(mu);
+        for (int i = 0; i < used; ++i)
+            if (cache[i].dev == dev && cache[i].smem == smem) {
+                out = cache[i].n;
+                return cudaSuccess;
+            }
+    }
+    cudaError_t e = rescan_attrs<kSampled, kCand, kPre, kMlp>();
+    if (e != cudaSuccess) return e;
+    int n = 0;
+    e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, rescan_kernel<kSampled, kCand, kPre, kMlp>, kRescanThreads, smem);
+    if (e != cudaSuccess) return e;
+    std::lock_guard<std::mutex> lk(mu);
+    if (used < 32) cache[used++] = Entry{dev, smem, n};
+    out = n;
+    return cudaSuccess;
+}
+
+template <bool kSampled, bool kCand, bool kMlp>
+static cudaError_t choose_hash(StepArgs &args, int split, int sms) {
+    const int32_t words = int32_t(((args.tile + 3) / 4 + 3) & ~3);  // one byte an end; 16-byte multiple
+    args.hash_words = 0;
+    // The hashing overlaps the preceding launch only when this launch's CTAs are resident early, which a
+    // grid of fewer CTAs than SMs is not, measured: the 8K rows (two CTAs a row, 128 CTAs) lose 0.1 us a
+    // launch with it, the 32K rows (512 CTAs) gain 0.1 us and the 128K rows (256 CTAs of 8.5K ends) 0.8 us.
+    if (int64_t(split) * args.B < int64_t(sms)) return cudaSuccess;
+    int without = 0, with = 0;
+    cudaError_t e = rescan_per_sm<kSampled, kCand, false, kMlp>(rescan_smem_bytes(args, split), without);
+    if (e != cudaSuccess) return e;
+    StepArgs h = args;
+    h.hash_words = words;
+    const size_t bytes = rescan_smem_bytes(h, split);
+    if (bytes > kRescanSmemBudget) return cudaSuccess;
+    e = rescan_per_sm<kSampled, kCand, true, kMlp>(bytes, with);
+    if (e != cudaSuccess) return e;
+    if (with >= 1 && with >= (without < kRescanMinBlocks ? without : kRescanMinBlocks)) args.hash_words = words;
+    return cudaSuccess;
+}
+
+template <bool kSampled, bool kCand>
+static cudaError_t choose_hash2(StepArgs &args, int split, int sms) {
+    return args.z1_part != nullptr ? choose_hash<kSampled, kCand, true>(args, split, sms)
+                                   : choose_hash<kSampled, kCand, false>(args, split, sms);
+}
+
+cudaError_t rescan_choose_hash(StepArgs &args, int split, int sms) {
+    if (args.W > 0) return choose_hash2<false, true>(args, split, sms);
+    return args.pv_p != nullptr ? choose_hash2<true, false>(args, split, sms)
+                                : choose_hash2<false, false>(args, split, sms);
+}
+
+template <bool kSampled, bool kCand>
+static cudaError_t launch_rescan2(const StepArgs &args, int split, cudaStream_t stream) {
+    const bool mlp = args.z1_part != nullptr;
+    if (args.hash_words > 0)
+        return mlp ? launch_rescan<kSampled, kCand, true, true>(args, split, stream)
+                   : launch_rescan<kSampled, kCand, true, false>(args, split, stream);
+    return mlp ? launch_rescan<kSampled, kCand, false, true>(args, split, stream)
+               : launch_rescan<kSampled, kCand, false, false>(args, split, stream);
 }
 
 cudaError_t launch_rescan_kernel(const StepArgs &args, int split, cudaStream_t stream) {
     // candidate verification is greedy (the candidates' targets are compared token by token)
-    if (args.W > 0) return launch_rescan<false, true>(args, split, stream);
-    return args.pv_p != nullptr ? launch_rescan<true, false>(args, split, stream)
-                                : launch_rescan<false, false>(args, split, stream);
+    if (args.W > 0) return launch_rescan2<false, true>(args, split, stream);
+    return args.pv_p != nullptr ? launch_rescan2<true, false>(args, split, stream)
+                                : launch_rescan2<false, false>(args, split, stream);
 }
 
 }  // namespace switchsd

@@ -18,11 +18,13 @@ constexpr int kMaxSplit = 16;
 constexpr unsigned long long kTimeoutBit = 1ull << 62;
 constexpr int kMaxCand = SWITCHSD_WMAX; // candidate mode: largest W
 constexpr int kProbeStage = 256;      // probe words (8 bf16) of w and of h staged per CTA; the rest is read directly
-// The rescan kernel (rescan.cu): four warps, at most 72 registers a thread, so that seven CTAs fit on an
-// SM and the next launch's CTAs are resident while this launch finishes.
+// The rescan kernel (rescan.cu): four warps, at most 64 registers a thread (eight CTAs' worth of an SM's
+// registers), so that the next launch's CTAs are resident while this launch finishes; the grid is sized
+// for seven CTAs per SM over two launches (a launch spreads unevenly, up to four CTAs on some SMs).
 constexpr int kRescanThreads = 128;
 constexpr int kRescanWarps = kRescanThreads / kWarp;
 constexpr int kRescanMinBlocks = 7;
+constexpr int kRescanLaunchBlocks = 8;  // the launch bound: 65,536 / (8 x 128) = 64 registers a thread
 constexpr int kRescanTileMax = 16384;  // largest CTA range of the rescan kernel (one bulk copy)
 constexpr size_t kRescanSmemBudget = 100 * 1024;
 constexpr int kRescanCapMax = 1 << 25;  // the rescan kernel's match keys hold an end below 2^25
@@ -60,6 +62,8 @@ struct StepArgs {
                                  // (pv_draft [B, W, D], pv_target [B, W, D+1], pv_len = their count [B])
     int32_t *out_choice;         // ... and the kept candidate [B]
     int32_t probe_words;         // rescan kernel: probe words of w and of h staged per CTA
+    int32_t hash_words;          // rescan kernel: words of the pre-wait hash bytes of the old ends (one byte
+                                 // an end, a multiple of 4 words), 0 = pass 1 hashes the tokens after the wait
     unsigned long long *counters;  // optional per-mode tallies (switchsd_params.counters), else null
     uint32_t msg_wait_polls;     // rescan kernel: polls of the leader's wait for the messages (kWaitLimit
                                  // normally; see msg_wait_polls() in step_api.cu)
@@ -92,5 +96,9 @@ cudaError_t launch_step_kernel(const StepArgs &args, bool cand, int split, cudaS
 // none), no candidates, no length bound; args.tile >= the largest CTA range, args.probe_words set.
 cudaError_t launch_rescan_kernel(const StepArgs &args, int split, cudaStream_t stream);
 size_t rescan_smem_bytes(const StepArgs &args, int split);
+// Sets args.hash_words: the pre-wait hash table when the grid has at least one CTA per SM (`sms` SMs) and
+// the table's shared memory keeps the launch's resident CTAs per SM at min(kRescanMinBlocks, what they are
+// without it), else 0.  args.tile, args.z1_part, args.W and args.pv_p must be set.
+cudaError_t rescan_choose_hash(StepArgs &args, int split, int sms);
 
 }  // namespace switchsd

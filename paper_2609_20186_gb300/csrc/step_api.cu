@@ -217,6 +217,7 @@ static int step_entry(int32_t *ctx_tokens, int32_t *ctx_lens, const uint16_t *hi
     args.wait_late = 0;
 
     args.probe_words = 0;
+    args.hash_words = 0;
     const int split = p->split > 0 ? p->split : choose_split(p->B, p->cap);
     // Tile: the largest CTA range (the last CTA may also cover a k + 1 token append), in one stage
     // up to kSingleTileMax ends (64 KB; one copy, and few enough bytes that a grid of two or four
@@ -267,6 +268,7 @@ static int step_entry(int32_t *ctx_tokens, int32_t *ctx_lens, const uint16_t *hi
             ra.out_cand = ra.out_cand_len = ra.out_ncand = ra.out_choice = nullptr;
             ra.pv_cand_len = nullptr;
         }
+        ra.hash_words = 0;
         rescan = rrange <= kRescanTileMax && rescan_smem_bytes(ra, rsplit) <= kRescanSmemBudget;
     }
     bool mlp_early = false;  // the first-layer kernel releases the step kernel at its start
@@ -340,6 +342,8 @@ static int step_entry(int32_t *ctx_tokens, int32_t *ctx_lens, const uint16_t *hi
         // launch's wait.  With it, that kernel releases this one at its start: this launch then reads
         // before its wait only what the caller's prefetch bits cover, and everything else after it.
         ra.wait_late = (args.z1_part != nullptr && !mlp_early) ? 1 : 0;
+        if (rescan_choose_hash(ra, rsplit, sm_count_cached() > 0 ? sm_count_cached() : 148) != cudaSuccess)
+            return SWITCHSD_ERR_CUDA;
         if (launch_rescan_kernel(ra, rsplit, stream) != cudaSuccess) return SWITCHSD_ERR_CUDA;
         return SWITCHSD_OK;
     }
