@@ -836,7 +836,9 @@ def run_ours(args, world, rank, local):
     m = measure_loop(base, args, dev, cs, l2, W, K, args.split, args.search, prefetch, sampled,
                      args.candidates, args.cand_len, world, headline=True, flush=flush)
     peaks = measured_peaks()
-    traffic = profiled_traffic(base.name)
+    # the committed summary profiles the greedy single-draft rescan instance: other modes get no traffic
+    profiled_mode = args.search == "scan" and args.candidates == 0 and args.verify == "greedy" and prefetch
+    traffic = profiled_traffic(base.name) if profiled_mode else None
     roof = roofline_of(m, peaks, "switchsd_verify_step" + (" (index)" if args.search == "index" else ""),
                        traffic)
 
