@@ -1,6 +1,6 @@
-// rescan.cu -- the rescan kernel: switchsd_step / switchsd_verify_step / switchsd_verify_sampled_step with
-// the linear probe (Eq. 3), laid out for a short chain of dependent phases after the grid-dependency
-// wait.
+// rescan.cu -- the rescan kernel: switchsd_step / switchsd_verify_step / switchsd_verify_sampled_step and the
+// candidate entry points, with the linear probe (Eq. 3) or the two-layer probe's finish, laid out for a
+// short chain of dependent phases after the grid-dependency wait.
 //
 // Paper: §3.3 (kappa-gram gate, recency-ranked copy candidates, Eq. 4 decision rule, parallel
 // verification), Eq. 3 (linear probe), Fig. 1 (three cases).
@@ -9,16 +9,19 @@
 // candidate ends [0, L_old - 1) are split into C contiguous 16-byte-aligned ranges; each CTA stages its
 // range (plus kHalo tokens of look-back and kFwd of look-ahead) with one bulk copy, and the row's last
 // kHalo tokens with another, as soon as it has read the row length -- before the grid-dependency wait
-// when the caller allows it.  The CTAs are small (four warps, at most 64 registers a thread) so that the
+// when the caller allows it -- and, in the hash instance, warps 1.. hash every staged old end into one
+// byte once the copy lands.  The CTAs are small (four warps, at most 64 registers a thread) so that the
 // next launch's CTAs are resident, with their copies in flight, while this launch finishes.
 //
-// After the wait there is no CTA-wide or cluster-wide barrier on the path:
+// After the wait no cluster-wide barrier is on the path, and no CTA-wide one outside candidate mode
+// (the hash instance's barrier on the hash bytes completes before the wait when the context is
+// prefetched):
 //  * every warp verifies the previous draft itself (the draft and the target are a few L2 lines), and
 //    keeps its own window of the row's last kHalo old tokens followed by the appended tokens: the new
 //    suffix and the appended positions come from it, so the staged tile is never patched;
-//  * every warp scans its share of the CTA's old ends (first-token filter, then the second token, then
-//    a backward compare against its suffix window), and the leader's warp 0 also tests the a+1 ends the
-//    append creates;
+//  * every warp scans its share of the CTA's old ends (a hash filter on the last F tokens -- computed
+//    from the tokens, or the pre-wait hash bytes -- then an exact test and a backward compare against
+//    its suffix window), and the leader's warp 0 also tests the a+1 ends the append creates;
 //  * every warp ships its best key, its share of the probe's dot product and its best match's
 //    continuation (from the staged tile, or from its window past the old length) to the row's leader CTA
 //    (the last one) with asynchronous DSMEM stores completing on the leader's mbarrier, and is done.
