@@ -43,8 +43,9 @@ static int choose_split(int B, int cap) {
 // CTAs per row of the rescan kernel: the largest power of two, at most kMaxSplit, that leaves every CTA
 // at least 4096 candidate ends while two launches' grids fit on the GPU at once (seven of its CTAs per
 // SM), so the next launch's copies are in flight while this one finishes; 1 at least.  Measured in the
-// benchmark's launch graph: the 32K-context rows 8 CTAs 4.74 us per launch (4: 5.04, 16: 6.85), the 8K
-// rows 2 CTAs 3.41 us (4: 3.43, 1: 4.19), the 128K rows 16 CTAs 5.87 us (8: 8.59).
+// benchmark's launch graph (256 launches): the 32K-context rows 8 CTAs 4.36 us per launch (4: 4.54,
+// 16: 6.59), the 8K rows 2 CTAs 3.06 us (1: 3.41, 4: 3.28), the 128K rows 16 CTAs 5.17 us (8: 8.74),
+// the 16K rows with the two-layer probe 2 CTAs 10.15 us per step (1: 15.83, 4: 11.45).
 static int choose_rescan_split(int B, int cap) {
     const int sms = sm_count_cached() > 0 ? sm_count_cached() : 148;
     int c = 1;
