@@ -2,7 +2,8 @@
 
 switchsd_step_host / switchsd_verify_step_host, and switchsd_plan replays of them, must give exactly
 what the device-buffer calls give (same contexts, outputs and accepted lengths, step after step) with
-the hidden states taken from host memory and the results delivered to host memory.  switchsd_harness_read must fold exactly the words it
+the hidden states taken from host memory and the results delivered to host memory; the plan replays
+(the benchmark's e2e path) are also held to the oracle directly.  switchsd_harness_read must fold exactly the words it
 is documented to read (checked against numpy)."""
 import numpy as np
 import pytest
@@ -198,4 +199,52 @@ def test_sampled_host_staged_and_plan_match_device_calls(use_index):
         assert np.array_equal(out_c.numpy(), want), t
     assert np.array_equal(a.ctx.cpu().numpy(), b.ctx.cpu().numpy())
     assert np.array_equal(a.ctx.cpu().numpy(), c.ctx.cpu().numpy())
+    plan.close()
+
+
+@pytest.mark.parametrize("name", ["zipf_32k", "code_16k"])
+def test_plan_replays_match_the_oracle(name):
+    """The e2e path itself -- switchsd_plan replays of switchsd_verify_step_host, the hidden states taken
+    from pinned host memory and the results read back into it, prefetch on -- against the oracle step by
+    step (lockstep.compare: bit-exact integers, logits within 1e-3)."""
+    import torch
+    from tests import lockstep
+    wl = synth.WORKLOADS[name].scaled(B=8, L0=6001, steps=10)
+    s = _session(wl, True)
+    B, d, k = wl.B, wl.d, wl.k
+    dev_h = torch.empty(B, d, dtype=torch.bfloat16, device="cuda")
+    host_h = torch.empty(B, d, dtype=torch.int16).pin_memory()
+    host_out = torch.empty(B * (k + 3), dtype=torch.int32).pin_memory()
+    first = s.host_plan(host_h, dev_h, host_out, verify=False, debug=True)
+    plan = s.host_plan(host_h, dev_h, host_out, verify=True, debug=True)
+    g_trace = []
+    for t in range(wl.steps):
+        host_h.copy_(torch.from_numpy(wl.hidden(t).view(np.int16)))
+        if t == 0:
+            first.run(host_h, host_out)
+        else:
+            s.harness(t - 1)
+            plan.run(host_h, host_out)
+        torch.cuda.synchronize()
+        res = host_out.numpy().copy()                   # mode [B], len [B], accept [B], draft [B, k]
+        out = s.step_outputs()
+        assert np.array_equal(res[:B], out["mode"]) and np.array_equal(res[B:2 * B], out["len"])
+        if t > 0:                                       # this replay verified the previous step's draft
+            st = out["status"]
+            g_trace[-1]["accept"] = res[2 * B:3 * B]
+            g_trace[-1]["vstatus"] = np.where((st == 1) | (st == 2), st, 0)
+            g_trace[-1]["lens_after"] = s.lens.cpu().numpy()
+        out["draft"] = res[3 * B:].reshape(B, k)
+        g_trace.append(out)
+    s.harness(wl.steps - 1)
+    s.verify()
+    torch.cuda.synchronize()
+    g_trace[-1]["accept"] = s.accept.cpu().numpy()
+    g_trace[-1]["vstatus"] = s.vstatus.cpu().numpy()
+    g_trace[-1]["lens_after"] = s.lens.cpu().numpy()
+    rows = range(B)
+    o_trace, o_ctx, _ = lockstep.oracle_trace(wl, rows, wl.steps)
+    flips, stats = lockstep.compare(wl, o_trace, g_trace, rows, o_ctx, s.ctx.cpu().numpy())
+    assert stats["checked"] > 0 and len(flips) <= 1
+    first.close()
     plan.close()
